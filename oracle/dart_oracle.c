@@ -1,0 +1,501 @@
+/*
+ * DARTree draft-tree construction: plain fp64 CPU oracle.
+ *
+ * TEST INFRASTRUCTURE ONLY.  The tests, the smoke check and the benchmark's
+ * CPU-baseline leg load this library; the product (CUDA) path never does and
+ * shares no code with it.  Everything here is written to be read against the
+ * paper, not to be fast: fp64 throughout, one straightforward loop per
+ * formula, no blocking or fusion.  OpenMP only splits independent vocabulary
+ * rows / output features across threads; every reduction that could depend
+ * on the thread count (log-sum-exp, top-k, sorting) runs serially.
+ *
+ * What it computes (paper: "DARTree: Speculative Diffusion Decoding with
+ * Autoregressive Draft Trees", arXiv 2608.13524):
+ *   - Algorithm 1 (depth-wise fixed-width supertree construction) with the
+ *     full vocabulary as candidate set and a per-node top-k (Appendix D,
+ *     "Full" candidate vocabulary);
+ *   - the path score of Eq. 5, s_beta(u_{1:d}) = sum_i log q~_i(u_i) + beta d;
+ *   - deferred pruning, T = TopB_{u in S} s_beta(u) (Algorithm 1, final step);
+ *   - the best-first heap of Sec. 3.3 / Lemma 1 (used to check that the top-B
+ *     selection equals heap selection when beta <= 0);
+ *   - flattening into the verification tree with an ancestor mask
+ *     (Sec. 3.3, tree verification).
+ * Readings where the paper is silent:
+ *   - correction head g = fallback head
+ *       h_c = RMSNorm(h_p + W_o SiLU(W_i [h_p ; E[t_c]])),  RMSNorm without gain;
+ *   - corrected child distribution of a node with state h at depth d-1:
+ *       z[v] = (Dlog[d-1][v] + E[v] . h) / T'   (T' = T if T > 0 else 1),
+ *       log q~[v] = min(z[v] - logsumexp(z), 0)  (clamp keeps Lemma 1 exact);
+ *   - ties: per-node top-k by (log q~ desc, token asc); frontier by
+ *     (score desc, parent slot asc, rank-in-parent-list asc); pruning by
+ *     (score desc, node id asc) with node id = (depth-1)*W + frontier rank, so
+ *     ancestors always have smaller ids (the "ancestors preferred" rule of
+ *     Lemma 1);
+ *   - candidates with score -inf (probability zero) are never retained.
+ */
+#include <math.h>
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+#ifdef _OPENMP
+#include <omp.h>
+#endif
+
+typedef struct {
+    int V, d, L, W, k, B, nseq, pos_offset, wdtype; /* wdtype 0: float32, 1: bf16 bits */
+    double beta, temperature, rms_eps;
+} orc_cfg;
+
+int orc_num_threads(void) {
+#ifdef _OPENMP
+    return omp_get_max_threads();
+#else
+    return 1;
+#endif
+}
+
+/* ---------------------------------------------------------------- weights */
+
+static double bf16_to_double(uint16_t b) {
+    uint32_t u = (uint32_t)b << 16;
+    float f;
+    memcpy(&f, &u, sizeof f);
+    return (double)f;
+}
+
+static double wval(const void *w, int dt, size_t i) {
+    return dt == 0 ? (double)((const float *)w)[i] : bf16_to_double(((const uint16_t *)w)[i]);
+}
+
+/* sum_j w[off + j] * x[j], j < n, accumulated in fp64 in index order. */
+static double wdot(const void *w, int dt, size_t off, const double *x, int n) {
+    double acc = 0.0;
+    if (dt == 0) {
+        const float *p = (const float *)w + off;
+        for (int j = 0; j < n; j++) acc += (double)p[j] * x[j];
+    } else {
+        const uint16_t *p = (const uint16_t *)w + off;
+        for (int j = 0; j < n; j++) acc += bf16_to_double(p[j]) * x[j];
+    }
+    return acc;
+}
+
+/* ------------------------------------------------------ correction head g */
+
+/* Fallback head: x = [h_p ; E[tok]] (2d), u = W_i x, a = SiLU(u), y = W_o a,
+ * h_c = RMSNorm(h_p + y) = r / sqrt(mean(r^2) + eps).  W_i is [d][2d], W_o is
+ * [d][d], both row-major with the output feature as the row. */
+void orc_head(const orc_cfg *c, const void *Wi, const void *Wo, const void *E,
+              const double *hp, int tok, double *hc) {
+    const int d = c->d, dt = c->wdtype;
+    double *x = (double *)malloc(sizeof(double) * 2 * (size_t)d);
+    double *a = (double *)malloc(sizeof(double) * (size_t)d);
+    double *r = (double *)malloc(sizeof(double) * (size_t)d);
+    for (int j = 0; j < d; j++) {
+        x[j] = hp[j];
+        x[d + j] = wval(E, dt, (size_t)tok * d + j);
+    }
+#pragma omp parallel for schedule(static)
+    for (int i = 0; i < d; i++) {
+        double u = wdot(Wi, dt, (size_t)i * 2 * d, x, 2 * d);
+        a[i] = u / (1.0 + exp(-u));
+    }
+#pragma omp parallel for schedule(static)
+    for (int i = 0; i < d; i++) r[i] = hp[i] + wdot(Wo, dt, (size_t)i * d, a, d);
+    double ss = 0.0;
+    for (int i = 0; i < d; i++) ss += r[i] * r[i];
+    double inv = 1.0 / sqrt(ss / d + c->rms_eps);
+    for (int i = 0; i < d; i++) hc[i] = r[i] * inv;
+    free(x);
+    free(a);
+    free(r);
+}
+
+/* ------------------------------------------- corrected child distribution */
+
+/* z[v] = (Dlog_row[v] + E[v] . h) / T' for every token v of the vocabulary. */
+void orc_child_logits(const orc_cfg *c, const void *E, const float *dlog_row,
+                      const double *h, double *z) {
+    const double Tp = c->temperature > 0.0 ? c->temperature : 1.0;
+    const int d = c->d, dt = c->wdtype;
+#pragma omp parallel for schedule(static)
+    for (int v = 0; v < c->V; v++)
+        z[v] = ((double)dlog_row[v] + wdot(E, dt, (size_t)v * d, h, d)) / Tp;
+}
+
+/* log q~[v] = min(z[v] - logsumexp(z), 0); returns logsumexp(z).  A row whose
+ * logits are all -inf has no child with nonzero probability. */
+double orc_log_softmax(const double *z, int V, double *logq) {
+    double m = -INFINITY;
+    for (int v = 0; v < V; v++)
+        if (z[v] > m) m = z[v];
+    if (m == -INFINITY) {
+        for (int v = 0; v < V; v++) logq[v] = -INFINITY;
+        return -INFINITY;
+    }
+    double s = 0.0;
+    for (int v = 0; v < V; v++) s += exp(z[v] - m);
+    const double lse = m + log(s);
+    for (int v = 0; v < V; v++) {
+        double t = z[v] - lse;
+        logq[v] = t < 0.0 ? t : 0.0;
+    }
+    return lse;
+}
+
+static int better(double a, int ia, double b, int ib) {
+    return a > b || (a == b && ia < ib);
+}
+
+/* Indices of the kk best entries of x by (value desc, index asc), best first. */
+void orc_topk(const double *x, int n, int kk, int *idx) {
+    int cnt = 0;
+    for (int v = 0; v < n; v++) {
+        if (cnt == kk && !better(x[v], v, x[idx[kk - 1]], idx[kk - 1])) continue;
+        int pos = cnt < kk ? cnt++ : kk - 1;
+        while (pos > 0 && better(x[v], v, x[idx[pos - 1]], idx[pos - 1])) {
+            idx[pos] = idx[pos - 1];
+            pos--;
+        }
+        idx[pos] = v;
+    }
+}
+
+/* ------------------------------------------------------------ Algorithm 1 */
+
+typedef struct {
+    double score;
+    int p, j, tok;
+} cand_t;
+
+static int cand_cmp(const void *a_, const void *b_) {
+    const cand_t *a = (const cand_t *)a_, *b = (const cand_t *)b_;
+    if (a->score > b->score) return -1;
+    if (a->score < b->score) return 1;
+    if (a->p != b->p) return a->p < b->p ? -1 : 1;
+    if (a->j != b->j) return a->j < b->j ? -1 : 1;
+    return 0;
+}
+
+typedef struct {
+    double score;
+    int id;
+} node_t;
+
+static int node_cmp(const void *a_, const void *b_) {
+    const node_t *a = (const node_t *)a_, *b = (const node_t *)b_;
+    if (a->score > b->score) return -1;
+    if (a->score < b->score) return 1;
+    return a->id < b->id ? -1 : (a->id > b->id);
+}
+
+static int kx_of(const orc_cfg *c) { return c->k + 1 <= c->V ? c->k + 1 : c->V; }
+
+/* Emission for one sequence: global top-B over the supertree (Algorithm 1,
+ * final step), flattened in ascending node id, which is a topological order.
+ * Output rows beyond the selected count are padding.  Returns 0, or -1 if a
+ * selected node's parent was not selected (impossible when beta <= 0). */
+static int prune_emit_one(const orc_cfg *c, int s, const int *st_tok, const int *st_parent,
+                          const double *st_score, const int *st_count, int *o_tok, int *o_par,
+                          int *o_dep, int *o_pos, double *o_score, int *o_n, uint64_t *o_mask,
+                          double *prune_gap) {
+    const int L = c->L, W = c->W, B = c->B, nw = (B + 63) / 64;
+    const int base = s * L * W;
+    node_t *nodes = (node_t *)malloc(sizeof(node_t) * (size_t)L * W + 1);
+    int total = 0;
+    for (int dep = 1; dep <= L; dep++)
+        for (int r = 0; r < st_count[s * L + dep - 1]; r++) {
+            int id = (dep - 1) * W + r;
+            nodes[total].score = st_score[base + id];
+            nodes[total].id = id;
+            total++;
+        }
+    qsort(nodes, (size_t)total, sizeof(node_t), node_cmp);
+    const int beff = total < B ? total : B;
+    prune_gap[s] = total > beff ? nodes[beff - 1].score - nodes[beff].score : INFINITY;
+    int *out_idx = (int *)malloc(sizeof(int) * (size_t)L * W);
+    char *sel = (char *)calloc((size_t)L * W, 1);
+    for (int i = 0; i < L * W; i++) out_idx[i] = -1;
+    for (int i = 0; i < beff; i++) sel[nodes[i].id] = 1;
+    int rc = 0, n = 0;
+    for (int id = 0; id < L * W; id++) {
+        if (!sel[id]) continue;
+        out_idx[id] = n;
+        const int dep = id / W + 1;
+        int par = -1;
+        if (dep > 1) {
+            int pid = (dep - 2) * W + st_parent[base + id];
+            par = out_idx[pid];
+            if (par < 0) rc = -1;
+        }
+        const size_t o = (size_t)s * B + n;
+        o_tok[o] = st_tok[base + id];
+        o_par[o] = par;
+        o_dep[o] = dep;
+        o_pos[o] = c->pos_offset + dep;
+        o_score[o] = st_score[base + id];
+        uint64_t *row = o_mask + o * nw;
+        memset(row, 0, sizeof(uint64_t) * nw);
+        /* bit j of row n is set iff j is n itself or one of its ancestors */
+        row[n / 64] |= 1ull << (n % 64);
+        int a = par;
+        while (a >= 0) {
+            row[a / 64] |= 1ull << (a % 64);
+            a = o_par[(size_t)s * B + a];
+        }
+        n++;
+    }
+    for (int i = n; i < B; i++) {
+        const size_t o = (size_t)s * B + i;
+        o_tok[o] = -1;
+        o_par[o] = -2;
+        o_dep[o] = 0;
+        o_pos[o] = -1;
+        o_score[o] = -INFINITY;
+        memset(o_mask + o * nw, 0, sizeof(uint64_t) * nw);
+    }
+    o_n[s] = n;
+    free(nodes);
+    free(out_idx);
+    free(sel);
+    return rc;
+}
+
+/* Top-B pruning + emission of every sequence of a given supertree. */
+int orc_prune_emit(const orc_cfg *c, const int *st_tok, const int *st_parent,
+                   const double *st_score, const int *st_count, int *o_tok, int *o_par,
+                   int *o_dep, int *o_pos, double *o_score, int *o_n, uint64_t *o_mask,
+                   double *prune_gap) {
+    int rc = 0;
+    for (int s = 0; s < c->nseq; s++)
+        if (prune_emit_one(c, s, st_tok, st_parent, st_score, st_count, o_tok, o_par, o_dep,
+                           o_pos, o_score, o_n, o_mask, prune_gap))
+            rc = -1;
+    return rc;
+}
+
+/* Algorithm 1 for every sequence, followed by pruning and emission.
+ * Arrays (all caller-allocated, row-major):
+ *   Dlog [nseq][L][V] float, h0 [nseq][d] float;
+ *   supertree st_tok / st_parent (slot in the previous depth, -1 = root) /
+ *     st_score [nseq][L][W], st_count [nseq][L];
+ *   per expanded node p of depth d-1 (index [s][d-1][p]): nd_lse, and its
+ *     kx = min(k+1, V) best children nd_tok / nd_logq [..][kx];
+ *   fr_score [nseq][L][W+1]: the W+1 best candidate scores at each depth;
+ *   emitted tree o_* [nseq][B], o_mask [nseq][B][ceil(B/64)], o_n [nseq],
+ *   prune_gap [nseq] (score gap at the budget cut, +inf if nothing was cut).
+ * Returns 0 on success. */
+int orc_build_tree(const orc_cfg *c, const void *Wi, const void *Wo, const void *E,
+                   const float *Dlog, const float *h0, int *st_tok, int *st_parent,
+                   double *st_score, int *st_count, double *nd_lse, int *nd_tok,
+                   double *nd_logq, double *fr_score, int *o_tok, int *o_par, int *o_dep,
+                   int *o_pos, double *o_score, int *o_n, uint64_t *o_mask, double *prune_gap) {
+    const int V = c->V, d = c->d, L = c->L, W = c->W, k = c->k, kx = kx_of(c);
+    double *hs = (double *)malloc(sizeof(double) * (size_t)W * d);
+    double *hn = (double *)malloc(sizeof(double) * (size_t)W * d);
+    double *z = (double *)malloc(sizeof(double) * (size_t)V);
+    double *logq = (double *)malloc(sizeof(double) * (size_t)V);
+    int *idx = (int *)malloc(sizeof(int) * (size_t)kx);
+    cand_t *cand = (cand_t *)malloc(sizeof(cand_t) * (size_t)W * k + 1);
+    double pscore[1024], nscore[1024];
+    int rc = 0;
+    for (int s = 0; s < c->nseq; s++) {
+        /* S_0 = {root}, r(root) = h_0, s_beta(root) = 0 */
+        for (int j = 0; j < d; j++) hs[j] = (double)h0[(size_t)s * d + j];
+        pscore[0] = 0.0;
+        int pcount = 1;
+        for (int dep = 1; dep <= L; dep++) {
+            const float *row = Dlog + ((size_t)s * L + dep - 1) * V;
+            const size_t nb = ((size_t)s * L + dep - 1) * W;
+            int ncand = 0;
+            for (int p = 0; p < W; p++) {
+                nd_lse[nb + p] = -INFINITY;
+                for (int j = 0; j < kx; j++) {
+                    nd_tok[(nb + p) * kx + j] = -1;
+                    nd_logq[(nb + p) * kx + j] = -INFINITY;
+                }
+            }
+            /* score every child of every retained prefix in S_{d-1} */
+            for (int p = 0; p < pcount; p++) {
+                orc_child_logits(c, E, row, hs + (size_t)p * d, z);
+                nd_lse[nb + p] = orc_log_softmax(z, V, logq);
+                orc_topk(logq, V, kx, idx);
+                for (int j = 0; j < kx; j++) {
+                    nd_tok[(nb + p) * kx + j] = idx[j];
+                    nd_logq[(nb + p) * kx + j] = logq[idx[j]];
+                }
+                for (int j = 0; j < k; j++) {
+                    cand[ncand].score = pscore[p] + logq[idx[j]] + c->beta; /* Eq. 5 */
+                    cand[ncand].p = p;
+                    cand[ncand].j = j;
+                    cand[ncand].tok = idx[j];
+                    ncand++;
+                }
+            }
+            qsort(cand, (size_t)ncand, sizeof(cand_t), cand_cmp);
+            int nvalid = 0;
+            while (nvalid < ncand && cand[nvalid].score > -INFINITY) nvalid++;
+            const int cnt = nvalid < W ? nvalid : W; /* global top-W -> S_d */
+            for (int r = 0; r <= W; r++)
+                fr_score[((size_t)s * L + dep - 1) * (W + 1) + r] =
+                    r < nvalid ? cand[r].score : -INFINITY;
+            const size_t sb = ((size_t)s * L + dep - 1) * W;
+            for (int r = 0; r < W; r++) {
+                st_tok[sb + r] = r < cnt ? cand[r].tok : -1;
+                st_parent[sb + r] = r < cnt ? cand[r].p : -1;
+                st_score[sb + r] = r < cnt ? cand[r].score : -INFINITY;
+            }
+            st_count[s * L + dep - 1] = cnt;
+            /* carry the correction states of the retained children */
+            if (dep < L)
+                for (int r = 0; r < cnt; r++)
+                    orc_head(c, Wi, Wo, E, hs + (size_t)cand[r].p * d, cand[r].tok,
+                             hn + (size_t)r * d);
+            for (int r = 0; r < cnt; r++) nscore[r] = cand[r].score;
+            memcpy(pscore, nscore, sizeof(double) * (size_t)cnt);
+            double *t = hs;
+            hs = hn;
+            hn = t;
+            pcount = cnt;
+        }
+    }
+    if (orc_prune_emit(c, st_tok, st_parent, st_score, st_count, o_tok, o_par, o_dep, o_pos,
+                       o_score, o_n, o_mask, prune_gap))
+        rc = -1;
+    free(hs);
+    free(hn);
+    free(z);
+    free(logq);
+    free(idx);
+    free(cand);
+    return rc;
+}
+
+/* ----------------------------------------------- best-first heap (Lemma 1) */
+
+/* Best-first selection over a materialised supertree of sequence s: a max-heap
+ * seeded with the root's children; each pop emits the best prefix and pushes
+ * its materialised children; stops after min(B, |S|) pops.  Writes the popped
+ * node ids in pop order and returns their count. */
+int orc_heap_select(const orc_cfg *c, const int *st_parent, const double *st_score,
+                    const int *st_count, int s, int *popped) {
+    const int L = c->L, W = c->W;
+    const int base = s * L * W;
+    int total = 0;
+    for (int dep = 1; dep <= L; dep++) total += st_count[s * L + dep - 1];
+    const int beff = total < c->B ? total : c->B;
+    node_t *heap = (node_t *)malloc(sizeof(node_t) * ((size_t)L * W + 1));
+    int hn = 0, np = 0;
+#define HBETTER(a, b) ((a).score > (b).score || ((a).score == (b).score && (a).id < (b).id))
+#define HPUSH(nd)                                                  \
+    do {                                                           \
+        int i_ = hn++;                                             \
+        heap[i_] = (nd);                                           \
+        while (i_ > 0 && HBETTER(heap[i_], heap[(i_ - 1) / 2])) {  \
+            node_t t_ = heap[i_];                                  \
+            heap[i_] = heap[(i_ - 1) / 2];                         \
+            heap[(i_ - 1) / 2] = t_;                               \
+            i_ = (i_ - 1) / 2;                                     \
+        }                                                          \
+    } while (0)
+    for (int r = 0; r < st_count[s * L]; r++) {
+        node_t nd = {st_score[base + r], r};
+        HPUSH(nd);
+    }
+    while (np < beff && hn > 0) {
+        node_t top = heap[0];
+        heap[0] = heap[--hn];
+        int i = 0;
+        for (;;) {
+            int l = 2 * i + 1, rr = l + 1, b = i;
+            if (l < hn && HBETTER(heap[l], heap[b])) b = l;
+            if (rr < hn && HBETTER(heap[rr], heap[b])) b = rr;
+            if (b == i) break;
+            node_t t = heap[i];
+            heap[i] = heap[b];
+            heap[b] = t;
+            i = b;
+        }
+        popped[np++] = top.id;
+        const int dep = top.id / W + 1, slot = top.id % W;
+        if (dep < L)
+            for (int r = 0; r < st_count[s * L + dep]; r++)
+                if (st_parent[base + dep * W + r] == slot) {
+                    node_t ch = {st_score[base + dep * W + r], dep * W + r};
+                    HPUSH(ch);
+                }
+    }
+#undef HPUSH
+#undef HBETTER
+    free(heap);
+    return np;
+}
+
+/* ----------------------------------------------- teacher-forced path tools */
+
+/* State r(u) of the prefix u = path[0..len) of sequence (Dlog_seq, h0_seq),
+ * obtained by running the correction head from the root along the path. */
+void orc_path_state(const orc_cfg *c, const void *Wi, const void *Wo, const void *E,
+                    const float *h0_seq, const int *path, int len, double *h_out) {
+    const int d = c->d;
+    double *h = (double *)malloc(sizeof(double) * (size_t)d);
+    double *t = (double *)malloc(sizeof(double) * (size_t)d);
+    for (int j = 0; j < d; j++) h[j] = (double)h0_seq[j];
+    for (int i = 0; i < len; i++) {
+        orc_head(c, Wi, Wo, E, h, path[i], t);
+        memcpy(h, t, sizeof(double) * (size_t)d);
+    }
+    memcpy(h_out, h, sizeof(double) * (size_t)d);
+    free(h);
+    free(t);
+}
+
+/* Children of the prefix path[0..len): its corrected log-probabilities over
+ * the whole vocabulary (logq_all, may be NULL), their log-sum-exp, and the kk
+ * best children by (log q~ desc, token asc). */
+double orc_node_children(const orc_cfg *c, const void *Wi, const void *Wo, const void *E,
+                         const float *Dlog_seq, const float *h0_seq, const int *path, int len,
+                         int kk, int *tok_out, double *logq_out, double *logq_all) {
+    const int V = c->V, d = c->d;
+    double *h = (double *)malloc(sizeof(double) * (size_t)d);
+    double *z = (double *)malloc(sizeof(double) * (size_t)V);
+    double *lq = logq_all ? logq_all : (double *)malloc(sizeof(double) * (size_t)V);
+    orc_path_state(c, Wi, Wo, E, h0_seq, path, len, h);
+    orc_child_logits(c, E, Dlog_seq + (size_t)len * V, h, z);
+    double lse = orc_log_softmax(z, V, lq);
+    if (kk > 0) {
+        orc_topk(lq, V, kk, tok_out);
+        for (int j = 0; j < kk; j++) logq_out[j] = lq[tok_out[j]];
+    }
+    free(h);
+    free(z);
+    if (!logq_all) free(lq);
+    return lse;
+}
+
+/* Eq. 5 along a path: scores[i] = sum_{i' <= i} log q~(path[i']) + beta (i+1). */
+void orc_path_scores(const orc_cfg *c, const void *Wi, const void *Wo, const void *E,
+                     const float *Dlog_seq, const float *h0_seq, const int *path, int len,
+                     double *scores) {
+    const int V = c->V, d = c->d;
+    double *h = (double *)malloc(sizeof(double) * (size_t)d);
+    double *t = (double *)malloc(sizeof(double) * (size_t)d);
+    double *z = (double *)malloc(sizeof(double) * (size_t)V);
+    double *lq = (double *)malloc(sizeof(double) * (size_t)V);
+    for (int j = 0; j < d; j++) h[j] = (double)h0_seq[j];
+    double s = 0.0;
+    for (int i = 0; i < len; i++) {
+        orc_child_logits(c, E, Dlog_seq + (size_t)i * V, h, z);
+        orc_log_softmax(z, V, lq);
+        s += lq[path[i]] + c->beta;
+        scores[i] = s;
+        if (i + 1 < len) {
+            orc_head(c, Wi, Wo, E, h, path[i], t);
+            memcpy(h, t, sizeof(double) * (size_t)d);
+        }
+    }
+    free(h);
+    free(t);
+    free(z);
+    free(lq);
+}

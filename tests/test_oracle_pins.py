@@ -1,0 +1,368 @@
+"""Pins of the fp64 oracle against what the paper and mathematics fix.
+
+Nothing here retypes the oracle's code: every check compares it with a
+library routine, exhaustive enumeration, a closed form, or a structural
+invariant the paper states (Lemma 1, prefix closure, monotone scores).
+"""
+import itertools
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from refs import TorchHead, all_path_scores, child_logq, ddtree_topB, weights64
+from workloads import TOY, Config, bf16_bits_to_f32, f32_to_bf16_bits, make_inputs
+
+
+def tiny(**kw):
+    base = dict(name="tiny", nseq=1, V=5, d=8, L=3, W=125, k=5, B=20, wdtype="f32",
+                temperature=0.0, seed=77)
+    base.update(kw)
+    return Config(**base)
+
+
+def rand_inputs(cfg, e_std=0.7, seed=None):
+    """Seeded inputs with a large E so the correction head visibly matters."""
+    g = np.random.Generator(np.random.PCG64(cfg.seed if seed is None else seed))
+    d = cfg.d
+    Wi = (g.standard_normal((d, 2 * d)) / np.sqrt(2 * d)).astype(np.float32)
+    Wo = (g.standard_normal((d, d)) / np.sqrt(d)).astype(np.float32)
+    E = (g.standard_normal((cfg.V, d)) * e_std).astype(np.float32)
+    Dlog = (g.standard_normal((cfg.nseq, cfg.L, cfg.V)) * 1.5).astype(np.float32)
+    h0 = g.standard_normal((cfg.nseq, d)).astype(np.float32)
+    if cfg.wdtype == "bf16":
+        Wi, Wo, E = f32_to_bf16_bits(Wi), f32_to_bf16_bits(Wo), f32_to_bf16_bits(E)
+    return dict(Wi=Wi, Wo=Wo, E=E, Dlog=Dlog, h0=h0)
+
+
+def run(cfg, x):
+    return oracle.build_tree(cfg, x["Wi"], x["Wo"], x["E"], x["Dlog"], x["h0"])
+
+
+# --------------------------------------------------------------- pieces
+
+@pytest.mark.parametrize("wdtype", ["f32", "bf16"])
+def test_head_matches_library_modules(wdtype):
+    cfg = tiny(d=48, V=11, wdtype=wdtype)
+    x = rand_inputs(cfg)
+    ref = TorchHead(cfg, x["Wi"], x["Wo"], x["E"])
+    g = np.random.Generator(np.random.PCG64(5))
+    for tok in (0, 3, 10):
+        hp = g.standard_normal(cfg.d)
+        got = oracle.head(cfg, x["Wi"], x["Wo"], x["E"], hp, tok)
+        want = ref(torch.from_numpy(hp), tok).numpy()
+        np.testing.assert_allclose(got, want, rtol=0, atol=1e-12)
+        # RMSNorm without gain: mean square is 1 up to eps
+        assert abs(np.mean(got ** 2) - 1.0) < 1e-5
+
+
+def test_child_logits_and_log_softmax_match_torch():
+    cfg = tiny(V=300, d=32, temperature=0.7)
+    x = rand_inputs(cfg)
+    h = np.random.Generator(np.random.PCG64(9)).standard_normal(cfg.d)
+    z = oracle.child_logits(cfg, x["E"], x["Dlog"][0, 1], h)
+    zt = (torch.from_numpy(x["Dlog"][0, 1].astype(np.float64))
+          + weights64(cfg, x["E"]) @ torch.from_numpy(h)) / 0.7
+    np.testing.assert_allclose(z, zt.numpy(), rtol=0, atol=1e-12)
+    lq, lse = oracle.log_softmax(z)
+    np.testing.assert_allclose(lq, child_logq(cfg, weights64(cfg, x["E"]), x["Dlog"][0, 1],
+                                              torch.from_numpy(h)).numpy(), atol=1e-12)
+    assert abs(np.exp(lq).sum() - 1.0) < 1e-12
+    assert np.all(lq <= 0.0)
+    assert abs(lse - float(torch.logsumexp(zt, 0))) < 1e-12
+
+
+def test_log_softmax_clamp_and_neg_inf():
+    # a single finite logit: log q = 0 exactly (clamped), others -inf
+    z = np.array([-np.inf, 3.0, -np.inf])
+    lq, lse = oracle.log_softmax(z)
+    assert lq[1] == 0.0 and np.isneginf(lq[0]) and np.isneginf(lq[2]) and lse == 3.0
+    lq, lse = oracle.log_softmax(np.full(4, -np.inf))
+    assert np.all(np.isneginf(lq)) and np.isneginf(lse)
+
+
+def test_topk_matches_lexsort_with_ties():
+    g = np.random.Generator(np.random.PCG64(3))
+    x = np.round(g.standard_normal(500), 1)          # many exact ties
+    x[[7, 99]] = -np.inf
+    for kk in (1, 5, 37, 500):
+        want = np.lexsort((np.arange(x.size), -x))[:kk]   # value desc, index asc
+        np.testing.assert_array_equal(oracle.topk(x, kk), want)
+
+
+# ------------------------------------------------- brute force on tiny V/L
+
+@pytest.mark.parametrize("temperature,beta", [(0.0, -0.2), (0.7, 0.0)])
+def test_bruteforce_full_supertree(temperature, beta):
+    """W = V^L, k = V: the supertree is every prefix; each node's score must
+    equal an independent per-path recomputation, and the pruned tree must be
+    the brute-force top-B."""
+    cfg = tiny(temperature=temperature, beta=beta)
+    x = rand_inputs(cfg)
+    r = run(cfg, x)
+    brute = all_path_scores(cfg, x["Wi"], x["Wo"], x["E"], x["Dlog"][0], x["h0"][0], cfg.L)
+    paths = oracle.node_paths(r["st_tok"], r["st_parent"], r["st_count"], 0, cfg.W)
+    assert len(paths) == len(brute) == 5 + 25 + 125
+    for nid, p in paths.items():
+        assert abs(r["st_score"][0].reshape(-1)[nid] - brute[p]) < 1e-12
+    ranked = sorted(brute.items(), key=lambda kv: -kv[1])
+    assert ranked[cfg.B - 1][1] - ranked[cfg.B][1] > 1e-9
+    want = {p for p, _ in ranked[:cfg.B]}
+    emitted = set()
+    for i in range(r["n_nodes"][0]):
+        path = []
+        j = i
+        while j >= 0:
+            path.append(int(r["tokens"][0, j]))
+            j = int(r["parents"][0, j])
+        emitted.add(tuple(reversed(path)))
+    assert emitted == want
+
+
+@pytest.mark.parametrize("V,W,k", [(6, 4, 4), (6, 5, 2), (7, 3, 7)])
+def test_bruteforce_beam_levels(V, W, k):
+    """Each S_d is the top-W (by Eq. 5 score) among the per-node top-k
+    children of S_{d-1}, every child scored by an independent recomputation.
+    For k >= W this is the same as the top-W over all V children."""
+    cfg = tiny(V=V, W=W, k=k, L=4, B=7, d=6, seed=11)
+    x = rand_inputs(cfg)
+    r = run(cfg, x)
+    head = TorchHead(cfg, x["Wi"], x["Wo"], x["E"])
+    E64 = head.E
+    frontier = [((), 0.0, torch.from_numpy(x["h0"][0].astype(np.float64)))]
+    for dep in range(1, cfg.L + 1):
+        cands = []
+        for pi, (path, s, h) in enumerate(frontier):
+            lq = child_logq(cfg, E64, x["Dlog"][0, dep - 1], h).numpy()
+            order = np.lexsort((np.arange(V), -lq))
+            allowed = order[:k] if k < W else order   # k >= W: all children
+            for t in allowed:
+                cands.append((s + lq[t] + cfg.beta, path + (int(t),), h, int(t)))
+        cands.sort(key=lambda c: -c[0])
+        keep = cands[:W]
+        got = [tuple(oracle.node_paths(r["st_tok"], r["st_parent"], r["st_count"], 0, W)
+                     [(dep - 1) * W + j]) for j in range(int(r["st_count"][0, dep - 1]))]
+        assert got == [c[1] for c in keep]
+        np.testing.assert_allclose(r["st_score"][0, dep - 1, :len(keep)],
+                                   [c[0] for c in keep], atol=1e-12)
+        frontier = [(c[1], c[0], head(c[2], c[3])) for c in keep]
+
+
+# ---------------------------------------------------------- special cases
+
+def test_zero_E_is_ddtree_optimal_tree():
+    """E = 0 makes q~ path independent (Sec. 2.3): scores reduce to
+    sum_i log_softmax(Dlog_i)[u_i] + beta d, and with W, k >= B the pruned
+    tree equals DDTree's best-first top-B prefixes."""
+    cfg = tiny(V=40, d=16, L=5, W=12, k=12, B=12, beta=-0.2)
+    x = rand_inputs(cfg)
+    x["E"] = np.zeros_like(x["E"])
+    r = run(cfg, x)
+    rows = [torch.log_softmax(torch.from_numpy(x["Dlog"][0, i].astype(np.float64)), 0).numpy()
+            + cfg.beta for i in range(cfg.L)]
+    want = ddtree_topB(rows, cfg.B)
+    got = {}
+    for i in range(r["n_nodes"][0]):
+        path, j = [], i
+        while j >= 0:
+            path.append(int(r["tokens"][0, j]))
+            j = int(r["parents"][0, j])
+        got[tuple(reversed(path))] = r["scores"][0, i]
+    assert set(got) == {p for p, _ in want}
+    for p, s in want:
+        assert abs(got[p] - s) < 1e-12
+
+
+def test_greedy_chain_W1_k1():
+    """W = k = 1: the tree is the greedy corrected chain; each step is the
+    argmax of a library log-softmax, the state advanced by the library head."""
+    cfg = tiny(V=64, d=24, L=6, W=1, k=1, B=6, temperature=1.0)
+    x = rand_inputs(cfg)
+    r = run(cfg, x)
+    head = TorchHead(cfg, x["Wi"], x["Wo"], x["E"])
+    h = torch.from_numpy(x["h0"][0].astype(np.float64))
+    s = 0.0
+    for i in range(cfg.L):
+        lq = child_logq(cfg, head.E, x["Dlog"][0, i], h)
+        t = int(torch.argmax(lq))
+        s += float(lq[t]) + cfg.beta
+        assert r["tokens"][0, i] == t and r["parents"][0, i] == i - 1
+        assert abs(r["scores"][0, i] - s) < 1e-12
+        h = head(h, t)
+
+
+def test_single_depth_is_topk_of_log_softmax():
+    cfg = tiny(V=500, d=32, L=1, W=9, k=12, B=6)
+    x = rand_inputs(cfg)
+    r = run(cfg, x)
+    lq = child_logq(cfg, weights64(cfg, x["E"]), x["Dlog"][0, 0],
+                    torch.from_numpy(x["h0"][0].astype(np.float64)))
+    vals, idx = torch.topk(lq, 6)
+    np.testing.assert_array_equal(r["tokens"][0, :6], idx.numpy())
+    np.testing.assert_allclose(r["scores"][0, :6], vals.numpy() + cfg.beta, atol=1e-12)
+    assert np.all(r["parents"][0, :6] == -1) and np.all(r["depths"][0, :6] == 1)
+
+
+# ------------------------------------------------------------ Lemma 1 etc.
+
+def _check_tree_structure(cfg, r):
+    """Prefix closure, monotone scores, depths, position ids and the ancestor
+    mask (transitive closure of the parent relation, diagonal set)."""
+    nw = (cfg.B + 63) // 64
+    for s in range(cfg.nseq):
+        n = int(r["n_nodes"][s])
+        par = r["parents"][s]
+        for i in range(n):
+            p = int(par[i])
+            assert -1 <= p < i
+            if p >= 0:
+                assert r["depths"][s, i] == r["depths"][s, p] + 1
+                assert r["scores"][s, i] <= r["scores"][s, p]
+            else:
+                assert r["depths"][s, i] == 1
+            assert r["pos_ids"][s, i] == cfg.pos_offset + r["depths"][s, i]
+            anc = {i}
+            j = p
+            while j >= 0:
+                anc.add(j)
+                j = int(par[j])
+            bits = {b for b in range(cfg.B) if (int(r["mask"][s, i, b // 64]) >> (b % 64)) & 1}
+            assert bits == anc
+            assert len(bits) == r["depths"][s, i]
+        for i in range(n, cfg.B):
+            assert r["tokens"][s, i] == -1 and r["parents"][s, i] == -2
+            assert r["depths"][s, i] == 0 and np.all(r["mask"][s, i] == 0)
+        assert r["mask"].shape[-1] == nw
+
+
+@pytest.mark.parametrize("beta", [0.0, -0.2, -1.5])
+def test_lemma1_heap_equals_topB(beta):
+    cfg = tiny(V=9, d=12, L=6, W=7, k=4, B=19, beta=beta, nseq=3, pos_offset=100)
+    x = rand_inputs(cfg)
+    r = run(cfg, x)
+    _check_tree_structure(cfg, r)
+    for s in range(cfg.nseq):
+        popped = oracle.heap_select(cfg, r["st_parent"], r["st_score"], r["st_count"], s)
+        order = sorted(((r["st_score"][s].reshape(-1)[i], i) for dep in range(cfg.L)
+                        for i in [dep * cfg.W + j for j in range(r["st_count"][s, dep])]),
+                       key=lambda t: (-t[0], t[1]))
+        sel = [i for _, i in order[:cfg.B]]
+        assert set(popped.tolist()) == set(sel)
+
+
+def test_lemma1_with_exact_ties():
+    """Quantised drafter logits and E = 0 give many exactly tied scores; with
+    the node-id tie-break the heap and the top-B still agree."""
+    cfg = tiny(V=6, d=8, L=5, W=9, k=6, B=23, beta=0.0)
+    x = rand_inputs(cfg)
+    x["E"] = np.zeros_like(x["E"])
+    x["Dlog"] = np.round(x["Dlog"]).astype(np.float32)
+    x["Dlog"][:, :, 0] = x["Dlog"][:, :, 1]
+    r = run(cfg, x)
+    sc = r["st_score"][0].reshape(-1)
+    ids = [dep * cfg.W + j for dep in range(cfg.L) for j in range(r["st_count"][0, dep])]
+    vals = [sc[i] for i in ids]
+    assert len(vals) - len(set(vals)) > 5          # there really are ties
+    popped = oracle.heap_select(cfg, r["st_parent"], r["st_score"], r["st_count"], 0)
+    top = sorted(ids, key=lambda i: (-sc[i], i))[:cfg.B]
+    assert popped.tolist() == top                  # identical pop order too
+    _check_tree_structure(cfg, r)
+
+
+def test_positive_beta_breaks_heap_equivalence():
+    """Lemma 1 needs beta <= 0: a hand-built supertree where a child
+    outranks its parent makes top-B not prefix closed."""
+    cfg = tiny(V=3, L=2, W=2, k=2, B=1, beta=0.5)
+    st_tok = np.array([[[0, -1], [1, -1]]], np.int32)
+    st_parent = np.array([[[-1, -1], [0, -1]]], np.int32)
+    st_score = np.array([[[-0.1, -np.inf], [0.3, -np.inf]]])
+    st_count = np.array([[1, 1]], np.int32)
+    popped = oracle.heap_select(cfg, st_parent, st_score, st_count, 0)
+    assert popped.tolist() == [0]                  # the heap can only pop the root child
+    r = oracle.prune_emit(cfg, st_tok, st_parent, st_score, st_count)
+    assert r["rc"] == -1                           # top-1 picked the orphan child
+
+
+def test_prune_emit_hand_example():
+    """A 6-node supertree with known answer: B = 4 keeps ids {0,1,2,4}."""
+    cfg = tiny(V=10, L=3, W=2, k=2, B=4, beta=-0.2, pos_offset=7)
+    st_tok = np.array([[[5, 6], [7, 8], [9, 1]]], np.int32)
+    st_parent = np.array([[[-1, -1], [0, 1], [0, 1]]], np.int32)
+    st_score = np.array([[[-0.3, -0.5], [-0.9, -0.6], [-1.2, -0.7]]])
+    st_count = np.array([[2, 2, 2]], np.int32)
+    r = oracle.prune_emit(cfg, st_tok, st_parent, st_score, st_count)
+    assert r["rc"] == 0 and r["n_nodes"][0] == 4
+    # selected ids by (score desc, id asc): 0(-0.3) 1(-0.5) 3(-0.6) 5(-0.7)
+    np.testing.assert_array_equal(r["tokens"][0], [5, 6, 8, 1])
+    np.testing.assert_array_equal(r["parents"][0], [-1, -1, 1, 2])
+    np.testing.assert_array_equal(r["depths"][0], [1, 1, 2, 3])
+    np.testing.assert_array_equal(r["pos_ids"][0], [8, 8, 9, 10])
+    np.testing.assert_array_equal(r["mask"][0, :, 0], [0b1, 0b10, 0b110, 0b1110])
+    assert abs(r["prune_gap"][0] - (-0.7 + 0.9)) < 1e-15
+
+
+def test_neg_inf_children_are_never_retained():
+    cfg = tiny(V=8, d=8, L=3, W=6, k=4, B=30)
+    x = rand_inputs(cfg)
+    x["Dlog"][0, 1, 2:] = -np.inf        # depth 2: only tokens 0, 1 possible
+    r = run(cfg, x)
+    c = r["st_count"][0]
+    assert c[1] == min(cfg.W, 2 * c[0])
+    assert set(r["st_tok"][0, 1, :c[1]].tolist()) <= {0, 1}
+    assert np.all(np.isfinite(r["st_score"][0, 1, :c[1]]))
+    _check_tree_structure(cfg, r)
+
+
+def test_toy_config_structure():
+    x = make_inputs(TOY)
+    r = run(TOY, x)
+    assert r["n_nodes"][0] == 16 and list(r["st_count"][0]) == [4, 4, 4, 4]
+    _check_tree_structure(TOY, r)
+    # teacher-forced helpers agree with the construction
+    paths = oracle.node_paths(r["st_tok"], r["st_parent"], r["st_count"], 0, TOY.W)
+    for nid in (0, 5, 15):
+        p = paths[nid]
+        sc = oracle.path_scores(TOY, x["Wi"], x["Wo"], x["E"], x["Dlog"][0], x["h0"][0], p)
+        assert abs(sc[-1] - r["st_score"][0].reshape(-1)[nid]) < 1e-9
+        tok, lq, lse, _ = oracle.node_children(TOY, x["Wi"], x["Wo"], x["E"], x["Dlog"][0],
+                                               x["h0"][0], p[:-1], TOY.k + 1)
+        dep = len(p)
+        par = r["st_parent"][0, dep - 1, nid % TOY.W] if dep > 1 else 0
+        np.testing.assert_array_equal(tok, r["nd_tok"][0, dep - 1, par])
+        np.testing.assert_allclose(lq, r["nd_logq"][0, dep - 1, par], atol=1e-12)
+
+
+def test_bf16_roundtrip_helper():
+    x = np.array([1.0, 1.00390625, 1.005859375, -3.0e-3, 0.0], np.float32)
+    b = f32_to_bf16_bits(x)
+    y = bf16_bits_to_f32(b)
+    # 1.00390625 is the exact midpoint 1 + 2^-8 -> rounds to even (1.0)
+    assert y[0] == 1.0 and y[1] == 1.0 and y[2] == np.float32(1.0078125)
+    assert abs(y[3] - x[3]) <= abs(x[3]) * 2 ** -8
+
+
+def test_prune_tiebreak_inside_tied_group():
+    """Budget cuts that fall inside a group of exactly tied scores: the
+    emitted nodes must be the smallest ids of the group (ancestors first),
+    matching both a library sort by (score desc, id asc) and the heap."""
+    cfg0 = tiny(V=6, d=8, L=5, W=9, k=6, B=23, beta=0.0)
+    x = rand_inputs(cfg0)
+    x["E"] = np.zeros_like(x["E"])
+    x["Dlog"] = np.round(x["Dlog"]).astype(np.float32)
+    x["Dlog"][:, :, 0] = x["Dlog"][:, :, 1]
+    r = run(cfg0, x)
+    sc = r["st_score"][0].reshape(-1)
+    ids = [dep * cfg0.W + j for dep in range(cfg0.L) for j in range(r["st_count"][0, dep])]
+    order = sorted(ids, key=lambda i: (-sc[i], i))
+    cuts = [b for b in range(1, len(order)) if sc[order[b - 1]] == sc[order[b]]]
+    assert len(cuts) >= 3
+    for B in cuts:
+        cfg = cfg0.replace(B=B)
+        e = oracle.prune_emit(cfg, r["st_tok"], r["st_parent"], r["st_score"], r["st_count"])
+        assert e["rc"] == 0
+        keep = sorted(order[:B])
+        np.testing.assert_array_equal(e["tokens"][0, :B], r["st_tok"][0].reshape(-1)[keep])
+        np.testing.assert_array_equal(e["depths"][0, :B], [i // cfg.W + 1 for i in keep])
+        popped = oracle.heap_select(cfg, r["st_parent"], r["st_score"], r["st_count"], 0)
+        assert sorted(popped.tolist()) == keep

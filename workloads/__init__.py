@@ -1,0 +1,192 @@
+"""Seeded synthetic workloads for DARTree draft-tree construction.
+
+This module only draws random inputs.  It holds none of the method's
+arithmetic, so both the CPU oracle and the CUDA path can consume exactly the
+same bits without sharing any code that computes the tree.
+
+The shapes follow the paper's experimental setting (Qwen3-4B / Qwen3-8B
+vocabulary and hidden sizes, a 16-token draft block, the width / budget
+ranges of the hyper-parameter study, Sec. 5.1 and Sec. 5.3).  The paper's
+drafter, correction head and datasets are not available, so:
+
+* the correction head is the fallback head
+  h_c = RMSNorm(h_p + W_o . SiLU(W_i . [h_p ; E[t_c]])) with
+  W_i ~ N(0, 1/(2d)), W_o ~ N(0, 1/d), E ~ N(0, 0.02^2) (the LM head is tied to E);
+* drafter marginal logits are 3 . N(0,1) per position plus a spike at one
+  seeded random token per position (+8 for the fp32 toy, +6 at positions 0-7
+  and +3 at positions 8-15 for the bf16 shapes, mimicking decaying drafter
+  confidence along the block);
+* the anchor state h_0 ~ N(0,1).
+
+bf16 weights are drawn in fp32 and rounded to nearest-even bf16; they are
+returned as uint16 bit patterns.  Every array is generated from numpy's PCG64
+with a fixed seed per (config, tensor, row chunk), so the values do not depend
+on the number of threads used to draw them or on the machine.
+"""
+from __future__ import annotations
+
+import concurrent.futures as _cf
+import dataclasses
+import os
+
+import numpy as np
+
+BETA_DEFAULT = -0.2      # depth bonus of the pruned variant (Sec. 5.1)
+RMS_EPS = 1e-6
+
+
+@dataclasses.dataclass(frozen=True)
+class Config:
+    name: str
+    nseq: int
+    V: int
+    d: int
+    L: int
+    W: int
+    k: int
+    B: int
+    wdtype: str            # "f32" or "bf16"
+    temperature: float     # 0 = greedy scoring (no scaling)
+    seed: int
+    beta: float = BETA_DEFAULT
+    rms_eps: float = RMS_EPS
+    pos_offset: int = 0
+    spike_early: float = 6.0   # positions 0..7
+    spike_late: float = 3.0    # positions 8..
+
+    def replace(self, **kw) -> "Config":
+        return dataclasses.replace(self, **kw)
+
+    @property
+    def bpe(self) -> int:
+        return 4 if self.wdtype == "f32" else 2
+
+    def caps(self):
+        """Maximum frontier size |S_d| for d = 0..L (|S_0| = 1)."""
+        c = [1]
+        for _ in range(self.L):
+            c.append(min(self.W, c[-1] * self.k))
+        return c
+
+    def expansions_per_round(self) -> int:
+        """Nodes whose children are scored in one round: sum_d nseq*|S_{d-1}|."""
+        c = self.caps()
+        return self.nseq * sum(c[:self.L])
+
+    def lmhead_bytes_per_depth(self) -> int:
+        """Algorithmic HBM bytes of one LM-head pass: E once + the drafter row."""
+        return self.V * self.d * self.bpe + self.nseq * self.V * 4
+
+
+# Base seed 2608 + index, in the order the workloads are listed.
+TOY = Config("toy", 1, 4096, 256, 4, 4, 4, 16, "f32", 0.0, 2608,
+             spike_early=8.0, spike_late=8.0)
+Q4B = Config("qwen3-4b", 1, 151936, 2560, 16, 8, 8, 64, "bf16", 0.0, 2609)
+Q8B = Config("qwen3-8b", 1, 151936, 4096, 16, 16, 16, 256, "bf16", 1.0, 2610)
+SWEEP_BASE = Config("sweep", 1, 151936, 2560, 16, 8, 8, 32, "bf16", 0.0, 2611)
+BATCHED = Config("batched", 8, 151936, 4096, 16, 32, 32, 512, "bf16", 1.0, 2612)
+
+
+def sweep_configs():
+    out = []
+    for W in (8, 16, 32, 64):
+        for B in (32, 128, 512, 1024):
+            out.append(SWEEP_BASE.replace(name=f"sweep-W{W}-B{B}", W=W, k=W, B=B))
+    return out
+
+
+NAMED = {c.name: c for c in (TOY, Q4B, Q8B, BATCHED)}
+for _c in sweep_configs():
+    NAMED[_c.name] = _c
+
+
+# --------------------------------------------------------------------------
+# bit helpers (no method arithmetic: only storage conversions)
+
+def f32_to_bf16_bits(x: np.ndarray) -> np.ndarray:
+    """Round float32 to bfloat16 (nearest even); returns uint16 bit patterns."""
+    u = np.ascontiguousarray(x, dtype=np.float32).view(np.uint32)
+    out = np.empty(u.shape, dtype=np.uint16)
+    flat_u = u.reshape(-1)
+    flat_o = out.reshape(-1)
+    step = 1 << 24
+    for s in range(0, flat_u.size, step):
+        c = flat_u[s:s + step]
+        r = (c >> np.uint32(16)) & np.uint32(1)
+        flat_o[s:s + step] = ((c + np.uint32(0x7FFF) + r) >> np.uint32(16)).astype(np.uint16)
+    return out
+
+
+def bf16_bits_to_f32(b: np.ndarray) -> np.ndarray:
+    return (np.ascontiguousarray(b, dtype=np.uint16).astype(np.uint32) << np.uint32(16)).view(np.float32)
+
+
+# --------------------------------------------------------------------------
+# generators
+
+_ROWS_PER_CHUNK = 4096
+
+
+def _normal_rows(seed: int, tag: int, rows: int, cols: int, std: float,
+                 threads: int | None = None) -> np.ndarray:
+    """rows x cols float32 N(0, std^2); chunk c of rows uses PCG64([seed, tag, c])."""
+    out = np.empty((rows, cols), dtype=np.float32)
+    nchunk = (rows + _ROWS_PER_CHUNK - 1) // _ROWS_PER_CHUNK
+
+    def work(c):
+        r0 = c * _ROWS_PER_CHUNK
+        r1 = min(rows, r0 + _ROWS_PER_CHUNK)
+        g = np.random.Generator(np.random.PCG64([seed, tag, c]))
+        blk = out[r0:r1]
+        g.standard_normal(out=blk, dtype=np.float32)
+        blk *= np.float32(std)
+
+    if threads is None:
+        threads = min(32, os.cpu_count() or 1)
+    if nchunk == 1 or threads <= 1:
+        for c in range(nchunk):
+            work(c)
+    else:
+        with _cf.ThreadPoolExecutor(threads) as ex:
+            list(ex.map(work, range(nchunk)))
+    return out
+
+
+def make_weights(cfg: Config, zero_E: bool = False):
+    """Fallback-head weights: W_i [d,2d], W_o [d,d], E [V,d] (tied LM head).
+
+    Returned as float32 arrays for fp32 configs, uint16 bf16 bit patterns for
+    bf16 configs.
+    """
+    d = cfg.d
+    Wi = _normal_rows(cfg.seed, 1, d, 2 * d, (1.0 / (2 * d)) ** 0.5)
+    Wo = _normal_rows(cfg.seed, 2, d, d, (1.0 / d) ** 0.5)
+    if zero_E:
+        E = np.zeros((cfg.V, d), dtype=np.float32)
+    else:
+        E = _normal_rows(cfg.seed, 3, cfg.V, d, 0.02)
+    if cfg.wdtype == "bf16":
+        return f32_to_bf16_bits(Wi), f32_to_bf16_bits(Wo), f32_to_bf16_bits(E)
+    return Wi, Wo, E
+
+
+def make_sequences(cfg: Config):
+    """Per-sequence drafter logits Dlog [nseq, L, V] and anchors h0 [nseq, d]."""
+    Dlog = np.empty((cfg.nseq, cfg.L, cfg.V), dtype=np.float32)
+    h0 = np.empty((cfg.nseq, cfg.d), dtype=np.float32)
+    for s in range(cfg.nseq):
+        g = np.random.Generator(np.random.PCG64(cfg.seed * 1000 + s))
+        h0[s] = g.standard_normal(cfg.d, dtype=np.float32)
+        noise = g.standard_normal((cfg.L, cfg.V), dtype=np.float32)
+        Dlog[s] = noise * np.float32(3.0)
+        spikes = g.integers(0, cfg.V, size=cfg.L)
+        for i in range(cfg.L):
+            amp = cfg.spike_early if i < 8 else cfg.spike_late
+            Dlog[s, i, spikes[i]] += np.float32(amp)
+    return Dlog, h0
+
+
+def make_inputs(cfg: Config, zero_E: bool = False):
+    Wi, Wo, E = make_weights(cfg, zero_E=zero_E)
+    Dlog, h0 = make_sequences(cfg)
+    return dict(Wi=Wi, Wo=Wo, E=E, Dlog=Dlog, h0=h0)
