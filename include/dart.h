@@ -1,0 +1,178 @@
+/*
+ * dart.h -- C ABI of the GB300 (sm_103a) DARTree draft-tree construction path.
+ *
+ * The library builds the verification tree of one speculative-decoding round
+ * from a block drafter's position-wise logits, following the paper "DARTree:
+ * Speculative Diffusion Decoding with Autoregressive Draft Trees"
+ * (arXiv 2608.13524):
+ *   - Algorithm 1: for every depth d = 1..L, all retained prefixes S_{d-1}
+ *     are scored in one batch by the correction head, every child is ranked
+ *     by the Eq. 5 path score s_beta = sum_i log q~_i(u_i) + beta*d, the
+ *     global top-W children form S_d, and their correction states are
+ *     updated;
+ *   - Sec. 3.3 / Lemma 1: the complete supertree S is pruned to the budget B
+ *     with one global top-B (equal to best-first heap selection for
+ *     beta <= 0), and flattened for tree-attention verification (Sec. 2.3).
+ *
+ * Correction head (the paper leaves its form open; this is the fallback head):
+ *   h_c = RMSNorm(h_p + W_o . SiLU(W_i . [h_p ; E[t_c]]))   (no gain)
+ * Corrected child distribution of a node with state h at depth d-1:
+ *   z[v]  = (Dlog[d-1][v] + E[v] . h) / T'   (T' = T if T > 0, else 1)
+ *   log q~[v] = min(z[v] - logsumexp_v z, 0)
+ * The LM head is tied to the embedding table E.  The candidate set is the
+ * whole vocabulary ("Full" in Appendix D); each node keeps its top-k
+ * children by (log q~ desc, token asc), and S_d is the top-W of those
+ * candidates by (score desc, parent slot asc, rank asc).  For k >= W this
+ * equals the top-W over all children.  Candidates of score -inf are never
+ * retained, so |S_d| <= min(W, |S_{d-1}| * k).
+ *
+ * Node ids: id = (depth-1)*W + rank within S_depth; ancestors always have
+ * smaller ids.  Pruning keeps the top-B by (score desc, id asc).  Emission
+ * lists the kept nodes in ascending id (a topological order).
+ *
+ * Conventions for every entry point:
+ *   - all pointers are DEVICE pointers unless the name says _host;
+ *   - `stream` is a cudaStream_t (NULL = legacy default stream); work is
+ *     enqueued asynchronously and no call synchronises unless documented;
+ *   - return value: DART_OK or a negative dart_status; argument errors are
+ *     detected on the host before anything is enqueued;
+ *   - a handle must not be used from two streams or threads at once.
+ */
+#ifndef DART_H
+#define DART_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct dart_handle dart_handle; /* opaque; owns its device workspace */
+
+typedef enum {
+    DART_OK = 0,
+    DART_ERR_INVALID = -1,     /* bad argument, shape or pointer alignment */
+    DART_ERR_CUDA = -2,        /* a CUDA runtime/driver call failed */
+    DART_ERR_NOMEM = -3,       /* device or host allocation failed */
+    DART_ERR_TIMEOUT = -4,     /* a device-side wait gave up (reported by dart_status_sync) */
+    DART_ERR_STATE = -5,       /* call out of order (e.g. depth skipped) */
+    DART_ERR_UNSUPPORTED = -6  /* device is not sm_103 / missing driver entry point */
+} dart_status;
+
+typedef enum { DART_F32 = 0, DART_BF16 = 1 } dart_dtype;
+
+/* Problem definition (Algorithm 1 inputs).
+ *   V      vocabulary size, 1 <= V < 2^24, V >= k
+ *   d      hidden size of the correction head, multiple of 64, 64 <= d <= 16384
+ *   L      draft block length gamma (number of depths), 1 <= L, L*W <= 1024
+ *   W      layer width (frontier size), 1 <= W <= 64
+ *   k      per-node candidate count, 1 <= k <= 64, W*k <= 4096
+ *   B      verification budget (non-root nodes kept), 1 <= B <= 1024
+ *   nseq   independent sequences sharing the weights, nseq*W <= 256
+ *   beta   depth bonus of Eq. 5, beta <= 0 (Lemma 1 precondition)
+ *   temperature  T >= 0; T > 0 divides the logits by T, T = 0 is greedy
+ *          scoring (no scaling)
+ *   rms_eps      RMSNorm epsilon (> 0)
+ *   pos_offset   position id of the root; a node at depth d gets pos_offset+d */
+typedef struct {
+    int V, d, L, W, k, B, nseq;
+    float beta, temperature, rms_eps;
+    int pos_offset;
+} dart_config;
+
+/* Emitted verification tree, caller-allocated, per sequence s:
+ *   tokens [nseq][B]  token id of each kept node (-1 in unused rows)
+ *   parents[nseq][B]  row of the parent in this array, -1 if the parent is
+ *                     the root (the committed context), -2 in unused rows
+ *   depths [nseq][B]  1..L (0 in unused rows)
+ *   pos_ids[nseq][B]  pos_offset + depth (-1 in unused rows)
+ *   scores [nseq][B]  Eq. 5 path score s_beta (-inf in unused rows)
+ *   n_nodes[nseq]     number of used rows, min(B, |S|)
+ *   mask   [nseq][B][ceil(B/64)]  ancestor bit mask: bit j of row i is set
+ *                     iff row j is row i or one of its ancestors (the root /
+ *                     context column is implicit and always visible); rows
+ *                     beyond n_nodes are zero.  u64 words, bit j%64 of word j/64. */
+typedef struct {
+    int32_t *tokens, *parents, *depths, *pos_ids;
+    float *scores;
+    int32_t *n_nodes;
+    uint64_t *mask;
+} dart_tree_out;
+
+/* Creates a handle for `cfg` and registers the head weights (Algorithm 1
+ * input g, plus the tied LM head).  Weights are borrowed, never copied, and
+ * must stay valid and unchanged for the handle's life:
+ *   W_i [d][2d], W_o [d][d], E [V][d], row-major, of type `wdtype`
+ *   (DART_BF16: bfloat16 with fp32 accumulation; DART_F32: float32 with
+ *   fp32 arithmetic throughout).  Pointers must be 16-byte aligned.
+ * Allocates the workspace for the worst case of cfg (synchronous
+ * allocation).  Requires a compute capability 10.3 device (GB300).
+ * On success *out receives the handle; on failure *out is NULL. */
+int dart_init_head(dart_handle **out, const dart_config *cfg, int wdtype,
+                   const void *W_i, const void *W_o, const void *E, void *stream);
+
+/* Algorithm 1, one iteration: expands depth `depth` (1..L, in order; depth 1
+ * restarts the round).  drafter_logits [nseq][L][V] float32 (row depth-1 is
+ * read), anchor_h [nseq][d] float32 = r_0 (read at depth 1 only, may be NULL
+ * afterwards).  Out of order -> DART_ERR_STATE. */
+int dart_expand_depth(dart_handle *h, int depth, const float *drafter_logits,
+                      const float *anchor_h, void *stream);
+
+/* Deferred pruning (Algorithm 1 final step, Lemma 1) and emission of the
+ * verification tree after depth L was expanded; else DART_ERR_STATE. */
+int dart_prune_and_emit(dart_handle *h, const dart_tree_out *out, void *stream);
+
+/* The whole round: dart_expand_depth for 1..L, then dart_prune_and_emit.
+ * Launched as one cached CUDA graph per distinct (inputs, outputs) pointer
+ * set unless the stream is being captured by the caller. */
+int dart_build_tree(dart_handle *h, const float *drafter_logits, const float *anchor_h,
+                    const dart_tree_out *out, void *stream);
+
+/* dart_build_tree on HOST buffers: copies drafter_logits_host [nseq][L][V]
+ * and anchor_host [nseq][d] to handle-owned device staging, builds the tree
+ * and copies it back into the host arrays of out_host (same layout as
+ * dart_tree_out).  Synchronises `stream` before returning.  Pinned host
+ * memory makes the copies asynchronous. */
+int dart_build_tree_host(dart_handle *h, const float *drafter_logits_host,
+                         const float *anchor_host, const dart_tree_out *out_host,
+                         void *stream);
+
+/* Test hook: copies S_depth of every sequence (after that depth was
+ * expanded): tok / parent_slot / score [nseq][W] (rank order; parent_slot
+ * -1 for children of the root, unused ranks tok -1, score -inf) and count
+ * [nseq].  Any output pointer may be NULL. */
+int dart_get_frontier(dart_handle *h, int depth, int32_t *tok, int32_t *parent_slot,
+                      float *score, int32_t *count, void *stream);
+
+/* Test hook: per expanded node of the most recent depth (rows
+ * s*P + p, P = max |S_{depth-1}|): its k best children tok/logq [rows][k] and
+ * the log-sum-exp of its scaled logits lse [rows].  *rows receives the row
+ * count (host int).  NULL outputs are skipped. */
+int dart_get_node_topk(dart_handle *h, int32_t *tok, float *logq, float *lse, int *rows,
+                       void *stream);
+
+/* Test hook: correction states r(u) [rows][d] float32 of the most recently
+ * retained frontier (after the head update of depth < L).  *rows as above. */
+int dart_get_states(dart_handle *h, float *states, int *rows, void *stream);
+
+/* Synchronises `stream` and returns (then clears) the device status word:
+ * DART_OK, or DART_ERR_TIMEOUT if a kernel's bounded wait gave up. */
+int dart_status_sync(dart_handle *h, void *stream);
+
+/* Profiling: when enabled, CUDA events bracket every LM-head scoring launch
+ * (forces non-graph launches); dart_profile_read returns the summed device
+ * time in ms and the launch count since the last read, and resets them. */
+int dart_set_profiling(dart_handle *h, int enable);
+int dart_profile_read(dart_handle *h, float *lmhead_ms, int *lmhead_launches);
+
+/* Number of kernel launches one dart_build_tree enqueues for this handle. */
+int dart_launches_per_round(dart_handle *h);
+
+void dart_destroy(dart_handle *h);
+const char *dart_status_string(int code);
+int dart_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* DART_H */

@@ -1,0 +1,748 @@
+// C ABI of the DARTree construction path: argument validation, workspace,
+// TMA tensor maps, per-depth orchestration of the kernels (Algorithm 1),
+// pruning/emission, CUDA-graph caching of whole rounds, the host-buffer
+// variant and the test hooks.  See include/dart.h for the contract.
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+
+#include <algorithm>
+#include <cmath>
+#include <cstdint>
+#include <cstdlib>
+#include <cstring>
+#include <new>
+#include <vector>
+
+#include "../../include/dart.h"
+#include "dart_device.cuh"
+#include "dart_kernels.h"
+
+using namespace dart;
+
+namespace {
+
+constexpr int kVersion = 1;
+constexpr int kMaxW = 64, kMaxK = 64, kMaxWK = 4096, kMaxSuper = 1024, kMaxB = 1024;
+constexpr int kMaxD = 16384;
+constexpr int kMaxV = (1 << 24) - 1;
+constexpr int kMaxProfilePairs = 8192;
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                  const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+    static EncodeTiledFn fn = nullptr;
+    if (!fn) {
+        void* p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<EncodeTiledFn>(p);
+    }
+    return fn;
+}
+
+// 2-D bf16 tensor [rows][inner] with a (64 x box_rows) box and 128-byte swizzle.
+bool encode_bf16_2d(CUtensorMap* m, const void* base, uint64_t inner, uint64_t rows, uint32_t box_rows) {
+    EncodeTiledFn fn = encode_fn();
+    if (!fn) return false;
+    cuuint64_t dims[2] = {inner, rows};
+    cuuint64_t strides[1] = {inner * 2};
+    cuuint32_t box[2] = {static_cast<cuuint32_t>(kBlockK), box_rows};
+    cuuint32_t estr[2] = {1, 1};
+    return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
+              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+bool aligned4(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 3u) == 0; }
+
+int ng_index(int NG) { return NG == 16 ? 0 : (NG == 32 ? 1 : 2); }
+
+struct DepthPlan {
+    int N, P, NG, G, nV, stages, smem;  // LM-head scoring
+    int Nc, Pn;                          // children (head update) at this depth
+    GemmArgs g1, g2;                     // head GEMMs (depth < L)
+    int g1_smem, g2_smem;
+};
+
+struct GraphEntry {
+    const void* key[9];
+    cudaGraphExec_t exec;
+};
+
+}  // namespace
+
+struct dart_handle {
+    dart_config cfg;
+    int wdtype;
+    const void *Wi, *Wo, *E;
+    int dev, num_sms, smem_optin;
+    std::vector<int> caps;
+    std::vector<DepthPlan> plans;
+    int next_depth;  // 1..L+1 (L+1 = all depths expanded)
+    int cur;         // which state buffer holds the current frontier
+    int last_rows;
+    // workspace
+    float* hbuf[2];
+    __nv_bfloat16 *HL, *XL, *AL;
+    float *X32, *A32;
+    float* part;
+    float2* part_ms;
+    uint64_t* part_key;
+    float *node_logq, *node_lse;
+    int* node_tok;
+    int *tree_tok, *tree_parent, *tree_count;
+    float* tree_score;
+    int *child_prow, *child_tok, *seq_ticket, *status;
+    std::vector<void*> allocs;
+    CUtensorMap tmE, tmWi, tmWo, tmH[3], tmX[3], tmA[3];
+    // host-buffer staging
+    float *st_dlog, *st_anchor;
+    dart_tree_out st_out;
+    bool staged;
+    // graphs
+    cudaStream_t cap_stream;
+    std::vector<GraphEntry> graphs;
+    // profiling
+    bool profiling;
+    std::vector<cudaEvent_t> ev;
+    int ev_used;
+};
+
+namespace {
+
+int cuda_err(cudaError_t e) { return e == cudaSuccess ? DART_OK : DART_ERR_CUDA; }
+
+template <typename T>
+int dalloc(dart_handle* h, T** p, size_t count) {
+    void* q = nullptr;
+    if (count == 0) count = 1;
+    if (cudaMalloc(&q, count * sizeof(T)) != cudaSuccess) return DART_ERR_NOMEM;
+    h->allocs.push_back(q);
+    *p = static_cast<T*>(q);
+    return DART_OK;
+}
+
+int validate_cfg(const dart_config* c) {
+    if (!c) return DART_ERR_INVALID;
+    if (c->V < 1 || c->V > kMaxV) return DART_ERR_INVALID;
+    if (c->d < 64 || c->d > kMaxD || c->d % 64) return DART_ERR_INVALID;
+    if (c->L < 1 || c->W < 1 || c->W > kMaxW || c->L * c->W > kMaxSuper) return DART_ERR_INVALID;
+    if (c->k < 1 || c->k > kMaxK || c->k > c->V || c->W * c->k > kMaxWK) return DART_ERR_INVALID;
+    if (c->B < 1 || c->B > kMaxB) return DART_ERR_INVALID;
+    if (c->nseq < 1 || c->nseq * c->W > kNPadMax) return DART_ERR_INVALID;
+    if (!(c->beta <= 0.0f) || !std::isfinite(c->beta)) return DART_ERR_INVALID;  // Lemma 1 needs beta <= 0
+    if (!(c->temperature >= 0.0f) || !std::isfinite(c->temperature)) return DART_ERR_INVALID;
+    if (!(c->rms_eps > 0.0f) || !std::isfinite(c->rms_eps)) return DART_ERR_INVALID;
+    return DART_OK;
+}
+
+int pick_ng_tc(int N) { return N <= 16 ? 16 : (N <= 32 ? 32 : 64); }
+int pick_ng_f32(int N) { return N <= 16 ? 16 : 32; }
+
+// Split-K GEMM plan: M = d output features, K reduction, Nc nodes.
+GemmArgs gemm_plan(const dart_handle* h, int K, int Nc, int lo_kb_end, bool tc) {
+    GemmArgs g;
+    std::memset(&g, 0, sizeof g);
+    const int d = h->cfg.d;
+    g.M = d;
+    g.K = K;
+    g.N = Nc;
+    g.KB = K / kBlockK;
+    g.lo_kb_end = lo_kb_end;
+    g.bhalf = kNPadMax;
+    if (tc) {
+        g.NG = pick_ng_tc(Nc);
+        g.G = (Nc + g.NG - 1) / g.NG;
+        g.MT = (d + kTileM - 1) / kTileM;
+        g.S = std::max(1, std::min(g.KB, h->num_sms / (g.MT * g.G)));
+    } else {
+        g.NG = 16;
+        g.G = (Nc + 15) / 16;
+        g.MT = (d + 63) / 64;
+        g.S = std::max(1, std::min(K / 32, (2 * h->num_sms) / (g.MT * g.G)));
+    }
+    return g;
+}
+
+int tc_stages(int smem_optin, int stage_bytes, int fixed) {
+    int s = (smem_optin - fixed) / stage_bytes;
+    return std::min(16, s);
+}
+
+int build_plans(dart_handle* h) {
+    const dart_config& c = h->cfg;
+    const bool tc = h->wdtype == DART_BF16;
+    h->caps.assign(c.L + 1, 1);
+    for (int i = 1; i <= c.L; i++) h->caps[i] = std::min(c.W, h->caps[i - 1] * c.k);
+    h->plans.resize(c.L + 1);
+    const int tiles = (c.V + kTileM - 1) / kTileM;
+    for (int dep = 1; dep <= c.L; dep++) {
+        DepthPlan& p = h->plans[dep];
+        p.P = h->caps[dep - 1];
+        p.N = c.nseq * p.P;
+        p.NG = tc ? pick_ng_tc(p.N) : pick_ng_f32(p.N);
+        p.G = (p.N + p.NG - 1) / p.NG;
+        p.nV = std::max(1, std::min(h->num_sms / p.G, tiles));
+        if (tc) {
+            const int fixed = lmhead_tc_fixed_smem(p.NG, c.k, 16);
+            p.stages = tc_stages(h->smem_optin, tc_stage_bytes(p.NG), fixed);
+            if (p.stages < 2) return DART_ERR_UNSUPPORTED;
+            p.smem = lmhead_tc_fixed_smem(p.NG, c.k, p.stages) + p.stages * tc_stage_bytes(p.NG);
+        } else {
+            p.stages = 0;
+            p.smem = lmhead_f32_smem(p.NG, c.k);
+            if (p.smem > h->smem_optin) return DART_ERR_UNSUPPORTED;
+        }
+        p.Pn = h->caps[dep];
+        p.Nc = c.nseq * p.Pn;
+        if (dep < c.L) {
+            p.g1 = gemm_plan(h, 2 * c.d, p.Nc, c.d / kBlockK, tc);
+            p.g2 = gemm_plan(h, c.d, p.Nc, c.d / kBlockK, tc);
+            if (tc) {
+                const int sb = tc_stage_bytes(p.g1.NG);
+                p.g1.stages = std::min(tc_stages(h->smem_optin, sb, gemm_tc_fixed_smem(16)), 8);
+                p.g2.stages = p.g1.stages;
+                if (p.g1.stages < 2) return DART_ERR_UNSUPPORTED;
+                p.g1_smem = gemm_tc_fixed_smem(p.g1.stages) + p.g1.stages * sb;
+                p.g2_smem = p.g1_smem;
+            }
+        }
+    }
+    return DART_OK;
+}
+
+size_t max_part_floats(const dart_handle* h) {
+    size_t m = 1;
+    for (int dep = 1; dep < h->cfg.L; dep++) {
+        const DepthPlan& p = h->plans[dep];
+        m = std::max(m, static_cast<size_t>(p.g1.S) * p.Nc * h->cfg.d);
+        m = std::max(m, static_cast<size_t>(p.g2.S) * p.Nc * h->cfg.d);
+    }
+    return m;
+}
+
+int alloc_workspace(dart_handle* h) {
+    const dart_config& c = h->cfg;
+    const size_t d = c.d;
+    int rc = DART_OK;
+    size_t max_nvn = 1;
+    int max_nV = 1;
+    for (int dep = 1; dep <= c.L; dep++) {
+        max_nvn = std::max(max_nvn, static_cast<size_t>(h->plans[dep].nV) * h->plans[dep].N);
+        max_nV = std::max(max_nV, h->plans[dep].nV);
+    }
+    const size_t super = static_cast<size_t>(c.nseq) * c.L * c.W;
+#define DART_ALLOC(ptr, n) \
+    if (rc == DART_OK) rc = dalloc(h, &(ptr), (n));
+    DART_ALLOC(h->hbuf[0], kNPadMax * d)
+    DART_ALLOC(h->hbuf[1], kNPadMax * d)
+    if (h->wdtype == DART_BF16) {
+        DART_ALLOC(h->HL, 2 * kNPadMax * d)
+        DART_ALLOC(h->XL, 2 * kNPadMax * 2 * d)
+        DART_ALLOC(h->AL, 2 * kNPadMax * d)
+    } else {
+        DART_ALLOC(h->X32, kNPadMax * 2 * d)
+        DART_ALLOC(h->A32, kNPadMax * d)
+    }
+    DART_ALLOC(h->part, max_part_floats(h))
+    DART_ALLOC(h->part_ms, max_nvn)
+    DART_ALLOC(h->part_key, max_nvn * c.k)
+    DART_ALLOC(h->node_logq, static_cast<size_t>(kNPadMax) * c.k)
+    DART_ALLOC(h->node_tok, static_cast<size_t>(kNPadMax) * c.k)
+    DART_ALLOC(h->node_lse, kNPadMax)
+    DART_ALLOC(h->tree_tok, super)
+    DART_ALLOC(h->tree_parent, super)
+    DART_ALLOC(h->tree_score, super)
+    DART_ALLOC(h->tree_count, static_cast<size_t>(c.nseq) * c.L)
+    DART_ALLOC(h->child_prow, kNPadMax)
+    DART_ALLOC(h->child_tok, kNPadMax)
+    DART_ALLOC(h->seq_ticket, c.nseq)
+    DART_ALLOC(h->status, 1)
+#undef DART_ALLOC
+    if (rc != DART_OK) return rc;
+    // zeroed once: stale rows of the operand buffers are always finite
+    for (void* p : {static_cast<void*>(h->hbuf[0]), static_cast<void*>(h->hbuf[1])})
+        if (cudaMemset(p, 0, kNPadMax * d * sizeof(float)) != cudaSuccess) return DART_ERR_CUDA;
+    if (h->wdtype == DART_BF16) {
+        if (cudaMemset(h->HL, 0, 2 * kNPadMax * d * 2) != cudaSuccess) return DART_ERR_CUDA;
+        if (cudaMemset(h->XL, 0, 2 * kNPadMax * 2 * d * 2) != cudaSuccess) return DART_ERR_CUDA;
+        if (cudaMemset(h->AL, 0, 2 * kNPadMax * d * 2) != cudaSuccess) return DART_ERR_CUDA;
+    } else {
+        if (cudaMemset(h->X32, 0, kNPadMax * 2 * d * 4) != cudaSuccess) return DART_ERR_CUDA;
+        if (cudaMemset(h->A32, 0, kNPadMax * d * 4) != cudaSuccess) return DART_ERR_CUDA;
+    }
+    if (cudaMemset(h->seq_ticket, 0, c.nseq * sizeof(int)) != cudaSuccess) return DART_ERR_CUDA;
+    if (cudaMemset(h->status, 0, sizeof(int)) != cudaSuccess) return DART_ERR_CUDA;
+    if (cudaMemset(h->tree_count, 0, c.nseq * c.L * sizeof(int)) != cudaSuccess) return DART_ERR_CUDA;
+    // one-time kernel attributes
+    int max_sel = 0;
+    for (int dep = 1; dep <= c.L; dep++) max_sel = std::max(max_sel, merge_select_smem(h->plans[dep].nV, c.k, c.W));
+    if (select_set_smem_limits(std::max(max_sel, 48 * 1024)) != cudaSuccess) return DART_ERR_CUDA;
+    if (h->wdtype == DART_BF16) {
+        if (tc_set_smem_limits(h->smem_optin) != cudaSuccess) return DART_ERR_CUDA;
+    } else {
+        if (f32_set_smem_limits(h->smem_optin) != cudaSuccess) return DART_ERR_CUDA;
+    }
+    (void)max_nV;
+    return DART_OK;
+}
+
+int make_tensor_maps(dart_handle* h) {
+    const dart_config& c = h->cfg;
+    const uint64_t d = c.d;
+    bool ok = encode_bf16_2d(&h->tmE, h->E, d, c.V, kTileM) && encode_bf16_2d(&h->tmWi, h->Wi, 2 * d, d, kTileM) &&
+              encode_bf16_2d(&h->tmWo, h->Wo, d, d, kTileM);
+    const int ngs[3] = {16, 32, 64};
+    for (int i = 0; i < 3 && ok; i++) {
+        ok = encode_bf16_2d(&h->tmH[i], h->HL, d, 2 * kNPadMax, ngs[i]) &&
+             encode_bf16_2d(&h->tmX[i], h->XL, 2 * d, 2 * kNPadMax, ngs[i]) &&
+             encode_bf16_2d(&h->tmA[i], h->AL, d, 2 * kNPadMax, ngs[i]);
+    }
+    return ok ? DART_OK : DART_ERR_UNSUPPORTED;
+}
+
+void release(dart_handle* h) {
+    for (auto& g : h->graphs) cudaGraphExecDestroy(g.exec);
+    h->graphs.clear();
+    for (cudaEvent_t e : h->ev) cudaEventDestroy(e);
+    h->ev.clear();
+    if (h->cap_stream) cudaStreamDestroy(h->cap_stream);
+    h->cap_stream = nullptr;
+    for (void* p : h->allocs) cudaFree(p);
+    h->allocs.clear();
+}
+
+// ---------------------------------------------------------------- enqueue
+
+int enqueue_depth(dart_handle* h, int dep, const float* dlog, const float* anchor, cudaStream_t st) {
+    const dart_config& c = h->cfg;
+    const DepthPlan& p = h->plans[dep];
+    const bool tc = h->wdtype == DART_BF16;
+    cudaError_t e = cudaSuccess;
+    if (dep == 1) {
+        e = launch_prep_anchor(anchor, c.nseq, c.d, h->hbuf[0], tc ? h->HL : nullptr, kNPadMax, st);
+        if (e != cudaSuccess) return DART_ERR_CUDA;
+        h->cur = 0;
+    }
+    // 1) LM-head scoring of every prefix in S_{dep-1} (fused log-sum-exp / top-k)
+    LmheadArgs la;
+    std::memset(&la, 0, sizeof la);
+    la.V = c.V;
+    la.d = c.d;
+    la.N = p.N;
+    la.NG = p.NG;
+    la.G = p.G;
+    la.nV = p.nV;
+    la.k = c.k;
+    la.tiles = (c.V + kTileM - 1) / kTileM;
+    la.P = p.P;
+    la.invT = c.temperature > 0.0f ? 1.0f / c.temperature : 1.0f;
+    la.dlog = dlog;
+    la.dlog_seq_stride = static_cast<long long>(c.L) * c.V;
+    la.dlog_row_off = static_cast<long long>(dep - 1) * c.V;
+    la.bhalf = kNPadMax;
+    la.stages = p.stages;
+    la.part_ms = h->part_ms;
+    la.part_key = h->part_key;
+    la.status = h->status;
+    la.h32 = h->hbuf[h->cur];
+    la.E32 = static_cast<const float*>(h->E);
+    const bool prof = h->profiling && h->ev_used + 2 <= kMaxProfilePairs * 2;
+    if (prof) {
+        while (static_cast<int>(h->ev.size()) < h->ev_used + 2) {
+            cudaEvent_t ev;
+            if (cudaEventCreate(&ev) != cudaSuccess) return DART_ERR_CUDA;
+            h->ev.push_back(ev);
+        }
+        cudaEventRecord(h->ev[h->ev_used], st);
+    }
+    e = tc ? launch_lmhead_tc(&h->tmE, &h->tmH[ng_index(p.NG)], la, p.smem, st) : launch_lmhead_f32(la, st);
+    if (e != cudaSuccess) return DART_ERR_CUDA;
+    if (prof) {
+        cudaEventRecord(h->ev[h->ev_used + 1], st);
+        h->ev_used += 2;
+    }
+    // 2) merge partials, log q~, Eq. 5 scores, global top-W -> S_dep
+    SelectArgs sa;
+    std::memset(&sa, 0, sizeof sa);
+    sa.N = p.N;
+    sa.P = p.P;
+    sa.k = c.k;
+    sa.nV = p.nV;
+    sa.W = c.W;
+    sa.L = c.L;
+    sa.nseq = c.nseq;
+    sa.dep = dep;
+    sa.Pn = p.Pn;
+    sa.beta = c.beta;
+    sa.part_ms = h->part_ms;
+    sa.part_key = h->part_key;
+    sa.node_logq = h->node_logq;
+    sa.node_tok = h->node_tok;
+    sa.node_lse = h->node_lse;
+    sa.tree_tok = h->tree_tok;
+    sa.tree_parent = h->tree_parent;
+    sa.tree_score = h->tree_score;
+    sa.tree_count = h->tree_count;
+    sa.child_prow = h->child_prow;
+    sa.child_tok = h->child_tok;
+    sa.seq_ticket = h->seq_ticket;
+    sa.status = h->status;
+    if (launch_merge_select(sa, st) != cudaSuccess) return DART_ERR_CUDA;
+    h->last_rows = p.N;
+    if (dep == c.L) return DART_OK;
+    // 3) correction-head update of the retained children (Algorithm 1, state update)
+    const float* hcur = h->hbuf[h->cur];
+    float* hnext = h->hbuf[1 - h->cur];
+    if (launch_gather_x(p.Nc, c.d, h->child_prow, h->child_tok, hcur, h->E, tc ? 1 : 0, h->XL, kNPadMax, h->X32,
+                        st) != cudaSuccess)
+        return DART_ERR_CUDA;
+    GemmArgs g1 = p.g1, g2 = p.g2;
+    g1.out = h->part;
+    g2.out = h->part;
+    g1.status = g2.status = h->status;
+    if (tc) {
+        e = launch_gemm_tc(&h->tmWi, &h->tmX[ng_index(g1.NG)], g1, p.g1_smem, st);
+    } else {
+        g1.A32 = static_cast<const float*>(h->Wi);
+        g1.B32 = h->X32;
+        e = launch_gemm_f32(g1, st);
+    }
+    if (e != cudaSuccess) return DART_ERR_CUDA;
+    if (launch_silu_split(p.Nc, c.d, g1.S, h->part, tc ? h->AL : nullptr, kNPadMax, h->A32, st) != cudaSuccess)
+        return DART_ERR_CUDA;
+    if (tc) {
+        e = launch_gemm_tc(&h->tmWo, &h->tmA[ng_index(g2.NG)], g2, p.g2_smem, st);
+    } else {
+        g2.A32 = static_cast<const float*>(h->Wo);
+        g2.B32 = h->A32;
+        e = launch_gemm_f32(g2, st);
+    }
+    if (e != cudaSuccess) return DART_ERR_CUDA;
+    if (launch_residual_norm(p.Nc, c.d, g2.S, h->part, h->child_prow, hcur, c.rms_eps, hnext, tc ? h->HL : nullptr,
+                             kNPadMax, st) != cudaSuccess)
+        return DART_ERR_CUDA;
+    h->cur = 1 - h->cur;
+    h->last_rows = p.Nc;
+    return DART_OK;
+}
+
+int check_out(const dart_tree_out* o) {
+    if (!o || !o->tokens || !o->parents || !o->depths || !o->pos_ids || !o->scores || !o->n_nodes || !o->mask)
+        return DART_ERR_INVALID;
+    if (!aligned4(o->tokens) || !aligned4(o->parents) || !aligned4(o->depths) || !aligned4(o->pos_ids) ||
+        !aligned4(o->scores) || !aligned4(o->n_nodes) || (reinterpret_cast<uintptr_t>(o->mask) & 7u))
+        return DART_ERR_INVALID;
+    return DART_OK;
+}
+
+int enqueue_emit(dart_handle* h, const dart_tree_out* o, cudaStream_t st) {
+    const dart_config& c = h->cfg;
+    EmitArgs a;
+    a.L = c.L;
+    a.W = c.W;
+    a.B = c.B;
+    a.nseq = c.nseq;
+    a.pos_offset = c.pos_offset;
+    a.tree_tok = h->tree_tok;
+    a.tree_parent = h->tree_parent;
+    a.tree_score = h->tree_score;
+    a.tree_count = h->tree_count;
+    a.tokens = o->tokens;
+    a.parents = o->parents;
+    a.depths = o->depths;
+    a.pos_ids = o->pos_ids;
+    a.n_nodes = o->n_nodes;
+    a.scores = o->scores;
+    a.mask = o->mask;
+    a.status = h->status;
+    return launch_prune_emit(a, st) == cudaSuccess ? DART_OK : DART_ERR_CUDA;
+}
+
+int enqueue_round(dart_handle* h, const float* dlog, const float* anchor, const dart_tree_out* out, cudaStream_t st) {
+    for (int dep = 1; dep <= h->cfg.L; dep++) {
+        int rc = enqueue_depth(h, dep, dlog, anchor, st);
+        if (rc != DART_OK) return rc;
+    }
+    h->next_depth = h->cfg.L + 1;
+    return enqueue_emit(h, out, st);
+}
+
+int check_inputs(const dart_handle* h, const float* dlog, const float* anchor, bool need_anchor) {
+    if (!dlog || !aligned4(dlog)) return DART_ERR_INVALID;
+    if (need_anchor && (!anchor || !aligned4(anchor))) return DART_ERR_INVALID;
+    (void)h;
+    return DART_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+int dart_version(void) { return kVersion; }
+
+const char* dart_status_string(int code) {
+    switch (code) {
+        case DART_OK: return "ok";
+        case DART_ERR_INVALID: return "invalid argument";
+        case DART_ERR_CUDA: return "CUDA error";
+        case DART_ERR_NOMEM: return "out of memory";
+        case DART_ERR_TIMEOUT: return "device wait timed out";
+        case DART_ERR_STATE: return "call out of order";
+        case DART_ERR_UNSUPPORTED: return "unsupported device or configuration";
+        default: return "unknown status";
+    }
+}
+
+int dart_init_head(dart_handle** out, const dart_config* cfg, int wdtype, const void* W_i, const void* W_o,
+                   const void* E, void* stream) {
+    (void)stream;
+    if (!out) return DART_ERR_INVALID;
+    *out = nullptr;
+    int rc = validate_cfg(cfg);
+    if (rc != DART_OK) return rc;
+    if (wdtype != DART_F32 && wdtype != DART_BF16) return DART_ERR_INVALID;
+    if (!W_i || !W_o || !E || !aligned16(W_i) || !aligned16(W_o) || !aligned16(E)) return DART_ERR_INVALID;
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return DART_ERR_CUDA;
+    int major = 0, minor = 0, sms = 0, optin = 0;
+    if (cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) != cudaSuccess)
+        return DART_ERR_CUDA;
+    if (major != 10 || minor != 3) return DART_ERR_UNSUPPORTED;  // built for sm_103a only
+    dart_handle* h = new (std::nothrow) dart_handle();
+    if (!h) return DART_ERR_NOMEM;
+    h->cfg = *cfg;
+    h->wdtype = wdtype;
+    h->Wi = W_i;
+    h->Wo = W_o;
+    h->E = E;
+    h->dev = dev;
+    h->num_sms = sms;
+    h->smem_optin = optin;
+    h->next_depth = 1;
+    rc = build_plans(h);
+    if (rc == DART_OK) rc = alloc_workspace(h);
+    if (rc == DART_OK && wdtype == DART_BF16) rc = make_tensor_maps(h);
+    if (rc == DART_OK && cudaStreamCreateWithFlags(&h->cap_stream, cudaStreamNonBlocking) != cudaSuccess)
+        rc = DART_ERR_CUDA;
+    if (rc == DART_OK && cudaDeviceSynchronize() != cudaSuccess) rc = DART_ERR_CUDA;
+    if (rc != DART_OK) {
+        release(h);
+        delete h;
+        return rc;
+    }
+    *out = h;
+    return DART_OK;
+}
+
+int dart_expand_depth(dart_handle* h, int depth, const float* drafter_logits, const float* anchor_h, void* stream) {
+    if (!h) return DART_ERR_INVALID;
+    if (depth < 1 || depth > h->cfg.L) return DART_ERR_INVALID;
+    int rc = check_inputs(h, drafter_logits, anchor_h, depth == 1);
+    if (rc != DART_OK) return rc;
+    if (depth != 1 && depth != h->next_depth) return DART_ERR_STATE;
+    rc = enqueue_depth(h, depth, drafter_logits, anchor_h, static_cast<cudaStream_t>(stream));
+    h->next_depth = rc == DART_OK ? depth + 1 : 1;
+    return rc;
+}
+
+int dart_prune_and_emit(dart_handle* h, const dart_tree_out* out, void* stream) {
+    if (!h) return DART_ERR_INVALID;
+    int rc = check_out(out);
+    if (rc != DART_OK) return rc;
+    if (h->next_depth != h->cfg.L + 1) return DART_ERR_STATE;
+    return enqueue_emit(h, out, static_cast<cudaStream_t>(stream));
+}
+
+int dart_build_tree(dart_handle* h, const float* drafter_logits, const float* anchor_h, const dart_tree_out* out,
+                    void* stream) {
+    if (!h) return DART_ERR_INVALID;
+    int rc = check_inputs(h, drafter_logits, anchor_h, true);
+    if (rc == DART_OK) rc = check_out(out);
+    if (rc != DART_OK) return rc;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+    if (cudaStreamIsCapturing(st, &cs) != cudaSuccess) return DART_ERR_CUDA;
+    if (h->profiling || cs != cudaStreamCaptureStatusNone) {
+        rc = enqueue_round(h, drafter_logits, anchor_h, out, st);
+        if (rc != DART_OK) h->next_depth = 1;
+        return rc;
+    }
+    const void* key[9] = {drafter_logits, anchor_h, out->tokens, out->parents, out->depths,
+                          out->pos_ids,   out->scores, out->n_nodes, out->mask};
+    for (auto& g : h->graphs) {
+        if (std::memcmp(g.key, key, sizeof key) == 0) {
+            h->next_depth = h->cfg.L + 1;
+            h->last_rows = h->plans[h->cfg.L].N;
+            return cuda_err(cudaGraphLaunch(g.exec, st));
+        }
+    }
+    cudaGraph_t graph = nullptr;
+    if (cudaStreamBeginCapture(h->cap_stream, cudaStreamCaptureModeThreadLocal) != cudaSuccess) return DART_ERR_CUDA;
+    rc = enqueue_round(h, drafter_logits, anchor_h, out, h->cap_stream);
+    cudaError_t ce = cudaStreamEndCapture(h->cap_stream, &graph);
+    if (rc != DART_OK || ce != cudaSuccess) {
+        if (graph) cudaGraphDestroy(graph);
+        h->next_depth = 1;
+        return rc != DART_OK ? rc : DART_ERR_CUDA;
+    }
+    GraphEntry ge;
+    std::memcpy(ge.key, key, sizeof key);
+    ce = cudaGraphInstantiate(&ge.exec, graph, 0);
+    cudaGraphDestroy(graph);
+    if (ce != cudaSuccess) {
+        h->next_depth = 1;
+        return DART_ERR_CUDA;
+    }
+    h->graphs.push_back(ge);
+    return cuda_err(cudaGraphLaunch(ge.exec, st));
+}
+
+int dart_build_tree_host(dart_handle* h, const float* drafter_logits_host, const float* anchor_host,
+                         const dart_tree_out* out_host, void* stream) {
+    if (!h || !drafter_logits_host || !anchor_host) return DART_ERR_INVALID;
+    int rc = check_out(out_host);
+    if (rc != DART_OK) return rc;
+    const dart_config& c = h->cfg;
+    const size_t n_dlog = static_cast<size_t>(c.nseq) * c.L * c.V;
+    const size_t n_anchor = static_cast<size_t>(c.nseq) * c.d;
+    const size_t nB = static_cast<size_t>(c.nseq) * c.B;
+    const size_t nmask = nB * ((c.B + 63) / 64);
+    if (!h->staged) {
+        rc = dalloc(h, &h->st_dlog, n_dlog);
+        if (rc == DART_OK) rc = dalloc(h, &h->st_anchor, n_anchor);
+        if (rc == DART_OK) rc = dalloc(h, &h->st_out.tokens, nB);
+        if (rc == DART_OK) rc = dalloc(h, &h->st_out.parents, nB);
+        if (rc == DART_OK) rc = dalloc(h, &h->st_out.depths, nB);
+        if (rc == DART_OK) rc = dalloc(h, &h->st_out.pos_ids, nB);
+        if (rc == DART_OK) rc = dalloc(h, &h->st_out.scores, nB);
+        if (rc == DART_OK) rc = dalloc(h, &h->st_out.n_nodes, static_cast<size_t>(c.nseq));
+        if (rc == DART_OK) rc = dalloc(h, &h->st_out.mask, nmask);
+        if (rc != DART_OK) return rc;
+        h->staged = true;
+    }
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    if (cudaMemcpyAsync(h->st_dlog, drafter_logits_host, n_dlog * 4, cudaMemcpyHostToDevice, st) != cudaSuccess ||
+        cudaMemcpyAsync(h->st_anchor, anchor_host, n_anchor * 4, cudaMemcpyHostToDevice, st) != cudaSuccess)
+        return DART_ERR_CUDA;
+    rc = dart_build_tree(h, h->st_dlog, h->st_anchor, &h->st_out, stream);
+    if (rc != DART_OK) return rc;
+    const dart_tree_out& d = h->st_out;
+    const dart_tree_out& o = *out_host;
+    cudaError_t e = cudaSuccess;
+    e = cudaMemcpyAsync(o.tokens, d.tokens, nB * 4, cudaMemcpyDeviceToHost, st);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(o.parents, d.parents, nB * 4, cudaMemcpyDeviceToHost, st);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(o.depths, d.depths, nB * 4, cudaMemcpyDeviceToHost, st);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(o.pos_ids, d.pos_ids, nB * 4, cudaMemcpyDeviceToHost, st);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(o.scores, d.scores, nB * 4, cudaMemcpyDeviceToHost, st);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(o.n_nodes, d.n_nodes, c.nseq * 4, cudaMemcpyDeviceToHost, st);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(o.mask, d.mask, nmask * 8, cudaMemcpyDeviceToHost, st);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+    return cuda_err(e);
+}
+
+int dart_get_frontier(dart_handle* h, int depth, int32_t* tok, int32_t* parent_slot, float* score, int32_t* count,
+                      void* stream) {
+    if (!h || depth < 1 || depth > h->cfg.L) return DART_ERR_INVALID;
+    if (depth >= h->next_depth) return DART_ERR_STATE;
+    const dart_config& c = h->cfg;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    const size_t W = c.W;
+    cudaError_t e = cudaSuccess;
+    for (int s = 0; s < c.nseq && e == cudaSuccess; s++) {
+        const size_t src = (static_cast<size_t>(s) * c.L + depth - 1) * W;
+        if (tok) e = cudaMemcpyAsync(tok + s * W, h->tree_tok + src, W * 4, cudaMemcpyDeviceToDevice, st);
+        if (parent_slot && e == cudaSuccess)
+            e = cudaMemcpyAsync(parent_slot + s * W, h->tree_parent + src, W * 4, cudaMemcpyDeviceToDevice, st);
+        if (score && e == cudaSuccess)
+            e = cudaMemcpyAsync(score + s * W, h->tree_score + src, W * 4, cudaMemcpyDeviceToDevice, st);
+        if (count && e == cudaSuccess)
+            e = cudaMemcpyAsync(count + s, h->tree_count + s * c.L + depth - 1, 4, cudaMemcpyDeviceToDevice, st);
+    }
+    return cuda_err(e);
+}
+
+int dart_get_node_topk(dart_handle* h, int32_t* tok, float* logq, float* lse, int* rows, void* stream) {
+    if (!h) return DART_ERR_INVALID;
+    if (h->next_depth < 2) return DART_ERR_STATE;
+    const int dep = h->next_depth - 1;
+    const int N = h->plans[dep].N;
+    if (rows) *rows = N;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    const size_t nk = static_cast<size_t>(N) * h->cfg.k;
+    cudaError_t e = cudaSuccess;
+    if (tok) e = cudaMemcpyAsync(tok, h->node_tok, nk * 4, cudaMemcpyDeviceToDevice, st);
+    if (logq && e == cudaSuccess) e = cudaMemcpyAsync(logq, h->node_logq, nk * 4, cudaMemcpyDeviceToDevice, st);
+    if (lse && e == cudaSuccess) e = cudaMemcpyAsync(lse, h->node_lse, N * 4, cudaMemcpyDeviceToDevice, st);
+    return cuda_err(e);
+}
+
+int dart_get_states(dart_handle* h, float* states, int* rows, void* stream) {
+    if (!h) return DART_ERR_INVALID;
+    if (h->next_depth < 2) return DART_ERR_STATE;
+    const int dep = h->next_depth - 1;
+    const int R = dep < h->cfg.L ? h->plans[dep].Nc : h->plans[dep].N;
+    if (rows) *rows = R;
+    if (!states) return DART_OK;
+    return cuda_err(cudaMemcpyAsync(states, h->hbuf[h->cur], static_cast<size_t>(R) * h->cfg.d * 4,
+                                    cudaMemcpyDeviceToDevice, static_cast<cudaStream_t>(stream)));
+}
+
+int dart_status_sync(dart_handle* h, void* stream) {
+    if (!h) return DART_ERR_INVALID;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    int word = 0;
+    if (cudaStreamSynchronize(st) != cudaSuccess) return DART_ERR_CUDA;
+    if (cudaMemcpy(&word, h->status, sizeof word, cudaMemcpyDeviceToHost) != cudaSuccess) return DART_ERR_CUDA;
+    if (cudaMemset(h->status, 0, sizeof word) != cudaSuccess) return DART_ERR_CUDA;
+    if (word & kDevTimeout) return DART_ERR_TIMEOUT;
+    if (word & kDevOrphan) return DART_ERR_STATE;
+    return DART_OK;
+}
+
+int dart_set_profiling(dart_handle* h, int enable) {
+    if (!h) return DART_ERR_INVALID;
+    h->profiling = enable != 0;
+    h->ev_used = 0;
+    return DART_OK;
+}
+
+int dart_profile_read(dart_handle* h, float* lmhead_ms, int* lmhead_launches) {
+    if (!h) return DART_ERR_INVALID;
+    float total = 0.0f;
+    const int pairs = h->ev_used / 2;
+    if (pairs > 0 && cudaEventSynchronize(h->ev[h->ev_used - 1]) != cudaSuccess) return DART_ERR_CUDA;
+    for (int i = 0; i < pairs; i++) {
+        float ms = 0.0f;
+        if (cudaEventElapsedTime(&ms, h->ev[2 * i], h->ev[2 * i + 1]) != cudaSuccess) return DART_ERR_CUDA;
+        total += ms;
+    }
+    if (lmhead_ms) *lmhead_ms = total;
+    if (lmhead_launches) *lmhead_launches = pairs;
+    h->ev_used = 0;
+    return DART_OK;
+}
+
+int dart_launches_per_round(dart_handle* h) {
+    if (!h) return DART_ERR_INVALID;
+    const int L = h->cfg.L;
+    return 1 + 2 * L + 5 * (L - 1) + 1;
+}
+
+void dart_destroy(dart_handle* h) {
+    if (!h) return;
+    cudaDeviceSynchronize();
+    release(h);
+    delete h;
+}
+
+}  // extern "C"

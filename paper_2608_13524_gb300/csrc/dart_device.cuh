@@ -1,0 +1,372 @@
+// Device-side building blocks of the DARTree construction path (sm_103a):
+// inline-PTX wrappers for mbarrier / TMA / tcgen05, order-preserving 64-bit
+// selection keys, a block-wide radix select, and the fused LM-head epilogue
+// (online log-sum-exp + per-node top-k) shared by the bf16 tensor-core kernel
+// and the fp32 CUDA-core kernel.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace dart {
+
+// Device status word bits (read back by dart_status_sync).
+constexpr int kDevTimeout = 1;      // a bounded wait gave up
+constexpr int kDevOrphan = 2;       // pruning kept a node whose parent was cut (impossible for beta <= 0)
+
+// A wait that has not completed after this long means a bug; give up.
+constexpr unsigned long long kWaitLimitNs = 2000000000ull;  // 2 s
+
+constexpr int kNPadMax = 256;       // max nodes per depth (nseq * W)
+constexpr int kTileM = 128;         // MMA M: vocabulary rows / output features per tile
+constexpr int kBlockK = 64;         // bf16 elements per 128-byte swizzled row
+constexpr int kCandCap = 128;       // per-node candidate slots per tile (one tile worth)
+constexpr int kEpiThreads = 128;    // 4 epilogue warps
+constexpr int kEpiBarrier = 1;      // named barrier id used by the epilogue warps
+
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+    return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+__device__ __forceinline__ unsigned long long globaltimer_ns() {
+    unsigned long long t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+
+__device__ __forceinline__ void named_bar_sync(int id, int nthreads) {
+    asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(nthreads) : "memory");
+}
+
+// ------------------------------------------------------------------ mbarrier
+
+__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count) : "memory");
+}
+__device__ __forceinline__ void fence_mbar_init() {
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t* bar, uint32_t bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)), "r"(bytes)
+                 : "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
+        " selp.u32 %0, 1, 0, p;\n}\n"
+        : "=r"(ok)
+        : "r"(smem_u32(bar)), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+// Waits for the phase with the given parity.  Gives up (returns false) when
+// *abort becomes nonzero or after kWaitLimitNs.
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort) {
+    if (mbar_try_wait(bar, parity)) return true;
+    const unsigned long long t0 = globaltimer_ns();
+    for (;;) {
+        if (mbar_try_wait(bar, parity)) return true;
+        if (*abort) return false;
+        if (globaltimer_ns() - t0 > kWaitLimitNs) return false;
+    }
+}
+
+// ----------------------------------------------------------------------- TMA
+
+__device__ __forceinline__ uint64_t l2_policy_evict_first() {
+    uint64_t p;
+    asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
+    return p;
+}
+__device__ __forceinline__ uint64_t l2_policy_evict_last() {
+    uint64_t p;
+    asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(p));
+    return p;
+}
+// 2-D tiled bulk copy global -> shared, completing on `bar` (x = innermost).
+__device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, uint64_t* bar, int x, int y,
+                                            uint64_t policy) {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint"
+        " [%0], [%1, {%3, %4}], [%2], %5;" ::"r"(smem_u32(dst)),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(smem_u32(bar)), "r"(x), "r"(y), "l"(policy)
+        : "memory");
+}
+
+// ------------------------------------------------------------------- tcgen05
+
+__device__ __forceinline__ void tmem_alloc(uint32_t* slot, uint32_t ncols) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(slot)),
+                 "r"(ncols)
+                 : "memory");
+}
+__device__ __forceinline__ void tmem_relinquish() {
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols) : "memory");
+}
+__device__ __forceinline__ void tc_fence_before() {
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tc_fence_after() {
+    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+// D[tmem] (+)= A[smem] * B[smem]^T, bf16 inputs, fp32 accumulation.
+__device__ __forceinline__ void tc_mma_bf16(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
+                                            uint32_t accumulate) {
+    asm volatile(
+        "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+        " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(tmem_d),
+        "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+        : "memory");
+}
+// Arrives once on `bar` when every tcgen05 op issued so far by this thread is done.
+__device__ __forceinline__ void tc_commit(uint64_t* bar) {
+    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
+                     smem_u32(bar))
+                 : "memory");
+}
+// 32 TMEM lanes x 16 consecutive 32-bit columns: thread i of the warp gets lane
+// (warp's lane quarter + i), columns [col, col+16).
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, float (&v)[16]) {
+    uint32_t r[16];
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15},"
+        " [%16];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+        : "r"(taddr));
+    // the registers are tied to the wait so no use can move above it
+    asm volatile("tcgen05.wait::ld.sync.aligned;"
+                 : "+r"(r[0]), "+r"(r[1]), "+r"(r[2]), "+r"(r[3]), "+r"(r[4]), "+r"(r[5]), "+r"(r[6]),
+                   "+r"(r[7]), "+r"(r[8]), "+r"(r[9]), "+r"(r[10]), "+r"(r[11]), "+r"(r[12]), "+r"(r[13]),
+                   "+r"(r[14]), "+r"(r[15])
+                 :
+                 : "memory");
+#pragma unroll
+    for (int i = 0; i < 16; i++) v[i] = __uint_as_float(r[i]);
+}
+
+// Shared-memory matrix descriptor of a K-major operand tile written by TMA
+// with 128-byte swizzling: rows of 128 bytes, 8-row groups 1024 bytes apart
+// (stride byte offset), tile base 1024-byte aligned; the leading byte offset
+// is unused because one MMA's K extent (32 bytes) stays inside a swizzle row.
+__device__ __forceinline__ uint64_t sdesc_sw128(uint32_t saddr) {
+    uint64_t d = 0;
+    d |= static_cast<uint64_t>((saddr >> 4) & 0x3FFFu);          // start address >> 4
+    d |= static_cast<uint64_t>((1024u >> 4) & 0x3FFFu) << 32;    // stride byte offset >> 4
+    d |= static_cast<uint64_t>(1u) << 46;                        // descriptor version (tcgen05)
+    d |= static_cast<uint64_t>(2u) << 61;                        // swizzle mode: 128B
+    return d;
+}
+// Instruction descriptor, kind::f16: D fp32, A and B bf16, both K-major.
+__host__ __device__ constexpr uint32_t idesc_bf16_f32(int M, int N) {
+    return (1u << 4) | (1u << 7) | (1u << 10) | (static_cast<uint32_t>(N >> 3) << 17) |
+           (static_cast<uint32_t>(M >> 4) << 24);
+}
+
+// ---------------------------------------------------------------- selection
+//
+// A candidate is a 64-bit key whose unsigned order is the selection order:
+// high word = order-preserving image of the fp32 value (larger value =
+// larger key), low word = ~index (smaller index wins ties).  Key 0 is below
+// every real candidate and marks empty slots.
+
+__device__ __forceinline__ uint32_t f32_ord(float f) {
+    uint32_t u = __float_as_uint(f);
+    return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+}
+__device__ __forceinline__ float f32_unord(uint32_t o) {
+    uint32_t u = (o & 0x80000000u) ? (o & 0x7FFFFFFFu) : ~o;
+    return __uint_as_float(u);
+}
+__device__ __forceinline__ uint64_t make_key(float v, uint32_t idx) {
+    if (v == 0.0f) v = 0.0f;  // -0 and +0 compare equal
+    return (static_cast<uint64_t>(f32_ord(v)) << 32) | static_cast<uint64_t>(0xFFFFFFFFu - idx);
+}
+__device__ __forceinline__ float key_val(uint64_t key) { return f32_unord(static_cast<uint32_t>(key >> 32)); }
+__device__ __forceinline__ uint32_t key_idx(uint64_t key) {
+    return 0xFFFFFFFFu - static_cast<uint32_t>(key & 0xFFFFFFFFull);
+}
+
+// Block-wide radix select: returns the kk-th largest of the n keys in shared
+// memory (1 <= kk <= n; keys distinct except for zeros).  Uses `hist` (256
+// u32) and `scal` (2 ints) of shared scratch.  Every thread of the block must
+// call it; it synchronises the block.
+__device__ __forceinline__ uint64_t block_kth_largest(const uint64_t* keys, int n, int kk, uint32_t* hist,
+                                                      int* scal) {
+    uint64_t prefix = 0, mask = 0;
+    int remaining = kk;
+    const int tid = threadIdx.x, nt = blockDim.x;
+    for (int shift = 56; shift >= 0; shift -= 8) {
+        for (int i = tid; i < 256; i += nt) hist[i] = 0;
+        __syncthreads();
+        for (int i = tid; i < n; i += nt) {
+            const uint64_t e = keys[i];
+            if ((e & mask) == prefix) atomicAdd(&hist[(e >> shift) & 255u], 1u);
+        }
+        __syncthreads();
+        if (tid < 32) {
+            // lane l owns digits 255-8l .. 248-8l (highest digits first)
+            uint32_t loc[8];
+            uint32_t sum = 0;
+#pragma unroll
+            for (int j = 0; j < 8; j++) {
+                loc[j] = hist[255 - 8 * tid - j];
+                sum += loc[j];
+            }
+            uint32_t incl = sum;
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+                uint32_t t = __shfl_up_sync(0xFFFFFFFFu, incl, o);
+                if (tid >= o) incl += t;
+            }
+            const unsigned hit = __ballot_sync(0xFFFFFFFFu, incl >= static_cast<uint32_t>(remaining));
+            const int lane = __ffs(hit) - 1;
+            if (tid == lane) {
+                uint32_t cum = incl - sum;
+                int digit = 255 - 8 * lane;
+#pragma unroll
+                for (int j = 0; j < 8; j++) {
+                    if (cum + loc[j] >= static_cast<uint32_t>(remaining)) {
+                        digit = 255 - 8 * lane - j;
+                        break;
+                    }
+                    cum += loc[j];
+                }
+                scal[0] = digit;
+                scal[1] = remaining - static_cast<int>(cum);
+            }
+        }
+        __syncthreads();
+        prefix |= static_cast<uint64_t>(scal[0]) << shift;
+        mask |= 255ull << shift;
+        remaining = scal[1];
+        __syncthreads();
+    }
+    return prefix;
+}
+
+// ------------------------------------------------ fused LM-head epilogue
+//
+// Per node (column) of a 128-row tile, every epilogue thread owns one
+// vocabulary row.  It keeps, per warp and node, a running (max, sum exp) for
+// the log-sum-exp, and per node a CTA-local top-k list of keys.  A value
+// enters the tile's candidate buffer only if it beats the node's current
+// k-th key; after the tile the buffers are merged into the lists by rank.
+
+struct EpiSmem {
+    uint64_t* list;   // [NG][k]   sorted desc, 0 = empty
+    uint64_t* cand;   // [NG][kCandCap]
+    int* cnt;         // [NG]
+    float2* stats;    // [4][NG]  (max, sum exp) per epilogue warp
+};
+
+__device__ __forceinline__ float warp_max(float v) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xFFFFFFFFu, v, o));
+    return v;
+}
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xFFFFFFFFu, v, o);
+    return v;
+}
+
+// (m, s) <- (m, s) (+) (m2, s2) for sums of exp relative to their maxima.
+__device__ __forceinline__ float2 lse_merge(float2 a, float2 b) {
+    if (b.x == -INFINITY) return a;
+    if (a.x == -INFINITY) return b;
+    const float m = fmaxf(a.x, b.x);
+    return make_float2(m, a.y * __expf(a.x - m) + b.y * __expf(b.x - m));
+}
+
+__device__ __forceinline__ void epi_init(const EpiSmem& e, int NG, int k, int etid) {
+    for (int i = etid; i < NG * k; i += kEpiThreads) e.list[i] = 0ull;
+    for (int i = etid; i < NG; i += kEpiThreads) e.cnt[i] = 0;
+    for (int i = etid; i < 4 * NG; i += kEpiThreads) e.stats[i] = make_float2(-INFINITY, 0.0f);
+}
+
+// One (row, node) value.  Must be called by all 32 lanes of the warp with the
+// same node.  `z` is the scaled logit, `valid` whether the row is < V.
+__device__ __forceinline__ void epi_value(const EpiSmem& e, int NG, int k, int ew, int lane, int node, float z,
+                                          bool valid, uint32_t row) {
+    const float m = warp_max(valid ? z : -INFINITY);
+    const float p = (valid && m != -INFINITY) ? __expf(z - m) : 0.0f;
+    const float s = warp_sum(p);
+    if (lane == 0) e.stats[ew * NG + node] = lse_merge(e.stats[ew * NG + node], make_float2(m, s));
+    const uint64_t key = valid ? make_key(z, row) : 0ull;
+    const bool pass = key > e.list[node * k + k - 1];
+    const unsigned bal = __ballot_sync(0xFFFFFFFFu, pass);
+    if (bal) {
+        int base = 0;
+        if (lane == 0) base = atomicAdd(&e.cnt[node], __popc(bal));
+        base = __shfl_sync(0xFFFFFFFFu, base, 0);
+        if (pass) e.cand[node * kCandCap + base + __popc(bal & ((1u << lane) - 1u))] = key;
+    }
+}
+
+// Merge every node's candidates into its list (after all values of a tile).
+// Called by all kEpiThreads epilogue threads.
+__device__ __forceinline__ void epi_merge(const EpiSmem& e, int NG, int k, int etid) {
+    named_bar_sync(kEpiBarrier, kEpiThreads);
+    for (int nd = 0; nd < NG; nd++) {
+        const int c = e.cnt[nd];
+        if (c == 0) continue;  // uniform: every thread reads the same count
+        uint64_t* Ln = e.list + nd * k;
+        const uint64_t* Cn = e.cand + nd * kCandCap;
+        const int total = k + c;
+        uint64_t x[2] = {0ull, 0ull};
+        int r[2] = {k, k};
+#pragma unroll
+        for (int it = 0; it < 2; it++) {
+            const int i = etid + it * kEpiThreads;
+            if (i < total) {
+                int rank = 0;
+                if (i < k) {
+                    x[it] = Ln[i];
+                    rank = i;
+                } else {
+                    x[it] = Cn[i - k];
+                    for (int j = 0; j < k; j++) rank += Ln[j] > x[it];
+                }
+                for (int j = 0; j < c; j++) rank += Cn[j] > x[it];
+                r[it] = rank;
+            }
+        }
+        named_bar_sync(kEpiBarrier, kEpiThreads);
+#pragma unroll
+        for (int it = 0; it < 2; it++)
+            if (r[it] < k) Ln[r[it]] = x[it];
+        if (etid == 0) e.cnt[nd] = 0;
+        named_bar_sync(kEpiBarrier, kEpiThreads);
+    }
+}
+
+// Writes this CTA's partial results for the nodes n0 .. n0+NG-1 (< N):
+// part_ms[vr][n] = (max, sum exp), part_key[vr][n][k] = top-k keys.
+__device__ __forceinline__ void epi_finalize(const EpiSmem& e, int NG, int k, int etid, int n0, int N, int vr,
+                                             float2* part_ms, uint64_t* part_key) {
+    named_bar_sync(kEpiBarrier, kEpiThreads);
+    for (int c = etid; c < NG; c += kEpiThreads) {
+        const int n = n0 + c;
+        if (n >= N) continue;
+        float2 a = e.stats[c];
+        for (int w = 1; w < 4; w++) a = lse_merge(a, e.stats[w * NG + c]);
+        part_ms[static_cast<size_t>(vr) * N + n] = a;
+    }
+    for (int i = etid; i < NG * k; i += kEpiThreads) {
+        const int c = i / k, j = i % k, n = n0 + c;
+        if (n >= N) continue;
+        part_key[(static_cast<size_t>(vr) * N + n) * k + j] = e.list[i];
+    }
+}
+
+}  // namespace dart

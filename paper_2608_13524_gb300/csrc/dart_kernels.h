@@ -1,0 +1,113 @@
+// Internal launch interface between the C-ABI layer and the kernels.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace dart {
+
+// LM-head scoring (Algorithm 1: correct every prefix of S_{d-1} over the full
+// vocabulary, Appendix D "Full"): per node n and vocabulary row v,
+//   z[n][v] = (Dlog[seq(n)][dep-1][v] + E[v] . h[n]) * invT,
+// reduced on chip to per-CTA (max, sum exp) and top-k keys.
+struct LmheadArgs {
+    int V, d, N;          // vocabulary, hidden, nodes at this depth
+    int NG, G;            // nodes per group (multiple of 16), groups
+    int nV;               // vocabulary ranges (CTAs per group)
+    int k;
+    int tiles;            // ceil(V / 128)
+    int P;                // nodes per sequence (node n belongs to sequence n / P)
+    float invT;
+    const float* dlog;    // [nseq][L][V]
+    long long dlog_seq_stride;  // L * V
+    long long dlog_row_off;     // (dep-1) * V
+    int bhalf;            // row offset of the lo half in the bf16 state operand
+    int stages;           // smem pipeline depth (tcgen05 kernel)
+    float2* part_ms;      // [nV][N]
+    uint64_t* part_key;   // [nV][N][k]
+    int* status;
+    const float* h32;     // fp32 states [N][d] (fp32 kernel)
+    const float* E32;     // fp32 table [V][d]   (fp32 kernel)
+};
+
+// Skinny split-K GEMM for the correction head: out[split][n][m] =
+// sum_{k in split} A[m][k] * B[n][k], B given as hi + lo bf16 halves.
+struct GemmArgs {
+    int M, K, N;          // output features, reduction length, nodes
+    int NG, G, MT, S;     // node group, groups, m tiles, k splits
+    int KB;               // K / 64
+    int lo_kb_end;        // k-blocks >= this have a zero lo half (skipped)
+    int bhalf;
+    int stages;
+    float* out;           // [S][N][M]
+    int* status;
+    const float* A32;     // fp32 path: A [M][K]
+    const float* B32;     // fp32 path: B [N][K]
+};
+
+// tcgen05 kernels (dart_tc.cu)
+cudaError_t launch_lmhead_tc(const CUtensorMap* tmE, const CUtensorMap* tmH, const LmheadArgs& a,
+                             int smem_bytes, cudaStream_t st);
+cudaError_t launch_gemm_tc(const CUtensorMap* tmA, const CUtensorMap* tmB, const GemmArgs& a, int smem_bytes,
+                           cudaStream_t st);
+int tc_stage_bytes(int NG);
+int lmhead_tc_fixed_smem(int NG, int k, int stages);
+int gemm_tc_fixed_smem(int stages);
+cudaError_t tc_set_smem_limits(int max_dyn);
+
+// fp32 CUDA-core kernels (dart_f32.cu)
+cudaError_t launch_lmhead_f32(const LmheadArgs& a, cudaStream_t st);
+cudaError_t launch_gemm_f32(const GemmArgs& a, cudaStream_t st);
+int lmhead_f32_smem(int NG, int k);
+cudaError_t f32_set_smem_limits(int max_dyn);
+
+// selection / emission / elementwise kernels (dart_select.cu)
+struct SelectArgs {
+    int N, P, k, nV, W, L, nseq, dep, Pn;  // Pn = max |S_dep| (child slots per sequence)
+    float beta;
+    const float2* part_ms;
+    const uint64_t* part_key;
+    float* node_logq;      // [N][k]
+    int* node_tok;         // [N][k]
+    float* node_lse;       // [N]
+    int* tree_tok;         // [nseq][L][W]
+    int* tree_parent;
+    float* tree_score;
+    int* tree_count;       // [nseq][L]
+    int* child_prow;       // [nseq*Pn]
+    int* child_tok;
+    int* seq_ticket;       // [nseq]
+    int* status;
+};
+cudaError_t launch_merge_select(const SelectArgs& a, cudaStream_t st);
+int merge_select_smem(int nV, int k, int W);
+cudaError_t select_set_smem_limits(int max_dyn);
+
+struct EmitArgs {
+    int L, W, B, nseq, pos_offset;
+    const int* tree_tok;
+    const int* tree_parent;
+    const float* tree_score;
+    const int* tree_count;
+    int32_t *tokens, *parents, *depths, *pos_ids, *n_nodes;
+    float* scores;
+    uint64_t* mask;
+    int* status;
+};
+cudaError_t launch_prune_emit(const EmitArgs& a, cudaStream_t st);
+
+// depth-1 preparation: states <- anchors, and their hi/lo bf16 split
+cudaError_t launch_prep_anchor(const float* anchor, int nseq, int d, float* h, __nv_bfloat16* HL, int bhalf,
+                               cudaStream_t st);
+// X[c] = [h[prow[c]] ; E[tok[c]]] (hi/lo bf16 or fp32)
+cudaError_t launch_gather_x(int Nc, int d, const int* prow, const int* tok, const float* h, const void* E,
+                            int wbf16, __nv_bfloat16* XL, int bhalf, float* X32, cudaStream_t st);
+// a = SiLU(sum_s part[s]) -> AL (hi/lo) or A32
+cudaError_t launch_silu_split(int Nc, int d, int S, const float* part, __nv_bfloat16* AL, int bhalf, float* A32,
+                              cudaStream_t st);
+// h_next[c] = RMSNorm(h[prow[c]] + sum_s part[s][c]) and its hi/lo split
+cudaError_t launch_residual_norm(int Nc, int d, int S, const float* part, const int* prow, const float* h,
+                                 float eps, float* h_next, __nv_bfloat16* HL, int bhalf, cudaStream_t st);
+
+}  // namespace dart

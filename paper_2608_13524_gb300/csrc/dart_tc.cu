@@ -1,0 +1,424 @@
+// tcgen05 / TMA kernels of the DARTree construction path (sm_103a).
+//
+// One warp-specialised mainloop serves two contractions with bf16 operands
+// in shared memory and fp32 accumulators in tensor memory:
+//   * LM-head scoring: A = E tile [128 vocabulary rows x 64], B = node states
+//     [NG nodes x 64] as hi + lo bf16 halves (both MMAs accumulate into the
+//     same TMEM tile, so states keep ~16 mantissa bits).  A persistent CTA
+//     walks a contiguous range of vocabulary tiles; two TMEM accumulators let
+//     the epilogue of tile i overlap the MMAs of tile i+1.  The epilogue adds
+//     the drafter row, scales by 1/T and reduces on chip to a running
+//     log-sum-exp and a top-k per node, so no [N,V] logits tensor is written.
+//   * Correction-head GEMMs (split-K): A = W_i or W_o tile, B = the node
+//     inputs; each CTA writes an fp32 partial tile.
+// Warp roles (192 threads): warp 0 = TMA producer, warp 1 = TMEM allocator
+// and single-thread MMA issuer, warps 2-5 = epilogue (TMEM lane quarters
+// warp%4).  Every wait is bounded: on timeout the CTA records kDevTimeout in
+// the status word, drains its own copies/MMAs (bounded), frees TMEM and exits.
+#include "dart_device.cuh"
+#include "dart_kernels.h"
+
+namespace dart {
+
+namespace {
+
+constexpr int kThreads = 192;
+constexpr int kATileBytes = kTileM * kBlockK * 2;  // 16 KB
+
+struct Work {
+    int ntiles;     // consecutive A tiles handled by this CTA
+    int row0;       // row coordinate of the first tile
+    int kb0, kb1;   // k-block range
+    int brow;       // B row of this node group (hi half); lo half at + bhalf
+    int lo_kb_end;  // k-blocks >= this carry no lo half
+};
+
+template <int NG>
+struct Layout {
+    static constexpr int kStage = kATileBytes + 2 * NG * 128;
+};
+
+__device__ __forceinline__ void record_timeout(int* status, volatile int* abort) {
+    *abort = 1;
+    atomicOr(status, kDevTimeout);
+}
+
+// Bounded wait that ignores the abort flag (used while draining).
+__device__ __forceinline__ void drain_wait(uint64_t* bar, uint32_t parity) {
+    const unsigned long long t0 = globaltimer_ns();
+    while (!mbar_try_wait(bar, parity)) {
+        if (globaltimer_ns() - t0 > kWaitLimitNs) return;
+    }
+}
+
+template <int NG>
+__device__ __forceinline__ void producer(const CUtensorMap* tmA, const CUtensorMap* tmB, const Work& w, int bhalf,
+                                         uint8_t* ring, int stages, uint64_t* full, uint64_t* empty,
+                                         volatile int* abort, int* status) {
+    const uint64_t pol_a = l2_policy_evict_first();  // streamed once
+    const uint64_t pol_b = l2_policy_evict_last();   // re-read by every tile
+    uint32_t stage = 0, phase = 0, fills = 0;
+    bool ok = true;
+    for (int i = 0; i < w.ntiles && ok; i++) {
+        const int row = w.row0 + i * kTileM;
+        for (int kb = w.kb0; kb < w.kb1; kb++) {
+            if (!mbar_wait(&empty[stage], phase ^ 1u, abort)) {
+                record_timeout(status, abort);
+                ok = false;
+                break;
+            }
+            const bool lo = kb < w.lo_kb_end;
+            uint8_t* sA = ring + stage * Layout<NG>::kStage;
+            uint8_t* sH = sA + kATileBytes;
+            uint8_t* sL = sH + NG * 128;
+            mbar_arrive_expect_tx(&full[stage], kATileBytes + NG * 128 * (lo ? 2 : 1));
+            tma_load_2d(sA, tmA, &full[stage], kb * kBlockK, row, pol_a);
+            tma_load_2d(sH, tmB, &full[stage], kb * kBlockK, w.brow, pol_b);
+            if (lo) tma_load_2d(sL, tmB, &full[stage], kb * kBlockK, bhalf + w.brow, pol_b);
+            fills++;
+            if (++stage == static_cast<uint32_t>(stages)) {
+                stage = 0;
+                phase ^= 1u;
+            }
+        }
+    }
+    if (!ok) {
+        // wait for this thread's copies still in flight before the CTA exits
+        const uint32_t first = fills > static_cast<uint32_t>(stages) ? fills - stages : 0;
+        for (uint32_t f = first; f < fills; f++) drain_wait(&full[f % stages], (f / stages) & 1u);
+    }
+}
+
+template <int NG>
+__device__ __forceinline__ void mma_issuer(const Work& w, uint8_t* ring, int stages, uint64_t* full,
+                                           uint64_t* empty, uint64_t* tfull, uint64_t* tempty, uint64_t* tdown,
+                                           uint32_t tmem_base, int acc_stride, volatile int* abort,
+                                           int* status) {
+    constexpr uint32_t idesc = idesc_bf16_f32(kTileM, NG);
+    uint32_t stage = 0, phase = 0;
+    bool ok = true;
+    for (int i = 0; i < w.ntiles && ok; i++) {
+        const int acc = i & 1;
+        const uint32_t aph = (i >> 1) & 1;
+        if (!mbar_wait(&tempty[acc], aph ^ 1u, abort)) {
+            record_timeout(status, abort);
+            ok = false;
+            break;
+        }
+        tc_fence_after();
+        const uint32_t d_tmem = tmem_base + acc * acc_stride;
+        for (int kb = w.kb0; kb < w.kb1; kb++) {
+            if (!mbar_wait(&full[stage], phase, abort)) {
+                record_timeout(status, abort);
+                ok = false;
+                break;
+            }
+            tc_fence_after();
+            const bool lo = kb < w.lo_kb_end;
+            const uint32_t a = smem_u32(ring + stage * Layout<NG>::kStage);
+            const uint32_t hb = a + kATileBytes;
+            const uint32_t lb = hb + NG * 128;
+#pragma unroll
+            for (int kk = 0; kk < kBlockK / 16; kk++) {
+                const uint64_t ad = sdesc_sw128(a + kk * 32);
+                tc_mma_bf16(d_tmem, ad, sdesc_sw128(hb + kk * 32), idesc, (kb > w.kb0 || kk > 0) ? 1u : 0u);
+                if (lo) tc_mma_bf16(d_tmem, ad, sdesc_sw128(lb + kk * 32), idesc, 1u);
+            }
+            tc_commit(&empty[stage]);  // frees the smem stage once these MMAs are done
+            if (++stage == static_cast<uint32_t>(stages)) {
+                stage = 0;
+                phase ^= 1u;
+            }
+        }
+        if (ok) tc_commit(&tfull[acc]);
+    }
+    if (!ok) {
+        // make sure no MMA still reads smem / writes TMEM before teardown
+        tc_commit(tdown);
+        drain_wait(tdown, 0);
+    }
+}
+
+struct Smem {
+    uint8_t* ring;
+    uint64_t *full, *empty, *tfull, *tempty, *tdown;
+    int* misc;  // [0] tmem base, [1] abort flag, [2] epilogue flag
+    uint8_t* tail;
+};
+
+template <int NG>
+__device__ __forceinline__ Smem carve(uint8_t* raw, int stages) {
+    Smem s;
+    const uint32_t off = (1024u - (smem_u32(raw) & 1023u)) & 1023u;
+    s.ring = raw + off;
+    s.full = reinterpret_cast<uint64_t*>(s.ring + stages * Layout<NG>::kStage);
+    s.empty = s.full + stages;
+    s.tfull = s.empty + stages;
+    s.tempty = s.tfull + 2;
+    s.tdown = s.tempty + 2;
+    s.misc = reinterpret_cast<int*>(s.tdown + 1);
+    s.tail = reinterpret_cast<uint8_t*>(s.misc + 4);
+    return s;
+}
+
+template <int NG>
+__device__ __forceinline__ uint32_t setup(const Smem& s, int stages, int ncols) {
+    const int warp = threadIdx.x >> 5;
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < stages; i++) {
+            mbar_init(&s.full[i], 1);
+            mbar_init(&s.empty[i], 1);
+        }
+        for (int i = 0; i < 2; i++) {
+            mbar_init(&s.tfull[i], 1);
+            mbar_init(&s.tempty[i], kEpiThreads);
+        }
+        mbar_init(s.tdown, 1);
+        s.misc[1] = 0;
+        s.misc[2] = 0;
+        fence_mbar_init();
+    }
+    if (warp == 1) {
+        tmem_alloc(reinterpret_cast<uint32_t*>(&s.misc[0]), ncols);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    return static_cast<uint32_t>(s.misc[0]);
+}
+
+__device__ __forceinline__ void teardown(uint32_t tmem_base, int ncols) {
+    tc_fence_before();
+    __syncthreads();
+    if ((threadIdx.x >> 5) == 1) {
+        __syncwarp();
+        tc_fence_after();
+        tmem_dealloc(tmem_base, ncols);
+    }
+}
+
+template <int NG>
+constexpr int acc_stride() {
+    return NG < 32 ? 32 : NG;
+}
+template <int NG>
+constexpr int tmem_cols() {
+    return 2 * acc_stride<NG>() <= 32 ? 32 : (2 * acc_stride<NG>() <= 64 ? 64 : (2 * acc_stride<NG>() <= 128 ? 128 : 256));
+}
+
+// ------------------------------------------------------------ LM-head kernel
+
+template <int NG>
+__global__ void __launch_bounds__(kThreads, 1)
+    lmhead_tc_kernel(const __grid_constant__ CUtensorMap tmE, const __grid_constant__ CUtensorMap tmH,
+                     const LmheadArgs a) {
+    extern __shared__ uint8_t smem_raw[];
+    const int stages = a.stages;
+    Smem s = carve<NG>(smem_raw, stages);
+    EpiSmem e;
+    e.list = reinterpret_cast<uint64_t*>(s.tail);
+    e.cand = e.list + NG * a.k;
+    e.stats = reinterpret_cast<float2*>(e.cand + NG * kCandCap);
+    e.cnt = reinterpret_cast<int*>(e.stats + 4 * NG);
+
+    const int g = blockIdx.x % a.G;
+    const int vr = blockIdx.x / a.G;
+    const int t0 = static_cast<int>((static_cast<long long>(vr) * a.tiles) / a.nV);
+    const int t1 = static_cast<int>((static_cast<long long>(vr + 1) * a.tiles) / a.nV);
+    Work w;
+    w.ntiles = t1 - t0;
+    w.row0 = t0 * kTileM;
+    w.kb0 = 0;
+    w.kb1 = a.d / kBlockK;
+    w.brow = g * NG;
+    w.lo_kb_end = w.kb1;
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const uint32_t tmem_base = setup<NG>(s, stages, tmem_cols<NG>());
+    volatile int* abort = &s.misc[1];
+
+    if (warp == 0) {
+        if (lane == 0) producer<NG>(&tmE, &tmH, w, a.bhalf, s.ring, stages, s.full, s.empty, abort, a.status);
+    } else if (warp == 1) {
+        if (lane == 0)
+            mma_issuer<NG>(w, s.ring, stages, s.full, s.empty, s.tfull, s.tempty, s.tdown, tmem_base,
+                           acc_stride<NG>(), abort, a.status);
+    } else {
+        const int etid = threadIdx.x - 64;
+        const int ew = warp - 2;
+        const int quarter = warp & 3;
+        epi_init(e, NG, a.k, etid);
+        for (int i = 0; i < w.ntiles; i++) {
+            const int acc = i & 1;
+            const uint32_t aph = (i >> 1) & 1;
+            if (etid == 0) {
+                const bool ok = mbar_wait(&s.tfull[acc], aph, abort);
+                if (!ok) record_timeout(a.status, abort);
+                s.misc[2] = ok ? 1 : 0;
+            }
+            named_bar_sync(kEpiBarrier, kEpiThreads);
+            if (s.misc[2] == 0) break;
+            tc_fence_after();
+            const int row_local = quarter * 32 + lane;
+            const int v = w.row0 + i * kTileM + row_local;
+            const bool valid = v < a.V;
+            int cur_seq = -1;
+            float dl = 0.0f;
+#pragma unroll
+            for (int c0 = 0; c0 < NG; c0 += 16) {
+                float vals[16];
+                tmem_ld16(tmem_base + acc * acc_stride<NG>() + c0 + (static_cast<uint32_t>(quarter * 32) << 16),
+                          vals);
+#pragma unroll
+                for (int j = 0; j < 16; j++) {
+                    const int node = c0 + j;
+                    const int n = g * NG + node;
+                    if (n < a.N) {
+                        const int seq = n / a.P;
+                        if (seq != cur_seq) {
+                            cur_seq = seq;
+                            dl = valid ? __ldg(a.dlog + seq * a.dlog_seq_stride + a.dlog_row_off + v) : 0.0f;
+                        }
+                        const float z = (vals[j] + dl) * a.invT;
+                        epi_value(e, NG, a.k, ew, lane, node, z, valid, static_cast<uint32_t>(v));
+                    }
+                }
+            }
+            tc_fence_before();
+            mbar_arrive(&s.tempty[acc]);
+            epi_merge(e, NG, a.k, etid);
+        }
+        epi_finalize(e, NG, a.k, etid, g * NG, a.N, vr, a.part_ms, a.part_key);
+    }
+    teardown(tmem_base, tmem_cols<NG>());
+}
+
+// --------------------------------------------------------------- GEMM kernel
+
+template <int NG>
+__global__ void __launch_bounds__(kThreads, 1)
+    gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                   const GemmArgs a) {
+    extern __shared__ uint8_t smem_raw[];
+    const int stages = a.stages;
+    Smem s = carve<NG>(smem_raw, stages);
+
+    const int mt = blockIdx.x % a.MT;
+    const int rest = blockIdx.x / a.MT;
+    const int g = rest % a.G;
+    const int split = rest / a.G;
+    Work w;
+    w.ntiles = 1;
+    w.row0 = mt * kTileM;
+    w.kb0 = static_cast<int>((static_cast<long long>(split) * a.KB) / a.S);
+    w.kb1 = static_cast<int>((static_cast<long long>(split + 1) * a.KB) / a.S);
+    w.brow = g * NG;
+    w.lo_kb_end = a.lo_kb_end;
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const uint32_t tmem_base = setup<NG>(s, stages, tmem_cols<NG>());
+    volatile int* abort = &s.misc[1];
+
+    if (warp == 0) {
+        if (lane == 0) producer<NG>(&tmA, &tmB, w, a.bhalf, s.ring, stages, s.full, s.empty, abort, a.status);
+    } else if (warp == 1) {
+        if (lane == 0)
+            mma_issuer<NG>(w, s.ring, stages, s.full, s.empty, s.tfull, s.tempty, s.tdown, tmem_base,
+                           acc_stride<NG>(), abort, a.status);
+    } else {
+        const int etid = threadIdx.x - 64;
+        const int quarter = warp & 3;
+        if (etid == 0) {
+            const bool ok = mbar_wait(&s.tfull[0], 0, abort);
+            if (!ok) record_timeout(a.status, abort);
+            s.misc[2] = ok ? 1 : 0;
+        }
+        named_bar_sync(kEpiBarrier, kEpiThreads);
+        if (s.misc[2] != 0) {
+            tc_fence_after();
+            const int m = w.row0 + quarter * 32 + lane;
+            const bool valid = m < a.M;
+            float* out = a.out + static_cast<size_t>(split) * a.N * a.M;
+#pragma unroll
+            for (int c0 = 0; c0 < NG; c0 += 16) {
+                float vals[16];
+                tmem_ld16(tmem_base + c0 + (static_cast<uint32_t>(quarter * 32) << 16), vals);
+#pragma unroll
+                for (int j = 0; j < 16; j++) {
+                    const int n = g * NG + c0 + j;
+                    if (valid && n < a.N) out[static_cast<size_t>(n) * a.M + m] = vals[j];
+                }
+            }
+        }
+    }
+    teardown(tmem_base, tmem_cols<NG>());
+}
+
+template <int NG>
+int lmhead_fixed(int k, int stages) {
+    return (2 * stages + 5) * 8 + 16 + NG * k * 8 + NG * kCandCap * 8 + 4 * NG * 8 + NG * 4;
+}
+
+template <int NG>
+cudaError_t launch_lmhead_ng(const CUtensorMap* tmE, const CUtensorMap* tmH, const LmheadArgs& a, int smem,
+                             cudaStream_t st) {
+    lmhead_tc_kernel<NG><<<a.nV * a.G, kThreads, smem, st>>>(*tmE, *tmH, a);
+    return cudaGetLastError();
+}
+template <int NG>
+cudaError_t launch_gemm_ng(const CUtensorMap* tmA, const CUtensorMap* tmB, const GemmArgs& a, int smem,
+                           cudaStream_t st) {
+    gemm_tc_kernel<NG><<<a.MT * a.G * a.S, kThreads, smem, st>>>(*tmA, *tmB, a);
+    return cudaGetLastError();
+}
+
+}  // namespace
+
+int tc_stage_bytes(int NG) { return kATileBytes + 2 * NG * 128; }
+
+int lmhead_tc_fixed_smem(int NG, int k, int stages) {
+    switch (NG) {
+        case 16: return lmhead_fixed<16>(k, stages) + 1024;
+        case 32: return lmhead_fixed<32>(k, stages) + 1024;
+        default: return lmhead_fixed<64>(k, stages) + 1024;
+    }
+}
+
+int gemm_tc_fixed_smem(int stages) { return (2 * stages + 5) * 8 + 16 + 1024; }
+
+cudaError_t tc_set_smem_limits(int max_dyn) {
+    cudaError_t e = cudaSuccess;
+#define DART_SET(fn)                                                                                   \
+    if (e == cudaSuccess) e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, max_dyn);
+    DART_SET(lmhead_tc_kernel<16>)
+    DART_SET(lmhead_tc_kernel<32>)
+    DART_SET(lmhead_tc_kernel<64>)
+    DART_SET(gemm_tc_kernel<16>)
+    DART_SET(gemm_tc_kernel<32>)
+    DART_SET(gemm_tc_kernel<64>)
+#undef DART_SET
+    return e;
+}
+
+cudaError_t launch_lmhead_tc(const CUtensorMap* tmE, const CUtensorMap* tmH, const LmheadArgs& a, int smem,
+                             cudaStream_t st) {
+    switch (a.NG) {
+        case 16: return launch_lmhead_ng<16>(tmE, tmH, a, smem, st);
+        case 32: return launch_lmhead_ng<32>(tmE, tmH, a, smem, st);
+        case 64: return launch_lmhead_ng<64>(tmE, tmH, a, smem, st);
+        default: return cudaErrorInvalidValue;
+    }
+}
+
+cudaError_t launch_gemm_tc(const CUtensorMap* tmA, const CUtensorMap* tmB, const GemmArgs& a, int smem,
+                           cudaStream_t st) {
+    switch (a.NG) {
+        case 16: return launch_gemm_ng<16>(tmA, tmB, a, smem, st);
+        case 32: return launch_gemm_ng<32>(tmA, tmB, a, smem, st);
+        case 64: return launch_gemm_ng<64>(tmA, tmB, a, smem, st);
+        default: return cudaErrorInvalidValue;
+    }
+}
+
+}  // namespace dart

@@ -1,0 +1,244 @@
+"""Thin ctypes binding of the DARTree C ABI (include/dart.h).
+
+Argument marshalling only: every step of the construction runs in the CUDA
+kernels of ``libdart.so``.  Functions keep the C names; tensors are passed by
+``data_ptr()`` and streams by their CUDA handle.  There is no fallback: if the
+library is missing, importing the binding raises.
+"""
+from __future__ import annotations
+
+import ctypes as C
+import os
+
+import torch
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "libdart.so")
+
+DART_OK = 0
+DART_ERR_INVALID = -1
+DART_ERR_CUDA = -2
+DART_ERR_NOMEM = -3
+DART_ERR_TIMEOUT = -4
+DART_ERR_STATE = -5
+DART_ERR_UNSUPPORTED = -6
+DART_F32 = 0
+DART_BF16 = 1
+
+
+class DartConfig(C.Structure):
+    _fields_ = [("V", C.c_int), ("d", C.c_int), ("L", C.c_int), ("W", C.c_int), ("k", C.c_int),
+                ("B", C.c_int), ("nseq", C.c_int), ("beta", C.c_float),
+                ("temperature", C.c_float), ("rms_eps", C.c_float), ("pos_offset", C.c_int)]
+
+
+class DartTreeOut(C.Structure):
+    _fields_ = [("tokens", C.c_void_p), ("parents", C.c_void_p), ("depths", C.c_void_p),
+                ("pos_ids", C.c_void_p), ("scores", C.c_void_p), ("n_nodes", C.c_void_p),
+                ("mask", C.c_void_p)]
+
+
+class DartError(RuntimeError):
+    def __init__(self, code, what):
+        super().__init__(f"{what}: {status_string(code)} ({code})")
+        self.code = code
+
+
+_lib = None
+
+
+def lib():
+    """Loads libdart.so (raises if it was not built)."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(LIB_PATH):
+            raise RuntimeError(f"{LIB_PATH} not found: build it with __graft_entry__.build()")
+        L = C.CDLL(LIB_PATH)
+        vp, i, f = C.c_void_p, C.c_int, C.c_float
+        sig = {
+            "dart_init_head": (i, [C.POINTER(vp), C.POINTER(DartConfig), i, vp, vp, vp, vp]),
+            "dart_expand_depth": (i, [vp, i, vp, vp, vp]),
+            "dart_prune_and_emit": (i, [vp, C.POINTER(DartTreeOut), vp]),
+            "dart_build_tree": (i, [vp, vp, vp, C.POINTER(DartTreeOut), vp]),
+            "dart_build_tree_host": (i, [vp, vp, vp, C.POINTER(DartTreeOut), vp]),
+            "dart_get_frontier": (i, [vp, i, vp, vp, vp, vp, vp]),
+            "dart_get_node_topk": (i, [vp, vp, vp, vp, C.POINTER(i), vp]),
+            "dart_get_states": (i, [vp, vp, C.POINTER(i), vp]),
+            "dart_status_sync": (i, [vp, vp]),
+            "dart_set_profiling": (i, [vp, i]),
+            "dart_profile_read": (i, [vp, C.POINTER(f), C.POINTER(i)]),
+            "dart_launches_per_round": (i, [vp]),
+            "dart_destroy": (None, [vp]),
+            "dart_status_string": (C.c_char_p, [i]),
+            "dart_version": (i, []),
+        }
+        for name, (res, args) in sig.items():
+            fn = getattr(L, name)
+            fn.restype = res
+            fn.argtypes = args
+        _lib = L
+    return _lib
+
+
+def status_string(code: int) -> str:
+    return lib().dart_status_string(int(code)).decode()
+
+
+def _check(code, what):
+    if code != DART_OK:
+        raise DartError(code, what)
+
+
+def _ptr(t):
+    return None if t is None else C.c_void_p(t.data_ptr())
+
+
+def _stream(stream):
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return C.c_void_p(stream.cuda_stream if hasattr(stream, "cuda_stream") else int(stream))
+
+
+def make_config(cfg) -> DartConfig:
+    """From any object with V, d, L, W, k, B, nseq, beta, temperature,
+    rms_eps, pos_offset."""
+    return DartConfig(int(cfg.V), int(cfg.d), int(cfg.L), int(cfg.W), int(cfg.k), int(cfg.B),
+                      int(cfg.nseq), float(cfg.beta), float(cfg.temperature), float(cfg.rms_eps),
+                      int(cfg.pos_offset))
+
+
+def alloc_tree_out(cfg, device="cuda", pin=False):
+    """Allocates the emitted-tree arrays; returns (dict of tensors, DartTreeOut)."""
+    ns, B = cfg.nseq, cfg.B
+    nw = (B + 63) // 64
+    kw = dict(device=device)
+    if pin:
+        kw = dict(device="cpu", pin_memory=True)
+    t = dict(tokens=torch.empty((ns, B), dtype=torch.int32, **kw),
+             parents=torch.empty((ns, B), dtype=torch.int32, **kw),
+             depths=torch.empty((ns, B), dtype=torch.int32, **kw),
+             pos_ids=torch.empty((ns, B), dtype=torch.int32, **kw),
+             scores=torch.empty((ns, B), dtype=torch.float32, **kw),
+             n_nodes=torch.empty((ns,), dtype=torch.int32, **kw),
+             mask=torch.empty((ns, B, nw), dtype=torch.int64, **kw))
+    out = DartTreeOut(*(t[k].data_ptr() for k in
+                        ("tokens", "parents", "depths", "pos_ids", "scores", "n_nodes", "mask")))
+    return t, out
+
+
+# ----------------------------------------------------------------- the ABI
+
+def dart_init_head(cfg, wdtype, W_i, W_o, E, stream=None):
+    """Returns an opaque handle (int).  W_i/W_o/E are device tensors of the
+    weight dtype (torch.bfloat16 or torch.float32)."""
+    h = C.c_void_p()
+    c = make_config(cfg)
+    _check(lib().dart_init_head(C.byref(h), C.byref(c), int(wdtype), _ptr(W_i), _ptr(W_o), _ptr(E),
+                                _stream(stream)), "dart_init_head")
+    return h
+
+
+def dart_expand_depth(h, depth, drafter_logits, anchor_h=None, stream=None):
+    _check(lib().dart_expand_depth(h, int(depth), _ptr(drafter_logits), _ptr(anchor_h),
+                                   _stream(stream)), "dart_expand_depth")
+
+
+def dart_prune_and_emit(h, out: DartTreeOut, stream=None):
+    _check(lib().dart_prune_and_emit(h, C.byref(out), _stream(stream)), "dart_prune_and_emit")
+
+
+def dart_build_tree(h, drafter_logits, anchor_h, out: DartTreeOut, stream=None):
+    _check(lib().dart_build_tree(h, _ptr(drafter_logits), _ptr(anchor_h), C.byref(out),
+                                 _stream(stream)), "dart_build_tree")
+
+
+def dart_build_tree_host(h, drafter_logits_host, anchor_host, out_host: DartTreeOut, stream=None):
+    _check(lib().dart_build_tree_host(h, _ptr(drafter_logits_host), _ptr(anchor_host),
+                                      C.byref(out_host), _stream(stream)), "dart_build_tree_host")
+
+
+def dart_get_frontier(h, depth, cfg, stream=None):
+    dev = "cuda"
+    tok = torch.empty((cfg.nseq, cfg.W), dtype=torch.int32, device=dev)
+    par = torch.empty_like(tok)
+    score = torch.empty((cfg.nseq, cfg.W), dtype=torch.float32, device=dev)
+    count = torch.empty((cfg.nseq,), dtype=torch.int32, device=dev)
+    _check(lib().dart_get_frontier(h, int(depth), _ptr(tok), _ptr(par), _ptr(score), _ptr(count),
+                                   _stream(stream)), "dart_get_frontier")
+    return tok, par, score, count
+
+
+def dart_get_node_topk(h, cfg, stream=None):
+    rows = C.c_int()
+    _check(lib().dart_get_node_topk(h, None, None, None, C.byref(rows), _stream(stream)),
+           "dart_get_node_topk")
+    n = rows.value
+    tok = torch.empty((n, cfg.k), dtype=torch.int32, device="cuda")
+    logq = torch.empty((n, cfg.k), dtype=torch.float32, device="cuda")
+    lse = torch.empty((n,), dtype=torch.float32, device="cuda")
+    _check(lib().dart_get_node_topk(h, _ptr(tok), _ptr(logq), _ptr(lse), C.byref(rows),
+                                    _stream(stream)), "dart_get_node_topk")
+    return tok, logq, lse
+
+
+def dart_get_states(h, cfg, stream=None):
+    rows = C.c_int()
+    _check(lib().dart_get_states(h, None, C.byref(rows), _stream(stream)), "dart_get_states")
+    st = torch.empty((rows.value, cfg.d), dtype=torch.float32, device="cuda")
+    _check(lib().dart_get_states(h, _ptr(st), C.byref(rows), _stream(stream)), "dart_get_states")
+    return st
+
+
+def dart_status_sync(h, stream=None):
+    return int(lib().dart_status_sync(h, _stream(stream)))
+
+
+def dart_set_profiling(h, enable):
+    _check(lib().dart_set_profiling(h, int(bool(enable))), "dart_set_profiling")
+
+
+def dart_profile_read(h):
+    ms = C.c_float()
+    n = C.c_int()
+    _check(lib().dart_profile_read(h, C.byref(ms), C.byref(n)), "dart_profile_read")
+    return float(ms.value), int(n.value)
+
+
+def dart_launches_per_round(h):
+    return int(lib().dart_launches_per_round(h))
+
+
+def dart_destroy(h):
+    if h:
+        lib().dart_destroy(h)
+
+
+class Dart:
+    """Owns one handle plus the weight tensors it borrows."""
+
+    def __init__(self, cfg, W_i, W_o, E, stream=None):
+        if W_i.dtype == torch.bfloat16:
+            wd = DART_BF16
+        elif W_i.dtype == torch.float32:
+            wd = DART_F32
+        else:
+            raise TypeError("weights must be bfloat16 or float32")
+        self.cfg = cfg
+        self._keep = (W_i, W_o, E)
+        self.h = dart_init_head(cfg, wd, W_i, W_o, E, stream)
+        self.out_t, self.out = alloc_tree_out(cfg)
+
+    def build_tree(self, drafter_logits, anchor_h, stream=None):
+        dart_build_tree(self.h, drafter_logits, anchor_h, self.out, stream)
+        return self.out_t
+
+    def close(self):
+        dart_destroy(self.h)
+        self.h = None
+
+    def __del__(self):
+        try:
+            if self.h:
+                self.close()
+        except Exception:
+            pass

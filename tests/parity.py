@@ -1,0 +1,209 @@
+"""GPU-vs-oracle comparison helpers.
+
+Rules (the contract of the parity tests):
+  * path scores within `tol` (2e-3 for bf16 weights, 1e-5 for fp32);
+  * topology compared as sets of token paths, required equal at every depth
+    whose relevant oracle rank gap (frontier cut, or the k-th / (k+1)-th cut
+    of a node whose k-th child is kept) is >= tol; after a near tie the
+    comparison switches to validity checks;
+  * the emitted arrays (tokens, parents, depths, pos_ids, mask, n_nodes) are
+    required bit-exact when no oracle rank gap anywhere is below tol;
+  * the GPU tree is always checked for structural validity.
+"""
+from __future__ import annotations
+
+import numpy as np
+import torch
+
+import oracle
+
+
+def to_device(cfg, x, dev="cuda"):
+    if cfg.wdtype == "bf16":
+        t = lambda a: torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).to(dev).view(torch.bfloat16)
+    else:
+        t = lambda a: torch.from_numpy(np.ascontiguousarray(a)).to(dev)
+    return dict(Wi=t(x["Wi"]), Wo=t(x["Wo"]), E=t(x["E"]),
+                Dlog=torch.from_numpy(x["Dlog"]).to(dev), h0=torch.from_numpy(x["h0"]).to(dev))
+
+
+def tol_of(cfg):
+    return 2e-3 if cfg.wdtype == "bf16" else 1e-5
+
+
+def gpu_supertree(dart, h, cfg):
+    st_tok = np.empty((cfg.nseq, cfg.L, cfg.W), np.int32)
+    st_par = np.empty_like(st_tok)
+    st_score = np.empty((cfg.nseq, cfg.L, cfg.W), np.float32)
+    st_count = np.empty((cfg.nseq, cfg.L), np.int32)
+    for dep in range(1, cfg.L + 1):
+        tok, par, sc, cnt = dart.dart_get_frontier(h, dep, cfg)
+        st_tok[:, dep - 1] = tok.cpu().numpy()
+        st_par[:, dep - 1] = par.cpu().numpy()
+        st_score[:, dep - 1] = sc.cpu().numpy()
+        st_count[:, dep - 1] = cnt.cpu().numpy()
+    return dict(st_tok=st_tok, st_parent=st_par, st_score=st_score, st_count=st_count)
+
+
+def tree_to_numpy(t):
+    return {k: v.cpu().numpy() for k, v in t.items()}
+
+
+def emitted_paths(g, s):
+    out = {}
+    for i in range(int(g["n_nodes"][s])):
+        path, j = [], i
+        while j >= 0:
+            path.append(int(g["tokens"][s, j]))
+            j = int(g["parents"][s, j])
+        out[tuple(reversed(path))] = float(g["scores"][s, i])
+    return out
+
+
+def check_structure(cfg, g):
+    """Prefix closure, monotone scores, depths, position ids, ancestor mask
+    and padding of an emitted tree."""
+    nw = (cfg.B + 63) // 64
+    for s in range(cfg.nseq):
+        n = int(g["n_nodes"][s])
+        assert 0 <= n <= cfg.B
+        par = g["parents"][s]
+        for i in range(n):
+            p = int(par[i])
+            assert -1 <= p < i, (s, i, p)
+            if p >= 0:
+                assert g["depths"][s, i] == g["depths"][s, p] + 1
+                assert g["scores"][s, i] <= g["scores"][s, p]
+            else:
+                assert g["depths"][s, i] == 1
+            assert g["pos_ids"][s, i] == cfg.pos_offset + g["depths"][s, i]
+            assert np.isfinite(g["scores"][s, i])
+            anc = {i}
+            j = p
+            while j >= 0:
+                anc.add(j)
+                j = int(par[j])
+            row = g["mask"][s, i].view(np.uint64)
+            bits = {b for b in range(cfg.B) if (int(row[b // 64]) >> (b % 64)) & 1}
+            assert bits == anc, (s, i)
+        for i in range(n, cfg.B):
+            assert g["tokens"][s, i] == -1 and g["parents"][s, i] == -2
+            assert g["depths"][s, i] == 0 and g["pos_ids"][s, i] == -1
+            assert np.isneginf(g["scores"][s, i]) and not np.any(g["mask"][s, i])
+        assert g["mask"].shape[-1] == nw
+
+
+def relevant_gaps(cfg, ref, s, dep):
+    """(cut gap, min adjacent gap among kept) of the oracle at this depth."""
+    W, k = cfg.W, cfg.k
+    fr = ref["fr_score"][s, dep - 1]
+    cnt = int(ref["st_count"][s, dep - 1])
+    cut = np.inf
+    if cnt == W and np.isfinite(fr[W]):
+        cut = fr[W - 1] - fr[W]
+    # a node whose k-th child is kept: its k-th / (k+1)-th cut decides the set
+    kx = ref["nd_tok"].shape[-1]
+    if kx > k:
+        for r in range(cnt):
+            p = int(ref["st_parent"][s, dep - 1, r]) if dep > 1 else 0
+            t = int(ref["st_tok"][s, dep - 1, r])
+            if ref["nd_tok"][s, dep - 1, p, k - 1] == t:
+                g = ref["nd_logq"][s, dep - 1, p, k - 1] - ref["nd_logq"][s, dep - 1, p, k]
+                cut = min(cut, g)
+    adj = np.diff(-fr[:cnt]) if cnt > 1 else np.array([np.inf])
+    return cut, float(np.min(adj)) if adj.size else np.inf
+
+
+def compare_with_oracle(cfg, ref, gst, g, tol):
+    """Compares the GPU supertree `gst` and emitted tree `g` with the oracle
+    run `ref`.  Returns a report dict; raises AssertionError on a mismatch
+    the rank gaps do not excuse."""
+    rep = dict(near_tie=[], order_ties=0, arrays_exact=None, bit_identical=None)
+    all_exact = True
+    for s in range(cfg.nseq):
+        rp = oracle.node_paths(ref["st_tok"], ref["st_parent"], ref["st_count"], s, cfg.W)
+        gp = oracle.node_paths(gst["st_tok"], gst["st_parent"], gst["st_count"], s, cfg.W)
+        sets_equal = True
+        for dep in range(1, cfg.L + 1):
+            rc = int(ref["st_count"][s, dep - 1])
+            gc = int(gst["st_count"][s, dep - 1])
+            r_paths = [rp[(dep - 1) * cfg.W + r] for r in range(rc)]
+            g_paths = [gp[(dep - 1) * cfg.W + r] for r in range(gc)]
+            cut, adj = relevant_gaps(cfg, ref, s, dep)
+            if set(r_paths) != set(g_paths):
+                assert cut < tol, f"seq {s} depth {dep}: frontier differs with oracle cut gap {cut}"
+                rep["near_tie"].append((s, dep, float(cut)))
+                sets_equal = False
+                all_exact = False
+                break
+            rs = {p: ref["st_score"][s, dep - 1, r] for r, p in enumerate(r_paths)}
+            for r, p in enumerate(g_paths):
+                d = abs(float(gst["st_score"][s, dep - 1, r]) - rs[p])
+                assert d <= tol, f"seq {s} depth {dep} path score off by {d}"
+            if adj < tol:
+                rep["order_ties"] += 1
+                all_exact = False
+                for i in range(len(g_paths) - 1):
+                    assert rs[g_paths[i]] >= rs[g_paths[i + 1]] - tol
+            else:
+                assert r_paths == g_paths, f"seq {s} depth {dep}: rank order differs"
+        if sets_equal:
+            if ref["prune_gap"][s] < tol:
+                all_exact = False
+                rep["near_tie"].append((s, "prune", float(ref["prune_gap"][s])))
+            else:
+                ge = emitted_paths(g, s)
+                re_ = emitted_paths(ref, s)
+                assert set(ge) == set(re_), f"seq {s}: pruned tree differs"
+                for p, sc in ge.items():
+                    assert abs(sc - re_[p]) <= tol
+    keys = ("tokens", "parents", "depths", "pos_ids", "n_nodes")
+    same = all(np.array_equal(g[k], ref[k]) for k in keys) and np.array_equal(
+        g["mask"].view(np.uint64), ref["mask"])
+    rep["bit_identical"] = bool(same)
+    rep["arrays_exact"] = all_exact
+    if all_exact:
+        assert same, "emitted arrays differ although every oracle rank gap exceeds the tolerance"
+        ok = np.isfinite(ref["scores"])
+        assert np.max(np.abs(g["scores"][ok] - ref["scores"][ok]), initial=0.0) <= tol
+    check_structure(cfg, g)
+    return rep
+
+
+def validate_frontier_teacher_forced(cfg, x, gst, s, dep, tol_step, ref_logq=None):
+    """Checks S_dep of the GPU against the oracle given the GPU's own parents:
+    every parent's children are recomputed from its token path; each kept
+    child's score increment must be within tol_step of log q~ + beta, and the
+    kept set must be a valid top-W of the candidates (per-node top-k)."""
+    W, k = cfg.W, cfg.k
+    gp = oracle.node_paths(gst["st_tok"], gst["st_parent"], gst["st_count"], s, W)
+    npar = 1 if dep == 1 else int(gst["st_count"][s, dep - 2])
+    cands = []
+    for p in range(npar):
+        path = () if dep == 1 else gp[(dep - 2) * W + p]
+        ps = 0.0 if dep == 1 else float(gst["st_score"][s, dep - 2, p])
+        tok, lq, lse, allq = oracle.node_children(cfg, x["Wi"], x["Wo"], x["E"], x["Dlog"][s], x["h0"][s],
+                                                  np.array(path, np.int32), min(k + 1, cfg.V),
+                                                  want_all=True)
+        for j in range(min(k + 1, cfg.V)):
+            cands.append((ps + lq[j] + cfg.beta, p, j, int(tok[j]), j < k))
+        if ref_logq is not None:
+            ref_logq[(s, dep, p)] = allq
+    gc = int(gst["st_count"][s, dep - 1])
+    kept = set()
+    for r in range(gc):
+        t = int(gst["st_tok"][s, dep - 1, r])
+        p = 0 if dep == 1 else int(gst["st_parent"][s, dep - 1, r])
+        match = [c for c in cands if c[1] == p and c[3] == t]
+        assert match, f"seq {s} depth {dep}: kept child ({p},{t}) is not among the parent's top-(k+1)"
+        c = match[0]
+        got = float(gst["st_score"][s, dep - 1, r])
+        assert abs(got - c[0]) <= tol_step, f"seq {s} depth {dep} rank {r}: score step off by {abs(got - c[0])}"
+        kept.add((p, t))
+    finite = [c for c in cands if c[4] and np.isfinite(c[0])]
+    assert gc == min(W, len(finite))
+    if gc:
+        lo = min(c[0] for c in cands if (c[1], c[3]) in kept)
+        others = [c[0] for c in cands if (c[1], c[3]) not in kept and c[4]]
+        if others:
+            assert lo >= max(others) - 2 * tol_step, f"seq {s} depth {dep}: kept set is not a top-W"

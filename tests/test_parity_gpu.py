@@ -1,0 +1,212 @@
+"""GPU parity: the CUDA path (through the C ABI) against the fp64 oracle.
+
+Small and mid-size cases are compared with a full oracle run (exact topology
+where the oracle's rank gaps exceed the tolerance, scores within tolerance);
+the full-size workloads are checked on sampled depths by teacher-forced
+oracle recomputation plus structural invariants.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from parity import (check_structure, compare_with_oracle, gpu_supertree, to_device, tol_of, tree_to_numpy,
+                    validate_frontier_teacher_forced)
+from workloads import BATCHED, Q4B, Q8B, TOY, Config, make_inputs, sweep_configs
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def dart():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2608_13524_gb300 import dart as d
+    d.lib()
+    return d
+
+
+def C(name, nseq, V, d, L, W, k, B, wdtype="bf16", T=0.0, seed=1, **kw):
+    return Config(name, nseq, V, d, L, W, k, B, wdtype, T, seed, **kw)
+
+
+SMALL = [
+    C("f32-small", 1, 1000, 128, 4, 4, 4, 10, "f32", 0.0, 11),
+    C("f32-groups", 3, 1500, 64, 3, 12, 4, 20, "f32", 0.7, 12),
+    C("bf16-small", 2, 1000, 128, 3, 4, 4, 7, "bf16", 1.0, 13),
+    C("bf16-mid", 1, 5003, 512, 5, 8, 8, 24, "bf16", 0.0, 14),
+    C("bf16-multitile", 1, 50000, 256, 4, 6, 7, 15, "bf16", 0.7, 15),
+    C("bf16-groups", 4, 3000, 256, 3, 24, 24, 50, "bf16", 1.0, 16),
+    C("bf16-N256", 8, 2000, 128, 3, 32, 8, 40, "bf16", 0.0, 17),
+    C("bf16-k64", 1, 4000, 128, 3, 64, 64, 100, "bf16", 0.0, 18),
+    C("bf16-d64", 1, 777, 64, 2, 3, 5, 4, "bf16", 0.0, 19),
+    C("bf16-L1", 2, 900, 128, 1, 5, 9, 3, "bf16", 0.0, 20),
+    C("bf16-chain", 1, 600, 128, 6, 1, 1, 6, "bf16", 0.0, 21),
+    C("bf16-B1", 1, 600, 128, 4, 4, 4, 1, "bf16", 0.0, 22),
+    C("bf16-Vk", 1, 8, 64, 4, 8, 8, 30, "bf16", 0.0, 23),
+    C("bf16-beta0", 1, 1200, 128, 4, 6, 3, 11, "bf16", 0.0, 24, beta=0.0),
+    C("bf16-kltW", 2, 1200, 128, 4, 9, 2, 25, "bf16", 0.0, 25, pos_offset=37),
+    TOY,
+]
+
+
+def run_depthwise(dart, cfg, dx):
+    """Expands depth by depth, collecting node lists / frontiers / states."""
+    h = dart.dart_init_head(cfg, dart.DART_BF16 if cfg.wdtype == "bf16" else dart.DART_F32,
+                            dx["Wi"], dx["Wo"], dx["E"])
+    per = []
+    try:
+        for dep in range(1, cfg.L + 1):
+            dart.dart_expand_depth(h, dep, dx["Dlog"], dx["h0"])
+            tok, lq, lse = dart.dart_get_node_topk(h, cfg)
+            st = dart.dart_get_states(h, cfg)
+            per.append(dict(tok=tok.cpu().numpy(), logq=lq.cpu().numpy(), lse=lse.cpu().numpy(),
+                            states=st.cpu().numpy()))
+        out_t, out = dart.alloc_tree_out(cfg)
+        dart.dart_prune_and_emit(h, out)
+        assert dart.dart_status_sync(h) == 0
+        gst = gpu_supertree(dart, h, cfg)
+        g = tree_to_numpy(out_t)
+    finally:
+        dart.dart_destroy(h)
+    return per, gst, g
+
+
+@pytest.mark.parametrize("cfg", SMALL, ids=[c.name for c in SMALL])
+def test_depthwise_parity(dart, cfg):
+    x = make_inputs(cfg)
+    dx = to_device(cfg, x)
+    ref = oracle.build_tree(cfg, x["Wi"], x["Wo"], x["E"], x["Dlog"], x["h0"])
+    per, gst, g = run_depthwise(dart, cfg, dx)
+    tol = tol_of(cfg)
+    rep = compare_with_oracle(cfg, ref, gst, g, tol)
+    print(cfg.name, rep)
+    # node-level lists and states while the frontiers agree exactly
+    caps = cfg.caps()
+    for dep in range(1, cfg.L + 1):
+        if any(t[0] == s and (t[1] == "prune" or t[1] <= dep - 1) for s in range(cfg.nseq) for t in rep["near_tie"]):
+            break
+        P = caps[dep - 1]
+        d = per[dep - 1]
+        for s in range(cfg.nseq):
+            npar = 1 if dep == 1 else int(ref["st_count"][s, dep - 2])
+            for p in range(npar):
+                row = s * P + p
+                rl = ref["nd_logq"][s, dep - 1, p, :cfg.k]
+                rt = ref["nd_tok"][s, dep - 1, p, :cfg.k]
+                assert abs(float(d["lse"][row]) - ref["nd_lse"][s, dep - 1, p]) <= tol
+                fin = np.isfinite(rl)
+                assert np.all(np.abs(d["logq"][row][fin] - rl[fin]) <= tol)
+                gaps = -np.diff(ref["nd_logq"][s, dep - 1, p])
+                if np.all(gaps[:cfg.k] >= tol):
+                    np.testing.assert_array_equal(d["tok"][row], rt)
+        if dep < cfg.L:
+            # states of the retained children vs teacher-forced oracle states
+            stol = 5e-4 if cfg.wdtype == "bf16" else 2e-5
+            for s in range(min(cfg.nseq, 2)):
+                paths = oracle.node_paths(ref["st_tok"], ref["st_parent"], ref["st_count"], s, cfg.W)
+                for r in range(min(int(ref["st_count"][s, dep - 1]), 4)):
+                    hs = oracle.path_state(cfg, x["Wi"], x["Wo"], x["E"], x["h0"][s],
+                                           np.array(paths[(dep - 1) * cfg.W + r], np.int32))
+                    got = d["states"][s * caps[dep] + r]
+                    assert np.max(np.abs(got - hs)) <= stol, (dep, s, r, np.max(np.abs(got - hs)))
+
+
+@pytest.mark.parametrize("cfg", SMALL[:6], ids=[c.name for c in SMALL[:6]])
+def test_build_tree_graph_matches_depthwise(dart, cfg):
+    """dart_build_tree (one cached CUDA graph) equals the depth-by-depth
+    calls, is deterministic across repeated launches, and the host-buffer
+    variant returns the same tree."""
+    x = make_inputs(cfg)
+    dx = to_device(cfg, x)
+    _, gst_ref, g_ref = run_depthwise(dart, cfg, dx)
+    eng = dart.Dart(cfg, dx["Wi"], dx["Wo"], dx["E"])
+    try:
+        for it in range(3):
+            out = eng.build_tree(dx["Dlog"], dx["h0"])
+            torch.cuda.synchronize()
+            g = tree_to_numpy(out)
+            for k in g:
+                np.testing.assert_array_equal(g[k], g_ref[k], err_msg=f"{k} (launch {it})")
+        assert dart.dart_status_sync(eng.h) == 0
+        ht, hout = dart.alloc_tree_out(cfg, pin=True)
+        Dh = dx["Dlog"].cpu().pin_memory()
+        h0h = dx["h0"].cpu().pin_memory()
+        dart.dart_build_tree_host(eng.h, Dh, h0h, hout)
+        for k in g_ref:
+            np.testing.assert_array_equal(ht[k].numpy(), g_ref[k], err_msg=k)
+    finally:
+        eng.close()
+
+
+def test_neg_inf_drafter_logits(dart):
+    cfg = C("neginf", 2, 700, 128, 4, 6, 4, 40, "bf16", 0.0, 31)
+    x = make_inputs(cfg)
+    x["Dlog"][0, 1, 3:] = -np.inf      # depth 2 of seq 0: only tokens 0..2 possible
+    x["Dlog"][1, 0, :] = -np.inf       # depth 1 of seq 1: no child at all
+    x["Dlog"][1, 0, 5] = 0.0           #   ... except token 5
+    dx = to_device(cfg, x)
+    ref = oracle.build_tree(cfg, x["Wi"], x["Wo"], x["E"], x["Dlog"], x["h0"])
+    _, gst, g = run_depthwise(dart, cfg, dx)
+    compare_with_oracle(cfg, ref, gst, g, tol_of(cfg))
+    assert int(gst["st_count"][1, 0]) == 1
+
+
+def test_call_order_and_argument_errors(dart):
+    cfg = C("err", 1, 500, 64, 3, 2, 2, 4, "bf16", 0.0, 41)
+    x = make_inputs(cfg)
+    dx = to_device(cfg, x)
+    h = dart.dart_init_head(cfg, dart.DART_BF16, dx["Wi"], dx["Wo"], dx["E"])
+    try:
+        out_t, out = dart.alloc_tree_out(cfg)
+        with pytest.raises(dart.DartError) as e:
+            dart.dart_expand_depth(h, 2, dx["Dlog"], dx["h0"])
+        assert e.value.code == dart.DART_ERR_STATE
+        with pytest.raises(dart.DartError) as e:
+            dart.dart_prune_and_emit(h, out)
+        assert e.value.code == dart.DART_ERR_STATE
+        dart.dart_expand_depth(h, 1, dx["Dlog"], dx["h0"])
+        with pytest.raises(dart.DartError) as e:
+            dart.dart_expand_depth(h, 3, dx["Dlog"], dx["h0"])
+        assert e.value.code == dart.DART_ERR_STATE
+        with pytest.raises(dart.DartError) as e:
+            dart.dart_expand_depth(h, 1, dx["Dlog"], None)   # anchor needed at depth 1
+        assert e.value.code == dart.DART_ERR_INVALID
+        dart.dart_expand_depth(h, 1, dx["Dlog"], dx["h0"])
+        dart.dart_expand_depth(h, 2, dx["Dlog"], None)
+        dart.dart_expand_depth(h, 3, dx["Dlog"], None)
+        dart.dart_prune_and_emit(h, out)
+        assert dart.dart_status_sync(h) == 0
+    finally:
+        dart.dart_destroy(h)
+
+
+# ----------------------------------------------------------------- full size
+
+FULL = [Q8B, Q4B, BATCHED, [c for c in sweep_configs() if c.W == 64 and c.B == 512][0]]
+
+
+@pytest.mark.parametrize("cfg", FULL, ids=[c.name for c in FULL])
+def test_full_size_sampled(dart, cfg):
+    """Full-size workloads in the launch configuration the benchmark times
+    (dart_build_tree, graph launch): structural invariants on every sequence,
+    teacher-forced oracle checks of the frontier and score increments at
+    sampled depths of the first sequence."""
+    x = make_inputs(cfg)
+    dx = to_device(cfg, x)
+    eng = dart.Dart(cfg, dx["Wi"], dx["Wo"], dx["E"])
+    try:
+        out = eng.build_tree(dx["Dlog"], dx["h0"])
+        assert dart.dart_status_sync(eng.h) == 0
+        g = tree_to_numpy(out)
+        gst = gpu_supertree(dart, eng.h, cfg)
+    finally:
+        eng.close()
+    check_structure(cfg, g)
+    caps = cfg.caps()
+    for s in range(cfg.nseq):
+        assert list(gst["st_count"][s]) == caps[1:]
+        assert g["n_nodes"][s] == min(cfg.B, sum(caps[1:]))
+    tol_step = tol_of(cfg) / cfg.L
+    for dep in sorted({1, 2, cfg.L}):
+        validate_frontier_teacher_forced(cfg, x, gst, 0, dep, tol_step)
