@@ -284,9 +284,12 @@ def main():
     pe1.record(stream)
     barrier()
     prof_ms_round = pe0.elapsed_time(pe1) / args.steps
-    k1_ms, k1_n = dart.dart_profile_read(h)
+    kinds = dart.dart_profile_read_kinds(h)
     dart.dart_set_profiling(h, False)
+    k1_ms, k1_n = kinds["lmhead"]
     k1_avg_s = k1_ms / 1e3 / max(1, k1_n)
+    breakdown = {k: {"us_per_round": v[0] * 1e3 / args.steps, "launches_per_round": v[1] / args.steps,
+                     "us_per_launch": v[0] * 1e3 / max(1, v[1])} for k, v in kinds.items() if v[1]}
 
     exp_round = cfg.expansions_per_round()
     value = exp_round * world / (ms / 1e3)
@@ -344,6 +347,7 @@ def main():
                          "traffic": traffic, "bytes_per_launch": bytes_launch,
                          "avg_launch_us": k1_avg_s * 1e6, "launches": k1_n,
                          "profiled_us_per_round": prof_ms_round * 1e3},
+            "kernel_breakdown": breakdown,
             "gpu_launches": launches * args.steps,
             "clocks": clk,
             "e2e": e2e,

@@ -165,6 +165,14 @@ int dart_status_sync(dart_handle *h, void *stream);
 int dart_set_profiling(dart_handle *h, int enable);
 int dart_profile_read(dart_handle *h, float *lmhead_ms, int *lmhead_launches);
 
+/* Per-kind breakdown of the same profiling events (every launch is
+ * bracketed while profiling is enabled).  Kinds: 0 LM-head scoring,
+ * 1 merge + frontier select, 2 head-input gather, 3 head GEMM W_i,
+ * 4 SiLU + split, 5 head GEMM W_o, 6 residual + RMSNorm, 7 depth-1 anchor
+ * preparation, 8 prune + emit.  ms[i] / launches[i] receive the summed device
+ * time and count of kind i for i < nkinds (nkinds <= 9); resets the events. */
+int dart_profile_read_kinds(dart_handle *h, float *ms, int *launches, int nkinds);
+
 /* Number of kernel launches one dart_build_tree enqueues for this handle. */
 int dart_launches_per_round(dart_handle *h);
 

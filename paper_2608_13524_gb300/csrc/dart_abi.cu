@@ -111,6 +111,7 @@ struct dart_handle {
     // profiling
     bool profiling;
     std::vector<cudaEvent_t> ev;
+    std::vector<int> ev_kind;
     int ev_used;
 };
 
@@ -190,8 +191,18 @@ int build_plans(dart_handle* h) {
         p.G = (p.N + p.NG - 1) / p.NG;
         p.nV = std::max(1, std::min(h->num_sms / p.G, tiles));
         if (tc) {
+            // Two CTAs per SM when both fit with >= 4 pipeline stages each: two
+            // independent TMA streams per SM, and one CTA's epilogue / start-up /
+            // tail overlaps the other's stream.
             const int fixed = lmhead_tc_fixed_smem(p.NG, c.k, 16);
-            p.stages = tc_stages(h->smem_optin, tc_stage_bytes(p.NG), fixed);
+            const int half = h->smem_optin / 2 - 2048;
+            const int st2 = tc_stages(half, tc_stage_bytes(p.NG), fixed);
+            if (st2 >= 4) {
+                p.stages = st2;
+                p.nV = std::max(1, std::min(2 * h->num_sms / p.G, tiles));
+            } else {
+                p.stages = tc_stages(h->smem_optin, tc_stage_bytes(p.NG), fixed);
+            }
             if (p.stages < 2) return DART_ERR_UNSUPPORTED;
             p.smem = lmhead_tc_fixed_smem(p.NG, c.k, p.stages) + p.stages * tc_stage_bytes(p.NG);
         } else {
@@ -320,13 +331,37 @@ void release(dart_handle* h) {
 
 // ---------------------------------------------------------------- enqueue
 
+enum Kind { kLmhead = 0, kSelect, kGather, kGemm1, kSilu, kGemm2, kNorm, kPrep, kEmit, kNumKinds };
+
+// Opens an event pair around the next launch when profiling (no-op otherwise).
+int prof_begin(dart_handle* h, int kind, cudaStream_t st) {
+    if (!h->profiling || h->ev_used + 2 > kMaxProfilePairs * 2) return -1;
+    while (static_cast<int>(h->ev.size()) < h->ev_used + 2) {
+        cudaEvent_t e;
+        if (cudaEventCreate(&e) != cudaSuccess) return -1;
+        h->ev.push_back(e);
+        h->ev_kind.push_back(-1);
+    }
+    const int i = h->ev_used;
+    h->ev_kind[i] = kind;
+    cudaEventRecord(h->ev[i], st);
+    return i;
+}
+void prof_end(dart_handle* h, int i, cudaStream_t st) {
+    if (i < 0) return;
+    cudaEventRecord(h->ev[i + 1], st);
+    h->ev_used = i + 2;
+}
+
 int enqueue_depth(dart_handle* h, int dep, const float* dlog, const float* anchor, cudaStream_t st) {
     const dart_config& c = h->cfg;
     const DepthPlan& p = h->plans[dep];
     const bool tc = h->wdtype == DART_BF16;
     cudaError_t e = cudaSuccess;
     if (dep == 1) {
+        const int pi = prof_begin(h, kPrep, st);
         e = launch_prep_anchor(anchor, c.nseq, c.d, h->hbuf[0], tc ? h->HL : nullptr, kNPadMax, st);
+        prof_end(h, pi, st);
         if (e != cudaSuccess) return DART_ERR_CUDA;
         h->cur = 0;
     }
@@ -353,21 +388,10 @@ int enqueue_depth(dart_handle* h, int dep, const float* dlog, const float* ancho
     la.status = h->status;
     la.h32 = h->hbuf[h->cur];
     la.E32 = static_cast<const float*>(h->E);
-    const bool prof = h->profiling && h->ev_used + 2 <= kMaxProfilePairs * 2;
-    if (prof) {
-        while (static_cast<int>(h->ev.size()) < h->ev_used + 2) {
-            cudaEvent_t ev;
-            if (cudaEventCreate(&ev) != cudaSuccess) return DART_ERR_CUDA;
-            h->ev.push_back(ev);
-        }
-        cudaEventRecord(h->ev[h->ev_used], st);
-    }
+    int pi = prof_begin(h, kLmhead, st);
     e = tc ? launch_lmhead_tc(&h->tmE, &h->tmH[ng_index(p.NG)], la, p.smem, st) : launch_lmhead_f32(la, st);
+    prof_end(h, pi, st);
     if (e != cudaSuccess) return DART_ERR_CUDA;
-    if (prof) {
-        cudaEventRecord(h->ev[h->ev_used + 1], st);
-        h->ev_used += 2;
-    }
     // 2) merge partials, log q~, Eq. 5 scores, global top-W -> S_dep
     SelectArgs sa;
     std::memset(&sa, 0, sizeof sa);
@@ -394,19 +418,24 @@ int enqueue_depth(dart_handle* h, int dep, const float* dlog, const float* ancho
     sa.child_tok = h->child_tok;
     sa.seq_ticket = h->seq_ticket;
     sa.status = h->status;
-    if (launch_merge_select(sa, st) != cudaSuccess) return DART_ERR_CUDA;
+    pi = prof_begin(h, kSelect, st);
+    e = launch_merge_select(sa, st);
+    prof_end(h, pi, st);
+    if (e != cudaSuccess) return DART_ERR_CUDA;
     h->last_rows = p.N;
     if (dep == c.L) return DART_OK;
     // 3) correction-head update of the retained children (Algorithm 1, state update)
     const float* hcur = h->hbuf[h->cur];
     float* hnext = h->hbuf[1 - h->cur];
-    if (launch_gather_x(p.Nc, c.d, h->child_prow, h->child_tok, hcur, h->E, tc ? 1 : 0, h->XL, kNPadMax, h->X32,
-                        st) != cudaSuccess)
-        return DART_ERR_CUDA;
+    pi = prof_begin(h, kGather, st);
+    e = launch_gather_x(p.Nc, c.d, h->child_prow, h->child_tok, hcur, h->E, tc ? 1 : 0, h->XL, kNPadMax, h->X32, st);
+    prof_end(h, pi, st);
+    if (e != cudaSuccess) return DART_ERR_CUDA;
     GemmArgs g1 = p.g1, g2 = p.g2;
     g1.out = h->part;
     g2.out = h->part;
     g1.status = g2.status = h->status;
+    pi = prof_begin(h, kGemm1, st);
     if (tc) {
         e = launch_gemm_tc(&h->tmWi, &h->tmX[ng_index(g1.NG)], g1, p.g1_smem, st);
     } else {
@@ -414,9 +443,13 @@ int enqueue_depth(dart_handle* h, int dep, const float* dlog, const float* ancho
         g1.B32 = h->X32;
         e = launch_gemm_f32(g1, st);
     }
+    prof_end(h, pi, st);
     if (e != cudaSuccess) return DART_ERR_CUDA;
-    if (launch_silu_split(p.Nc, c.d, g1.S, h->part, tc ? h->AL : nullptr, kNPadMax, h->A32, st) != cudaSuccess)
-        return DART_ERR_CUDA;
+    pi = prof_begin(h, kSilu, st);
+    e = launch_silu_split(p.Nc, c.d, g1.S, h->part, tc ? h->AL : nullptr, kNPadMax, h->A32, st);
+    prof_end(h, pi, st);
+    if (e != cudaSuccess) return DART_ERR_CUDA;
+    pi = prof_begin(h, kGemm2, st);
     if (tc) {
         e = launch_gemm_tc(&h->tmWo, &h->tmA[ng_index(g2.NG)], g2, p.g2_smem, st);
     } else {
@@ -424,10 +457,13 @@ int enqueue_depth(dart_handle* h, int dep, const float* dlog, const float* ancho
         g2.B32 = h->A32;
         e = launch_gemm_f32(g2, st);
     }
+    prof_end(h, pi, st);
     if (e != cudaSuccess) return DART_ERR_CUDA;
-    if (launch_residual_norm(p.Nc, c.d, g2.S, h->part, h->child_prow, hcur, c.rms_eps, hnext, tc ? h->HL : nullptr,
-                             kNPadMax, st) != cudaSuccess)
-        return DART_ERR_CUDA;
+    pi = prof_begin(h, kNorm, st);
+    e = launch_residual_norm(p.Nc, c.d, g2.S, h->part, h->child_prow, hcur, c.rms_eps, hnext, tc ? h->HL : nullptr,
+                             kNPadMax, st);
+    prof_end(h, pi, st);
+    if (e != cudaSuccess) return DART_ERR_CUDA;
     h->cur = 1 - h->cur;
     h->last_rows = p.Nc;
     return DART_OK;
@@ -462,7 +498,10 @@ int enqueue_emit(dart_handle* h, const dart_tree_out* o, cudaStream_t st) {
     a.scores = o->scores;
     a.mask = o->mask;
     a.status = h->status;
-    return launch_prune_emit(a, st) == cudaSuccess ? DART_OK : DART_ERR_CUDA;
+    const int pi = prof_begin(h, kEmit, st);
+    const cudaError_t e = launch_prune_emit(a, st);
+    prof_end(h, pi, st);
+    return e == cudaSuccess ? DART_OK : DART_ERR_CUDA;
 }
 
 int enqueue_round(dart_handle* h, const float* dlog, const float* anchor, const dart_tree_out* out, cudaStream_t st) {
@@ -716,20 +755,31 @@ int dart_set_profiling(dart_handle* h, int enable) {
     return DART_OK;
 }
 
-int dart_profile_read(dart_handle* h, float* lmhead_ms, int* lmhead_launches) {
-    if (!h) return DART_ERR_INVALID;
-    float total = 0.0f;
+int dart_profile_read_kinds(dart_handle* h, float* ms, int* launches, int nkinds) {
+    if (!h || nkinds < 0 || nkinds > kNumKinds) return DART_ERR_INVALID;
+    float tot[kNumKinds] = {0};
+    int cnt[kNumKinds] = {0};
     const int pairs = h->ev_used / 2;
     if (pairs > 0 && cudaEventSynchronize(h->ev[h->ev_used - 1]) != cudaSuccess) return DART_ERR_CUDA;
     for (int i = 0; i < pairs; i++) {
-        float ms = 0.0f;
-        if (cudaEventElapsedTime(&ms, h->ev[2 * i], h->ev[2 * i + 1]) != cudaSuccess) return DART_ERR_CUDA;
-        total += ms;
+        float t = 0.0f;
+        if (cudaEventElapsedTime(&t, h->ev[2 * i], h->ev[2 * i + 1]) != cudaSuccess) return DART_ERR_CUDA;
+        const int k = h->ev_kind[2 * i];
+        if (k >= 0 && k < kNumKinds) {
+            tot[k] += t;
+            cnt[k]++;
+        }
     }
-    if (lmhead_ms) *lmhead_ms = total;
-    if (lmhead_launches) *lmhead_launches = pairs;
+    for (int k = 0; k < nkinds; k++) {
+        if (ms) ms[k] = tot[k];
+        if (launches) launches[k] = cnt[k];
+    }
     h->ev_used = 0;
     return DART_OK;
+}
+
+int dart_profile_read(dart_handle* h, float* lmhead_ms, int* lmhead_launches) {
+    return dart_profile_read_kinds(h, lmhead_ms, lmhead_launches, 1);
 }
 
 int dart_launches_per_round(dart_handle* h) {

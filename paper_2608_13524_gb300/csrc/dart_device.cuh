@@ -36,6 +36,14 @@ __device__ __forceinline__ unsigned long long globaltimer_ns() {
     return t;
 }
 
+// Programmatic dependent launch.  pdl_trigger lets the next kernel of the
+// stream start its prologue early; pdl_wait blocks until every prerequisite
+// kernel has completed and its memory is visible.  Every kernel calls
+// pdl_wait before it touches data written by an earlier kernel (or data an
+// earlier kernel still reads), so completion is transitive along the stream.
+__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
 __device__ __forceinline__ void named_bar_sync(int id, int nthreads) {
     asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(nthreads) : "memory");
 }
@@ -256,29 +264,28 @@ __device__ __forceinline__ uint64_t block_kth_largest(const uint64_t* keys, int 
 
 // ------------------------------------------------ fused LM-head epilogue
 //
-// Per node (column) of a 128-row tile, every epilogue thread owns one
-// vocabulary row.  It keeps, per warp and node, a running (max, sum exp) for
-// the log-sum-exp, and per node a CTA-local top-k list of keys.  A value
-// enters the tile's candidate buffer only if it beats the node's current
-// k-th key; after the tile the buffers are merged into the lists by rank.
+// Every epilogue thread owns one vocabulary row of a 128-row tile and sees
+// the scaled logits of its row for the CTA's node group, 16 nodes (one
+// "chunk") at a time.  Per node it keeps:
+//   * log-sum-exp: per warp, a reference max m_ref (shared memory) and a
+//     running sum of exp(z - m_ref) (a register of the lanes 2j, 2j+1 after
+//     the butterfly reduction).  m_ref is raised -- and the sum rescaled --
+//     only when some logit exceeds it by more than kRefSlack, so after the
+//     first tile the exact warp max is almost never needed;
+//   * top-k: a CTA-wide list of keys (shared memory, sorted).  A logit
+//     enters the tile's candidate buffer only if it beats the node's current
+//     k-th key; after the tile one warp per node merges the candidates.
+
+constexpr unsigned kFull = 0xFFFFFFFFu;
+constexpr float kRefSlack = 30.0f;  // exp(30) ~ 1e13: sums stay far from fp32 overflow
 
 struct EpiSmem {
     uint64_t* list;   // [NG][k]   sorted desc, 0 = empty
     uint64_t* cand;   // [NG][kCandCap]
     int* cnt;         // [NG]
-    float2* stats;    // [4][NG]  (max, sum exp) per epilogue warp
+    float* mref;      // [4][NG]  per-warp reference max
+    float2* stats;    // [4][NG]  (reference, sum exp) per epilogue warp at the end
 };
-
-__device__ __forceinline__ float warp_max(float v) {
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xFFFFFFFFu, v, o));
-    return v;
-}
-__device__ __forceinline__ float warp_sum(float v) {
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xFFFFFFFFu, v, o);
-    return v;
-}
 
 // (m, s) <- (m, s) (+) (m2, s2) for sums of exp relative to their maxima.
 __device__ __forceinline__ float2 lse_merge(float2 a, float2 b) {
@@ -288,65 +295,202 @@ __device__ __forceinline__ float2 lse_merge(float2 a, float2 b) {
     return make_float2(m, a.y * __expf(a.x - m) + b.y * __expf(b.x - m));
 }
 
+__device__ __forceinline__ float warp_max(float v) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(kFull, v, o));
+    return v;
+}
+
+// Butterfly reduction of 16 values per lane over the warp: returns, in
+// lanes 2j and 2j+1, the reduction of v[j] over all 32 lanes (16 shuffles).
+template <bool kMax>
+__device__ __forceinline__ float bfly16(const float (&v)[16], int lane) {
+    auto op = [](float x, float y) { return kMax ? fmaxf(x, y) : x + y; };
+    float a[8], b[4], c[2];
+    const bool h4 = lane & 16, h3 = lane & 8, h2 = lane & 4, h1 = lane & 2;
+#pragma unroll
+    for (int i = 0; i < 8; i++) a[i] = op(h4 ? v[8 + i] : v[i], __shfl_xor_sync(kFull, h4 ? v[i] : v[8 + i], 16));
+#pragma unroll
+    for (int i = 0; i < 4; i++) b[i] = op(h3 ? a[4 + i] : a[i], __shfl_xor_sync(kFull, h3 ? a[i] : a[4 + i], 8));
+#pragma unroll
+    for (int i = 0; i < 2; i++) c[i] = op(h2 ? b[2 + i] : b[i], __shfl_xor_sync(kFull, h2 ? b[i] : b[2 + i], 4));
+    const float d = op(h1 ? c[1] : c[0], __shfl_xor_sync(kFull, h1 ? c[0] : c[1], 2));
+    return op(d, __shfl_xor_sync(kFull, d, 1));
+}
+
 __device__ __forceinline__ void epi_init(const EpiSmem& e, int NG, int k, int etid) {
     for (int i = etid; i < NG * k; i += kEpiThreads) e.list[i] = 0ull;
     for (int i = etid; i < NG; i += kEpiThreads) e.cnt[i] = 0;
-    for (int i = etid; i < 4 * NG; i += kEpiThreads) e.stats[i] = make_float2(-INFINITY, 0.0f);
+    for (int i = etid; i < 4 * NG; i += kEpiThreads) e.mref[i] = -INFINITY;
 }
 
-// One (row, node) value.  Must be called by all 32 lanes of the warp with the
-// same node.  `z` is the scaled logit, `valid` whether the row is < V.
-__device__ __forceinline__ void epi_value(const EpiSmem& e, int NG, int k, int ew, int lane, int node, float z,
-                                          bool valid, uint32_t row) {
-    const float m = warp_max(valid ? z : -INFINITY);
-    const float p = (valid && m != -INFINITY) ? __expf(z - m) : 0.0f;
-    const float s = warp_sum(p);
-    if (lane == 0) e.stats[ew * NG + node] = lse_merge(e.stats[ew * NG + node], make_float2(m, s));
-    const uint64_t key = valid ? make_key(z, row) : 0ull;
-    const bool pass = key > e.list[node * k + k - 1];
-    const unsigned bal = __ballot_sync(0xFFFFFFFFu, pass);
-    if (bal) {
-        int base = 0;
-        if (lane == 0) base = atomicAdd(&e.cnt[node], __popc(bal));
-        base = __shfl_sync(0xFFFFFFFFu, base, 0);
-        if (pass) e.cand[node * kCandCap + base + __popc(bal & ((1u << lane) - 1u))] = key;
+// One 16-node chunk of this thread's row (all 32 lanes, same chunk).
+// z[j]: scaled logit of node c0+j of the group; node j exists iff bit j of
+// nodemask is set; rowvalid: the row is < V.  ssum: the running sum of this
+// lane's node (c0 + lane/2).
+__device__ __forceinline__ void epi_chunk(const EpiSmem& e, int NG, int k, int ew, int lane, int c0,
+                                          float (&z)[16], uint32_t nodemask, bool rowvalid, uint32_t row,
+                                          float& ssum) {
+    bool ok[16];
+#pragma unroll
+    for (int j = 0; j < 16; j++) {
+        ok[j] = rowvalid && ((nodemask >> j) & 1u);
+        if (!ok[j]) z[j] = -INFINITY;
+        else if (z[j] == 0.0f) z[j] = 0.0f;  // -0 -> +0
+    }
+    float* mr = e.mref + ew * NG + c0;
+    bool slow = false;
+#pragma unroll
+    for (int j = 0; j < 16; j++) slow |= z[j] > mr[j] + kRefSlack;
+    if (__any_sync(kFull, slow)) {
+        const float mx = bfly16<true>(z, lane);
+        const int me = lane >> 1;
+        const float old = mr[me];
+        const float nm = fmaxf(old, mx);
+        if (old != -INFINITY && nm > old) ssum *= __expf(old - nm);
+        __syncwarp();
+        if ((lane & 1) == 0) mr[me] = nm;
+        __syncwarp();
+    }
+    float p[16];
+#pragma unroll
+    for (int j = 0; j < 16; j++) p[j] = z[j] != -INFINITY ? __expf(z[j] - mr[j]) : 0.0f;
+    ssum += bfly16<false>(p, lane);
+    uint64_t key[16];
+    bool pass[16];
+    bool anyp = false;
+#pragma unroll
+    for (int j = 0; j < 16; j++) {
+        key[j] = ok[j] ? make_key(z[j], row) : 0ull;
+        pass[j] = key[j] > e.list[(c0 + j) * k + k - 1];
+        anyp |= pass[j];
+    }
+    if (__any_sync(kFull, anyp)) {
+#pragma unroll
+        for (int j = 0; j < 16; j++) {
+            const unsigned bal = __ballot_sync(kFull, pass[j]);
+            if (bal) {
+                int base = 0;
+                if (lane == 0) base = atomicAdd(&e.cnt[c0 + j], __popc(bal));
+                base = __shfl_sync(kFull, base, 0);
+                if (pass[j]) e.cand[(c0 + j) * kCandCap + base + __popc(bal & ((1u << lane) - 1u))] = key[j];
+            }
+        }
     }
 }
 
-// Merge every node's candidates into its list (after all values of a tile).
-// Called by all kEpiThreads epilogue threads.
-__device__ __forceinline__ void epi_merge(const EpiSmem& e, int NG, int k, int etid) {
-    named_bar_sync(kEpiBarrier, kEpiThreads);
-    for (int nd = 0; nd < NG; nd++) {
-        const int c = e.cnt[nd];
-        if (c == 0) continue;  // uniform: every thread reads the same count
-        uint64_t* Ln = e.list + nd * k;
-        const uint64_t* Cn = e.cand + nd * kCandCap;
-        const int total = k + c;
-        uint64_t x[2] = {0ull, 0ull};
-        int r[2] = {k, k};
+__device__ __forceinline__ uint64_t shfl_u64(uint64_t v, int src) {
+    const uint32_t lo = __shfl_sync(kFull, static_cast<uint32_t>(v), src);
+    const uint32_t hi = __shfl_sync(kFull, static_cast<uint32_t>(v >> 32), src);
+    return (static_cast<uint64_t>(hi) << 32) | lo;
+}
+__device__ __forceinline__ uint64_t shfl_xor_u64(uint64_t v, int m) {
+    const uint32_t lo = __shfl_xor_sync(kFull, static_cast<uint32_t>(v), m);
+    const uint32_t hi = __shfl_xor_sync(kFull, static_cast<uint32_t>(v >> 32), m);
+    return (static_cast<uint64_t>(hi) << 32) | lo;
+}
+__device__ __forceinline__ uint64_t shfl_up_u64(uint64_t v, int dlt) {
+    const uint32_t lo = __shfl_up_sync(kFull, static_cast<uint32_t>(v), dlt);
+    const uint32_t hi = __shfl_up_sync(kFull, static_cast<uint32_t>(v >> 32), dlt);
+    return (static_cast<uint64_t>(hi) << 32) | lo;
+}
+
+// Merges the c candidate keys C[0..c) into the sorted list L[0..k) (k <= 64)
+// with one warp.  Keys are distinct; 0 marks empty slots.
+__device__ __forceinline__ void warp_merge(uint64_t* L, const uint64_t* C, int c, int k, int lane) {
+    if (c <= 4) {
+        // few candidates: insert one at a time into the register-held list
+        uint64_t a0 = lane < k ? L[lane] : 0ull;
+        uint64_t a1 = lane + 32 < k ? L[lane + 32] : 0ull;
+        for (int i = 0; i < c; i++) {
+            const uint64_t x = C[i];
+            const int p = __popc(__ballot_sync(kFull, a0 > x)) + __popc(__ballot_sync(kFull, a1 > x));
+            if (p >= k) continue;
+            const uint64_t u0 = shfl_up_u64(a0, 1), u1 = shfl_up_u64(a1, 1), l0 = shfl_u64(a0, 31);
+            const uint64_t n0 = lane > p ? u0 : (lane == p ? x : a0);
+            const uint64_t n1 = lane + 32 > p ? (lane == 0 ? l0 : u1) : (lane + 32 == p ? x : a1);
+            a0 = n0;
+            a1 = n1;
+        }
+        __syncwarp();
+        if (lane < k) L[lane] = a0;
+        if (lane + 32 < k) L[lane + 32] = a1;
+        __syncwarp();
+        return;
+    }
+    for (int b = 0; b < c; b += 32) {
+        const int nb = min(32, c - b);
+        uint64_t x = lane < nb ? C[b + lane] : 0ull;
+        // bitonic sort of the batch, descending across lanes
 #pragma unroll
-        for (int it = 0; it < 2; it++) {
-            const int i = etid + it * kEpiThreads;
-            if (i < total) {
-                int rank = 0;
-                if (i < k) {
-                    x[it] = Ln[i];
-                    rank = i;
-                } else {
-                    x[it] = Cn[i - k];
-                    for (int j = 0; j < k; j++) rank += Ln[j] > x[it];
-                }
-                for (int j = 0; j < c; j++) rank += Cn[j] > x[it];
-                r[it] = rank;
+        for (int size = 2; size <= 32; size <<= 1) {
+#pragma unroll
+            for (int stride = size >> 1; stride > 0; stride >>= 1) {
+                const uint64_t y = shfl_xor_u64(x, stride);
+                const bool desc_block = (lane & size) == 0;
+                const bool lower = (lane & stride) == 0;
+                const bool keep_max = lower == desc_block;
+                x = keep_max ? (x > y ? x : y) : (x < y ? x : y);
             }
         }
-        named_bar_sync(kEpiBarrier, kEpiThreads);
+        // new position of the batch element = #{list > x} + its rank in the batch
+        int lo = 0, hi = k;
+        while (lo < hi) {
+            const int mid = (lo + hi) >> 1;
+            if (L[mid] > x)
+                lo = mid + 1;
+            else
+                hi = mid;
+        }
+        const int posx = lo + lane;
+        // new position of a list element = old position + #{batch > element}
+        uint64_t ent[2];
+        int posn[2];
 #pragma unroll
-        for (int it = 0; it < 2; it++)
-            if (r[it] < k) Ln[r[it]] = x[it];
-        if (etid == 0) e.cnt[nd] = 0;
-        named_bar_sync(kEpiBarrier, kEpiThreads);
+        for (int t = 0; t < 2; t++) {
+            const int pos = lane + 32 * t;
+            ent[t] = pos < k ? L[pos] : 0ull;
+            int l2 = 0, h2 = 32;
+#pragma unroll
+            for (int it = 0; it < 6; it++) {
+                const int mid = (l2 + h2) >> 1;
+                const uint64_t bm = shfl_u64(x, mid & 31);
+                if (l2 < h2) {
+                    if (bm > ent[t])
+                        l2 = mid + 1;
+                    else
+                        h2 = mid;
+                }
+            }
+            posn[t] = pos + l2;
+        }
+        __syncwarp();
+        if (posx < k && x != 0ull) L[posx] = x;
+#pragma unroll
+        for (int t = 0; t < 2; t++)
+            if (lane + 32 * t < k && posn[t] < k) L[posn[t]] = ent[t];
+        __syncwarp();
+    }
+}
+
+// Merges every node's tile candidates into its list: one warp per node, no
+// block barrier between nodes.  Called by all epilogue threads.
+__device__ __forceinline__ void epi_merge(const EpiSmem& e, int NG, int k, int ew, int lane) {
+    named_bar_sync(kEpiBarrier, kEpiThreads);
+    for (int nd = ew; nd < NG; nd += 4) {
+        const int c = e.cnt[nd];
+        if (c == 0) continue;
+        warp_merge(e.list + nd * k, e.cand + nd * kCandCap, c, k, lane);
+        if (lane == 0) e.cnt[nd] = 0;
+    }
+    named_bar_sync(kEpiBarrier, kEpiThreads);
+}
+
+// Records this warp's (reference, sum) of chunk cc's nodes.
+__device__ __forceinline__ void epi_stash(const EpiSmem& e, int NG, int ew, int lane, int c0, float ssum) {
+    if ((lane & 1) == 0) {
+        const int nd = c0 + (lane >> 1);
+        e.stats[ew * NG + nd] = make_float2(e.mref[ew * NG + nd], ssum);
     }
 }
 

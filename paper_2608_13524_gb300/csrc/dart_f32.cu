@@ -16,13 +16,16 @@ constexpr int kEPad = kBlockK + 1;  // padded row of the staged E tile (no bank 
 template <int NG>
 __global__ void __launch_bounds__(kEpiThreads) lmhead_f32_kernel(const LmheadArgs a) {
     extern __shared__ float smf[];
+    pdl_trigger();
+    pdl_wait();
     float* Es = smf;                     // [128][65]
     float* Hs = Es + kTileM * kEPad;     // [NG][64]
     EpiSmem e;
     e.list = reinterpret_cast<uint64_t*>(Hs + NG * kBlockK);
     e.cand = e.list + NG * a.k;
     e.stats = reinterpret_cast<float2*>(e.cand + NG * kCandCap);
-    e.cnt = reinterpret_cast<int*>(e.stats + 4 * NG);
+    e.mref = reinterpret_cast<float*>(e.stats + 4 * NG);
+    e.cnt = reinterpret_cast<int*>(e.mref + 4 * NG);
 
     const int g = blockIdx.x % a.G;
     const int vr = blockIdx.x / a.G;
@@ -31,6 +34,9 @@ __global__ void __launch_bounds__(kEpiThreads) lmhead_f32_kernel(const LmheadArg
     const int tid = threadIdx.x, lane = tid & 31, ew = tid >> 5;
     const int KB = a.d / kBlockK;
     epi_init(e, NG, a.k, tid);
+    float ssum[NG / 16];
+#pragma unroll
+    for (int c = 0; c < NG / 16; c++) ssum[c] = 0.0f;
 
     for (int t = t0; t < t1; t++) {
         float acc[NG];
@@ -69,19 +75,29 @@ __global__ void __launch_bounds__(kEpiThreads) lmhead_f32_kernel(const LmheadArg
         int cur_seq = -1;
         float dl = 0.0f;
 #pragma unroll
-        for (int j = 0; j < NG; j++) {
-            const int n = g * NG + j;
-            if (n < a.N) {
-                const int seq = n / a.P;
-                if (seq != cur_seq) {
-                    cur_seq = seq;
-                    dl = valid ? __ldg(a.dlog + seq * a.dlog_seq_stride + a.dlog_row_off + v) : 0.0f;
+        for (int c0 = 0; c0 < NG; c0 += 16) {
+            float z[16];
+            uint32_t nodemask = 0;
+#pragma unroll
+            for (int j = 0; j < 16; j++) {
+                const int n = g * NG + c0 + j;
+                z[j] = 0.0f;
+                if (n < a.N) {
+                    nodemask |= 1u << j;
+                    const int seq = n / a.P;
+                    if (seq != cur_seq) {
+                        cur_seq = seq;
+                        dl = valid ? __ldg(a.dlog + seq * a.dlog_seq_stride + a.dlog_row_off + v) : 0.0f;
+                    }
+                    z[j] = (acc[c0 + j] + dl) * a.invT;
                 }
-                epi_value(e, NG, a.k, ew, lane, j, (acc[j] + dl) * a.invT, valid, static_cast<uint32_t>(v));
             }
+            epi_chunk(e, NG, a.k, ew, lane, c0, z, nodemask, valid, static_cast<uint32_t>(v), ssum[c0 / 16]);
         }
-        epi_merge(e, NG, a.k, tid);
+        epi_merge(e, NG, a.k, ew, lane);
     }
+#pragma unroll
+    for (int c0 = 0; c0 < NG; c0 += 16) epi_stash(e, NG, ew, lane, c0, ssum[c0 / 16]);
     epi_finalize(e, NG, a.k, tid, g * NG, a.N, vr, a.part_ms, a.part_key);
 }
 
@@ -92,6 +108,8 @@ constexpr int kGM = 64, kGN = 16, kGK = 32;
 __global__ void __launch_bounds__(256) gemm_f32_kernel(const GemmArgs a) {
     __shared__ float As[kGM][kGK + 1];
     __shared__ float Bs[kGN][kGK + 1];
+    pdl_trigger();
+    pdl_wait();
     const int mt = blockIdx.x % a.MT;
     const int rest = blockIdx.x / a.MT;
     const int g = rest % a.G;
@@ -135,7 +153,7 @@ __global__ void __launch_bounds__(256) gemm_f32_kernel(const GemmArgs a) {
 
 template <int NG>
 int smem_ng(int k) {
-    return (kTileM * kEPad + NG * kBlockK) * 4 + NG * k * 8 + NG * kCandCap * 8 + 4 * NG * 8 + NG * 4;
+    return (kTileM * kEPad + NG * kBlockK) * 4 + NG * k * 8 + NG * kCandCap * 8 + 4 * NG * 8 + 4 * NG * 4 + NG * 4;
 }
 
 }  // namespace
@@ -151,18 +169,13 @@ cudaError_t f32_set_smem_limits(int max_dyn) {
 
 cudaError_t launch_lmhead_f32(const LmheadArgs& a, cudaStream_t st) {
     const int smem = lmhead_f32_smem(a.NG, a.k);
-    if (a.NG == 16)
-        lmhead_f32_kernel<16><<<a.nV * a.G, kEpiThreads, smem, st>>>(a);
-    else if (a.NG == 32)
-        lmhead_f32_kernel<32><<<a.nV * a.G, kEpiThreads, smem, st>>>(a);
-    else
-        return cudaErrorInvalidValue;
-    return cudaGetLastError();
+    if (a.NG == 16) return launch_pdl(lmhead_f32_kernel<16>, dim3(a.nV * a.G), dim3(kEpiThreads), smem, st, a);
+    if (a.NG == 32) return launch_pdl(lmhead_f32_kernel<32>, dim3(a.nV * a.G), dim3(kEpiThreads), smem, st, a);
+    return cudaErrorInvalidValue;
 }
 
 cudaError_t launch_gemm_f32(const GemmArgs& a, cudaStream_t st) {
-    gemm_f32_kernel<<<a.MT * a.G * a.S, 256, 0, st>>>(a);
-    return cudaGetLastError();
+    return launch_pdl(gemm_f32_kernel, dim3(a.MT * a.G * a.S), dim3(256), 0, st, a);
 }
 
 }  // namespace dart

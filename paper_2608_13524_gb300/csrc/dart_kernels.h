@@ -7,6 +7,26 @@
 
 namespace dart {
 
+// Launches `kernel` with programmatic stream serialization (PDL), so its
+// prologue can overlap the tail of the previous kernel in the stream.
+bool pdl_enabled();
+
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t st,
+                       Args&&... args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = pdl_enabled() ? 1 : 0;
+    return cudaLaunchKernelEx(&cfg, kernel, static_cast<Args&&>(args)...);
+}
+
 // LM-head scoring (Algorithm 1: correct every prefix of S_{d-1} over the full
 // vocabulary, Appendix D "Full"): per node n and vocabulary row v,
 //   z[n][v] = (Dlog[seq(n)][dep-1][v] + E[v] . h[n]) * invT,

@@ -12,6 +12,8 @@
 //       ancestor bit mask.
 //   prep / gather / silu / residual_norm: the elementwise parts of the
 //       fallback correction head around the two GEMMs.
+#include <cstdlib>
+
 #include "dart_device.cuh"
 #include "dart_kernels.h"
 
@@ -46,38 +48,80 @@ __device__ __forceinline__ float block_sum_float(float v, float* red) {
     return t;
 }
 
-// Selects the kk largest nonzero keys (kk >= 1, at least kk nonzero keys
-// present) and writes them in descending order to out[0..kk).
-__device__ __forceinline__ void block_topk_sorted(const uint64_t* keys, int n, int kk, uint64_t* out,
-                                                  uint64_t* sel, uint32_t* hist, int* scal) {
-    const uint64_t kth = block_kth_largest(keys, n, kk, hist, scal);
-    if (threadIdx.x == 0) scal[2] = 0;
-    __syncthreads();
-    for (int i = threadIdx.x; i < n; i += blockDim.x) {
-        const uint64_t x = keys[i];
-        if (x != 0ull && x >= kth) sel[atomicAdd(&scal[2], 1)] = x;
+constexpr int kRankMax = 1024;  // candidate count up to which an O(n^2 / threads) rank sort is used
+
+// Writes the kk largest nonzero keys, in descending order, to out[0..kk).
+// `keys` holds nlists lists of `len` keys, each sorted in descending order
+// with zeros (empty slots) last; at least kk keys are nonzero.  A key can
+// only be among the kk largest if it is >= the kk-th largest list head, and
+// only the kk lists whose heads reach that threshold can hold such keys, so
+// at most kk*len keys survive the filter; the survivors are ranked by
+// counting.  A block-wide radix select handles any larger survivor set.
+// `surv` has kRankMax slots.  Every thread of the block must call this.
+__device__ __forceinline__ void topk_of_sorted_lists(const uint64_t* keys, int nlists, int len, int kk,
+                                                     uint64_t* out, uint64_t* surv, uint64_t* thr,
+                                                     uint32_t* hist, int* scal) {
+    const int tid = threadIdx.x, nt = blockDim.x;
+    const int n = nlists * len;
+    if (tid == 0) {
+        *thr = 0ull;
+        scal[2] = 0;
     }
     __syncthreads();
-    for (int i = threadIdx.x; i < kk; i += blockDim.x) {
-        const uint64_t x = sel[i];
+    if (n > kRankMax && nlists > kk) {
+        for (int r = tid; r < nlists; r += nt) {
+            const uint64_t h = keys[r * len];
+            if (h == 0ull) continue;
+            int rank = 0;
+            for (int q = 0; q < nlists; q++) rank += keys[q * len] > h;
+            if (rank == kk - 1) *thr = h;
+        }
+        __syncthreads();
+    }
+    const uint64_t T = *thr;
+    for (int i = tid; i < n; i += nt) {
+        const uint64_t x = keys[i];
+        if (x != 0ull && x >= T) {
+            const int pos = atomicAdd(&scal[2], 1);
+            if (pos < kRankMax) surv[pos] = x;
+        }
+    }
+    __syncthreads();
+    const int m = scal[2];
+    if (m > kRankMax) {
+        const uint64_t kth = block_kth_largest(keys, n, kk, hist, scal);
+        if (tid == 0) scal[2] = 0;
+        __syncthreads();
+        for (int i = tid; i < n; i += nt) {
+            const uint64_t x = keys[i];
+            if (x != 0ull && x >= kth) surv[atomicAdd(&scal[2], 1)] = x;
+        }
+        __syncthreads();
+    }
+    const int mm = m > kRankMax ? kk : m;
+    for (int i = tid; i < mm; i += nt) {
+        const uint64_t x = surv[i];
         int r = 0;
-        for (int j = 0; j < kk; j++) r += sel[j] > x;
-        out[r] = x;
+        for (int j = 0; j < mm; j++) r += surv[j] > x;
+        if (r < kk) out[r] = x;
     }
     __syncthreads();
 }
 
 __global__ void __launch_bounds__(kSelThreads) merge_select_kernel(const SelectArgs a) {
-    extern __shared__ uint64_t keys[];  // max(nV*k, W*k) keys, then 2 x 64 selection slots
+    pdl_trigger();
+    pdl_wait();
+    extern __shared__ uint64_t keys[];  // max(nV*k, W*k) keys, kRankMax survivors, 64 outputs
     __shared__ uint32_t hist[256];
     __shared__ int scal[4];
+    __shared__ uint64_t thr;
     __shared__ float redf[32];
     __shared__ float redm[32];
     __shared__ int redi[32];
     __shared__ int ticket;
     const int cap = max(a.nV * a.k, a.W * a.k);
-    uint64_t* sel = keys + cap;
-    uint64_t* top = sel + 64;
+    uint64_t* surv = keys + cap;
+    uint64_t* top = surv + kRankMax;
 
     const int n = blockIdx.x, tid = threadIdx.x;
     const int s = n / a.P, p = n % a.P;
@@ -87,25 +131,22 @@ __global__ void __launch_bounds__(kSelThreads) merge_select_kernel(const SelectA
         // log-sum-exp of the node's scaled logits from the per-CTA partials
         float2 acc = make_float2(-INFINITY, 0.0f);
         for (int r = tid; r < a.nV; r += kSelThreads) acc = lse_merge(acc, a.part_ms[static_cast<size_t>(r) * a.N + n]);
-        const float gm = [&] {
-            float m = warp_max(acc.x);
-            if ((tid & 31) == 0) redm[tid >> 5] = m;
-            __syncthreads();
-            float t = -INFINITY;
-            for (int i = 0; i < kSelThreads / 32; i++) t = fmaxf(t, redm[i]);
-            return t;
-        }();
+        float m = warp_max(acc.x);
+        if ((tid & 31) == 0) redm[tid >> 5] = m;
+        __syncthreads();
+        float gm = -INFINITY;
+        for (int i = 0; i < kSelThreads / 32; i++) gm = fmaxf(gm, redm[i]);
         const float part = acc.x == -INFINITY ? 0.0f : acc.y * __expf(acc.x - gm);
         const float ssum = block_sum_float(part, redf);
         const float lse = gm == -INFINITY ? -INFINITY : gm + logf(ssum);
-        // top-k over every CTA's top-k
+        // top-k over every CTA's (sorted) top-k list
         const int nk = a.nV * a.k;
         for (int i = tid; i < nk; i += kSelThreads) {
             const int r = i / a.k, j = i % a.k;
             keys[i] = a.part_key[(static_cast<size_t>(r) * a.N + n) * a.k + j];
         }
         __syncthreads();
-        block_topk_sorted(keys, nk, a.k, top, sel, hist, scal);
+        topk_of_sorted_lists(keys, a.nV, a.k, a.k, top, surv, &thr, hist, scal);
         for (int j = tid; j < a.k; j += kSelThreads) {
             const uint64_t x = top[j];
             const float z = key_val(x);
@@ -132,6 +173,7 @@ __global__ void __launch_bounds__(kSelThreads) merge_select_kernel(const SelectA
     __threadfence();
     if (tid == 0) a.seq_ticket[s] = 0;
 
+    // candidates (p, j): parent p's list is sorted by log q~, hence by score
     const int ncand = prev_count * a.k;
     int valid = 0;
     for (int c = tid; c < ncand; c += kSelThreads) {
@@ -145,7 +187,7 @@ __global__ void __launch_bounds__(kSelThreads) merge_select_kernel(const SelectA
     }
     const int nvalid = block_sum_int(valid, redi);
     const int cnt = min(a.W, nvalid);
-    if (cnt > 0) block_topk_sorted(keys, ncand, cnt, top, sel, hist, scal);
+    if (cnt > 0) topk_of_sorted_lists(keys, prev_count, a.k, cnt, top, surv, &thr, hist, scal);
     const size_t tb = (static_cast<size_t>(s) * a.L + a.dep - 1) * a.W;
     for (int r = tid; r < a.W; r += kSelThreads) {
         if (r < cnt) {
@@ -173,31 +215,55 @@ __global__ void __launch_bounds__(kSelThreads) merge_select_kernel(const SelectA
     if (tid == 0) a.tree_count[s * a.L + a.dep - 1] = cnt;
 }
 
+// Number of keys > x in the descending list l[0..n) (binary search).
+__device__ __forceinline__ int count_greater(const uint64_t* l, int n, uint64_t x) {
+    int lo = 0, hi = n;
+    while (lo < hi) {
+        const int mid = (lo + hi) >> 1;
+        if (l[mid] > x)
+            lo = mid + 1;
+        else
+            hi = mid;
+    }
+    return lo;
+}
+
 __global__ void __launch_bounds__(kEmitThreads) prune_emit_kernel(const EmitArgs a) {
+    pdl_trigger();
+    pdl_wait();
     __shared__ uint64_t keys[1024];
     __shared__ int outidx[1024];
     __shared__ int par_out[1024];
-    __shared__ uint32_t hist[256];
-    __shared__ int scal[4];
+    __shared__ int cnts[1024];
     __shared__ int redi[32];
     __shared__ int wsum[32];
     const int s = blockIdx.x, tid = threadIdx.x;
     const int T = a.L * a.W;
     const size_t tb = static_cast<size_t>(s) * T;
+    for (int dd = tid; dd < a.L; dd += kEmitThreads) cnts[dd] = a.tree_count[s * a.L + dd];
+    __syncthreads();
     int valid = 0;
+    uint64_t my = 0ull;
     if (tid < T) {
         const int dep = tid / a.W + 1, r = tid % a.W;
-        const bool ok = r < a.tree_count[s * a.L + dep - 1];
-        keys[tid] = ok ? make_key(a.tree_score[tb + tid], static_cast<uint32_t>(tid)) : 0ull;
+        const bool ok = r < cnts[dep - 1];
+        my = ok ? make_key(a.tree_score[tb + tid], static_cast<uint32_t>(tid)) : 0ull;
+        keys[tid] = my;
         valid = ok;
     }
-    const int nvalid = block_sum_int(valid, redi);
+    const int nvalid = block_sum_int(valid, redi);  // synchronises: keys visible
     const int beff = min(a.B, nvalid);
-    uint64_t kth = ~0ull;
-    if (beff > 0) kth = block_kth_largest(keys, T, beff, hist, scal);
-    // compaction in ascending node id (exclusive scan of the selection flags)
+    // Rank of a node = number of nodes with a larger key.  Each depth's list
+    // is sorted (frontier rank order is score order, ties by id), so the rank
+    // is a sum of L binary searches (Algorithm 1 final step: TopB by s_beta).
+    int flag = 0;
+    if (tid < T && my != 0ull) {
+        int rank = 0;
+        for (int dd = 0; dd < a.L; dd++) rank += count_greater(keys + dd * a.W, cnts[dd], my);
+        flag = rank < beff;
+    }
+    // compaction in ascending node id (exclusive scan of the flags)
     const int lane = tid & 31, warp = tid >> 5;
-    const int flag = (tid < T && keys[tid] != 0ull && keys[tid] >= kth) ? 1 : 0;
     int incl = flag;
 #pragma unroll
     for (int o = 1; o < 32; o <<= 1) {
@@ -256,94 +322,149 @@ __device__ __forceinline__ void split_bf16(float x, __nv_bfloat16& hi, __nv_bflo
     lo = __float2bfloat16_rn(x - __bfloat162float(hi));
 }
 
-__global__ void prep_anchor_kernel(const float* anchor, int d, float* h, __nv_bfloat16* HL, int bhalf) {
-    const int s = blockIdx.x;
-    for (int j = threadIdx.x; j < d; j += blockDim.x) {
-        const float x = anchor[static_cast<size_t>(s) * d + j];
-        h[static_cast<size_t>(s) * d + j] = x;
-        if (HL) {
-            __nv_bfloat16 hi, lo;
-            split_bf16(x, hi, lo);
-            HL[static_cast<size_t>(s) * d + j] = hi;
-            HL[static_cast<size_t>(bhalf + s) * d + j] = lo;
-        }
+// 4 consecutive floats -> 4 hi and 4 lo bf16 (8-byte stores)
+__device__ __forceinline__ void split4(const float4 v, __nv_bfloat16* hi, __nv_bfloat16* lo) {
+    __align__(8) __nv_bfloat16 h[4], l[4];
+    split_bf16(v.x, h[0], l[0]);
+    split_bf16(v.y, h[1], l[1]);
+    split_bf16(v.z, h[2], l[2]);
+    split_bf16(v.w, h[3], l[3]);
+    *reinterpret_cast<uint2*>(hi) = *reinterpret_cast<const uint2*>(h);
+    *reinterpret_cast<uint2*>(lo) = *reinterpret_cast<const uint2*>(l);
+}
+
+__global__ void prep_anchor_kernel(const float* anchor, int nseq, int d, float* h, __nv_bfloat16* HL, int bhalf) {
+    pdl_trigger();
+    pdl_wait();
+    const int q4 = d / 4;
+    const int total = nseq * q4;
+    for (int u = blockIdx.x * blockDim.x + threadIdx.x; u < total; u += gridDim.x * blockDim.x) {
+        const int s = u / q4, j = (u % q4) * 4;
+        const float4 x = *reinterpret_cast<const float4*>(anchor + static_cast<size_t>(s) * d + j);
+        *reinterpret_cast<float4*>(h + static_cast<size_t>(s) * d + j) = x;
+        if (HL) split4(x, HL + static_cast<size_t>(s) * d + j, HL + static_cast<size_t>(bhalf + s) * d + j);
     }
 }
 
-__global__ void gather_x_kernel(int d, const int* prow, const int* tok, const float* h, const void* E, int wbf16,
-                                __nv_bfloat16* XL, int bhalf, float* X32) {
-    const int c = blockIdx.x;
-    const int pr = prow[c];
-    const int t = tok[c];
-    const size_t xo = static_cast<size_t>(c) * 2 * d;
-    const size_t xl = static_cast<size_t>(bhalf + c) * 2 * d;
-    for (int j = threadIdx.x; j < d; j += blockDim.x) {
-        const float x = pr >= 0 ? h[static_cast<size_t>(pr) * d + j] : 0.0f;
-        if (wbf16) {
-            __nv_bfloat16 hi, lo;
-            split_bf16(x, hi, lo);
-            XL[xo + j] = hi;
-            XL[xl + j] = lo;
-            const __nv_bfloat16 ev = pr >= 0 ? reinterpret_cast<const __nv_bfloat16*>(E)[static_cast<size_t>(t) * d + j]
-                                             : __float2bfloat16_rn(0.0f);
-            XL[xo + d + j] = ev;
-            XL[xl + d + j] = __float2bfloat16_rn(0.0f);
+// X[c] = [h[prow[c]] ; E[tok[c]]]: one thread per 4 columns.
+__global__ void gather_x_kernel(int Nc, int d, const int* prow, const int* tok, const float* h, const void* E,
+                                int wbf16, __nv_bfloat16* XL, int bhalf, float* X32) {
+    pdl_trigger();
+    pdl_wait();
+    const int q4 = (2 * d) / 4;
+    const int total = Nc * q4;
+    for (int u = blockIdx.x * blockDim.x + threadIdx.x; u < total; u += gridDim.x * blockDim.x) {
+        const int c = u / q4, j = (u % q4) * 4;
+        const int pr = prow[c];
+        const size_t xo = static_cast<size_t>(c) * 2 * d + j;
+        const size_t xl = static_cast<size_t>(bhalf + c) * 2 * d + j;
+        if (j < d) {
+            float4 x = make_float4(0.f, 0.f, 0.f, 0.f);
+            if (pr >= 0) x = *reinterpret_cast<const float4*>(h + static_cast<size_t>(pr) * d + j);
+            if (wbf16)
+                split4(x, XL + xo, XL + xl);
+            else
+                *reinterpret_cast<float4*>(X32 + xo) = x;
         } else {
-            X32[xo + j] = x;
-            X32[xo + d + j] = pr >= 0 ? reinterpret_cast<const float*>(E)[static_cast<size_t>(t) * d + j] : 0.0f;
+            const size_t eo = static_cast<size_t>(tok[c]) * d + (j - d);
+            if (wbf16) {
+                uint2 e = make_uint2(0u, 0u);
+                if (pr >= 0) e = *reinterpret_cast<const uint2*>(reinterpret_cast<const __nv_bfloat16*>(E) + eo);
+                *reinterpret_cast<uint2*>(XL + xo) = e;
+                *reinterpret_cast<uint2*>(XL + xl) = make_uint2(0u, 0u);
+            } else {
+                float4 e = make_float4(0.f, 0.f, 0.f, 0.f);
+                if (pr >= 0) e = *reinterpret_cast<const float4*>(reinterpret_cast<const float*>(E) + eo);
+                *reinterpret_cast<float4*>(X32 + xo) = e;
+            }
         }
     }
 }
 
 __global__ void silu_split_kernel(int Nc, int d, int S, const float* part, __nv_bfloat16* AL, int bhalf, float* A32) {
+    pdl_trigger();
+    pdl_wait();
     const size_t total = static_cast<size_t>(Nc) * d;
-    for (size_t q = blockIdx.x * static_cast<size_t>(blockDim.x) + threadIdx.x; q < total;
-         q += static_cast<size_t>(gridDim.x) * blockDim.x) {
-        float u = 0.0f;
-        for (int s = 0; s < S; s++) u += part[static_cast<size_t>(s) * total + q];
-        const float act = u / (1.0f + expf(-u));
-        if (AL) {
-            __nv_bfloat16 hi, lo;
-            split_bf16(act, hi, lo);
-            AL[q] = hi;
-            AL[static_cast<size_t>(bhalf) * d + q] = lo;
-        } else {
-            A32[q] = act;
+    const size_t t4 = total / 4;
+    for (size_t u = blockIdx.x * static_cast<size_t>(blockDim.x) + threadIdx.x; u < t4;
+         u += static_cast<size_t>(gridDim.x) * blockDim.x) {
+        const size_t q = u * 4;
+        float4 v = *reinterpret_cast<const float4*>(part + q);
+        for (int s = 1; s < S; s++) {
+            const float4 w = *reinterpret_cast<const float4*>(part + static_cast<size_t>(s) * total + q);
+            v.x += w.x;
+            v.y += w.y;
+            v.z += w.z;
+            v.w += w.w;
         }
+        v.x = v.x / (1.0f + expf(-v.x));
+        v.y = v.y / (1.0f + expf(-v.y));
+        v.z = v.z / (1.0f + expf(-v.z));
+        v.w = v.w / (1.0f + expf(-v.w));
+        if (AL)
+            split4(v, AL + q, AL + static_cast<size_t>(bhalf) * d + q);
+        else
+            *reinterpret_cast<float4*>(A32 + q) = v;
     }
 }
 
-__global__ void residual_norm_kernel(int d, int S, int Nc, const float* part, const int* prow, const float* h,
-                                     float eps, float* h_next, __nv_bfloat16* HL, int bhalf) {
+constexpr int kNormThreads = 1024;
+
+// One block per child: r = h[prow] + sum_s part[s], h_next = r / rms(r).
+__global__ void __launch_bounds__(kNormThreads) residual_norm_kernel(int d, int S, int Nc, const float* part,
+                                                                     const int* prow, const float* h, float eps,
+                                                                     float* h_next, __nv_bfloat16* HL, int bhalf) {
+    pdl_trigger();
+    pdl_wait();
     __shared__ float red[32];
     const int c = blockIdx.x;
     const int pr = prow[c];
     const size_t total = static_cast<size_t>(Nc) * d;
+    constexpr int kMaxPer = 4;  // d <= 16384 = 4 * 4 * 1024
+    float4 r[kMaxPer];
     float ss = 0.0f;
-    for (int i = threadIdx.x; i < d; i += blockDim.x) {
-        float y = 0.0f;
-        for (int s = 0; s < S; s++) y += part[static_cast<size_t>(s) * total + static_cast<size_t>(c) * d + i];
-        const float r = pr >= 0 ? h[static_cast<size_t>(pr) * d + i] + y : 0.0f;
-        h_next[static_cast<size_t>(c) * d + i] = r;
-        ss += r * r;
+#pragma unroll
+    for (int it = 0; it < kMaxPer; it++) {
+        const int j = (it * kNormThreads + threadIdx.x) * 4;
+        r[it] = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (j < d && pr >= 0) {
+            float4 v = *reinterpret_cast<const float4*>(h + static_cast<size_t>(pr) * d + j);
+            for (int s = 0; s < S; s++) {
+                const float4 w = *reinterpret_cast<const float4*>(part + static_cast<size_t>(s) * total +
+                                                                  static_cast<size_t>(c) * d + j);
+                v.x += w.x;
+                v.y += w.y;
+                v.z += w.z;
+                v.w += w.w;
+            }
+            r[it] = v;
+            ss += v.x * v.x + v.y * v.y + v.z * v.z + v.w * v.w;
+        }
     }
     const float tot = block_sum_float(ss, red);
     const float inv = 1.0f / sqrtf(tot / static_cast<float>(d) + eps);
-    for (int i = threadIdx.x; i < d; i += blockDim.x) {
-        const float x = h_next[static_cast<size_t>(c) * d + i] * inv;
-        h_next[static_cast<size_t>(c) * d + i] = x;
-        if (HL) {
-            __nv_bfloat16 hi, lo;
-            split_bf16(x, hi, lo);
-            HL[static_cast<size_t>(c) * d + i] = hi;
-            HL[static_cast<size_t>(bhalf + c) * d + i] = lo;
+#pragma unroll
+    for (int it = 0; it < kMaxPer; it++) {
+        const int j = (it * kNormThreads + threadIdx.x) * 4;
+        if (j < d) {
+            const float4 v = make_float4(r[it].x * inv, r[it].y * inv, r[it].z * inv, r[it].w * inv);
+            *reinterpret_cast<float4*>(h_next + static_cast<size_t>(c) * d + j) = v;
+            if (HL) split4(v, HL + static_cast<size_t>(c) * d + j, HL + static_cast<size_t>(bhalf + c) * d + j);
         }
     }
 }
 
 }  // namespace
 
-int merge_select_smem(int nV, int k, int W) { return (max(nV * k, W * k) + 128) * 8; }
+bool pdl_enabled() {
+    static const bool on = [] {
+        const char* e = getenv("DART_DISABLE_PDL");
+        return !(e && e[0] && e[0] != '0');
+    }();
+    return on;
+}
+
+int merge_select_smem(int nV, int k, int W) { return (max(nV * k, W * k) + kRankMax + 64) * 8; }
 
 cudaError_t select_set_smem_limits(int max_dyn) {
     return cudaFuncSetAttribute(merge_select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, max_dyn);
@@ -351,40 +472,40 @@ cudaError_t select_set_smem_limits(int max_dyn) {
 
 cudaError_t launch_merge_select(const SelectArgs& a, cudaStream_t st) {
     const int smem = merge_select_smem(a.nV, a.k, a.W);
-    merge_select_kernel<<<a.N, kSelThreads, smem, st>>>(a);
-    return cudaGetLastError();
+    return launch_pdl(merge_select_kernel, dim3(a.N), dim3(kSelThreads), smem, st, a);
 }
 
 cudaError_t launch_prune_emit(const EmitArgs& a, cudaStream_t st) {
-    prune_emit_kernel<<<a.nseq, kEmitThreads, 0, st>>>(a);
-    return cudaGetLastError();
+    return launch_pdl(prune_emit_kernel, dim3(a.nseq), dim3(kEmitThreads), 0, st, a);
+}
+
+static int grid_for(size_t units) {
+    size_t b = (units + 255) / 256;
+    return static_cast<int>(b < 1 ? 1 : (b > 2048 ? 2048 : b));
 }
 
 cudaError_t launch_prep_anchor(const float* anchor, int nseq, int d, float* h, __nv_bfloat16* HL, int bhalf,
                                cudaStream_t st) {
-    prep_anchor_kernel<<<nseq, 256, 0, st>>>(anchor, d, h, HL, bhalf);
-    return cudaGetLastError();
+    return launch_pdl(prep_anchor_kernel, dim3(grid_for(static_cast<size_t>(nseq) * d / 4)), dim3(256), 0, st, anchor,
+                      nseq, d, h, HL, bhalf);
 }
 
 cudaError_t launch_gather_x(int Nc, int d, const int* prow, const int* tok, const float* h, const void* E,
                             int wbf16, __nv_bfloat16* XL, int bhalf, float* X32, cudaStream_t st) {
-    gather_x_kernel<<<Nc, 256, 0, st>>>(d, prow, tok, h, E, wbf16, XL, bhalf, X32);
-    return cudaGetLastError();
+    return launch_pdl(gather_x_kernel, dim3(grid_for(static_cast<size_t>(Nc) * 2 * d / 4)), dim3(256), 0, st, Nc, d,
+                      prow, tok, h, E, wbf16, XL, bhalf, X32);
 }
 
 cudaError_t launch_silu_split(int Nc, int d, int S, const float* part, __nv_bfloat16* AL, int bhalf, float* A32,
                               cudaStream_t st) {
-    const size_t total = static_cast<size_t>(Nc) * d;
-    int blocks = static_cast<int>((total + 255) / 256);
-    if (blocks > 4096) blocks = 4096;
-    silu_split_kernel<<<blocks, 256, 0, st>>>(Nc, d, S, part, AL, bhalf, A32);
-    return cudaGetLastError();
+    return launch_pdl(silu_split_kernel, dim3(grid_for(static_cast<size_t>(Nc) * d / 4)), dim3(256), 0, st, Nc, d, S,
+                      part, AL, bhalf, A32);
 }
 
 cudaError_t launch_residual_norm(int Nc, int d, int S, const float* part, const int* prow, const float* h,
                                  float eps, float* h_next, __nv_bfloat16* HL, int bhalf, cudaStream_t st) {
-    residual_norm_kernel<<<Nc, 256, 0, st>>>(d, S, Nc, part, prow, h, eps, h_next, HL, bhalf);
-    return cudaGetLastError();
+    return launch_pdl(residual_norm_kernel, dim3(Nc), dim3(kNormThreads), 0, st, d, S, Nc, part, prow, h, eps, h_next,
+                      HL, bhalf);
 }
 
 }  // namespace dart

@@ -57,29 +57,45 @@ __device__ __forceinline__ void producer(const CUtensorMap* tmA, const CUtensorM
                                          volatile int* abort, int* status) {
     const uint64_t pol_a = l2_policy_evict_first();  // streamed once
     const uint64_t pol_b = l2_policy_evict_last();   // re-read by every tile
-    uint32_t stage = 0, phase = 0, fills = 0;
+    const int kbs = w.kb1 - w.kb0;
+    const uint32_t total = static_cast<uint32_t>(w.ntiles * kbs);
+    // The A operand (E or a head weight) never depends on an earlier kernel:
+    // its first `pre` stages are requested before waiting on the previous
+    // kernel; the B operand (node states) only after.
+    const uint32_t pre = total < static_cast<uint32_t>(stages) ? total : static_cast<uint32_t>(stages);
+    for (uint32_t f = 0; f < pre; f++) {
+        const int i = static_cast<int>(f) / kbs, kb = w.kb0 + static_cast<int>(f) % kbs;
+        const bool lo = kb < w.lo_kb_end;
+        mbar_arrive_expect_tx(&full[f], kATileBytes + NG * 128 * (lo ? 2 : 1));
+        tma_load_2d(ring + f * Layout<NG>::kStage, tmA, &full[f], kb * kBlockK, w.row0 + i * kTileM, pol_a);
+    }
+    pdl_wait();
+    for (uint32_t f = 0; f < pre; f++) {
+        const int kb = w.kb0 + static_cast<int>(f) % kbs;
+        uint8_t* sH = ring + f * Layout<NG>::kStage + kATileBytes;
+        tma_load_2d(sH, tmB, &full[f], kb * kBlockK, w.brow, pol_b);
+        if (kb < w.lo_kb_end) tma_load_2d(sH + NG * 128, tmB, &full[f], kb * kBlockK, bhalf + w.brow, pol_b);
+    }
+    uint32_t stage = pre % stages, phase = (pre / stages) & 1u, fills = pre;
     bool ok = true;
-    for (int i = 0; i < w.ntiles && ok; i++) {
-        const int row = w.row0 + i * kTileM;
-        for (int kb = w.kb0; kb < w.kb1; kb++) {
-            if (!mbar_wait(&empty[stage], phase ^ 1u, abort)) {
-                record_timeout(status, abort);
-                ok = false;
-                break;
-            }
-            const bool lo = kb < w.lo_kb_end;
-            uint8_t* sA = ring + stage * Layout<NG>::kStage;
-            uint8_t* sH = sA + kATileBytes;
-            uint8_t* sL = sH + NG * 128;
-            mbar_arrive_expect_tx(&full[stage], kATileBytes + NG * 128 * (lo ? 2 : 1));
-            tma_load_2d(sA, tmA, &full[stage], kb * kBlockK, row, pol_a);
-            tma_load_2d(sH, tmB, &full[stage], kb * kBlockK, w.brow, pol_b);
-            if (lo) tma_load_2d(sL, tmB, &full[stage], kb * kBlockK, bhalf + w.brow, pol_b);
-            fills++;
-            if (++stage == static_cast<uint32_t>(stages)) {
-                stage = 0;
-                phase ^= 1u;
-            }
+    for (uint32_t f = pre; f < total; f++) {
+        if (!mbar_wait(&empty[stage], phase ^ 1u, abort)) {
+            record_timeout(status, abort);
+            ok = false;
+            break;
+        }
+        const int i = static_cast<int>(f) / kbs, kb = w.kb0 + static_cast<int>(f) % kbs;
+        const bool lo = kb < w.lo_kb_end;
+        uint8_t* sA = ring + stage * Layout<NG>::kStage;
+        uint8_t* sH = sA + kATileBytes;
+        mbar_arrive_expect_tx(&full[stage], kATileBytes + NG * 128 * (lo ? 2 : 1));
+        tma_load_2d(sA, tmA, &full[stage], kb * kBlockK, w.row0 + i * kTileM, pol_a);
+        tma_load_2d(sH, tmB, &full[stage], kb * kBlockK, w.brow, pol_b);
+        if (lo) tma_load_2d(sH + NG * 128, tmB, &full[stage], kb * kBlockK, bhalf + w.brow, pol_b);
+        fills++;
+        if (++stage == static_cast<uint32_t>(stages)) {
+            stage = 0;
+            phase ^= 1u;
         }
     }
     if (!ok) {
@@ -214,13 +230,15 @@ __global__ void __launch_bounds__(kThreads, 1)
     lmhead_tc_kernel(const __grid_constant__ CUtensorMap tmE, const __grid_constant__ CUtensorMap tmH,
                      const LmheadArgs a) {
     extern __shared__ uint8_t smem_raw[];
+    pdl_trigger();
     const int stages = a.stages;
     Smem s = carve<NG>(smem_raw, stages);
     EpiSmem e;
     e.list = reinterpret_cast<uint64_t*>(s.tail);
     e.cand = e.list + NG * a.k;
     e.stats = reinterpret_cast<float2*>(e.cand + NG * kCandCap);
-    e.cnt = reinterpret_cast<int*>(e.stats + 4 * NG);
+    e.mref = reinterpret_cast<float*>(e.stats + 4 * NG);
+    e.cnt = reinterpret_cast<int*>(e.mref + 4 * NG);
 
     const int g = blockIdx.x % a.G;
     const int vr = blockIdx.x / a.G;
@@ -248,7 +266,11 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int etid = threadIdx.x - 64;
         const int ew = warp - 2;
         const int quarter = warp & 3;
+        pdl_wait();
         epi_init(e, NG, a.k, etid);
+        float ssum[NG / 16];
+#pragma unroll
+        for (int c = 0; c < NG / 16; c++) ssum[c] = 0.0f;
         for (int i = 0; i < w.ntiles; i++) {
             const int acc = i & 1;
             const uint32_t aph = (i >> 1) & 1;
@@ -267,28 +289,30 @@ __global__ void __launch_bounds__(kThreads, 1)
             float dl = 0.0f;
 #pragma unroll
             for (int c0 = 0; c0 < NG; c0 += 16) {
-                float vals[16];
-                tmem_ld16(tmem_base + acc * acc_stride<NG>() + c0 + (static_cast<uint32_t>(quarter * 32) << 16),
-                          vals);
+                float z[16];
+                tmem_ld16(tmem_base + acc * acc_stride<NG>() + c0 + (static_cast<uint32_t>(quarter * 32) << 16), z);
+                uint32_t nodemask = 0;
 #pragma unroll
                 for (int j = 0; j < 16; j++) {
-                    const int node = c0 + j;
-                    const int n = g * NG + node;
+                    const int n = g * NG + c0 + j;
                     if (n < a.N) {
+                        nodemask |= 1u << j;
                         const int seq = n / a.P;
                         if (seq != cur_seq) {
                             cur_seq = seq;
                             dl = valid ? __ldg(a.dlog + seq * a.dlog_seq_stride + a.dlog_row_off + v) : 0.0f;
                         }
-                        const float z = (vals[j] + dl) * a.invT;
-                        epi_value(e, NG, a.k, ew, lane, node, z, valid, static_cast<uint32_t>(v));
+                        z[j] = (z[j] + dl) * a.invT;
                     }
                 }
+                epi_chunk(e, NG, a.k, ew, lane, c0, z, nodemask, valid, static_cast<uint32_t>(v), ssum[c0 / 16]);
             }
             tc_fence_before();
             mbar_arrive(&s.tempty[acc]);
-            epi_merge(e, NG, a.k, etid);
+            epi_merge(e, NG, a.k, ew, lane);
         }
+#pragma unroll
+        for (int c0 = 0; c0 < NG; c0 += 16) epi_stash(e, NG, ew, lane, c0, ssum[c0 / 16]);
         epi_finalize(e, NG, a.k, etid, g * NG, a.N, vr, a.part_ms, a.part_key);
     }
     teardown(tmem_base, tmem_cols<NG>());
@@ -301,6 +325,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                    const GemmArgs a) {
     extern __shared__ uint8_t smem_raw[];
+    pdl_trigger();
     const int stages = a.stages;
     Smem s = carve<NG>(smem_raw, stages);
 
@@ -329,6 +354,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     } else {
         const int etid = threadIdx.x - 64;
         const int quarter = warp & 3;
+        pdl_wait();
         if (etid == 0) {
             const bool ok = mbar_wait(&s.tfull[0], 0, abort);
             if (!ok) record_timeout(a.status, abort);
@@ -357,20 +383,18 @@ __global__ void __launch_bounds__(kThreads, 1)
 
 template <int NG>
 int lmhead_fixed(int k, int stages) {
-    return (2 * stages + 5) * 8 + 16 + NG * k * 8 + NG * kCandCap * 8 + 4 * NG * 8 + NG * 4;
+    return (2 * stages + 5) * 8 + 16 + NG * k * 8 + NG * kCandCap * 8 + 4 * NG * 8 + 4 * NG * 4 + NG * 4;
 }
 
 template <int NG>
 cudaError_t launch_lmhead_ng(const CUtensorMap* tmE, const CUtensorMap* tmH, const LmheadArgs& a, int smem,
                              cudaStream_t st) {
-    lmhead_tc_kernel<NG><<<a.nV * a.G, kThreads, smem, st>>>(*tmE, *tmH, a);
-    return cudaGetLastError();
+    return launch_pdl(lmhead_tc_kernel<NG>, dim3(a.nV * a.G), dim3(kThreads), smem, st, *tmE, *tmH, a);
 }
 template <int NG>
 cudaError_t launch_gemm_ng(const CUtensorMap* tmA, const CUtensorMap* tmB, const GemmArgs& a, int smem,
                            cudaStream_t st) {
-    gemm_tc_kernel<NG><<<a.MT * a.G * a.S, kThreads, smem, st>>>(*tmA, *tmB, a);
-    return cudaGetLastError();
+    return launch_pdl(gemm_tc_kernel<NG>, dim3(a.MT * a.G * a.S), dim3(kThreads), smem, st, *tmA, *tmB, a);
 }
 
 }  // namespace

@@ -67,6 +67,7 @@ def lib():
             "dart_status_sync": (i, [vp, vp]),
             "dart_set_profiling": (i, [vp, i]),
             "dart_profile_read": (i, [vp, C.POINTER(f), C.POINTER(i)]),
+            "dart_profile_read_kinds": (i, [vp, vp, vp, i]),
             "dart_launches_per_round": (i, [vp]),
             "dart_destroy": (None, [vp]),
             "dart_status_string": (C.c_char_p, [i]),
@@ -202,6 +203,20 @@ def dart_profile_read(h):
     n = C.c_int()
     _check(lib().dart_profile_read(h, C.byref(ms), C.byref(n)), "dart_profile_read")
     return float(ms.value), int(n.value)
+
+
+KIND_NAMES = ("lmhead", "merge_select", "gather", "gemm_wi", "silu_split", "gemm_wo", "residual_norm",
+              "prep_anchor", "prune_emit")
+
+
+def dart_profile_read_kinds(h):
+    """{kind name: (total ms, launches)} since the last read."""
+    n = len(KIND_NAMES)
+    ms = (C.c_float * n)()
+    cnt = (C.c_int * n)()
+    _check(lib().dart_profile_read_kinds(h, C.cast(ms, C.c_void_p), C.cast(cnt, C.c_void_p), n),
+           "dart_profile_read_kinds")
+    return {KIND_NAMES[i]: (float(ms[i]), int(cnt[i])) for i in range(n)}
 
 
 def dart_launches_per_round(h):

@@ -46,6 +46,9 @@ SMALL = [
     C("bf16-Vk", 1, 8, 64, 4, 8, 8, 30, "bf16", 0.0, 23),
     C("bf16-beta0", 1, 1200, 128, 4, 6, 3, 11, "bf16", 0.0, 24, beta=0.0),
     C("bf16-kltW", 2, 1200, 128, 4, 9, 2, 25, "bf16", 0.0, 25, pos_offset=37),
+    C("bf16-manytiles", 1, 320000, 128, 3, 8, 16, 20, "bf16", 1.0, 26),
+    C("bf16-k64-many", 1, 200000, 64, 2, 64, 64, 80, "bf16", 0.0, 27),
+    C("f32-manytiles", 2, 150000, 64, 3, 16, 16, 30, "f32", 0.0, 28),
     TOY,
 ]
 
