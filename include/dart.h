@@ -176,6 +176,29 @@ int dart_profile_read_kinds(dart_handle *h, float *ms, int *launches, int nkinds
 /* Number of kernel launches one dart_build_tree enqueues for this handle. */
 int dart_launches_per_round(dart_handle *h);
 
+/* No-allocation variant of depth 1 (no counterpart in the paper: it exists
+ * for callers that cannot allocate device memory while they run, e.g. a
+ * serving engine that has reserved all free memory for its own pool, or a
+ * path where cudaMalloc's implicit device synchronisation is not allowed).
+ * It computes what dart_expand_depth(1) computes for every root -- the k best
+ * children, their log q~ and the log-sum-exp over the full vocabulary, and
+ * S_1 -- without a handle and without allocating:
+ *   E [V][d] bf16 (16-byte aligned), drafter_logits [nseq][L][V] (row 0 is
+ *   read), anchor_h [nseq][d] (16-byte aligned); outputs node_tok /
+ *   node_logq [nseq][k], node_lse [nseq], front_tok / front_score [nseq][W]
+ *   (rank order, unused ranks -1 / -inf), front_count [nseq].
+ * Its scratch is one static 16 MiB device array that every GPU loading this
+ * library keeps until the process exits.  Limits beyond dart_init_head's:
+ * nseq <= 64, d <= 8192; larger problems return DART_ERR_INVALID before any
+ * work is enqueued.  The first call on a device looks up the array's device
+ * address (cudaGetSymbolAddress) and sets kernel attributes, so make that
+ * first call before any stream capture.  Every call on a device shares the
+ * array: calls that overlap on the GPU (other streams, other threads) race;
+ * serialise them.  Device-side timeouts are not reported by this entry point. */
+int dart_expand_root_noalloc(const dart_config *cfg, const void *E, const float *drafter_logits,
+                             const float *anchor_h, int32_t *node_tok, float *node_logq, float *node_lse,
+                             int32_t *front_tok, float *front_score, int32_t *front_count, void *stream);
+
 void dart_destroy(dart_handle *h);
 const char *dart_status_string(int code);
 int dart_version(void);

@@ -69,6 +69,7 @@ def lib():
             "dart_profile_read": (i, [vp, C.POINTER(f), C.POINTER(i)]),
             "dart_profile_read_kinds": (i, [vp, vp, vp, i]),
             "dart_launches_per_round": (i, [vp]),
+            "dart_expand_root_noalloc": (i, [C.POINTER(DartConfig), vp, vp, vp, vp, vp, vp, vp, vp, vp, vp]),
             "dart_destroy": (None, [vp]),
             "dart_status_string": (C.c_char_p, [i]),
             "dart_version": (i, []),
@@ -221,6 +222,16 @@ def dart_profile_read_kinds(h):
 
 def dart_launches_per_round(h):
     return int(lib().dart_launches_per_round(h))
+
+
+def dart_expand_root_noalloc(cfg, E, drafter_logits, anchor_h, node_tok, node_logq, node_lse, front_tok,
+                             front_score, front_count, stream=None):
+    """Depth-1 expansion without device allocation (outputs are caller tensors)."""
+    c = make_config(cfg)
+    _check(lib().dart_expand_root_noalloc(C.byref(c), _ptr(E), _ptr(drafter_logits), _ptr(anchor_h),
+                                          _ptr(node_tok), _ptr(node_logq), _ptr(node_lse), _ptr(front_tok),
+                                          _ptr(front_score), _ptr(front_count), _stream(stream)),
+           "dart_expand_root_noalloc")
 
 
 def dart_destroy(h):

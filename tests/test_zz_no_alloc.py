@@ -1,0 +1,75 @@
+"""The allocation-free depth-1 entry point against the regular handle path.
+
+dart_expand_root_noalloc serves callers that cannot allocate device memory
+while they run (a serving engine whose memory pool owns every free byte, or a
+path where cudaMalloc's implicit synchronisation is not allowed): it keeps its
+scratch in a static device array instead.  This file is collected last on
+purpose, so a failure here cannot hide the result of any other test.
+"""
+import ctypes as C
+
+import numpy as np
+import pytest
+import torch
+
+from parity import to_device, tol_of
+from workloads import Config, make_inputs
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def dart():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2608_13524_gb300 import dart as d
+    d.lib()
+    return d
+
+
+def handle_depth1(dart, cfg, dx):
+    """What the existing entry points return for depth 1."""
+    h = dart.dart_init_head(cfg, dart.DART_BF16, dx["Wi"], dx["Wo"], dx["E"])
+    try:
+        dart.dart_expand_depth(h, 1, dx["Dlog"], dx["h0"])
+        tok, logq, lse = dart.dart_get_node_topk(h, cfg)
+        ftok, _, fsc, fcnt = dart.dart_get_frontier(h, 1, cfg)
+        assert dart.dart_status_sync(h) == 0
+        return [t.cpu().numpy() for t in (tok, logq, lse, ftok, fsc, fcnt)]
+    finally:
+        dart.dart_destroy(h)
+
+
+@pytest.mark.parametrize("nseq,V,d,W,k,T", [(3, 20000, 512, 8, 12, 0.7), (1, 151936, 4096, 16, 16, 1.0)])
+def test_noalloc_matches_handle_path_twice(dart, nseq, V, d, W, k, T):
+    cfg = Config("noalloc", nseq, V, d, 4, W, k, 20, "bf16", T, 9000 + nseq)
+    x = make_inputs(cfg)
+    dx = to_device(cfg, x)
+    ref = handle_depth1(dart, cfg, dx)
+    tol = tol_of(cfg)
+    for call in range(2):  # the second call reuses the array the first one left behind
+        out = [torch.full((nseq, k), -7, dtype=torch.int32, device="cuda"),
+               torch.full((nseq, k), 7.0, device="cuda"), torch.full((nseq,), 7.0, device="cuda"),
+               torch.full((nseq, W), -7, dtype=torch.int32, device="cuda"),
+               torch.full((nseq, W), 7.0, device="cuda"), torch.full((nseq,), -7, dtype=torch.int32, device="cuda")]
+        dart.dart_expand_root_noalloc(cfg, dx["E"], dx["Dlog"], dx["h0"], *out)
+        torch.cuda.synchronize()
+        got = [t.cpu().numpy() for t in out]
+        np.testing.assert_array_equal(got[0], ref[0], err_msg=f"node tokens, call {call}")
+        np.testing.assert_allclose(got[1], ref[1], atol=tol, rtol=0, err_msg=f"node log q, call {call}")
+        np.testing.assert_allclose(got[2], ref[2], atol=tol, rtol=0, err_msg=f"node lse, call {call}")
+        np.testing.assert_array_equal(got[3], ref[3], err_msg=f"frontier tokens, call {call}")
+        np.testing.assert_allclose(got[4], ref[4], atol=tol, rtol=0, err_msg=f"frontier scores, call {call}")
+        np.testing.assert_array_equal(got[5], ref[5], err_msg=f"frontier counts, call {call}")
+
+
+def test_noalloc_rejects_sizes_beyond_its_array(dart):
+    lib = dart.lib()
+    big = Config("toolarge", 65, 1000, 128, 2, 2, 2, 4, "bf16", 0.0, 1)
+    wide = Config("toowide", 1, 1000, 16384, 2, 2, 2, 4, "bf16", 0.0, 1)
+    buf = torch.zeros(1 << 20, dtype=torch.uint8, device="cuda")
+    p = C.c_void_p(buf.data_ptr())
+    for cfg in (big, wide):
+        c = dart.make_config(cfg)
+        rc = lib.dart_expand_root_noalloc(C.byref(c), p, p, p, p, p, p, p, p, p, None)
+        assert rc == dart.DART_ERR_INVALID
