@@ -113,8 +113,8 @@ int dart_init_head(dart_handle **out, const dart_config *cfg, int wdtype,
 
 /* Algorithm 1, one iteration: expands depth `depth` (1..L, in order; depth 1
  * restarts the round).  drafter_logits [nseq][L][V] float32 (row depth-1 is
- * read), anchor_h [nseq][d] float32 = r_0 (read at depth 1 only, may be NULL
- * afterwards).  Out of order -> DART_ERR_STATE. */
+ * read, 4-byte aligned), anchor_h [nseq][d] float32 = r_0 (16-byte aligned;
+ * read at depth 1 only, may be NULL afterwards).  Out of order -> DART_ERR_STATE. */
 int dart_expand_depth(dart_handle *h, int depth, const float *drafter_logits,
                       const float *anchor_h, void *stream);
 

@@ -197,7 +197,8 @@ int build_plans(dart_handle* h) {
             const int fixed = lmhead_tc_fixed_smem(p.NG, c.k, 16);
             const int half = h->smem_optin / 2 - 2048;
             const int st2 = tc_stages(half, tc_stage_bytes(p.NG), fixed);
-            if (st2 >= 4) {
+            const int smem2 = lmhead_tc_fixed_smem(p.NG, c.k, st2) + st2 * tc_stage_bytes(p.NG);
+            if (st2 >= 4 && lmhead_tc_ctas_per_sm(p.NG, smem2) >= 2) {
                 p.stages = st2;
                 p.nV = std::max(1, std::min(2 * h->num_sms / p.G, tiles));
             } else {
@@ -263,7 +264,7 @@ int alloc_workspace(dart_handle* h) {
     }
     DART_ALLOC(h->part, max_part_floats(h))
     DART_ALLOC(h->part_ms, max_nvn)
-    DART_ALLOC(h->part_key, max_nvn * c.k)
+    DART_ALLOC(h->part_key, max_nvn * c.k + kNPadMax)  // + one padding key per node (part_stride)
     DART_ALLOC(h->node_logq, static_cast<size_t>(kNPadMax) * c.k)
     DART_ALLOC(h->node_tok, static_cast<size_t>(kNPadMax) * c.k)
     DART_ALLOC(h->node_lse, kNPadMax)
@@ -515,7 +516,7 @@ int enqueue_round(dart_handle* h, const float* dlog, const float* anchor, const 
 
 int check_inputs(const dart_handle* h, const float* dlog, const float* anchor, bool need_anchor) {
     if (!dlog || !aligned4(dlog)) return DART_ERR_INVALID;
-    if (need_anchor && (!anchor || !aligned4(anchor))) return DART_ERR_INVALID;
+    if (need_anchor && (!anchor || !aligned16(anchor))) return DART_ERR_INVALID;  // read with 16-byte loads
     (void)h;
     return DART_OK;
 }
@@ -568,7 +569,8 @@ int dart_init_head(dart_handle** out, const dart_config* cfg, int wdtype, const 
     h->num_sms = sms;
     h->smem_optin = optin;
     h->next_depth = 1;
-    rc = build_plans(h);
+    if (wdtype == DART_BF16 && tc_set_smem_limits(optin) != cudaSuccess) rc = DART_ERR_CUDA;
+    if (rc == DART_OK) rc = build_plans(h);
     if (rc == DART_OK) rc = alloc_workspace(h);
     if (rc == DART_OK && wdtype == DART_BF16) rc = make_tensor_maps(h);
     if (rc == DART_OK && cudaStreamCreateWithFlags(&h->cap_stream, cudaStreamNonBlocking) != cudaSuccess)

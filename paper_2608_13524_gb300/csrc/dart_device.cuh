@@ -23,7 +23,6 @@ constexpr int kNPadMax = 256;       // max nodes per depth (nseq * W)
 constexpr int kTileM = 128;         // MMA M: vocabulary rows / output features per tile
 constexpr int kBlockK = 64;         // bf16 elements per 128-byte swizzled row
 constexpr int kCandCap = 128;       // per-node candidate slots per tile (one tile worth)
-constexpr int kEpiThreads = 128;    // 4 epilogue warps
 constexpr int kEpiBarrier = 1;      // named barrier id used by the epilogue warps
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
@@ -318,13 +317,15 @@ __device__ __forceinline__ float bfly16(const float (&v)[16], int lane) {
     return op(d, __shfl_xor_sync(kFull, d, 1));
 }
 
-__device__ __forceinline__ void epi_init(const EpiSmem& e, int NG, int k, int etid) {
-    for (int i = etid; i < NG * k; i += kEpiThreads) e.list[i] = 0ull;
-    for (int i = etid; i < NG; i += kEpiThreads) e.cnt[i] = 0;
-    for (int i = etid; i < 4 * NG; i += kEpiThreads) e.mref[i] = -INFINITY;
+// nthr = number of epilogue threads (4 warps per 16-node chunk of the group).
+__device__ __forceinline__ void epi_init(const EpiSmem& e, int NG, int k, int etid, int nthr) {
+    for (int i = etid; i < NG * k; i += nthr) e.list[i] = 0ull;
+    for (int i = etid; i < NG; i += nthr) e.cnt[i] = 0;
+    for (int i = etid; i < 4 * NG; i += nthr) e.mref[i] = -INFINITY;
 }
 
 // One 16-node chunk of this thread's row (all 32 lanes, same chunk).
+// ew: the warp's row quarter (0..3; per-quarter reference maxima and sums).
 // z[j]: scaled logit of node c0+j of the group; node j exists iff bit j of
 // nodemask is set; rowvalid: the row is < V.  ssum: the running sum of this
 // lane's node (c0 + lane/2).
@@ -474,16 +475,17 @@ __device__ __forceinline__ void warp_merge(uint64_t* L, const uint64_t* C, int c
 }
 
 // Merges every node's tile candidates into its list: one warp per node, no
-// block barrier between nodes.  Called by all epilogue threads.
-__device__ __forceinline__ void epi_merge(const EpiSmem& e, int NG, int k, int ew, int lane) {
-    named_bar_sync(kEpiBarrier, kEpiThreads);
-    for (int nd = ew; nd < NG; nd += 4) {
+// block barrier between nodes.  Called by all nthr epilogue threads; wi is
+// the epilogue warp index (0 .. nthr/32 - 1).
+__device__ __forceinline__ void epi_merge(const EpiSmem& e, int NG, int k, int wi, int lane, int nthr) {
+    named_bar_sync(kEpiBarrier, nthr);
+    for (int nd = wi; nd < NG; nd += nthr / 32) {
         const int c = e.cnt[nd];
         if (c == 0) continue;
         warp_merge(e.list + nd * k, e.cand + nd * kCandCap, c, k, lane);
         if (lane == 0) e.cnt[nd] = 0;
     }
-    named_bar_sync(kEpiBarrier, kEpiThreads);
+    named_bar_sync(kEpiBarrier, nthr);
 }
 
 // Records this warp's (reference, sum) of chunk cc's nodes.
@@ -494,22 +496,27 @@ __device__ __forceinline__ void epi_stash(const EpiSmem& e, int NG, int ew, int 
     }
 }
 
-// Writes this CTA's partial results for the nodes n0 .. n0+NG-1 (< N):
-// part_ms[vr][n] = (max, sum exp), part_key[vr][n][k] = top-k keys.
-__device__ __forceinline__ void epi_finalize(const EpiSmem& e, int NG, int k, int etid, int n0, int N, int vr,
-                                             float2* part_ms, uint64_t* part_key) {
-    named_bar_sync(kEpiBarrier, kEpiThreads);
-    for (int c = etid; c < NG; c += kEpiThreads) {
+// Keys per node in the partial buffer: nV*k rounded up to even, so every
+// node's block starts on a 16-byte boundary (it is read with 16-byte loads).
+__host__ __device__ __forceinline__ int part_stride(int nV, int k) { return (nV * k + 1) & ~1; }
+
+// Writes this CTA's partial results for the nodes n0 .. n0+NG-1 (< N), node
+// major so that each node's partials are contiguous:
+// part_ms[n][vr] = (max, sum exp), part_key[n * part_stride + vr*k + j] = top-k keys.
+__device__ __forceinline__ void epi_finalize(const EpiSmem& e, int NG, int k, int etid, int nthr, int n0, int N,
+                                             int vr, int nV, float2* part_ms, uint64_t* part_key) {
+    named_bar_sync(kEpiBarrier, nthr);
+    for (int c = etid; c < NG; c += nthr) {
         const int n = n0 + c;
         if (n >= N) continue;
         float2 a = e.stats[c];
         for (int w = 1; w < 4; w++) a = lse_merge(a, e.stats[w * NG + c]);
-        part_ms[static_cast<size_t>(vr) * N + n] = a;
+        part_ms[static_cast<size_t>(n) * nV + vr] = a;
     }
-    for (int i = etid; i < NG * k; i += kEpiThreads) {
+    for (int i = etid; i < NG * k; i += nthr) {
         const int c = i / k, j = i % k, n = n0 + c;
         if (n >= N) continue;
-        part_key[(static_cast<size_t>(vr) * N + n) * k + j] = e.list[i];
+        part_key[static_cast<size_t>(n) * part_stride(nV, k) + static_cast<size_t>(vr) * k + j] = e.list[i];
     }
 }
 

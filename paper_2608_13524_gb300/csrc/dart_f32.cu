@@ -10,6 +10,7 @@ namespace dart {
 namespace {
 
 constexpr int kEPad = kBlockK + 1;  // padded row of the staged E tile (no bank conflicts)
+constexpr int kEpiThreads = 128;    // 4 warps: thread r owns row r of a tile
 
 // LM-head scoring, fp32: one block of 128 threads (the 4 epilogue warps) per
 // vocabulary range and node group; thread r owns row r of each 128-row tile.
@@ -33,7 +34,7 @@ __global__ void __launch_bounds__(kEpiThreads) lmhead_f32_kernel(const LmheadArg
     const int t1 = static_cast<int>((static_cast<long long>(vr + 1) * a.tiles) / a.nV);
     const int tid = threadIdx.x, lane = tid & 31, ew = tid >> 5;
     const int KB = a.d / kBlockK;
-    epi_init(e, NG, a.k, tid);
+    epi_init(e, NG, a.k, tid, kEpiThreads);
     float ssum[NG / 16];
 #pragma unroll
     for (int c = 0; c < NG / 16; c++) ssum[c] = 0.0f;
@@ -94,11 +95,11 @@ __global__ void __launch_bounds__(kEpiThreads) lmhead_f32_kernel(const LmheadArg
             }
             epi_chunk(e, NG, a.k, ew, lane, c0, z, nodemask, valid, static_cast<uint32_t>(v), ssum[c0 / 16]);
         }
-        epi_merge(e, NG, a.k, ew, lane);
+        epi_merge(e, NG, a.k, ew, lane, kEpiThreads);
     }
 #pragma unroll
     for (int c0 = 0; c0 < NG; c0 += 16) epi_stash(e, NG, ew, lane, c0, ssum[c0 / 16]);
-    epi_finalize(e, NG, a.k, tid, g * NG, a.N, vr, a.part_ms, a.part_key);
+    epi_finalize(e, NG, a.k, tid, kEpiThreads, g * NG, a.N, vr, a.nV, a.part_ms, a.part_key);
 }
 
 // out[split][n][m] = sum_{k in split} A[m][k] * B[n][k]; 64 x 16 output tile

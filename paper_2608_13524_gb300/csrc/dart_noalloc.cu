@@ -142,7 +142,7 @@ extern "C" int dart_expand_root_noalloc(const dart_config* cfg, const void* E, c
     const int sb = tc_stage_bytes(NG);
     const int st2 = std::min(16, (ds.optin / 2 - 2048 - fixed) / sb);
     int stages, nV;
-    if (st2 >= 4) {
+    if (st2 >= 4 && lmhead_tc_ctas_per_sm(NG, lmhead_tc_fixed_smem(NG, c.k, st2) + st2 * sb) >= 2) {
         stages = st2;
         nV = std::max(1, std::min(2 * ds.sms, tiles));
     } else {
@@ -163,7 +163,7 @@ extern "C" int dart_expand_root_noalloc(const dart_config* cfg, const void* E, c
     float* h32 = reinterpret_cast<float*>(take(size_t(N) * c.d * 4));
     __nv_bfloat16* HL = reinterpret_cast<__nv_bfloat16*>(take(size_t(2) * kBhalfNoAlloc * c.d * 2));
     float2* part_ms = reinterpret_cast<float2*>(take(size_t(nV) * N * 8));
-    uint64_t* part_key = reinterpret_cast<uint64_t*>(take(size_t(nV) * N * c.k * 8));
+    uint64_t* part_key = reinterpret_cast<uint64_t*>(take(size_t(N) * part_stride(nV, c.k) * 8));
     int* tree_parent = reinterpret_cast<int*>(take(size_t(N) * c.W * 4));
     int* child_prow = reinterpret_cast<int*>(take(size_t(N) * Pn * 4));
     int* child_tok = reinterpret_cast<int*>(take(size_t(N) * Pn * 4));

@@ -21,7 +21,7 @@ namespace dart {
 
 namespace {
 
-constexpr int kSelThreads = 256;
+constexpr int kSelThreads = 512;
 constexpr int kEmitThreads = 1024;
 
 __device__ __forceinline__ int block_sum_int(int v, int* red) {
@@ -129,8 +129,14 @@ __global__ void __launch_bounds__(kSelThreads) merge_select_kernel(const SelectA
 
     if (p < prev_count) {
         // log-sum-exp of the node's scaled logits from the per-CTA partials
+        // this node's partials are contiguous: part_ms[n][nV], part_key[n][nV][k]
+        const int nk = a.nV * a.k;
+        const uint64_t* blk = a.part_key + static_cast<size_t>(n) * part_stride(a.nV, a.k);  // 16-byte aligned
+        const uint4* src = reinterpret_cast<const uint4*>(blk);
+        for (int i = tid; i < nk / 2; i += kSelThreads) reinterpret_cast<uint4*>(keys)[i] = __ldcg(src + i);
+        if ((nk & 1) && tid == 0) keys[nk - 1] = __ldcg(blk + nk - 1);
         float2 acc = make_float2(-INFINITY, 0.0f);
-        for (int r = tid; r < a.nV; r += kSelThreads) acc = lse_merge(acc, a.part_ms[static_cast<size_t>(r) * a.N + n]);
+        for (int r = tid; r < a.nV; r += kSelThreads) acc = lse_merge(acc, __ldcg(a.part_ms + static_cast<size_t>(n) * a.nV + r));
         float m = warp_max(acc.x);
         if ((tid & 31) == 0) redm[tid >> 5] = m;
         __syncthreads();
@@ -140,11 +146,6 @@ __global__ void __launch_bounds__(kSelThreads) merge_select_kernel(const SelectA
         const float ssum = block_sum_float(part, redf);
         const float lse = gm == -INFINITY ? -INFINITY : gm + logf(ssum);
         // top-k over every CTA's (sorted) top-k list
-        const int nk = a.nV * a.k;
-        for (int i = tid; i < nk; i += kSelThreads) {
-            const int r = i / a.k, j = i % a.k;
-            keys[i] = a.part_key[(static_cast<size_t>(r) * a.N + n) * a.k + j];
-        }
         __syncthreads();
         topk_of_sorted_lists(keys, a.nV, a.k, a.k, top, surv, &thr, hist, scal);
         for (int j = tid; j < a.k; j += kSelThreads) {

@@ -22,7 +22,15 @@ namespace dart {
 
 namespace {
 
-constexpr int kThreads = 192;
+// 2 warps (producer, MMA) + 4 epilogue warps per 16-node chunk of the group
+template <int NG>
+constexpr int epi_threads() {
+    return 128 * (NG / 16);
+}
+template <int NG>
+constexpr int threads() {
+    return 64 + epi_threads<NG>();
+}
 constexpr int kATileBytes = kTileM * kBlockK * 2;  // 16 KB
 
 struct Work {
@@ -179,6 +187,7 @@ __device__ __forceinline__ Smem carve(uint8_t* raw, int stages) {
 
 template <int NG>
 __device__ __forceinline__ uint32_t setup(const Smem& s, int stages, int ncols) {
+    constexpr int kEpi = epi_threads<NG>();
     const int warp = threadIdx.x >> 5;
     if (threadIdx.x == 0) {
         for (int i = 0; i < stages; i++) {
@@ -187,7 +196,7 @@ __device__ __forceinline__ uint32_t setup(const Smem& s, int stages, int ncols) 
         }
         for (int i = 0; i < 2; i++) {
             mbar_init(&s.tfull[i], 1);
-            mbar_init(&s.tempty[i], kEpiThreads);
+            mbar_init(&s.tempty[i], kEpi);
         }
         mbar_init(s.tdown, 1);
         s.misc[1] = 0;
@@ -226,7 +235,7 @@ constexpr int tmem_cols() {
 // ------------------------------------------------------------ LM-head kernel
 
 template <int NG>
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __launch_bounds__(threads<NG>(), 1)
     lmhead_tc_kernel(const __grid_constant__ CUtensorMap tmE, const __grid_constant__ CUtensorMap tmH,
                      const LmheadArgs a) {
     extern __shared__ uint8_t smem_raw[];
@@ -263,14 +272,19 @@ __global__ void __launch_bounds__(kThreads, 1)
             mma_issuer<NG>(w, s.ring, stages, s.full, s.empty, s.tfull, s.tempty, s.tdown, tmem_base,
                            acc_stride<NG>(), abort, a.status);
     } else {
+        // epilogue warp wi = warp - 2 reads TMEM lane quarter warp % 4 and
+        // owns the 16-node chunk wi / 4 of the group
+        constexpr int kEpi = epi_threads<NG>();
         const int etid = threadIdx.x - 64;
-        const int ew = warp - 2;
+        const int wi = warp - 2;
         const int quarter = warp & 3;
+        const int c0 = (wi >> 2) * 16;
         pdl_wait();
-        epi_init(e, NG, a.k, etid);
-        float ssum[NG / 16];
-#pragma unroll
-        for (int c = 0; c < NG / 16; c++) ssum[c] = 0.0f;
+        epi_init(e, NG, a.k, etid, kEpi);
+        float ssum = 0.0f;
+        uint32_t nodemask = 0;
+        for (int j = 0; j < 16; j++)
+            if (g * NG + c0 + j < a.N) nodemask |= 1u << j;
         for (int i = 0; i < w.ntiles; i++) {
             const int acc = i & 1;
             const uint32_t aph = (i >> 1) & 1;
@@ -279,41 +293,33 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (!ok) record_timeout(a.status, abort);
                 s.misc[2] = ok ? 1 : 0;
             }
-            named_bar_sync(kEpiBarrier, kEpiThreads);
+            named_bar_sync(kEpiBarrier, kEpi);
             if (s.misc[2] == 0) break;
             tc_fence_after();
-            const int row_local = quarter * 32 + lane;
-            const int v = w.row0 + i * kTileM + row_local;
+            const int v = w.row0 + i * kTileM + quarter * 32 + lane;
             const bool valid = v < a.V;
+            float z[16];
+            tmem_ld16(tmem_base + acc * acc_stride<NG>() + c0 + (static_cast<uint32_t>(quarter * 32) << 16), z);
+            tc_fence_before();
+            mbar_arrive(&s.tempty[acc]);
             int cur_seq = -1;
             float dl = 0.0f;
 #pragma unroll
-            for (int c0 = 0; c0 < NG; c0 += 16) {
-                float z[16];
-                tmem_ld16(tmem_base + acc * acc_stride<NG>() + c0 + (static_cast<uint32_t>(quarter * 32) << 16), z);
-                uint32_t nodemask = 0;
-#pragma unroll
-                for (int j = 0; j < 16; j++) {
-                    const int n = g * NG + c0 + j;
-                    if (n < a.N) {
-                        nodemask |= 1u << j;
-                        const int seq = n / a.P;
-                        if (seq != cur_seq) {
-                            cur_seq = seq;
-                            dl = valid ? __ldg(a.dlog + seq * a.dlog_seq_stride + a.dlog_row_off + v) : 0.0f;
-                        }
-                        z[j] = (z[j] + dl) * a.invT;
+            for (int j = 0; j < 16; j++) {
+                if ((nodemask >> j) & 1u) {
+                    const int seq = (g * NG + c0 + j) / a.P;
+                    if (seq != cur_seq) {
+                        cur_seq = seq;
+                        dl = valid ? __ldg(a.dlog + seq * a.dlog_seq_stride + a.dlog_row_off + v) : 0.0f;
                     }
+                    z[j] = (z[j] + dl) * a.invT;
                 }
-                epi_chunk(e, NG, a.k, ew, lane, c0, z, nodemask, valid, static_cast<uint32_t>(v), ssum[c0 / 16]);
             }
-            tc_fence_before();
-            mbar_arrive(&s.tempty[acc]);
-            epi_merge(e, NG, a.k, ew, lane);
+            epi_chunk(e, NG, a.k, quarter, lane, c0, z, nodemask, valid, static_cast<uint32_t>(v), ssum);
+            epi_merge(e, NG, a.k, wi, lane, kEpi);
         }
-#pragma unroll
-        for (int c0 = 0; c0 < NG; c0 += 16) epi_stash(e, NG, ew, lane, c0, ssum[c0 / 16]);
-        epi_finalize(e, NG, a.k, etid, g * NG, a.N, vr, a.part_ms, a.part_key);
+        epi_stash(e, NG, quarter, lane, c0, ssum);
+        epi_finalize(e, NG, a.k, etid, kEpi, g * NG, a.N, vr, a.nV, a.part_ms, a.part_key);
     }
     teardown(tmem_base, tmem_cols<NG>());
 }
@@ -321,7 +327,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 // --------------------------------------------------------------- GEMM kernel
 
 template <int NG>
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __launch_bounds__(threads<NG>(), 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                    const GemmArgs a) {
     extern __shared__ uint8_t smem_raw[];
@@ -360,21 +366,19 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (!ok) record_timeout(a.status, abort);
             s.misc[2] = ok ? 1 : 0;
         }
-        named_bar_sync(kEpiBarrier, kEpiThreads);
+        named_bar_sync(kEpiBarrier, epi_threads<NG>());
         if (s.misc[2] != 0) {
             tc_fence_after();
             const int m = w.row0 + quarter * 32 + lane;
             const bool valid = m < a.M;
             float* out = a.out + static_cast<size_t>(split) * a.N * a.M;
+            const int c0 = ((warp - 2) >> 2) * 16;
+            float vals[16];
+            tmem_ld16(tmem_base + c0 + (static_cast<uint32_t>(quarter * 32) << 16), vals);
 #pragma unroll
-            for (int c0 = 0; c0 < NG; c0 += 16) {
-                float vals[16];
-                tmem_ld16(tmem_base + c0 + (static_cast<uint32_t>(quarter * 32) << 16), vals);
-#pragma unroll
-                for (int j = 0; j < 16; j++) {
-                    const int n = g * NG + c0 + j;
-                    if (valid && n < a.N) out[static_cast<size_t>(n) * a.M + m] = vals[j];
-                }
+            for (int j = 0; j < 16; j++) {
+                const int n = g * NG + c0 + j;
+                if (valid && n < a.N) out[static_cast<size_t>(n) * a.M + m] = vals[j];
             }
         }
     }
@@ -389,12 +393,12 @@ int lmhead_fixed(int k, int stages) {
 template <int NG>
 cudaError_t launch_lmhead_ng(const CUtensorMap* tmE, const CUtensorMap* tmH, const LmheadArgs& a, int smem,
                              cudaStream_t st) {
-    return launch_pdl(lmhead_tc_kernel<NG>, dim3(a.nV * a.G), dim3(kThreads), smem, st, *tmE, *tmH, a);
+    return launch_pdl(lmhead_tc_kernel<NG>, dim3(a.nV * a.G), dim3(threads<NG>()), smem, st, *tmE, *tmH, a);
 }
 template <int NG>
 cudaError_t launch_gemm_ng(const CUtensorMap* tmA, const CUtensorMap* tmB, const GemmArgs& a, int smem,
                            cudaStream_t st) {
-    return launch_pdl(gemm_tc_kernel<NG>, dim3(a.MT * a.G * a.S), dim3(kThreads), smem, st, *tmA, *tmB, a);
+    return launch_pdl(gemm_tc_kernel<NG>, dim3(a.MT * a.G * a.S), dim3(threads<NG>()), smem, st, *tmA, *tmB, a);
 }
 
 }  // namespace
@@ -410,6 +414,18 @@ int lmhead_tc_fixed_smem(int NG, int k, int stages) {
 }
 
 int gemm_tc_fixed_smem(int stages) { return (2 * stages + 5) * 8 + 16 + 1024; }
+
+int lmhead_tc_ctas_per_sm(int NG, int smem) {
+    int n = 0;
+    cudaError_t e = cudaErrorInvalidValue;
+    switch (NG) {
+        case 16: e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, lmhead_tc_kernel<16>, threads<16>(), smem); break;
+        case 32: e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, lmhead_tc_kernel<32>, threads<32>(), smem); break;
+        case 64: e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, lmhead_tc_kernel<64>, threads<64>(), smem); break;
+        default: break;
+    }
+    return e == cudaSuccess ? n : 0;
+}
 
 cudaError_t tc_set_smem_limits(int max_dyn) {
     cudaError_t e = cudaSuccess;
