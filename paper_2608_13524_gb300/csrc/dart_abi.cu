@@ -217,12 +217,24 @@ int build_plans(dart_handle* h) {
             p.g1 = gemm_plan(h, 2 * c.d, p.Nc, c.d / kBlockK, tc);
             p.g2 = gemm_plan(h, c.d, p.Nc, c.d / kBlockK, tc);
             if (tc) {
+                // two CTAs per SM when both fit with >= 4 stages: twice the
+                // independent weight streams, k split twice as finely
                 const int sb = tc_stage_bytes(p.g1.NG);
-                p.g1.stages = std::min(tc_stages(h->smem_optin, sb, gemm_tc_fixed_smem(16)), 8);
+                const int st2 = std::min(tc_stages(h->smem_optin / 2 - 2048, sb, gemm_tc_fixed_smem(16)), 8);
+                const int smem2 = gemm_tc_fixed_smem(st2) + st2 * sb;
+                int cps = 1;
+                if (st2 >= 4 && gemm_tc_ctas_per_sm(p.g1.NG, smem2) >= 2) {
+                    cps = 2;
+                    p.g1.stages = st2;
+                } else {
+                    p.g1.stages = std::min(tc_stages(h->smem_optin, sb, gemm_tc_fixed_smem(16)), 8);
+                }
                 p.g2.stages = p.g1.stages;
                 if (p.g1.stages < 2) return DART_ERR_UNSUPPORTED;
                 p.g1_smem = gemm_tc_fixed_smem(p.g1.stages) + p.g1.stages * sb;
                 p.g2_smem = p.g1_smem;
+                p.g1.S = std::max(1, std::min(p.g1.KB, cps * h->num_sms / (p.g1.MT * p.g1.G)));
+                p.g2.S = std::max(1, std::min(p.g2.KB, cps * h->num_sms / (p.g2.MT * p.g2.G)));
             }
         }
     }

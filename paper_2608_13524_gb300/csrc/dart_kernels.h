@@ -74,7 +74,8 @@ cudaError_t launch_gemm_tc(const CUtensorMap* tmA, const CUtensorMap* tmB, const
 int tc_stage_bytes(int NG);
 int lmhead_tc_fixed_smem(int NG, int k, int stages);
 int gemm_tc_fixed_smem(int stages);
-int lmhead_tc_ctas_per_sm(int NG, int smem);  // resident CTAs per SM (occupancy API; needs limits set)
+int lmhead_tc_ctas_per_sm(int NG, int smem);
+int gemm_tc_ctas_per_sm(int NG, int smem);  // resident CTAs per SM (occupancy API; needs limits set)
 cudaError_t tc_set_smem_limits(int max_dyn);
 
 // fp32 CUDA-core kernels (dart_f32.cu)

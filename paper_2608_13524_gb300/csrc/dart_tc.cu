@@ -415,6 +415,18 @@ int lmhead_tc_fixed_smem(int NG, int k, int stages) {
 
 int gemm_tc_fixed_smem(int stages) { return (2 * stages + 5) * 8 + 16 + 1024; }
 
+int gemm_tc_ctas_per_sm(int NG, int smem) {
+    int n = 0;
+    cudaError_t e = cudaErrorInvalidValue;
+    switch (NG) {
+        case 16: e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, gemm_tc_kernel<16>, threads<16>(), smem); break;
+        case 32: e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, gemm_tc_kernel<32>, threads<32>(), smem); break;
+        case 64: e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, gemm_tc_kernel<64>, threads<64>(), smem); break;
+        default: break;
+    }
+    return e == cudaSuccess ? n : 0;
+}
+
 int lmhead_tc_ctas_per_sm(int NG, int smem) {
     int n = 0;
     cudaError_t e = cudaErrorInvalidValue;
