@@ -193,12 +193,16 @@ int build_plans(dart_handle* h) {
         if (tc) {
             // Two CTAs per SM when both fit with >= 4 pipeline stages each: two
             // independent TMA streams per SM, and one CTA's epilogue / start-up /
-            // tail overlaps the other's stream.
+            // tail overlaps the other's stream.  Measured on GB300 it pays for
+            // short rows (d = 2560: -4 % per round) but not for d = 4096, where
+            // the deeper single-CTA pipeline and half as many partial lists win.
             const int fixed = lmhead_tc_fixed_smem(p.NG, c.k, 16);
             const int half = h->smem_optin / 2 - 2048;
             const int st2 = tc_stages(half, tc_stage_bytes(p.NG), fixed);
             const int smem2 = lmhead_tc_fixed_smem(p.NG, c.k, st2) + st2 * tc_stage_bytes(p.NG);
-            if (st2 >= 4 && lmhead_tc_ctas_per_sm(p.NG, smem2) >= 2) {
+            const char* force = getenv("DART_LMHEAD_CTAS_PER_SM");  // tuning override: 1 or 2
+            const bool want2 = force ? atoi(force) == 2 : c.d <= 3072;
+            if (want2 && st2 >= 4 && lmhead_tc_ctas_per_sm(p.NG, smem2) >= 2) {
                 p.stages = st2;
                 p.nV = std::max(1, std::min(2 * h->num_sms / p.G, tiles));
             } else {

@@ -357,24 +357,20 @@ __device__ __forceinline__ void epi_chunk(const EpiSmem& e, int NG, int k, int e
 #pragma unroll
     for (int j = 0; j < 16; j++) p[j] = z[j] != -INFINITY ? __expf(z[j] - mr[j]) : 0.0f;
     ssum += bfly16<false>(p, lane);
-    uint64_t key[16];
-    bool pass[16];
-    bool anyp = false;
+    uint32_t passmask = 0;  // bit j: this row's key beats node j's current k-th key
 #pragma unroll
-    for (int j = 0; j < 16; j++) {
-        key[j] = ok[j] ? make_key(z[j], row) : 0ull;
-        pass[j] = key[j] > e.list[(c0 + j) * k + k - 1];
-        anyp |= pass[j];
-    }
-    if (__any_sync(kFull, anyp)) {
+    for (int j = 0; j < 16; j++)
+        if (ok[j] && make_key(z[j], row) > e.list[(c0 + j) * k + k - 1]) passmask |= 1u << j;
+    if (__any_sync(kFull, passmask != 0u)) {
 #pragma unroll
         for (int j = 0; j < 16; j++) {
-            const unsigned bal = __ballot_sync(kFull, pass[j]);
+            const bool pass = (passmask >> j) & 1u;
+            const unsigned bal = __ballot_sync(kFull, pass);
             if (bal) {
                 int base = 0;
                 if (lane == 0) base = atomicAdd(&e.cnt[c0 + j], __popc(bal));
                 base = __shfl_sync(kFull, base, 0);
-                if (pass[j]) e.cand[(c0 + j) * kCandCap + base + __popc(bal & ((1u << lane) - 1u))] = key[j];
+                if (pass) e.cand[(c0 + j) * kCandCap + base + __popc(bal & ((1u << lane) - 1u))] = make_key(z[j], row);
             }
         }
     }

@@ -15,6 +15,10 @@
 // and single-thread MMA issuer, warps 2-5 = epilogue (TMEM lane quarters
 // warp%4).  Every wait is bounded: on timeout the CTA records kDevTimeout in
 // the status word, drains its own copies/MMAs (bounded), frees TMEM and exits.
+#include <algorithm>
+#include <cstdio>
+#include <cstdlib>
+
 #include "dart_device.cuh"
 #include "dart_kernels.h"
 
@@ -415,34 +419,51 @@ int lmhead_tc_fixed_smem(int NG, int k, int stages) {
 
 int gemm_tc_fixed_smem(int stages) { return (2 * stages + 5) * 8 + 16 + 1024; }
 
+// Resident CTAs per SM for a kernel with `smem` bytes of dynamic shared
+// memory, from the device limits (shared memory with the per-block
+// reservation, register file at 8-register granularity, threads).
+static int ctas_per_sm(const void* fn, int nthreads, int smem) {
+    int dev = 0, sm_smem = 0, reserved = 0, sm_regs = 0, sm_threads = 0;
+    cudaFuncAttributes fa;
+    if (cudaGetDevice(&dev) != cudaSuccess || cudaFuncGetAttributes(&fa, fn) != cudaSuccess ||
+        cudaDeviceGetAttribute(&sm_smem, cudaDevAttrMaxSharedMemoryPerMultiprocessor, dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&reserved, cudaDevAttrReservedSharedMemoryPerBlock, dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&sm_regs, cudaDevAttrMaxRegistersPerMultiprocessor, dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&sm_threads, cudaDevAttrMaxThreadsPerMultiProcessor, dev) != cudaSuccess)
+        return 1;
+    const int per_smem = smem + static_cast<int>(fa.sharedSizeBytes) + reserved;
+    const int per_regs = ((fa.numRegs + 7) / 8) * 8 * nthreads;
+    int n = per_smem > 0 ? sm_smem / per_smem : 1;
+    if (per_regs > 0) n = std::min(n, sm_regs / per_regs);
+    n = std::min(n, sm_threads / nthreads);
+    if (getenv("DART_DEBUG_PLAN"))
+        fprintf(stderr, "dart: smem %d (+%zu static, +%d reserved) of %d, regs %d x %d of %d -> %d CTAs/SM\n", smem,
+                fa.sharedSizeBytes, reserved, sm_smem, fa.numRegs, nthreads, sm_regs, n);
+    return std::max(n, 1);
+}
+
 int gemm_tc_ctas_per_sm(int NG, int smem) {
-    int n = 0;
-    cudaError_t e = cudaErrorInvalidValue;
     switch (NG) {
-        case 16: e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, gemm_tc_kernel<16>, threads<16>(), smem); break;
-        case 32: e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, gemm_tc_kernel<32>, threads<32>(), smem); break;
-        case 64: e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, gemm_tc_kernel<64>, threads<64>(), smem); break;
-        default: break;
+        case 16: return ctas_per_sm(reinterpret_cast<const void*>(gemm_tc_kernel<16>), threads<16>(), smem);
+        case 32: return ctas_per_sm(reinterpret_cast<const void*>(gemm_tc_kernel<32>), threads<32>(), smem);
+        default: return ctas_per_sm(reinterpret_cast<const void*>(gemm_tc_kernel<64>), threads<64>(), smem);
     }
-    return e == cudaSuccess ? n : 0;
 }
 
 int lmhead_tc_ctas_per_sm(int NG, int smem) {
-    int n = 0;
-    cudaError_t e = cudaErrorInvalidValue;
     switch (NG) {
-        case 16: e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, lmhead_tc_kernel<16>, threads<16>(), smem); break;
-        case 32: e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, lmhead_tc_kernel<32>, threads<32>(), smem); break;
-        case 64: e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, lmhead_tc_kernel<64>, threads<64>(), smem); break;
-        default: break;
+        case 16: return ctas_per_sm(reinterpret_cast<const void*>(lmhead_tc_kernel<16>), threads<16>(), smem);
+        case 32: return ctas_per_sm(reinterpret_cast<const void*>(lmhead_tc_kernel<32>), threads<32>(), smem);
+        default: return ctas_per_sm(reinterpret_cast<const void*>(lmhead_tc_kernel<64>), threads<64>(), smem);
     }
-    return e == cudaSuccess ? n : 0;
 }
 
 cudaError_t tc_set_smem_limits(int max_dyn) {
     cudaError_t e = cudaSuccess;
 #define DART_SET(fn)                                                                                   \
-    if (e == cudaSuccess) e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, max_dyn);
+    if (e == cudaSuccess) e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, max_dyn); \
+    if (e == cudaSuccess)                                                                              \
+        e = cudaFuncSetAttribute(fn, cudaFuncAttributePreferredSharedMemoryCarveout, cudaSharedmemCarveoutMaxShared);
     DART_SET(lmhead_tc_kernel<16>)
     DART_SET(lmhead_tc_kernel<32>)
     DART_SET(lmhead_tc_kernel<64>)
