@@ -60,6 +60,24 @@ def dist_env():
     return rank, world, local
 
 
+def allreduce_max(x, world, device=None):
+    """Max of a float over all ranks (the timing rule: the job is as slow as
+    its slowest rank).  No-op for a single process."""
+    if world <= 1:
+        return float(x)
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([float(x)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def whole_job_rate(units_per_step_per_rank, world, seconds_per_step):
+    """Units of all ranks per second (weak scaling: every rank does the same
+    amount of independent work)."""
+    return units_per_step_per_rank * world / seconds_per_step
+
+
 def measured_peak():
     p = os.path.join(ROOT, "MEASURED_PEAKS.json")
     try:
@@ -215,7 +233,7 @@ def main():
     from paper_2608_13524_gb300 import dart
     from workloads import make_inputs
 
-    x = make_inputs(cfg)
+    x = make_inputs(cfg, rank=rank)  # each replica builds its own sequences
     tb = lambda a: torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).to(dev).view(torch.bfloat16)
     tf = lambda a: torch.from_numpy(np.ascontiguousarray(a)).to(dev)
     conv = tb if cfg.wdtype == "bf16" else tf
@@ -259,12 +277,8 @@ def main():
         eng.build_tree(D, h0, stream)
     ev1.record(stream)
     barrier()
-    ms = ev0.elapsed_time(ev1) / args.steps
+    ms = allreduce_max(ev0.elapsed_time(ev1) / args.steps, world, dev)
     clk = clocks.stop()
-    if world > 1:
-        t = torch.tensor([ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
     rc = dart.dart_status_sync(h, stream)
     if rc != 0:
         raise RuntimeError(f"device status {rc} after timed region")
@@ -292,7 +306,7 @@ def main():
                      "us_per_launch": v[0] * 1e3 / max(1, v[1])} for k, v in kinds.items() if v[1]}
 
     exp_round = cfg.expansions_per_round()
-    value = exp_round * world / (ms / 1e3)
+    value = whole_job_rate(exp_round, world, ms / 1e3)
     bytes_launch = cfg.lmhead_bytes_per_depth()
     lm_bytes_round = cfg.L * cfg.V * cfg.d * cfg.bpe
     peak, peak_kind = measured_peak()
@@ -313,14 +327,10 @@ def main():
         for _ in range(args.steps):
             dart.dart_build_tree_host(h, Dh, hh, hout, stream)
         barrier()
-        e2e_s = (time.perf_counter() - t0) / args.steps
-        if world > 1:
-            t = torch.tensor([e2e_s], device=dev)
-            dist.all_reduce(t, op=dist.ReduceOp.MAX)
-            e2e_s = float(t.item())
+        e2e_s = allreduce_max((time.perf_counter() - t0) / args.steps, world, dev)
         h2d = Dh.numel() * 4 + hh.numel() * 4
         d2h = sum(v.numel() * v.element_size() for v in ht.values())
-        e2e = {"value": exp_round * world / e2e_s, "unit": UNIT, "h2d_bytes_per_step": h2d,
+        e2e = {"value": whole_job_rate(exp_round, world, e2e_s), "unit": UNIT, "h2d_bytes_per_step": h2d,
                "d2h_bytes_per_step": d2h, "ms_per_step": e2e_s * 1e3}
 
     cpu = None

@@ -170,12 +170,15 @@ def make_weights(cfg: Config, zero_E: bool = False):
     return Wi, Wo, E
 
 
-def make_sequences(cfg: Config):
-    """Per-sequence drafter logits Dlog [nseq, L, V] and anchors h0 [nseq, d]."""
+def make_sequences(cfg: Config, rank: int = 0):
+    """Per-sequence drafter logits Dlog [nseq, L, V] and anchors h0 [nseq, d].
+
+    `rank` selects a disjoint block of sequences (seed cfg.seed*1000 +
+    rank*nseq + s), so replicas on different GPUs build different trees."""
     Dlog = np.empty((cfg.nseq, cfg.L, cfg.V), dtype=np.float32)
     h0 = np.empty((cfg.nseq, cfg.d), dtype=np.float32)
     for s in range(cfg.nseq):
-        g = np.random.Generator(np.random.PCG64(cfg.seed * 1000 + s))
+        g = np.random.Generator(np.random.PCG64(cfg.seed * 1000 + rank * cfg.nseq + s))
         h0[s] = g.standard_normal(cfg.d, dtype=np.float32)
         noise = g.standard_normal((cfg.L, cfg.V), dtype=np.float32)
         Dlog[s] = noise * np.float32(3.0)
@@ -186,7 +189,7 @@ def make_sequences(cfg: Config):
     return Dlog, h0
 
 
-def make_inputs(cfg: Config, zero_E: bool = False):
+def make_inputs(cfg: Config, zero_E: bool = False, rank: int = 0):
     Wi, Wo, E = make_weights(cfg, zero_E=zero_E)
-    Dlog, h0 = make_sequences(cfg)
+    Dlog, h0 = make_sequences(cfg, rank=rank)
     return dict(Wi=Wi, Wo=Wo, E=E, Dlog=Dlog, h0=h0)
