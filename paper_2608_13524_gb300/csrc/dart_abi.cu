@@ -99,6 +99,7 @@ struct dart_handle {
     int *tree_tok, *tree_parent, *tree_count;
     float* tree_score;
     int *child_prow, *child_tok, *seq_ticket, *status;
+    uint64_t* gthr;  // [L][kNPadMax] cross-CTA top-k bounds of every depth, zeroed per round
     std::vector<void*> allocs;
     CUtensorMap tmE, tmWi, tmWo, tmH[3], tmX[3], tmA[3];
     // host-buffer staging
@@ -292,6 +293,7 @@ int alloc_workspace(dart_handle* h) {
     DART_ALLOC(h->child_tok, kNPadMax)
     DART_ALLOC(h->seq_ticket, c.nseq)
     DART_ALLOC(h->status, 1)
+    DART_ALLOC(h->gthr, static_cast<size_t>(c.L) * kNPadMax)
 #undef DART_ALLOC
     if (rc != DART_OK) return rc;
     // zeroed once: stale rows of the operand buffers are always finite
@@ -377,7 +379,8 @@ int enqueue_depth(dart_handle* h, int dep, const float* dlog, const float* ancho
     cudaError_t e = cudaSuccess;
     if (dep == 1) {
         const int pi = prof_begin(h, kPrep, st);
-        e = launch_prep_anchor(anchor, c.nseq, c.d, h->hbuf[0], tc ? h->HL : nullptr, kNPadMax, st);
+        e = launch_prep_anchor(anchor, c.nseq, c.d, h->hbuf[0], tc ? h->HL : nullptr, kNPadMax, h->gthr,
+                               c.L * kNPadMax, st);
         prof_end(h, pi, st);
         if (e != cudaSuccess) return DART_ERR_CUDA;
         h->cur = 0;
@@ -405,6 +408,7 @@ int enqueue_depth(dart_handle* h, int dep, const float* dlog, const float* ancho
     la.status = h->status;
     la.h32 = h->hbuf[h->cur];
     la.E32 = static_cast<const float*>(h->E);
+    la.gthr = h->gthr + static_cast<size_t>(dep - 1) * kNPadMax;
     int pi = prof_begin(h, kLmhead, st);
     e = tc ? launch_lmhead_tc(&h->tmE, &h->tmH[ng_index(p.NG)], la, p.smem, st) : launch_lmhead_f32(la, st);
     prof_end(h, pi, st);

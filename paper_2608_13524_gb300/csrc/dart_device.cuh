@@ -281,6 +281,7 @@ constexpr float kRefSlack = 30.0f;  // exp(30) ~ 1e13: sums stay far from fp32 o
 struct EpiSmem {
     uint64_t* list;   // [NG][k]   sorted desc, 0 = empty
     uint64_t* cand;   // [NG][kCandCap]
+    uint64_t* gcache; // [NG]  last seen cross-CTA bound (see epi_merge)
     int* cnt;         // [NG]
     float* mref;      // [4][NG]  per-warp reference max
     float2* stats;    // [4][NG]  (reference, sum exp) per epilogue warp at the end
@@ -320,7 +321,10 @@ __device__ __forceinline__ float bfly16(const float (&v)[16], int lane) {
 // nthr = number of epilogue threads (4 warps per 16-node chunk of the group).
 __device__ __forceinline__ void epi_init(const EpiSmem& e, int NG, int k, int etid, int nthr) {
     for (int i = etid; i < NG * k; i += nthr) e.list[i] = 0ull;
-    for (int i = etid; i < NG; i += nthr) e.cnt[i] = 0;
+    for (int i = etid; i < NG; i += nthr) {
+        e.cnt[i] = 0;
+        e.gcache[i] = 0ull;
+    }
     for (int i = etid; i < 4 * NG; i += nthr) e.mref[i] = -INFINITY;
 }
 
@@ -357,10 +361,12 @@ __device__ __forceinline__ void epi_chunk(const EpiSmem& e, int NG, int k, int e
 #pragma unroll
     for (int j = 0; j < 16; j++) p[j] = z[j] != -INFINITY ? __expf(z[j] - mr[j]) : 0.0f;
     ssum += bfly16<false>(p, lane);
-    uint32_t passmask = 0;  // bit j: this row's key beats node j's current k-th key
+    uint32_t passmask = 0;  // bit j: this row's key beats node j's current threshold
 #pragma unroll
-    for (int j = 0; j < 16; j++)
-        if (ok[j] && make_key(z[j], row) > e.list[(c0 + j) * k + k - 1]) passmask |= 1u << j;
+    for (int j = 0; j < 16; j++) {
+        const uint64_t l = e.list[(c0 + j) * k + k - 1], g = e.gcache[c0 + j];
+        if (ok[j] && make_key(z[j], row) > (l > g ? l : g)) passmask |= 1u << j;
+    }
     if (__any_sync(kFull, passmask != 0u)) {
 #pragma unroll
         for (int j = 0; j < 16; j++) {
@@ -473,15 +479,31 @@ __device__ __forceinline__ void warp_merge(uint64_t* L, const uint64_t* C, int c
 // Merges every node's tile candidates into its list: one warp per node, no
 // block barrier between nodes.  Called by all nthr epilogue threads; wi is
 // the epilogue warp index (0 .. nthr/32 - 1).
-__device__ __forceinline__ void epi_merge(const EpiSmem& e, int NG, int k, int wi, int lane, int nthr) {
+//
+// Cross-CTA filter: gthr[n] (global, zeroed before the launch) holds the
+// largest k-th key any CTA has published for node n.  A CTA holding k keys
+// >= b proves that no key <= b can be among the node's k best children of
+// the whole vocabulary, so candidates must beat max(own k-th key, gthr[n]);
+// keys are distinct, so the test is exact.  Each merge publishes the CTA's
+// k-th key (atomicMax) and fetches gthr[n] for the next tile's filter.
+__device__ __forceinline__ void epi_merge(const EpiSmem& e, int NG, int k, int wi, int lane, int nthr, int etid,
+                                          uint64_t* gthr, int n0, int N) {
     named_bar_sync(kEpiBarrier, nthr);
+    uint64_t g = 0ull;
+    if (gthr && etid < NG && n0 + etid < N) g = __ldcg(reinterpret_cast<const unsigned long long*>(gthr) + n0 + etid);
     for (int nd = wi; nd < NG; nd += nthr / 32) {
         const int c = e.cnt[nd];
         if (c == 0) continue;
         warp_merge(e.list + nd * k, e.cand + nd * kCandCap, c, k, lane);
-        if (lane == 0) e.cnt[nd] = 0;
+        if (lane == 0) {
+            e.cnt[nd] = 0;
+            const uint64_t kth = e.list[nd * k + k - 1];
+            if (gthr && kth != 0ull && n0 + nd < N)
+                atomicMax(reinterpret_cast<unsigned long long*>(gthr) + n0 + nd, static_cast<unsigned long long>(kth));
+        }
     }
     named_bar_sync(kEpiBarrier, nthr);
+    if (etid < NG) e.gcache[etid] = g;  // read by the next tile's filter, after its first barrier
 }
 
 // Records this warp's (reference, sum) of chunk cc's nodes.

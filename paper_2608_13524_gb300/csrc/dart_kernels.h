@@ -49,6 +49,7 @@ struct LmheadArgs {
     int* status;
     const float* h32;     // fp32 states [N][d] (fp32 kernel)
     const float* E32;     // fp32 table [V][d]   (fp32 kernel)
+    uint64_t* gthr;       // [N] cross-CTA top-k bounds, zero before the launch (may be null)
 };
 
 // Skinny split-K GEMM for the correction head: out[split][n][m] =
@@ -121,7 +122,7 @@ cudaError_t launch_prune_emit(const EmitArgs& a, cudaStream_t st);
 
 // depth-1 preparation: states <- anchors, and their hi/lo bf16 split
 cudaError_t launch_prep_anchor(const float* anchor, int nseq, int d, float* h, __nv_bfloat16* HL, int bhalf,
-                               cudaStream_t st);
+                               uint64_t* gthr_all, int n_gthr, cudaStream_t st);
 // X[c] = [h[prow[c]] ; E[tok[c]]] (hi/lo bf16 or fp32)
 cudaError_t launch_gather_x(int Nc, int d, const int* prow, const int* tok, const float* h, const void* E,
                             int wbf16, __nv_bfloat16* XL, int bhalf, float* X32, cudaStream_t st);

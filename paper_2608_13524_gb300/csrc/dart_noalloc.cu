@@ -169,6 +169,7 @@ extern "C" int dart_expand_root_noalloc(const dart_config* cfg, const void* E, c
     int* child_tok = reinterpret_cast<int*>(take(size_t(N) * Pn * 4));
     int* seq_ticket = reinterpret_cast<int*>(take(size_t(N) * 4));
     int* status = reinterpret_cast<int*>(take(4));
+    uint64_t* gthr = reinterpret_cast<uint64_t*>(take(size_t(N) * 8));
     if (off > kScratchBytes) return DART_ERR_INVALID;
 
     CUtensorMap tmE, tmH;
@@ -180,7 +181,7 @@ extern "C" int dart_expand_root_noalloc(const dart_config* cfg, const void* E, c
     if (cudaMemsetAsync(seq_ticket, 0, size_t(N) * 4, st) != cudaSuccess ||
         cudaMemsetAsync(status, 0, 4, st) != cudaSuccess)
         return DART_ERR_CUDA;
-    if (launch_prep_anchor(anchor_h, N, c.d, h32, HL, kBhalfNoAlloc, st) != cudaSuccess) return DART_ERR_CUDA;
+    if (launch_prep_anchor(anchor_h, N, c.d, h32, HL, kBhalfNoAlloc, gthr, N, st) != cudaSuccess) return DART_ERR_CUDA;
 
     LmheadArgs la;
     std::memset(&la, 0, sizeof la);
@@ -202,6 +203,7 @@ extern "C" int dart_expand_root_noalloc(const dart_config* cfg, const void* E, c
     la.part_ms = part_ms;
     la.part_key = part_key;
     la.status = status;
+    la.gthr = gthr;
     if (launch_lmhead_tc(&tmE, &tmH, la, smem, st) != cudaSuccess) return DART_ERR_CUDA;
 
     SelectArgs sa;

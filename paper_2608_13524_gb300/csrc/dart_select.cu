@@ -334,9 +334,11 @@ __device__ __forceinline__ void split4(const float4 v, __nv_bfloat16* hi, __nv_b
     *reinterpret_cast<uint2*>(lo) = *reinterpret_cast<const uint2*>(l);
 }
 
-__global__ void prep_anchor_kernel(const float* anchor, int nseq, int d, float* h, __nv_bfloat16* HL, int bhalf) {
+__global__ void prep_anchor_kernel(const float* anchor, int nseq, int d, float* h, __nv_bfloat16* HL, int bhalf,
+                                   uint64_t* gthr_all, int n_gthr) {
     pdl_trigger();
     pdl_wait();
+    for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < n_gthr; i += gridDim.x * blockDim.x) gthr_all[i] = 0ull;
     const int q4 = d / 4;
     const int total = nseq * q4;
     for (int u = blockIdx.x * blockDim.x + threadIdx.x; u < total; u += gridDim.x * blockDim.x) {
@@ -486,9 +488,9 @@ static int grid_for(size_t units) {
 }
 
 cudaError_t launch_prep_anchor(const float* anchor, int nseq, int d, float* h, __nv_bfloat16* HL, int bhalf,
-                               cudaStream_t st) {
+                               uint64_t* gthr_all, int n_gthr, cudaStream_t st) {
     return launch_pdl(prep_anchor_kernel, dim3(grid_for(static_cast<size_t>(nseq) * d / 4)), dim3(256), 0, st, anchor,
-                      nseq, d, h, HL, bhalf);
+                      nseq, d, h, HL, bhalf, gthr_all, n_gthr);
 }
 
 cudaError_t launch_gather_x(int Nc, int d, const int* prow, const int* tok, const float* h, const void* E,

@@ -249,7 +249,8 @@ __global__ void __launch_bounds__(threads<NG>(), 1)
     EpiSmem e;
     e.list = reinterpret_cast<uint64_t*>(s.tail);
     e.cand = e.list + NG * a.k;
-    e.stats = reinterpret_cast<float2*>(e.cand + NG * kCandCap);
+    e.gcache = e.cand + NG * kCandCap;
+    e.stats = reinterpret_cast<float2*>(e.gcache + NG);
     e.mref = reinterpret_cast<float*>(e.stats + 4 * NG);
     e.cnt = reinterpret_cast<int*>(e.mref + 4 * NG);
 
@@ -320,7 +321,7 @@ __global__ void __launch_bounds__(threads<NG>(), 1)
                 }
             }
             epi_chunk(e, NG, a.k, quarter, lane, c0, z, nodemask, valid, static_cast<uint32_t>(v), ssum);
-            epi_merge(e, NG, a.k, wi, lane, kEpi);
+            epi_merge(e, NG, a.k, wi, lane, kEpi, etid, a.gthr, g * NG, a.N);
         }
         epi_stash(e, NG, quarter, lane, c0, ssum);
         epi_finalize(e, NG, a.k, etid, kEpi, g * NG, a.N, vr, a.nV, a.part_ms, a.part_key);
@@ -391,7 +392,7 @@ __global__ void __launch_bounds__(threads<NG>(), 1)
 
 template <int NG>
 int lmhead_fixed(int k, int stages) {
-    return (2 * stages + 5) * 8 + 16 + NG * k * 8 + NG * kCandCap * 8 + 4 * NG * 8 + 4 * NG * 4 + NG * 4;
+    return (2 * stages + 5) * 8 + 16 + NG * k * 8 + NG * kCandCap * 8 + NG * 8 + 4 * NG * 8 + 4 * NG * 4 + NG * 4;
 }
 
 template <int NG>
