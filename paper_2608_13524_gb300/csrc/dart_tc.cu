@@ -3,8 +3,10 @@
 // One warp-specialised mainloop serves two contractions with bf16 operands
 // in shared memory and fp32 accumulators in tensor memory:
 //   * LM-head scoring: A = E tile [128 vocabulary rows x 64], B = node states
-//     [NG nodes x 64] as hi + lo bf16 halves (both MMAs accumulate into the
-//     same TMEM tile, so states keep ~16 mantissa bits).  A persistent CTA
+//     [NG nodes x 64] as hi + lo bf16 halves stored as 2*NG consecutive rows,
+//     so ONE MMA with N = 2*NG computes both products (TMEM columns [0, NG)
+//     = A.hi, [NG, 2NG) = A.lo; the epilogue adds them: states keep ~16
+//     mantissa bits at half the MMA instruction count).  A persistent CTA
 //     walks a contiguous range of vocabulary tiles; two TMEM accumulators let
 //     the epilogue of tile i overlap the MMAs of tile i+1.  The epilogue adds
 //     the drafter row, scales by 1/T and reduces on chip to a running
@@ -122,7 +124,8 @@ __device__ __forceinline__ void mma_issuer(const Work& w, uint8_t* ring, int sta
                                            uint64_t* empty, uint64_t* tfull, uint64_t* tempty, uint64_t* tdown,
                                            uint32_t tmem_base, int acc_stride, volatile int* abort,
                                            int* status) {
-    constexpr uint32_t idesc = idesc_bf16_f32(kTileM, NG);
+    constexpr uint32_t idesc2 = idesc_bf16_f32(kTileM, 2 * NG);  // hi and lo rows together
+    constexpr uint32_t idesc1 = idesc_bf16_f32(kTileM, NG);      // hi rows only (no lo half)
     uint32_t stage = 0, phase = 0;
     bool ok = true;
     for (int i = 0; i < w.ntiles && ok; i++) {
@@ -142,16 +145,13 @@ __device__ __forceinline__ void mma_issuer(const Work& w, uint8_t* ring, int sta
                 break;
             }
             tc_fence_after();
-            const bool lo = kb < w.lo_kb_end;
+            const uint32_t idesc = kb < w.lo_kb_end ? idesc2 : idesc1;
             const uint32_t a = smem_u32(ring + stage * Layout<NG>::kStage);
             const uint32_t hb = a + kATileBytes;
-            const uint32_t lb = hb + NG * 128;
 #pragma unroll
-            for (int kk = 0; kk < kBlockK / 16; kk++) {
-                const uint64_t ad = sdesc_sw128(a + kk * 32);
-                tc_mma_bf16(d_tmem, ad, sdesc_sw128(hb + kk * 32), idesc, (kb > w.kb0 || kk > 0) ? 1u : 0u);
-                if (lo) tc_mma_bf16(d_tmem, ad, sdesc_sw128(lb + kk * 32), idesc, 1u);
-            }
+            for (int kk = 0; kk < kBlockK / 16; kk++)
+                tc_mma_bf16(d_tmem, sdesc_sw128(a + kk * 32), sdesc_sw128(hb + kk * 32), idesc,
+                            (kb > w.kb0 || kk > 0) ? 1u : 0u);
             tc_commit(&empty[stage]);  // frees the smem stage once these MMAs are done
             if (++stage == static_cast<uint32_t>(stages)) {
                 stage = 0;
@@ -227,9 +227,10 @@ __device__ __forceinline__ void teardown(uint32_t tmem_base, int ncols) {
     }
 }
 
+// One accumulator = 2*NG fp32 columns (hi products, then lo products).
 template <int NG>
 constexpr int acc_stride() {
-    return NG < 32 ? 32 : NG;
+    return 2 * NG < 32 ? 32 : 2 * NG;
 }
 template <int NG>
 constexpr int tmem_cols() {
@@ -303,10 +304,13 @@ __global__ void __launch_bounds__(threads<NG>(), 1)
             tc_fence_after();
             const int v = w.row0 + i * kTileM + quarter * 32 + lane;
             const bool valid = v < a.V;
-            float z[16];
-            tmem_ld16(tmem_base + acc * acc_stride<NG>() + c0 + (static_cast<uint32_t>(quarter * 32) << 16), z);
+            float z[16], zl[16];
+            const uint32_t tcol = tmem_base + acc * acc_stride<NG>() + c0 + (static_cast<uint32_t>(quarter * 32) << 16);
+            tmem_ld16_pair(tcol, tcol + NG, z, zl);
             tc_fence_before();
             mbar_arrive(&s.tempty[acc]);
+#pragma unroll
+            for (int j = 0; j < 16; j++) z[j] += zl[j];
             int cur_seq = -1;
             float dl = 0.0f;
 #pragma unroll
@@ -378,8 +382,14 @@ __global__ void __launch_bounds__(threads<NG>(), 1)
             const bool valid = m < a.M;
             float* out = a.out + static_cast<size_t>(split) * a.N * a.M;
             const int c0 = ((warp - 2) >> 2) * 16;
-            float vals[16];
-            tmem_ld16(tmem_base + c0 + (static_cast<uint32_t>(quarter * 32) << 16), vals);
+            float vals[16], lov[16];
+            const uint32_t tcol = tmem_base + c0 + (static_cast<uint32_t>(quarter * 32) << 16);
+            tmem_ld16_pair(tcol, tcol + NG, vals, lov);
+            // lo columns were written only if this split saw a k-block with a lo half
+            if (w.kb0 < w.lo_kb_end) {
+#pragma unroll
+                for (int j = 0; j < 16; j++) vals[j] += lov[j];
+            }
 #pragma unroll
             for (int j = 0; j < 16; j++) {
                 const int n = g * NG + c0 + j;
