@@ -428,6 +428,7 @@ int enqueue_depth(dart_handle* h, int dep, const float* dlog, const float* ancho
     sa.beta = c.beta;
     sa.part_ms = h->part_ms;
     sa.part_key = h->part_key;
+    sa.gthr = la.gthr;
     sa.node_logq = h->node_logq;
     sa.node_tok = h->node_tok;
     sa.node_lse = h->node_lse;

@@ -91,6 +91,7 @@ struct SelectArgs {
     float beta;
     const float2* part_ms;
     const uint64_t* part_key;
+    const uint64_t* gthr;  // [N] largest published k-th key per node (may be null)
     float* node_logq;      // [N][k]
     int* node_tok;         // [N][k]
     float* node_lse;       // [N]

@@ -220,6 +220,7 @@ extern "C" int dart_expand_root_noalloc(const dart_config* cfg, const void* E, c
     sa.beta = c.beta;
     sa.part_ms = part_ms;
     sa.part_key = part_key;
+    sa.gthr = gthr;
     sa.node_logq = node_logq;
     sa.node_tok = node_tok;
     sa.node_lse = node_lse;

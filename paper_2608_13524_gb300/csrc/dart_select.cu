@@ -52,14 +52,15 @@ constexpr int kRankMax = 1024;  // candidate count up to which an O(n^2 / thread
 
 // Writes the kk largest nonzero keys, in descending order, to out[0..kk).
 // `keys` holds nlists lists of `len` keys, each sorted in descending order
-// with zeros (empty slots) last; at least kk keys are nonzero.  A key can
-// only be among the kk largest if it is >= the kk-th largest list head, and
-// only the kk lists whose heads reach that threshold can hold such keys, so
-// at most kk*len keys survive the filter; the survivors are ranked by
-// counting.  A block-wide radix select handles any larger survivor set.
+// with zeros (empty slots) last; at least kk keys are nonzero.  Only keys
+// >= a threshold T can be among the kk largest, where T is the larger of
+// `bound` (0, or a key known to have kk keys >= it, such as the largest
+// k-th key any LM-head CTA published for the node) and the kk-th largest
+// list head (some kk lists reach it); the survivors are ranked by counting.
+// A block-wide radix select handles a survivor set larger than kRankMax.
 // `surv` has kRankMax slots.  Every thread of the block must call this.
 __device__ __forceinline__ void topk_of_sorted_lists(const uint64_t* keys, int nlists, int len, int kk,
-                                                     uint64_t* out, uint64_t* surv, uint64_t* thr,
+                                                     uint64_t bound, uint64_t* out, uint64_t* surv, uint64_t* thr,
                                                      uint32_t* hist, int* scal) {
     const int tid = threadIdx.x, nt = blockDim.x;
     const int n = nlists * len;
@@ -68,17 +69,22 @@ __device__ __forceinline__ void topk_of_sorted_lists(const uint64_t* keys, int n
         scal[2] = 0;
     }
     __syncthreads();
-    if (n > kRankMax && nlists > kk) {
+    if (nlists >= kk && nlists > 1) {
         for (int r = tid; r < nlists; r += nt) {
             const uint64_t h = keys[r * len];
             if (h == 0ull) continue;
             int rank = 0;
-            for (int q = 0; q < nlists; q++) rank += keys[q * len] > h;
+            int q = 0;
+            for (; q + 8 <= nlists; q += 8) {
+#pragma unroll
+                for (int u = 0; u < 8; u++) rank += keys[(q + u) * len] > h;
+            }
+            for (; q < nlists; q++) rank += keys[q * len] > h;
             if (rank == kk - 1) *thr = h;
         }
         __syncthreads();
     }
-    const uint64_t T = *thr;
+    const uint64_t T = *thr > bound ? *thr : bound;
     for (int i = tid; i < n; i += nt) {
         const uint64_t x = keys[i];
         if (x != 0ull && x >= T) {
@@ -102,7 +108,12 @@ __device__ __forceinline__ void topk_of_sorted_lists(const uint64_t* keys, int n
     for (int i = tid; i < mm; i += nt) {
         const uint64_t x = surv[i];
         int r = 0;
-        for (int j = 0; j < mm; j++) r += surv[j] > x;
+        int j = 0;
+        for (; j + 8 <= mm; j += 8) {
+#pragma unroll
+            for (int u = 0; u < 8; u++) r += surv[j + u] > x;
+        }
+        for (; j < mm; j++) r += surv[j] > x;
         if (r < kk) out[r] = x;
     }
     __syncthreads();
@@ -111,7 +122,8 @@ __device__ __forceinline__ void topk_of_sorted_lists(const uint64_t* keys, int n
 __global__ void __launch_bounds__(kSelThreads) merge_select_kernel(const SelectArgs a) {
     pdl_trigger();
     pdl_wait();
-    extern __shared__ uint64_t keys[];  // max(nV*k, W*k) keys, kRankMax survivors, 64 outputs
+    // dynamic: max(nV*k, W*k) keys, kRankMax survivors, 64 outputs, W*k candidate tokens
+    extern __shared__ uint64_t keys[];
     __shared__ uint32_t hist[256];
     __shared__ int scal[4];
     __shared__ uint64_t thr;
@@ -122,21 +134,51 @@ __global__ void __launch_bounds__(kSelThreads) merge_select_kernel(const SelectA
     const int cap = max(a.nV * a.k, a.W * a.k);
     uint64_t* surv = keys + cap;
     uint64_t* top = surv + kRankMax;
+    int* ctok = reinterpret_cast<int*>(top + 64);
 
     const int n = blockIdx.x, tid = threadIdx.x;
     const int s = n / a.P, p = n % a.P;
-    const int prev_count = a.dep == 1 ? 1 : a.tree_count[s * a.L + a.dep - 2];
+    // this node's partials are contiguous: part_ms[n][nV], part_key[n][nV][k];
+    // they are loaded before the frontier size is known (rows past it hold
+    // stale but harmless data)
+    const int nk = a.nV * a.k;
+    const uint64_t* blk = a.part_key + static_cast<size_t>(n) * part_stride(a.nV, a.k);  // 16-byte aligned
+    const uint4* src = reinterpret_cast<const uint4*>(blk);
+    const int prev_count = a.dep == 1 ? 1 : __ldcg(a.tree_count + s * a.L + a.dep - 2);
+    const uint64_t bound = a.gthr ? __ldcg(reinterpret_cast<const unsigned long long*>(a.gthr) + n) : 0ull;
+    float2 acc = make_float2(-INFINITY, 0.0f);
+    {
+        // every load of this thread is issued before the first use: one
+        // L2 round trip instead of one per loop iteration
+        constexpr int kBatch = 8;
+        float2 ms[2];
+#pragma unroll
+        for (int u = 0; u < 2; u++) {
+            const int r = tid + u * kSelThreads;
+            ms[u] = r < a.nV ? __ldcg(a.part_ms + static_cast<size_t>(n) * a.nV + r) : make_float2(-INFINITY, 0.0f);
+        }
+        for (int r = tid + 2 * kSelThreads; r < a.nV; r += kSelThreads)
+            acc = lse_merge(acc, __ldcg(a.part_ms + static_cast<size_t>(n) * a.nV + r));
+        for (int i0 = 0; i0 < nk / 2; i0 += kBatch * kSelThreads) {
+            uint4 v[kBatch];
+#pragma unroll
+            for (int u = 0; u < kBatch; u++) {
+                const int i = i0 + u * kSelThreads + tid;
+                if (i < nk / 2) v[u] = __ldcg(src + i);
+            }
+#pragma unroll
+            for (int u = 0; u < kBatch; u++) {
+                const int i = i0 + u * kSelThreads + tid;
+                if (i < nk / 2) reinterpret_cast<uint4*>(keys)[i] = v[u];
+            }
+        }
+        if ((nk & 1) && tid == 0) keys[nk - 1] = __ldcg(blk + nk - 1);
+        acc = lse_merge(acc, ms[0]);
+        acc = lse_merge(acc, ms[1]);
+    }
 
     if (p < prev_count) {
         // log-sum-exp of the node's scaled logits from the per-CTA partials
-        // this node's partials are contiguous: part_ms[n][nV], part_key[n][nV][k]
-        const int nk = a.nV * a.k;
-        const uint64_t* blk = a.part_key + static_cast<size_t>(n) * part_stride(a.nV, a.k);  // 16-byte aligned
-        const uint4* src = reinterpret_cast<const uint4*>(blk);
-        for (int i = tid; i < nk / 2; i += kSelThreads) reinterpret_cast<uint4*>(keys)[i] = __ldcg(src + i);
-        if ((nk & 1) && tid == 0) keys[nk - 1] = __ldcg(blk + nk - 1);
-        float2 acc = make_float2(-INFINITY, 0.0f);
-        for (int r = tid; r < a.nV; r += kSelThreads) acc = lse_merge(acc, __ldcg(a.part_ms + static_cast<size_t>(n) * a.nV + r));
         float m = warp_max(acc.x);
         if ((tid & 31) == 0) redm[tid >> 5] = m;
         __syncthreads();
@@ -146,8 +188,7 @@ __global__ void __launch_bounds__(kSelThreads) merge_select_kernel(const SelectA
         const float ssum = block_sum_float(part, redf);
         const float lse = gm == -INFINITY ? -INFINITY : gm + logf(ssum);
         // top-k over every CTA's (sorted) top-k list
-        __syncthreads();
-        topk_of_sorted_lists(keys, a.nV, a.k, a.k, top, surv, &thr, hist, scal);
+        topk_of_sorted_lists(keys, a.nV, a.k, a.k, bound, top, surv, &thr, hist, scal);
         for (int j = tid; j < a.k; j += kSelThreads) {
             const uint64_t x = top[j];
             const float z = key_val(x);
@@ -179,8 +220,10 @@ __global__ void __launch_bounds__(kSelThreads) merge_select_kernel(const SelectA
     int valid = 0;
     for (int c = tid; c < ncand; c += kSelThreads) {
         const int pp = c / a.k, j = c % a.k;
+        const size_t src_i = static_cast<size_t>(s * a.P + pp) * a.k + j;
         const float ps = a.dep == 1 ? 0.0f : a.tree_score[(static_cast<size_t>(s) * a.L + a.dep - 2) * a.W + pp];
-        const float lq = __ldcg(a.node_logq + static_cast<size_t>(s * a.P + pp) * a.k + j);
+        const float lq = __ldcg(a.node_logq + src_i);
+        ctok[c] = __ldcg(a.node_tok + src_i);
         const float sc = (ps + lq) + a.beta;  // Eq. 5, one more depth
         const bool ok = sc > -INFINITY;
         keys[c] = ok ? make_key(sc, static_cast<uint32_t>(c)) : 0ull;
@@ -188,14 +231,14 @@ __global__ void __launch_bounds__(kSelThreads) merge_select_kernel(const SelectA
     }
     const int nvalid = block_sum_int(valid, redi);
     const int cnt = min(a.W, nvalid);
-    if (cnt > 0) topk_of_sorted_lists(keys, prev_count, a.k, cnt, top, surv, &thr, hist, scal);
+    if (cnt > 0) topk_of_sorted_lists(keys, prev_count, a.k, cnt, 0ull, top, surv, &thr, hist, scal);
     const size_t tb = (static_cast<size_t>(s) * a.L + a.dep - 1) * a.W;
     for (int r = tid; r < a.W; r += kSelThreads) {
         if (r < cnt) {
             const uint64_t x = top[r];
             const int c = static_cast<int>(key_idx(x));
-            const int pp = c / a.k, j = c % a.k;
-            const int tok = __ldcg(a.node_tok + static_cast<size_t>(s * a.P + pp) * a.k + j);
+            const int pp = c / a.k;
+            const int tok = ctok[c];
             a.tree_tok[tb + r] = tok;
             a.tree_parent[tb + r] = a.dep == 1 ? -1 : pp;
             a.tree_score[tb + r] = key_val(x);
@@ -467,7 +510,7 @@ bool pdl_enabled() {
     return on;
 }
 
-int merge_select_smem(int nV, int k, int W) { return (max(nV * k, W * k) + kRankMax + 64) * 8; }
+int merge_select_smem(int nV, int k, int W) { return (max(nV * k, W * k) + kRankMax + 64) * 8 + W * k * 4; }
 
 cudaError_t select_set_smem_limits(int max_dyn) {
     return cudaFuncSetAttribute(merge_select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, max_dyn);
