@@ -9,6 +9,7 @@
 #include <algorithm>
 #include <cmath>
 #include <cstdint>
+#include <cstdio>
 #include <cstdlib>
 #include <cstring>
 #include <new>
@@ -238,8 +239,31 @@ int build_plans(dart_handle* h) {
                 if (p.g1.stages < 2) return DART_ERR_UNSUPPORTED;
                 p.g1_smem = gemm_tc_fixed_smem(p.g1.stages) + p.g1.stages * sb;
                 p.g2_smem = p.g1_smem;
-                p.g1.S = std::max(1, std::min(p.g1.KB, cps * h->num_sms / (p.g1.MT * p.g1.G)));
-                p.g2.S = std::max(1, std::min(p.g2.KB, cps * h->num_sms / (p.g2.MT * p.g2.G)));
+                // One node group of <= 16 nodes: k split over every resident
+                // CTA, partial tiles summed by the SiLU / residual-norm kernels
+                // (the small kernel between the GEMMs is where the W_o GEMM's
+                // CTAs become resident and fetch their first weight tiles).
+                // Larger node sets: the k splits of a tile are one cluster
+                // (the largest <= 8 whose clusters all fit on the GPU at
+                // once) and are summed on chip, with SiLU applied there.
+                const bool cluster = p.Nc > 16;
+                for (GemmArgs* g : {&p.g1, &p.g2}) {
+                    const int tiles_mg = g->MT * g->G;
+                    const int cap = cps * h->num_sms;
+                    if (cluster) {
+                        int sc = std::max(1, std::min({kMaxClusterK, g->KB, cap / tiles_mg}));
+                        for (; sc > 1; sc--)
+                            if (gemm_tc_max_clusters(g->NG, p.g1_smem, sc) >= tiles_mg) break;
+                        g->S = sc;
+                    } else {
+                        g->S = std::max(1, std::min(g->KB, cap / tiles_mg));
+                    }
+                    if (getenv("DART_DEBUG_PLAN"))
+                        fprintf(stderr, "dart: depth %d gemm K=%d tiles %d x k-splits %d%s, %d CTAs/SM\n", dep, g->K,
+                                tiles_mg, g->S, cluster ? " (cluster)" : "", cps);
+                }
+                p.g1.mode = cluster ? kGemmSiluSplit : kGemmPartials;
+                p.g2.mode = cluster ? kGemmSum : kGemmPartials;
             }
         }
     }
@@ -455,6 +479,7 @@ int enqueue_depth(dart_handle* h, int dep, const float* dlog, const float* ancho
     if (e != cudaSuccess) return DART_ERR_CUDA;
     GemmArgs g1 = p.g1, g2 = p.g2;
     g1.out = h->part;
+    g1.outL = h->AL;
     g2.out = h->part;
     g1.status = g2.status = h->status;
     pi = prof_begin(h, kGemm1, st);
@@ -467,10 +492,13 @@ int enqueue_depth(dart_handle* h, int dep, const float* dlog, const float* ancho
     }
     prof_end(h, pi, st);
     if (e != cudaSuccess) return DART_ERR_CUDA;
-    pi = prof_begin(h, kSilu, st);
-    e = launch_silu_split(p.Nc, c.d, g1.S, h->part, tc ? h->AL : nullptr, kNPadMax, h->A32, st);
-    prof_end(h, pi, st);
-    if (e != cudaSuccess) return DART_ERR_CUDA;
+    const bool fused = tc && g1.mode != kGemmPartials;  // SiLU applied in the GEMM's cluster reduction
+    if (!fused) {
+        pi = prof_begin(h, kSilu, st);
+        e = launch_silu_split(p.Nc, c.d, g1.S, h->part, tc ? h->AL : nullptr, kNPadMax, h->A32, st);
+        prof_end(h, pi, st);
+        if (e != cudaSuccess) return DART_ERR_CUDA;
+    }
     pi = prof_begin(h, kGemm2, st);
     if (tc) {
         e = launch_gemm_tc(&h->tmWo, &h->tmA[ng_index(g2.NG)], g2, p.g2_smem, st);
@@ -482,7 +510,7 @@ int enqueue_depth(dart_handle* h, int dep, const float* dlog, const float* ancho
     prof_end(h, pi, st);
     if (e != cudaSuccess) return DART_ERR_CUDA;
     pi = prof_begin(h, kNorm, st);
-    e = launch_residual_norm(p.Nc, c.d, g2.S, h->part, h->child_prow, hcur, c.rms_eps, hnext, tc ? h->HL : nullptr,
+    e = launch_residual_norm(p.Nc, c.d, fused ? 1 : g2.S, h->part, h->child_prow, hcur, c.rms_eps, hnext, tc ? h->HL : nullptr,
                              kNPadMax, st);
     prof_end(h, pi, st);
     if (e != cudaSuccess) return DART_ERR_CUDA;
@@ -808,7 +836,11 @@ int dart_profile_read(dart_handle* h, float* lmhead_ms, int* lmhead_launches) {
 int dart_launches_per_round(dart_handle* h) {
     if (!h) return DART_ERR_INVALID;
     const int L = h->cfg.L;
-    return 1 + 2 * L + 5 * (L - 1) + 1;
+    // prep, (LM-head + select) per depth, (gather, W_i GEMM, [SiLU,] W_o GEMM,
+    // residual-norm) per depth but the last, prune-emit
+    int n = 1 + 2 * L + 1;
+    for (int dep = 1; dep < L; dep++) n += (h->wdtype == DART_BF16 && h->plans[dep].g1.mode != kGemmPartials) ? 4 : 5;
+    return n;
 }
 
 void dart_destroy(dart_handle* h) {

@@ -2,6 +2,7 @@
 #pragma once
 
 #include <cuda.h>
+#include <cuda_bf16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -24,6 +25,27 @@ cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t s
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = pdl_enabled() ? 1 : 0;
+    return cudaLaunchKernelEx(&cfg, kernel, static_cast<Args&&>(args)...);
+}
+
+// The same with thread-block clusters of `cluster_x` consecutive CTAs.
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl_cluster(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t st,
+                               int cluster_x, Args&&... args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[2];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = static_cast<unsigned>(cluster_x);
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[1].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = pdl_enabled() ? 2 : 1;
     return cudaLaunchKernelEx(&cfg, kernel, static_cast<Args&&>(args)...);
 }
 
@@ -61,11 +83,18 @@ struct GemmArgs {
     int lo_kb_end;        // k-blocks >= this have a zero lo half (skipped)
     int bhalf;
     int stages;
-    float* out;           // [S][N][M]
+    int mode;             // tcgen05 path: kGemmPartials, or kGemmSiluSplit / kGemmSum (the k splits are one cluster)
+    float* out;           // fp32 path: partials [S][N][M]; kGemmSum: the sum [N][M]
+    __nv_bfloat16* outL;  // kGemmSiluSplit: SiLU of the sum as hi rows [N][M], lo rows from row bhalf
     int* status;
     const float* A32;     // fp32 path: A [M][K]
     const float* B32;     // fp32 path: B [N][K]
 };
+
+constexpr int kGemmPartials = 0;   // out[split] = partial A . B^T over the split's k range
+constexpr int kGemmSiluSplit = 1;  // out = split(SiLU(A . B^T)) (correction-head W_i layer)
+constexpr int kGemmSum = 2;        // out = A . B^T in fp32 (correction-head W_o layer)
+constexpr int kMaxClusterK = 8;    // k splits of one tile reduced on chip (portable cluster size)
 
 // tcgen05 kernels (dart_tc.cu)
 cudaError_t launch_lmhead_tc(const CUtensorMap* tmE, const CUtensorMap* tmH, const LmheadArgs& a,
@@ -76,7 +105,8 @@ int tc_stage_bytes(int NG);
 int lmhead_tc_fixed_smem(int NG, int k, int stages);
 int gemm_tc_fixed_smem(int stages);
 int lmhead_tc_ctas_per_sm(int NG, int smem);
-int gemm_tc_ctas_per_sm(int NG, int smem);  // resident CTAs per SM (occupancy API; needs limits set)
+int gemm_tc_ctas_per_sm(int NG, int smem);
+int gemm_tc_max_clusters(int NG, int smem, int cluster);  // resident CTAs per SM (occupancy API; needs limits set)
 cudaError_t tc_set_smem_limits(int max_dyn);
 
 // fp32 CUDA-core kernels (dart_f32.cu)

@@ -361,11 +361,6 @@ __global__ void __launch_bounds__(kEmitThreads) prune_emit_kernel(const EmitArgs
     if (tid == 0) a.n_nodes[s] = beff;
 }
 
-__device__ __forceinline__ void split_bf16(float x, __nv_bfloat16& hi, __nv_bfloat16& lo) {
-    hi = __float2bfloat16_rn(x);
-    lo = __float2bfloat16_rn(x - __bfloat162float(hi));
-}
-
 // 4 consecutive floats -> 4 hi and 4 lo bf16 (8-byte stores)
 __device__ __forceinline__ void split4(const float4 v, __nv_bfloat16* hi, __nv_bfloat16* lo) {
     __align__(8) __nv_bfloat16 h[4], l[4];
@@ -454,24 +449,26 @@ __global__ void silu_split_kernel(int Nc, int d, int S, const float* part, __nv_
     }
 }
 
-constexpr int kNormThreads = 1024;
-
 // One block per child: r = h[prow] + sum_s part[s], h_next = r / rms(r).
-__global__ void __launch_bounds__(kNormThreads) residual_norm_kernel(int d, int S, int Nc, const float* part,
-                                                                     const int* prow, const float* h, float eps,
-                                                                     float* h_next, __nv_bfloat16* HL, int bhalf) {
+// NT = 1024 threads when S partial tiles are summed (many loads in flight),
+// 256 for one summed tile (few registers, so blocks can become resident
+// beside the GEMM before it ends).
+template <int NT>
+__global__ void __launch_bounds__(NT) residual_norm_kernel(int d, int S, int Nc, const float* part, const int* prow,
+                                                           const float* h, float eps, float* h_next,
+                                                           __nv_bfloat16* HL, int bhalf) {
     pdl_trigger();
     pdl_wait();
     __shared__ float red[32];
     const int c = blockIdx.x;
     const int pr = prow[c];
     const size_t total = static_cast<size_t>(Nc) * d;
-    constexpr int kMaxPer = 4;  // d <= 16384 = 4 * 4 * 1024
+    constexpr int kMaxPer = 16384 / (4 * NT);  // d <= 16384
     float4 r[kMaxPer];
     float ss = 0.0f;
 #pragma unroll
     for (int it = 0; it < kMaxPer; it++) {
-        const int j = (it * kNormThreads + threadIdx.x) * 4;
+        const int j = (it * NT + threadIdx.x) * 4;
         r[it] = make_float4(0.f, 0.f, 0.f, 0.f);
         if (j < d && pr >= 0) {
             float4 v = *reinterpret_cast<const float4*>(h + static_cast<size_t>(pr) * d + j);
@@ -491,7 +488,7 @@ __global__ void __launch_bounds__(kNormThreads) residual_norm_kernel(int d, int 
     const float inv = 1.0f / sqrtf(tot / static_cast<float>(d) + eps);
 #pragma unroll
     for (int it = 0; it < kMaxPer; it++) {
-        const int j = (it * kNormThreads + threadIdx.x) * 4;
+        const int j = (it * NT + threadIdx.x) * 4;
         if (j < d) {
             const float4 v = make_float4(r[it].x * inv, r[it].y * inv, r[it].z * inv, r[it].w * inv);
             *reinterpret_cast<float4*>(h_next + static_cast<size_t>(c) * d + j) = v;
@@ -550,7 +547,10 @@ cudaError_t launch_silu_split(int Nc, int d, int S, const float* part, __nv_bflo
 
 cudaError_t launch_residual_norm(int Nc, int d, int S, const float* part, const int* prow, const float* h,
                                  float eps, float* h_next, __nv_bfloat16* HL, int bhalf, cudaStream_t st) {
-    return launch_pdl(residual_norm_kernel, dim3(Nc), dim3(kNormThreads), 0, st, d, S, Nc, part, prow, h, eps, h_next,
+    if (S > 1)
+        return launch_pdl(residual_norm_kernel<1024>, dim3(Nc), dim3(1024), 0, st, d, S, Nc, part, prow, h, eps,
+                          h_next, HL, bhalf);
+    return launch_pdl(residual_norm_kernel<256>, dim3(Nc), dim3(256), 0, st, d, S, Nc, part, prow, h, eps, h_next,
                       HL, bhalf);
 }
 

@@ -334,6 +334,17 @@ __global__ void __launch_bounds__(threads<NG>(), 1)
 }
 
 // --------------------------------------------------------------- GEMM kernel
+//
+// Correction-head layer out = A . B^T with A = W_i or W_o [M x K] and B the
+// node inputs [N x K], split over K into a.S parts.
+//   kGemmPartials:  every CTA writes its fp32 partial tile to out[split]; the
+//                   elementwise kernels that follow sum the splits.
+//   kGemmSiluSplit, kGemmSum: the S splits of one (M tile, node group) form
+//                   a thread-block cluster: every CTA stages its fp32 tile in
+//                   shared memory, and after a cluster barrier CTA r sums
+//                   rows [r*R, (r+1)*R) of the tile over the S CTAs in rank
+//                   order (deterministic) and writes outL = hi/lo bf16 split
+//                   of SiLU(sum) (input of W_o), or out = sum in fp32.
 
 template <int NG>
 __global__ void __launch_bounds__(threads<NG>(), 1)
@@ -344,21 +355,24 @@ __global__ void __launch_bounds__(threads<NG>(), 1)
     const int stages = a.stages;
     Smem s = carve<NG>(smem_raw, stages);
 
-    const int mt = blockIdx.x % a.MT;
-    const int rest = blockIdx.x / a.MT;
-    const int g = rest % a.G;
-    const int split = rest / a.G;
+    // block = (g * MT + mt) * S + split: the S splits of a tile are consecutive,
+    // i.e. one cluster
+    const int tile = blockIdx.x / a.S;
+    const int mt_c = tile % a.MT, g_c = tile / a.MT, split_c = blockIdx.x % a.S;
     Work w;
     w.ntiles = 1;
-    w.row0 = mt * kTileM;
-    w.kb0 = static_cast<int>((static_cast<long long>(split) * a.KB) / a.S);
-    w.kb1 = static_cast<int>((static_cast<long long>(split + 1) * a.KB) / a.S);
-    w.brow = g * NG;
+    w.row0 = mt_c * kTileM;
+    w.kb0 = static_cast<int>((static_cast<long long>(split_c) * a.KB) / a.S);
+    w.kb1 = static_cast<int>((static_cast<long long>(split_c + 1) * a.KB) / a.S);
+    w.brow = g_c * NG;
     w.lo_kb_end = a.lo_kb_end;
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const uint32_t tmem_base = setup<NG>(s, stages, tmem_cols<NG>());
     volatile int* abort = &s.misc[1];
+    // staging tile [NG nodes][128 rows] fp32, in the pipeline ring (free once
+    // the last MMA has completed)
+    float* stage_tile = reinterpret_cast<float*>(s.ring);
 
     if (warp == 0) {
         if (lane == 0) producer<NG>(&tmA, &tmB, w, a.bhalf, s.ring, stages, s.full, s.empty, abort, a.status);
@@ -378,9 +392,6 @@ __global__ void __launch_bounds__(threads<NG>(), 1)
         named_bar_sync(kEpiBarrier, epi_threads<NG>());
         if (s.misc[2] != 0) {
             tc_fence_after();
-            const int m = w.row0 + quarter * 32 + lane;
-            const bool valid = m < a.M;
-            float* out = a.out + static_cast<size_t>(split) * a.N * a.M;
             const int c0 = ((warp - 2) >> 2) * 16;
             float vals[16], lov[16];
             const uint32_t tcol = tmem_base + c0 + (static_cast<uint32_t>(quarter * 32) << 16);
@@ -390,14 +401,54 @@ __global__ void __launch_bounds__(threads<NG>(), 1)
 #pragma unroll
                 for (int j = 0; j < 16; j++) vals[j] += lov[j];
             }
+            if (a.mode == kGemmPartials) {
+                const int m = w.row0 + quarter * 32 + lane;
+                float* out = a.out + static_cast<size_t>(split_c) * a.N * a.M;
 #pragma unroll
-            for (int j = 0; j < 16; j++) {
-                const int n = g * NG + c0 + j;
-                if (valid && n < a.N) out[static_cast<size_t>(n) * a.M + m] = vals[j];
+                for (int j = 0; j < 16; j++) {
+                    const int n = g_c * NG + c0 + j;
+                    if (m < a.M && n < a.N) out[static_cast<size_t>(n) * a.M + m] = vals[j];
+                }
+            } else {
+#pragma unroll
+                for (int j = 0; j < 16; j++) stage_tile[(c0 + j) * kTileM + quarter * 32 + lane] = vals[j];
             }
         }
     }
     teardown(tmem_base, tmem_cols<NG>());
+    if (a.mode == kGemmPartials) return;  // launched without clusters
+    cluster_sync_all();  // every split's tile is staged
+    {
+        const int S = a.S;
+        const uint32_t r = cluster_ctarank();
+        const int R = (kTileM + S - 1) / S;
+        const int nthr = threads<NG>();
+        const uint32_t base = smem_u32(stage_tile);
+        for (int idx = threadIdx.x; idx < R * NG; idx += nthr) {
+            const int nl = idx / R, row = static_cast<int>(r) * R + idx % R;
+            const int m = w.row0 + row, n = g_c * NG + nl;
+            if (row >= kTileM || m >= a.M || n >= a.N) continue;
+            const uint32_t off = base + static_cast<uint32_t>((nl * kTileM + row) * 4);
+            float v[kMaxClusterK];
+#pragma unroll
+            for (int q = 0; q < kMaxClusterK; q++) v[q] = q < S ? ld_cluster_f32(off, static_cast<uint32_t>(q)) : 0.0f;
+            float acc = 0.0f;
+#pragma unroll
+            for (int q = 0; q < kMaxClusterK; q++)
+                if (q < S) acc += v[q];
+            const size_t o = static_cast<size_t>(n) * a.M + m;
+            if (a.mode == kGemmSiluSplit) {
+                const float act = acc / (1.0f + expf(-acc));
+                __nv_bfloat16 hi, lo;
+                split_bf16(act, hi, lo);
+                a.outL[o] = hi;
+                a.outL[static_cast<size_t>(a.bhalf) * a.M + o] = lo;
+            } else {
+                a.out[o] = acc;
+            }
+        }
+    }
+    cluster_sync_all();  // no CTA leaves while a peer still reads its staging tile
 }
 
 template <int NG>
@@ -413,7 +464,31 @@ cudaError_t launch_lmhead_ng(const CUtensorMap* tmE, const CUtensorMap* tmH, con
 template <int NG>
 cudaError_t launch_gemm_ng(const CUtensorMap* tmA, const CUtensorMap* tmB, const GemmArgs& a, int smem,
                            cudaStream_t st) {
-    return launch_pdl(gemm_tc_kernel<NG>, dim3(a.MT * a.G * a.S), dim3(threads<NG>()), smem, st, *tmA, *tmB, a);
+    if (a.mode == kGemmPartials)
+        return launch_pdl(gemm_tc_kernel<NG>, dim3(a.MT * a.G * a.S), dim3(threads<NG>()), smem, st, *tmA, *tmB, a);
+    return launch_pdl_cluster(gemm_tc_kernel<NG>, dim3(a.MT * a.G * a.S), dim3(threads<NG>()), smem, st, a.S, *tmA,
+                              *tmB, a);
+}
+
+template <int NG>
+int max_clusters_ng(int smem, int cluster) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(cluster * 1024);
+    cfg.blockDim = dim3(threads<NG>());
+    cfg.dynamicSmemBytes = smem;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = static_cast<unsigned>(cluster);
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    int n = 0;
+    if (cudaOccupancyMaxActiveClusters(&n, gemm_tc_kernel<NG>, &cfg) != cudaSuccess) {
+        cudaGetLastError();
+        return 0;
+    }
+    return n;
 }
 
 }  // namespace
@@ -458,6 +533,14 @@ int gemm_tc_ctas_per_sm(int NG, int smem) {
         case 16: return ctas_per_sm(reinterpret_cast<const void*>(gemm_tc_kernel<16>), threads<16>(), smem);
         case 32: return ctas_per_sm(reinterpret_cast<const void*>(gemm_tc_kernel<32>), threads<32>(), smem);
         default: return ctas_per_sm(reinterpret_cast<const void*>(gemm_tc_kernel<64>), threads<64>(), smem);
+    }
+}
+
+int gemm_tc_max_clusters(int NG, int smem, int cluster) {
+    switch (NG) {
+        case 16: return max_clusters_ng<16>(smem, cluster);
+        case 32: return max_clusters_ng<32>(smem, cluster);
+        default: return max_clusters_ng<64>(smem, cluster);
     }
 }
 
