@@ -49,7 +49,7 @@ def build(force: bool = False) -> str:
 class _Cfg(C.Structure):
     _fields_ = [("V", C.c_int), ("d", C.c_int), ("L", C.c_int), ("W", C.c_int),
                 ("k", C.c_int), ("B", C.c_int), ("nseq", C.c_int),
-                ("pos_offset", C.c_int), ("wdtype", C.c_int),
+                ("pos_offset", C.c_int), ("wdtype", C.c_int), ("cand_k", C.c_int),
                 ("beta", C.c_double), ("temperature", C.c_double),
                 ("rms_eps", C.c_double)]
 
@@ -57,7 +57,8 @@ class _Cfg(C.Structure):
 def _cfg(cfg) -> _Cfg:
     return _Cfg(int(cfg.V), int(cfg.d), int(cfg.L), int(cfg.W), int(cfg.k), int(cfg.B),
                 int(cfg.nseq), int(cfg.pos_offset), 0 if cfg.wdtype == "f32" else 1,
-                float(cfg.beta), float(cfg.temperature), float(cfg.rms_eps))
+                int(getattr(cfg, "cand_k", 0)), float(cfg.beta), float(cfg.temperature),
+                float(cfg.rms_eps))
 
 
 def lib():
@@ -116,6 +117,20 @@ def log_softmax(z):
     return out, float(lse)
 
 
+def cand_count(cfg) -> int:
+    """Entries scored per node: the candidate-set size K, or V (full vocabulary)."""
+    K = int(getattr(cfg, "cand_k", 0))
+    return K if K > 0 else int(cfg.V)
+
+
+def candidates(cfg, dlog_row):
+    """C_d = TopK(L_d^base, K) of Algorithm 1, sorted by token id."""
+    dlog_row = np.ascontiguousarray(dlog_row, dtype=np.float32)
+    out = np.empty(int(cfg.cand_k), dtype=np.int32)
+    lib().orc_candidates(C.byref(_cfg(cfg)), _p(dlog_row), _p(out))
+    return out
+
+
 def topk(x, kk):
     x = np.ascontiguousarray(x, dtype=np.float64)
     idx = np.empty(kk, dtype=np.int32)
@@ -132,7 +147,7 @@ def build_tree(cfg, Wi, Wo, E, Dlog, h0):
     Dlog = np.ascontiguousarray(Dlog, dtype=np.float32)
     h0 = np.ascontiguousarray(h0, dtype=np.float32)
     ns, L, W, B = cfg.nseq, cfg.L, cfg.W, cfg.B
-    kx = min(cfg.k + 1, cfg.V)
+    kx = min(cfg.k + 1, cand_count(cfg))
     nw = (B + 63) // 64
     r = dict(
         st_tok=np.empty((ns, L, W), np.int32), st_parent=np.empty((ns, L, W), np.int32),

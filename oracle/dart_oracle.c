@@ -11,9 +11,10 @@
  *
  * What it computes (paper: "DARTree: Speculative Diffusion Decoding with
  * Autoregressive Draft Trees", arXiv 2608.13524):
- *   - Algorithm 1 (depth-wise fixed-width supertree construction) with the
- *     full vocabulary as candidate set and a per-node top-k (Appendix D,
- *     "Full" candidate vocabulary);
+ *   - Algorithm 1 (depth-wise fixed-width supertree construction) with a
+ *     per-node top-k, over either the full vocabulary (Appendix D, "Full")
+ *     or the candidate set C_d = TopK(L_d^base, K) of Algorithm 1 (cand_k =
+ *     K > 0; the paper's default is K = 64, Sec. 4.1);
  *   - the path score of Eq. 5, s_beta(u_{1:d}) = sum_i log q~_i(u_i) + beta d;
  *   - deferred pruning, T = TopB_{u in S} s_beta(u) (Algorithm 1, final step);
  *   - the best-first heap of Sec. 3.3 / Lemma 1 (used to check that the top-B
@@ -25,7 +26,12 @@
  *       h_c = RMSNorm(h_p + W_o SiLU(W_i [h_p ; E[t_c]])),  RMSNorm without gain;
  *   - corrected child distribution of a node with state h at depth d-1:
  *       z[v] = (Dlog[d-1][v] + E[v] . h) / T'   (T' = T if T > 0 else 1),
- *       log q~[v] = min(z[v] - logsumexp(z), 0)  (clamp keeps Lemma 1 exact);
+ *       log q~[v] = min(z[v] - logsumexp(z), 0)  (clamp keeps Lemma 1 exact),
+ *     the log-sum-exp running over the vocabulary, or over C_d when the
+ *     candidate set is restricted (q~ renormalised over C_d: Algorithm 1
+ *     evaluates g only on C_d, so tokens outside C_d have no probability);
+ *   - C_d = the K tokens of largest drafter logit Dlog[d-1][v] (ties: token
+ *     asc), the same for every node of the depth;
  *   - ties: per-node top-k by (log q~ desc, token asc); frontier by
  *     (score desc, parent slot asc, rank-in-parent-list asc); pruning by
  *     (score desc, node id asc) with node id = (depth-1)*W + frontier rank, so
@@ -43,6 +49,7 @@
 
 typedef struct {
     int V, d, L, W, k, B, nseq, pos_offset, wdtype; /* wdtype 0: float32, 1: bf16 bits */
+    int cand_k;                                     /* K of Algorithm 1; 0 = full vocabulary */
     double beta, temperature, rms_eps;
 } orc_cfg;
 
@@ -143,6 +150,64 @@ double orc_log_softmax(const double *z, int V, double *logq) {
     return lse;
 }
 
+/* ------------------------------------------ restricted candidate set C_d */
+
+static int int_cmp(const void *a_, const void *b_) {
+    const int a = *(const int *)a_, b = *(const int *)b_;
+    return (a > b) - (a < b);
+}
+
+void orc_topk(const double *x, int n, int kk, int *idx);
+
+/* C_d = TopK(L_d^base, K) (Algorithm 1): the cand_k tokens with the largest
+ * base (drafter) logits of this position, ties by token asc, returned sorted
+ * by token id. */
+void orc_candidates(const orc_cfg *c, const float *dlog_row, int *cand) {
+    double *x = (double *)malloc(sizeof(double) * (size_t)c->V);
+    for (int v = 0; v < c->V; v++) x[v] = (double)dlog_row[v];
+    orc_topk(x, c->V, c->cand_k, cand);
+    qsort(cand, (size_t)c->cand_k, sizeof(int), int_cmp);
+    free(x);
+}
+
+/* Corrected child distribution over the candidates only (Algorithm 1 applies
+ * g to C_d): z_i = (Dlog[C_i] + E[C_i] . h) / T', log q~_i = min(z_i -
+ * logsumexp_i z, 0).  Returns the log-sum-exp over C_d. */
+double orc_restricted_logq(const orc_cfg *c, const void *E, const float *dlog_row,
+                           const int *cand, const double *h, double *lq) {
+    const double Tp = c->temperature > 0.0 ? c->temperature : 1.0;
+    const int K = c->cand_k, d = c->d, dt = c->wdtype;
+    double *z = (double *)malloc(sizeof(double) * (size_t)K);
+    for (int i = 0; i < K; i++)
+        z[i] = ((double)dlog_row[cand[i]] + wdot(E, dt, (size_t)cand[i] * d, h, d)) / Tp;
+    double lse = orc_log_softmax(z, K, lq);
+    free(z);
+    return lse;
+}
+
+/* Corrected log-probabilities of every token (tokens outside C_d: -inf) and
+ * the log-sum-exp; full vocabulary when cand_k = 0. */
+static double child_logq_all(const orc_cfg *c, const void *E, const float *dlog_row, const double *h,
+                             double *lq_all) {
+    const int V = c->V;
+    if (c->cand_k <= 0) {
+        double *z = (double *)malloc(sizeof(double) * (size_t)V);
+        orc_child_logits(c, E, dlog_row, h, z);
+        double lse = orc_log_softmax(z, V, lq_all);
+        free(z);
+        return lse;
+    }
+    int *cand = (int *)malloc(sizeof(int) * (size_t)c->cand_k);
+    double *lq = (double *)malloc(sizeof(double) * (size_t)c->cand_k);
+    orc_candidates(c, dlog_row, cand);
+    double lse = orc_restricted_logq(c, E, dlog_row, cand, h, lq);
+    for (int v = 0; v < V; v++) lq_all[v] = -INFINITY;
+    for (int i = 0; i < c->cand_k; i++) lq_all[cand[i]] = lq[i];
+    free(cand);
+    free(lq);
+    return lse;
+}
+
 static int better(double a, int ia, double b, int ib) {
     return a > b || (a == b && ia < ib);
 }
@@ -189,7 +254,12 @@ static int node_cmp(const void *a_, const void *b_) {
     return a->id < b->id ? -1 : (a->id > b->id);
 }
 
-static int kx_of(const orc_cfg *c) { return c->k + 1 <= c->V ? c->k + 1 : c->V; }
+/* Children listed per node: k + 1 (one more than kept, for rank-gap checks),
+ * at most the number of candidates. */
+static int kx_of(const orc_cfg *c) {
+    const int n = c->cand_k > 0 ? c->cand_k : c->V;
+    return c->k + 1 <= n ? c->k + 1 : n;
+}
 
 /* Emission for one sequence: global top-B over the supertree (Algorithm 1,
  * final step), flattened in ascending node id, which is a topological order.
@@ -291,11 +361,16 @@ int orc_build_tree(const orc_cfg *c, const void *Wi, const void *Wo, const void 
                    double *nd_logq, double *fr_score, int *o_tok, int *o_par, int *o_dep,
                    int *o_pos, double *o_score, int *o_n, uint64_t *o_mask, double *prune_gap) {
     const int V = c->V, d = c->d, L = c->L, W = c->W, k = c->k, kx = kx_of(c);
+    /* entries scored per node: every token, or the candidate set C_d
+     * (ent[i] = token of entry i, ascending) */
+    const int nent = c->cand_k > 0 ? c->cand_k : V;
     double *hs = (double *)malloc(sizeof(double) * (size_t)W * d);
     double *hn = (double *)malloc(sizeof(double) * (size_t)W * d);
     double *z = (double *)malloc(sizeof(double) * (size_t)V);
     double *logq = (double *)malloc(sizeof(double) * (size_t)V);
+    int *ent = (int *)malloc(sizeof(int) * (size_t)nent);
     int *idx = (int *)malloc(sizeof(int) * (size_t)kx);
+    for (int i = 0; i < nent; i++) ent[i] = i;
     cand_t *cand = (cand_t *)malloc(sizeof(cand_t) * (size_t)W * k + 1);
     double pscore[1024], nscore[1024];
     int rc = 0;
@@ -307,6 +382,7 @@ int orc_build_tree(const orc_cfg *c, const void *Wi, const void *Wo, const void 
         for (int dep = 1; dep <= L; dep++) {
             const float *row = Dlog + ((size_t)s * L + dep - 1) * V;
             const size_t nb = ((size_t)s * L + dep - 1) * W;
+            if (c->cand_k > 0) orc_candidates(c, row, ent); /* C_d = TopK(L_d^base, K) */
             int ncand = 0;
             for (int p = 0; p < W; p++) {
                 nd_lse[nb + p] = -INFINITY;
@@ -317,18 +393,23 @@ int orc_build_tree(const orc_cfg *c, const void *Wi, const void *Wo, const void 
             }
             /* score every child of every retained prefix in S_{d-1} */
             for (int p = 0; p < pcount; p++) {
-                orc_child_logits(c, E, row, hs + (size_t)p * d, z);
-                nd_lse[nb + p] = orc_log_softmax(z, V, logq);
-                orc_topk(logq, V, kx, idx);
+                if (c->cand_k > 0) {
+                    nd_lse[nb + p] = orc_restricted_logq(c, E, row, ent, hs + (size_t)p * d, logq);
+                } else {
+                    orc_child_logits(c, E, row, hs + (size_t)p * d, z);
+                    nd_lse[nb + p] = orc_log_softmax(z, V, logq);
+                }
+                /* entries are in token order, so index ties are token ties */
+                orc_topk(logq, nent, kx, idx);
                 for (int j = 0; j < kx; j++) {
-                    nd_tok[(nb + p) * kx + j] = idx[j];
+                    nd_tok[(nb + p) * kx + j] = ent[idx[j]];
                     nd_logq[(nb + p) * kx + j] = logq[idx[j]];
                 }
                 for (int j = 0; j < k; j++) {
                     cand[ncand].score = pscore[p] + logq[idx[j]] + c->beta; /* Eq. 5 */
                     cand[ncand].p = p;
                     cand[ncand].j = j;
-                    cand[ncand].tok = idx[j];
+                    cand[ncand].tok = ent[idx[j]];
                     ncand++;
                 }
             }
@@ -366,6 +447,7 @@ int orc_build_tree(const orc_cfg *c, const void *Wi, const void *Wo, const void 
     free(hn);
     free(z);
     free(logq);
+    free(ent);
     free(idx);
     free(cand);
     return rc;
@@ -458,17 +540,30 @@ double orc_node_children(const orc_cfg *c, const void *Wi, const void *Wo, const
                          int kk, int *tok_out, double *logq_out, double *logq_all) {
     const int V = c->V, d = c->d;
     double *h = (double *)malloc(sizeof(double) * (size_t)d);
-    double *z = (double *)malloc(sizeof(double) * (size_t)V);
     double *lq = logq_all ? logq_all : (double *)malloc(sizeof(double) * (size_t)V);
     orc_path_state(c, Wi, Wo, E, h0_seq, path, len, h);
-    orc_child_logits(c, E, Dlog_seq + (size_t)len * V, h, z);
-    double lse = orc_log_softmax(z, V, lq);
+    const float *row = Dlog_seq + (size_t)len * V;
+    double lse = child_logq_all(c, E, row, h, lq);
     if (kk > 0) {
-        orc_topk(lq, V, kk, tok_out);
-        for (int j = 0; j < kk; j++) logq_out[j] = lq[tok_out[j]];
+        if (c->cand_k > 0) {
+            /* the kk best candidates (kk <= cand_k), ties by token asc */
+            int *cand = (int *)malloc(sizeof(int) * (size_t)c->cand_k);
+            double *lc = (double *)malloc(sizeof(double) * (size_t)c->cand_k);
+            orc_candidates(c, row, cand);
+            for (int i = 0; i < c->cand_k; i++) lc[i] = lq[cand[i]];
+            orc_topk(lc, c->cand_k, kk, tok_out);
+            for (int j = 0; j < kk; j++) {
+                logq_out[j] = lc[tok_out[j]];
+                tok_out[j] = cand[tok_out[j]];
+            }
+            free(cand);
+            free(lc);
+        } else {
+            orc_topk(lq, V, kk, tok_out);
+            for (int j = 0; j < kk; j++) logq_out[j] = lq[tok_out[j]];
+        }
     }
     free(h);
-    free(z);
     if (!logq_all) free(lq);
     return lse;
 }
@@ -480,13 +575,11 @@ void orc_path_scores(const orc_cfg *c, const void *Wi, const void *Wo, const voi
     const int V = c->V, d = c->d;
     double *h = (double *)malloc(sizeof(double) * (size_t)d);
     double *t = (double *)malloc(sizeof(double) * (size_t)d);
-    double *z = (double *)malloc(sizeof(double) * (size_t)V);
     double *lq = (double *)malloc(sizeof(double) * (size_t)V);
     for (int j = 0; j < d; j++) h[j] = (double)h0_seq[j];
     double s = 0.0;
     for (int i = 0; i < len; i++) {
-        orc_child_logits(c, E, Dlog_seq + (size_t)i * V, h, z);
-        orc_log_softmax(z, V, lq);
+        child_logq_all(c, E, Dlog_seq + (size_t)i * V, h, lq);
         s += lq[path[i]] + c->beta;
         scores[i] = s;
         if (i + 1 < len) {
@@ -496,6 +589,5 @@ void orc_path_scores(const orc_cfg *c, const void *Wi, const void *Wo, const voi
     }
     free(h);
     free(t);
-    free(z);
     free(lq);
 }

@@ -51,19 +51,45 @@ def child_logq(cfg, E64, dlog_row, h):
     return torch.clamp(torch.log_softmax(z, dim=0), max=0.0)
 
 
+def topK_candidates(dlog_row, K):
+    """C = the K largest base logits, ties by token asc (numpy lexsort), as a
+    sorted token array."""
+    row = np.asarray(dlog_row, np.float64)
+    order = np.lexsort((np.arange(row.size), -row))
+    return np.sort(order[:K])
+
+
+def child_logq_restricted(cfg, E64, dlog_row, h, cand):
+    """Clamped log-softmax over the candidate subset only (torch fp64); a
+    full-vocabulary tensor with -inf outside the subset."""
+    Tp = cfg.temperature if cfg.temperature > 0 else 1.0
+    idx = torch.from_numpy(np.asarray(cand, np.int64))
+    z = (torch.from_numpy(np.asarray(dlog_row, np.float64))[idx] + E64[idx] @ h) / Tp
+    out = torch.full((cfg.V,), float("-inf"), dtype=torch.float64)
+    out[idx] = torch.clamp(torch.log_softmax(z, dim=0), max=0.0)
+    return out
+
+
 def all_path_scores(cfg, Wi, Wo, E, Dlog_seq, h0_seq, max_len):
     """Exhaustive enumeration: Eq. 5 score of every token path of length
-    1..max_len, each recomputed from the root on its own (no shared state)."""
+    1..max_len, each recomputed from the root on its own (no shared state).
+    With cfg.cand_k = K > 0 the paths run over the candidate sets C_i (the K
+    largest base logits of position i) and q~ is renormalised over C_i."""
     head = TorchHead(cfg, Wi, Wo, E)
     E64 = head.E
     h0 = torch.from_numpy(np.asarray(h0_seq, np.float64))
+    K = int(getattr(cfg, "cand_k", 0))
+    cands = [topK_candidates(Dlog_seq[i], K) if K > 0 else np.arange(cfg.V) for i in range(max_len)]
     out = {}
     for n in range(1, max_len + 1):
-        for path in itertools.product(range(cfg.V), repeat=n):
+        for path in itertools.product(*[[int(t) for t in cands[i]] for i in range(n)]):
             h = h0.clone()
             s = 0.0
             for i, t in enumerate(path):
-                lq = child_logq(cfg, E64, Dlog_seq[i], h)
+                if K > 0:
+                    lq = child_logq_restricted(cfg, E64, Dlog_seq[i], h, cands[i])
+                else:
+                    lq = child_logq(cfg, E64, Dlog_seq[i], h)
                 s += float(lq[t]) + cfg.beta
                 h = head(h, t)
             out[path] = s

@@ -11,7 +11,8 @@ import pytest
 import torch
 
 import oracle
-from refs import TorchHead, all_path_scores, child_logq, ddtree_topB, weights64
+from refs import (TorchHead, all_path_scores, child_logq, child_logq_restricted, ddtree_topB,
+                  topK_candidates, weights64)
 from workloads import TOY, Config, bf16_bits_to_f32, f32_to_bf16_bits, make_inputs
 
 
@@ -366,3 +367,126 @@ def test_prune_tiebreak_inside_tied_group():
         np.testing.assert_array_equal(e["depths"][0, :B], [i // cfg.W + 1 for i in keep])
         popped = oracle.heap_select(cfg, r["st_parent"], r["st_score"], r["st_count"], 0)
         assert sorted(popped.tolist()) == keep
+
+
+# ------------------------------------- candidate-restricted scoring (K)
+
+def _emitted_paths(r, s=0):
+    out = {}
+    for i in range(r["n_nodes"][s]):
+        path, j = [], i
+        while j >= 0:
+            path.append(int(r["tokens"][s, j]))
+            j = int(r["parents"][s, j])
+        out[tuple(reversed(path))] = r["scores"][s, i]
+    return out
+
+
+def test_candidates_match_lexsort_with_ties():
+    """C_d = TopK(L_d^base, K): the K largest base logits, ties by token asc."""
+    cfg = tiny(V=300, cand_k=37)
+    g = np.random.default_rng(5)
+    row = np.round(g.standard_normal(cfg.V) * 2) .astype(np.float32) / 2  # many exact ties
+    got = oracle.candidates(cfg, row)
+    np.testing.assert_array_equal(got, topK_candidates(row, cfg.cand_k))
+    assert np.all(np.diff(got) > 0)
+
+
+def test_restricted_with_K_equal_V_is_full_vocabulary():
+    """K = V restricts nothing: the tree equals the full-vocabulary tree."""
+    cfg = tiny(V=50, d=12, L=4, W=6, k=6, B=15, temperature=0.8, seed=21)
+    x = rand_inputs(cfg)
+    full = run(cfg, x)
+    rest = run(cfg.replace(cand_k=cfg.V), x)
+    for key in ("st_tok", "st_parent", "st_count", "tokens", "parents", "depths", "mask", "n_nodes"):
+        np.testing.assert_array_equal(full[key], rest[key])
+    np.testing.assert_allclose(full["st_score"], rest["st_score"], atol=1e-12)
+    np.testing.assert_allclose(full["nd_lse"], rest["nd_lse"], atol=1e-12)
+
+
+@pytest.mark.parametrize("temperature,beta", [(0.0, -0.2), (0.9, 0.0)])
+def test_restricted_bruteforce_full_supertree(temperature, beta):
+    """V = 7, K = 3, W = K^L, k = K: the supertree is every path through the
+    candidate sets; each node's score must equal an independent per-path
+    recomputation with q~ renormalised over C_d (library log_softmax on the
+    subset), and the pruned tree must be the brute-force top-B."""
+    cfg = tiny(V=7, L=3, W=27, k=3, B=17, cand_k=3, temperature=temperature, beta=beta, seed=31)
+    x = rand_inputs(cfg)
+    r = run(cfg, x)
+    brute = all_path_scores(cfg, x["Wi"], x["Wo"], x["E"], x["Dlog"][0], x["h0"][0], cfg.L)
+    paths = oracle.node_paths(r["st_tok"], r["st_parent"], r["st_count"], 0, cfg.W)
+    assert len(paths) == len(brute) == 3 + 9 + 27
+    for nid, p in paths.items():
+        assert abs(r["st_score"][0].reshape(-1)[nid] - brute[p]) < 1e-12
+    ranked = sorted(brute.items(), key=lambda kv: -kv[1])
+    assert ranked[cfg.B - 1][1] - ranked[cfg.B][1] > 1e-9
+    assert set(_emitted_paths(r)) == {p for p, _ in ranked[:cfg.B]}
+
+
+def test_restricted_beam_levels_and_normalisation():
+    """Each S_d is the top-W of the K candidates of every node of S_{d-1},
+    scored by an independent recomputation; q~ sums to one over C_d and is
+    zero outside it."""
+    cfg = tiny(V=60, d=10, L=4, W=5, k=5, B=9, cand_k=8, temperature=0.7, seed=41)
+    x = rand_inputs(cfg)
+    r = run(cfg, x)
+    head = TorchHead(cfg, x["Wi"], x["Wo"], x["E"])
+    frontier = [((), 0.0, torch.from_numpy(x["h0"][0].astype(np.float64)))]
+    for dep in range(1, cfg.L + 1):
+        cand = topK_candidates(x["Dlog"][0, dep - 1], cfg.cand_k)
+        cands = []
+        for path, s, h in frontier:
+            lq = child_logq_restricted(cfg, head.E, x["Dlog"][0, dep - 1], h, cand).numpy()
+            assert abs(np.exp(lq[cand]).sum() - 1.0) < 1e-12
+            for t in cand:
+                cands.append((s + lq[t] + cfg.beta, path + (int(t),), h, int(t)))
+        cands.sort(key=lambda c: -c[0])
+        keep = cands[:cfg.W]
+        got = [tuple(oracle.node_paths(r["st_tok"], r["st_parent"], r["st_count"], 0, cfg.W)
+                     [(dep - 1) * cfg.W + j]) for j in range(int(r["st_count"][0, dep - 1]))]
+        assert got == [c[1] for c in keep]
+        np.testing.assert_allclose(r["st_score"][0, dep - 1, :len(keep)], [c[0] for c in keep],
+                                   atol=1e-12)
+        frontier = [(c[1], c[0], head(c[2], c[3])) for c in keep]
+    # the oracle's own per-node distribution: zero outside C_d, sums to one over it
+    tok, lq, lse, lq_all = oracle.node_children(cfg, x["Wi"], x["Wo"], x["E"], x["Dlog"][0], x["h0"][0],
+                                                np.array([], np.int32), cfg.k, want_all=True)
+    cand = topK_candidates(x["Dlog"][0, 0], cfg.cand_k)
+    outside = np.setdiff1d(np.arange(cfg.V), cand)
+    assert np.all(np.isneginf(lq_all[outside]))
+    assert abs(np.exp(lq_all[cand]).sum() - 1.0) < 1e-12
+    assert set(tok.tolist()) <= set(cand.tolist())
+
+
+def test_restricted_zero_E_is_ddtree_over_candidates():
+    """E = 0: q~ is the base distribution renormalised over C_d, path
+    independent, so with W, k >= B the pruned tree equals DDTree's best-first
+    top-B over the restricted marginals."""
+    cfg = tiny(V=80, d=16, L=5, W=12, k=12, B=12, cand_k=16, beta=-0.2, seed=51)
+    x = rand_inputs(cfg)
+    x["E"] = np.zeros_like(x["E"])
+    r = run(cfg, x)
+    rows = []
+    for i in range(cfg.L):
+        cand = topK_candidates(x["Dlog"][0, i], cfg.cand_k)
+        row = np.full(cfg.V, -np.inf)
+        row[cand] = torch.log_softmax(torch.from_numpy(x["Dlog"][0, i, cand].astype(np.float64)), 0).numpy()
+        rows.append(row + cfg.beta)
+    want = ddtree_topB(rows, cfg.B)
+    got = _emitted_paths(r)
+    assert set(got) == {p for p, _ in want}
+    for p, s in want:
+        assert abs(got[p] - s) < 1e-12
+
+
+def test_restricted_tree_structure():
+    """Prefix closure, monotone scores, depths, position ids and the mask hold
+    in the restricted mode too, and every token lies in its depth's C_d."""
+    cfg = tiny(V=200, d=16, L=6, W=6, k=6, B=20, cand_k=10, temperature=1.0, seed=61, nseq=2)
+    x = rand_inputs(cfg)
+    r = run(cfg, x)
+    _check_tree_structure(cfg, r)
+    for s in range(cfg.nseq):
+        for i in range(r["n_nodes"][s]):
+            dep = int(r["depths"][s, i])
+            assert r["tokens"][s, i] in set(topK_candidates(x["Dlog"][s, dep - 1], cfg.cand_k).tolist())

@@ -53,6 +53,7 @@ class Config:
     pos_offset: int = 0
     spike_early: float = 6.0   # positions 0..7
     spike_late: float = 3.0    # positions 8..
+    cand_k: int = 0            # K of Algorithm 1 (candidate-set size); 0 = full vocabulary
 
     def replace(self, **kw) -> "Config":
         return dataclasses.replace(self, **kw)
