@@ -20,11 +20,15 @@
  *   z[v]  = (Dlog[d-1][v] + E[v] . h) / T'   (T' = T if T > 0, else 1)
  *   log q~[v] = min(z[v] - logsumexp_v z, 0)
  * The LM head is tied to the embedding table E.  The candidate set is the
- * whole vocabulary ("Full" in Appendix D); each node keeps its top-k
- * children by (log q~ desc, token asc), and S_d is the top-W of those
- * candidates by (score desc, parent slot asc, rank asc).  For k >= W this
- * equals the top-W over all children.  Candidates of score -inf are never
- * retained, so |S_d| <= min(W, |S_{d-1}| * k).
+ * whole vocabulary ("Full" in Appendix D) when cand_k = 0, or, as in
+ * Algorithm 1 with K = cand_k (the paper's default K = 64, Sec. 4.1), the
+ * set C_d = TopK(L_d^base, K) of the K largest drafter logits of position d
+ * (ties: token asc), shared by every node of the depth; then v runs over
+ * C_d only and q~ is renormalised over C_d (logsumexp over C_d).  Each node
+ * keeps its top-k children by (log q~ desc, token asc), and S_d is the top-W
+ * of those candidates by (score desc, parent slot asc, rank asc).  For
+ * k >= W this equals the top-W over all children.  Candidates of score -inf
+ * are never retained, so |S_d| <= min(W, |S_{d-1}| * k).
  *
  * Node ids: id = (depth-1)*W + rank within S_depth; ancestors always have
  * smaller ids.  Pruning keeps the top-B by (score desc, id asc).  Emission
@@ -73,11 +77,14 @@ typedef enum { DART_F32 = 0, DART_BF16 = 1 } dart_dtype;
  *   temperature  T >= 0; T > 0 divides the logits by T, T = 0 is greedy
  *          scoring (no scaling)
  *   rms_eps      RMSNorm epsilon (> 0)
- *   pos_offset   position id of the root; a node at depth d gets pos_offset+d */
+ *   pos_offset   position id of the root; a node at depth d gets pos_offset+d
+ *   cand_k K of Algorithm 1: 0 scores every node over the full vocabulary;
+ *          k <= cand_k <= min(V, 1024) scores it over C_d only */
 typedef struct {
     int V, d, L, W, k, B, nseq;
     float beta, temperature, rms_eps;
     int pos_offset;
+    int cand_k;
 } dart_config;
 
 /* Emitted verification tree, caller-allocated, per sequence s:
@@ -114,7 +121,9 @@ int dart_init_head(dart_handle **out, const dart_config *cfg, int wdtype,
 /* Algorithm 1, one iteration: expands depth `depth` (1..L, in order; depth 1
  * restarts the round).  drafter_logits [nseq][L][V] float32 (row depth-1 is
  * read, 4-byte aligned), anchor_h [nseq][d] float32 = r_0 (16-byte aligned;
- * read at depth 1 only, may be NULL afterwards).  Out of order -> DART_ERR_STATE. */
+ * read at depth 1 only, may be NULL afterwards).  With cand_k > 0 the
+ * candidate sets C_d of all L positions are taken at depth 1 from that
+ * call's drafter_logits.  Out of order -> DART_ERR_STATE. */
 int dart_expand_depth(dart_handle *h, int depth, const float *drafter_logits,
                       const float *anchor_h, void *stream);
 
@@ -169,8 +178,10 @@ int dart_profile_read(dart_handle *h, float *lmhead_ms, int *lmhead_launches);
  * bracketed while profiling is enabled).  Kinds: 0 LM-head scoring,
  * 1 merge + frontier select, 2 head-input gather, 3 head GEMM W_i,
  * 4 SiLU + split, 5 head GEMM W_o, 6 residual + RMSNorm, 7 depth-1 anchor
- * preparation, 8 prune + emit.  ms[i] / launches[i] receive the summed device
- * time and count of kind i for i < nkinds (nkinds <= 9); resets the events. */
+ * preparation, 8 prune + emit, 9 candidate sets C_d (cand_k > 0, once per
+ * round), 10 candidate scoring (cand_k > 0, per depth).  ms[i] / launches[i]
+ * receive the summed device time and count of kind i for i < nkinds
+ * (nkinds <= 11); resets the events. */
 int dart_profile_read_kinds(dart_handle *h, float *ms, int *launches, int nkinds);
 
 /* Number of kernel launches one dart_build_tree enqueues for this handle. */
@@ -189,7 +200,8 @@ int dart_launches_per_round(dart_handle *h);
  *   (rank order, unused ranks -1 / -inf), front_count [nseq].
  * Its scratch is one static 16 MiB device array that every GPU loading this
  * library keeps until the process exits.  Limits beyond dart_init_head's:
- * nseq <= 64, d <= 8192; larger problems return DART_ERR_INVALID before any
+ * nseq <= 64, d <= 8192, full-vocabulary scoring only (cand_k = 0); other
+ * problems return DART_ERR_INVALID before any
  * work is enqueued.  The first call on a device looks up the array's device
  * address (cudaGetSymbolAddress) and sets kernel attributes, so make that
  * first call before any stream capture.  Every call on a device shares the

@@ -26,6 +26,7 @@ namespace {
 constexpr int kVersion = 1;
 constexpr int kMaxW = 64, kMaxK = 64, kMaxWK = 4096, kMaxSuper = 1024, kMaxB = 1024;
 constexpr int kMaxD = 16384;
+constexpr int kMaxCandK = 1024;  // candidate-set size K of the restricted scoring
 constexpr int kMaxV = (1 << 24) - 1;
 constexpr int kMaxProfilePairs = 8192;
 
@@ -66,6 +67,7 @@ int ng_index(int NG) { return NG == 16 ? 0 : (NG == 32 ? 1 : 2); }
 
 struct DepthPlan {
     int N, P, NG, G, nV, stages, smem;  // LM-head scoring
+    int nlist, klist;                    // sorted key lists per node and their length (merge input)
     int Nc, Pn;                          // children (head update) at this depth
     GemmArgs g1, g2;                     // head GEMMs (depth < L)
     int g1_smem, g2_smem;
@@ -101,6 +103,7 @@ struct dart_handle {
     float* tree_score;
     int *child_prow, *child_tok, *seq_ticket, *status;
     uint64_t* gthr;  // [L][kNPadMax] cross-CTA top-k bounds of every depth, zeroed per round
+    int* cand_tok;   // [nseq][L][cand_k] candidate sets C_d (cand_k > 0)
     std::vector<void*> allocs;
     CUtensorMap tmE, tmWi, tmWo, tmH[3], tmX[3], tmA[3];
     // host-buffer staging
@@ -142,6 +145,7 @@ int validate_cfg(const dart_config* c) {
     if (!(c->beta <= 0.0f) || !std::isfinite(c->beta)) return DART_ERR_INVALID;  // Lemma 1 needs beta <= 0
     if (!(c->temperature >= 0.0f) || !std::isfinite(c->temperature)) return DART_ERR_INVALID;
     if (!(c->rms_eps > 0.0f) || !std::isfinite(c->rms_eps)) return DART_ERR_INVALID;
+    if (c->cand_k != 0 && (c->cand_k < c->k || c->cand_k > c->V || c->cand_k > kMaxCandK)) return DART_ERR_INVALID;
     return DART_OK;
 }
 
@@ -217,6 +221,8 @@ int build_plans(dart_handle* h) {
             p.smem = lmhead_f32_smem(p.NG, c.k);
             if (p.smem > h->smem_optin) return DART_ERR_UNSUPPORTED;
         }
+        p.nlist = c.cand_k > 0 ? c.cand_k : p.nV;  // one single-key list per candidate of C_d
+        p.klist = c.cand_k > 0 ? 1 : c.k;
         p.Pn = h->caps[dep];
         p.Nc = c.nseq * p.Pn;
         if (dep < c.L) {
@@ -284,11 +290,11 @@ int alloc_workspace(dart_handle* h) {
     const dart_config& c = h->cfg;
     const size_t d = c.d;
     int rc = DART_OK;
-    size_t max_nvn = 1;
-    int max_nV = 1;
+    size_t max_nvn = 1, max_keys = 1;  // key lists x nodes; keys incl. one padding key per node
     for (int dep = 1; dep <= c.L; dep++) {
-        max_nvn = std::max(max_nvn, static_cast<size_t>(h->plans[dep].nV) * h->plans[dep].N);
-        max_nV = std::max(max_nV, h->plans[dep].nV);
+        const DepthPlan& p = h->plans[dep];
+        max_nvn = std::max(max_nvn, static_cast<size_t>(p.nlist) * p.N);
+        max_keys = std::max(max_keys, (static_cast<size_t>(p.nlist) * p.klist + 1) * p.N);
     }
     const size_t super = static_cast<size_t>(c.nseq) * c.L * c.W;
 #define DART_ALLOC(ptr, n) \
@@ -305,7 +311,7 @@ int alloc_workspace(dart_handle* h) {
     }
     DART_ALLOC(h->part, max_part_floats(h))
     DART_ALLOC(h->part_ms, max_nvn)
-    DART_ALLOC(h->part_key, max_nvn * c.k + kNPadMax)  // + one padding key per node (part_stride)
+    DART_ALLOC(h->part_key, max_keys)  // part_stride(nlist, klist) keys per node
     DART_ALLOC(h->node_logq, static_cast<size_t>(kNPadMax) * c.k)
     DART_ALLOC(h->node_tok, static_cast<size_t>(kNPadMax) * c.k)
     DART_ALLOC(h->node_lse, kNPadMax)
@@ -318,6 +324,7 @@ int alloc_workspace(dart_handle* h) {
     DART_ALLOC(h->seq_ticket, c.nseq)
     DART_ALLOC(h->status, 1)
     DART_ALLOC(h->gthr, static_cast<size_t>(c.L) * kNPadMax)
+    if (c.cand_k > 0) DART_ALLOC(h->cand_tok, static_cast<size_t>(c.nseq) * c.L * c.cand_k)
 #undef DART_ALLOC
     if (rc != DART_OK) return rc;
     // zeroed once: stale rows of the operand buffers are always finite
@@ -336,14 +343,16 @@ int alloc_workspace(dart_handle* h) {
     if (cudaMemset(h->tree_count, 0, c.nseq * c.L * sizeof(int)) != cudaSuccess) return DART_ERR_CUDA;
     // one-time kernel attributes
     int max_sel = 0;
-    for (int dep = 1; dep <= c.L; dep++) max_sel = std::max(max_sel, merge_select_smem(h->plans[dep].nV, c.k, c.W));
+    for (int dep = 1; dep <= c.L; dep++)
+        max_sel = std::max(max_sel, merge_select_smem(h->plans[dep].nlist, h->plans[dep].klist, c.k, c.W));
+    if (max_sel > h->smem_optin) return DART_ERR_UNSUPPORTED;
     if (select_set_smem_limits(std::max(max_sel, 48 * 1024)) != cudaSuccess) return DART_ERR_CUDA;
+    if (c.cand_k > 0 && cand_set_smem_limits(cand_topk_smem(c.cand_k)) != cudaSuccess) return DART_ERR_CUDA;
     if (h->wdtype == DART_BF16) {
         if (tc_set_smem_limits(h->smem_optin) != cudaSuccess) return DART_ERR_CUDA;
     } else {
         if (f32_set_smem_limits(h->smem_optin) != cudaSuccess) return DART_ERR_CUDA;
     }
-    (void)max_nV;
     return DART_OK;
 }
 
@@ -374,7 +383,7 @@ void release(dart_handle* h) {
 
 // ---------------------------------------------------------------- enqueue
 
-enum Kind { kLmhead = 0, kSelect, kGather, kGemm1, kSilu, kGemm2, kNorm, kPrep, kEmit, kNumKinds };
+enum Kind { kLmhead = 0, kSelect, kGather, kGemm1, kSilu, kGemm2, kNorm, kPrep, kEmit, kCandTopk, kCandScore, kNumKinds };
 
 // Opens an event pair around the next launch when profiling (no-op otherwise).
 int prof_begin(dart_handle* h, int kind, cudaStream_t st) {
@@ -408,6 +417,13 @@ int enqueue_depth(dart_handle* h, int dep, const float* dlog, const float* ancho
         prof_end(h, pi, st);
         if (e != cudaSuccess) return DART_ERR_CUDA;
         h->cur = 0;
+        if (c.cand_k > 0) {
+            // C_d = TopK(L_d^base, K) of every position of every sequence
+            const int pc = prof_begin(h, kCandTopk, st);
+            e = launch_cand_topk(dlog, c.nseq * c.L, c.V, c.cand_k, h->cand_tok, st);
+            prof_end(h, pc, st);
+            if (e != cudaSuccess) return DART_ERR_CUDA;
+        }
     }
     // 1) LM-head scoring of every prefix in S_{dep-1} (fused log-sum-exp / top-k)
     LmheadArgs la;
@@ -433,8 +449,33 @@ int enqueue_depth(dart_handle* h, int dep, const float* dlog, const float* ancho
     la.h32 = h->hbuf[h->cur];
     la.E32 = static_cast<const float*>(h->E);
     la.gthr = h->gthr + static_cast<size_t>(dep - 1) * kNPadMax;
-    int pi = prof_begin(h, kLmhead, st);
-    e = tc ? launch_lmhead_tc(&h->tmE, &h->tmH[ng_index(p.NG)], la, p.smem, st) : launch_lmhead_f32(la, st);
+    int pi;
+    if (c.cand_k > 0) {
+        // candidate-restricted scoring: every node against its sequence's C_d
+        CandArgs ca;
+        std::memset(&ca, 0, sizeof ca);
+        ca.K = c.cand_k;
+        ca.P = p.P;
+        ca.d = c.d;
+        ca.L = c.L;
+        ca.dep = dep;
+        ca.nseq = c.nseq;
+        ca.wbf16 = tc ? 1 : 0;
+        ca.invT = la.invT;
+        ca.cand_tok = h->cand_tok;
+        ca.dlog = dlog;
+        ca.dlog_seq_stride = la.dlog_seq_stride;
+        ca.dlog_row_off = la.dlog_row_off;
+        ca.h = h->hbuf[h->cur];
+        ca.E = h->E;
+        ca.part_ms = h->part_ms;
+        ca.part_key = h->part_key;
+        pi = prof_begin(h, kCandScore, st);
+        e = launch_cand_score(ca, st);
+    } else {
+        pi = prof_begin(h, kLmhead, st);
+        e = tc ? launch_lmhead_tc(&h->tmE, &h->tmH[ng_index(p.NG)], la, p.smem, st) : launch_lmhead_f32(la, st);
+    }
     prof_end(h, pi, st);
     if (e != cudaSuccess) return DART_ERR_CUDA;
     // 2) merge partials, log q~, Eq. 5 scores, global top-W -> S_dep
@@ -443,7 +484,8 @@ int enqueue_depth(dart_handle* h, int dep, const float* dlog, const float* ancho
     sa.N = p.N;
     sa.P = p.P;
     sa.k = c.k;
-    sa.nV = p.nV;
+    sa.nV = p.nlist;
+    sa.klist = p.klist;
     sa.W = c.W;
     sa.L = c.L;
     sa.nseq = c.nseq;
@@ -452,7 +494,7 @@ int enqueue_depth(dart_handle* h, int dep, const float* dlog, const float* ancho
     sa.beta = c.beta;
     sa.part_ms = h->part_ms;
     sa.part_key = h->part_key;
-    sa.gthr = la.gthr;
+    sa.gthr = c.cand_k > 0 ? nullptr : la.gthr;
     sa.node_logq = h->node_logq;
     sa.node_tok = h->node_tok;
     sa.node_lse = h->node_lse;
@@ -838,7 +880,7 @@ int dart_launches_per_round(dart_handle* h) {
     const int L = h->cfg.L;
     // prep, (LM-head + select) per depth, (gather, W_i GEMM, [SiLU,] W_o GEMM,
     // residual-norm) per depth but the last, prune-emit
-    int n = 1 + 2 * L + 1;
+    int n = 1 + 2 * L + 1 + (h->cfg.cand_k > 0 ? 1 : 0);
     for (int dep = 1; dep < L; dep++) n += (h->wdtype == DART_BF16 && h->plans[dep].g1.mode != kGemmPartials) ? 4 : 5;
     return n;
 }

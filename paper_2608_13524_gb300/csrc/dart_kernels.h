@@ -117,7 +117,9 @@ cudaError_t f32_set_smem_limits(int max_dyn);
 
 // selection / emission / elementwise kernels (dart_select.cu)
 struct SelectArgs {
-    int N, P, k, nV, W, L, nseq, dep, Pn;  // Pn = max |S_dep| (child slots per sequence)
+    // nV sorted key lists of klist keys per node (LM-head CTAs, or one key
+    // per candidate of C_d); Pn = max |S_dep| (child slots per sequence)
+    int N, P, k, nV, klist, W, L, nseq, dep, Pn;
     float beta;
     const float2* part_ms;
     const uint64_t* part_key;
@@ -135,8 +137,26 @@ struct SelectArgs {
     int* status;
 };
 cudaError_t launch_merge_select(const SelectArgs& a, cudaStream_t st);
-int merge_select_smem(int nV, int k, int W);
+int merge_select_smem(int nV, int klist, int k, int W);
 cudaError_t select_set_smem_limits(int max_dyn);
+
+// candidate-restricted scoring (dart_cand.cu)
+struct CandArgs {
+    int K, P, d, L, dep, nseq, wbf16;
+    float invT;
+    const int* cand_tok;        // [nseq][L][K] C_d of every position, ascending tokens
+    const float* dlog;          // [nseq][L][V]
+    long long dlog_seq_stride;  // L * V
+    long long dlog_row_off;     // (dep-1) * V
+    const float* h;             // [nseq*P][d] fp32 states of S_{dep-1}
+    const void* E;              // [V][d] bf16 or fp32
+    float2* part_ms;            // [nseq*P][K]  (z, 1)
+    uint64_t* part_key;         // [nseq*P][part_stride(K, 1)]  key(z, token)
+};
+cudaError_t launch_cand_topk(const float* dlog, int rows, int V, int K, int* cand_tok, cudaStream_t st);
+cudaError_t launch_cand_score(const CandArgs& a, cudaStream_t st);
+int cand_topk_smem(int K);
+cudaError_t cand_set_smem_limits(int max_dyn);
 
 struct EmitArgs {
     int L, W, B, nseq, pos_offset;

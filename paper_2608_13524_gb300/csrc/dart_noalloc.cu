@@ -120,6 +120,7 @@ extern "C" int dart_expand_root_noalloc(const dart_config* cfg, const void* E, c
         !std::isfinite(c.temperature))
         return DART_ERR_INVALID;
     if (c.nseq > kMaxSeqNoAlloc || c.d > kMaxDNoAlloc) return DART_ERR_INVALID;
+    if (c.cand_k != 0) return DART_ERR_INVALID;  // full-vocabulary scoring only
     if ((reinterpret_cast<uintptr_t>(E) & 15u) || (reinterpret_cast<uintptr_t>(drafter_logits) & 3u) ||
         (reinterpret_cast<uintptr_t>(anchor_h) & 15u))
         return DART_ERR_INVALID;
@@ -212,6 +213,7 @@ extern "C" int dart_expand_root_noalloc(const dart_config* cfg, const void* E, c
     sa.P = 1;
     sa.k = c.k;
     sa.nV = nV;
+    sa.klist = c.k;
     sa.W = c.W;
     sa.L = 1;
     sa.nseq = N;

@@ -131,18 +131,18 @@ __global__ void __launch_bounds__(kSelThreads) merge_select_kernel(const SelectA
     __shared__ float redm[32];
     __shared__ int redi[32];
     __shared__ int ticket;
-    const int cap = max(a.nV * a.k, a.W * a.k);
+    const int cap = max(a.nV * a.klist, a.W * a.k);
     uint64_t* surv = keys + cap;
     uint64_t* top = surv + kRankMax;
     int* ctok = reinterpret_cast<int*>(top + 64);
 
     const int n = blockIdx.x, tid = threadIdx.x;
     const int s = n / a.P, p = n % a.P;
-    // this node's partials are contiguous: part_ms[n][nV], part_key[n][nV][k];
+    // this node's partials are contiguous: part_ms[n][nV], part_key[n][nV][klist];
     // they are loaded before the frontier size is known (rows past it hold
     // stale but harmless data)
-    const int nk = a.nV * a.k;
-    const uint64_t* blk = a.part_key + static_cast<size_t>(n) * part_stride(a.nV, a.k);  // 16-byte aligned
+    const int nk = a.nV * a.klist;
+    const uint64_t* blk = a.part_key + static_cast<size_t>(n) * part_stride(a.nV, a.klist);  // 16-byte aligned
     const uint4* src = reinterpret_cast<const uint4*>(blk);
     const int prev_count = a.dep == 1 ? 1 : __ldcg(a.tree_count + s * a.L + a.dep - 2);
     const uint64_t bound = a.gthr ? __ldcg(reinterpret_cast<const unsigned long long*>(a.gthr) + n) : 0ull;
@@ -188,7 +188,7 @@ __global__ void __launch_bounds__(kSelThreads) merge_select_kernel(const SelectA
         const float ssum = block_sum_float(part, redf);
         const float lse = gm == -INFINITY ? -INFINITY : gm + logf(ssum);
         // top-k over every CTA's (sorted) top-k list
-        topk_of_sorted_lists(keys, a.nV, a.k, a.k, bound, top, surv, &thr, hist, scal);
+        topk_of_sorted_lists(keys, a.nV, a.klist, a.k, bound, top, surv, &thr, hist, scal);
         for (int j = tid; j < a.k; j += kSelThreads) {
             const uint64_t x = top[j];
             const float z = key_val(x);
@@ -507,14 +507,16 @@ bool pdl_enabled() {
     return on;
 }
 
-int merge_select_smem(int nV, int k, int W) { return (max(nV * k, W * k) + kRankMax + 64) * 8 + W * k * 4; }
+int merge_select_smem(int nV, int klist, int k, int W) {
+    return (max(nV * klist, W * k) + kRankMax + 64) * 8 + W * k * 4;
+}
 
 cudaError_t select_set_smem_limits(int max_dyn) {
     return cudaFuncSetAttribute(merge_select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, max_dyn);
 }
 
 cudaError_t launch_merge_select(const SelectArgs& a, cudaStream_t st) {
-    const int smem = merge_select_smem(a.nV, a.k, a.W);
+    const int smem = merge_select_smem(a.nV, a.klist, a.k, a.W);
     return launch_pdl(merge_select_kernel, dim3(a.N), dim3(kSelThreads), smem, st, a);
 }
 

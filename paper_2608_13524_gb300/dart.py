@@ -29,7 +29,8 @@ DART_BF16 = 1
 class DartConfig(C.Structure):
     _fields_ = [("V", C.c_int), ("d", C.c_int), ("L", C.c_int), ("W", C.c_int), ("k", C.c_int),
                 ("B", C.c_int), ("nseq", C.c_int), ("beta", C.c_float),
-                ("temperature", C.c_float), ("rms_eps", C.c_float), ("pos_offset", C.c_int)]
+                ("temperature", C.c_float), ("rms_eps", C.c_float), ("pos_offset", C.c_int),
+                ("cand_k", C.c_int)]
 
 
 class DartTreeOut(C.Structure):
@@ -103,10 +104,10 @@ def _stream(stream):
 
 def make_config(cfg) -> DartConfig:
     """From any object with V, d, L, W, k, B, nseq, beta, temperature,
-    rms_eps, pos_offset."""
+    rms_eps, pos_offset and optionally cand_k (0: full vocabulary)."""
     return DartConfig(int(cfg.V), int(cfg.d), int(cfg.L), int(cfg.W), int(cfg.k), int(cfg.B),
                       int(cfg.nseq), float(cfg.beta), float(cfg.temperature), float(cfg.rms_eps),
-                      int(cfg.pos_offset))
+                      int(cfg.pos_offset), int(getattr(cfg, "cand_k", 0)))
 
 
 def alloc_tree_out(cfg, device="cuda", pin=False):
@@ -207,7 +208,7 @@ def dart_profile_read(h):
 
 
 KIND_NAMES = ("lmhead", "merge_select", "gather", "gemm_wi", "silu_split", "gemm_wo", "residual_norm",
-              "prep_anchor", "prune_emit")
+              "prep_anchor", "prune_emit", "cand_topk", "cand_score")
 
 
 def dart_profile_read_kinds(h):

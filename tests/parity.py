@@ -183,9 +183,9 @@ def validate_frontier_teacher_forced(cfg, x, gst, s, dep, tol_step, ref_logq=Non
         path = () if dep == 1 else gp[(dep - 2) * W + p]
         ps = 0.0 if dep == 1 else float(gst["st_score"][s, dep - 2, p])
         tok, lq, lse, allq = oracle.node_children(cfg, x["Wi"], x["Wo"], x["E"], x["Dlog"][s], x["h0"][s],
-                                                  np.array(path, np.int32), min(k + 1, cfg.V),
+                                                  np.array(path, np.int32), min(k + 1, oracle.cand_count(cfg)),
                                                   want_all=True)
-        for j in range(min(k + 1, cfg.V)):
+        for j in range(min(k + 1, oracle.cand_count(cfg))):
             cands.append((ps + lq[j] + cfg.beta, p, j, int(tok[j]), j < k))
         if ref_logq is not None:
             ref_logq[(s, dep, p)] = allq

@@ -41,7 +41,7 @@ def test_status_strings_and_version():
 class Cfg:
     def __init__(self, **kw):
         base = dict(V=1000, d=128, L=4, W=4, k=4, B=16, nseq=1, beta=-0.2, temperature=0.0,
-                    rms_eps=1e-6, pos_offset=0)
+                    rms_eps=1e-6, pos_offset=0, cand_k=0)
         base.update(kw)
         self.__dict__.update(base)
 
@@ -49,7 +49,7 @@ class Cfg:
 BAD = [dict(V=0), dict(d=100), dict(d=32), dict(L=0), dict(W=0), dict(W=65), dict(k=0), dict(k=65),
        dict(V=10, k=11), dict(W=64, k=65), dict(L=17, W=64), dict(B=0), dict(B=1025), dict(nseq=0),
        dict(nseq=5, W=64), dict(beta=0.1), dict(beta=float("nan")), dict(temperature=-1.0),
-       dict(rms_eps=0.0)]
+       dict(rms_eps=0.0), dict(cand_k=3), dict(cand_k=-1), dict(cand_k=1001), dict(V=5000, cand_k=1025)]
 
 
 @pytest.mark.parametrize("bad", BAD, ids=[str(b) for b in BAD])

@@ -12,7 +12,7 @@ import torch
 import oracle
 from parity import (check_structure, compare_with_oracle, gpu_supertree, to_device, tol_of, tree_to_numpy,
                     validate_frontier_teacher_forced)
-from workloads import BATCHED, Q4B, Q8B, TOY, Config, make_inputs, sweep_configs
+from workloads import BATCHED, NAMED, Q4B, Q8B, TOY, Config, make_inputs, sweep_configs
 
 pytestmark = pytest.mark.gpu
 
@@ -52,6 +52,17 @@ SMALL = [
     TOY,
 ]
 
+# candidate-restricted scoring (Algorithm 1 with K = cand_k)
+RESTRICTED = [
+    C("cand-f32", 1, 3000, 128, 4, 4, 4, 10, "f32", 0.0, 51, cand_k=64),
+    C("cand-bf16", 2, 20000, 256, 5, 8, 8, 24, "bf16", 1.0, 52, cand_k=64),
+    C("cand-bf16-N256", 8, 5000, 128, 3, 32, 32, 60, "bf16", 0.0, 53, cand_k=64),
+    C("cand-odd-K", 1, 4000, 192, 4, 6, 5, 20, "bf16", 0.7, 54, cand_k=37),
+    C("cand-K1024", 1, 9000, 128, 3, 16, 16, 40, "bf16", 0.0, 55, cand_k=1024),
+    C("cand-K=k", 2, 2500, 64, 4, 8, 8, 30, "bf16", 0.0, 56, cand_k=8),
+    C("cand-K=V", 1, 300, 64, 3, 5, 5, 12, "f32", 0.0, 57, cand_k=300),
+]
+
 
 def run_depthwise(dart, cfg, dx):
     """Expands depth by depth, collecting node lists / frontiers / states."""
@@ -75,7 +86,7 @@ def run_depthwise(dart, cfg, dx):
     return per, gst, g
 
 
-@pytest.mark.parametrize("cfg", SMALL, ids=[c.name for c in SMALL])
+@pytest.mark.parametrize("cfg", SMALL + RESTRICTED, ids=[c.name for c in SMALL + RESTRICTED])
 def test_depthwise_parity(dart, cfg):
     x = make_inputs(cfg)
     dx = to_device(cfg, x)
@@ -115,7 +126,10 @@ def test_depthwise_parity(dart, cfg):
                     assert np.max(np.abs(got - hs)) <= stol, (dep, s, r, np.max(np.abs(got - hs)))
 
 
-@pytest.mark.parametrize("cfg", SMALL[:6], ids=[c.name for c in SMALL[:6]])
+GRAPH = SMALL[:6] + RESTRICTED[:3]
+
+
+@pytest.mark.parametrize("cfg", GRAPH, ids=[c.name for c in GRAPH])
 def test_build_tree_graph_matches_depthwise(dart, cfg):
     """dart_build_tree (one cached CUDA graph) equals the depth-by-depth
     calls, is deterministic across repeated launches, and the host-buffer
@@ -155,6 +169,23 @@ def test_neg_inf_drafter_logits(dart):
     assert int(gst["st_count"][1, 0]) == 1
 
 
+def test_restricted_candidates_and_neg_inf(dart):
+    """Restricted scoring with -inf drafter logits: C_d still holds K tokens
+    (the -inf ones by token id), their children have probability zero and are
+    never retained."""
+    cfg = C("cand-neginf", 2, 700, 128, 4, 6, 4, 40, "bf16", 0.0, 58, cand_k=16)
+    x = make_inputs(cfg)
+    x["Dlog"][0, 1, 3:] = -np.inf      # depth 2 of seq 0: only tokens 0..2 possible
+    x["Dlog"][1, 0, :] = -np.inf       # depth 1 of seq 1: no child at all
+    x["Dlog"][1, 0, 5] = 0.0           #   ... except token 5
+    dx = to_device(cfg, x)
+    ref = oracle.build_tree(cfg, x["Wi"], x["Wo"], x["E"], x["Dlog"], x["h0"])
+    _, gst, g = run_depthwise(dart, cfg, dx)
+    compare_with_oracle(cfg, ref, gst, g, tol_of(cfg))
+    assert int(gst["st_count"][1, 0]) == 1
+    assert int(gst["st_tok"][1, 0, 0]) == 5
+
+
 def test_call_order_and_argument_errors(dart):
     cfg = C("err", 1, 500, 64, 3, 2, 2, 4, "bf16", 0.0, 41)
     x = make_inputs(cfg)
@@ -186,7 +217,8 @@ def test_call_order_and_argument_errors(dart):
 
 # ----------------------------------------------------------------- full size
 
-FULL = [Q8B, Q4B, BATCHED, [c for c in sweep_configs() if c.W == 64 and c.B == 512][0]]
+FULL = [Q8B, Q4B, BATCHED, [c for c in sweep_configs() if c.W == 64 and c.B == 512][0],
+        NAMED["qwen3-8b-k64"], NAMED["batched-k64"]]
 
 
 @pytest.mark.parametrize("cfg", FULL, ids=[c.name for c in FULL])

@@ -96,8 +96,13 @@ def sweep_configs():
     return out
 
 
+# The same shapes and inputs with Algorithm 1's candidate restriction at the
+# paper's default K = 64 (Sec. 4.1).
+RESTRICTED = [Q8B.replace(name="qwen3-8b-k64", cand_k=64), Q4B.replace(name="qwen3-4b-k64", cand_k=64),
+              BATCHED.replace(name="batched-k64", cand_k=64)]
+
 NAMED = {c.name: c for c in (TOY, Q4B, Q8B, BATCHED)}
-for _c in sweep_configs():
+for _c in sweep_configs() + RESTRICTED:
     NAMED[_c.name] = _c
 
 
