@@ -68,6 +68,7 @@ int ng_index(int NG) { return NG == 16 ? 0 : (NG == 32 ? 1 : 2); }
 struct DepthPlan {
     int N, P, NG, G, nV, stages, smem;  // LM-head scoring
     int nlist, klist;                    // sorted key lists per node and their length (merge input)
+    int cand_ds;                         // candidate scoring: d slices per candidate group
     int Nc, Pn;                          // children (head update) at this depth
     GemmArgs g1, g2;                     // head GEMMs (depth < L)
     int g1_smem, g2_smem;
@@ -104,6 +105,8 @@ struct dart_handle {
     int *child_prow, *child_tok, *seq_ticket, *status;
     uint64_t* gthr;  // [L][kNPadMax] cross-CTA top-k bounds of every depth, zeroed per round
     int* cand_tok;   // [nseq][L][cand_k] candidate sets C_d (cand_k > 0)
+    float* cand_scratch;  // candidate scoring partial dot products
+    int* cand_ticket;     // [nseq][ceil(cand_k/8)]
     std::vector<void*> allocs;
     CUtensorMap tmE, tmWi, tmWo, tmH[3], tmX[3], tmA[3];
     // host-buffer staging
@@ -223,6 +226,11 @@ int build_plans(dart_handle* h) {
         }
         p.nlist = c.cand_k > 0 ? c.cand_k : p.nV;  // one single-key list per candidate of C_d
         p.klist = c.cand_k > 0 ? 1 : c.k;
+        p.cand_ds = 0;
+        if (c.cand_k > 0) {
+            p.cand_ds = cand_score_slices(p.P, c.d, c.nseq, c.cand_k, h->smem_optin);
+            if (p.cand_ds == 0) return DART_ERR_UNSUPPORTED;
+        }
         p.Pn = h->caps[dep];
         p.Nc = c.nseq * p.Pn;
         if (dep < c.L) {
@@ -324,7 +332,14 @@ int alloc_workspace(dart_handle* h) {
     DART_ALLOC(h->seq_ticket, c.nseq)
     DART_ALLOC(h->status, 1)
     DART_ALLOC(h->gthr, static_cast<size_t>(c.L) * kNPadMax)
-    if (c.cand_k > 0) DART_ALLOC(h->cand_tok, static_cast<size_t>(c.nseq) * c.L * c.cand_k)
+    if (c.cand_k > 0) {
+        size_t scr = 1;
+        for (int dep = 1; dep <= c.L; dep++)
+            scr = std::max(scr, static_cast<size_t>(h->plans[dep].cand_ds) * h->plans[dep].N * c.cand_k);
+        DART_ALLOC(h->cand_tok, static_cast<size_t>(c.nseq) * c.L * c.cand_k)
+        DART_ALLOC(h->cand_scratch, scr)
+        DART_ALLOC(h->cand_ticket, static_cast<size_t>(c.nseq) * ((c.cand_k + 7) / 8))
+    }
 #undef DART_ALLOC
     if (rc != DART_OK) return rc;
     // zeroed once: stale rows of the operand buffers are always finite
@@ -347,7 +362,15 @@ int alloc_workspace(dart_handle* h) {
         max_sel = std::max(max_sel, merge_select_smem(h->plans[dep].nlist, h->plans[dep].klist, c.k, c.W));
     if (max_sel > h->smem_optin) return DART_ERR_UNSUPPORTED;
     if (select_set_smem_limits(std::max(max_sel, 48 * 1024)) != cudaSuccess) return DART_ERR_CUDA;
-    if (c.cand_k > 0 && cand_set_smem_limits(cand_topk_smem(c.cand_k)) != cudaSuccess) return DART_ERR_CUDA;
+    if (c.cand_k > 0) {
+        int score_smem = 48 * 1024;
+        for (int dep = 1; dep <= c.L; dep++)
+            score_smem = std::max(score_smem, cand_score_smem(h->plans[dep].P, c.d, h->plans[dep].cand_ds));
+        if (cudaMemset(h->cand_ticket, 0, c.nseq * ((c.cand_k + 7) / 8) * sizeof(int)) != cudaSuccess)
+            return DART_ERR_CUDA;
+        if (cand_set_smem_limits(std::max(cand_topk_smem(c.cand_k), 48 * 1024), score_smem) != cudaSuccess)
+            return DART_ERR_CUDA;
+    }
     if (h->wdtype == DART_BF16) {
         if (tc_set_smem_limits(h->smem_optin) != cudaSuccess) return DART_ERR_CUDA;
     } else {
@@ -461,6 +484,7 @@ int enqueue_depth(dart_handle* h, int dep, const float* dlog, const float* ancho
         ca.dep = dep;
         ca.nseq = c.nseq;
         ca.wbf16 = tc ? 1 : 0;
+        ca.V = c.V;
         ca.invT = la.invT;
         ca.cand_tok = h->cand_tok;
         ca.dlog = dlog;
@@ -470,6 +494,9 @@ int enqueue_depth(dart_handle* h, int dep, const float* dlog, const float* ancho
         ca.E = h->E;
         ca.part_ms = h->part_ms;
         ca.part_key = h->part_key;
+        ca.DS = p.cand_ds;
+        ca.scratch = h->cand_scratch;
+        ca.ticket = h->cand_ticket;
         pi = prof_begin(h, kCandScore, st);
         e = launch_cand_score(ca, st);
     } else {

@@ -142,7 +142,7 @@ cudaError_t select_set_smem_limits(int max_dyn);
 
 // candidate-restricted scoring (dart_cand.cu)
 struct CandArgs {
-    int K, P, d, L, dep, nseq, wbf16;
+    int K, P, d, L, dep, nseq, wbf16, V;
     float invT;
     const int* cand_tok;        // [nseq][L][K] C_d of every position, ascending tokens
     const float* dlog;          // [nseq][L][V]
@@ -152,11 +152,16 @@ struct CandArgs {
     const void* E;              // [V][d] bf16 or fp32
     float2* part_ms;            // [nseq*P][K]  (z, 1)
     uint64_t* part_key;         // [nseq*P][part_stride(K, 1)]  key(z, token)
+    int DS;                     // d slices (blocks per candidate group), see cand_score_slices
+    float* scratch;             // [DS][nseq*P][K] partial dot products
+    int* ticket;                // [nseq][ceil(K/8)] zero between launches
 };
 cudaError_t launch_cand_topk(const float* dlog, int rows, int V, int K, int* cand_tok, cudaStream_t st);
 cudaError_t launch_cand_score(const CandArgs& a, cudaStream_t st);
 int cand_topk_smem(int K);
-cudaError_t cand_set_smem_limits(int max_dyn);
+int cand_score_slices(int P, int d, int nseq, int K, int max_smem);  // 0: does not fit
+int cand_score_smem(int P, int d, int DS);
+cudaError_t cand_set_smem_limits(int topk_smem, int score_smem);
 
 struct EmitArgs {
     int L, W, B, nseq, pos_offset;

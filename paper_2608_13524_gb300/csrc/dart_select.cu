@@ -48,77 +48,6 @@ __device__ __forceinline__ float block_sum_float(float v, float* red) {
     return t;
 }
 
-constexpr int kRankMax = 1024;  // candidate count up to which an O(n^2 / threads) rank sort is used
-
-// Writes the kk largest nonzero keys, in descending order, to out[0..kk).
-// `keys` holds nlists lists of `len` keys, each sorted in descending order
-// with zeros (empty slots) last; at least kk keys are nonzero.  Only keys
-// >= a threshold T can be among the kk largest, where T is the larger of
-// `bound` (0, or a key known to have kk keys >= it, such as the largest
-// k-th key any LM-head CTA published for the node) and the kk-th largest
-// list head (some kk lists reach it); the survivors are ranked by counting.
-// A block-wide radix select handles a survivor set larger than kRankMax.
-// `surv` has kRankMax slots.  Every thread of the block must call this.
-__device__ __forceinline__ void topk_of_sorted_lists(const uint64_t* keys, int nlists, int len, int kk,
-                                                     uint64_t bound, uint64_t* out, uint64_t* surv, uint64_t* thr,
-                                                     uint32_t* hist, int* scal) {
-    const int tid = threadIdx.x, nt = blockDim.x;
-    const int n = nlists * len;
-    if (tid == 0) {
-        *thr = 0ull;
-        scal[2] = 0;
-    }
-    __syncthreads();
-    if (nlists >= kk && nlists > 1) {
-        for (int r = tid; r < nlists; r += nt) {
-            const uint64_t h = keys[r * len];
-            if (h == 0ull) continue;
-            int rank = 0;
-            int q = 0;
-            for (; q + 8 <= nlists; q += 8) {
-#pragma unroll
-                for (int u = 0; u < 8; u++) rank += keys[(q + u) * len] > h;
-            }
-            for (; q < nlists; q++) rank += keys[q * len] > h;
-            if (rank == kk - 1) *thr = h;
-        }
-        __syncthreads();
-    }
-    const uint64_t T = *thr > bound ? *thr : bound;
-    for (int i = tid; i < n; i += nt) {
-        const uint64_t x = keys[i];
-        if (x != 0ull && x >= T) {
-            const int pos = atomicAdd(&scal[2], 1);
-            if (pos < kRankMax) surv[pos] = x;
-        }
-    }
-    __syncthreads();
-    const int m = scal[2];
-    if (m > kRankMax) {
-        const uint64_t kth = block_kth_largest(keys, n, kk, hist, scal);
-        if (tid == 0) scal[2] = 0;
-        __syncthreads();
-        for (int i = tid; i < n; i += nt) {
-            const uint64_t x = keys[i];
-            if (x != 0ull && x >= kth) surv[atomicAdd(&scal[2], 1)] = x;
-        }
-        __syncthreads();
-    }
-    const int mm = m > kRankMax ? kk : m;
-    for (int i = tid; i < mm; i += nt) {
-        const uint64_t x = surv[i];
-        int r = 0;
-        int j = 0;
-        for (; j + 8 <= mm; j += 8) {
-#pragma unroll
-            for (int u = 0; u < 8; u++) r += surv[j + u] > x;
-        }
-        for (; j < mm; j++) r += surv[j] > x;
-        if (r < kk) out[r] = x;
-    }
-    __syncthreads();
-}
-
 __global__ void __launch_bounds__(kSelThreads) merge_select_kernel(const SelectArgs a) {
     pdl_trigger();
     pdl_wait();
