@@ -63,7 +63,7 @@ bool encode_bf16_2d(CUtensorMap* m, const void* base, uint64_t inner, uint64_t r
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 bool aligned4(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 3u) == 0; }
 
-int ng_index(int NG) { return NG == 16 ? 0 : (NG == 32 ? 1 : 2); }
+int ng_index(int NG) { return NG == 16 ? 0 : (NG == 32 ? 1 : (NG == 64 ? 2 : 3)); }
 
 struct DepthPlan {
     int N, P, NG, G, nV, stages, smem;  // LM-head scoring
@@ -108,7 +108,7 @@ struct dart_handle {
     float* cand_scratch;  // candidate scoring partial dot products
     int* cand_ticket;     // [nseq][ceil(cand_k/8)]
     std::vector<void*> allocs;
-    CUtensorMap tmE, tmWi, tmWo, tmH[3], tmX[3], tmA[3];
+    CUtensorMap tmE, tmWi, tmWo, tmH[4], tmX[3], tmA[3];
     // host-buffer staging
     float *st_dlog, *st_anchor;
     dart_tree_out st_out;
@@ -152,7 +152,10 @@ int validate_cfg(const dart_config* c) {
     return DART_OK;
 }
 
-int pick_ng_tc(int N) { return N <= 16 ? 16 : (N <= 32 ? 32 : 64); }
+// Node group of the LM-head kernel (up to 128: one MMA of N = 256 covers the
+// hi and lo products of 128 nodes) and of the head GEMMs (up to 64).
+int pick_ng_tc(int N) { return N <= 16 ? 16 : (N <= 32 ? 32 : (N <= 64 ? 64 : 128)); }
+int pick_ng_gemm(int N) { return N <= 16 ? 16 : (N <= 32 ? 32 : 64); }
 int pick_ng_f32(int N) { return N <= 16 ? 16 : 32; }
 
 // Split-K GEMM plan: M = d output features, K reduction, Nc nodes.
@@ -167,7 +170,7 @@ GemmArgs gemm_plan(const dart_handle* h, int K, int Nc, int lo_kb_end, bool tc) 
     g.lo_kb_end = lo_kb_end;
     g.bhalf = kNPadMax;
     if (tc) {
-        g.NG = pick_ng_tc(Nc);
+        g.NG = pick_ng_gemm(Nc);
         g.G = (Nc + g.NG - 1) / g.NG;
         g.MT = (d + kTileM - 1) / kTileM;
         g.S = std::max(1, std::min(g.KB, h->num_sms / (g.MT * g.G)));
@@ -211,7 +214,8 @@ int build_plans(dart_handle* h) {
             const int smem2 = lmhead_tc_fixed_smem(p.NG, c.k, st2) + st2 * tc_stage_bytes(p.NG);
             const char* force = getenv("DART_LMHEAD_CTAS_PER_SM");  // tuning override: 1 or 2
             const bool want2 = force ? atoi(force) == 2 : c.d <= 3072;
-            if (want2 && st2 >= 4 && lmhead_tc_ctas_per_sm(p.NG, smem2) >= 2) {
+            if (want2 && st2 >= 4 && 2 * lmhead_tc_tmem_cols(p.NG) <= 512 &&
+                lmhead_tc_ctas_per_sm(p.NG, smem2) >= 2) {
                 p.stages = st2;
                 p.nV = std::max(1, std::min(2 * h->num_sms / p.G, tiles));
             } else {
@@ -390,6 +394,7 @@ int make_tensor_maps(dart_handle* h) {
              encode_bf16_2d(&h->tmX[i], h->XL, 2 * d, 2 * kNPadMax, ngs[i]) &&
              encode_bf16_2d(&h->tmA[i], h->AL, d, 2 * kNPadMax, ngs[i]);
     }
+    if (ok) ok = encode_bf16_2d(&h->tmH[3], h->HL, d, 2 * kNPadMax, 128);  // LM-head 128-node groups
     return ok ? DART_OK : DART_ERR_UNSUPPORTED;
 }
 

@@ -23,6 +23,7 @@ constexpr int kNPadMax = 256;       // max nodes per depth (nseq * W)
 constexpr int kTileM = 128;         // MMA M: vocabulary rows / output features per tile
 constexpr int kBlockK = 64;         // bf16 elements per 128-byte swizzled row
 constexpr int kCandCap = 128;       // per-node candidate slots per tile (one tile worth)
+constexpr int kCandCapLarge = 32;   // slots per node for 128-node groups (overflow: more merge rounds)
 constexpr int kEpiBarrier = 1;      // named barrier id used by the epilogue warps
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
@@ -410,11 +411,13 @@ constexpr float kRefSlack = 30.0f;  // exp(30) ~ 1e13: sums stay far from fp32 o
 
 struct EpiSmem {
     uint64_t* list;   // [NG][k]   sorted desc, 0 = empty
-    uint64_t* cand;   // [NG][kCandCap]
+    uint64_t* cand;   // [NG][cap]
     uint64_t* gcache; // [NG]  last seen cross-CTA bound (see epi_merge)
-    int* cnt;         // [NG]
+    int* cnt;         // [NG]  candidates offered this round (may exceed cap)
+    int* more;        // [2]   "a candidate found no free slot" flags of alternate merge rounds
     float* mref;      // [4][NG]  per-warp reference max
     float2* stats;    // [4][NG]  (reference, sum exp) per epilogue warp at the end
+    int cap;          // candidate slots per node
 };
 
 // (m, s) <- (m, s) (+) (m2, s2) for sums of exp relative to their maxima.
@@ -455,15 +458,59 @@ __device__ __forceinline__ void epi_init(const EpiSmem& e, int NG, int k, int et
         e.cnt[i] = 0;
         e.gcache[i] = 0ull;
     }
+    if (etid < 2) e.more[etid] = 0;
     for (int i = etid; i < 4 * NG; i += nthr) e.mref[i] = -INFINITY;
+}
+
+// Appends, for every node j whose bit is set in `offer`, this lane's key
+// key(z[j], row) to node j's candidate slots; returns the bits of the keys
+// that found no free slot (offered again after the next merge).
+__device__ __forceinline__ uint32_t epi_offer(const EpiSmem& e, int c0, const float (&z)[16], uint32_t offer,
+                                              uint32_t row, int lane) {
+    uint32_t pend = 0;
+    if (__any_sync(kFull, offer != 0u)) {
+#pragma unroll
+        for (int j = 0; j < 16; j++) {
+            const bool pass = (offer >> j) & 1u;
+            const unsigned bal = __ballot_sync(kFull, pass);
+            if (bal) {
+                int base = 0;
+                if (lane == 0) base = atomicAdd(&e.cnt[c0 + j], __popc(bal));
+                base = __shfl_sync(kFull, base, 0);
+                const int pos = base + __popc(bal & ((1u << lane) - 1u));
+                if (pass) {
+                    if (pos < e.cap)
+                        e.cand[(c0 + j) * e.cap + pos] = make_key(z[j], row);
+                    else
+                        pend |= 1u << j;
+                }
+            }
+        }
+    }
+    return pend;
+}
+
+// The subset of `pend` whose keys still beat their node's (raised) threshold.
+__device__ __forceinline__ uint32_t epi_still_pass(const EpiSmem& e, int k, int c0, const float (&z)[16],
+                                                   uint32_t pend, uint32_t row) {
+    uint32_t keep = 0;
+#pragma unroll
+    for (int j = 0; j < 16; j++) {
+        if ((pend >> j) & 1u) {
+            const uint64_t l = e.list[(c0 + j) * k + k - 1], g = e.gcache[c0 + j];
+            if (make_key(z[j], row) > (l > g ? l : g)) keep |= 1u << j;
+        }
+    }
+    return keep;
 }
 
 // One 16-node chunk of this thread's row (all 32 lanes, same chunk).
 // ew: the warp's row quarter (0..3; per-quarter reference maxima and sums).
 // z[j]: scaled logit of node c0+j of the group; node j exists iff bit j of
 // nodemask is set; rowvalid: the row is < V.  ssum: the running sum of this
-// lane's node (c0 + lane/2).
-__device__ __forceinline__ void epi_chunk(const EpiSmem& e, int NG, int k, int ew, int lane, int c0,
+// lane's node (c0 + lane/2).  Returns the bits of the candidates that found
+// no free slot (only possible when e.cap < the tile's rows).
+__device__ __forceinline__ uint32_t epi_chunk(const EpiSmem& e, int NG, int k, int ew, int lane, int c0,
                                           float (&z)[16], uint32_t nodemask, bool rowvalid, uint32_t row,
                                           float& ssum) {
     bool ok[16];
@@ -497,19 +544,7 @@ __device__ __forceinline__ void epi_chunk(const EpiSmem& e, int NG, int k, int e
         const uint64_t l = e.list[(c0 + j) * k + k - 1], g = e.gcache[c0 + j];
         if (ok[j] && make_key(z[j], row) > (l > g ? l : g)) passmask |= 1u << j;
     }
-    if (__any_sync(kFull, passmask != 0u)) {
-#pragma unroll
-        for (int j = 0; j < 16; j++) {
-            const bool pass = (passmask >> j) & 1u;
-            const unsigned bal = __ballot_sync(kFull, pass);
-            if (bal) {
-                int base = 0;
-                if (lane == 0) base = atomicAdd(&e.cnt[c0 + j], __popc(bal));
-                base = __shfl_sync(kFull, base, 0);
-                if (pass) e.cand[(c0 + j) * kCandCap + base + __popc(bal & ((1u << lane) - 1u))] = make_key(z[j], row);
-            }
-        }
-    }
+    return epi_offer(e, c0, z, passmask, row, lane);
 }
 
 __device__ __forceinline__ uint64_t shfl_u64(uint64_t v, int src) {
@@ -617,14 +652,15 @@ __device__ __forceinline__ void warp_merge(uint64_t* L, const uint64_t* C, int c
 // keys are distinct, so the test is exact.  Each merge publishes the CTA's
 // k-th key (atomicMax) and fetches gthr[n] for the next tile's filter.
 __device__ __forceinline__ void epi_merge(const EpiSmem& e, int NG, int k, int wi, int lane, int nthr, int etid,
-                                          uint64_t* gthr, int n0, int N) {
+                                          uint64_t* gthr, int n0, int N, int* reset_flag = nullptr) {
     named_bar_sync(kEpiBarrier, nthr);
+    if (reset_flag && etid == 0) *reset_flag = 0;  // every thread read it before this barrier
     uint64_t g = 0ull;
     if (gthr && etid < NG && n0 + etid < N) g = __ldcg(reinterpret_cast<const unsigned long long*>(gthr) + n0 + etid);
     for (int nd = wi; nd < NG; nd += nthr / 32) {
-        const int c = e.cnt[nd];
+        const int c = min(e.cnt[nd], e.cap);
         if (c == 0) continue;
-        warp_merge(e.list + nd * k, e.cand + nd * kCandCap, c, k, lane);
+        warp_merge(e.list + nd * k, e.cand + nd * e.cap, c, k, lane);
         if (lane == 0) {
             e.cnt[nd] = 0;
             const uint64_t kth = e.list[nd * k + k - 1];

@@ -22,12 +22,14 @@ __global__ void __launch_bounds__(kEpiThreads) lmhead_f32_kernel(const LmheadArg
     float* Es = smf;                     // [128][65]
     float* Hs = Es + kTileM * kEPad;     // [NG][64]
     EpiSmem e;
+    e.cap = kCandCap;  // a whole tile: every candidate always fits
     e.list = reinterpret_cast<uint64_t*>(Hs + NG * kBlockK);
     e.cand = e.list + NG * a.k;
     e.gcache = e.cand + NG * kCandCap;
     e.stats = reinterpret_cast<float2*>(e.gcache + NG);
     e.mref = reinterpret_cast<float*>(e.stats + 4 * NG);
     e.cnt = reinterpret_cast<int*>(e.mref + 4 * NG);
+    e.more = e.cnt + NG;
 
     const int g = blockIdx.x % a.G;
     const int vr = blockIdx.x / a.G;
@@ -94,7 +96,7 @@ __global__ void __launch_bounds__(kEpiThreads) lmhead_f32_kernel(const LmheadArg
                     z[j] = (acc[c0 + j] + dl) * a.invT;
                 }
             }
-            epi_chunk(e, NG, a.k, ew, lane, c0, z, nodemask, valid, static_cast<uint32_t>(v), ssum[c0 / 16]);
+            (void)epi_chunk(e, NG, a.k, ew, lane, c0, z, nodemask, valid, static_cast<uint32_t>(v), ssum[c0 / 16]);
         }
         epi_merge(e, NG, a.k, ew, lane, kEpiThreads, tid, a.gthr, g * NG, a.N);
     }
@@ -155,7 +157,8 @@ __global__ void __launch_bounds__(256) gemm_f32_kernel(const GemmArgs a) {
 
 template <int NG>
 int smem_ng(int k) {
-    return (kTileM * kEPad + NG * kBlockK) * 4 + NG * k * 8 + NG * kCandCap * 8 + NG * 8 + 4 * NG * 8 + 4 * NG * 4 + NG * 4;
+    return (kTileM * kEPad + NG * kBlockK) * 4 + NG * k * 8 + NG * kCandCap * 8 + NG * 8 + 4 * NG * 8 + 4 * NG * 4 + NG * 4 +
+           8;
 }
 
 }  // namespace

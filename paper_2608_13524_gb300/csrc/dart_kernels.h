@@ -102,6 +102,7 @@ cudaError_t launch_lmhead_tc(const CUtensorMap* tmE, const CUtensorMap* tmH, con
 cudaError_t launch_gemm_tc(const CUtensorMap* tmA, const CUtensorMap* tmB, const GemmArgs& a, int smem_bytes,
                            cudaStream_t st);
 int tc_stage_bytes(int NG);
+int lmhead_tc_tmem_cols(int NG);  // TMEM columns one LM-head CTA allocates
 int lmhead_tc_fixed_smem(int NG, int k, int stages);
 int gemm_tc_fixed_smem(int stages);
 int lmhead_tc_ctas_per_sm(int NG, int smem);

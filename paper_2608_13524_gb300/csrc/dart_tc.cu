@@ -28,10 +28,22 @@ namespace dart {
 
 namespace {
 
-// 2 warps (producer, MMA) + 4 epilogue warps per 16-node chunk of the group
+// 2 warps (producer, MMA) + 4 epilogue warps (one per TMEM lane quarter) per
+// 16-node chunk of the group, at most 16 epilogue warps: in 128-node groups
+// every epilogue warp handles two chunks.
 template <int NG>
 constexpr int epi_threads() {
-    return 128 * (NG / 16);
+    return 128 * (NG / 16 < 4 ? NG / 16 : 4);
+}
+template <int NG>
+constexpr int epi_chunks() {
+    return NG > 64 ? NG / 64 : 1;
+}
+// Candidate slots per node: a whole tile (nothing can overflow) up to 64-node
+// groups; 128-node groups keep fewer and merge in rounds when they overflow.
+template <int NG>
+constexpr int lm_cand_cap() {
+    return NG > 64 ? kCandCapLarge : kCandCap;
 }
 template <int NG>
 constexpr int threads() {
@@ -234,7 +246,11 @@ constexpr int acc_stride() {
 }
 template <int NG>
 constexpr int tmem_cols() {
-    return 2 * acc_stride<NG>() <= 32 ? 32 : (2 * acc_stride<NG>() <= 64 ? 64 : (2 * acc_stride<NG>() <= 128 ? 128 : 256));
+    return 2 * acc_stride<NG>() <= 32 ? 32
+                                      : (2 * acc_stride<NG>() <= 64 ? 64
+                                                                    : (2 * acc_stride<NG>() <= 128
+                                                                           ? 128
+                                                                           : (2 * acc_stride<NG>() <= 256 ? 256 : 512)));
 }
 
 // ------------------------------------------------------------ LM-head kernel
@@ -247,13 +263,16 @@ __global__ void __launch_bounds__(threads<NG>(), 1)
     pdl_trigger();
     const int stages = a.stages;
     Smem s = carve<NG>(smem_raw, stages);
+    constexpr int kCap = lm_cand_cap<NG>();
     EpiSmem e;
+    e.cap = kCap;
     e.list = reinterpret_cast<uint64_t*>(s.tail);
     e.cand = e.list + NG * a.k;
-    e.gcache = e.cand + NG * kCandCap;
+    e.gcache = e.cand + NG * kCap;
     e.stats = reinterpret_cast<float2*>(e.gcache + NG);
     e.mref = reinterpret_cast<float*>(e.stats + 4 * NG);
     e.cnt = reinterpret_cast<int*>(e.mref + 4 * NG);
+    e.more = e.cnt + NG;
 
     const int g = blockIdx.x % a.G;
     const int vr = blockIdx.x / a.G;
@@ -279,18 +298,48 @@ __global__ void __launch_bounds__(threads<NG>(), 1)
                            acc_stride<NG>(), abort, a.status);
     } else {
         // epilogue warp wi = warp - 2 reads TMEM lane quarter warp % 4 and
-        // owns the 16-node chunk wi / 4 of the group
+        // owns the 16-node chunks wi / 4 + 4 * ci (ci < kChunks) of the group
         constexpr int kEpi = epi_threads<NG>();
+        constexpr int kChunks = epi_chunks<NG>();
         const int etid = threadIdx.x - 64;
         const int wi = warp - 2;
         const int quarter = warp & 3;
-        const int c0 = (wi >> 2) * 16;
         pdl_wait();
         epi_init(e, NG, a.k, etid, kEpi);
-        float ssum = 0.0f;
-        uint32_t nodemask = 0;
-        for (int j = 0; j < 16; j++)
-            if (g * NG + c0 + j < a.N) nodemask |= 1u << j;
+        float ssum[kChunks];
+        uint32_t nodemask[kChunks];
+#pragma unroll
+        for (int ci = 0; ci < kChunks; ci++) {
+            const int c0 = ((wi >> 2) + 4 * ci) * 16;
+            ssum[ci] = 0.0f;
+            nodemask[ci] = 0;
+            for (int j = 0; j < 16; j++)
+                if (g * NG + c0 + j < a.N) nodemask[ci] |= 1u << j;
+        }
+        // scaled logits of this thread's row v for chunk ci from accumulator acc:
+        // hi + lo products, drafter row added, 1/T applied
+        auto load_z = [&](int acc, int ci, int v, bool valid, float (&z)[16]) {
+            const int c0 = ((wi >> 2) + 4 * ci) * 16;
+            float zl[16];
+            const uint32_t tcol =
+                tmem_base + acc * acc_stride<NG>() + c0 + (static_cast<uint32_t>(quarter * 32) << 16);
+            tmem_ld16_pair(tcol, tcol + NG, z, zl);
+#pragma unroll
+            for (int j = 0; j < 16; j++) z[j] += zl[j];
+            int cur_seq = -1;
+            float dl = 0.0f;
+#pragma unroll
+            for (int j = 0; j < 16; j++) {
+                if ((nodemask[ci] >> j) & 1u) {
+                    const int seq = (g * NG + c0 + j) / a.P;
+                    if (seq != cur_seq) {
+                        cur_seq = seq;
+                        dl = valid ? __ldg(a.dlog + seq * a.dlog_seq_stride + a.dlog_row_off + v) : 0.0f;
+                    }
+                    z[j] = (z[j] + dl) * a.invT;
+                }
+            }
+        };
         for (int i = 0; i < w.ntiles; i++) {
             const int acc = i & 1;
             const uint32_t aph = (i >> 1) & 1;
@@ -304,30 +353,56 @@ __global__ void __launch_bounds__(threads<NG>(), 1)
             tc_fence_after();
             const int v = w.row0 + i * kTileM + quarter * 32 + lane;
             const bool valid = v < a.V;
-            float z[16], zl[16];
-            const uint32_t tcol = tmem_base + acc * acc_stride<NG>() + c0 + (static_cast<uint32_t>(quarter * 32) << 16);
-            tmem_ld16_pair(tcol, tcol + NG, z, zl);
-            tc_fence_before();
-            mbar_arrive(&s.tempty[acc]);
+            if constexpr (kCap >= kTileM) {
+                // every candidate of the tile fits: one merge, and the
+                // accumulator is released as soon as it has been read
+                float z[16];
+                load_z(acc, 0, v, valid, z);
+                tc_fence_before();
+                mbar_arrive(&s.tempty[acc]);
+                (void)epi_chunk(e, NG, a.k, quarter, lane, (wi >> 2) * 16, z, nodemask[0], valid,
+                                static_cast<uint32_t>(v), ssum[0]);
+                epi_merge(e, NG, a.k, wi, lane, kEpi, etid, a.gthr, g * NG, a.N);
+            } else {
+                uint32_t pend[kChunks];
 #pragma unroll
-            for (int j = 0; j < 16; j++) z[j] += zl[j];
-            int cur_seq = -1;
-            float dl = 0.0f;
-#pragma unroll
-            for (int j = 0; j < 16; j++) {
-                if ((nodemask >> j) & 1u) {
-                    const int seq = (g * NG + c0 + j) / a.P;
-                    if (seq != cur_seq) {
-                        cur_seq = seq;
-                        dl = valid ? __ldg(a.dlog + seq * a.dlog_seq_stride + a.dlog_row_off + v) : 0.0f;
-                    }
-                    z[j] = (z[j] + dl) * a.invT;
+                for (int ci = 0; ci < kChunks; ci++) {
+                    float z[16];
+                    load_z(acc, ci, v, valid, z);
+                    pend[ci] = epi_chunk(e, NG, a.k, quarter, lane, ((wi >> 2) + 4 * ci) * 16, z, nodemask[ci],
+                                         valid, static_cast<uint32_t>(v), ssum[ci]);
                 }
+                // Merge rounds while some candidate found no free slot: those
+                // still beating the raised thresholds are read again from the
+                // accumulator (kept until the last round) and offered again.
+                // A round's flag is set before epi_merge's first barrier, read
+                // after its second, and cleared in the next round after that
+                // round's first barrier.
+                for (int round = 0;; round++) {
+                    bool any = false;
+#pragma unroll
+                    for (int ci = 0; ci < kChunks; ci++) any |= pend[ci] != 0u;
+                    if (__any_sync(kFull, any) && lane == 0) atomicOr(&e.more[round & 1], 1);
+                    epi_merge(e, NG, a.k, wi, lane, kEpi, etid, a.gthr, g * NG, a.N,
+                              round > 0 ? &e.more[(round + 1) & 1] : nullptr);
+                    if (e.more[round & 1] == 0) break;
+#pragma unroll
+                    for (int ci = 0; ci < kChunks; ci++) {
+                        if (__any_sync(kFull, pend[ci] != 0u)) {
+                            const int c0 = ((wi >> 2) + 4 * ci) * 16;
+                            float z[16];
+                            load_z(acc, ci, v, valid, z);
+                            pend[ci] = epi_offer(e, c0, z, epi_still_pass(e, a.k, c0, z, pend[ci], static_cast<uint32_t>(v)),
+                                                 static_cast<uint32_t>(v), lane);
+                        }
+                    }
+                }
+                tc_fence_before();
+                mbar_arrive(&s.tempty[acc]);
             }
-            epi_chunk(e, NG, a.k, quarter, lane, c0, z, nodemask, valid, static_cast<uint32_t>(v), ssum);
-            epi_merge(e, NG, a.k, wi, lane, kEpi, etid, a.gthr, g * NG, a.N);
         }
-        epi_stash(e, NG, quarter, lane, c0, ssum);
+#pragma unroll
+        for (int ci = 0; ci < kChunks; ci++) epi_stash(e, NG, quarter, lane, ((wi >> 2) + 4 * ci) * 16, ssum[ci]);
         epi_finalize(e, NG, a.k, etid, kEpi, g * NG, a.N, vr, a.nV, a.part_ms, a.part_key);
     }
     teardown(tmem_base, tmem_cols<NG>());
@@ -453,7 +528,8 @@ __global__ void __launch_bounds__(threads<NG>(), 1)
 
 template <int NG>
 int lmhead_fixed(int k, int stages) {
-    return (2 * stages + 5) * 8 + 16 + NG * k * 8 + NG * kCandCap * 8 + NG * 8 + 4 * NG * 8 + 4 * NG * 4 + NG * 4;
+    return (2 * stages + 5) * 8 + 16 + NG * k * 8 + NG * lm_cand_cap<NG>() * 8 + NG * 8 + 4 * NG * 8 + 4 * NG * 4 +
+           NG * 4 + 8;
 }
 
 template <int NG>
@@ -495,11 +571,21 @@ int max_clusters_ng(int smem, int cluster) {
 
 int tc_stage_bytes(int NG) { return kATileBytes + 2 * NG * 128; }
 
+int lmhead_tc_tmem_cols(int NG) {
+    switch (NG) {
+        case 16: return tmem_cols<16>();
+        case 32: return tmem_cols<32>();
+        case 64: return tmem_cols<64>();
+        default: return tmem_cols<128>();
+    }
+}
+
 int lmhead_tc_fixed_smem(int NG, int k, int stages) {
     switch (NG) {
         case 16: return lmhead_fixed<16>(k, stages) + 1024;
         case 32: return lmhead_fixed<32>(k, stages) + 1024;
-        default: return lmhead_fixed<64>(k, stages) + 1024;
+        case 64: return lmhead_fixed<64>(k, stages) + 1024;
+        default: return lmhead_fixed<128>(k, stages) + 1024;
     }
 }
 
@@ -548,7 +634,8 @@ int lmhead_tc_ctas_per_sm(int NG, int smem) {
     switch (NG) {
         case 16: return ctas_per_sm(reinterpret_cast<const void*>(lmhead_tc_kernel<16>), threads<16>(), smem);
         case 32: return ctas_per_sm(reinterpret_cast<const void*>(lmhead_tc_kernel<32>), threads<32>(), smem);
-        default: return ctas_per_sm(reinterpret_cast<const void*>(lmhead_tc_kernel<64>), threads<64>(), smem);
+        case 64: return ctas_per_sm(reinterpret_cast<const void*>(lmhead_tc_kernel<64>), threads<64>(), smem);
+        default: return ctas_per_sm(reinterpret_cast<const void*>(lmhead_tc_kernel<128>), threads<128>(), smem);
     }
 }
 
@@ -561,6 +648,7 @@ cudaError_t tc_set_smem_limits(int max_dyn) {
     DART_SET(lmhead_tc_kernel<16>)
     DART_SET(lmhead_tc_kernel<32>)
     DART_SET(lmhead_tc_kernel<64>)
+    DART_SET(lmhead_tc_kernel<128>)
     DART_SET(gemm_tc_kernel<16>)
     DART_SET(gemm_tc_kernel<32>)
     DART_SET(gemm_tc_kernel<64>)
@@ -574,6 +662,7 @@ cudaError_t launch_lmhead_tc(const CUtensorMap* tmE, const CUtensorMap* tmH, con
         case 16: return launch_lmhead_ng<16>(tmE, tmH, a, smem, st);
         case 32: return launch_lmhead_ng<32>(tmE, tmH, a, smem, st);
         case 64: return launch_lmhead_ng<64>(tmE, tmH, a, smem, st);
+        case 128: return launch_lmhead_ng<128>(tmE, tmH, a, smem, st);
         default: return cudaErrorInvalidValue;
     }
 }
