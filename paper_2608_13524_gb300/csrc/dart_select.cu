@@ -351,6 +351,27 @@ __global__ void gather_x_kernel(int Nc, int d, const int* prow, const int* tok, 
     }
 }
 
+// v += p[0] + p[stride] + ... (n terms, in this order), with up to 8 of the
+// 16-byte loads in flight at once (a plain loop issues them one at a time).
+__device__ __forceinline__ void add_splits(float4& v, const float* p, size_t stride, int n) {
+    constexpr int kBatch = 8;
+    for (int s0 = 0; s0 < n; s0 += kBatch) {
+        float4 w[kBatch];
+#pragma unroll
+        for (int u = 0; u < kBatch; u++)
+            if (s0 + u < n) w[u] = *reinterpret_cast<const float4*>(p + static_cast<size_t>(s0 + u) * stride);
+#pragma unroll
+        for (int u = 0; u < kBatch; u++) {
+            if (s0 + u < n) {
+                v.x += w[u].x;
+                v.y += w[u].y;
+                v.z += w[u].z;
+                v.w += w[u].w;
+            }
+        }
+    }
+}
+
 __global__ void silu_split_kernel(int Nc, int d, int S, const float* part, __nv_bfloat16* AL, int bhalf, float* A32) {
     pdl_trigger();
     pdl_wait();
@@ -360,13 +381,7 @@ __global__ void silu_split_kernel(int Nc, int d, int S, const float* part, __nv_
          u += static_cast<size_t>(gridDim.x) * blockDim.x) {
         const size_t q = u * 4;
         float4 v = *reinterpret_cast<const float4*>(part + q);
-        for (int s = 1; s < S; s++) {
-            const float4 w = *reinterpret_cast<const float4*>(part + static_cast<size_t>(s) * total + q);
-            v.x += w.x;
-            v.y += w.y;
-            v.z += w.z;
-            v.w += w.w;
-        }
+        add_splits(v, part + total + q, total, S - 1);
         v.x = v.x / (1.0f + expf(-v.x));
         v.y = v.y / (1.0f + expf(-v.y));
         v.z = v.z / (1.0f + expf(-v.z));
@@ -401,14 +416,7 @@ __global__ void __launch_bounds__(NT) residual_norm_kernel(int d, int S, int Nc,
         r[it] = make_float4(0.f, 0.f, 0.f, 0.f);
         if (j < d && pr >= 0) {
             float4 v = *reinterpret_cast<const float4*>(h + static_cast<size_t>(pr) * d + j);
-            for (int s = 0; s < S; s++) {
-                const float4 w = *reinterpret_cast<const float4*>(part + static_cast<size_t>(s) * total +
-                                                                  static_cast<size_t>(c) * d + j);
-                v.x += w.x;
-                v.y += w.y;
-                v.z += w.z;
-                v.w += w.w;
-            }
+            add_splits(v, part + static_cast<size_t>(c) * d + j, total, S);
             r[it] = v;
             ss += v.x * v.x + v.y * v.y + v.z * v.z + v.w * v.w;
         }
