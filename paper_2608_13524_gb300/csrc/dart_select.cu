@@ -15,6 +15,7 @@
 #include <cstdlib>
 
 #include "dart_device.cuh"
+#include "dart_frontier.cuh"
 #include "dart_kernels.h"
 
 namespace dart {
@@ -23,30 +24,6 @@ namespace {
 
 constexpr int kSelThreads = 512;
 constexpr int kEmitThreads = 1024;
-
-__device__ __forceinline__ int block_sum_int(int v, int* red) {
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xFFFFFFFFu, v, o);
-    __syncthreads();
-    if (lane == 0) red[warp] = v;
-    __syncthreads();
-    int t = 0;
-    for (int i = 0; i < nw; i++) t += red[i];
-    return t;
-}
-
-__device__ __forceinline__ float block_sum_float(float v, float* red) {
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xFFFFFFFFu, v, o);
-    __syncthreads();
-    if (lane == 0) red[warp] = v;
-    __syncthreads();
-    float t = 0.0f;
-    for (int i = 0; i < nw; i++) t += red[i];
-    return t;
-}
 
 __global__ void __launch_bounds__(kSelThreads) merge_select_kernel(const SelectArgs a) {
     pdl_trigger();
@@ -144,48 +121,7 @@ __global__ void __launch_bounds__(kSelThreads) merge_select_kernel(const SelectA
     __threadfence();
     if (tid == 0) a.seq_ticket[s] = 0;
 
-    // candidates (p, j): parent p's list is sorted by log q~, hence by score
-    const int ncand = prev_count * a.k;
-    int valid = 0;
-    for (int c = tid; c < ncand; c += kSelThreads) {
-        const int pp = c / a.k, j = c % a.k;
-        const size_t src_i = static_cast<size_t>(s * a.P + pp) * a.k + j;
-        const float ps = a.dep == 1 ? 0.0f : a.tree_score[(static_cast<size_t>(s) * a.L + a.dep - 2) * a.W + pp];
-        const float lq = __ldcg(a.node_logq + src_i);
-        ctok[c] = __ldcg(a.node_tok + src_i);
-        const float sc = (ps + lq) + a.beta;  // Eq. 5, one more depth
-        const bool ok = sc > -INFINITY;
-        keys[c] = ok ? make_key(sc, static_cast<uint32_t>(c)) : 0ull;
-        valid += ok;
-    }
-    const int nvalid = block_sum_int(valid, redi);
-    const int cnt = min(a.W, nvalid);
-    if (cnt > 0) topk_of_sorted_lists(keys, prev_count, a.k, cnt, 0ull, top, surv, &thr, hist, scal);
-    const size_t tb = (static_cast<size_t>(s) * a.L + a.dep - 1) * a.W;
-    for (int r = tid; r < a.W; r += kSelThreads) {
-        if (r < cnt) {
-            const uint64_t x = top[r];
-            const int c = static_cast<int>(key_idx(x));
-            const int pp = c / a.k;
-            const int tok = ctok[c];
-            a.tree_tok[tb + r] = tok;
-            a.tree_parent[tb + r] = a.dep == 1 ? -1 : pp;
-            a.tree_score[tb + r] = key_val(x);
-            if (r < a.Pn) {
-                a.child_prow[s * a.Pn + r] = s * a.P + pp;
-                a.child_tok[s * a.Pn + r] = tok;
-            }
-        } else {
-            a.tree_tok[tb + r] = -1;
-            a.tree_parent[tb + r] = -1;
-            a.tree_score[tb + r] = -INFINITY;
-            if (r < a.Pn) {
-                a.child_prow[s * a.Pn + r] = -1;
-                a.child_tok[s * a.Pn + r] = 0;
-            }
-        }
-    }
-    if (tid == 0) a.tree_count[s * a.L + a.dep - 1] = cnt;
+    select_frontier(a, s, prev_count, keys, ctok, surv, top, &thr, hist, scal, redi);
 }
 
 // Number of keys > x in the descending list l[0..n) (binary search).
