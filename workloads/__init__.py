@@ -199,3 +199,95 @@ def make_inputs(cfg: Config, zero_E: bool = False, rank: int = 0):
     Wi, Wo, E = make_weights(cfg, zero_E=zero_E)
     Dlog, h0 = make_sequences(cfg, rank=rank)
     return dict(Wi=Wi, Wo=Wo, E=E, Dlog=Dlog, h0=h0)
+
+
+# --------------------------------------------------------------------------
+# tree-attention verification inputs (Sec. 2.2: one target forward pass over
+# the flattened tree).  The target model is not available: one attention
+# layer with Qwen3-4B/8B head geometry (32 query heads, 8 key/value heads,
+# head dim 128, RoPE base 1e6) on N(0,1) queries, keys and values, and a
+# verified context of C tokens whose keys are a (rotated) KV cache.  The
+# tree is a random prefix tree shaped like DARTree's supertree: depth levels
+# 1..L of at most W nodes, each node's parent drawn uniformly from the level
+# above, ids in level order (a topological order, as emitted).
+
+@dataclasses.dataclass(frozen=True)
+class AttnConfig:
+    name: str
+    nseq: int
+    B: int          # tree rows per sequence (the budget)
+    C: int          # context keys per sequence
+    L: int          # maximum depth
+    W: int          # maximum nodes per depth level
+    seed: int
+    Hq: int = 32
+    Hkv: int = 8
+    dh: int = 128
+    rope_theta: float = 1.0e6
+    pos_offset: int = -1     # < 0: the context length C, so depth d sits at position C + d
+    fill: float = 1.0        # fraction of the B rows used by the tree (n_nodes)
+
+    def replace(self, **kw) -> "AttnConfig":
+        return dataclasses.replace(self, **kw)
+
+    @property
+    def scale(self) -> float:
+        return 1.0 / float(self.dh) ** 0.5
+
+    @property
+    def offset(self) -> int:
+        return self.C if self.pos_offset < 0 else self.pos_offset
+
+
+ATTN_Q8B = AttnConfig("verify-qwen3-8b", 1, 256, 2048, 16, 16, 2620)
+ATTN_Q4B = AttnConfig("verify-qwen3-4b", 1, 64, 2048, 16, 8, 2621)
+ATTN_BATCHED = AttnConfig("verify-batched", 8, 512, 2048, 16, 32, 2622)
+ATTN_NAMED = {c.name: c for c in (ATTN_Q8B, ATTN_Q4B, ATTN_BATCHED)}
+
+
+def random_tree(B: int, L: int, W: int, n: int, g: np.random.Generator):
+    """parents [B] (-1: child of the root, -2: unused row) and depths [B]
+    (0 for unused rows) of a random n-node prefix tree in level order."""
+    parents = np.full(B, -2, dtype=np.int32)
+    depths = np.zeros(B, dtype=np.int32)
+    prev = [-1]
+    i = 0
+    d = 1
+    while i < n and d <= L:
+        cnt = min(W, n - i)
+        if d == L:
+            cnt = n - i  # the last level takes what is left
+        picks = np.sort(g.integers(0, len(prev), size=cnt))
+        level = []
+        for pk in picks:
+            parents[i] = prev[pk]
+            depths[i] = d
+            level.append(i)
+            i += 1
+        prev = level
+        d += 1
+    return parents, depths
+
+
+def make_attn_inputs(cfg: AttnConfig):
+    """Q, K, V of the tree rows and the context (uint16 bf16 bit patterns,
+    N(0,1) before rounding) and the tree structure (parents, depths, n_nodes)."""
+    g = np.random.Generator(np.random.PCG64([cfg.seed, 7]))
+
+    def bf(*shape):
+        return f32_to_bf16_bits(g.standard_normal(shape, dtype=np.float32))
+
+    q = bf(cfg.nseq, cfg.B, cfg.Hq, cfg.dh)
+    k_tree = bf(cfg.nseq, cfg.B, cfg.Hkv, cfg.dh)
+    v_tree = bf(cfg.nseq, cfg.B, cfg.Hkv, cfg.dh)
+    k_ctx = bf(cfg.nseq, cfg.C, cfg.Hkv, cfg.dh)
+    v_ctx = bf(cfg.nseq, cfg.C, cfg.Hkv, cfg.dh)
+    parents = np.empty((cfg.nseq, cfg.B), dtype=np.int32)
+    depths = np.empty((cfg.nseq, cfg.B), dtype=np.int32)
+    n_nodes = np.empty(cfg.nseq, dtype=np.int32)
+    for s in range(cfg.nseq):
+        n = max(0, min(cfg.B, int(round(cfg.fill * cfg.B)) - (s % 3 if cfg.fill < 1.0 else 0)))
+        parents[s], depths[s] = random_tree(cfg.B, cfg.L, cfg.W, n, g)
+        n_nodes[s] = int((parents[s] != -2).sum())
+    return dict(q=q, k_tree=k_tree, v_tree=v_tree, k_ctx=k_ctx, v_ctx=v_ctx, parents=parents,
+                depths=depths, n_nodes=n_nodes)
