@@ -60,13 +60,14 @@ def root_path(parents: np.ndarray, i: int) -> list:
 
 
 def tree_attention(q, k_tree, v_tree, k_ctx, v_ctx, parents, depths, n_nodes, pos_offset: int,
-                   rope_theta: float, scale: float) -> np.ndarray:
+                   rope_theta: float, scale: float, rows=None) -> np.ndarray:
     """One tree-attention layer (see module docstring).
 
     q [nseq, B, Hq, dh]; k_tree, v_tree [nseq, B, Hkv, dh]; k_ctx, v_ctx
     [nseq, C, Hkv, dh] (k_ctx rotated); parents, depths [nseq, B];
     n_nodes [nseq].  Returns out [nseq, B, Hq, dh] float64 with zero rows
-    for i >= n_nodes.
+    for i >= n_nodes.  `rows`, a list of (s, i), restricts the evaluation to
+    those tree rows (the others stay zero).
     """
     q = np.asarray(q, dtype=np.float64)
     k_tree = np.asarray(k_tree, dtype=np.float64)
@@ -77,10 +78,13 @@ def tree_attention(q, k_tree, v_tree, k_ctx, v_ctx, parents, depths, n_nodes, po
     Hkv = k_tree.shape[2]
     G = Hq // Hkv
     out = np.zeros((nseq, B, Hq, dh), dtype=np.float64)
+    want = None if rows is None else {(int(s), int(i)) for s, i in rows}
     for s in range(nseq):
         n = int(n_nodes[s])
         pos = pos_offset + np.asarray(depths[s], dtype=np.int64)
         for i in range(n):
+            if want is not None and (s, i) not in want:
+                continue
             path = root_path(parents[s], i)
             for h in range(Hq):
                 g = h // G

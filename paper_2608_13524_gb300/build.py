@@ -17,7 +17,8 @@ CSRC = os.path.join(HERE, "csrc")
 LIB = os.path.join(HERE, "libdart.so")
 BUILD_DIR = os.path.join(HERE, "_build")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
-SOURCES = ["dart_abi.cu", "dart_tc.cu", "dart_f32.cu", "dart_select.cu", "dart_noalloc.cu", "dart_cand.cu"]
+SOURCES = ["dart_abi.cu", "dart_tc.cu", "dart_f32.cu", "dart_select.cu", "dart_noalloc.cu", "dart_cand.cu",
+           "dart_attn.cu"]
 
 
 def _nvcc() -> str:

@@ -19,22 +19,7 @@
 #include "dart_device.cuh"
 #include "dart_kernels.h"
 
-using namespace dart;
-
-namespace {
-
-constexpr int kVersion = 1;
-constexpr int kMaxW = 64, kMaxK = 64, kMaxWK = 4096, kMaxSuper = 1024, kMaxB = 1024;
-constexpr int kMaxD = 16384;
-constexpr int kMaxCandK = 1024;  // candidate-set size K of the restricted scoring
-constexpr int kMaxV = (1 << 24) - 1;
-constexpr int kMaxProfilePairs = 8192;
-
-typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
-                                  const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
-                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
-
-EncodeTiledFn encode_fn() {
+dart::EncodeTiledFn dart::tensor_map_encoder() {
     static EncodeTiledFn fn = nullptr;
     if (!fn) {
         void* p = nullptr;
@@ -46,6 +31,19 @@ EncodeTiledFn encode_fn() {
     }
     return fn;
 }
+
+using namespace dart;
+
+namespace {
+
+constexpr int kVersion = 1;
+constexpr int kMaxW = 64, kMaxK = 64, kMaxWK = 4096, kMaxSuper = 1024, kMaxB = 1024;
+constexpr int kMaxD = 16384;
+constexpr int kMaxCandK = 1024;  // candidate-set size K of the restricted scoring
+constexpr int kMaxV = (1 << 24) - 1;
+constexpr int kMaxProfilePairs = 8192;
+
+EncodeTiledFn encode_fn() { return tensor_map_encoder(); }
 
 // 2-D bf16 tensor [rows][inner] with a (64 x box_rows) box and 128-byte swizzle.
 bool encode_bf16_2d(CUtensorMap* m, const void* base, uint64_t inner, uint64_t rows, uint32_t box_rows) {

@@ -8,6 +8,12 @@
 
 namespace dart {
 
+// cuTensorMapEncodeTiled from the driver (NULL if unavailable), looked up once.
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                  const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+EncodeTiledFn tensor_map_encoder();
+
 // Launches `kernel` with programmatic stream serialization (PDL), so its
 // prologue can overlap the tail of the previous kernel in the stream.
 bool pdl_enabled();

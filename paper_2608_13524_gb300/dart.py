@@ -39,6 +39,11 @@ class DartTreeOut(C.Structure):
                 ("mask", C.c_void_p)]
 
 
+class DartAttnConfig(C.Structure):
+    _fields_ = [("nseq", C.c_int), ("B", C.c_int), ("C", C.c_int), ("Hq", C.c_int), ("Hkv", C.c_int),
+                ("dh", C.c_int), ("rope_theta", C.c_float), ("scale", C.c_float)]
+
+
 class DartError(RuntimeError):
     def __init__(self, code, what):
         super().__init__(f"{what}: {status_string(code)} ({code})")
@@ -71,6 +76,10 @@ def lib():
             "dart_profile_read_kinds": (i, [vp, vp, vp, i]),
             "dart_launches_per_round": (i, [vp]),
             "dart_expand_root_noalloc": (i, [C.POINTER(DartConfig), vp, vp, vp, vp, vp, vp, vp, vp, vp, vp]),
+            "dart_tree_attention_workspace": (C.c_size_t, [C.POINTER(DartAttnConfig)]),
+            "dart_tree_attention": (i, [C.POINTER(DartAttnConfig), vp, vp, vp, vp, vp, vp, vp, vp, vp, vp,
+                                        C.c_size_t, vp, vp]),
+            "dart_ancestor_mask": (i, [vp, vp, i, i, vp, vp]),
             "dart_destroy": (None, [vp]),
             "dart_status_string": (C.c_char_p, [i]),
             "dart_version": (i, []),
@@ -269,3 +278,49 @@ class Dart:
                 self.close()
         except Exception:
             pass
+
+
+# ------------------------------------------- tree-attention verification (dart_verify.h)
+
+def make_attn_config(nseq, B, C_ctx, Hq, Hkv, dh, rope_theta, scale) -> DartAttnConfig:
+    return DartAttnConfig(int(nseq), int(B), int(C_ctx), int(Hq), int(Hkv), int(dh), float(rope_theta),
+                          float(scale))
+
+
+def dart_tree_attention_workspace(acfg: DartAttnConfig) -> int:
+    return int(lib().dart_tree_attention_workspace(C.byref(acfg)))
+
+
+def dart_tree_attention(acfg: DartAttnConfig, q, k_tree, v_tree, k_ctx, v_ctx, pos_ids, mask, n_nodes, out,
+                        workspace, status=None, stream=None):
+    """One tree-attention layer; every tensor is a caller-owned device tensor
+    (bf16 q/k/v, int32 pos_ids/n_nodes, int64 mask, fp32 out, uint8 workspace)."""
+    _check(lib().dart_tree_attention(C.byref(acfg), _ptr(q), _ptr(k_tree), _ptr(v_tree), _ptr(k_ctx),
+                                     _ptr(v_ctx), _ptr(pos_ids), _ptr(mask), _ptr(n_nodes), _ptr(out),
+                                     _ptr(workspace), C.c_size_t(workspace.numel() * workspace.element_size()),
+                                     _ptr(status), _stream(stream)), "dart_tree_attention")
+
+
+def dart_ancestor_mask(parents, n_nodes, mask, stream=None):
+    nseq, B = parents.shape
+    _check(lib().dart_ancestor_mask(_ptr(parents), _ptr(n_nodes), int(nseq), int(B), _ptr(mask),
+                                    _stream(stream)), "dart_ancestor_mask")
+
+
+class TreeAttention:
+    """Owns the workspace of one tree-attention shape."""
+
+    def __init__(self, nseq, B, C_ctx, Hq=32, Hkv=8, dh=128, rope_theta=1.0e6, scale=None):
+        self.cfg = make_attn_config(nseq, B, C_ctx, Hq, Hkv, dh, rope_theta,
+                                    scale if scale is not None else dh ** -0.5)
+        n = dart_tree_attention_workspace(self.cfg)
+        if n == 0:
+            raise DartError(DART_ERR_INVALID, "dart_tree_attention_workspace")
+        self.workspace = torch.empty(n, dtype=torch.uint8, device="cuda")
+        c = self.cfg
+        self.out = torch.empty((c.nseq, c.B, c.Hq, c.dh), dtype=torch.float32, device="cuda")
+
+    def __call__(self, q, k_tree, v_tree, k_ctx, v_ctx, pos_ids, mask, n_nodes, status=None, stream=None):
+        dart_tree_attention(self.cfg, q, k_tree, v_tree, k_ctx, v_ctx, pos_ids, mask, n_nodes, self.out,
+                            self.workspace, status, stream)
+        return self.out

@@ -85,3 +85,43 @@ def test_null_handle_is_rejected():
     assert lib.dart_build_tree(None, None, None, C.byref(out), None) == dart.DART_ERR_INVALID
     assert lib.dart_status_sync(None, None) == dart.DART_ERR_INVALID
     lib.dart_destroy(None)  # no-op
+
+
+ATTN_BAD = [dict(nseq=0), dict(B=0), dict(B=1025), dict(C_ctx=-1), dict(Hq=12, Hkv=8), dict(Hq=24, Hkv=8),
+            dict(Hq=4, Hkv=8), dict(dh=64), dict(rope_theta=1.0), dict(rope_theta=float("inf")), dict(scale=0.0),
+            dict(scale=float("nan"))]
+
+
+def attn_cfg(**kw):
+    base = dict(nseq=1, B=64, C_ctx=128, Hq=32, Hkv=8, dh=128, rope_theta=1.0e6, scale=128 ** -0.5)
+    base.update(kw)
+    return dart.make_attn_config(**base)
+
+
+@pytest.mark.parametrize("bad", ATTN_BAD, ids=[str(b) for b in ATTN_BAD])
+def test_tree_attention_rejects_bad_config_on_host(bad):
+    lib = dart.lib()
+    cfg = attn_cfg(**bad)
+    assert lib.dart_tree_attention_workspace(C.byref(cfg)) == 0
+    buf = (C.c_uint8 * 1024)()
+    p = (C.cast(buf, C.c_void_p).value + 255) & ~255
+    rc = lib.dart_tree_attention(C.byref(cfg), p, p, p, p, p, p, p, p, p, p, 1 << 40, None, None)
+    assert rc == dart.DART_ERR_INVALID
+
+
+def test_tree_attention_rejects_null_and_misaligned_pointers():
+    lib = dart.lib()
+    cfg = attn_cfg()
+    buf = (C.c_uint8 * 1024)()
+    p = (C.cast(buf, C.c_void_p).value + 255) & ~255
+    args = [p] * 10
+    for i in range(10):
+        a = list(args)
+        a[i] = None  # context K/V (3, 4) may be NULL only when C = 0
+        assert lib.dart_tree_attention(C.byref(cfg), *a, 1 << 40, None, None) == dart.DART_ERR_INVALID
+        a[i] = p + 8
+        assert lib.dart_tree_attention(C.byref(cfg), *a, 1 << 40, None, None) == dart.DART_ERR_INVALID
+    assert lib.dart_ancestor_mask(None, p, 1, 8, p, None) == dart.DART_ERR_INVALID
+    assert lib.dart_ancestor_mask(p, p, 1, 0, p, None) == dart.DART_ERR_INVALID
+    assert lib.dart_ancestor_mask(p, p, 0, 8, p, None) == dart.DART_ERR_INVALID
+    assert lib.dart_ancestor_mask(p, p, 1, 1025, p, None) == dart.DART_ERR_INVALID
