@@ -86,6 +86,16 @@ int dart_tree_attention(const dart_attn_config *cfg, const void *q, const void *
                         const int32_t *n_nodes, float *out, void *workspace, size_t workspace_bytes,
                         int *status, void *stream);
 
+/* dart_tree_attention followed by a synchronisation of `stream`; *ms_rope
+ * and *ms_attn receive the device time of the RoPE pre-pass and of the
+ * attention kernel (CUDA events recorded around each launch on `stream`).
+ * For benchmarking; same arguments and errors, plus DART_ERR_INVALID for a
+ * NULL ms_rope / ms_attn. */
+int dart_tree_attention_timed(const dart_attn_config *cfg, const void *q, const void *k_tree, const void *v_tree,
+                              const void *k_ctx, const void *v_ctx, const int32_t *pos_ids, const uint64_t *mask,
+                              const int32_t *n_nodes, float *out, void *workspace, size_t workspace_bytes,
+                              int *status, float *ms_rope, float *ms_attn, void *stream);
+
 /* Ancestor bitmask of flattened trees given by parent indices:
  * parents [nseq][B] int32 with -1 for a child of the root and
  * 0 <= parents[i] < i otherwise (a topological order, as emitted);

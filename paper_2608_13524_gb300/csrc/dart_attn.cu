@@ -4,23 +4,25 @@
 // hands the pruned tree to that single forward pass).  Contract:
 // include/dart_verify.h.
 //
-// Three launches per call:
-//   attn_rope_kernel   rotates the tree queries and keys by their position
-//                      ids (rotate-half RoPE, fp32, rounded to bf16) into the
-//                      workspace; queries are regrouped so the Hq/Hkv query
-//                      heads of one kv head are adjacent rows;
+// Two launches per call:
+//   attn_prep_kernel   the RoPE (cos, sin) table of every tree position and
+//                      the rotated tree keys (rotate-half RoPE in fp32,
+//                      rounded to bf16) in the workspace;
 //   tree_attn_kernel   flash attention on the tensor cores (tcgen05, TMEM
 //                      accumulators, TMA-staged K/V).  A CTA owns 128 query
 //                      rows = 128/G tree rows x the G query heads sharing one
-//                      kv head, so each K/V tile feeds all G heads.  Its key
+//                      kv head, so each K/V tile feeds all G heads; the
+//                      softmax warps rotate the query tile in shared memory
+//                      before the first MMA.  Its key
 //                      tiles are the context tiles (all visible, ragged tail
 //                      masked) followed by the tree tiles up to its last row
 //                      (ancestors precede their descendants, so later tiles
-//                      are invisible), masked by the ancestor bitmask.  Long
-//                      key lists are split over `splits` CTAs whose last
-//                      finisher merges the partial (max, sum, O) in split
-//                      order (deterministic, nobody waits);
-//   ancestor mask      (dart_ancestor_mask only) one block per sequence.
+//                      are invisible), masked by the ancestor bitmask.  When
+//                      there are fewer (sequence, kv head, query tile) blocks
+//                      than SMs, the key list is split over a thread-block
+//                      cluster whose CTAs merge their partial (max, sum, O)
+//                      over distributed shared memory, in rank order;
+// and dart_ancestor_mask's own kernel, one block per sequence.
 // Warp roles of tree_attn_kernel (192 threads): warp 0 TMA producer, warp 1
 // TMEM allocator + single-thread MMA issuer, warps 2-5 softmax, thread =
 // query row = TMEM lane.  TMEM: two S buffers (128 columns each, so the
@@ -50,35 +52,34 @@ constexpr int kRows = 128;                // query rows per CTA (MMA M)
 constexpr int kKeys = 128;                // keys per tile (MMA N of S = QK^T, K of O += PV)
 constexpr int kAttnThreads = 192;
 constexpr int kSoftThreads = 128;
-constexpr int kKvStages = 2;
+constexpr int kKStages = 3;                  // K ring: the S MMA needs K two tiles ahead of its load
+constexpr int kVStages = 2;
 constexpr int kHalf = kRows * 64 * 2;     // 16 KB: 128 rows x 64 bf16, one 128-byte swizzle column
 constexpr int kTileBytes = 2 * kHalf;     // 32 KB: 128 rows x dh bf16
-constexpr int kMaxSplits = 16;
+constexpr int kMaxSplits = 8;                // cluster size limit (portable)
 constexpr int kTmemCols = 512;            // S0 [0,128), S1 [128,256), O [256,384)
 constexpr int kOCol = 256;
 constexpr float kRescaleSlack = 8.0f;     // log2 units: P <= 2^8 between rescales
-constexpr int kSmemUsed = kTileBytes * (1 + 2 * kKvStages + 1) + 16 * 8 + 4 * 4;
+constexpr int kNumBars = 1 + 2 * kKStages + 2 * kVStages + 4 + 4;
+constexpr int kSmemUsed = kTileBytes * (1 + kKStages + kVStages + 1) + kNumBars * 8 + 4 * 4;  // Q, K/V rings, P, barriers
 constexpr int kAttnSmem = kSmemUsed + 1024;  // + alignment slack of the 1024-byte swizzle atoms
 
 struct AttnArgs {
     int B, C, Hq, Hkv, G, qpt, nqt, splits, mw, nct;
     float sl2;                // scale * log2(e)
+    const float2* cs;         // [nseq][B][dh/2] RoPE (cos, sin) of the tree positions
     const int32_t* n_nodes;   // [nseq]
     const uint64_t* mask;     // [nseq][B][mw]
     float* out;               // [nseq][B][Hq][dh]
-    float* part_o;            // [blocks][splits][dh][128]
-    float2* part_ml;          // [blocks][splits][128] (running max in log2 units, sum)
-    int* ticket;              // [blocks], zero on entry
     int* status;
 };
 
-struct RopeArgs {
-    int nseq, B, Hq, Hkv, G;
-    const __nv_bfloat16* q;   // [nseq][B][Hq][dh]
+struct PrepArgs {
+    int nseq, B, Hkv;
     const __nv_bfloat16* kt;  // [nseq][B][Hkv][dh]
     const int32_t* pos_ids;   // [nseq][B]
-    __nv_bfloat16* qr;        // [nseq][Hkv][B][G][dh]
-    __nv_bfloat16* kr;        // [nseq][B][Hkv][dh]
+    __nv_bfloat16* kr;        // [nseq][B][Hkv][dh] rotated tree keys
+    float2* cs;               // [nseq][B][dh/2] (cos, sin) of every tree position and frequency
     float inv_freq[kDh / 2];
 };
 
@@ -142,6 +143,26 @@ __device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, volati
     return __all_sync(0xFFFFFFFFu, got);
 }
 
+// Stores into the shared memory of cluster CTA `rank` at the offset of the
+// local shared address `local` (distributed shared memory).
+__device__ __forceinline__ void st_cluster_f32x4(uint32_t local, int rank, float x, float y, float z, float w) {
+    uint32_t remote;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(remote) : "r"(local), "r"(rank));
+    asm volatile("st.shared::cluster.v4.f32 [%0], {%1, %2, %3, %4};" ::"r"(remote), "f"(x), "f"(y), "f"(z), "f"(w)
+                 : "memory");
+}
+__device__ __forceinline__ void st_cluster_f32x2(uint32_t local, int rank, float x, float y) {
+    uint32_t remote;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(remote) : "r"(local), "r"(rank));
+    asm volatile("st.shared::cluster.v2.f32 [%0], {%1, %2};" ::"r"(remote), "f"(x), "f"(y) : "memory");
+}
+
+// Column slice [slice_lo(j), slice_lo(j + 1)) merged by cluster CTA j of
+// `splits` (multiples of 4 columns), and the padded row stride (floats) of a
+// received slice: an odd number of 16-byte units.
+__device__ __forceinline__ int slice_lo(int j, int splits) { return 4 * ((j * (kDh / 4)) / splits); }
+__device__ __forceinline__ int slice_stride(int ncol) { return ((ncol / 4) & 1) ? ncol : ncol + 4; }
+
 __device__ __forceinline__ uint32_t pack_bf16(float a, float b) {
     const __nv_bfloat162 h = __floats2bfloat162_rn(a, b);
     return *reinterpret_cast<const uint32_t*>(&h);
@@ -149,46 +170,71 @@ __device__ __forceinline__ uint32_t pack_bf16(float a, float b) {
 
 // ------------------------------------------------------------ RoPE pre-pass
 
-__global__ void __launch_bounds__(256) attn_rope_kernel(const RopeArgs a) {
+// One warp per tree row (s, b): the (cos, sin) of its position for the 64
+// frequencies (two per lane) go to the table the attention kernel rotates its
+// queries with, and the Hkv key rows of (s, b) are rotated into kr.
+__global__ void __launch_bounds__(256) attn_prep_kernel(const PrepArgs a) {
     pdl_trigger();
     pdl_wait();
-    constexpr int kPairs = kDh / 4;  // threads per row: two rotation pairs each
-    const long long qrows = static_cast<long long>(a.nseq) * a.B * a.Hq;
-    const long long rows = qrows + static_cast<long long>(a.nseq) * a.B * a.Hkv;
-    for (long long u = blockIdx.x * static_cast<long long>(blockDim.x) + threadIdx.x; u < rows * kPairs;
-         u += static_cast<long long>(gridDim.x) * blockDim.x) {
-        const long long row = u / kPairs;
-        const int t = static_cast<int>(u % kPairs) * 2;
-        const __nv_bfloat16* src;
-        __nv_bfloat16* dst;
-        int sb;  // s * B + b
-        if (row < qrows) {
-            const int h = static_cast<int>(row % a.Hq);
-            sb = static_cast<int>(row / a.Hq);
-            const int s = sb / a.B, b = sb % a.B, kvh = h / a.G, g = h % a.G;
-            src = a.q + row * kDh;
-            dst = a.qr + ((((static_cast<long long>(s) * a.Hkv + kvh) * a.B + b) * a.G + g) * kDh);
-        } else {
-            const long long kr = row - qrows;
-            sb = static_cast<int>(kr / a.Hkv);
-            src = a.kt + kr * kDh;
-            dst = a.kr + kr * kDh;
-        }
-        const float pos = static_cast<float>(a.pos_ids[sb]);
-        const __nv_bfloat162 x1 = *reinterpret_cast<const __nv_bfloat162*>(src + t);
-        const __nv_bfloat162 x2 = *reinterpret_cast<const __nv_bfloat162*>(src + t + kDh / 2);
+    const int lane = threadIdx.x & 31, t = lane * 2;
+    const int rows = a.nseq * a.B;
+    const int wstride = gridDim.x * (blockDim.x >> 5);
+    for (int sb = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); sb < rows; sb += wstride) {
+        const float pos = static_cast<float>(__ldg(a.pos_ids + sb));
         float s0, c0, s1, c1;
         sincosf(pos * a.inv_freq[t], &s0, &c0);
         sincosf(pos * a.inv_freq[t + 1], &s1, &c1);
-        const float a0 = __low2float(x1), a1 = __high2float(x1);
-        const float b0 = __low2float(x2), b1 = __high2float(x2);
-        *reinterpret_cast<__nv_bfloat162*>(dst + t) = __floats2bfloat162_rn(a0 * c0 - b0 * s0, a1 * c1 - b1 * s1);
-        *reinterpret_cast<__nv_bfloat162*>(dst + t + kDh / 2) =
-            __floats2bfloat162_rn(b0 * c0 + a0 * s0, b1 * c1 + a1 * s1);
+        *reinterpret_cast<float4*>(a.cs + static_cast<size_t>(sb) * (kDh / 2) + t) = make_float4(c0, s0, c1, s1);
+        for (int kvh = 0; kvh < a.Hkv; kvh++) {
+            const size_t row = (static_cast<size_t>(sb) * a.Hkv + kvh) * kDh;
+            const __nv_bfloat162 x1 = *reinterpret_cast<const __nv_bfloat162*>(a.kt + row + t);
+            const __nv_bfloat162 x2 = *reinterpret_cast<const __nv_bfloat162*>(a.kt + row + t + kDh / 2);
+            const float a0 = __low2float(x1), a1 = __high2float(x1);
+            const float b0 = __low2float(x2), b1 = __high2float(x2);
+            *reinterpret_cast<__nv_bfloat162*>(a.kr + row + t) =
+                __floats2bfloat162_rn(a0 * c0 - b0 * s0, a1 * c1 - b1 * s1);
+            *reinterpret_cast<__nv_bfloat162*>(a.kr + row + t + kDh / 2) =
+                __floats2bfloat162_rn(b0 * c0 + a0 * s0, b1 * c1 + a1 * s1);
+        }
     }
 }
 
 // ------------------------------------------------------------ attention
+
+// 128 consecutive 32-bit TMEM columns of this thread's lane into registers
+// (four x32 loads, one wait; the registers are tied to the wait so no use can
+// move above it).
+__device__ __forceinline__ void tmem_ld128(uint32_t taddr, float (&v)[128]) {
+    uint32_t r[128];
+    asm volatile("tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+                 : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+                 : "r"(taddr + 0));
+    asm volatile("tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+                 : "=r"(r[32]), "=r"(r[33]), "=r"(r[34]), "=r"(r[35]), "=r"(r[36]), "=r"(r[37]), "=r"(r[38]), "=r"(r[39]), "=r"(r[40]), "=r"(r[41]), "=r"(r[42]), "=r"(r[43]), "=r"(r[44]), "=r"(r[45]), "=r"(r[46]), "=r"(r[47]), "=r"(r[48]), "=r"(r[49]), "=r"(r[50]), "=r"(r[51]), "=r"(r[52]), "=r"(r[53]), "=r"(r[54]), "=r"(r[55]), "=r"(r[56]), "=r"(r[57]), "=r"(r[58]), "=r"(r[59]), "=r"(r[60]), "=r"(r[61]), "=r"(r[62]), "=r"(r[63])
+                 : "r"(taddr + 32));
+    asm volatile("tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+                 : "=r"(r[64]), "=r"(r[65]), "=r"(r[66]), "=r"(r[67]), "=r"(r[68]), "=r"(r[69]), "=r"(r[70]), "=r"(r[71]), "=r"(r[72]), "=r"(r[73]), "=r"(r[74]), "=r"(r[75]), "=r"(r[76]), "=r"(r[77]), "=r"(r[78]), "=r"(r[79]), "=r"(r[80]), "=r"(r[81]), "=r"(r[82]), "=r"(r[83]), "=r"(r[84]), "=r"(r[85]), "=r"(r[86]), "=r"(r[87]), "=r"(r[88]), "=r"(r[89]), "=r"(r[90]), "=r"(r[91]), "=r"(r[92]), "=r"(r[93]), "=r"(r[94]), "=r"(r[95])
+                 : "r"(taddr + 64));
+    asm volatile("tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+                 : "=r"(r[96]), "=r"(r[97]), "=r"(r[98]), "=r"(r[99]), "=r"(r[100]), "=r"(r[101]), "=r"(r[102]), "=r"(r[103]), "=r"(r[104]), "=r"(r[105]), "=r"(r[106]), "=r"(r[107]), "=r"(r[108]), "=r"(r[109]), "=r"(r[110]), "=r"(r[111]), "=r"(r[112]), "=r"(r[113]), "=r"(r[114]), "=r"(r[115]), "=r"(r[116]), "=r"(r[117]), "=r"(r[118]), "=r"(r[119]), "=r"(r[120]), "=r"(r[121]), "=r"(r[122]), "=r"(r[123]), "=r"(r[124]), "=r"(r[125]), "=r"(r[126]), "=r"(r[127])
+                 : "r"(taddr + 96));
+    asm volatile("tcgen05.wait::ld.sync.aligned;"
+                 : "+r"(r[0]), "+r"(r[1]), "+r"(r[2]), "+r"(r[3]), "+r"(r[4]), "+r"(r[5]), "+r"(r[6]), "+r"(r[7]), "+r"(r[8]), "+r"(r[9]), "+r"(r[10]), "+r"(r[11]), "+r"(r[12]), "+r"(r[13]), "+r"(r[14]), "+r"(r[15]), "+r"(r[16]), "+r"(r[17]), "+r"(r[18]), "+r"(r[19]), "+r"(r[20]), "+r"(r[21]), "+r"(r[22]), "+r"(r[23]), "+r"(r[24]), "+r"(r[25]), "+r"(r[26]), "+r"(r[27]), "+r"(r[28]), "+r"(r[29]), "+r"(r[30]), "+r"(r[31]), "+r"(r[32]), "+r"(r[33]), "+r"(r[34]), "+r"(r[35]), "+r"(r[36]), "+r"(r[37]), "+r"(r[38]), "+r"(r[39]), "+r"(r[40]), "+r"(r[41]), "+r"(r[42]), "+r"(r[43]), "+r"(r[44]), "+r"(r[45]), "+r"(r[46]), "+r"(r[47]), "+r"(r[48]), "+r"(r[49]), "+r"(r[50]), "+r"(r[51]), "+r"(r[52]), "+r"(r[53]), "+r"(r[54]), "+r"(r[55]), "+r"(r[56]), "+r"(r[57]), "+r"(r[58]), "+r"(r[59]), "+r"(r[60]), "+r"(r[61]), "+r"(r[62]), "+r"(r[63]), "+r"(r[64]), "+r"(r[65]), "+r"(r[66]), "+r"(r[67]), "+r"(r[68]), "+r"(r[69]), "+r"(r[70]), "+r"(r[71]), "+r"(r[72]), "+r"(r[73]), "+r"(r[74]), "+r"(r[75]), "+r"(r[76]), "+r"(r[77]), "+r"(r[78]), "+r"(r[79]), "+r"(r[80]), "+r"(r[81]), "+r"(r[82]), "+r"(r[83]), "+r"(r[84]), "+r"(r[85]), "+r"(r[86]), "+r"(r[87]), "+r"(r[88]), "+r"(r[89]), "+r"(r[90]), "+r"(r[91]), "+r"(r[92]), "+r"(r[93]), "+r"(r[94]), "+r"(r[95]), "+r"(r[96]), "+r"(r[97]), "+r"(r[98]), "+r"(r[99]), "+r"(r[100]), "+r"(r[101]), "+r"(r[102]), "+r"(r[103]), "+r"(r[104]), "+r"(r[105]), "+r"(r[106]), "+r"(r[107]), "+r"(r[108]), "+r"(r[109]), "+r"(r[110]), "+r"(r[111]), "+r"(r[112]), "+r"(r[113]), "+r"(r[114]), "+r"(r[115]), "+r"(r[116]), "+r"(r[117]), "+r"(r[118]), "+r"(r[119]), "+r"(r[120]), "+r"(r[121]), "+r"(r[122]), "+r"(r[123]), "+r"(r[124]), "+r"(r[125]), "+r"(r[126]), "+r"(r[127])
+                 :
+                 : "memory");
+#pragma unroll
+    for (int k = 0; k < 128; k++) v[k] = __uint_as_float(r[k]);
+}
+
+__device__ __forceinline__ float ex2(float x) {
+    float y;
+    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+
+__device__ __forceinline__ bool key_visible(uint64_t w0, uint64_t w1, int c) {
+    return ((c < 64 ? w0 : w1) >> (c & 63)) & 1ull;
+}
 
 __global__ void __launch_bounds__(kAttnThreads, 1)
     tree_attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmKc,
@@ -198,22 +244,27 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
     pdl_trigger();
     const uint32_t off = (1024u - (smem_u32(attn_smem_raw) & 1023u)) & 1023u;
     uint8_t* sQ = attn_smem_raw + off;
-    uint8_t* sKV = sQ + kTileBytes;  // stage st: K at st * 2 * kTileBytes, V right after
-    uint8_t* sP = sKV + kKvStages * 2 * kTileBytes;
+    uint8_t* sK = sQ + kTileBytes;                    // [kKStages] K stages
+    uint8_t* sV = sK + kKStages * kTileBytes;         // [kVStages] V stages
+    uint8_t* sP = sV + kVStages * kTileBytes;
     uint64_t* bars = reinterpret_cast<uint64_t*>(sP + kTileBytes);
     uint64_t* q_full = bars;
-    uint64_t* k_full = bars + 1;     // [2]
-    uint64_t* v_full = bars + 3;     // [2]
-    uint64_t* kv_empty = bars + 5;   // [2]
-    uint64_t* s_full = bars + 7;     // [2]
-    uint64_t* s_empty = bars + 9;    // [2]
-    uint64_t* p_full = bars + 11;
-    uint64_t* pv_done = bars + 12;
-    uint64_t* tdown = bars + 13;
-    int* misc = reinterpret_cast<int*>(bars + 16);  // [0] TMEM base, [1] abort, [2] last split
+    uint64_t* k_full = bars + 1;                      // [kKStages]
+    uint64_t* k_empty = k_full + kKStages;            // [kKStages] S of the stage's tile done
+    uint64_t* v_full = k_empty + kKStages;            // [kVStages]
+    uint64_t* v_empty = v_full + kVStages;            // [kVStages] PV of the stage's tile done
+    uint64_t* s_full = v_empty + kVStages;            // [2]
+    uint64_t* s_empty = s_full + 2;                   // [2]
+    uint64_t* p_full = s_empty + 2;
+    uint64_t* pv_done = p_full + 1;
+    uint64_t* tdown = pv_done + 1;
+    uint64_t* q_ready = tdown + 1;                    // queries rotated in place
+    int* misc = reinterpret_cast<int*>(bars + kNumBars);  // [0] TMEM base, [1] abort
     volatile int* abort = &misc[1];
 
-    const int split = blockIdx.x % a.splits;
+    // cluster of `splits` CTAs = one (sequence, kv head, query tile); the
+    // cluster rank is the key-range split
+    const int split = a.splits > 1 ? static_cast<int>(cluster_ctarank()) : 0;
     const int blk = blockIdx.x / a.splits;
     const int qt = blk % a.nqt;
     const int kvh = (blk / a.nqt) % a.Hkv;
@@ -223,18 +274,23 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
 
     if (threadIdx.x == 0) {
         mbar_init(q_full, 1);
-        for (int i = 0; i < 2; i++) {
+        for (int i = 0; i < kKStages; i++) {
             mbar_init(&k_full[i], 1);
+            mbar_init(&k_empty[i], 1);
+        }
+        for (int i = 0; i < kVStages; i++) {
             mbar_init(&v_full[i], 1);
-            mbar_init(&kv_empty[i], 1);
+            mbar_init(&v_empty[i], 1);
+        }
+        for (int i = 0; i < 2; i++) {
             mbar_init(&s_full[i], 1);
             mbar_init(&s_empty[i], kSoftThreads);
         }
         mbar_init(p_full, kSoftThreads);
         mbar_init(pv_done, 1);
         mbar_init(tdown, 1);
+        mbar_init(q_ready, kSoftThreads);
         misc[1] = 0;
-        misc[2] = 0;
         fence_mbar_init();
     }
     if (warp == 1) {
@@ -245,127 +301,169 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = static_cast<uint32_t>(misc[0]);
-    pdl_wait();  // rotated queries / keys and the tree arrays come from earlier kernels
+    pdl_wait();  // the key table, rotated keys and the tree arrays come from earlier kernels
 
     const int nn = min(max(__ldg(a.n_nodes + s), 0), a.B);
     const int qlast = min(q0 + a.qpt, nn) - 1;  // last tree row of this CTA with a query (-1: none)
     const int T = qlast >= 0 ? a.nct + qlast / kKeys + 1 : 0;
-    const int j0 = static_cast<int>((static_cast<long long>(split) * T) / a.splits);
-    const int nt = static_cast<int>((static_cast<long long>(split + 1) * T) / a.splits) - j0;
+    const int j0 = (split * T) / a.splits;
+    const int nt = ((split + 1) * T) / a.splits - j0;
+
+    // softmax state (warps 2-5), kept for the epilogue
+    const int qd = warp & 3;
+    const int r = qd * 32 + lane;  // query row = TMEM lane
+    const int b = q0 + r / a.G, g = r % a.G;
+    const bool row_ok = b < nn;
+    const uint32_t tl = tmem + (static_cast<uint32_t>(qd * 32) << 16);
+    float m_run = -INFINITY, l = 0.0f;
+    bool ok = true;
 
     if (warp == 0) {
         // ---------------------------------------------------------- producer
         if (lane == 0 && nt > 0) {
             const uint64_t pol_q = l2_policy_evict_first();
             const uint64_t pol_kv = l2_policy_evict_last();  // re-read by the other query tiles
-            const int qrow = ((s * a.Hkv + kvh) * a.B + q0) * a.G;
+            // rows (tree row q0 + r / G, head kvh * G + r % G)
             mbar_arrive_expect_tx(q_full, kTileBytes);
-            tma_load_2d(sQ, &tmQ, q_full, 0, qrow, pol_q);
-            tma_load_2d(sQ + kHalf, &tmQ, q_full, 64, qrow, pol_q);
-            int issued = 0;
-            for (int i = 0; i < nt; i++) {
-                const int st = i & 1;
-                const uint32_t u = static_cast<uint32_t>(i >> 1);
-                if (!mbar_wait(&kv_empty[st], (u & 1u) ^ 1u, abort)) {
-                    attn_timeout(a.status, abort);
-                    break;
-                }
+            tma_load_4d(sQ, &tmQ, q_full, 0, kvh * a.G, q0, s, pol_q);
+            tma_load_4d(sQ + kHalf, &tmQ, q_full, 64, kvh * a.G, q0, s, pol_q);
+            // K runs up to kKStages tiles ahead, V up to kVStages: issue
+            // whichever is due, K first
+            int kdone = 0, vdone = 0;
+            while ((kdone < nt || vdone < nt) && !*abort) {
+                const bool do_k = kdone < nt && kdone < vdone + kKStages;
+                const int i = do_k ? kdone : vdone;
                 const int j = j0 + i;
                 const bool ctx = j < a.nct;
                 const int key0 = (ctx ? j : j - a.nct) * kKeys;
-                const CUtensorMap* mk = ctx ? &tmKc : &tmKt;
-                const CUtensorMap* mv = ctx ? &tmVc : &tmVt;
-                uint8_t* sK = sKV + st * 2 * kTileBytes;
-                uint8_t* sV = sK + kTileBytes;
-                mbar_arrive_expect_tx(&k_full[st], kTileBytes);
-                tma_load_4d(sK, mk, &k_full[st], 0, kvh, key0, s, pol_kv);
-                tma_load_4d(sK + kHalf, mk, &k_full[st], 64, kvh, key0, s, pol_kv);
-                mbar_arrive_expect_tx(&v_full[st], kTileBytes);
-                tma_load_4d(sV, mv, &v_full[st], 0, kvh, key0, s, pol_kv);
-                tma_load_4d(sV + kHalf, mv, &v_full[st], 64, kvh, key0, s, pol_kv);
-                issued = i + 1;
+                if (do_k) {
+                    const int st = i % kKStages;
+                    if (!mbar_wait(&k_empty[st], (static_cast<uint32_t>(i / kKStages) & 1u) ^ 1u, abort)) {
+                        attn_timeout(a.status, abort);
+                        break;
+                    }
+                    uint8_t* dk = sK + st * kTileBytes;
+                    mbar_arrive_expect_tx(&k_full[st], kTileBytes);
+                    tma_load_4d(dk, ctx ? &tmKc : &tmKt, &k_full[st], 0, kvh, key0, s, pol_kv);
+                    tma_load_4d(dk + kHalf, ctx ? &tmKc : &tmKt, &k_full[st], 64, kvh, key0, s, pol_kv);
+                    kdone++;
+                } else {
+                    const int st = i % kVStages;
+                    if (!mbar_wait(&v_empty[st], (static_cast<uint32_t>(i / kVStages) & 1u) ^ 1u, abort)) {
+                        attn_timeout(a.status, abort);
+                        break;
+                    }
+                    uint8_t* dv = sV + st * kTileBytes;
+                    mbar_arrive_expect_tx(&v_full[st], kTileBytes);
+                    tma_load_4d(dv, ctx ? &tmVc : &tmVt, &v_full[st], 0, kvh, key0, s, pol_kv);
+                    tma_load_4d(dv + kHalf, ctx ? &tmVc : &tmVt, &v_full[st], 64, kvh, key0, s, pol_kv);
+                    vdone++;
+                }
             }
             if (*abort) {
                 // copies still in flight must land before the CTA exits
                 attn_drain(q_full, 0);
-                for (int i = issued > kKvStages ? issued - kKvStages : 0; i < issued; i++) {
-                    attn_drain(&k_full[i & 1], static_cast<uint32_t>(i >> 1) & 1u);
-                    attn_drain(&v_full[i & 1], static_cast<uint32_t>(i >> 1) & 1u);
-                }
+                for (int i = kdone > kKStages ? kdone - kKStages : 0; i < kdone; i++)
+                    attn_drain(&k_full[i % kKStages], static_cast<uint32_t>(i / kKStages) & 1u);
+                for (int i = vdone > kVStages ? vdone - kVStages : 0; i < vdone; i++)
+                    attn_drain(&v_full[i % kVStages], static_cast<uint32_t>(i / kVStages) & 1u);
             }
         }
     } else if (warp == 1) {
         // ---------------------------------------------------------- MMA issuer
+        // order: S(0), S(1), then per tile i: PV(i) as soon as P(i) is ready,
+        // then S(i+2) into the S buffer softmax(i) has released
         if (lane == 0 && nt > 0) {
             constexpr uint32_t idesc_s = idesc_bf16_f32(kRows, kKeys);
             constexpr uint32_t idesc_pv = idesc_bf16_f32(kRows, kDh) | (1u << 16);  // B (= V) MN-major
             const uint32_t q_addr = smem_u32(sQ), p_addr = smem_u32(sP);
-            bool ok = mbar_wait(q_full, 0, abort);
-            if (!ok) attn_timeout(a.status, abort);
-            tc_fence_after();
+            bool mok = mbar_wait(q_ready, 0, abort);
             auto issue_s = [&](int i) -> bool {
-                const int st = i & 1;
-                const uint32_t u = static_cast<uint32_t>(i >> 1);
-                if (!mbar_wait(&k_full[st], u & 1u, abort) || !mbar_wait(&s_empty[st], (u & 1u) ^ 1u, abort)) {
-                    attn_timeout(a.status, abort);
+                const int sb = i & 1, st = i % kKStages;
+                // S buffer sb was last read by softmax(i - 2)
+                if (!mbar_wait(&k_full[st], static_cast<uint32_t>(i / kKStages) & 1u, abort) ||
+                    !mbar_wait(&s_empty[sb], (static_cast<uint32_t>(i >> 1) & 1u) ^ 1u, abort))
                     return false;
-                }
                 tc_fence_after();
-                const uint32_t k_addr = smem_u32(sKV + st * 2 * kTileBytes);
+                const uint32_t k_addr = smem_u32(sK + st * kTileBytes);
 #pragma unroll
                 for (int kk = 0; kk < kDh / 16; kk++) {
                     const uint32_t o = (kk >> 2) * kHalf + (kk & 3) * 32;
-                    tc_mma_bf16(tmem + st * kKeys, sdesc_sw128(q_addr + o), sdesc_sw128(k_addr + o), idesc_s,
+                    tc_mma_bf16(tmem + sb * kKeys, sdesc_sw128(q_addr + o), sdesc_sw128(k_addr + o), idesc_s,
                                 kk > 0 ? 1u : 0u);
                 }
-                tc_commit(&s_full[st]);
+                tc_commit(&s_full[sb]);
+                tc_commit(&k_empty[st]);
                 return true;
             };
-            auto issue_pv = [&](int i) -> bool {
-                const int st = i & 1;
+            if (mok) tc_fence_after();
+            if (mok) mok = issue_s(0);
+            if (mok && nt > 1) mok = issue_s(1);
+            for (int i = 0; i < nt && mok; i++) {
+                const int st = i % kVStages;
                 if (!mbar_wait(p_full, static_cast<uint32_t>(i) & 1u, abort) ||
-                    !mbar_wait(&v_full[st], static_cast<uint32_t>(i >> 1) & 1u, abort)) {
-                    attn_timeout(a.status, abort);
-                    return false;
+                    !mbar_wait(&v_full[st], static_cast<uint32_t>(i / kVStages) & 1u, abort)) {
+                    mok = false;
+                    break;
                 }
                 tc_fence_after();
-                const uint32_t v_addr = smem_u32(sKV + st * 2 * kTileBytes + kTileBytes);
+                const uint32_t v_addr = smem_u32(sV + st * kTileBytes);
 #pragma unroll
                 for (int kk = 0; kk < kKeys / 16; kk++) {
                     const uint32_t o = (kk >> 2) * kHalf + (kk & 3) * 32;
                     tc_mma_bf16(tmem + kOCol, sdesc_sw128(p_addr + o), sdesc_sw128_mn(v_addr + kk * 2048, kHalf),
                                 idesc_pv, (i > 0 || kk > 0) ? 1u : 0u);
                 }
-                tc_commit(&kv_empty[st]);
+                tc_commit(&v_empty[st]);
                 tc_commit(pv_done);
-                return true;
-            };
-            if (ok) ok = issue_s(0);
-            for (int i = 1; i < nt && ok; i++) {
-                ok = issue_s(i);
-                if (ok) ok = issue_pv(i - 1);
+                if (i + 2 < nt) mok = issue_s(i + 2);
             }
-            if (ok) ok = issue_pv(nt - 1);
-            if (!ok) {
+            if (!mok) {
+                attn_timeout(a.status, abort);
                 tc_commit(tdown);
                 attn_drain(tdown, 0);
             }
         }
     } else {
         // ---------------------------------------------------------- softmax
-        const int qd = warp & 3;
-        const int r = qd * 32 + lane;          // query row = TMEM lane
-        const int b = q0 + r / a.G, g = r % a.G;
-        const bool row_ok = b < nn;
-        const uint32_t tl = tmem + (static_cast<uint32_t>(qd * 32) << 16);
         uint8_t* prow = sP + r * 128;
         const uint32_t swz = static_cast<uint32_t>(r & 7);
-        float m_run = -INFINITY, l = 0.0f;
-        bool ok = true;
-        for (int i = 0; i < nt; i++) {
+        if (nt > 0) {
+            // RoPE of this thread's query row, in place: element t of the
+            // first 64 and element t of the second 64 sit at the same
+            // swizzled position of the two 16 KB halves
+            if (!warp_wait(q_full, 0, abort)) {
+                attn_timeout(a.status, abort);
+                ok = false;
+            } else if (b < a.B) {
+                const float4* cs = reinterpret_cast<const float4*>(a.cs + (static_cast<size_t>(s) * a.B + b) * (kDh / 2));
+#pragma unroll
+                for (int c = 0; c < 8; c++) {
+                    uint8_t* p1 = sQ + r * 128 + ((static_cast<uint32_t>(c) ^ swz) << 4);
+                    uint4 x1 = *reinterpret_cast<const uint4*>(p1);
+                    uint4 x2 = *reinterpret_cast<const uint4*>(p1 + kHalf);
+                    uint32_t* u1 = reinterpret_cast<uint32_t*>(&x1);
+                    uint32_t* u2 = reinterpret_cast<uint32_t*>(&x2);
+#pragma unroll
+                    for (int e = 0; e < 4; e++) {
+                        const float4 f = __ldg(cs + c * 4 + e);  // (cos, sin) of pairs 8c+2e, 8c+2e+1
+                        const __nv_bfloat162 h1 = *reinterpret_cast<const __nv_bfloat162*>(&u1[e]);
+                        const __nv_bfloat162 h2 = *reinterpret_cast<const __nv_bfloat162*>(&u2[e]);
+                        const float a0 = __low2float(h1), a1 = __high2float(h1);
+                        const float b0 = __low2float(h2), b1 = __high2float(h2);
+                        u1[e] = pack_bf16(a0 * f.x - b0 * f.y, a1 * f.z - b1 * f.w);
+                        u2[e] = pack_bf16(b0 * f.x + a0 * f.y, b1 * f.z + a1 * f.w);
+                    }
+                    *reinterpret_cast<uint4*>(p1) = x1;
+                    *reinterpret_cast<uint4*>(p1 + kHalf) = x2;
+                }
+            }
+            fence_async_smem();
+            mbar_arrive(q_ready);
+        }
+        for (int i = 0; i < nt && ok; i++) {
             const int j = j0 + i;
-            const int st = i & 1;
-            const uint32_t u = static_cast<uint32_t>(i >> 1);
+            const int sb = i & 1;
             // visible keys of this row in the tile, as two 64-bit words
             uint64_t w0 = 0ull, w1 = 0ull;
             if (row_ok) {
@@ -388,30 +486,33 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
                     w1 &= (1ull << (kvalid - 64)) - 1ull;
                 }
             }
-            if (!warp_wait(&s_full[st], u & 1u, abort)) {
+            const bool full = __all_sync(0xFFFFFFFFu, (w0 & w1) == ~0ull);  // whole warp sees every key
+            if (!warp_wait(&s_full[sb], static_cast<uint32_t>(i >> 1) & 1u, abort)) {
                 attn_timeout(a.status, abort);
                 ok = false;
                 break;
             }
             tc_fence_after();
-            const uint32_t ts = tl + st * kKeys;
+            float sv[kKeys];
+            tmem_ld128(tl + sb * kKeys, sv);
+            // S is in registers: the buffer is free for S(i + 2)
+            tc_fence_before();
+            mbar_arrive(&s_empty[sb]);
             float mx = -INFINITY;
+            if (full) {
 #pragma unroll
-            for (int c0 = 0; c0 < kKeys; c0 += 32) {
-                float va[16], vb[16];
-                tmem_ld16_pair(ts + c0, ts + c0 + 16, va, vb);
-                const uint64_t w = c0 < 64 ? w0 : w1;
-                const int sh = c0 & 63;
+                for (int c = 0; c < kKeys; c += 2) mx = fmaxf(mx, fmaxf(sv[c], sv[c + 1]));
+            } else {
 #pragma unroll
-                for (int e = 0; e < 16; e++) {
-                    if ((w >> (sh + e)) & 1ull) mx = fmaxf(mx, va[e]);
-                    if ((w >> (sh + 16 + e)) & 1ull) mx = fmaxf(mx, vb[e]);
+                for (int c = 0; c < kKeys; c++) {
+                    if (!key_visible(w0, w1, c)) sv[c] = -INFINITY;
+                    mx = fmaxf(mx, sv[c]);
                 }
             }
             const float mx2 = mx * a.sl2;
             const bool resc = mx2 > m_run + kRescaleSlack;
             const float m_new = resc ? mx2 : m_run;
-            const float alpha = resc ? exp2f(m_run - m_new) : 1.0f;
+            const float alpha = resc ? ex2(m_run - m_new) : 1.0f;
             if (i > 0) {
                 // PV of the previous tile must be done before P or O is touched
                 if (!warp_wait(pv_done, static_cast<uint32_t>(i - 1) & 1u, abort)) {
@@ -434,41 +535,25 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
             }
             l *= alpha;
             m_run = m_new;
-            // P = exp2(s * scale * log2 e - m) as bf16 into the swizzled K-major P tile
+            // P = 2^(s * scale * log2 e - m) as bf16 into the swizzled K-major P
+            // tile; masked keys hold -inf and give 0 (so does every key of a
+            // row that has seen no visible key yet: m = -inf)
+            const float nm = m_run == -INFINITY ? 0.0f : -m_run;
+            float lsum = 0.0f;
 #pragma unroll
-            for (int c0 = 0; c0 < kKeys; c0 += 32) {
-                float va[16], vb[16];
-                tmem_ld16_pair(ts + c0, ts + c0 + 16, va, vb);
-                const uint64_t w = c0 < 64 ? w0 : w1;
-                const int sh = c0 & 63;
-                uint32_t pk[16];
+            for (int c0 = 0; c0 < kKeys; c0 += 8) {
+                float p[8];
 #pragma unroll
-                for (int e = 0; e < 16; e += 2) {
-                    const float p0 = ((w >> (sh + e)) & 1ull) ? exp2f(fmaf(va[e], a.sl2, -m_run)) : 0.0f;
-                    const float p1 = ((w >> (sh + e + 1)) & 1ull) ? exp2f(fmaf(va[e + 1], a.sl2, -m_run)) : 0.0f;
-                    const float p2 = ((w >> (sh + 16 + e)) & 1ull) ? exp2f(fmaf(vb[e], a.sl2, -m_run)) : 0.0f;
-                    const float p3 =
-                        ((w >> (sh + 16 + e + 1)) & 1ull) ? exp2f(fmaf(vb[e + 1], a.sl2, -m_run)) : 0.0f;
-                    pk[e / 2] = pack_bf16(p0, p1);
-                    pk[8 + e / 2] = pack_bf16(p2, p3);
+                for (int e = 0; e < 8; e++) {
+                    p[e] = ex2(fmaf(sv[c0 + e], a.sl2, nm));
+                    lsum += p[e];
                 }
-                // the sum uses the rounded weights the tensor core multiplies
-#pragma unroll
-                for (int e = 0; e < 16; e++) {
-                    const __nv_bfloat162 h = *reinterpret_cast<const __nv_bfloat162*>(&pk[e]);
-                    l += __low2float(h) + __high2float(h);
-                }
-                // 32 keys = four 16-byte chunks of the 128-byte row of swizzle column c0 / 64
-                uint8_t* col = prow + (c0 >> 6) * kHalf;
-                const uint32_t ch0 = static_cast<uint32_t>((c0 & 63) >> 3);
-#pragma unroll
-                for (int q = 0; q < 4; q++) {
-                    uint4 v = make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]);
-                    *reinterpret_cast<uint4*>(col + (((ch0 + q) ^ swz) << 4)) = v;
-                }
+                const uint4 v = make_uint4(pack_bf16(p[0], p[1]), pack_bf16(p[2], p[3]), pack_bf16(p[4], p[5]),
+                                           pack_bf16(p[6], p[7]));
+                *reinterpret_cast<uint4*>(prow + (c0 >> 6) * kHalf +
+                                          (((static_cast<uint32_t>((c0 & 63) >> 3)) ^ swz) << 4)) = v;
             }
-            tc_fence_before();
-            mbar_arrive(&s_empty[st]);
+            l += lsum;
             fence_async_smem();
             mbar_arrive(p_full);
         }
@@ -479,91 +564,100 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
             }
             tc_fence_after();
         }
-        const int h = kvh * a.G + g;
-        if (a.splits == 1) {
-            if (ok) {
-                float* orow = a.out + ((static_cast<size_t>(s) * a.B + b) * a.Hq + h) * kDh;
-                const bool have = nt > 0;
-                const float inv = (row_ok && l > 0.0f) ? 1.0f / l : 0.0f;
+    }
+
+    const int h = kvh * a.G + g;
+    if (a.splits == 1) {
+        if (warp >= 2 && ok) {
+            float* orow = a.out + ((static_cast<size_t>(s) * a.B + b) * a.Hq + h) * kDh;
+            const float inv = (row_ok && l > 0.0f) ? 1.0f / l : 0.0f;
 #pragma unroll
-                for (int c0 = 0; c0 < kDh; c0 += 16) {
-                    float o[16];
-                    if (have) {
-                        tmem_ld16(tl + kOCol + c0, o);
-                    } else {
-#pragma unroll
-                        for (int e = 0; e < 16; e++) o[e] = 0.0f;
-                    }
-                    if (b < a.B) {
-#pragma unroll
-                        for (int e = 0; e < 16; e += 4)
-                            *reinterpret_cast<float4*>(orow + c0 + e) =
-                                make_float4(o[e] * inv, o[e + 1] * inv, o[e + 2] * inv, o[e + 3] * inv);
-                    }
-                }
-            }
-        } else {
-            // partial of this split: (m, l) and O unnormalised, column-major so
-            // that a warp's 32 rows are one 128-byte line.  Every softmax warp
-            // reaches both named barriers, also after a timeout.
-            const size_t pidx = static_cast<size_t>(blk) * a.splits + split;
-            a.part_ml[pidx * kRows + r] = make_float2(m_run, (ok && nt > 0) ? l : 0.0f);
-            if (ok && nt > 0) {
-                float* po = a.part_o + pidx * kDh * kRows + r;
-#pragma unroll
-                for (int c0 = 0; c0 < kDh; c0 += 16) {
-                    float o[16];
+            for (int c0 = 0; c0 < kDh; c0 += 16) {
+                float o[16];
+                if (nt > 0) {
                     tmem_ld16(tl + kOCol + c0, o);
+                } else {
 #pragma unroll
-                    for (int e = 0; e < 16; e++) po[(c0 + e) * kRows] = o[e];
+                    for (int e = 0; e < 16; e++) o[e] = 0.0f;
                 }
-            }
-            __threadfence();
-            named_bar_sync(kEpiBarrier, kSoftThreads);
-            if (r == 0) {
-                const int tk = atomicAdd(&a.ticket[blk], 1);
-                misc[2] = tk == a.splits - 1;
-                if (tk == a.splits - 1) a.ticket[blk] = 0;
-            }
-            named_bar_sync(kEpiBarrier, kSoftThreads);
-            if (misc[2]) {
-                __threadfence();
-                // merge the splits in order: O = sum_p 2^(m_p - M) O_p / sum_p 2^(m_p - M) l_p
-                const size_t p0 = static_cast<size_t>(blk) * a.splits;
-                float M = -INFINITY;
-                for (int p = 0; p < a.splits; p++) {
-                    const float2 ml = __ldcg(a.part_ml + (p0 + p) * kRows + r);
-                    if (ml.y > 0.0f) M = fmaxf(M, ml.x);
-                }
-                float wsum = 0.0f;
-                float wp[kMaxSplits];
-#pragma unroll
-                for (int p = 0; p < kMaxSplits; p++) {
-                    wp[p] = 0.0f;
-                    if (p < a.splits) {
-                        const float2 ml = __ldcg(a.part_ml + (p0 + p) * kRows + r);
-                        if (ml.y > 0.0f) {
-                            wp[p] = exp2f(ml.x - M);
-                            wsum += wp[p] * ml.y;
-                        }
-                    }
-                }
-                const float inv = (row_ok && wsum > 0.0f) ? 1.0f / wsum : 0.0f;
                 if (b < a.B) {
-                    float* orow = a.out + ((static_cast<size_t>(s) * a.B + b) * a.Hq + h) * kDh;
-                    for (int c0 = 0; c0 < kDh; c0 += 4) {
-                        float o[4] = {0.0f, 0.0f, 0.0f, 0.0f};
 #pragma unroll
-                        for (int p = 0; p < kMaxSplits; p++) {
-                            if (p < a.splits && wp[p] != 0.0f) {
-                                const float* po = a.part_o + (p0 + p) * kDh * kRows + r;
+                    for (int e = 0; e < 16; e += 4)
+                        *reinterpret_cast<float4*>(orow + c0 + e) =
+                            make_float4(o[e] * inv, o[e + 1] * inv, o[e + 2] * inv, o[e + 3] * inv);
+                }
+            }
+        }
+    } else {
+        // Split key range.  Columns are owned in groups of 4: CTA j merges
+        // [c_lo(j), c_hi(j)).  After a cluster barrier (every CTA is past its
+        // main loop, so the K ring and P tile are free), every CTA p pushes,
+        // with 16-byte stores into the peers' shared memory, its (m, l) row
+        // to every peer and its unnormalised O row slices to their owners
+        // (row-major, row stride padded to an odd number of 16-byte units:
+        // conflict-free); after a second barrier CTA j merges locally, in
+        // rank order: O = sum_p 2^(m_p - M) O_p / sum_p 2^(m_p - M) l_p.
+        float* rbuf = reinterpret_cast<float*>(sK);     // [p][128 rows][stride]
+        float2* rml = reinterpret_cast<float2*>(sP);    // [p][128 rows]
+        __syncwarp();
+        cluster_sync_all();
+        if (warp >= 2) {
+            const bool have = ok && nt > 0;
+            for (int jj = 0; jj < a.splits; jj++)
+                st_cluster_f32x2(smem_u32(rml + split * kRows + r), jj, m_run, have ? l : 0.0f);
+            if (have) {
+                float o[kDh];
+                tmem_ld128(tl + kOCol, o);
+                for (int jj = 0; jj < a.splits; jj++) {
+                    const int lo = slice_lo(jj, a.splits), ncol = slice_lo(jj + 1, a.splits) - lo;
+                    const int stride = slice_stride(ncol);
+                    const uint32_t dst = smem_u32(rbuf + (split * kRows + r) * stride);
 #pragma unroll
-                                for (int e = 0; e < 4; e++) o[e] += wp[p] * __ldcg(po + (c0 + e) * kRows);
-                            }
-                        }
-                        *reinterpret_cast<float4*>(orow + c0) =
-                            make_float4(o[0] * inv, o[1] * inv, o[2] * inv, o[3] * inv);
+                    for (int c = 0; c < kDh; c += 4)
+                        if (c >= lo && c < lo + ncol)
+                            st_cluster_f32x4(dst + (c - lo) * 4, jj, o[c], o[c + 1], o[c + 2], o[c + 3]);
+                }
+            }
+        }
+        __syncwarp();
+        cluster_sync_all();  // every push has landed
+        if (warp >= 2) {
+            const int c_lo = slice_lo(split, a.splits), ncol = slice_lo(split + 1, a.splits) - c_lo;
+            const int stride = slice_stride(ncol);
+            float M = -INFINITY;
+            for (int p = 0; p < a.splits; p++) {
+                const float2 ml = rml[p * kRows + r];
+                if (ml.y > 0.0f) M = fmaxf(M, ml.x);
+            }
+            float wp[kMaxSplits];
+            float L = 0.0f;
+#pragma unroll
+            for (int p = 0; p < kMaxSplits; p++) {
+                wp[p] = 0.0f;
+                if (p < a.splits) {
+                    const float2 ml = rml[p * kRows + r];
+                    if (ml.y > 0.0f) {
+                        wp[p] = ex2(ml.x - M);
+                        L += wp[p] * ml.y;
                     }
+                }
+            }
+            const float inv = (row_ok && L > 0.0f) ? 1.0f / L : 0.0f;
+            if (b < a.B) {
+                float* orow = a.out + ((static_cast<size_t>(s) * a.B + b) * a.Hq + h) * kDh + c_lo;
+                for (int c = 0; c < ncol; c += 4) {
+                    float4 o = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+#pragma unroll
+                    for (int p = 0; p < kMaxSplits; p++) {
+                        if (wp[p] != 0.0f) {
+                            const float4 v = *reinterpret_cast<const float4*>(rbuf + (p * kRows + r) * stride + c);
+                            o.x += wp[p] * v.x;
+                            o.y += wp[p] * v.y;
+                            o.z += wp[p] * v.z;
+                            o.w += wp[p] * v.w;
+                        }
+                    }
+                    *reinterpret_cast<float4*>(orow + c) = make_float4(o.x * inv, o.y * inv, o.z * inv, o.w * inv);
                 }
             }
         }
@@ -608,7 +702,7 @@ __global__ void __launch_bounds__(kMaskThreads) ancestor_mask_kernel(const int32
 
 struct Plan {
     int G, qpt, nqt, blocks, splits, mw, nct;
-    size_t off_qr, off_kr, off_po, off_ml, off_ticket, total;
+    size_t off_kr, off_cs, total;
 };
 
 size_t align256(size_t x) { return (x + 255) & ~static_cast<size_t>(255); }
@@ -623,7 +717,7 @@ bool valid_cfg(const dart_attn_config* c) {
     if (!(c->rope_theta > 1.0f) || !std::isfinite(c->rope_theta)) return false;
     if (!(c->scale > 0.0f) || !std::isfinite(c->scale)) return false;
     // TMA coordinates and element counts stay in int range
-    if (static_cast<long long>(c->nseq) * c->Hq * c->B > (1ll << 30)) return false;
+    if (static_cast<long long>(c->nseq) * c->B * (c->Hq + c->Hkv) > (1ll << 30)) return false;
     if (static_cast<long long>(c->C) * c->Hkv * kDh > (1ll << 40)) return false;
     return true;
 }
@@ -634,21 +728,12 @@ int sm_count() {
     return n > 0 ? n : 148;
 }
 
-// Splits of the key list: the smallest modelled time ceil(CTAs / SMs) waves
-// x tiles per split, plus one tile for the merge when split.
+// Splits of the key list (= cluster size): as many as keep every CTA in one
+// wave (1 CTA per SM) with at least two key tiles per split.
 int pick_splits(int blocks, int max_tiles, int nsm) {
-    int best = 1;
-    long long best_cost = -1;
-    for (int sp = 1; sp <= kMaxSplits; sp++) {
-        if (sp > 1 && (max_tiles + sp - 1) / sp < 2) break;
-        const long long waves = (static_cast<long long>(blocks) * sp + nsm - 1) / nsm;
-        const long long cost = waves * ((max_tiles + sp - 1) / sp) + (sp > 1 ? 1 : 0);
-        if (best_cost < 0 || cost < best_cost) {
-            best_cost = cost;
-            best = sp;
-        }
-    }
-    return best;
+    int sp = 1;
+    while (sp < kMaxSplits && static_cast<long long>(blocks) * (sp + 1) <= nsm && max_tiles / (sp + 1) >= 2) sp++;
+    return sp;
 }
 
 Plan make_plan(const dart_attn_config* c, int nsm) {
@@ -660,28 +745,26 @@ Plan make_plan(const dart_attn_config* c, int nsm) {
     p.mw = (c->B + 63) / 64;
     p.nct = (c->C + kKeys - 1) / kKeys;
     p.splits = pick_splits(p.blocks, p.nct + (c->B + kKeys - 1) / kKeys, nsm);
-    const size_t qr = static_cast<size_t>(c->nseq) * c->B * c->Hq * kDh * 2;
     const size_t kr = static_cast<size_t>(c->nseq) * c->B * c->Hkv * kDh * 2;
-    const size_t po = p.splits > 1 ? static_cast<size_t>(p.blocks) * p.splits * kDh * kRows * 4 : 0;
-    const size_t ml = p.splits > 1 ? static_cast<size_t>(p.blocks) * p.splits * kRows * 8 : 0;
-    const size_t tk = p.splits > 1 ? static_cast<size_t>(p.blocks) * 4 : 0;
-    p.off_qr = 0;
-    p.off_kr = align256(p.off_qr + qr);
-    p.off_po = align256(p.off_kr + kr);
-    p.off_ml = align256(p.off_po + po);
-    p.off_ticket = align256(p.off_ml + ml);
-    p.total = align256(p.off_ticket + tk);
+    const size_t cs = static_cast<size_t>(c->nseq) * c->B * (kDh / 2) * 8;
+    p.off_kr = 0;
+    p.off_cs = align256(p.off_kr + kr);
+    p.total = align256(p.off_cs + cs);
     return p;
 }
 
-bool encode_2d(CUtensorMap* m, const void* base, uint64_t rows) {
+// Queries [nseq][B][Hq][dh] bf16 with a (64, G heads, qpt rows, 1) box: the
+// 128 box rows are (tree row, head) pairs, heads fastest.
+bool encode_q(CUtensorMap* m, const void* base, int nseq, int B, int Hq, int G, int qpt) {
     EncodeTiledFn fn = tensor_map_encoder();
     if (!fn) return false;
-    cuuint64_t dims[2] = {static_cast<cuuint64_t>(kDh), rows};
-    cuuint64_t strides[1] = {kDh * 2};
-    cuuint32_t box[2] = {64, kRows};
-    cuuint32_t estr[2] = {1, 1};
-    return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
+    cuuint64_t dims[4] = {static_cast<cuuint64_t>(kDh), static_cast<cuuint64_t>(Hq), static_cast<cuuint64_t>(B),
+                          static_cast<cuuint64_t>(nseq)};
+    cuuint64_t strides[3] = {static_cast<cuuint64_t>(kDh) * 2, static_cast<cuuint64_t>(Hq) * kDh * 2,
+                             static_cast<cuuint64_t>(B) * Hq * kDh * 2};
+    cuuint32_t box[4] = {64, static_cast<cuuint32_t>(G), static_cast<cuuint32_t>(qpt), 1};
+    cuuint32_t estr[4] = {1, 1, 1, 1};
+    return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(base), dims, strides, box, estr,
               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
@@ -703,22 +786,14 @@ bool encode_kv(CUtensorMap* m, const void* base, int nseq, int len, int Hkv) {
 
 bool al16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
-}  // namespace
-}  // namespace dart
 
-using namespace dart;
 
-extern "C" {
-
-size_t dart_tree_attention_workspace(const dart_attn_config* cfg) {
-    if (!valid_cfg(cfg)) return 0;
-    return make_plan(cfg, sm_count()).total;
-}
-
-int dart_tree_attention(const dart_attn_config* cfg, const void* q, const void* k_tree, const void* v_tree,
-                        const void* k_ctx, const void* v_ctx, const int32_t* pos_ids, const uint64_t* mask,
-                        const int32_t* n_nodes, float* out, void* workspace, size_t workspace_bytes, int* status,
-                        void* stream) {
+// Validates, then enqueues the pre-pass and the attention kernel; ev[0..2]
+// (optional) are recorded before the pre-pass, between the two and after.
+int enqueue_tree_attention(const dart_attn_config* cfg, const void* q, const void* k_tree, const void* v_tree,
+                           const void* k_ctx, const void* v_ctx, const int32_t* pos_ids, const uint64_t* mask,
+                           const int32_t* n_nodes, float* out, void* workspace, size_t workspace_bytes,
+                           int* status, void* stream, cudaEvent_t* ev) {
     if (!valid_cfg(cfg)) return DART_ERR_INVALID;
     const dart_attn_config& c = *cfg;
     if (!q || !k_tree || !v_tree || !pos_ids || !mask || !n_nodes || !out || !workspace) return DART_ERR_INVALID;
@@ -739,11 +814,11 @@ int dart_tree_attention(const dart_attn_config* cfg, const void* q, const void* 
     if (workspace_bytes < p.total) return DART_ERR_INVALID;
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     uint8_t* ws = static_cast<uint8_t*>(workspace);
-    __nv_bfloat16* qr = reinterpret_cast<__nv_bfloat16*>(ws + p.off_qr);
     __nv_bfloat16* kr = reinterpret_cast<__nv_bfloat16*>(ws + p.off_kr);
+    float2* cs = reinterpret_cast<float2*>(ws + p.off_cs);
 
     CUtensorMap tmQ, tmKc, tmVc, tmKt, tmVt;
-    if (!encode_2d(&tmQ, qr, static_cast<uint64_t>(c.nseq) * c.Hkv * c.B * p.G)) return DART_ERR_CUDA;
+    if (!encode_q(&tmQ, q, c.nseq, c.B, c.Hq, p.G, p.qpt)) return DART_ERR_CUDA;
     if (!encode_kv(&tmKt, kr, c.nseq, c.B, c.Hkv) || !encode_kv(&tmVt, v_tree, c.nseq, c.B, c.Hkv))
         return DART_ERR_CUDA;
     if (c.C > 0) {
@@ -754,18 +829,15 @@ int dart_tree_attention(const dart_attn_config* cfg, const void* q, const void* 
         tmVc = tmVt;
     }
 
-    RopeArgs ra;
+    PrepArgs ra;
     std::memset(&ra, 0, sizeof ra);
     ra.nseq = c.nseq;
     ra.B = c.B;
-    ra.Hq = c.Hq;
     ra.Hkv = c.Hkv;
-    ra.G = p.G;
-    ra.q = static_cast<const __nv_bfloat16*>(q);
     ra.kt = static_cast<const __nv_bfloat16*>(k_tree);
     ra.pos_ids = pos_ids;
-    ra.qr = qr;
     ra.kr = kr;
+    ra.cs = cs;
     for (int t = 0; t < kDh / 2; t++)
         ra.inv_freq[t] = static_cast<float>(std::pow(static_cast<double>(c.rope_theta), -2.0 * t / kDh));
 
@@ -782,26 +854,70 @@ int dart_tree_attention(const dart_attn_config* cfg, const void* q, const void* 
     aa.mw = p.mw;
     aa.nct = p.nct;
     aa.sl2 = static_cast<float>(static_cast<double>(c.scale) * 1.4426950408889634);
+    aa.cs = cs;
     aa.n_nodes = n_nodes;
     aa.mask = mask;
     aa.out = out;
-    aa.part_o = p.splits > 1 ? reinterpret_cast<float*>(ws + p.off_po) : nullptr;
-    aa.part_ml = p.splits > 1 ? reinterpret_cast<float2*>(ws + p.off_ml) : nullptr;
-    aa.ticket = p.splits > 1 ? reinterpret_cast<int*>(ws + p.off_ticket) : nullptr;
     aa.status = status;
 
-    if (p.splits > 1 && cudaMemsetAsync(aa.ticket, 0, static_cast<size_t>(p.blocks) * 4, st) != cudaSuccess)
-        return DART_ERR_CUDA;
-    const long long rope_threads = static_cast<long long>(c.nseq) * c.B * (c.Hq + c.Hkv) * (kDh / 4);
-    const int rope_blocks = static_cast<int>(std::min<long long>((rope_threads + 255) / 256, 8LL * (nsm > 0 ? nsm : 148)));
-    if (launch_pdl(attn_rope_kernel, dim3(rope_blocks), dim3(256), 0, st, ra) != cudaSuccess) return DART_ERR_CUDA;
     if (cudaFuncSetAttribute(tree_attn_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kAttnSmem) !=
         cudaSuccess)
         return DART_ERR_CUDA;
-    if (launch_pdl(tree_attn_kernel, dim3(p.blocks * p.splits), dim3(kAttnThreads), kAttnSmem, st, tmQ, tmKc, tmVc,
-                   tmKt, tmVt, aa) != cudaSuccess)
-        return DART_ERR_CUDA;
+    const int prep_blocks = static_cast<int>(std::min<long long>((static_cast<long long>(c.nseq) * c.B + 7) / 8,
+                                                                 16LL * (nsm > 0 ? nsm : 148)));  // 8 rows per block
+    if (ev && cudaEventRecord(ev[0], st) != cudaSuccess) return DART_ERR_CUDA;
+    if (launch_pdl(attn_prep_kernel, dim3(prep_blocks), dim3(256), 0, st, ra) != cudaSuccess) return DART_ERR_CUDA;
+    if (ev && cudaEventRecord(ev[1], st) != cudaSuccess) return DART_ERR_CUDA;
+    const cudaError_t le =
+        p.splits > 1 ? launch_pdl_cluster(tree_attn_kernel, dim3(p.blocks * p.splits), dim3(kAttnThreads), kAttnSmem,
+                                          st, p.splits, tmQ, tmKc, tmVc, tmKt, tmVt, aa)
+                     : launch_pdl(tree_attn_kernel, dim3(p.blocks), dim3(kAttnThreads), kAttnSmem, st, tmQ, tmKc,
+                                  tmVc, tmKt, tmVt, aa);
+    if (le != cudaSuccess) return DART_ERR_CUDA;
+    if (ev && cudaEventRecord(ev[2], st) != cudaSuccess) return DART_ERR_CUDA;
     return DART_OK;
+}
+
+}  // namespace
+}  // namespace dart
+
+using namespace dart;
+
+extern "C" {
+
+size_t dart_tree_attention_workspace(const dart_attn_config* cfg) {
+    if (!valid_cfg(cfg)) return 0;
+    return make_plan(cfg, sm_count()).total;
+}
+
+
+int dart_tree_attention(const dart_attn_config* cfg, const void* q, const void* k_tree, const void* v_tree,
+                        const void* k_ctx, const void* v_ctx, const int32_t* pos_ids, const uint64_t* mask,
+                        const int32_t* n_nodes, float* out, void* workspace, size_t workspace_bytes, int* status,
+                        void* stream) {
+    return enqueue_tree_attention(cfg, q, k_tree, v_tree, k_ctx, v_ctx, pos_ids, mask, n_nodes, out, workspace,
+                                  workspace_bytes, status, stream, nullptr);
+}
+
+int dart_tree_attention_timed(const dart_attn_config* cfg, const void* q, const void* k_tree, const void* v_tree,
+                              const void* k_ctx, const void* v_ctx, const int32_t* pos_ids, const uint64_t* mask,
+                              const int32_t* n_nodes, float* out, void* workspace, size_t workspace_bytes,
+                              int* status, float* ms_rope, float* ms_attn, void* stream) {
+    if (!ms_rope || !ms_attn) return DART_ERR_INVALID;
+    cudaEvent_t ev[3] = {nullptr, nullptr, nullptr};
+    int rc = DART_OK;
+    for (int i = 0; i < 3 && rc == DART_OK; i++)
+        if (cudaEventCreate(&ev[i]) != cudaSuccess) rc = DART_ERR_CUDA;
+    if (rc == DART_OK)
+        rc = enqueue_tree_attention(cfg, q, k_tree, v_tree, k_ctx, v_ctx, pos_ids, mask, n_nodes, out, workspace,
+                                    workspace_bytes, status, stream, ev);
+    if (rc == DART_OK && cudaEventSynchronize(ev[2]) != cudaSuccess) rc = DART_ERR_CUDA;
+    if (rc == DART_OK && (cudaEventElapsedTime(ms_rope, ev[0], ev[1]) != cudaSuccess ||
+                          cudaEventElapsedTime(ms_attn, ev[1], ev[2]) != cudaSuccess))
+        rc = DART_ERR_CUDA;
+    for (int i = 0; i < 3; i++)
+        if (ev[i]) cudaEventDestroy(ev[i]);
+    return rc;
 }
 
 int dart_ancestor_mask(const int32_t* parents, const int32_t* n_nodes, int nseq, int B, uint64_t* mask,

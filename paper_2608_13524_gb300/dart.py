@@ -79,6 +79,8 @@ def lib():
             "dart_tree_attention_workspace": (C.c_size_t, [C.POINTER(DartAttnConfig)]),
             "dart_tree_attention": (i, [C.POINTER(DartAttnConfig), vp, vp, vp, vp, vp, vp, vp, vp, vp, vp,
                                         C.c_size_t, vp, vp]),
+            "dart_tree_attention_timed": (i, [C.POINTER(DartAttnConfig), vp, vp, vp, vp, vp, vp, vp, vp, vp, vp,
+                                              C.c_size_t, vp, C.POINTER(f), C.POINTER(f), vp]),
             "dart_ancestor_mask": (i, [vp, vp, i, i, vp, vp]),
             "dart_destroy": (None, [vp]),
             "dart_status_string": (C.c_char_p, [i]),
@@ -301,6 +303,20 @@ def dart_tree_attention(acfg: DartAttnConfig, q, k_tree, v_tree, k_ctx, v_ctx, p
                                      _ptr(status), _stream(stream)), "dart_tree_attention")
 
 
+def dart_tree_attention_timed(acfg: DartAttnConfig, q, k_tree, v_tree, k_ctx, v_ctx, pos_ids, mask, n_nodes, out,
+                              workspace, status=None, stream=None):
+    """As dart_tree_attention, then synchronises; returns (ms of the RoPE
+    pre-pass, ms of the attention kernel)."""
+    a, b = C.c_float(), C.c_float()
+    _check(lib().dart_tree_attention_timed(C.byref(acfg), _ptr(q), _ptr(k_tree), _ptr(v_tree), _ptr(k_ctx),
+                                           _ptr(v_ctx), _ptr(pos_ids), _ptr(mask), _ptr(n_nodes), _ptr(out),
+                                           _ptr(workspace),
+                                           C.c_size_t(workspace.numel() * workspace.element_size()),
+                                           _ptr(status), C.byref(a), C.byref(b), _stream(stream)),
+           "dart_tree_attention_timed")
+    return float(a.value), float(b.value)
+
+
 def dart_ancestor_mask(parents, n_nodes, mask, stream=None):
     nseq, B = parents.shape
     _check(lib().dart_ancestor_mask(_ptr(parents), _ptr(n_nodes), int(nseq), int(B), _ptr(mask),
@@ -324,3 +340,7 @@ class TreeAttention:
         dart_tree_attention(self.cfg, q, k_tree, v_tree, k_ctx, v_ctx, pos_ids, mask, n_nodes, self.out,
                             self.workspace, status, stream)
         return self.out
+
+    def timed(self, q, k_tree, v_tree, k_ctx, v_ctx, pos_ids, mask, n_nodes, status=None, stream=None):
+        return dart_tree_attention_timed(self.cfg, q, k_tree, v_tree, k_ctx, v_ctx, pos_ids, mask, n_nodes,
+                                         self.out, self.workspace, status, stream)
