@@ -35,6 +35,7 @@
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 
+#include <atomic>
 #include <cmath>
 #include <cstdint>
 #include <cstring>
@@ -50,8 +51,9 @@ namespace {
 constexpr int kDh = 128;                  // head dimension (two 64-element swizzle columns)
 constexpr int kRows = 128;                // query rows per CTA (MMA M)
 constexpr int kKeys = 128;                // keys per tile (MMA N of S = QK^T, K of O += PV)
-constexpr int kAttnThreads = 192;
-constexpr int kSoftThreads = 128;
+constexpr int kSoftThreads = 256;             // two softmax warpgroups: key / O columns [0,64) and [64,128)
+constexpr int kAttnThreads = 64 + kSoftThreads;
+constexpr int kPairBarrier0 = 2;             // named barriers 2..5: the two warps of one TMEM lane quarter
 constexpr int kKStages = 3;                  // K ring: the S MMA needs K two tiles ahead of its load
 constexpr int kVStages = 2;
 constexpr int kHalf = kRows * 64 * 2;     // 16 KB: 128 rows x 64 bf16, one 128-byte swizzle column
@@ -61,7 +63,7 @@ constexpr int kTmemCols = 512;            // S0 [0,128), S1 [128,256), O [256,38
 constexpr int kOCol = 256;
 constexpr float kRescaleSlack = 8.0f;     // log2 units: P <= 2^8 between rescales
 constexpr int kNumBars = 1 + 2 * kKStages + 2 * kVStages + 4 + 4;
-constexpr int kSmemUsed = kTileBytes * (1 + kKStages + kVStages + 1) + kNumBars * 8 + 4 * 4;  // Q, K/V rings, P, barriers
+constexpr int kSmemUsed = kTileBytes * (1 + kKStages + kVStages + 1) + kNumBars * 8 + 4 * 4 + 2 * 128 * 4 + 8 * 4;  // Q, K/V rings, P, barriers, exchange
 constexpr int kAttnSmem = kSmemUsed + 1024;  // + alignment slack of the 1024-byte swizzle atoms
 
 struct AttnArgs {
@@ -170,60 +172,68 @@ __device__ __forceinline__ uint32_t pack_bf16(float a, float b) {
 
 // ------------------------------------------------------------ RoPE pre-pass
 
-// One warp per tree row (s, b): the (cos, sin) of its position for the 64
-// frequencies (two per lane) go to the table the attention kernel rotates its
-// queries with, and the Hkv key rows of (s, b) are rotated into kr.
+// sin and cos of x (|x| up to ~1e5): Cody-Waite reduction by 2*pi split
+// into two floats (the high part exactly representable, so k * hi is exact
+// inside the fma), then the hardware approximations on [-pi, pi] (absolute
+// error ~2^-21, far below the bf16 rounding of the rotated values).
+__device__ __forceinline__ void sincos_reduced(float x, float* sn, float* cs) {
+    constexpr float kInv2Pi = 0.159154943091895336f;
+    constexpr float k2PiHi = 6.28318548202514648f;  // float(2 pi)
+    constexpr float k2PiLo = -1.74845560e-7f;       // 2 pi - k2PiHi
+    const float k = rintf(x * kInv2Pi);
+    float r = fmaf(-k, k2PiHi, x);
+    r = fmaf(-k, k2PiLo, r);
+    __sincosf(r, sn, cs);
+}
+
+// One warp per tree key row (s, b, kv head) -- every row's loads in flight at
+// once: the row is rotated into kr (two of the 64 frequencies per lane), and
+// the kv-head-0 warp of (s, b) writes the (cos, sin) of its position to the
+// table the attention kernel rotates its queries with.
 __global__ void __launch_bounds__(256) attn_prep_kernel(const PrepArgs a) {
     pdl_trigger();
     pdl_wait();
     const int lane = threadIdx.x & 31, t = lane * 2;
-    const int rows = a.nseq * a.B;
+    const int rows = a.nseq * a.B * a.Hkv;
     const int wstride = gridDim.x * (blockDim.x >> 5);
-    for (int sb = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); sb < rows; sb += wstride) {
+    for (int row = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); row < rows; row += wstride) {
+        const int sb = row / a.Hkv;
+        const size_t off = static_cast<size_t>(row) * kDh;
+        const __nv_bfloat162 x1 = *reinterpret_cast<const __nv_bfloat162*>(a.kt + off + t);
+        const __nv_bfloat162 x2 = *reinterpret_cast<const __nv_bfloat162*>(a.kt + off + t + kDh / 2);
         const float pos = static_cast<float>(__ldg(a.pos_ids + sb));
         float s0, c0, s1, c1;
-        sincosf(pos * a.inv_freq[t], &s0, &c0);
-        sincosf(pos * a.inv_freq[t + 1], &s1, &c1);
-        *reinterpret_cast<float4*>(a.cs + static_cast<size_t>(sb) * (kDh / 2) + t) = make_float4(c0, s0, c1, s1);
-        for (int kvh = 0; kvh < a.Hkv; kvh++) {
-            const size_t row = (static_cast<size_t>(sb) * a.Hkv + kvh) * kDh;
-            const __nv_bfloat162 x1 = *reinterpret_cast<const __nv_bfloat162*>(a.kt + row + t);
-            const __nv_bfloat162 x2 = *reinterpret_cast<const __nv_bfloat162*>(a.kt + row + t + kDh / 2);
-            const float a0 = __low2float(x1), a1 = __high2float(x1);
-            const float b0 = __low2float(x2), b1 = __high2float(x2);
-            *reinterpret_cast<__nv_bfloat162*>(a.kr + row + t) =
-                __floats2bfloat162_rn(a0 * c0 - b0 * s0, a1 * c1 - b1 * s1);
-            *reinterpret_cast<__nv_bfloat162*>(a.kr + row + t + kDh / 2) =
-                __floats2bfloat162_rn(b0 * c0 + a0 * s0, b1 * c1 + a1 * s1);
-        }
+        sincos_reduced(pos * a.inv_freq[t], &s0, &c0);
+        sincos_reduced(pos * a.inv_freq[t + 1], &s1, &c1);
+        if (row % a.Hkv == 0)
+            *reinterpret_cast<float4*>(a.cs + static_cast<size_t>(sb) * (kDh / 2) + t) = make_float4(c0, s0, c1, s1);
+        const float a0 = __low2float(x1), a1 = __high2float(x1);
+        const float b0 = __low2float(x2), b1 = __high2float(x2);
+        *reinterpret_cast<__nv_bfloat162*>(a.kr + off + t) = __floats2bfloat162_rn(a0 * c0 - b0 * s0, a1 * c1 - b1 * s1);
+        *reinterpret_cast<__nv_bfloat162*>(a.kr + off + t + kDh / 2) =
+            __floats2bfloat162_rn(b0 * c0 + a0 * s0, b1 * c1 + a1 * s1);
     }
 }
 
 // ------------------------------------------------------------ attention
 
-// 128 consecutive 32-bit TMEM columns of this thread's lane into registers
-// (four x32 loads, one wait; the registers are tied to the wait so no use can
+// 64 consecutive 32-bit TMEM columns of this thread's lane into registers
+// (two x32 loads, one wait; the registers are tied to the wait so no use can
 // move above it).
-__device__ __forceinline__ void tmem_ld128(uint32_t taddr, float (&v)[128]) {
-    uint32_t r[128];
+__device__ __forceinline__ void tmem_ld64(uint32_t taddr, float (&v)[64]) {
+    uint32_t r[64];
     asm volatile("tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
                  : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
                  : "r"(taddr + 0));
     asm volatile("tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
                  : "=r"(r[32]), "=r"(r[33]), "=r"(r[34]), "=r"(r[35]), "=r"(r[36]), "=r"(r[37]), "=r"(r[38]), "=r"(r[39]), "=r"(r[40]), "=r"(r[41]), "=r"(r[42]), "=r"(r[43]), "=r"(r[44]), "=r"(r[45]), "=r"(r[46]), "=r"(r[47]), "=r"(r[48]), "=r"(r[49]), "=r"(r[50]), "=r"(r[51]), "=r"(r[52]), "=r"(r[53]), "=r"(r[54]), "=r"(r[55]), "=r"(r[56]), "=r"(r[57]), "=r"(r[58]), "=r"(r[59]), "=r"(r[60]), "=r"(r[61]), "=r"(r[62]), "=r"(r[63])
                  : "r"(taddr + 32));
-    asm volatile("tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
-                 : "=r"(r[64]), "=r"(r[65]), "=r"(r[66]), "=r"(r[67]), "=r"(r[68]), "=r"(r[69]), "=r"(r[70]), "=r"(r[71]), "=r"(r[72]), "=r"(r[73]), "=r"(r[74]), "=r"(r[75]), "=r"(r[76]), "=r"(r[77]), "=r"(r[78]), "=r"(r[79]), "=r"(r[80]), "=r"(r[81]), "=r"(r[82]), "=r"(r[83]), "=r"(r[84]), "=r"(r[85]), "=r"(r[86]), "=r"(r[87]), "=r"(r[88]), "=r"(r[89]), "=r"(r[90]), "=r"(r[91]), "=r"(r[92]), "=r"(r[93]), "=r"(r[94]), "=r"(r[95])
-                 : "r"(taddr + 64));
-    asm volatile("tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
-                 : "=r"(r[96]), "=r"(r[97]), "=r"(r[98]), "=r"(r[99]), "=r"(r[100]), "=r"(r[101]), "=r"(r[102]), "=r"(r[103]), "=r"(r[104]), "=r"(r[105]), "=r"(r[106]), "=r"(r[107]), "=r"(r[108]), "=r"(r[109]), "=r"(r[110]), "=r"(r[111]), "=r"(r[112]), "=r"(r[113]), "=r"(r[114]), "=r"(r[115]), "=r"(r[116]), "=r"(r[117]), "=r"(r[118]), "=r"(r[119]), "=r"(r[120]), "=r"(r[121]), "=r"(r[122]), "=r"(r[123]), "=r"(r[124]), "=r"(r[125]), "=r"(r[126]), "=r"(r[127])
-                 : "r"(taddr + 96));
     asm volatile("tcgen05.wait::ld.sync.aligned;"
-                 : "+r"(r[0]), "+r"(r[1]), "+r"(r[2]), "+r"(r[3]), "+r"(r[4]), "+r"(r[5]), "+r"(r[6]), "+r"(r[7]), "+r"(r[8]), "+r"(r[9]), "+r"(r[10]), "+r"(r[11]), "+r"(r[12]), "+r"(r[13]), "+r"(r[14]), "+r"(r[15]), "+r"(r[16]), "+r"(r[17]), "+r"(r[18]), "+r"(r[19]), "+r"(r[20]), "+r"(r[21]), "+r"(r[22]), "+r"(r[23]), "+r"(r[24]), "+r"(r[25]), "+r"(r[26]), "+r"(r[27]), "+r"(r[28]), "+r"(r[29]), "+r"(r[30]), "+r"(r[31]), "+r"(r[32]), "+r"(r[33]), "+r"(r[34]), "+r"(r[35]), "+r"(r[36]), "+r"(r[37]), "+r"(r[38]), "+r"(r[39]), "+r"(r[40]), "+r"(r[41]), "+r"(r[42]), "+r"(r[43]), "+r"(r[44]), "+r"(r[45]), "+r"(r[46]), "+r"(r[47]), "+r"(r[48]), "+r"(r[49]), "+r"(r[50]), "+r"(r[51]), "+r"(r[52]), "+r"(r[53]), "+r"(r[54]), "+r"(r[55]), "+r"(r[56]), "+r"(r[57]), "+r"(r[58]), "+r"(r[59]), "+r"(r[60]), "+r"(r[61]), "+r"(r[62]), "+r"(r[63]), "+r"(r[64]), "+r"(r[65]), "+r"(r[66]), "+r"(r[67]), "+r"(r[68]), "+r"(r[69]), "+r"(r[70]), "+r"(r[71]), "+r"(r[72]), "+r"(r[73]), "+r"(r[74]), "+r"(r[75]), "+r"(r[76]), "+r"(r[77]), "+r"(r[78]), "+r"(r[79]), "+r"(r[80]), "+r"(r[81]), "+r"(r[82]), "+r"(r[83]), "+r"(r[84]), "+r"(r[85]), "+r"(r[86]), "+r"(r[87]), "+r"(r[88]), "+r"(r[89]), "+r"(r[90]), "+r"(r[91]), "+r"(r[92]), "+r"(r[93]), "+r"(r[94]), "+r"(r[95]), "+r"(r[96]), "+r"(r[97]), "+r"(r[98]), "+r"(r[99]), "+r"(r[100]), "+r"(r[101]), "+r"(r[102]), "+r"(r[103]), "+r"(r[104]), "+r"(r[105]), "+r"(r[106]), "+r"(r[107]), "+r"(r[108]), "+r"(r[109]), "+r"(r[110]), "+r"(r[111]), "+r"(r[112]), "+r"(r[113]), "+r"(r[114]), "+r"(r[115]), "+r"(r[116]), "+r"(r[117]), "+r"(r[118]), "+r"(r[119]), "+r"(r[120]), "+r"(r[121]), "+r"(r[122]), "+r"(r[123]), "+r"(r[124]), "+r"(r[125]), "+r"(r[126]), "+r"(r[127])
+                 : "+r"(r[0]), "+r"(r[1]), "+r"(r[2]), "+r"(r[3]), "+r"(r[4]), "+r"(r[5]), "+r"(r[6]), "+r"(r[7]), "+r"(r[8]), "+r"(r[9]), "+r"(r[10]), "+r"(r[11]), "+r"(r[12]), "+r"(r[13]), "+r"(r[14]), "+r"(r[15]), "+r"(r[16]), "+r"(r[17]), "+r"(r[18]), "+r"(r[19]), "+r"(r[20]), "+r"(r[21]), "+r"(r[22]), "+r"(r[23]), "+r"(r[24]), "+r"(r[25]), "+r"(r[26]), "+r"(r[27]), "+r"(r[28]), "+r"(r[29]), "+r"(r[30]), "+r"(r[31]), "+r"(r[32]), "+r"(r[33]), "+r"(r[34]), "+r"(r[35]), "+r"(r[36]), "+r"(r[37]), "+r"(r[38]), "+r"(r[39]), "+r"(r[40]), "+r"(r[41]), "+r"(r[42]), "+r"(r[43]), "+r"(r[44]), "+r"(r[45]), "+r"(r[46]), "+r"(r[47]), "+r"(r[48]), "+r"(r[49]), "+r"(r[50]), "+r"(r[51]), "+r"(r[52]), "+r"(r[53]), "+r"(r[54]), "+r"(r[55]), "+r"(r[56]), "+r"(r[57]), "+r"(r[58]), "+r"(r[59]), "+r"(r[60]), "+r"(r[61]), "+r"(r[62]), "+r"(r[63])
                  :
                  : "memory");
 #pragma unroll
-    for (int k = 0; k < 128; k++) v[k] = __uint_as_float(r[k]);
+    for (int k = 0; k < 64; k++) v[k] = __uint_as_float(r[k]);
 }
 
 __device__ __forceinline__ float ex2(float x) {
@@ -309,12 +319,18 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
     const int j0 = (split * T) / a.splits;
     const int nt = ((split + 1) * T) / a.splits - j0;
 
-    // softmax state (warps 2-5), kept for the epilogue
+    // softmax state (warps 2-9), kept for the epilogue.  Warps w and w + 4
+    // share TMEM lane quarter w % 4 (the same 32 query rows); warpgroup wg
+    // handles key columns and O columns [64 wg, 64 wg + 64).
     const int qd = warp & 3;
+    const int wg = warp >= 2 ? (warp - 2) >> 2 : 0;
+    const int cb = wg * 64;
     const int r = qd * 32 + lane;  // query row = TMEM lane
     const int b = q0 + r / a.G, g = r % a.G;
     const bool row_ok = b < nn;
     const uint32_t tl = tmem + (static_cast<uint32_t>(qd * 32) << 16);
+    float* xch = reinterpret_cast<float*>(misc + 4);  // [2][128] row max / sum exchange of the two warpgroups
+    int* xok = misc + 4 + 2 * kRows;                   // [2][4] per-warp "no wait failed" exchange
     float m_run = -INFINITY, l = 0.0f;
     bool ok = true;
 
@@ -426,19 +442,22 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
         }
     } else {
         // ---------------------------------------------------------- softmax
-        uint8_t* prow = sP + r * 128;
+        uint8_t* prow = sP + wg * kHalf + r * 128;  // this warpgroup's 64 keys of row r
         const uint32_t swz = static_cast<uint32_t>(r & 7);
+        const int pair_bar = kPairBarrier0 + qd;
         if (nt > 0) {
             // RoPE of this thread's query row, in place: element t of the
             // first 64 and element t of the second 64 sit at the same
-            // swizzled position of the two 16 KB halves
+            // swizzled position of the two 16 KB halves; warpgroup wg
+            // rotates chunks 4 wg .. 4 wg + 3
             if (!warp_wait(q_full, 0, abort)) {
                 attn_timeout(a.status, abort);
                 ok = false;
             } else if (b < a.B) {
                 const float4* cs = reinterpret_cast<const float4*>(a.cs + (static_cast<size_t>(s) * a.B + b) * (kDh / 2));
 #pragma unroll
-                for (int c = 0; c < 8; c++) {
+                for (int cc = 0; cc < 4; cc++) {
+                    const int c = wg * 4 + cc;
                     uint8_t* p1 = sQ + r * 128 + ((static_cast<uint32_t>(c) ^ swz) << 4);
                     uint4 x1 = *reinterpret_cast<const uint4*>(p1);
                     uint4 x2 = *reinterpret_cast<const uint4*>(p1 + kHalf);
@@ -461,87 +480,96 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
             fence_async_smem();
             mbar_arrive(q_ready);
         }
-        for (int i = 0; i < nt && ok; i++) {
+        for (int i = 0; i < nt; i++) {
             const int j = j0 + i;
             const int sb = i & 1;
-            // visible keys of this row in the tile, as two 64-bit words
-            uint64_t w0 = 0ull, w1 = 0ull;
+            // visible keys of this row among this warpgroup's 64 keys of the tile
+            uint64_t w = 0ull;
             if (row_ok) {
                 int kvalid;
                 if (j < a.nct) {
                     kvalid = min(kKeys, a.C - j * kKeys);
-                    w0 = ~0ull;
-                    w1 = ~0ull;
+                    w = ~0ull;
                 } else {
                     const int t = j - a.nct;
                     kvalid = min(kKeys, nn - t * kKeys);
-                    const uint64_t* mrow = a.mask + (static_cast<size_t>(s) * a.B + b) * a.mw;
-                    w0 = __ldg(mrow + 2 * t);
-                    w1 = 2 * t + 1 < a.mw ? __ldg(mrow + 2 * t + 1) : 0ull;
+                    w = 2 * t + wg < a.mw ? __ldg(a.mask + (static_cast<size_t>(s) * a.B + b) * a.mw + 2 * t + wg) : 0ull;
                 }
-                if (kvalid < 64) {
-                    w0 &= (1ull << kvalid) - 1ull;
-                    w1 = 0ull;
-                } else if (kvalid < 128) {
-                    w1 &= (1ull << (kvalid - 64)) - 1ull;
-                }
+                kvalid -= cb;
+                if (kvalid <= 0)
+                    w = 0ull;
+                else if (kvalid < 64)
+                    w &= (1ull << kvalid) - 1ull;
             }
-            const bool full = __all_sync(0xFFFFFFFFu, (w0 & w1) == ~0ull);  // whole warp sees every key
-            if (!warp_wait(&s_full[sb], static_cast<uint32_t>(i >> 1) & 1u, abort)) {
+            const bool full = __all_sync(0xFFFFFFFFu, w == ~0ull);  // whole warp sees all 64 keys
+            // Both warps of the lane quarter reach both pair barriers of every
+            // iteration and leave the loop at the same point: a failed wait is
+            // exchanged with the row max and acted on after the barriers.
+            if (ok && !warp_wait(&s_full[sb], static_cast<uint32_t>(i >> 1) & 1u, abort)) {
                 attn_timeout(a.status, abort);
                 ok = false;
-                break;
             }
-            tc_fence_after();
-            float sv[kKeys];
-            tmem_ld128(tl + sb * kKeys, sv);
-            // S is in registers: the buffer is free for S(i + 2)
-            tc_fence_before();
-            mbar_arrive(&s_empty[sb]);
+            float sv[64];
             float mx = -INFINITY;
-            if (full) {
+            if (ok) {
+                tc_fence_after();
+                tmem_ld64(tl + sb * kKeys + cb, sv);
+                // S is in registers: the buffer is free for S(i + 2)
+                tc_fence_before();
+                mbar_arrive(&s_empty[sb]);
+                if (full) {
 #pragma unroll
-                for (int c = 0; c < kKeys; c += 2) mx = fmaxf(mx, fmaxf(sv[c], sv[c + 1]));
-            } else {
+                    for (int c = 0; c < 64; c += 2) mx = fmaxf(mx, fmaxf(sv[c], sv[c + 1]));
+                } else {
 #pragma unroll
-                for (int c = 0; c < kKeys; c++) {
-                    if (!key_visible(w0, w1, c)) sv[c] = -INFINITY;
-                    mx = fmaxf(mx, sv[c]);
+                    for (int c = 0; c < 64; c++) {
+                        if (!((w >> c) & 1ull)) sv[c] = -INFINITY;
+                        mx = fmaxf(mx, sv[c]);
+                    }
                 }
             }
+            xch[wg * kRows + r] = mx;
+            if (lane == 0) xok[wg * 4 + qd] = ok ? 1 : 0;
+            named_bar_sync(pair_bar, 64);
+            mx = fmaxf(mx, xch[(1 - wg) * kRows + r]);
+            ok = ok && xok[(1 - wg) * 4 + qd] != 0;
+            named_bar_sync(pair_bar, 64);  // both read before the next tile's write
+            if (!ok) break;
             const float mx2 = mx * a.sl2;
             const bool resc = mx2 > m_run + kRescaleSlack;
             const float m_new = resc ? mx2 : m_run;
             const float alpha = resc ? ex2(m_run - m_new) : 1.0f;
             if (i > 0) {
                 // PV of the previous tile must be done before P or O is touched
+                // (on a timeout this tile is skipped; the pair leaves the loop
+                // together at the next exchange)
                 if (!warp_wait(pv_done, static_cast<uint32_t>(i - 1) & 1u, abort)) {
                     attn_timeout(a.status, abort);
                     ok = false;
-                    break;
+                    continue;
                 }
                 tc_fence_after();
                 if (__any_sync(0xFFFFFFFFu, resc)) {
 #pragma unroll
-                    for (int c0 = 0; c0 < kDh; c0 += 16) {
+                    for (int c0 = 0; c0 < 64; c0 += 16) {
                         float o[16];
-                        tmem_ld16(tl + kOCol + c0, o);
+                        tmem_ld16(tl + kOCol + cb + c0, o);
 #pragma unroll
                         for (int e = 0; e < 16; e++) o[e] *= alpha;
-                        tmem_st16(tl + kOCol + c0, o);
+                        tmem_st16(tl + kOCol + cb + c0, o);
                     }
                     tmem_wait_st();
                 }
             }
             l *= alpha;
             m_run = m_new;
-            // P = 2^(s * scale * log2 e - m) as bf16 into the swizzled K-major P
-            // tile; masked keys hold -inf and give 0 (so does every key of a
-            // row that has seen no visible key yet: m = -inf)
+            // P = 2^(s * scale * log2 e - m) as bf16 into this warpgroup's half
+            // of the swizzled K-major P tile; masked keys hold -inf and give 0
+            // (so does every key of a row that has seen no visible key: m = -inf)
             const float nm = m_run == -INFINITY ? 0.0f : -m_run;
             float lsum = 0.0f;
 #pragma unroll
-            for (int c0 = 0; c0 < kKeys; c0 += 8) {
+            for (int c0 = 0; c0 < 64; c0 += 8) {
                 float p[8];
 #pragma unroll
                 for (int e = 0; e < 8; e++) {
@@ -550,8 +578,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
                 }
                 const uint4 v = make_uint4(pack_bf16(p[0], p[1]), pack_bf16(p[2], p[3]), pack_bf16(p[4], p[5]),
                                            pack_bf16(p[6], p[7]));
-                *reinterpret_cast<uint4*>(prow + (c0 >> 6) * kHalf +
-                                          (((static_cast<uint32_t>((c0 & 63) >> 3)) ^ swz) << 4)) = v;
+                *reinterpret_cast<uint4*>(prow + (((static_cast<uint32_t>(c0 >> 3)) ^ swz) << 4)) = v;
             }
             l += lsum;
             fence_async_smem();
@@ -564,18 +591,23 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
             }
             tc_fence_after();
         }
+        // the row sum is split over the two warpgroups
+        xch[wg * kRows + r] = l;
+        named_bar_sync(pair_bar, 64);
+        l += xch[(1 - wg) * kRows + r];
+        ok = __all_sync(0xFFFFFFFFu, ok);
     }
 
     const int h = kvh * a.G + g;
     if (a.splits == 1) {
         if (warp >= 2 && ok) {
-            float* orow = a.out + ((static_cast<size_t>(s) * a.B + b) * a.Hq + h) * kDh;
+            float* orow = a.out + ((static_cast<size_t>(s) * a.B + b) * a.Hq + h) * kDh + cb;
             const float inv = (row_ok && l > 0.0f) ? 1.0f / l : 0.0f;
 #pragma unroll
-            for (int c0 = 0; c0 < kDh; c0 += 16) {
+            for (int c0 = 0; c0 < 64; c0 += 16) {
                 float o[16];
                 if (nt > 0) {
-                    tmem_ld16(tl + kOCol + c0, o);
+                    tmem_ld16(tl + kOCol + cb + c0, o);
                 } else {
 #pragma unroll
                     for (int e = 0; e < 16; e++) o[e] = 0.0f;
@@ -603,19 +635,20 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
         cluster_sync_all();
         if (warp >= 2) {
             const bool have = ok && nt > 0;
-            for (int jj = 0; jj < a.splits; jj++)
-                st_cluster_f32x2(smem_u32(rml + split * kRows + r), jj, m_run, have ? l : 0.0f);
+            if (wg == 0)
+                for (int jj = 0; jj < a.splits; jj++)
+                    st_cluster_f32x2(smem_u32(rml + split * kRows + r), jj, m_run, have ? l : 0.0f);
             if (have) {
-                float o[kDh];
-                tmem_ld128(tl + kOCol, o);
+                float o[64];
+                tmem_ld64(tl + kOCol + cb, o);
                 for (int jj = 0; jj < a.splits; jj++) {
                     const int lo = slice_lo(jj, a.splits), ncol = slice_lo(jj + 1, a.splits) - lo;
                     const int stride = slice_stride(ncol);
                     const uint32_t dst = smem_u32(rbuf + (split * kRows + r) * stride);
 #pragma unroll
-                    for (int c = 0; c < kDh; c += 4)
-                        if (c >= lo && c < lo + ncol)
-                            st_cluster_f32x4(dst + (c - lo) * 4, jj, o[c], o[c + 1], o[c + 2], o[c + 3]);
+                    for (int c = 0; c < 64; c += 4)
+                        if (cb + c >= lo && cb + c < lo + ncol)
+                            st_cluster_f32x4(dst + (cb + c - lo) * 4, jj, o[c], o[c + 1], o[c + 2], o[c + 3]);
                 }
             }
         }
@@ -645,7 +678,8 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
             const float inv = (row_ok && L > 0.0f) ? 1.0f / L : 0.0f;
             if (b < a.B) {
                 float* orow = a.out + ((static_cast<size_t>(s) * a.B + b) * a.Hq + h) * kDh + c_lo;
-                for (int c = 0; c < ncol; c += 4) {
+                // the two warpgroups take alternate 4-column groups of the slice
+                for (int c = 4 * wg; c < ncol; c += 8) {
                     float4 o = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
 #pragma unroll
                     for (int p = 0; p < kMaxSplits; p++) {
@@ -786,6 +820,19 @@ bool encode_kv(CUtensorMap* m, const void* base, int nseq, int len, int Hkv) {
 
 bool al16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
+// The kernel's shared-memory opt-in, set once per device (a host call that
+// costs microseconds when repeated on every launch).
+bool attn_attr_set(int dev) {
+    static std::atomic<uint64_t> done{0};
+    const uint64_t bit = dev < 64 ? (1ull << dev) : 0ull;
+    if (bit && (done.load() & bit)) return true;
+    if (cudaFuncSetAttribute(tree_attn_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kAttnSmem) !=
+        cudaSuccess)
+        return false;
+    done.fetch_or(bit);
+    return true;
+}
+
 
 
 // Validates, then enqueues the pre-pass and the attention kernel; ev[0..2]
@@ -860,11 +907,9 @@ int enqueue_tree_attention(const dart_attn_config* cfg, const void* q, const voi
     aa.out = out;
     aa.status = status;
 
-    if (cudaFuncSetAttribute(tree_attn_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kAttnSmem) !=
-        cudaSuccess)
-        return DART_ERR_CUDA;
-    const int prep_blocks = static_cast<int>(std::min<long long>((static_cast<long long>(c.nseq) * c.B + 7) / 8,
-                                                                 16LL * (nsm > 0 ? nsm : 148)));  // 8 rows per block
+    if (!attn_attr_set(dev)) return DART_ERR_CUDA;
+    const int prep_blocks = static_cast<int>(std::min<long long>(
+        (static_cast<long long>(c.nseq) * c.B * c.Hkv + 7) / 8, 16LL * (nsm > 0 ? nsm : 148)));  // 8 rows per block
     if (ev && cudaEventRecord(ev[0], st) != cudaSuccess) return DART_ERR_CUDA;
     if (launch_pdl(attn_prep_kernel, dim3(prep_blocks), dim3(256), 0, st, ra) != cudaSuccess) return DART_ERR_CUDA;
     if (ev && cudaEventRecord(ev[1], st) != cudaSuccess) return DART_ERR_CUDA;
