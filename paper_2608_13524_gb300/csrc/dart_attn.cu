@@ -55,15 +55,16 @@ constexpr int kSoftThreads = 256;             // two softmax warpgroups: key / O
 constexpr int kAttnThreads = 64 + kSoftThreads;
 constexpr int kPairBarrier0 = 2;             // named barriers 2..5: the two warps of one TMEM lane quarter
 constexpr int kKStages = 3;                  // K ring: the S MMA needs K two tiles ahead of its load
-constexpr int kVStages = 2;
+constexpr int kVStages = 3;
 constexpr int kHalf = kRows * 64 * 2;     // 16 KB: 128 rows x 64 bf16, one 128-byte swizzle column
 constexpr int kTileBytes = 2 * kHalf;     // 32 KB: 128 rows x dh bf16
 constexpr int kMaxSplits = 8;                // cluster size limit (portable)
-constexpr int kTmemCols = 512;            // S0 [0,128), S1 [128,256), O [256,384)
+constexpr int kTmemCols = 512;            // S0 [0,128), S1 [128,256), O [256,384), P0 [384,448), P1 [448,512)
 constexpr int kOCol = 256;
+constexpr int kPCol = 384;                // P tiles: 128 keys as 64 columns of bf16 pairs
 constexpr float kRescaleSlack = 8.0f;     // log2 units: P <= 2^8 between rescales
-constexpr int kNumBars = 1 + 2 * kKStages + 2 * kVStages + 4 + 4;
-constexpr int kSmemUsed = kTileBytes * (1 + kKStages + kVStages + 1) + kNumBars * 8 + 4 * 4 + 2 * 128 * 4 + 8 * 4;  // Q, K/V rings, P, barriers, exchange
+constexpr int kNumBars = 1 + 2 * kKStages + 2 * kVStages + 4 + 5;
+constexpr int kSmemUsed = kTileBytes * (1 + kKStages + kVStages) + kNumBars * 8 + 4 * 4 + 2 * 128 * 4 + 8 * 4;  // Q, K/V rings, barriers, exchange
 constexpr int kAttnSmem = kSmemUsed + 1024;  // + alignment slack of the 1024-byte swizzle atoms
 
 struct AttnArgs {
@@ -123,6 +124,29 @@ __device__ __forceinline__ void tmem_st16(uint32_t taddr, const float (&v)[16]) 
         : "memory");
 }
 __device__ __forceinline__ void tmem_wait_st() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
+
+// D[tmem] (+)= A[tmem] * B[smem], bf16 inputs, fp32 accumulation (A: lane =
+// row, K along columns as bf16 pairs).
+__device__ __forceinline__ void tc_mma_bf16_ts(uint32_t tmem_d, uint32_t tmem_a, uint64_t bdesc, uint32_t idesc,
+                                               uint32_t accumulate) {
+    asm volatile(
+        "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+        " tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n}\n" ::"r"(tmem_d),
+        "r"(tmem_a), "l"(bdesc), "r"(idesc), "r"(accumulate)
+        : "memory");
+}
+
+// 32 consecutive 32-bit TMEM columns of this thread's lane from registers.
+__device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t (&v)[32]) {
+    asm volatile(
+        "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,"
+        "%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32};" ::"r"(taddr),
+        "r"(v[0]), "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7]), "r"(v[8]), "r"(v[9]),
+        "r"(v[10]), "r"(v[11]), "r"(v[12]), "r"(v[13]), "r"(v[14]), "r"(v[15]), "r"(v[16]), "r"(v[17]), "r"(v[18]),
+        "r"(v[19]), "r"(v[20]), "r"(v[21]), "r"(v[22]), "r"(v[23]), "r"(v[24]), "r"(v[25]), "r"(v[26]), "r"(v[27]),
+        "r"(v[28]), "r"(v[29]), "r"(v[30]), "r"(v[31])
+        : "memory");
+}
 
 // Generic-proxy shared-memory writes become visible to the tensor core.
 __device__ __forceinline__ void fence_async_smem() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
@@ -242,10 +266,6 @@ __device__ __forceinline__ float ex2(float x) {
     return y;
 }
 
-__device__ __forceinline__ bool key_visible(uint64_t w0, uint64_t w1, int c) {
-    return ((c < 64 ? w0 : w1) >> (c & 63)) & 1ull;
-}
-
 __global__ void __launch_bounds__(kAttnThreads, 1)
     tree_attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmKc,
                      const __grid_constant__ CUtensorMap tmVc, const __grid_constant__ CUtensorMap tmKt,
@@ -256,8 +276,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
     uint8_t* sQ = attn_smem_raw + off;
     uint8_t* sK = sQ + kTileBytes;                    // [kKStages] K stages
     uint8_t* sV = sK + kKStages * kTileBytes;         // [kVStages] V stages
-    uint8_t* sP = sV + kVStages * kTileBytes;
-    uint64_t* bars = reinterpret_cast<uint64_t*>(sP + kTileBytes);
+    uint64_t* bars = reinterpret_cast<uint64_t*>(sV + kVStages * kTileBytes);
     uint64_t* q_full = bars;
     uint64_t* k_full = bars + 1;                      // [kKStages]
     uint64_t* k_empty = k_full + kKStages;            // [kKStages] S of the stage's tile done
@@ -266,8 +285,8 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
     uint64_t* s_full = v_empty + kVStages;            // [2]
     uint64_t* s_empty = s_full + 2;                   // [2]
     uint64_t* p_full = s_empty + 2;
-    uint64_t* pv_done = p_full + 1;
-    uint64_t* tdown = pv_done + 1;
+    uint64_t* pv_done = p_full + 1;                   // [2] PV of a tile using P buffer b done
+    uint64_t* tdown = pv_done + 2;
     uint64_t* q_ready = tdown + 1;                    // queries rotated in place
     int* misc = reinterpret_cast<int*>(bars + kNumBars);  // [0] TMEM base, [1] abort
     volatile int* abort = &misc[1];
@@ -297,7 +316,8 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
             mbar_init(&s_empty[i], kSoftThreads);
         }
         mbar_init(p_full, kSoftThreads);
-        mbar_init(pv_done, 1);
+        mbar_init(&pv_done[0], 1);
+        mbar_init(&pv_done[1], 1);
         mbar_init(tdown, 1);
         mbar_init(q_ready, kSoftThreads);
         misc[1] = 0;
@@ -392,7 +412,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
         if (lane == 0 && nt > 0) {
             constexpr uint32_t idesc_s = idesc_bf16_f32(kRows, kKeys);
             constexpr uint32_t idesc_pv = idesc_bf16_f32(kRows, kDh) | (1u << 16);  // B (= V) MN-major
-            const uint32_t q_addr = smem_u32(sQ), p_addr = smem_u32(sP);
+            const uint32_t q_addr = smem_u32(sQ);
             bool mok = mbar_wait(q_ready, 0, abort);
             auto issue_s = [&](int i) -> bool {
                 const int sb = i & 1, st = i % kKStages;
@@ -424,14 +444,13 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
                 }
                 tc_fence_after();
                 const uint32_t v_addr = smem_u32(sV + st * kTileBytes);
+                const uint32_t p_tmem = tmem + kPCol + (i & 1) * (kKeys / 2);
 #pragma unroll
-                for (int kk = 0; kk < kKeys / 16; kk++) {
-                    const uint32_t o = (kk >> 2) * kHalf + (kk & 3) * 32;
-                    tc_mma_bf16(tmem + kOCol, sdesc_sw128(p_addr + o), sdesc_sw128_mn(v_addr + kk * 2048, kHalf),
-                                idesc_pv, (i > 0 || kk > 0) ? 1u : 0u);
-                }
+                for (int kk = 0; kk < kKeys / 16; kk++)  // 16 keys = 8 columns of bf16 pairs
+                    tc_mma_bf16_ts(tmem + kOCol, p_tmem + kk * 8, sdesc_sw128_mn(v_addr + kk * 2048, kHalf), idesc_pv,
+                                   (i > 0 || kk > 0) ? 1u : 0u);
                 tc_commit(&v_empty[st]);
-                tc_commit(pv_done);
+                tc_commit(&pv_done[i & 1]);
                 if (i + 2 < nt) mok = issue_s(i + 2);
             }
             if (!mok) {
@@ -442,7 +461,6 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
         }
     } else {
         // ---------------------------------------------------------- softmax
-        uint8_t* prow = sP + wg * kHalf + r * 128;  // this warpgroup's 64 keys of row r
         const uint32_t swz = static_cast<uint32_t>(r & 7);
         const int pair_bar = kPairBarrier0 + qd;
         if (nt > 0) {
@@ -539,17 +557,24 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
             const bool resc = mx2 > m_run + kRescaleSlack;
             const float m_new = resc ? mx2 : m_run;
             const float alpha = resc ? ex2(m_run - m_new) : 1.0f;
-            if (i > 0) {
-                // PV of the previous tile must be done before P or O is touched
-                // (on a timeout this tile is skipped; the pair leaves the loop
-                // together at the next exchange)
-                if (!warp_wait(pv_done, static_cast<uint32_t>(i - 1) & 1u, abort)) {
+            // P buffer i & 1 was last read by PV(i - 2); O must be stable (PV(i - 1)
+            // done) only when it is rescaled.  On a timeout this tile is
+            // skipped; the pair leaves the loop together at the next exchange.
+            if (i > 1 && !warp_wait(&pv_done[i & 1], (static_cast<uint32_t>(i >> 1) & 1u) ^ 1u, abort)) {
+                attn_timeout(a.status, abort);
+                ok = false;
+                continue;
+            }
+            tc_fence_after();
+            const bool any_resc = __any_sync(0xFFFFFFFFu, resc);
+            if (i > 0 && any_resc) {
+                if (!warp_wait(&pv_done[(i - 1) & 1], static_cast<uint32_t>((i - 1) >> 1) & 1u, abort)) {
                     attn_timeout(a.status, abort);
                     ok = false;
                     continue;
                 }
                 tc_fence_after();
-                if (__any_sync(0xFFFFFFFFu, resc)) {
+                {
 #pragma unroll
                     for (int c0 = 0; c0 < 64; c0 += 16) {
                         float o[16];
@@ -563,29 +588,28 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
             }
             l *= alpha;
             m_run = m_new;
-            // P = 2^(s * scale * log2 e - m) as bf16 into this warpgroup's half
-            // of the swizzled K-major P tile; masked keys hold -inf and give 0
-            // (so does every key of a row that has seen no visible key: m = -inf)
+            // P = 2^(s * scale * log2 e - m) as bf16 pairs into TMEM P buffer
+            // i & 1 (lane = row, keys 64 wg .. 64 wg + 63 in 32 columns); masked
+            // keys hold -inf and give 0 (so does every key of a row that has
+            // seen no visible key: m = -inf)
             const float nm = m_run == -INFINITY ? 0.0f : -m_run;
             float lsum = 0.0f;
+            uint32_t pk[32];
 #pragma unroll
-            for (int c0 = 0; c0 < 64; c0 += 8) {
-                float p[8];
-#pragma unroll
-                for (int e = 0; e < 8; e++) {
-                    p[e] = ex2(fmaf(sv[c0 + e], a.sl2, nm));
-                    lsum += p[e];
-                }
-                const uint4 v = make_uint4(pack_bf16(p[0], p[1]), pack_bf16(p[2], p[3]), pack_bf16(p[4], p[5]),
-                                           pack_bf16(p[6], p[7]));
-                *reinterpret_cast<uint4*>(prow + (((static_cast<uint32_t>(c0 >> 3)) ^ swz) << 4)) = v;
+            for (int c = 0; c < 64; c += 2) {
+                const float p0 = ex2(fmaf(sv[c], a.sl2, nm));
+                const float p1 = ex2(fmaf(sv[c + 1], a.sl2, nm));
+                lsum += p0 + p1;
+                pk[c >> 1] = pack_bf16(p0, p1);
             }
+            tmem_st32(tl + kPCol + (i & 1) * (kKeys / 2) + wg * 32, pk);
+            tmem_wait_st();
             l += lsum;
-            fence_async_smem();
+            tc_fence_before();
             mbar_arrive(p_full);
         }
         if (ok && nt > 0) {
-            if (!warp_wait(pv_done, static_cast<uint32_t>(nt - 1) & 1u, abort)) {
+            if (!warp_wait(&pv_done[(nt - 1) & 1], static_cast<uint32_t>((nt - 1) >> 1) & 1u, abort)) {
                 attn_timeout(a.status, abort);
                 ok = false;
             }
@@ -623,14 +647,14 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
     } else {
         // Split key range.  Columns are owned in groups of 4: CTA j merges
         // [c_lo(j), c_hi(j)).  After a cluster barrier (every CTA is past its
-        // main loop, so the K ring and P tile are free), every CTA p pushes,
+        // main loop, so the K and V rings are free), every CTA p pushes,
         // with 16-byte stores into the peers' shared memory, its (m, l) row
         // to every peer and its unnormalised O row slices to their owners
         // (row-major, row stride padded to an odd number of 16-byte units:
         // conflict-free); after a second barrier CTA j merges locally, in
         // rank order: O = sum_p 2^(m_p - M) O_p / sum_p 2^(m_p - M) l_p.
         float* rbuf = reinterpret_cast<float*>(sK);     // [p][128 rows][stride]
-        float2* rml = reinterpret_cast<float2*>(sP);    // [p][128 rows]
+        float2* rml = reinterpret_cast<float2*>(sV);    // [p][128 rows]
         __syncwarp();
         cluster_sync_all();
         if (warp >= 2) {
