@@ -59,11 +59,13 @@ constexpr int kVStages = 3;
 constexpr int kHalf = kRows * 64 * 2;     // 16 KB: 128 rows x 64 bf16, one 128-byte swizzle column
 constexpr int kTileBytes = 2 * kHalf;     // 32 KB: 128 rows x dh bf16
 constexpr int kMaxSplits = 8;                // cluster size limit (portable)
-constexpr int kTmemCols = 512;            // S0 [0,128), S1 [128,256), O [256,384), P0 [384,448), P1 [448,512)
-constexpr int kOCol = 256;
-constexpr int kPCol = 384;                // P tiles: 128 keys as 64 columns of bf16 pairs
+constexpr int kTmemCols = 512;            // S [0,128), O [128,256), P0 [256,320), P1 [320,384), Q [384,448)
+constexpr int kSCol = 0;
+constexpr int kOCol = 128;
+constexpr int kPCol = 256;                // P tiles: 128 keys as 64 columns of bf16 pairs
+constexpr int kQCol = 384;                // rotated query tile: dh = 128 as 64 columns of bf16 pairs
 constexpr float kRescaleSlack = 8.0f;     // log2 units: P <= 2^8 between rescales
-constexpr int kNumBars = 1 + 2 * kKStages + 2 * kVStages + 4 + 5;
+constexpr int kNumBars = 1 + 2 * kKStages + 2 * kVStages + 2 + 5;
 constexpr int kSmemUsed = kTileBytes * (1 + kKStages + kVStages) + kNumBars * 8 + 4 * 4 + 2 * 128 * 4 + 8 * 4;  // Q, K/V rings, barriers, exchange
 constexpr int kAttnSmem = kSmemUsed + 1024;  // + alignment slack of the 1024-byte swizzle atoms
 
@@ -136,6 +138,16 @@ __device__ __forceinline__ void tc_mma_bf16_ts(uint32_t tmem_d, uint32_t tmem_a,
         : "memory");
 }
 
+// 16 consecutive 32-bit TMEM columns of this thread's lane from registers.
+__device__ __forceinline__ void tmem_st16u(uint32_t taddr, const uint32_t (&v)[16]) {
+    asm volatile(
+        "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16};" ::"r"(
+            taddr),
+        "r"(v[0]), "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7]), "r"(v[8]), "r"(v[9]),
+        "r"(v[10]), "r"(v[11]), "r"(v[12]), "r"(v[13]), "r"(v[14]), "r"(v[15])
+        : "memory");
+}
+
 // 32 consecutive 32-bit TMEM columns of this thread's lane from registers.
 __device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t (&v)[32]) {
     asm volatile(
@@ -147,9 +159,6 @@ __device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t (&v)[32
         "r"(v[28]), "r"(v[29]), "r"(v[30]), "r"(v[31])
         : "memory");
 }
-
-// Generic-proxy shared-memory writes become visible to the tensor core.
-__device__ __forceinline__ void fence_async_smem() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
 
 __device__ __forceinline__ void attn_timeout(int* status, volatile int* abort) {
     *abort = 1;
@@ -282,9 +291,9 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
     uint64_t* k_empty = k_full + kKStages;            // [kKStages] S of the stage's tile done
     uint64_t* v_full = k_empty + kKStages;            // [kVStages]
     uint64_t* v_empty = v_full + kVStages;            // [kVStages] PV of the stage's tile done
-    uint64_t* s_full = v_empty + kVStages;            // [2]
-    uint64_t* s_empty = s_full + 2;                   // [2]
-    uint64_t* p_full = s_empty + 2;
+    uint64_t* s_full = v_empty + kVStages;
+    uint64_t* s_empty = s_full + 1;                   // softmax has S in registers
+    uint64_t* p_full = s_empty + 1;
     uint64_t* pv_done = p_full + 1;                   // [2] PV of a tile using P buffer b done
     uint64_t* tdown = pv_done + 2;
     uint64_t* q_ready = tdown + 1;                    // queries rotated in place
@@ -311,10 +320,8 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
             mbar_init(&v_full[i], 1);
             mbar_init(&v_empty[i], 1);
         }
-        for (int i = 0; i < 2; i++) {
-            mbar_init(&s_full[i], 1);
-            mbar_init(&s_empty[i], kSoftThreads);
-        }
+        mbar_init(s_full, 1);
+        mbar_init(s_empty, kSoftThreads);
         mbar_init(p_full, kSoftThreads);
         mbar_init(&pv_done[0], 1);
         mbar_init(&pv_done[1], 1);
@@ -407,35 +414,39 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
         }
     } else if (warp == 1) {
         // ---------------------------------------------------------- MMA issuer
-        // order: S(0), S(1), then per tile i: PV(i) as soon as P(i) is ready,
-        // then S(i+2) into the S buffer softmax(i) has released
+        // Q (rotated) and P are tensor-memory operands, K and V come from the
+        // shared-memory rings.  Order: S(0); then per tile i: S(i+1) once
+        // softmax(i) holds S(i) in registers (it runs during softmax(i)),
+        // PV(i) once P(i) is written (P is double-buffered).
         if (lane == 0 && nt > 0) {
             constexpr uint32_t idesc_s = idesc_bf16_f32(kRows, kKeys);
             constexpr uint32_t idesc_pv = idesc_bf16_f32(kRows, kDh) | (1u << 16);  // B (= V) MN-major
-            const uint32_t q_addr = smem_u32(sQ);
             bool mok = mbar_wait(q_ready, 0, abort);
             auto issue_s = [&](int i) -> bool {
-                const int sb = i & 1, st = i % kKStages;
-                // S buffer sb was last read by softmax(i - 2)
+                const int st = i % kKStages;
+                // the S columns were last read by softmax(i - 1)
                 if (!mbar_wait(&k_full[st], static_cast<uint32_t>(i / kKStages) & 1u, abort) ||
-                    !mbar_wait(&s_empty[sb], (static_cast<uint32_t>(i >> 1) & 1u) ^ 1u, abort))
+                    (i > 0 && !mbar_wait(s_empty, static_cast<uint32_t>(i - 1) & 1u, abort)))
                     return false;
                 tc_fence_after();
                 const uint32_t k_addr = smem_u32(sK + st * kTileBytes);
 #pragma unroll
                 for (int kk = 0; kk < kDh / 16; kk++) {
                     const uint32_t o = (kk >> 2) * kHalf + (kk & 3) * 32;
-                    tc_mma_bf16(tmem + sb * kKeys, sdesc_sw128(q_addr + o), sdesc_sw128(k_addr + o), idesc_s,
-                                kk > 0 ? 1u : 0u);
+                    tc_mma_bf16_ts(tmem + kSCol, tmem + kQCol + kk * 8, sdesc_sw128(k_addr + o), idesc_s,
+                                   kk > 0 ? 1u : 0u);
                 }
-                tc_commit(&s_full[sb]);
+                tc_commit(s_full);
                 tc_commit(&k_empty[st]);
                 return true;
             };
             if (mok) tc_fence_after();
             if (mok) mok = issue_s(0);
-            if (mok && nt > 1) mok = issue_s(1);
             for (int i = 0; i < nt && mok; i++) {
+                if (i + 1 < nt && !issue_s(i + 1)) {
+                    mok = false;
+                    break;
+                }
                 const int st = i % kVStages;
                 if (!mbar_wait(p_full, static_cast<uint32_t>(i) & 1u, abort) ||
                     !mbar_wait(&v_full[st], static_cast<uint32_t>(i / kVStages) & 1u, abort)) {
@@ -451,7 +462,6 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
                                    (i > 0 || kk > 0) ? 1u : 0u);
                 tc_commit(&v_empty[st]);
                 tc_commit(&pv_done[i & 1]);
-                if (i + 2 < nt) mok = issue_s(i + 2);
             }
             if (!mok) {
                 attn_timeout(a.status, abort);
@@ -471,16 +481,21 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
             if (!warp_wait(q_full, 0, abort)) {
                 attn_timeout(a.status, abort);
                 ok = false;
-            } else if (b < a.B) {
+            }
+            // rotated elements t (first half) and t + 64 (second half) of this
+            // warpgroup's t in [32 wg, 32 wg + 32), as bf16 pairs for the TMEM
+            // columns kQCol + t / 2 and kQCol + 32 + t / 2 (zeros past row B)
+            uint32_t q1[16], q2[16];
+            if (ok && b < a.B) {
                 const float4* cs = reinterpret_cast<const float4*>(a.cs + (static_cast<size_t>(s) * a.B + b) * (kDh / 2));
 #pragma unroll
                 for (int cc = 0; cc < 4; cc++) {
                     const int c = wg * 4 + cc;
-                    uint8_t* p1 = sQ + r * 128 + ((static_cast<uint32_t>(c) ^ swz) << 4);
-                    uint4 x1 = *reinterpret_cast<const uint4*>(p1);
-                    uint4 x2 = *reinterpret_cast<const uint4*>(p1 + kHalf);
-                    uint32_t* u1 = reinterpret_cast<uint32_t*>(&x1);
-                    uint32_t* u2 = reinterpret_cast<uint32_t*>(&x2);
+                    const uint8_t* p1 = sQ + r * 128 + ((static_cast<uint32_t>(c) ^ swz) << 4);
+                    const uint4 x1 = *reinterpret_cast<const uint4*>(p1);
+                    const uint4 x2 = *reinterpret_cast<const uint4*>(p1 + kHalf);
+                    const uint32_t* u1 = reinterpret_cast<const uint32_t*>(&x1);
+                    const uint32_t* u2 = reinterpret_cast<const uint32_t*>(&x2);
 #pragma unroll
                     for (int e = 0; e < 4; e++) {
                         const float4 f = __ldg(cs + c * 4 + e);  // (cos, sin) of pairs 8c+2e, 8c+2e+1
@@ -488,19 +503,22 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
                         const __nv_bfloat162 h2 = *reinterpret_cast<const __nv_bfloat162*>(&u2[e]);
                         const float a0 = __low2float(h1), a1 = __high2float(h1);
                         const float b0 = __low2float(h2), b1 = __high2float(h2);
-                        u1[e] = pack_bf16(a0 * f.x - b0 * f.y, a1 * f.z - b1 * f.w);
-                        u2[e] = pack_bf16(b0 * f.x + a0 * f.y, b1 * f.z + a1 * f.w);
+                        q1[cc * 4 + e] = pack_bf16(a0 * f.x - b0 * f.y, a1 * f.z - b1 * f.w);
+                        q2[cc * 4 + e] = pack_bf16(b0 * f.x + a0 * f.y, b1 * f.z + a1 * f.w);
                     }
-                    *reinterpret_cast<uint4*>(p1) = x1;
-                    *reinterpret_cast<uint4*>(p1 + kHalf) = x2;
                 }
+            } else {
+#pragma unroll
+                for (int k = 0; k < 16; k++) q1[k] = q2[k] = 0u;
             }
-            fence_async_smem();
+            tmem_st16u(tl + kQCol + wg * 16, q1);
+            tmem_st16u(tl + kQCol + 32 + wg * 16, q2);
+            tmem_wait_st();
+            tc_fence_before();
             mbar_arrive(q_ready);
         }
         for (int i = 0; i < nt; i++) {
             const int j = j0 + i;
-            const int sb = i & 1;
             // visible keys of this row among this warpgroup's 64 keys of the tile
             uint64_t w = 0ull;
             if (row_ok) {
@@ -523,7 +541,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
             // Both warps of the lane quarter reach both pair barriers of every
             // iteration and leave the loop at the same point: a failed wait is
             // exchanged with the row max and acted on after the barriers.
-            if (ok && !warp_wait(&s_full[sb], static_cast<uint32_t>(i >> 1) & 1u, abort)) {
+            if (ok && !warp_wait(s_full, static_cast<uint32_t>(i) & 1u, abort)) {
                 attn_timeout(a.status, abort);
                 ok = false;
             }
@@ -531,10 +549,10 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
             float mx = -INFINITY;
             if (ok) {
                 tc_fence_after();
-                tmem_ld64(tl + sb * kKeys + cb, sv);
+                tmem_ld64(tl + kSCol + cb, sv);
                 // S is in registers: the buffer is free for S(i + 2)
                 tc_fence_before();
-                mbar_arrive(&s_empty[sb]);
+                mbar_arrive(s_empty);
                 if (full) {
 #pragma unroll
                     for (int c = 0; c < 64; c += 2) mx = fmaxf(mx, fmaxf(sv[c], sv[c + 1]));
