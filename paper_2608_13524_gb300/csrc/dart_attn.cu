@@ -58,7 +58,7 @@ constexpr int kKStages = 3;                  // K ring: the S MMA needs K two ti
 constexpr int kVStages = 3;
 constexpr int kHalf = kRows * 64 * 2;     // 16 KB: 128 rows x 64 bf16, one 128-byte swizzle column
 constexpr int kTileBytes = 2 * kHalf;     // 32 KB: 128 rows x dh bf16
-constexpr int kMaxSplits = 8;                // cluster size limit (portable)
+constexpr int kMaxSplits = 4;                // cluster size: clusters of 4 fit a GPC in one wave beside each other
 constexpr int kTmemCols = 512;            // S [0,128), O [128,256), P0 [256,320), P1 [320,384), Q [384,448)
 constexpr int kSCol = 0;
 constexpr int kOCol = 128;
