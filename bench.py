@@ -231,7 +231,7 @@ def run_reference(args, cfg):
 
 
 # ------------------------------------------------------------------ tree attention
-# (the verification consumer of the emitted tree, Sec. 2.2: one attention
+# (the verification consumer of the emitted tree, Sec. 3.3: one attention
 # layer over [context ; tree] with the ancestor mask and the tree positions)
 
 ATTN_METRIC = "tree-attention verification layer: tree tokens/s (µs per call)"

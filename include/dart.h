@@ -10,9 +10,9 @@
  *     by the Eq. 5 path score s_beta = sum_i log q~_i(u_i) + beta*d, the
  *     global top-W children form S_d, and their correction states are
  *     updated;
- *   - Sec. 3.3 / Lemma 1: the complete supertree S is pruned to the budget B
+ *   - Sec. 4.3 / Lemma 1: the complete supertree S is pruned to the budget B
  *     with one global top-B (equal to best-first heap selection for
- *     beta <= 0), and flattened for tree-attention verification (Sec. 2.3).
+ *     beta <= 0), and flattened for tree-attention verification (Sec. 3.3).
  *
  * Correction head (the paper leaves its form open; this is the fallback head):
  *   h_c = RMSNorm(h_p + W_o . SiLU(W_i . [h_p ; E[t_c]]))   (no gain)
@@ -21,7 +21,7 @@
  *   log q~[v] = min(z[v] - logsumexp_v z, 0)
  * The LM head is tied to the embedding table E.  The candidate set is the
  * whole vocabulary ("Full" in Appendix D) when cand_k = 0, or, as in
- * Algorithm 1 with K = cand_k (the paper's default K = 64, Sec. 4.1), the
+ * Algorithm 1 with K = cand_k (the paper's default K = 64, Sec. 5.1), the
  * set C_d = TopK(L_d^base, K) of the K largest drafter logits of position d
  * (ties: token asc), shared by every node of the depth; then v runs over
  * C_d only and q~ is renormalised over C_d (logsumexp over C_d).  Each node

@@ -2,10 +2,10 @@
  * dart_verify.h -- tree-attention verification consumer of the emitted draft
  * tree (GB300, sm_103a).
  *
- * Sec. 2.2 of the paper ("Tree Verification and DDTree") flattens the draft
+ * Sec. 3.3 of the paper ("Tree Verification and DDTree") flattens the draft
  * tree and verifies every branch in ONE target forward pass: each tree node
  * attends to the verified context and to the tokens on its own root-to-node
- * path, and nothing else.  Sec. 3.3 (after Lemma 1) hands the pruned tree to
+ * path, and nothing else.  Sec. 4.3 (after Lemma 1) hands the pruned tree to
  * exactly that pass.  The target model is not available here, so this
  * library provides the part of the pass that the tree changes -- one
  * attention layer over [context ; tree] with the tree mask and the tree

@@ -14,10 +14,10 @@
  *   - Algorithm 1 (depth-wise fixed-width supertree construction) with a
  *     per-node top-k, over either the full vocabulary (Appendix D, "Full")
  *     or the candidate set C_d = TopK(L_d^base, K) of Algorithm 1 (cand_k =
- *     K > 0; the paper's default is K = 64, Sec. 4.1);
+ *     K > 0; the paper's default is K = 64, Sec. 5.1);
  *   - the path score of Eq. 5, s_beta(u_{1:d}) = sum_i log q~_i(u_i) + beta d;
  *   - deferred pruning, T = TopB_{u in S} s_beta(u) (Algorithm 1, final step);
- *   - the best-first heap of Sec. 3.3 / Lemma 1 (used to check that the top-B
+ *   - the best-first heap of Sec. 4.3 / Lemma 1 (used to check that the top-B
  *     selection equals heap selection when beta <= 0);
  *   - flattening into the verification tree with an ancestor mask
  *     (Sec. 3.3, tree verification).

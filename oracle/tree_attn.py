@@ -4,7 +4,7 @@ TEST INFRASTRUCTURE ONLY: the tests, ``__graft_entry__.smoke()`` and the
 benchmark's CPU-baseline leg may use this module; the product path never
 imports it.  It shares no code with the CUDA path.
 
-What it computes (Sec. 2.2 of the paper, "Tree Verification and DDTree"):
+What it computes (Sec. 3.3 of the paper, "Tree Verification and DDTree"):
 the draft tree is flattened and verified in one target forward pass in
 which every tree node attends to the verified context and to the tokens on
 its own root-to-node path.  The target model is not available, so the

@@ -1,6 +1,6 @@
-// Tree-attention verification consumer of the emitted draft tree (Sec. 2.2,
+// Tree-attention verification consumer of the emitted draft tree (Sec. 3.3,
 // "Tree Verification and DDTree": every flattened tree node attends to the
-// verified context and to the tokens on its root-to-node path; Sec. 3.3
+// verified context and to the tokens on its root-to-node path; Sec. 4.3
 // hands the pruned tree to that single forward pass).  Contract:
 // include/dart_verify.h.
 //

@@ -6,7 +6,7 @@
 //       log q~ = min(z - lse, 0); the last block of each sequence (atomic
 //       ticket, no waiting) then scores the candidates with Eq. 5 and keeps
 //       the top-W as S_d.
-//   prune_emit    (Algorithm 1 final step + Lemma 1, Sec. 2.3 flattening):
+//   prune_emit    (Algorithm 1 final step + Lemma 1, Sec. 3.3 flattening):
 //       one block per sequence: global top-B by (score desc, node id asc),
 //       compaction in id order, parent remap, depths, position ids and the
 //       ancestor bit mask.

@@ -97,7 +97,7 @@ def all_path_scores(cfg, Wi, Wo, E, Dlog_seq, h0_seq, max_len):
 
 
 def ddtree_topB(logq_rows, B):
-    """DDTree best-first over path-independent marginals (Sec. 2.3): pop the
+    """DDTree best-first over path-independent marginals (Sec. 3.3): pop the
     best prefix, push its next sibling and its first child.  Marginal rows are
     log-probabilities; the prefix score is their sum (beta folded in by the
     caller).  Returns the popped token paths in pop order."""

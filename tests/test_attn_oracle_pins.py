@@ -1,5 +1,5 @@
 """Pins of the tree-attention oracle (oracle/tree_attn.py) to facts that do
-not come from the oracle itself (Sec. 2.2: a tree node attends to the
+not come from the oracle itself (Sec. 3.3: a tree node attends to the
 verified context and to its own root-to-node path).
 
 * A branch of the tree is an ordinary causal sequence: for every node, the

@@ -153,7 +153,7 @@ def test_bruteforce_beam_levels(V, W, k):
 # ---------------------------------------------------------- special cases
 
 def test_zero_E_is_ddtree_optimal_tree():
-    """E = 0 makes q~ path independent (Sec. 2.3): scores reduce to
+    """E = 0 makes q~ path independent (Sec. 3.3): scores reduce to
     sum_i log_softmax(Dlog_i)[u_i] + beta d, and with W, k >= B the pruned
     tree equals DDTree's best-first top-B prefixes."""
     cfg = tiny(V=40, d=16, L=5, W=12, k=12, B=12, beta=-0.2)

@@ -97,7 +97,7 @@ def sweep_configs():
 
 
 # The same shapes and inputs with Algorithm 1's candidate restriction at the
-# paper's default K = 64 (Sec. 4.1).
+# paper's default K = 64 (Sec. 5.1).
 RESTRICTED = [Q8B.replace(name="qwen3-8b-k64", cand_k=64), Q4B.replace(name="qwen3-4b-k64", cand_k=64),
               BATCHED.replace(name="batched-k64", cand_k=64)]
 
@@ -202,7 +202,7 @@ def make_inputs(cfg: Config, zero_E: bool = False, rank: int = 0):
 
 
 # --------------------------------------------------------------------------
-# tree-attention verification inputs (Sec. 2.2: one target forward pass over
+# tree-attention verification inputs (Sec. 3.3: one target forward pass over
 # the flattened tree).  The target model is not available: one attention
 # layer with Qwen3-4B/8B head geometry (32 query heads, 8 key/value heads,
 # head dim 128, RoPE base 1e6) on N(0,1) queries, keys and values, and a
