@@ -437,7 +437,7 @@ constexpr float kRefSlack = 30.0f;  // exp(30) ~ 1e13: sums stay far from fp32 o
 struct EpiSmem {
     uint64_t* list;   // [NG][k]   sorted desc, 0 = empty
     uint64_t* cand;   // [NG][cap]
-    uint64_t* gcache; // [NG]  last seen cross-CTA bound (see epi_merge)
+    uint64_t* gcache; // [NG]  filter threshold: max(own k-th key, last seen cross-CTA bound) (see epi_merge)
     int* cnt;         // [NG]  candidates offered this round (may exceed cap)
     int* more;        // [2]   "a candidate found no free slot" flags of alternate merge rounds
     float* mref;      // [4][NG]  per-warp reference max
@@ -515,17 +515,15 @@ __device__ __forceinline__ uint32_t epi_offer(const EpiSmem& e, int c0, const fl
     return pend;
 }
 
-// The subset of `pend` whose keys still beat their node's (raised) threshold.
+// The subset of `pend` whose keys still beat their node's (raised)
+// threshold (a threshold read before its update is lower: a superset).
 __device__ __forceinline__ uint32_t epi_still_pass(const EpiSmem& e, int k, int c0, const float (&z)[16],
                                                    uint32_t pend, uint32_t row) {
+    (void)k;
     uint32_t keep = 0;
 #pragma unroll
-    for (int j = 0; j < 16; j++) {
-        if ((pend >> j) & 1u) {
-            const uint64_t l = e.list[(c0 + j) * k + k - 1], g = e.gcache[c0 + j];
-            if (make_key(z[j], row) > (l > g ? l : g)) keep |= 1u << j;
-        }
-    }
+    for (int j = 0; j < 16; j++)
+        if (((pend >> j) & 1u) && make_key(z[j], row) > e.gcache[c0 + j]) keep |= 1u << j;
     return keep;
 }
 
@@ -546,9 +544,12 @@ __device__ __forceinline__ uint32_t epi_chunk(const EpiSmem& e, int NG, int k, i
         else if (z[j] == 0.0f) z[j] = 0.0f;  // -0 -> +0
     }
     float* mr = e.mref + ew * NG + c0;
+    float m[16];
+#pragma unroll
+    for (int j = 0; j < 16; j++) m[j] = mr[j];
     bool slow = false;
 #pragma unroll
-    for (int j = 0; j < 16; j++) slow |= z[j] > mr[j] + kRefSlack;
+    for (int j = 0; j < 16; j++) slow |= z[j] > m[j] + kRefSlack;
     if (__any_sync(kFull, slow)) {
         const float mx = bfly16<true>(z, lane);
         const int me = lane >> 1;
@@ -558,17 +559,17 @@ __device__ __forceinline__ uint32_t epi_chunk(const EpiSmem& e, int NG, int k, i
         __syncwarp();
         if ((lane & 1) == 0) mr[me] = nm;
         __syncwarp();
+#pragma unroll
+        for (int j = 0; j < 16; j++) m[j] = mr[j];
     }
     float p[16];
 #pragma unroll
-    for (int j = 0; j < 16; j++) p[j] = z[j] != -INFINITY ? __expf(z[j] - mr[j]) : 0.0f;
+    for (int j = 0; j < 16; j++) p[j] = z[j] != -INFINITY ? __expf(z[j] - m[j]) : 0.0f;
     ssum += bfly16<false>(p, lane);
     uint32_t passmask = 0;  // bit j: this row's key beats node j's current threshold
 #pragma unroll
-    for (int j = 0; j < 16; j++) {
-        const uint64_t l = e.list[(c0 + j) * k + k - 1], g = e.gcache[c0 + j];
-        if (ok[j] && make_key(z[j], row) > (l > g ? l : g)) passmask |= 1u << j;
-    }
+    for (int j = 0; j < 16; j++)
+        if (ok[j] && make_key(z[j], row) > e.gcache[c0 + j]) passmask |= 1u << j;
     return epi_offer(e, c0, z, passmask, row, lane);
 }
 
@@ -694,7 +695,12 @@ __device__ __forceinline__ void epi_merge(const EpiSmem& e, int NG, int k, int w
         }
     }
     named_bar_sync(kEpiBarrier, nthr);
-    if (etid < NG) e.gcache[etid] = g;  // read by the next tile's filter, after its first barrier
+    // the filter threshold of the next tile (read after its first barrier):
+    // the larger of the node's own k-th key and the cross-CTA bound
+    if (etid < NG) {
+        const uint64_t l = e.list[etid * k + k - 1];
+        e.gcache[etid] = l > g ? l : g;
+    }
 }
 
 // Records this warp's (reference, sum) of chunk cc's nodes.
