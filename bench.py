@@ -88,12 +88,22 @@ def measured_peak():
         return FALLBACK_HBM_GBS, "fallback"
 
 
-def kernel_source_sha():
+def code_sha(files):
+    """Hash of CUDA sources with comments and blank space removed: a capture
+    stays valid across comment-only edits and is void after any code change."""
+    import re
     h = hashlib.sha256()
-    for f in ("dart_tc.cu", "dart_device.cuh"):
-        with open(os.path.join(ROOT, "paper_2608_13524_gb300", "csrc", f), "rb") as fh:
-            h.update(fh.read())
+    for f in files:
+        with open(os.path.join(ROOT, "paper_2608_13524_gb300", "csrc", f)) as fh:
+            src = fh.read()
+        src = re.sub(r"/\*.*?\*/", " ", src, flags=re.S)
+        src = re.sub(r"//[^\n]*", " ", src)
+        h.update(" ".join(src.split()).encode())
     return h.hexdigest()[:16]
+
+
+def kernel_source_sha():
+    return code_sha(("dart_tc.cu", "dart_device.cuh"))
 
 
 def recorded_traffic(workload):
@@ -248,11 +258,7 @@ def measured_tflops():
 
 
 def attn_source_sha():
-    h = hashlib.sha256()
-    for f in ("dart_attn.cu", "dart_device.cuh"):
-        with open(os.path.join(ROOT, "paper_2608_13524_gb300", "csrc", f), "rb") as fh:
-            h.update(fh.read())
-    return h.hexdigest()[:16]
+    return code_sha(("dart_attn.cu", "dart_device.cuh"))
 
 
 def attn_recorded_traffic(workload):

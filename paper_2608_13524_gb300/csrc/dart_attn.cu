@@ -9,28 +9,32 @@
 //                      the rotated tree keys (rotate-half RoPE in fp32,
 //                      rounded to bf16) in the workspace;
 //   tree_attn_kernel   flash attention on the tensor cores (tcgen05, TMEM
-//                      accumulators, TMA-staged K/V).  A CTA owns 128 query
-//                      rows = 128/G tree rows x the G query heads sharing one
-//                      kv head, so each K/V tile feeds all G heads; the
-//                      softmax warps rotate the query tile in shared memory
-//                      before the first MMA.  Its key
-//                      tiles are the context tiles (all visible, ragged tail
-//                      masked) followed by the tree tiles up to its last row
-//                      (ancestors precede their descendants, so later tiles
-//                      are invisible), masked by the ancestor bitmask.  When
-//                      there are fewer (sequence, kv head, query tile) blocks
-//                      than SMs, the key list is split over a thread-block
-//                      cluster whose CTAs merge their partial (max, sum, O)
-//                      over distributed shared memory, in rank order;
+//                      operands and accumulators, TMA-staged K/V).  A CTA
+//                      owns 128 query rows = 128/G tree rows x the G query
+//                      heads sharing one kv head, so each K/V tile feeds all
+//                      G heads.  Its key tiles are the context tiles (all
+//                      visible, ragged tail masked) followed by the tree
+//                      tiles up to its last row (ancestors precede their
+//                      descendants, so later tiles are invisible), masked by
+//                      the ancestor bitmask.  When there are fewer (sequence,
+//                      kv head, query tile) blocks than SMs, the key list is
+//                      split over a thread-block cluster of up to 4 CTAs
+//                      that merge their partial (max, sum, O) over
+//                      distributed shared memory, in rank order;
 // and dart_ancestor_mask's own kernel, one block per sequence.
-// Warp roles of tree_attn_kernel (192 threads): warp 0 TMA producer, warp 1
-// TMEM allocator + single-thread MMA issuer, warps 2-5 softmax, thread =
-// query row = TMEM lane.  TMEM: two S buffers (128 columns each, so the
-// S = Q K^T of tile i+1 overlaps the softmax of tile i) and the O accumulator
-// (128 columns).  O stays in TMEM for the whole key range; a row's running
-// max is raised (and O, l rescaled through tcgen05.ld/st) only when a tile
-// exceeds it by more than 2^8, so P = exp2(s - m) <= 256 and the rescale is
-// rare.  Every wait is bounded (status bit on timeout, then drain and exit).
+// tree_attn_kernel, 320 threads: warp 0 TMA producer (K ring 3 stages, V ring
+// 3 stages), warp 1 TMEM allocator + single-thread MMA issuer, warps 2-9 two
+// softmax warpgroups; thread = query row = TMEM lane, warpgroup wg owns key
+// columns and O columns [64 wg, 64 wg + 64) of the rows, the pair of warps of
+// a lane quarter exchanging row max and row sum through shared memory.
+// TMEM (512 columns): S [0,128), O [128,256), P double buffer [256,384), the
+// rotated query tile [384,448).  S = Q K^T and O += P V both take A from
+// TMEM (K K-major, V MN-major from shared memory); the softmax reads S into
+// registers at once, which frees it for the next tile's S while it works.
+// O stays in TMEM for the whole key range; a row's running max is raised
+// (and O, l rescaled through tcgen05.ld/st) only when a tile exceeds it by
+// more than 2^8, so P = exp2(s - m) <= 256 and the rescale is rare.  Every
+// wait is bounded (status bit on timeout, then drain and exit).
 #include <cuda.h>
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
