@@ -782,6 +782,10 @@ __global__ void __launch_bounds__(kMaskThreads) ancestor_mask_kernel(const int32
 
 struct Plan {
     int G, qpt, nqt, blocks, splits, mw, nct;
+};
+
+// Workspace: rotated tree keys, then the (cos, sin) table (no device query).
+struct WsLayout {
     size_t off_kr, off_cs, total;
 };
 
@@ -802,12 +806,6 @@ bool valid_cfg(const dart_attn_config* c) {
     return true;
 }
 
-int sm_count() {
-    int dev = 0, n = 148;
-    if (cudaGetDevice(&dev) == cudaSuccess) cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
-    return n > 0 ? n : 148;
-}
-
 // Splits of the key list (= cluster size): as many as keep every CTA in one
 // wave (1 CTA per SM) with at least two key tiles per split.
 int pick_splits(int blocks, int max_tiles, int nsm) {
@@ -825,12 +823,41 @@ Plan make_plan(const dart_attn_config* c, int nsm) {
     p.mw = (c->B + 63) / 64;
     p.nct = (c->C + kKeys - 1) / kKeys;
     p.splits = pick_splits(p.blocks, p.nct + (c->B + kKeys - 1) / kKeys, nsm);
+    return p;
+}
+
+WsLayout ws_layout(const dart_attn_config* c) {
+    WsLayout w;
     const size_t kr = static_cast<size_t>(c->nseq) * c->B * c->Hkv * kDh * 2;
     const size_t cs = static_cast<size_t>(c->nseq) * c->B * (kDh / 2) * 8;
-    p.off_kr = 0;
-    p.off_cs = align256(p.off_kr + kr);
-    p.total = align256(p.off_cs + cs);
-    return p;
+    w.off_kr = 0;
+    w.off_cs = align256(w.off_kr + kr);
+    w.total = align256(w.off_cs + cs);
+    return w;
+}
+
+// Compute capability, shared-memory opt-in and SM count of a device, queried
+// once per device.
+struct DevInfo {
+    int major, minor, optin, nsm;
+};
+bool dev_info(int dev, DevInfo* out) {
+    constexpr int kMaxDev = 64;
+    static DevInfo info[kMaxDev];
+    static std::atomic<int> ready[kMaxDev];
+    if (dev < 0 || dev >= kMaxDev) return false;
+    if (ready[dev].load(std::memory_order_acquire) == 0) {
+        DevInfo d{};
+        if (cudaDeviceGetAttribute(&d.major, cudaDevAttrComputeCapabilityMajor, dev) != cudaSuccess ||
+            cudaDeviceGetAttribute(&d.minor, cudaDevAttrComputeCapabilityMinor, dev) != cudaSuccess ||
+            cudaDeviceGetAttribute(&d.optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) != cudaSuccess ||
+            cudaDeviceGetAttribute(&d.nsm, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+            return false;
+        info[dev] = d;  // every thread that gets here writes the same values
+        ready[dev].store(1, std::memory_order_release);
+    }
+    *out = info[dev];
+    return true;
 }
 
 // Queries [nseq][B][Hq][dh] bf16 with a (64, G heads, qpt rows, 1) box: the
@@ -896,19 +923,18 @@ int enqueue_tree_attention(const dart_attn_config* cfg, const void* q, const voi
         return DART_ERR_INVALID;
     if (c.C > 0 && (!al16(k_ctx) || !al16(v_ctx))) return DART_ERR_INVALID;
     if (status && !al16(status)) return DART_ERR_INVALID;
-    int dev = 0, major = 0, minor = 0, optin = 0, nsm = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess) return DART_ERR_CUDA;
-    cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev);
-    cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev);
-    cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
-    cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev);
-    if (major != 10 || minor != 3 || optin < kAttnSmem) return DART_ERR_UNSUPPORTED;
-    const Plan p = make_plan(cfg, nsm > 0 ? nsm : 148);
-    if (workspace_bytes < p.total) return DART_ERR_INVALID;
+    const WsLayout wl = ws_layout(cfg);
+    if (workspace_bytes < wl.total) return DART_ERR_INVALID;
+    int dev = 0;
+    DevInfo di;
+    if (cudaGetDevice(&dev) != cudaSuccess || !dev_info(dev, &di)) return DART_ERR_CUDA;
+    if (di.major != 10 || di.minor != 3 || di.optin < kAttnSmem) return DART_ERR_UNSUPPORTED;
+    const int nsm = di.nsm > 0 ? di.nsm : 148;
+    const Plan p = make_plan(cfg, nsm);
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     uint8_t* ws = static_cast<uint8_t*>(workspace);
-    __nv_bfloat16* kr = reinterpret_cast<__nv_bfloat16*>(ws + p.off_kr);
-    float2* cs = reinterpret_cast<float2*>(ws + p.off_cs);
+    __nv_bfloat16* kr = reinterpret_cast<__nv_bfloat16*>(ws + wl.off_kr);
+    float2* cs = reinterpret_cast<float2*>(ws + wl.off_cs);
 
     CUtensorMap tmQ, tmKc, tmVc, tmKt, tmVt;
     if (!encode_q(&tmQ, q, c.nseq, c.B, c.Hq, p.G, p.qpt)) return DART_ERR_CUDA;
@@ -955,7 +981,7 @@ int enqueue_tree_attention(const dart_attn_config* cfg, const void* q, const voi
 
     if (!attn_attr_set(dev)) return DART_ERR_CUDA;
     const int prep_blocks = static_cast<int>(std::min<long long>(
-        (static_cast<long long>(c.nseq) * c.B * c.Hkv + 7) / 8, 16LL * (nsm > 0 ? nsm : 148)));  // 8 rows per block
+        (static_cast<long long>(c.nseq) * c.B * c.Hkv + 7) / 8, 16LL * nsm));  // 8 rows per block
     if (ev && cudaEventRecord(ev[0], st) != cudaSuccess) return DART_ERR_CUDA;
     if (launch_pdl(attn_prep_kernel, dim3(prep_blocks), dim3(256), 0, st, ra) != cudaSuccess) return DART_ERR_CUDA;
     if (ev && cudaEventRecord(ev[1], st) != cudaSuccess) return DART_ERR_CUDA;
@@ -978,7 +1004,7 @@ extern "C" {
 
 size_t dart_tree_attention_workspace(const dart_attn_config* cfg) {
     if (!valid_cfg(cfg)) return 0;
-    return make_plan(cfg, sm_count()).total;
+    return ws_layout(cfg).total;
 }
 
 

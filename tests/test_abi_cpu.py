@@ -125,3 +125,15 @@ def test_tree_attention_rejects_null_and_misaligned_pointers():
     assert lib.dart_ancestor_mask(p, p, 1, 0, p, None) == dart.DART_ERR_INVALID
     assert lib.dart_ancestor_mask(p, p, 0, 8, p, None) == dart.DART_ERR_INVALID
     assert lib.dart_ancestor_mask(p, p, 1, 1025, p, None) == dart.DART_ERR_INVALID
+
+
+def test_tree_attention_rejects_a_small_workspace_on_host():
+    lib = dart.lib()
+    cfg = attn_cfg()
+    need = lib.dart_tree_attention_workspace(C.byref(cfg))
+    # rotated tree keys (bf16) and the (cos, sin) table of the tree positions
+    assert need >= 1 * 64 * 8 * 128 * 2 + 1 * 64 * 64 * 8
+    buf = (C.c_uint8 * 1024)()
+    p = (C.cast(buf, C.c_void_p).value + 255) & ~255
+    rc = lib.dart_tree_attention(C.byref(cfg), p, p, p, p, p, p, p, p, p, p, need - 1, None, None)
+    assert rc == dart.DART_ERR_INVALID
