@@ -65,6 +65,7 @@ int ng_index(int NG) { return NG == 16 ? 0 : (NG == 32 ? 1 : (NG == 64 ? 2 : 3))
 
 struct DepthPlan {
     int N, P, NG, G, nV, stages, smem;  // LM-head scoring
+    int l2pf;                            // LM-head: E tiles per CTA prefetched into L2 before its wait
     int nlist, klist;                    // sorted key lists per node and their length (merge input)
     int cand_ds;                         // candidate scoring: d slices per candidate group
     int Nc, Pn;                          // children (head update) at this depth
@@ -181,6 +182,8 @@ GemmArgs gemm_plan(const dart_handle* h, int K, int Nc, int lo_kb_end, bool tc) 
     return g;
 }
 
+constexpr long long kL2PrefetchBytes = 64ll << 20;  // about half of the 126 MB L2
+
 int tc_stages(int smem_optin, int stage_bytes, int fixed) {
     int s = (smem_optin - fixed) / stage_bytes;
     return std::min(16, s);
@@ -221,8 +224,19 @@ int build_plans(dart_handle* h) {
             }
             if (p.stages < 2) return DART_ERR_UNSUPPORTED;
             p.smem = lmhead_tc_fixed_smem(p.NG, c.k, p.stages) + p.stages * tc_stage_bytes(p.NG);
+            // One node group: every CTA streams its own slice of E and the
+            // launch is HBM-bound.  Besides the stages it loads before
+            // waiting on the previous kernel (which is latency-bound and
+            // leaves HBM idle), each CTA then prefetches its next E tiles
+            // into L2, about kL2PrefetchBytes over all CTAs.  Measured on
+            // GB300: -0.4 % per round (d = 4096), -1.2 % (d = 2560); with
+            // several node groups (tensor-bound, each E tile read by every
+            // group) it costs +1 %, so it is off there.
+            p.l2pf = p.G == 1 ? static_cast<int>(kL2PrefetchBytes / (static_cast<long long>(kTileM) * kBlockK * 2) / p.nV)
+                              : 0;
         } else {
             p.stages = 0;
+            p.l2pf = 0;
             p.smem = lmhead_f32_smem(p.NG, c.k);
             if (p.smem > h->smem_optin) return DART_ERR_UNSUPPORTED;
         }
@@ -469,6 +483,7 @@ int enqueue_depth(dart_handle* h, int dep, const float* dlog, const float* ancho
     la.dlog_row_off = static_cast<long long>(dep - 1) * c.V;
     la.bhalf = kNPadMax;
     la.stages = p.stages;
+    la.l2pf = p.l2pf;
     la.part_ms = h->part_ms;
     la.part_key = h->part_key;
     la.status = h->status;

@@ -72,6 +72,7 @@ struct LmheadArgs {
     long long dlog_row_off;     // (dep-1) * V
     int bhalf;            // row offset of the lo half in the bf16 state operand
     int stages;           // smem pipeline depth (tcgen05 kernel)
+    int l2pf;             // A tiles prefetched into L2 before the wait on the previous kernel
     float2* part_ms;      // [nV][N]
     uint64_t* part_key;   // [nV][N][k]
     int* status;

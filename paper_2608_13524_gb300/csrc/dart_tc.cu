@@ -80,7 +80,7 @@ __device__ __forceinline__ void drain_wait(uint64_t* bar, uint32_t parity) {
 template <int NG>
 __device__ __forceinline__ void producer(const CUtensorMap* tmA, const CUtensorMap* tmB, const Work& w, int bhalf,
                                          uint8_t* ring, int stages, uint64_t* full, uint64_t* empty,
-                                         volatile int* abort, int* status) {
+                                         volatile int* abort, int* status, int l2pf = 0) {
     const uint64_t pol_a = l2_policy_evict_first();  // streamed once
     const uint64_t pol_b = l2_policy_evict_last();   // re-read by every tile
     const int kbs = w.kb1 - w.kb0;
@@ -94,6 +94,11 @@ __device__ __forceinline__ void producer(const CUtensorMap* tmA, const CUtensorM
         const bool lo = kb < w.lo_kb_end;
         mbar_arrive_expect_tx(&full[f], kATileBytes + NG * 128 * (lo ? 2 : 1));
         tma_load_2d(ring + f * Layout<NG>::kStage, tmA, &full[f], kb * kBlockK, w.row0 + i * kTileM, pol_a);
+    }
+    // and the next `l2pf` into L2, while the previous kernel still runs
+    for (uint32_t f = pre; f < pre + static_cast<uint32_t>(l2pf) && f < total; f++) {
+        const int i = static_cast<int>(f) / kbs, kb = w.kb0 + static_cast<int>(f) % kbs;
+        tma_prefetch_2d(tmA, kb * kBlockK, w.row0 + i * kTileM);
     }
     pdl_wait();
     for (uint32_t f = 0; f < pre; f++) {
@@ -291,7 +296,8 @@ __global__ void __launch_bounds__(threads<NG>(), 1)
     volatile int* abort = &s.misc[1];
 
     if (warp == 0) {
-        if (lane == 0) producer<NG>(&tmE, &tmH, w, a.bhalf, s.ring, stages, s.full, s.empty, abort, a.status);
+        if (lane == 0)
+            producer<NG>(&tmE, &tmH, w, a.bhalf, s.ring, stages, s.full, s.empty, abort, a.status, a.l2pf);
     } else if (warp == 1) {
         if (lane == 0)
             mma_issuer<NG>(w, s.ring, stages, s.full, s.empty, s.tfull, s.tempty, s.tdown, tmem_base,
