@@ -106,6 +106,8 @@ struct dart_handle {
     int* cand_tok;   // [nseq][L][cand_k] candidate sets C_d (cand_k > 0)
     float* cand_scratch;  // candidate scoring partial dot products
     int* cand_ticket;     // [nseq][ceil(cand_k/8)]
+    uint64_t* cand_part;  // [nseq * L][slices][cand_k] per-slice top keys of the candidate selection
+    int* cand_rticket;    // [nseq * L] slices finished per row
     std::vector<void*> allocs;
     CUtensorMap tmE, tmWi, tmWo, tmH[4], tmX[3], tmA[3];
     // host-buffer staging
@@ -355,6 +357,9 @@ int alloc_workspace(dart_handle* h) {
         DART_ALLOC(h->cand_tok, static_cast<size_t>(c.nseq) * c.L * c.cand_k)
         DART_ALLOC(h->cand_scratch, scr)
         DART_ALLOC(h->cand_ticket, static_cast<size_t>(c.nseq) * ((c.cand_k + 7) / 8))
+        DART_ALLOC(h->cand_part, static_cast<size_t>(c.nseq) * c.L *
+                                     cand_topk_slices(c.V, c.cand_k, c.nseq * c.L, h->num_sms) * c.cand_k)
+        DART_ALLOC(h->cand_rticket, static_cast<size_t>(c.nseq) * c.L)
     }
 #undef DART_ALLOC
     if (rc != DART_OK) return rc;
@@ -382,7 +387,8 @@ int alloc_workspace(dart_handle* h) {
         int score_smem = 48 * 1024;
         for (int dep = 1; dep <= c.L; dep++)
             score_smem = std::max(score_smem, cand_score_smem(h->plans[dep].P, c.d, h->plans[dep].cand_ds));
-        if (cudaMemset(h->cand_ticket, 0, c.nseq * ((c.cand_k + 7) / 8) * sizeof(int)) != cudaSuccess)
+        if (cudaMemset(h->cand_ticket, 0, c.nseq * ((c.cand_k + 7) / 8) * sizeof(int)) != cudaSuccess ||
+            cudaMemset(h->cand_rticket, 0, static_cast<size_t>(c.nseq) * c.L * sizeof(int)) != cudaSuccess)
             return DART_ERR_CUDA;
         if (cand_set_smem_limits(std::max(cand_topk_smem(c.cand_k), 48 * 1024), score_smem) != cudaSuccess)
             return DART_ERR_CUDA;
@@ -460,7 +466,9 @@ int enqueue_depth(dart_handle* h, int dep, const float* dlog, const float* ancho
         if (c.cand_k > 0) {
             // C_d = TopK(L_d^base, K) of every position of every sequence
             const int pc = prof_begin(h, kCandTopk, st);
-            e = launch_cand_topk(dlog, c.nseq * c.L, c.V, c.cand_k, h->cand_tok, st);
+            const int rows = c.nseq * c.L;
+            e = launch_cand_topk(dlog, rows, c.V, c.cand_k, cand_topk_slices(c.V, c.cand_k, rows, h->num_sms),
+                                 h->cand_tok, h->cand_part, h->cand_rticket, st);
             prof_end(h, pc, st);
             if (e != cudaSuccess) return DART_ERR_CUDA;
         }

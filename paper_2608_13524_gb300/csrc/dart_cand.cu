@@ -13,6 +13,8 @@
 //               part_ms[n][i] = (z, 1), part_key[n][i] = key(z, c), so the
 //               merge kernel computes log-sum-exp over C_d (q~ renormalised
 //               over the candidates) and the node's top-k unchanged.
+#include <algorithm>
+
 #include "dart_device.cuh"
 #include "dart_kernels.h"
 
@@ -102,19 +104,24 @@ __device__ __forceinline__ void for_row(const float* x, int V, F&& f) {
     }
 }
 
-// One block per (sequence, position) row; keys key(x, v) order by (value
-// desc, token asc).  Pass 1: every thread finds the largest key of its share
-// of the row.  Bound T: in every warp the m-th largest of these maxima
+// S blocks per (sequence, position) row, block j taking the slice
+// [V j / S, V (j + 1) / S) of the row; keys key(x, v) order by (value desc,
+// token asc).  Every block finds the exact top min(K, slice) keys of its
+// slice; the global top K is among them.  Pass 1: every thread finds the
+// largest key of its share of the slice.  Bound T: in every warp the m-th largest of these maxima
 // (m = ceil(K/32), warp bitonic sort), minimised over the warps -- at least
 // 32*m >= K threads hold a key >= T, so the K-th largest key is >= T, and
 // only a small multiple of K keys reach it.  Pass 2 gathers the keys >= T
-// (the row is now in L2) and the top K of them are ranked in shared memory.
-// If more than kCollCap keys reach T (pathological rows, e.g. many equal
-// values), an exact radix select over the row decides instead: 12 bits per
-// pass from the top, the keys above the threshold digit taken, and once the
-// threshold digit holds at most kCollCap keys they are gathered for an
-// in-memory select.
-__global__ void __launch_bounds__(kTopkThreads) cand_topk_kernel(const float* dlog, int V, int K, int* cand_tok) {
+// (the slice is now in L2) and the top K of them are ranked in shared
+// memory.  If more than kCollCap keys reach T (pathological rows, e.g. many
+// equal values), an exact radix select over the slice decides instead: 12
+// bits per pass from the top, the keys above the threshold digit taken, and
+// once the threshold digit holds at most kCollCap keys they are gathered for
+// an in-memory select.  With S > 1 each block publishes its keys (zeros past
+// its count) and the last block of the row to finish (atomic ticket; nobody
+// waits) selects the K largest of the S K published keys.
+__global__ void __launch_bounds__(kTopkThreads)
+    cand_topk_kernel(const float* dlog, int V, int K, int S, int* cand_tok, uint64_t* part, int* ticket) {
     pdl_trigger();
     pdl_wait();
     extern __shared__ uint64_t csm[];
@@ -127,17 +134,22 @@ __global__ void __launch_bounds__(kTopkThreads) cand_topk_kernel(const float* dl
     __shared__ uint64_t wmin[kTopkThreads / 32];
     __shared__ int dig[2];
     __shared__ int cnt[2];  // [0] keys taken into out, [1] keys gathered into coll
-    const float* x = dlog + static_cast<size_t>(blockIdx.x) * V;
+    __shared__ int last;
+    const int row = blockIdx.x / S, sl = blockIdx.x % S;
+    const int v0 = static_cast<int>(static_cast<long long>(V) * sl / S);
+    const int Vs = static_cast<int>(static_cast<long long>(V) * (sl + 1) / S) - v0;
+    const int Kl = min(K, Vs);  // keys this block selects from its slice
+    const float* x = dlog + static_cast<size_t>(row) * V + v0;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     if (tid == 0) cnt[0] = cnt[1] = 0;
     // pass 1: this thread's largest key
     uint64_t mx = 0ull;
-    for_row(x, V, [&](float xv, int v) {
-        const uint64_t k = make_key(xv, static_cast<uint32_t>(v));
+    for_row(x, Vs, [&](float xv, int v) {
+        const uint64_t k = make_key(xv, static_cast<uint32_t>(v0 + v));
         mx = k > mx ? k : mx;
     });
     {
-        const int m = (K + 31) / 32;
+        const int m = (Kl + 31) / 32;
         uint64_t hv = mx;
 #pragma unroll
         for (int size = 2; size <= 32; size <<= 1) {
@@ -156,8 +168,8 @@ __global__ void __launch_bounds__(kTopkThreads) cand_topk_kernel(const float* dl
     uint64_t T = wmin[0];
     for (int w = 1; w < kTopkThreads / 32; w++) T = wmin[w] < T ? wmin[w] : T;
     // pass 2: gather every key >= T
-    for_row(x, V, [&](float xv, int v) {
-        const uint64_t k = make_key(xv, static_cast<uint32_t>(v));
+    for_row(x, Vs, [&](float xv, int v) {
+        const uint64_t k = make_key(xv, static_cast<uint32_t>(v0 + v));
         if (k >= T) {
             const int pos = atomicAdd(&cnt[1], 1);
             if (pos < kCollCap) coll[pos] = k;
@@ -168,16 +180,16 @@ __global__ void __launch_bounds__(kTopkThreads) cand_topk_kernel(const float* dl
     const bool inexact = ng > kCollCap;
     __syncthreads();  // every thread has read the count before it is reused
     if (!inexact) {
-        // the K largest of the ng gathered keys (ng >= K, keys distinct)
+        // the Kl largest of the ng gathered keys (ng >= Kl, keys distinct)
         if (ng <= kRankMax) {
             for (int i = tid; i < ng; i += kTopkThreads) {
                 const uint64_t k = coll[i];
                 int r = 0;
                 for (int j = 0; j < ng; j++) r += coll[j] > k;
-                if (r < K) out[r] = k;
+                if (r < Kl) out[r] = k;
             }
         } else {
-            const uint64_t kth = block_kth_largest(coll, ng, K, hist8, scal);
+            const uint64_t kth = block_kth_largest(coll, ng, Kl, hist8, scal);
             for (int i = tid; i < ng; i += kTopkThreads)
                 if (coll[i] >= kth) out[atomicAdd(&cnt[0], 1)] = coll[i];
         }
@@ -187,7 +199,7 @@ __global__ void __launch_bounds__(kTopkThreads) cand_topk_kernel(const float* dl
         if (tid == 0) cnt[0] = cnt[1] = 0;
         __syncthreads();
         uint64_t prefix = 0, mask = 0;
-        int need = K;
+        int need = Kl;
         // at most 6 passes: after the 4-bit sixth digit the prefix is the whole
         // key, which is unique, so the threshold digit holds <= 1 key
         for (int level = 0, shift = 64 - kDigitBits; level < 6; level++, shift -= kDigitBits) {
@@ -195,8 +207,8 @@ __global__ void __launch_bounds__(kTopkThreads) cand_topk_kernel(const float* dl
             const uint64_t dmask = (shift > 0 ? static_cast<uint64_t>(kBins - 1) : ((1ull << (kDigitBits + shift)) - 1));
             for (int i = tid; i < kBins; i += kTopkThreads) hist[i] = 0;
             __syncthreads();
-            for (int v = tid; v < V; v += kTopkThreads) {
-                const uint64_t k = make_key(__ldg(x + v), static_cast<uint32_t>(v));
+            for (int v = tid; v < Vs; v += kTopkThreads) {
+                const uint64_t k = make_key(__ldg(x + v), static_cast<uint32_t>(v0 + v));
                 if ((k & mask) == prefix) atomicAdd(&hist[(k >> sh) & dmask], 1u);
             }
             __syncthreads();
@@ -206,8 +218,8 @@ __global__ void __launch_bounds__(kTopkThreads) cand_topk_kernel(const float* dl
             const int above = dig[1];
             const int m = static_cast<int>(hist[b]);
             const bool finish = m <= kCollCap;
-            for (int v = tid; v < V; v += kTopkThreads) {
-                const uint64_t k = make_key(__ldg(x + v), static_cast<uint32_t>(v));
+            for (int v = tid; v < Vs; v += kTopkThreads) {
+                const uint64_t k = make_key(__ldg(x + v), static_cast<uint32_t>(v0 + v));
                 if ((k & mask) != prefix) continue;
                 const uint64_t dg = (k >> sh) & dmask;
                 if (dg > b)
@@ -230,12 +242,36 @@ __global__ void __launch_bounds__(kTopkThreads) cand_topk_kernel(const float* dl
             __syncthreads();
         }
     }
+    if (S > 1) {
+        // publish this slice's keys; the last block of the row merges
+        uint64_t* pp = part + (static_cast<size_t>(row) * S + sl) * K;
+        for (int i = tid; i < K; i += kTopkThreads) pp[i] = i < Kl ? out[i] : 0ull;
+        __threadfence();
+        __syncthreads();
+        if (tid == 0) last = atomicAdd(&ticket[row], 1) == S - 1;
+        __syncthreads();
+        if (!last) return;
+        __threadfence();
+        if (tid == 0) {
+            ticket[row] = 0;
+            cnt[0] = 0;
+        }
+        // S K <= kCollCap keys, non-zero ones distinct, at least K of them
+        const int ng = S * K;
+        const uint64_t* rp = part + static_cast<size_t>(row) * S * K;
+        for (int i = tid; i < ng; i += kTopkThreads) coll[i] = __ldcg(rp + i);
+        __syncthreads();
+        const uint64_t kth = block_kth_largest(coll, ng, K, hist8, scal);
+        for (int i = tid; i < ng; i += kTopkThreads)
+            if (coll[i] >= kth && coll[i] != 0ull) out[atomicAdd(&cnt[0], 1)] = coll[i];
+        __syncthreads();
+    }
     // write the K tokens in ascending order (rank by counting)
     for (int i = tid; i < K; i += kTopkThreads) {
         const uint32_t tk = key_idx(out[i]);
         int r = 0;
         for (int j = 0; j < K; j++) r += key_idx(out[j]) < tk;
-        cand_tok[static_cast<size_t>(blockIdx.x) * K + r] = static_cast<int>(tk);
+        cand_tok[static_cast<size_t>(row) * K + r] = static_cast<int>(tk);
     }
 }
 
@@ -359,6 +395,16 @@ __global__ void __launch_bounds__(kScoreThreads) cand_score_kernel(const CandArg
 
 int cand_topk_smem(int K) { return (kCollCap + K + kRankMax) * 8 + kBins * 4; }
 
+// Blocks per row of the candidate top-K: slices of at least 4096 logits
+// (several per thread of the block), at most 8, S K keys within the merge's
+// shared-memory buffer, and rows x S within one block per SM (measured on
+// GB300: 8 slices of 16 rows -2 % per round at K = 64; 8 slices of 128 rows,
+// several waves, +2.4 %).
+int cand_topk_slices(int V, int K, int rows, int num_sms) {
+    const int s = std::min(std::min(8, V / 4096), std::min(kCollCap / K, num_sms / std::max(rows, 1)));
+    return std::max(1, s);
+}
+
 int cand_score_slices(int P, int d, int nseq, int K, int max_smem) {
     // slices of d per block: enough blocks to spread the loads (>= 128), the
     // staged slice within 64 KB, and d / DS a multiple of 4 floats
@@ -380,8 +426,10 @@ cudaError_t cand_set_smem_limits(int topk_smem, int score_smem) {
     return e;
 }
 
-cudaError_t launch_cand_topk(const float* dlog, int rows, int V, int K, int* cand_tok, cudaStream_t st) {
-    return launch_pdl(cand_topk_kernel, dim3(rows), dim3(kTopkThreads), cand_topk_smem(K), st, dlog, V, K, cand_tok);
+cudaError_t launch_cand_topk(const float* dlog, int rows, int V, int K, int S, int* cand_tok, uint64_t* part,
+                             int* ticket, cudaStream_t st) {
+    return launch_pdl(cand_topk_kernel, dim3(rows * S), dim3(kTopkThreads), cand_topk_smem(K), st, dlog, V, K, S,
+                      cand_tok, part, ticket);
 }
 
 cudaError_t launch_cand_score(const CandArgs& a, cudaStream_t st) {

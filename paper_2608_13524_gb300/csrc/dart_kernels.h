@@ -164,7 +164,12 @@ struct CandArgs {
     float* scratch;             // [DS][nseq*P][K] partial dot products
     int* ticket;                // [nseq][ceil(K/8)] zero between launches
 };
-cudaError_t launch_cand_topk(const float* dlog, int rows, int V, int K, int* cand_tok, cudaStream_t st);
+// S = cand_topk_slices(V, K, rows, SMs) blocks per row; part: [rows][S][K]
+// keys, ticket: [rows] ints, zero before the first launch (every launch
+// leaves them zero).
+cudaError_t launch_cand_topk(const float* dlog, int rows, int V, int K, int S, int* cand_tok, uint64_t* part,
+                             int* ticket, cudaStream_t st);
+int cand_topk_slices(int V, int K, int rows, int num_sms);
 cudaError_t launch_cand_score(const CandArgs& a, cudaStream_t st);
 int cand_topk_smem(int K);
 int cand_score_slices(int P, int d, int nseq, int K, int max_smem);  // 0: does not fit
