@@ -91,6 +91,7 @@ struct GemmArgs {
     int bhalf;
     int stages;
     int mode;             // tcgen05 path: kGemmPartials, or kGemmSiluSplit / kGemmSum (the k splits are one cluster)
+    int keep_a;           // load A (the weights) evict-last: it is read again at the next depth from L2
     float* out;           // fp32 path: partials [S][N][M]; kGemmSum: the sum [N][M]
     __nv_bfloat16* outL;  // kGemmSiluSplit: SiLU of the sum as hi rows [N][M], lo rows from row bhalf
     int* status;

@@ -80,8 +80,10 @@ __device__ __forceinline__ void drain_wait(uint64_t* bar, uint32_t parity) {
 template <int NG>
 __device__ __forceinline__ void producer(const CUtensorMap* tmA, const CUtensorMap* tmB, const Work& w, int bhalf,
                                          uint8_t* ring, int stages, uint64_t* full, uint64_t* empty,
-                                         volatile int* abort, int* status, int l2pf = 0) {
-    const uint64_t pol_a = l2_policy_evict_first();  // streamed once
+                                         volatile int* abort, int* status, int l2pf = 0, bool keep_a = false) {
+    // A: streamed once (E), or kept for the next depth (head weights when
+    // nothing else streams through L2)
+    const uint64_t pol_a = keep_a ? l2_policy_evict_last() : l2_policy_evict_first();
     const uint64_t pol_b = l2_policy_evict_last();   // re-read by every tile
     const int kbs = w.kb1 - w.kb0;
     const uint32_t total = static_cast<uint32_t>(w.ntiles * kbs);
@@ -456,7 +458,8 @@ __global__ void __launch_bounds__(threads<NG>(), 1)
     float* stage_tile = reinterpret_cast<float*>(s.ring);
 
     if (warp == 0) {
-        if (lane == 0) producer<NG>(&tmA, &tmB, w, a.bhalf, s.ring, stages, s.full, s.empty, abort, a.status);
+        if (lane == 0)
+            producer<NG>(&tmA, &tmB, w, a.bhalf, s.ring, stages, s.full, s.empty, abort, a.status, 0, a.keep_a != 0);
     } else if (warp == 1) {
         if (lane == 0)
             mma_issuer<NG>(w, s.ring, stages, s.full, s.empty, s.tfull, s.tempty, s.tdown, tmem_base,
