@@ -185,7 +185,7 @@ GemmArgs gemm_plan(const dart_handle* h, int K, int Nc, int lo_kb_end, bool tc) 
 }
 
 constexpr long long kL2PrefetchBytes = 64ll << 20;  // about half of the 126 MB L2
-constexpr long long kL2KeepBytes = 64ll << 20;      // head weights kept in L2 across depths, at most
+constexpr long long kL2KeepBytes = 72ll << 20;      // head weights kept in L2 across depths, at most
 
 int tc_stages(int smem_optin, int stage_bytes, int fixed) {
     int s = (smem_optin - fixed) / stage_bytes;
@@ -299,16 +299,23 @@ int build_plans(dart_handle* h) {
                 p.g2.mode = cluster ? kGemmSum : kGemmPartials;
                 // Candidate-restricted scoring streams nothing through L2
                 // between the depths: with <= 16 children (weight-bound
-                // GEMMs), head weights that fit in half of it (W_o, 2 d^2
-                // bytes, first; then W_i, 4 d^2) are loaded evict-last and
-                // read from HBM once per round instead of once per depth.
-                // Measured on GB300 (A/B, K = 64): -4.9 % per round at d =
-                // 2560 (both kept), -2.0 % at d = 4096 (W_o kept); both kept
-                // at d = 4096 (100 MB) +2.1 %; W_o kept with 256 children
+                // GEMMs) the largest of {W_i and W_o, W_i (4 d^2 bytes), W_o
+                // (2 d^2)} within kL2KeepBytes is loaded evict-last and read
+                // from HBM once per round instead of once per depth.
+                // Measured on GB300 (A/B, K = 64): d = 2560, both (39 MB):
+                // -4.9 % per round; d = 4096: W_i (67 MB) -6.0 %, W_o
+                // (34 MB) -2.0 %, both (101 MB) +2.1 %; W_o with 256 children
                 // (cluster GEMMs) +0.8 %.
                 const long long wo_bytes = 2ll * c.d * c.d, wi_bytes = 4ll * c.d * c.d;
-                p.g2.keep_a = c.cand_k > 0 && !cluster && wo_bytes <= kL2KeepBytes;
-                p.g1.keep_a = p.g2.keep_a && wo_bytes + wi_bytes <= kL2KeepBytes;
+                p.g1.keep_a = p.g2.keep_a = 0;
+                if (c.cand_k > 0 && !cluster) {
+                    if (wi_bytes + wo_bytes <= kL2KeepBytes)
+                        p.g1.keep_a = p.g2.keep_a = 1;
+                    else if (wi_bytes <= kL2KeepBytes)
+                        p.g1.keep_a = 1;
+                    else if (wo_bytes <= kL2KeepBytes)
+                        p.g2.keep_a = 1;
+                }
             }
         }
     }
