@@ -106,6 +106,20 @@ def kernel_source_sha():
     return code_sha(("dart_tc.cu", "dart_device.cuh"))
 
 
+def kept_head_weights(cfg):
+    """(W_i kept, W_o kept): the head weights the library loads evict-last
+    so that they stay in L2 across the depths of a round.  Mirrors its plan:
+    candidate-restricted scoring, <= 16 children, the largest of {both, W_i,
+    W_o} within 72 MiB (bf16 weights)."""
+    if cfg.cand_k == 0 or cfg.wdtype != "bf16" or cfg.nseq * cfg.W > 16:
+        return False, False
+    cap = 72 << 20
+    wi, wo = 4 * cfg.d * cfg.d, 2 * cfg.d * cfg.d
+    if wi + wo <= cap:
+        return True, True
+    return wi <= cap, wi > cap and wo <= cap
+
+
 def recorded_traffic(workload):
     """DRAM bytes per LM-head launch from the committed ncu summary, if it was
     taken on the current kernel source."""
@@ -606,8 +620,21 @@ def main():
     kinds = dart.dart_profile_read_kinds(h)
     dart.dart_set_profiling(h, False)
     # roofline kernel: the LM-head stream, or with candidate-restricted
-    # scoring the largest remaining HBM stream, the W_i GEMM (2*d*d weights)
-    rl_kind = "lmhead" if cfg.cand_k == 0 else "gemm_wi"
+    # scoring the head GEMM whose weights stream from HBM at every depth (W_i,
+    # 4 d^2 bytes, else W_o, 2 d^2); when both stay in L2 the W_i GEMM with
+    # its weights counted once per round (the HBM reads it needs)
+    wi_kept, wo_kept = kept_head_weights(cfg)
+    if cfg.cand_k == 0:
+        rl_kind, rl_name, bytes_launch, rl_note = "lmhead", "lmhead_tc_kernel", cfg.lmhead_bytes_per_depth(), None
+    elif not wi_kept:
+        rl_kind, rl_name, bytes_launch, rl_note = "gemm_wi", "gemm_tc_kernel (W_i)", 2 * cfg.d * cfg.d * cfg.bpe, None
+    elif not wo_kept:
+        rl_kind, rl_name, bytes_launch, rl_note = ("gemm_wo", "gemm_tc_kernel (W_o)", cfg.d * cfg.d * cfg.bpe,
+                                                   "W_i stays in L2 across depths; W_o streams from HBM")
+    else:
+        rl_kind, rl_name = "gemm_wi", "gemm_tc_kernel (W_i)"
+        bytes_launch = 2 * cfg.d * cfg.d * cfg.bpe / max(1, cfg.L - 1)
+        rl_note = "W_i and W_o stay in L2 across depths: W_i bytes counted once per round"
     k1_ms, k1_n = kinds[rl_kind]
     k1_avg_s = k1_ms / 1e3 / max(1, k1_n)
     breakdown = {k: {"us_per_round": v[0] * 1e3 / args.steps, "launches_per_round": v[1] / args.steps,
@@ -615,7 +642,6 @@ def main():
 
     exp_round = cfg.expansions_per_round()
     value = whole_job_rate(exp_round, world, ms / 1e3)
-    bytes_launch = cfg.lmhead_bytes_per_depth() if cfg.cand_k == 0 else 2 * cfg.d * cfg.d * cfg.bpe
     lm_bytes_round = cfg.L * cfg.V * cfg.d * cfg.bpe if cfg.cand_k == 0 else None
     peak, peak_kind = measured_peak()
     achieved = bytes_launch / k1_avg_s / 1e9
@@ -664,7 +690,7 @@ def main():
             "us_per_round": ms * 1e3,
             "lmhead_gbs": lm_bytes_round / (ms / 1e3) / 1e9 if lm_bytes_round else None,
             "lmhead_frac_of_8tbs": lm_bytes_round / (ms / 1e3) / 1e9 / NOMINAL_HBM_GBS if lm_bytes_round else None,
-            "roofline": {"kernel": "lmhead_tc_kernel" if cfg.cand_k == 0 else "gemm_tc_kernel (W_i)",
+            "roofline": {"kernel": rl_name, "note": rl_note,
                          "bound": "hbm", "achieved": achieved, "peak": peak,
                          "peak_kind": peak_kind, "unit": "GB/s", "frac": achieved / peak,
                          "traffic": traffic, "bytes_per_launch": bytes_launch,
