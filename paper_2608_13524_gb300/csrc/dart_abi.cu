@@ -227,16 +227,17 @@ int build_plans(dart_handle* h) {
             }
             if (p.stages < 2) return DART_ERR_UNSUPPORTED;
             p.smem = lmhead_tc_fixed_smem(p.NG, c.k, p.stages) + p.stages * tc_stage_bytes(p.NG);
-            // One node group: every CTA streams its own slice of E and the
-            // launch is HBM-bound.  Besides the stages it loads before
-            // waiting on the previous kernel (which is latency-bound and
-            // leaves HBM idle), each CTA then prefetches its next E tiles
-            // into L2, about kL2PrefetchBytes over all CTAs.  Measured on
-            // GB300: -0.4 % per round (d = 4096), -1.2 % (d = 2560); with
-            // several node groups (tensor-bound, each E tile read by every
-            // group) it costs +1 %, so it is off there.
-            p.l2pf = p.G == 1 ? static_cast<int>(kL2PrefetchBytes / (static_cast<long long>(kTileM) * kBlockK * 2) / p.nV)
-                              : 0;
+            // One group of <= 16 nodes: every CTA streams its own slice of
+            // E and the launch is HBM-bound.  Besides the stages it loads
+            // before waiting on the previous kernel (which is latency-bound
+            // and leaves HBM idle), each CTA then prefetches its next E
+            // tiles into L2, about kL2PrefetchBytes over all CTAs.  Measured
+            // on GB300 (A/B per round): -0.55 % at d = 4096, -1.0 % at
+            // d = 2560, -0.8 % with 16 nodes at d = 2560; with 32 or 64
+            // nodes (+2.5 %, +1.0 %) or several groups (+1 %) it is off.
+            p.l2pf = (p.G == 1 && p.NG <= 16)
+                         ? static_cast<int>(kL2PrefetchBytes / (static_cast<long long>(kTileM) * kBlockK * 2) / p.nV)
+                         : 0;
         } else {
             p.stages = 0;
             p.l2pf = 0;
