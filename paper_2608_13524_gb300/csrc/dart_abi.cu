@@ -45,12 +45,14 @@ constexpr int kMaxProfilePairs = 8192;
 
 EncodeTiledFn encode_fn() { return tensor_map_encoder(); }
 
-// 2-D bf16 tensor [rows][inner] with a (64 x box_rows) box and 128-byte swizzle.
-bool encode_bf16_2d(CUtensorMap* m, const void* base, uint64_t inner, uint64_t rows, uint32_t box_rows) {
+// 2-D bf16 tensor [rows][inner] (row pitch `pitch` elements, default inner)
+// with a (64 x box_rows) box and 128-byte swizzle.
+bool encode_bf16_2d(CUtensorMap* m, const void* base, uint64_t inner, uint64_t rows, uint32_t box_rows,
+                    uint64_t pitch = 0) {
     EncodeTiledFn fn = encode_fn();
     if (!fn) return false;
     cuuint64_t dims[2] = {inner, rows};
-    cuuint64_t strides[1] = {inner * 2};
+    cuuint64_t strides[1] = {(pitch ? pitch : inner) * 2};
     cuuint32_t box[2] = {static_cast<cuuint32_t>(kBlockK), box_rows};
     cuuint32_t estr[2] = {1, 1};
     return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
@@ -69,6 +71,7 @@ struct DepthPlan {
     int nlist, klist;                    // sorted key lists per node and their length (merge input)
     int cand_ds;                         // candidate scoring: d slices per candidate group
     int Nc, Pn;                          // children (head update) at this depth
+    int split;                           // g1 = W_i[:, 0:d] . h over the N parents; E half from the Q table
     GemmArgs g1, g2;                     // head GEMMs (depth < L)
     int g1_smem, g2_smem;
 };
@@ -108,8 +111,10 @@ struct dart_handle {
     int* cand_ticket;     // [nseq][ceil(cand_k/8)]
     uint64_t* cand_part;  // [nseq * L][slices][cand_k] per-slice top keys of the candidate selection
     int* cand_rticket;    // [nseq * L] slices finished per row
+    float* Qtab;          // [V][d] fp32: Q[t] = W_i[:, d:2d] . E[t] (split first head layer), or null
     std::vector<void*> allocs;
     CUtensorMap tmE, tmWi, tmWo, tmH[4], tmX[3], tmA[3];
+    CUtensorMap tmWiR, tmEB;  // Q table: A = W_i[:, d:2d] (128-row box), B = E rows as 64-node groups
     // host-buffer staging
     float *st_dlog, *st_anchor;
     dart_tree_out st_out;
@@ -253,8 +258,18 @@ int build_plans(dart_handle* h) {
         }
         p.Pn = h->caps[dep];
         p.Nc = c.nseq * p.Pn;
+        p.split = 0;
         if (dep < c.L) {
-            p.g1 = gemm_plan(h, 2 * c.d, p.Nc, c.d / kBlockK, tc);
+            // Split first head layer (full vocabulary, <= 16 children, bf16):
+            //   W_i . [h_p ; E[t_c]] = W_i[:, 0:d] . h_p + Q[t_c],
+            // Q = the per-token table computed once per handle.  The GEMM then
+            // runs over the parents' states, which the LM-head already holds
+            // as hi/lo rows (no gather of the inputs), streams half of W_i
+            // (its first tiles while merge + select runs), and Q[t_c] is
+            // added in the SiLU kernel.  DART_SPLIT_HEAD=0 turns it off.
+            const char* sh = getenv("DART_SPLIT_HEAD");
+            p.split = (tc && c.cand_k == 0 && p.Nc <= 16 && !(sh && sh[0] == '0')) ? 1 : 0;
+            p.g1 = p.split ? gemm_plan(h, c.d, p.N, c.d / kBlockK, tc) : gemm_plan(h, 2 * c.d, p.Nc, c.d / kBlockK, tc);
             p.g2 = gemm_plan(h, c.d, p.Nc, c.d / kBlockK, tc);
             if (tc) {
                 // two CTAs per SM when both fit with >= 4 stages: twice the
@@ -371,6 +386,9 @@ int alloc_workspace(dart_handle* h) {
     DART_ALLOC(h->seq_ticket, c.nseq)
     DART_ALLOC(h->status, 1)
     DART_ALLOC(h->gthr, static_cast<size_t>(c.L) * kNPadMax)
+    bool any_split = false;
+    for (int dep = 1; dep < c.L; dep++) any_split = any_split || h->plans[dep].split;
+    if (any_split) DART_ALLOC(h->Qtab, static_cast<size_t>(c.V) * d)
     if (c.cand_k > 0) {
         size_t scr = 1;
         for (int dep = 1; dep <= c.L; dep++)
@@ -434,7 +452,42 @@ int make_tensor_maps(dart_handle* h) {
              encode_bf16_2d(&h->tmA[i], h->AL, d, 2 * kNPadMax, ngs[i]);
     }
     if (ok) ok = encode_bf16_2d(&h->tmH[3], h->HL, d, 2 * kNPadMax, 128);  // LM-head 128-node groups
+    if (ok && h->Qtab) {
+        ok = encode_bf16_2d(&h->tmWiR, static_cast<const __nv_bfloat16*>(h->Wi) + d, d, d, kTileM, 2 * d) &&
+             encode_bf16_2d(&h->tmEB, h->E, d, c.V, 64);
+    }
     return ok ? DART_OK : DART_ERR_UNSUPPORTED;
+}
+
+// Q[t][j] = sum_k W_i[j][d + k] * E[t][k] for every token t: one launch of
+// the head GEMM kernel with the roles of the operands swapped (A = the
+// second half of W_i, M = d output features; B = E, V rows as nodes in
+// groups of 64, no lo half since E is exact in bf16), k not split, so its
+// partial tile is the result, written as [V][d].
+int compute_qtab(dart_handle* h, cudaStream_t st) {
+    const dart_config& c = h->cfg;
+    GemmArgs q;
+    std::memset(&q, 0, sizeof q);
+    q.M = c.d;
+    q.K = c.d;
+    q.N = c.V;
+    q.NG = 64;
+    q.G = (c.V + 63) / 64;
+    q.MT = (c.d + kTileM - 1) / kTileM;
+    q.S = 1;
+    q.KB = c.d / kBlockK;
+    q.lo_kb_end = 0;
+    q.bhalf = 0;
+    const int sb = tc_stage_bytes(64);
+    const int st2 = std::min(tc_stages(h->smem_optin / 2 - 2048, sb, gemm_tc_fixed_smem(16)), 8);
+    q.stages = st2 >= 3 ? st2 : std::min(tc_stages(h->smem_optin, sb, gemm_tc_fixed_smem(16)), 8);
+    if (q.stages < 2) return DART_ERR_UNSUPPORTED;
+    q.mode = kGemmPartials;
+    q.keep_a = 1;  // the 2 d^2-byte A operand is read by every node group
+    q.out = h->Qtab;
+    q.status = h->status;
+    const int smem = gemm_tc_fixed_smem(q.stages) + q.stages * sb;
+    return cuda_err(launch_gemm_tc(&h->tmWiR, &h->tmEB, q, smem, st));
 }
 
 void release(dart_handle* h) {
@@ -450,7 +503,10 @@ void release(dart_handle* h) {
 
 // ---------------------------------------------------------------- enqueue
 
-enum Kind { kLmhead = 0, kSelect, kGather, kGemm1, kSilu, kGemm2, kNorm, kPrep, kEmit, kCandTopk, kCandScore, kNumKinds };
+enum Kind {
+    kLmhead = 0, kSelect, kGather, kGemm1, kSilu, kGemm2, kNorm, kPrep, kEmit, kCandTopk, kCandScore, kGatherSilu,
+    kNumKinds
+};
 
 // Opens an event pair around the next launch when profiling (no-op otherwise).
 int prof_begin(dart_handle* h, int kind, cudaStream_t st) {
@@ -589,17 +645,23 @@ int enqueue_depth(dart_handle* h, int dep, const float* dlog, const float* ancho
     // 3) correction-head update of the retained children (Algorithm 1, state update)
     const float* hcur = h->hbuf[h->cur];
     float* hnext = h->hbuf[1 - h->cur];
-    pi = prof_begin(h, kGather, st);
-    e = launch_gather_x(p.Nc, c.d, h->child_prow, h->child_tok, hcur, h->E, tc ? 1 : 0, h->XL, kNPadMax, h->X32, st);
-    prof_end(h, pi, st);
-    if (e != cudaSuccess) return DART_ERR_CUDA;
+    if (!p.split) {
+        pi = prof_begin(h, kGather, st);
+        e = launch_gather_x(p.Nc, c.d, h->child_prow, h->child_tok, hcur, h->E, tc ? 1 : 0, h->XL, kNPadMax, h->X32,
+                            st);
+        prof_end(h, pi, st);
+        if (e != cudaSuccess) return DART_ERR_CUDA;
+    }
     GemmArgs g1 = p.g1, g2 = p.g2;
     g1.out = h->part;
     g1.outL = h->AL;
     g2.out = h->part;
     g1.status = g2.status = h->status;
     pi = prof_begin(h, kGemm1, st);
-    if (tc) {
+    if (p.split) {
+        // W_i[:, 0:d] . h over the parents: B = their hi/lo rows of the LM-head
+        e = launch_gemm_tc(&h->tmWi, &h->tmH[ng_index(g1.NG)], g1, p.g1_smem, st);
+    } else if (tc) {
         e = launch_gemm_tc(&h->tmWi, &h->tmX[ng_index(g1.NG)], g1, p.g1_smem, st);
     } else {
         g1.A32 = static_cast<const float*>(h->Wi);
@@ -609,7 +671,13 @@ int enqueue_depth(dart_handle* h, int dep, const float* dlog, const float* ancho
     prof_end(h, pi, st);
     if (e != cudaSuccess) return DART_ERR_CUDA;
     const bool fused = tc && g1.mode != kGemmPartials;  // SiLU applied in the GEMM's cluster reduction
-    if (!fused) {
+    if (p.split) {
+        pi = prof_begin(h, kGatherSilu, st);
+        e = launch_gather_silu(p.Nc, c.d, g1.S, g1.N, h->part, h->child_prow, h->child_tok, c.V, h->Qtab, h->AL,
+                               kNPadMax, st);
+        prof_end(h, pi, st);
+        if (e != cudaSuccess) return DART_ERR_CUDA;
+    } else if (!fused) {
         pi = prof_begin(h, kSilu, st);
         e = launch_silu_split(p.Nc, c.d, g1.S, h->part, tc ? h->AL : nullptr, kNPadMax, h->A32, st);
         prof_end(h, pi, st);
@@ -707,7 +775,6 @@ const char* dart_status_string(int code) {
 
 int dart_init_head(dart_handle** out, const dart_config* cfg, int wdtype, const void* W_i, const void* W_o,
                    const void* E, void* stream) {
-    (void)stream;
     if (!out) return DART_ERR_INVALID;
     *out = nullptr;
     int rc = validate_cfg(cfg);
@@ -738,6 +805,7 @@ int dart_init_head(dart_handle** out, const dart_config* cfg, int wdtype, const 
     if (rc == DART_OK) rc = build_plans(h);
     if (rc == DART_OK) rc = alloc_workspace(h);
     if (rc == DART_OK && wdtype == DART_BF16) rc = make_tensor_maps(h);
+    if (rc == DART_OK && h->Qtab) rc = compute_qtab(h, static_cast<cudaStream_t>(stream));
     if (rc == DART_OK && cudaStreamCreateWithFlags(&h->cap_stream, cudaStreamNonBlocking) != cudaSuccess)
         rc = DART_ERR_CUDA;
     if (rc == DART_OK && cudaDeviceSynchronize() != cudaSuccess) rc = DART_ERR_CUDA;
@@ -952,10 +1020,13 @@ int dart_profile_read(dart_handle* h, float* lmhead_ms, int* lmhead_launches) {
 int dart_launches_per_round(dart_handle* h) {
     if (!h) return DART_ERR_INVALID;
     const int L = h->cfg.L;
-    // prep, (LM-head + select) per depth, (gather, W_i GEMM, [SiLU,] W_o GEMM,
-    // residual-norm) per depth but the last, prune-emit
+    // prep, (LM-head + select) per depth, then per depth but the last:
+    // gather, W_i GEMM, [SiLU,] W_o GEMM, residual-norm; or with the split
+    // first layer: W_i[:, 0:d] GEMM, gather + SiLU, W_o GEMM, residual-norm;
+    // prune-emit
     int n = 1 + 2 * L + 1 + (h->cfg.cand_k > 0 ? 1 : 0);
-    for (int dep = 1; dep < L; dep++) n += (h->wdtype == DART_BF16 && h->plans[dep].g1.mode != kGemmPartials) ? 4 : 5;
+    for (int dep = 1; dep < L; dep++)
+        n += (h->plans[dep].split || (h->wdtype == DART_BF16 && h->plans[dep].g1.mode != kGemmPartials)) ? 4 : 5;
     return n;
 }
 

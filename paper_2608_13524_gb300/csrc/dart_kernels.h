@@ -199,6 +199,9 @@ cudaError_t launch_gather_x(int Nc, int d, const int* prow, const int* tok, cons
 // a = SiLU(sum_s part[s]) -> AL (hi/lo) or A32
 cudaError_t launch_silu_split(int Nc, int d, int S, const float* part, __nv_bfloat16* AL, int bhalf, float* A32,
                               cudaStream_t st);
+// a = SiLU(Q[tok[c]] + sum_s part[s][prow[c]]) -> AL (hi/lo); part: [S][Np][d]
+cudaError_t launch_gather_silu(int Nc, int d, int S, int Np, const float* part, const int* prow, const int* tok,
+                               int V, const float* Q, __nv_bfloat16* AL, int bhalf, cudaStream_t st);
 // h_next[c] = RMSNorm(h[prow[c]] + sum_s part[s][c]) and its hi/lo split
 cudaError_t launch_residual_norm(int Nc, int d, int S, const float* part, const int* prow, const float* h,
                                  float eps, float* h_next, __nv_bfloat16* HL, int bhalf, cudaStream_t st);

@@ -329,6 +329,35 @@ __global__ void silu_split_kernel(int Nc, int d, int S, const float* part, __nv_
     }
 }
 
+// First head layer with the E half taken from the per-token table
+// Q[t] = W_i[:, d:2d] . E[t] (computed once per handle):
+//   a_c = SiLU(Q[tok[c]] + sum_s part[s][prow[c]]),
+// where part holds the S k-split partials of W_i[:, 0:d] . h over the Np
+// parents, then the hi/lo bf16 split of a_c (input of the W_o GEMM).  Empty
+// child slots (prow < 0) and tokens outside [0, V) give a_c = 0.
+__global__ void gather_silu_kernel(int Nc, int d, int S, int Np, const float* part, const int* prow, const int* tok,
+                                   int V, const float* Q, __nv_bfloat16* AL, int bhalf) {
+    pdl_trigger();
+    pdl_wait();
+    const size_t stride = static_cast<size_t>(Np) * d;
+    const int q4 = d / 4;
+    const int total = Nc * q4;
+    for (int u = blockIdx.x * blockDim.x + threadIdx.x; u < total; u += gridDim.x * blockDim.x) {
+        const int c = u / q4, j = (u % q4) * 4;
+        const int pr = prow[c], t = tok[c];
+        float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (pr >= 0 && static_cast<unsigned>(t) < static_cast<unsigned>(V)) {
+            v = *reinterpret_cast<const float4*>(Q + static_cast<size_t>(t) * d + j);
+            add_splits(v, part + static_cast<size_t>(pr) * d + j, stride, S);
+            v.x = v.x / (1.0f + expf(-v.x));
+            v.y = v.y / (1.0f + expf(-v.y));
+            v.z = v.z / (1.0f + expf(-v.z));
+            v.w = v.w / (1.0f + expf(-v.w));
+        }
+        split4(v, AL + static_cast<size_t>(c) * d + j, AL + static_cast<size_t>(bhalf + c) * d + j);
+    }
+}
+
 // One block per child: r = h[prow] + sum_s part[s], h_next = r / rms(r).
 // NT = 1024 threads when S partial tiles are summed (many loads in flight),
 // 256 for one summed tile (few registers, so blocks can become resident
@@ -418,6 +447,12 @@ cudaError_t launch_silu_split(int Nc, int d, int S, const float* part, __nv_bflo
                               cudaStream_t st) {
     return launch_pdl(silu_split_kernel, dim3(grid_for(static_cast<size_t>(Nc) * d / 4)), dim3(256), 0, st, Nc, d, S,
                       part, AL, bhalf, A32);
+}
+
+cudaError_t launch_gather_silu(int Nc, int d, int S, int Np, const float* part, const int* prow, const int* tok,
+                               int V, const float* Q, __nv_bfloat16* AL, int bhalf, cudaStream_t st) {
+    return launch_pdl(gather_silu_kernel, dim3(grid_for(static_cast<size_t>(Nc) * d / 4)), dim3(256), 0, st, Nc, d, S,
+                      Np, part, prow, tok, V, Q, AL, bhalf);
 }
 
 cudaError_t launch_residual_norm(int Nc, int d, int S, const float* part, const int* prow, const float* h,

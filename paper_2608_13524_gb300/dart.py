@@ -219,7 +219,7 @@ def dart_profile_read(h):
 
 
 KIND_NAMES = ("lmhead", "merge_select", "gather", "gemm_wi", "silu_split", "gemm_wo", "residual_norm",
-              "prep_anchor", "prune_emit", "cand_topk", "cand_score")
+              "prep_anchor", "prune_emit", "cand_topk", "cand_score", "gather_silu")
 
 
 def dart_profile_read_kinds(h):
