@@ -72,6 +72,7 @@ struct DepthPlan {
     int cand_ds;                         // candidate scoring: d slices per candidate group
     int Nc, Pn;                          // children (head update) at this depth
     int split;                           // g1 = W_i[:, 0:d] . h over the N parents; E half from the Q table
+    int side;                            // split: g1 runs on the side stream beside merge + select
     GemmArgs g1, g2;                     // head GEMMs (depth < L)
     int g1_smem, g2_smem;
 };
@@ -119,6 +120,10 @@ struct dart_handle {
     float *st_dlog, *st_anchor;
     dart_tree_out st_out;
     bool staged;
+    // side stream of the split first head layer (fork after the LM-head,
+    // join before gather_silu)
+    cudaStream_t side;
+    cudaEvent_t ev_fork, ev_join;
     // graphs
     cudaStream_t cap_stream;
     std::vector<GraphEntry> graphs;
@@ -258,7 +263,7 @@ int build_plans(dart_handle* h) {
         }
         p.Pn = h->caps[dep];
         p.Nc = c.nseq * p.Pn;
-        p.split = 0;
+        p.split = p.side = 0;
         if (dep < c.L) {
             // Split first head layer (full vocabulary, <= 16 children, bf16):
             //   W_i . [h_p ; E[t_c]] = W_i[:, 0:d] . h_p + Q[t_c],
@@ -269,6 +274,8 @@ int build_plans(dart_handle* h) {
             // added in the SiLU kernel.  DART_SPLIT_HEAD=0 turns it off.
             const char* sh = getenv("DART_SPLIT_HEAD");
             p.split = (tc && c.cand_k == 0 && p.Nc <= 16 && !(sh && sh[0] == '0')) ? 1 : 0;
+            const char* ss = getenv("DART_SPLIT_SIDE");  // tuning override: 0 = after merge + select, same stream
+            p.side = (p.split && !(ss && ss[0] == '0')) ? 1 : 0;
             p.g1 = p.split ? gemm_plan(h, c.d, p.N, c.d / kBlockK, tc) : gemm_plan(h, 2 * c.d, p.Nc, c.d / kBlockK, tc);
             p.g2 = gemm_plan(h, c.d, p.Nc, c.d / kBlockK, tc);
             if (tc) {
@@ -497,6 +504,11 @@ void release(dart_handle* h) {
     h->ev.clear();
     if (h->cap_stream) cudaStreamDestroy(h->cap_stream);
     h->cap_stream = nullptr;
+    if (h->side) cudaStreamDestroy(h->side);
+    h->side = nullptr;
+    if (h->ev_fork) cudaEventDestroy(h->ev_fork);
+    if (h->ev_join) cudaEventDestroy(h->ev_join);
+    h->ev_fork = h->ev_join = nullptr;
     for (void* p : h->allocs) cudaFree(p);
     h->allocs.clear();
 }
@@ -608,6 +620,23 @@ int enqueue_depth(dart_handle* h, int dep, const float* dlog, const float* ancho
     }
     prof_end(h, pi, st);
     if (e != cudaSuccess) return DART_ERR_CUDA;
+    if (p.side) {
+        // Split first head layer: U = W_i[:, 0:d] . h over the parents needs
+        // only their states (the hi/lo rows the LM-head just read), so it runs
+        // on the side stream while merge + select finds the children; it
+        // writes `part`, whose last reader (residual_norm of the previous
+        // depth) finished before the LM-head did.  Joined before gather_silu.
+        GemmArgs g1 = p.g1;
+        g1.out = h->part;
+        g1.outL = h->AL;
+        g1.status = h->status;
+        if (cudaEventRecord(h->ev_fork, st) != cudaSuccess || cudaStreamWaitEvent(h->side, h->ev_fork, 0) != cudaSuccess)
+            return DART_ERR_CUDA;
+        pi = prof_begin(h, kGemm1, h->side);
+        e = launch_gemm_tc(&h->tmWi, &h->tmH[ng_index(g1.NG)], g1, p.g1_smem, h->side);
+        prof_end(h, pi, h->side);
+        if (e != cudaSuccess || cudaEventRecord(h->ev_join, h->side) != cudaSuccess) return DART_ERR_CUDA;
+    }
     // 2) merge partials, log q~, Eq. 5 scores, global top-W -> S_dep
     SelectArgs sa;
     std::memset(&sa, 0, sizeof sa);
@@ -657,21 +686,23 @@ int enqueue_depth(dart_handle* h, int dep, const float* dlog, const float* ancho
     g1.outL = h->AL;
     g2.out = h->part;
     g1.status = g2.status = h->status;
-    pi = prof_begin(h, kGemm1, st);
-    if (p.split) {
-        // W_i[:, 0:d] . h over the parents: B = their hi/lo rows of the LM-head
-        e = launch_gemm_tc(&h->tmWi, &h->tmH[ng_index(g1.NG)], g1, p.g1_smem, st);
-    } else if (tc) {
-        e = launch_gemm_tc(&h->tmWi, &h->tmX[ng_index(g1.NG)], g1, p.g1_smem, st);
-    } else {
-        g1.A32 = static_cast<const float*>(h->Wi);
-        g1.B32 = h->X32;
-        e = launch_gemm_f32(g1, st);
+    if (!p.side) {  // (on the side stream it was launched after the LM-head)
+        pi = prof_begin(h, kGemm1, st);
+        if (p.split) {
+            e = launch_gemm_tc(&h->tmWi, &h->tmH[ng_index(g1.NG)], g1, p.g1_smem, st);
+        } else if (tc) {
+            e = launch_gemm_tc(&h->tmWi, &h->tmX[ng_index(g1.NG)], g1, p.g1_smem, st);
+        } else {
+            g1.A32 = static_cast<const float*>(h->Wi);
+            g1.B32 = h->X32;
+            e = launch_gemm_f32(g1, st);
+        }
+        prof_end(h, pi, st);
+        if (e != cudaSuccess) return DART_ERR_CUDA;
     }
-    prof_end(h, pi, st);
-    if (e != cudaSuccess) return DART_ERR_CUDA;
     const bool fused = tc && g1.mode != kGemmPartials;  // SiLU applied in the GEMM's cluster reduction
     if (p.split) {
+        if (p.side && cudaStreamWaitEvent(st, h->ev_join, 0) != cudaSuccess) return DART_ERR_CUDA;
         pi = prof_begin(h, kGatherSilu, st);
         e = launch_gather_silu(p.Nc, c.d, g1.S, g1.N, h->part, h->child_prow, h->child_tok, c.V, h->Qtab, h->AL,
                                kNPadMax, st);
@@ -807,6 +838,11 @@ int dart_init_head(dart_handle** out, const dart_config* cfg, int wdtype, const 
     if (rc == DART_OK && wdtype == DART_BF16) rc = make_tensor_maps(h);
     if (rc == DART_OK && h->Qtab) rc = compute_qtab(h, static_cast<cudaStream_t>(stream));
     if (rc == DART_OK && cudaStreamCreateWithFlags(&h->cap_stream, cudaStreamNonBlocking) != cudaSuccess)
+        rc = DART_ERR_CUDA;
+    if (rc == DART_OK && h->Qtab &&
+        (cudaStreamCreateWithFlags(&h->side, cudaStreamNonBlocking) != cudaSuccess ||
+         cudaEventCreateWithFlags(&h->ev_fork, cudaEventDisableTiming) != cudaSuccess ||
+         cudaEventCreateWithFlags(&h->ev_join, cudaEventDisableTiming) != cudaSuccess))
         rc = DART_ERR_CUDA;
     if (rc == DART_OK && cudaDeviceSynchronize() != cudaSuccess) rc = DART_ERR_CUDA;
     if (rc != DART_OK) {
