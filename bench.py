@@ -106,15 +106,26 @@ def kernel_source_sha():
     return code_sha(("dart_tc.cu", "dart_device.cuh"))
 
 
+def split_head(cfg):
+    """True when the library splits the first head layer (bf16 weights):
+    each depth streams W_i[:, 0:d] (2 d^2 bytes) instead of all of W_i."""
+    return cfg.wdtype == "bf16" and os.environ.get("DART_SPLIT_HEAD", "1")[:1] != "0"
+
+
+def wi_bytes_per_depth(cfg):
+    return (1 if split_head(cfg) else 2) * cfg.d * cfg.d * cfg.bpe
+
+
 def kept_head_weights(cfg):
     """(W_i kept, W_o kept): the head weights the library loads evict-last
     so that they stay in L2 across the depths of a round.  Mirrors its plan:
-    candidate-restricted scoring, <= 16 children, the largest of {both, W_i,
-    W_o} within 72 MiB (bf16 weights)."""
+    candidate-restricted scoring, <= 16 children, the largest of {both, W_i
+    (its first half with the split first layer), W_o} within 72 MiB (bf16
+    weights)."""
     if cfg.cand_k == 0 or cfg.wdtype != "bf16" or cfg.nseq * cfg.W > 16:
         return False, False
     cap = 72 << 20
-    wi, wo = 4 * cfg.d * cfg.d, 2 * cfg.d * cfg.d
+    wi, wo = wi_bytes_per_depth(cfg), 2 * cfg.d * cfg.d
     if wi + wo <= cap:
         return True, True
     return wi <= cap, wi > cap and wo <= cap
@@ -620,20 +631,21 @@ def main():
     kinds = dart.dart_profile_read_kinds(h)
     dart.dart_set_profiling(h, False)
     # roofline kernel: the LM-head stream, or with candidate-restricted
-    # scoring the head GEMM whose weights stream from HBM at every depth (W_i,
-    # 4 d^2 bytes, else W_o, 2 d^2); when both stay in L2 the W_i GEMM with
-    # its weights counted once per round (the HBM reads it needs)
+    # scoring the head GEMM whose weights stream from HBM at every depth (W_i
+    # or, with the split first layer, its first half W_i[:, 0:d], else W_o);
+    # when both stay in L2 the W_i GEMM with its weights counted once per
+    # round (the HBM reads it needs)
     wi_kept, wo_kept = kept_head_weights(cfg)
     if cfg.cand_k == 0:
         rl_kind, rl_name, bytes_launch, rl_note = "lmhead", "lmhead_tc_kernel", cfg.lmhead_bytes_per_depth(), None
     elif not wi_kept:
-        rl_kind, rl_name, bytes_launch, rl_note = "gemm_wi", "gemm_tc_kernel (W_i)", 2 * cfg.d * cfg.d * cfg.bpe, None
+        rl_kind, rl_name, bytes_launch, rl_note = "gemm_wi", "gemm_tc_kernel (W_i)", wi_bytes_per_depth(cfg), None
     elif not wo_kept:
         rl_kind, rl_name, bytes_launch, rl_note = ("gemm_wo", "gemm_tc_kernel (W_o)", cfg.d * cfg.d * cfg.bpe,
                                                    "W_i stays in L2 across depths; W_o streams from HBM")
     else:
         rl_kind, rl_name = "gemm_wi", "gemm_tc_kernel (W_i)"
-        bytes_launch = 2 * cfg.d * cfg.d * cfg.bpe / max(1, cfg.L - 1)
+        bytes_launch = wi_bytes_per_depth(cfg) / max(1, cfg.L - 1)
         rl_note = "W_i and W_o stay in L2 across depths: W_i bytes counted once per round"
     k1_ms, k1_n = kinds[rl_kind]
     k1_avg_s = k1_ms / 1e3 / max(1, k1_n)
@@ -685,8 +697,8 @@ def main():
                        "l2": ("inputs larger than L2: E (%.2f GB) streamed once per depth" %
                               (cfg.V * cfg.d * cfg.bpe / 1e9)) if cfg.cand_k == 0 else
                              ("L2 flushed before every timed round (untimed 512 MB write, then a 512 MB read "
-                              "that takes the write-back); the round's head weights (%.0f MB) would fit in L2" %
-                              (3 * cfg.d * cfg.d * cfg.bpe / 1e6))},
+                              "that takes the write-back); the head weights a depth reads (%.0f MB) would fit in L2" %
+                              ((wi_bytes_per_depth(cfg) + cfg.d * cfg.d * cfg.bpe) / 1e6))},
             "us_per_round": ms * 1e3,
             "lmhead_gbs": lm_bytes_round / (ms / 1e3) / 1e9 if lm_bytes_round else None,
             "lmhead_frac_of_8tbs": lm_bytes_round / (ms / 1e3) / 1e9 / NOMINAL_HBM_GBS if lm_bytes_round else None,

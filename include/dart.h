@@ -113,12 +113,11 @@ typedef struct {
  *   (DART_BF16: bfloat16 with fp32 accumulation; DART_F32: float32 with
  *   fp32 arithmetic throughout).  Pointers must be 16-byte aligned.
  * Allocates the workspace for the worst case of cfg (synchronous
- * allocation).  With DART_BF16 weights, cand_k = 0 and at most 16 children
- * per depth (nseq * W <= 16), it also computes on `stream` the per-token
- * table Q[t] = W_i[:, d:2d] . E[t] (fp32, V * d floats: 2.5 GB at V = 151936,
- * d = 4096), so that each state update adds one row of Q per child instead
- * of streaming the second half of W_i again; the call returns after it is
- * done.  Requires a compute capability 10.3 device (GB300).
+ * allocation).  With DART_BF16 weights it also computes on `stream` the
+ * per-token table Q[t] = W_i[:, d:2d] . E[t] (fp32, V * d floats: 2.5 GB at
+ * V = 151936, d = 4096), so that each state update adds one row of Q per
+ * child instead of streaming the second half of W_i again; the call returns
+ * after it is done.  Requires a compute capability 10.3 device (GB300).
  * On success *out receives the handle; on failure *out is NULL. */
 int dart_init_head(dart_handle **out, const dart_config *cfg, int wdtype,
                    const void *W_i, const void *W_o, const void *E, void *stream);

@@ -265,15 +265,15 @@ int build_plans(dart_handle* h) {
         p.Nc = c.nseq * p.Pn;
         p.split = p.side = 0;
         if (dep < c.L) {
-            // Split first head layer (full vocabulary, <= 16 children, bf16):
+            // Split first head layer (bf16 weights):
             //   W_i . [h_p ; E[t_c]] = W_i[:, 0:d] . h_p + Q[t_c],
             // Q = the per-token table computed once per handle.  The GEMM then
-            // runs over the parents' states, which the LM-head already holds
-            // as hi/lo rows (no gather of the inputs), streams half of W_i
-            // (its first tiles while merge + select runs), and Q[t_c] is
-            // added in the SiLU kernel.  DART_SPLIT_HEAD=0 turns it off.
+            // runs over the parents' states, which are already held as hi/lo
+            // rows (no gather of the inputs), with half of W_i, beside the
+            // selection of the children, and Q[t_c] is added in the SiLU
+            // kernel.  DART_SPLIT_HEAD=0 turns it off.
             const char* sh = getenv("DART_SPLIT_HEAD");
-            p.split = (tc && c.cand_k == 0 && p.Nc <= 16 && !(sh && sh[0] == '0')) ? 1 : 0;
+            p.split = (tc && !(sh && sh[0] == '0')) ? 1 : 0;
             const char* ss = getenv("DART_SPLIT_SIDE");  // tuning override: 0 = after merge + select, same stream
             p.side = (p.split && !(ss && ss[0] == '0')) ? 1 : 0;
             p.g1 = p.split ? gemm_plan(h, c.d, p.N, c.d / kBlockK, tc) : gemm_plan(h, 2 * c.d, p.Nc, c.d / kBlockK, tc);
@@ -281,11 +281,14 @@ int build_plans(dart_handle* h) {
             if (tc) {
                 // two CTAs per SM when both fit with >= 4 stages: twice the
                 // independent weight streams, k split twice as finely
-                const int sb = tc_stage_bytes(p.g1.NG);
+                // (the split layer's GEMM runs over the parents, fewer nodes
+                // than the W_o GEMM's children: size both for the larger group)
+                const int ngmax = std::max(p.g1.NG, p.g2.NG);
+                const int sb = tc_stage_bytes(ngmax);
                 const int st2 = std::min(tc_stages(h->smem_optin / 2 - 2048, sb, gemm_tc_fixed_smem(16)), 8);
                 const int smem2 = gemm_tc_fixed_smem(st2) + st2 * sb;
                 int cps = 1;
-                if (st2 >= 4 && gemm_tc_ctas_per_sm(p.g1.NG, smem2) >= 2) {
+                if (st2 >= 4 && gemm_tc_ctas_per_sm(ngmax, smem2) >= 2) {
                     cps = 2;
                     p.g1.stages = st2;
                 } else {
@@ -301,12 +304,16 @@ int build_plans(dart_handle* h) {
                 // CTAs become resident and fetch their first weight tiles).
                 // Larger node sets: the k splits of a tile are one cluster
                 // (the largest <= 8 whose clusters all fit on the GPU at
-                // once) and are summed on chip, with SiLU applied there.
+                // once) and are summed on chip, with SiLU applied there (the
+                // split layer's GEMM writes the plain sum; SiLU follows the
+                // addition of Q[t_c]).
                 const bool cluster = p.Nc > 16;
+                const bool cluster1 = p.split ? p.N > 16 : cluster;
                 for (GemmArgs* g : {&p.g1, &p.g2}) {
                     const int tiles_mg = g->MT * g->G;
                     const int cap = cps * h->num_sms;
-                    if (cluster) {
+                    const bool cl = g == &p.g1 ? cluster1 : cluster;
+                    if (cl) {
                         int sc = std::max(1, std::min({kMaxClusterK, g->KB, cap / tiles_mg}));
                         for (; sc > 1; sc--)
                             if (gemm_tc_max_clusters(g->NG, p.g1_smem, sc) >= tiles_mg) break;
@@ -316,20 +323,21 @@ int build_plans(dart_handle* h) {
                     }
                     if (getenv("DART_DEBUG_PLAN"))
                         fprintf(stderr, "dart: depth %d gemm K=%d tiles %d x k-splits %d%s, %d CTAs/SM\n", dep, g->K,
-                                tiles_mg, g->S, cluster ? " (cluster)" : "", cps);
+                                tiles_mg, g->S, cl ? " (cluster)" : "", cps);
                 }
-                p.g1.mode = cluster ? kGemmSiluSplit : kGemmPartials;
+                p.g1.mode = cluster1 ? (p.split ? kGemmSum : kGemmSiluSplit) : kGemmPartials;
                 p.g2.mode = cluster ? kGemmSum : kGemmPartials;
                 // Candidate-restricted scoring streams nothing through L2
                 // between the depths: with <= 16 children (weight-bound
-                // GEMMs) the largest of {W_i and W_o, W_i (4 d^2 bytes), W_o
-                // (2 d^2)} within kL2KeepBytes is loaded evict-last and read
-                // from HBM once per round instead of once per depth.
+                // GEMMs) the largest of {W_i and W_o, W_i (4 d^2 bytes, 2 d^2
+                // for the split layer), W_o (2 d^2)} within kL2KeepBytes is
+                // loaded evict-last and read from HBM once per round instead
+                // of once per depth.
                 // Measured on GB300 (A/B, K = 64): d = 2560, both (39 MB):
                 // -4.9 % per round; d = 4096: W_i (67 MB) -6.0 %, W_o
                 // (34 MB) -2.0 %, both (101 MB) +2.1 %; W_o with 256 children
                 // (cluster GEMMs) +0.8 %.
-                const long long wo_bytes = 2ll * c.d * c.d, wi_bytes = 4ll * c.d * c.d;
+                const long long wo_bytes = 2ll * c.d * c.d, wi_bytes = (p.split ? 2ll : 4ll) * c.d * c.d;
                 p.g1.keep_a = p.g2.keep_a = 0;
                 if (c.cand_k > 0 && !cluster) {
                     if (wi_bytes + wo_bytes <= kL2KeepBytes)
@@ -704,8 +712,9 @@ int enqueue_depth(dart_handle* h, int dep, const float* dlog, const float* ancho
     if (p.split) {
         if (p.side && cudaStreamWaitEvent(st, h->ev_join, 0) != cudaSuccess) return DART_ERR_CUDA;
         pi = prof_begin(h, kGatherSilu, st);
-        e = launch_gather_silu(p.Nc, c.d, g1.S, g1.N, h->part, h->child_prow, h->child_tok, c.V, h->Qtab, h->AL,
-                               kNPadMax, st);
+        // (a cluster GEMM wrote the summed U: one "split")
+        e = launch_gather_silu(p.Nc, c.d, g1.mode == kGemmPartials ? g1.S : 1, g1.N, h->part, h->child_prow,
+                               h->child_tok, c.V, h->Qtab, h->AL, kNPadMax, st);
         prof_end(h, pi, st);
         if (e != cudaSuccess) return DART_ERR_CUDA;
     } else if (!fused) {
@@ -725,7 +734,8 @@ int enqueue_depth(dart_handle* h, int dep, const float* dlog, const float* ancho
     prof_end(h, pi, st);
     if (e != cudaSuccess) return DART_ERR_CUDA;
     pi = prof_begin(h, kNorm, st);
-    e = launch_residual_norm(p.Nc, c.d, fused ? 1 : g2.S, h->part, h->child_prow, hcur, c.rms_eps, hnext, tc ? h->HL : nullptr,
+    const int s2 = tc && g2.mode != kGemmPartials ? 1 : g2.S;  // the W_o cluster GEMM wrote the sum
+    e = launch_residual_norm(p.Nc, c.d, s2, h->part, h->child_prow, hcur, c.rms_eps, hnext, tc ? h->HL : nullptr,
                              kNPadMax, st);
     prof_end(h, pi, st);
     if (e != cudaSuccess) return DART_ERR_CUDA;
