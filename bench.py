@@ -700,8 +700,11 @@ def main():
                               "that takes the write-back); the head weights a depth reads (%.0f MB) would fit in L2" %
                               ((wi_bytes_per_depth(cfg) + cfg.d * cfg.d * cfg.bpe) / 1e6))},
             "us_per_round": ms * 1e3,
+            # the round's LM-head bytes over the whole round's time (head updates,
+            # selection and pruning included), and the LM-head kernel alone
             "lmhead_gbs": lm_bytes_round / (ms / 1e3) / 1e9 if lm_bytes_round else None,
             "lmhead_frac_of_8tbs": lm_bytes_round / (ms / 1e3) / 1e9 / NOMINAL_HBM_GBS if lm_bytes_round else None,
+            "lmhead_kernel_frac_of_8tbs": achieved / NOMINAL_HBM_GBS if lm_bytes_round else None,
             "roofline": {"kernel": rl_name, "note": rl_note,
                          "bound": "hbm", "achieved": achieved, "peak": peak,
                          "peak_kind": peak_kind, "unit": "GB/s", "frac": achieved / peak,
