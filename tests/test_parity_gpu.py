@@ -156,6 +156,34 @@ def test_build_tree_graph_matches_depthwise(dart, cfg):
         eng.close()
 
 
+VARIANT_CFGS = [SMALL[2], SMALL[5], SMALL[6], RESTRICTED[1]]
+
+
+@pytest.mark.parametrize("env", [{"DART_SPLIT_HEAD": "0"}, {"DART_SPLIT_SIDE": "0"}], ids=["unsplit", "same-stream"])
+@pytest.mark.parametrize("cfg", VARIANT_CFGS, ids=[c.name for c in VARIANT_CFGS])
+def test_head_update_variants(dart, cfg, env, monkeypatch):
+    """The head-update variants the library keeps behind its tuning switches
+    (read when a handle is created): the unsplit first layer (gather of
+    [h_p ; E[t_c]] and the full W_i GEMM) and the split layer's GEMM on the
+    main stream.  Each matches the oracle, and the graph launch equals the
+    depth-by-depth calls."""
+    for k, v in env.items():
+        monkeypatch.setenv(k, v)
+    x = make_inputs(cfg)
+    dx = to_device(cfg, x)
+    ref = oracle.build_tree(cfg, x["Wi"], x["Wo"], x["E"], x["Dlog"], x["h0"])
+    _, gst, g_ref = run_depthwise(dart, cfg, dx)
+    compare_with_oracle(cfg, ref, gst, g_ref, tol_of(cfg))
+    eng = dart.Dart(cfg, dx["Wi"], dx["Wo"], dx["E"])
+    try:
+        g = tree_to_numpy(eng.build_tree(dx["Dlog"], dx["h0"]))
+        assert dart.dart_status_sync(eng.h) == 0
+    finally:
+        eng.close()
+    for k in g_ref:
+        np.testing.assert_array_equal(g[k], g_ref[k], err_msg=k)
+
+
 def test_neg_inf_drafter_logits(dart):
     cfg = C("neginf", 2, 700, 128, 4, 6, 4, 40, "bf16", 0.0, 31)
     x = make_inputs(cfg)
