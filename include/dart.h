@@ -117,7 +117,8 @@ typedef struct {
  * per-token table Q[t] = W_i[:, d:2d] . E[t] (fp32, V * d floats: 2.5 GB at
  * V = 151936, d = 4096), so that each state update adds one row of Q per
  * child instead of streaming the second half of W_i again; the call returns
- * after it is done.  Requires a compute capability 10.3 device (GB300).
+ * after it is done (DART_ERR_TIMEOUT if a device-side wait of that GEMM gave
+ * up).  Requires a compute capability 10.3 device (GB300).
  * On success *out receives the handle; on failure *out is NULL. */
 int dart_init_head(dart_handle **out, const dart_config *cfg, int wdtype,
                    const void *W_i, const void *W_o, const void *E, void *stream);

@@ -855,6 +855,14 @@ int dart_init_head(dart_handle** out, const dart_config* cfg, int wdtype, const 
          cudaEventCreateWithFlags(&h->ev_join, cudaEventDisableTiming) != cudaSuccess))
         rc = DART_ERR_CUDA;
     if (rc == DART_OK && cudaDeviceSynchronize() != cudaSuccess) rc = DART_ERR_CUDA;
+    if (rc == DART_OK && h->Qtab) {
+        // the table's GEMM waits with a time limit: one that gave up left Q incomplete
+        int word = 0;
+        if (cudaMemcpy(&word, h->status, sizeof word, cudaMemcpyDeviceToHost) != cudaSuccess)
+            rc = DART_ERR_CUDA;
+        else if (word & kDevTimeout)
+            rc = DART_ERR_TIMEOUT;
+    }
     if (rc != DART_OK) {
         release(h);
         delete h;
