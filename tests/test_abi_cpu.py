@@ -49,7 +49,9 @@ class Cfg:
 BAD = [dict(V=0), dict(d=100), dict(d=32), dict(L=0), dict(W=0), dict(W=65), dict(k=0), dict(k=65),
        dict(V=10, k=11), dict(W=64, k=65), dict(L=17, W=64), dict(B=0), dict(B=1025), dict(nseq=0),
        dict(nseq=5, W=64), dict(beta=0.1), dict(beta=float("nan")), dict(temperature=-1.0),
-       dict(rms_eps=0.0), dict(cand_k=3), dict(cand_k=-1), dict(cand_k=1001), dict(V=5000, cand_k=1025)]
+       dict(rms_eps=0.0), dict(cand_k=3), dict(cand_k=-1), dict(cand_k=1001), dict(V=5000, cand_k=1025),
+       dict(d=16448), dict(V=1 << 24), dict(L=1025, W=1), dict(temperature=float("inf")),
+       dict(rms_eps=float("nan"))]
 
 
 @pytest.mark.parametrize("bad", BAD, ids=[str(b) for b in BAD])
