@@ -1,0 +1,136 @@
+"""Planted mistakes in the oracle must fail at least one of its pins (CPU).
+
+Each case copies ``oracle/dart_oracle.c``, changes one spot the way a
+plausible slip would (a swapped concatenation, a dropped term, a wrong index
+or drafter row, a reversed tie-break, ...), compiles the copy and points the
+oracle's ctypes wrapper at it for the duration of the test, then runs every
+pin of ``test_oracle_pins.py``.  A planted mistake that passes every pin
+would mean the pins cannot tell that part of the oracle from a wrong one.
+The oracle source itself carries no switches for this.
+"""
+import inspect
+import itertools
+import os
+import shutil
+import subprocess
+
+import pytest
+
+import oracle
+import test_oracle_pins as pins
+
+# (name, exact text of the oracle, planted replacement)
+MUTANTS = [
+    ("head: [E[t]; h_p] instead of [h_p; E[t]]",
+     "        x[j] = hp[j];\n        x[d + j] = wval(E, dt, (size_t)tok * d + j);",
+     "        x[d + j] = hp[j];\n        x[j] = wval(E, dt, (size_t)tok * d + j);"),
+    ("head: residual h_p dropped",
+     "r[i] = hp[i] + wdot(Wo, dt, (size_t)i * d, a, d);",
+     "r[i] = wdot(Wo, dt, (size_t)i * d, a, d);"),
+    ("head: RMSNorm epsilon dropped",
+     "sqrt(ss / d + c->rms_eps)",
+     "sqrt(ss / d)"),
+    ("head: ReLU instead of SiLU",
+     "a[i] = u / (1.0 + exp(-u));",
+     "a[i] = u > 0.0 ? u : 0.0;"),
+    ("scoring: temperature not applied",
+     "z[v] = ((double)dlog_row[v] + wdot(E, dt, (size_t)v * d, h, d)) / Tp;",
+     "z[v] = ((double)dlog_row[v] + wdot(E, dt, (size_t)v * d, h, d));"),
+    ("scoring: drafter row of position d instead of d-1",
+     "const float *row = Dlog + ((size_t)s * L + dep - 1) * V;",
+     "const float *row = Dlog + ((size_t)s * L + (dep < L ? dep : dep - 1)) * V;"),
+    ("Eq. 5: depth bonus beta dropped",
+     "cand[ncand].score = pscore[p] + logq[idx[j]] + c->beta; /* Eq. 5 */",
+     "cand[ncand].score = pscore[p] + logq[idx[j]]; /* Eq. 5 */"),
+    ("Eq. 5: parent's path score not accumulated",
+     "cand[ncand].score = pscore[p] + logq[idx[j]] + c->beta; /* Eq. 5 */",
+     "cand[ncand].score = logq[idx[j]] + c->beta; /* Eq. 5 */"),
+    ("state update: child state from the first parent",
+     "orc_head(c, Wi, Wo, E, hs + (size_t)cand[r].p * d, cand[r].tok,",
+     "orc_head(c, Wi, Wo, E, hs, cand[r].tok,"),
+    ("top-k: ties by token desc",
+     "return a > b || (a == b && ia < ib);",
+     "return a > b || (a == b && ia > ib);"),
+    ("frontier: ties by parent slot desc",
+     "if (a->p != b->p) return a->p < b->p ? -1 : 1;",
+     "if (a->p != b->p) return a->p > b->p ? -1 : 1;"),
+    ("pruning: ties by node id desc",
+     "return a->id < b->id ? -1 : (a->id > b->id);",
+     "return a->id > b->id ? -1 : (a->id < b->id);"),
+    ("emission: position id = pos_offset + depth - 1",
+     "o_pos[o] = c->pos_offset + dep;",
+     "o_pos[o] = c->pos_offset + dep - 1;"),
+    ("emission: mask row holds the parent only",
+     "            a = o_par[(size_t)s * B + a];",
+     "            a = -1;"),
+    ("heap: ties popped by node id desc",
+     "((a).score == (b).score && (a).id < (b).id))",
+     "((a).score == (b).score && (a).id > (b).id))"),
+    ("candidate set: the K smallest drafter logits",
+     "for (int v = 0; v < c->V; v++) x[v] = (double)dlog_row[v];",
+     "for (int v = 0; v < c->V; v++) x[v] = -(double)dlog_row[v];"),
+]
+
+
+def pin_cases():
+    """(id, function, kwargs) for every pin, parametrisations expanded."""
+    out = []
+    for name, fn in inspect.getmembers(pins, inspect.isfunction):
+        if not name.startswith("test_") or fn.__module__ != pins.__name__:
+            continue
+        marks = [m for m in getattr(fn, "pytestmark", []) if m.name == "parametrize"]
+        grids = []
+        for m in marks:
+            names = [a.strip() for a in m.args[0].split(",")] if isinstance(m.args[0], str) else list(m.args[0])
+            vals = [v if len(names) > 1 else (v,) for v in m.args[1]]
+            grids.append([dict(zip(names, v)) for v in vals])
+        params = set(inspect.signature(fn).parameters)
+        for combo in itertools.product(*grids) if grids else [()]:
+            kw = {}
+            for part in combo:
+                kw.update(part)
+            if set(kw) != params:
+                continue  # needs a fixture: not a pure pin
+            out.append((f"{name}{sorted(kw.items()) if kw else ''}", fn, kw))
+    return out
+
+
+def build_mutant(tmp_path, old, new):
+    src = open(oracle._SRC).read()
+    assert src.count(old) == 1, "the planted spot must occur exactly once in the oracle"
+    msrc = tmp_path / "dart_oracle_mut.c"
+    msrc.write_text(src.replace(old, new))
+    mlib = tmp_path / "libdart_oracle_mut.so"
+    cmd = ["gcc", "-O2", "-std=c11", "-shared", "-fPIC", str(msrc), "-o", str(mlib), "-lm"]
+    r = subprocess.run(cmd[:1] + ["-fopenmp"] + cmd[1:], capture_output=True)
+    if r.returncode != 0:
+        subprocess.run(cmd, check=True, capture_output=True)
+    return msrc, mlib
+
+
+def failing_pins():
+    failed = []
+    for cid, fn, kw in pin_cases():
+        try:
+            fn(**kw)
+        except Exception as e:  # an assertion, or a crash on nonsense output
+            failed.append(f"{cid}: {type(e).__name__}")
+    return failed
+
+
+@pytest.mark.skipif(shutil.which("gcc") is None, reason="gcc not available")
+def test_unmodified_oracle_passes_every_pin():
+    assert len(pin_cases()) >= 25
+    assert failing_pins() == []
+
+
+@pytest.mark.skipif(shutil.which("gcc") is None, reason="gcc not available")
+@pytest.mark.parametrize("name,old,new", MUTANTS, ids=[m[0] for m in MUTANTS])
+def test_planted_mistake_fails_a_pin(tmp_path, monkeypatch, name, old, new):
+    msrc, mlib = build_mutant(tmp_path, old, new)
+    monkeypatch.setattr(oracle, "_SRC", str(msrc))
+    monkeypatch.setattr(oracle, "_LIB", str(mlib))
+    monkeypatch.setattr(oracle, "_lib", None)
+    failed = failing_pins()
+    print(name, "->", failed)
+    assert failed, f"planted mistake passed every pin: {name}"

@@ -303,6 +303,37 @@ def test_prune_emit_hand_example():
     assert abs(r["prune_gap"][0] - (-0.7 + 0.9)) < 1e-15
 
 
+def test_frontier_ties_across_parents_by_parent_slot():
+    """Exact score ties at the W-th cut, across parents (the reading of the
+    frontier order: score desc, parent slot asc, rank in the parent's list
+    asc).  With E = 0 the head has no effect and log q~ is the log-softmax of
+    the drafter row.  Depth 1: row [2, 2, -5, -5] makes tokens 0 and 1 equal,
+    so slots 0 and 1 carry the same path score, and the cut at W = 3 falls
+    inside the tie {2, 3} (rank asc keeps token 2).  Depth 2: row [3, 0, 0, 0]
+    gives both of those parents the same children's scores; the two best are
+    (slot 0, token 0) and (slot 1, token 0), and the third comes from the tie
+    group {tokens 1, 2, 3} x {slots 0, 1}: slot 0, token 1."""
+    cfg = tiny(V=4, d=8, L=2, W=3, k=4, B=6, beta=-0.2)
+    x = rand_inputs(cfg)
+    x["E"][:] = 0.0
+    x["Dlog"][0, 0] = [2.0, 2.0, -5.0, -5.0]
+    x["Dlog"][0, 1] = [3.0, 0.0, 0.0, 0.0]
+    r = run(cfg, x)
+    np.testing.assert_array_equal(r["st_count"][0], [3, 3])
+    np.testing.assert_array_equal(r["st_tok"][0, 0], [0, 1, 2])
+    np.testing.assert_array_equal(r["st_tok"][0, 1], [0, 0, 1])
+    np.testing.assert_array_equal(r["st_parent"][0, 1], [0, 1, 0])
+    # the ties are exact, and the scores are the closed form of Eq. 5
+    l1 = torch.log_softmax(torch.tensor([2.0, 2.0, -5.0, -5.0], dtype=torch.float64), 0).numpy()
+    l2 = torch.log_softmax(torch.tensor([3.0, 0.0, 0.0, 0.0], dtype=torch.float64), 0).numpy()
+    assert r["st_score"][0, 0, 0] == r["st_score"][0, 0, 1]
+    assert r["st_score"][0, 1, 0] == r["st_score"][0, 1, 1]
+    np.testing.assert_allclose(r["st_score"][0, 0], l1[[0, 1, 2]] - 0.2, atol=1e-12)
+    np.testing.assert_allclose(r["st_score"][0, 1], [l1[0] + l2[0] - 0.4, l1[1] + l2[0] - 0.4, l1[0] + l2[1] - 0.4],
+                               atol=1e-12)
+    _check_tree_structure(cfg, r)
+
+
 def test_neg_inf_children_are_never_retained():
     cfg = tiny(V=8, d=8, L=3, W=6, k=4, B=30)
     x = rand_inputs(cfg)
