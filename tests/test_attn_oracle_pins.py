@@ -35,6 +35,24 @@ def rope_complex(x, pos, theta):
     return np.concatenate([r.real, r.imag], axis=-1)
 
 
+def branch(parents, i):
+    """Root-to-node path of node i written independently of the oracle: the
+    ancestor set of i (i included) ordered by distance from the root."""
+    anc = {int(i)}
+    frontier = int(i)
+    while int(parents[frontier]) >= 0:
+        frontier = int(parents[frontier])
+        anc.add(frontier)
+
+    def dist(j):
+        n = 0
+        while int(parents[j]) >= 0:
+            j = int(parents[j])
+            n += 1
+        return n
+    return sorted(anc, key=dist)
+
+
 def make_case(seed, nseq=2, B=12, C=5, Hq=4, Hkv=2, dh=8, L=4, W=4, fill=None, theta=1.0e4):
     g = np.random.Generator(np.random.PCG64(seed))
     q = g.standard_normal((nseq, B, Hq, dh))
@@ -94,7 +112,7 @@ def test_branch_is_a_causal_sequence(seed, kw):
     case = make_case(seed, **kw)
     off = case["C"] + 7
     got = run_oracle(case, off)
-    ref = causal_reference(case, off, ta.root_path)
+    ref = causal_reference(case, off, branch)
     np.testing.assert_allclose(got, ref, rtol=0, atol=1e-12)
     for s in range(case["q"].shape[0]):
         assert np.all(got[s, int(case["n_nodes"][s]):] == 0.0)
@@ -104,7 +122,7 @@ def test_chain_tree_is_plain_causal_attention():
     case = make_case(5, B=6, L=6, W=1)
     assert list(case["parents"][0]) == [-1, 0, 1, 2, 3, 4]
     got = run_oracle(case, case["C"])
-    ref = causal_reference(case, case["C"], ta.root_path)
+    ref = causal_reference(case, case["C"], branch)
     np.testing.assert_allclose(got, ref, rtol=0, atol=1e-12)
 
 
@@ -161,14 +179,12 @@ def test_relabelling_permutes_outputs():
 def test_planted_sibling_leak_fails_the_causal_pin(monkeypatch):
     case = make_case(8, nseq=1, B=12, C=2, L=3, W=6)
 
-    honest = ta.root_path
-
     def with_sibling(parents, i):
-        path = honest(parents, i)
+        path = branch(parents, i)
         sib = [j for j in range(len(parents)) if parents[j] == parents[i] and j != i and parents[j] != -2]
         return path[:-1] + sib[:1] + path[-1:] if sib else path
 
     monkeypatch.setattr(ta, "root_path", with_sibling)
     got = run_oracle(case, 2)
-    ref = causal_reference(case, 2, honest)
+    ref = causal_reference(case, 2, branch)
     assert np.max(np.abs(got - ref)) > 1e-3

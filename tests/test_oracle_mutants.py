@@ -1,13 +1,16 @@
-"""Planted mistakes in the oracle must fail at least one of its pins (CPU).
+"""Planted mistakes in the oracles must fail at least one of their pins (CPU).
 
-Each case copies ``oracle/dart_oracle.c``, changes one spot the way a
-plausible slip would (a swapped concatenation, a dropped term, a wrong index
-or drafter row, a reversed tie-break, ...), compiles the copy and points the
-oracle's ctypes wrapper at it for the duration of the test, then runs every
-pin of ``test_oracle_pins.py``.  A planted mistake that passes every pin
-would mean the pins cannot tell that part of the oracle from a wrong one.
-The oracle source itself carries no switches for this.
+Construction oracle: each case copies ``oracle/dart_oracle.c``, changes one
+spot the way a plausible slip would (a swapped concatenation, a dropped term,
+a wrong index or drafter row, a reversed tie-break, ...), compiles the copy
+and points the oracle's ctypes wrapper at it for the duration of the test,
+then runs every pin of ``test_oracle_pins.py``.  Tree-attention oracle: the
+same with a changed copy of ``oracle/tree_attn.py`` loaded as a module and
+the pins of ``test_attn_oracle_pins.py``.  A planted mistake that passes
+every pin would mean the pins cannot tell that part of an oracle from a
+wrong one.  The oracle sources themselves carry no switches for this.
 """
+import importlib.util
 import inspect
 import itertools
 import os
@@ -17,7 +20,9 @@ import subprocess
 import pytest
 
 import oracle
+import test_attn_oracle_pins as attn_pins
 import test_oracle_pins as pins
+from oracle import tree_attn
 
 # (name, exact text of the oracle, planted replacement)
 MUTANTS = [
@@ -72,11 +77,47 @@ MUTANTS = [
 ]
 
 
-def pin_cases():
+# the tree-attention oracle (numpy): (name, exact text, planted replacement)
+ATTN_MUTANTS = [
+    ("RoPE: rotation by -angle",
+     "return np.concatenate([x1 * c - x2 * s, x2 * c + x1 * s], axis=-1)",
+     "return np.concatenate([x1 * c + x2 * s, x2 * c - x1 * s], axis=-1)"),
+    ("RoPE: frequencies theta^(-t/dh)",
+     "inv_freq = float(theta) ** (-2.0 * np.arange(half, dtype=np.float64) / dh)",
+     "inv_freq = float(theta) ** (-1.0 * np.arange(half, dtype=np.float64) / dh)"),
+    ("GQA: query head h reads kv head h % Hkv",
+     "g = h // G",
+     "g = h % Hkv"),
+    ("positions: pos_offset + depth - 1",
+     "pos = pos_offset + np.asarray(depths[s], dtype=np.int64)",
+     "pos = pos_offset + np.asarray(depths[s], dtype=np.int64) - 1"),
+    ("logits: scale dropped",
+     "logits = scale * (keys @ qi)",
+     "logits = keys @ qi"),
+    ("path: the node itself left out",
+     "    j = int(i)\n    while j >= 0:",
+     "    j = int(parents[i])\n    while j >= 0:"),
+    ("context: keys and values left out",
+     "keys = np.concatenate([k_ctx[s, :, g], kt], axis=0)\n"
+     "                vals = np.concatenate([v_ctx[s, :, g], v_tree[s, path, g]], axis=0)",
+     "keys = kt\n                vals = v_tree[s, path, g]"),
+    ("context: values of kv head 0",
+     "vals = np.concatenate([v_ctx[s, :, g], v_tree[s, path, g]], axis=0)",
+     "vals = np.concatenate([v_ctx[s, :, 0], v_tree[s, path, g]], axis=0)"),
+    ("query not rotated",
+     "qi = rope(q[s, i, h], pos[i], rope_theta)",
+     "qi = q[s, i, h]"),
+    ("tree keys rotated at the query's position",
+     "kt = rope(k_tree[s, path, g], pos[path], rope_theta)",
+     "kt = rope(k_tree[s, path, g], pos[i], rope_theta)"),
+]
+
+
+def pin_cases(module=pins):
     """(id, function, kwargs) for every pin, parametrisations expanded."""
     out = []
-    for name, fn in inspect.getmembers(pins, inspect.isfunction):
-        if not name.startswith("test_") or fn.__module__ != pins.__name__:
+    for name, fn in inspect.getmembers(module, inspect.isfunction):
+        if not name.startswith("test_") or fn.__module__ != module.__name__:
             continue
         marks = [m for m in getattr(fn, "pytestmark", []) if m.name == "parametrize"]
         grids = []
@@ -108,9 +149,9 @@ def build_mutant(tmp_path, old, new):
     return msrc, mlib
 
 
-def failing_pins():
+def failing_pins(module=pins):
     failed = []
-    for cid, fn, kw in pin_cases():
+    for cid, fn, kw in pin_cases(module):
         try:
             fn(**kw)
         except Exception as e:  # an assertion, or a crash on nonsense output
@@ -132,5 +173,25 @@ def test_planted_mistake_fails_a_pin(tmp_path, monkeypatch, name, old, new):
     monkeypatch.setattr(oracle, "_LIB", str(mlib))
     monkeypatch.setattr(oracle, "_lib", None)
     failed = failing_pins()
+    print(name, "->", failed)
+    assert failed, f"planted mistake passed every pin: {name}"
+
+
+def test_unmodified_attention_oracle_passes_every_pin():
+    assert len(pin_cases(attn_pins)) >= 8
+    assert failing_pins(attn_pins) == []
+
+
+@pytest.mark.parametrize("name,old,new", ATTN_MUTANTS, ids=[m[0] for m in ATTN_MUTANTS])
+def test_planted_attention_mistake_fails_a_pin(tmp_path, monkeypatch, name, old, new):
+    src = open(tree_attn.__file__).read()
+    assert src.count(old) == 1, "the planted spot must occur exactly once in the oracle"
+    path = tmp_path / "tree_attn_mut.py"
+    path.write_text(src.replace(old, new))
+    spec = importlib.util.spec_from_file_location("tree_attn_mut", path)
+    mut = importlib.util.module_from_spec(spec)
+    spec.loader.exec_module(mut)
+    monkeypatch.setattr(attn_pins, "ta", mut)
+    failed = failing_pins(attn_pins)
     print(name, "->", failed)
     assert failed, f"planted mistake passed every pin: {name}"
