@@ -74,6 +74,17 @@ MUTANTS = [
     ("candidate set: the K smallest drafter logits",
      "for (int v = 0; v < c->V; v++) x[v] = (double)dlog_row[v];",
      "for (int v = 0; v < c->V; v++) x[v] = -(double)dlog_row[v];"),
+    ("candidate set: left in rank order instead of token order",
+     "    qsort(cand, (size_t)c->cand_k, sizeof(int), int_cmp);\n",
+     ""),
+    ("restricted q~: normalised over the full vocabulary",
+     "    double lse = orc_log_softmax(z, K, lq);\n    free(z);",
+     "    double *zf = (double *)malloc(sizeof(double) * (size_t)c->V);\n"
+     "    double *lf = (double *)malloc(sizeof(double) * (size_t)c->V);\n"
+     "    orc_child_logits(c, E, dlog_row, h, zf);\n"
+     "    double lse = orc_log_softmax(zf, c->V, lf);\n"
+     "    for (int i = 0; i < K; i++) lq[i] = z[i] - lse < 0.0 ? z[i] - lse : 0.0;\n"
+     "    free(zf);\n    free(lf);\n    free(z);"),
 ]
 
 
