@@ -38,6 +38,10 @@
  *   - all pointers are DEVICE pointers unless the name says _host;
  *   - `stream` is a cudaStream_t (NULL = legacy default stream); work is
  *     enqueued asynchronously and no call synchronises unless documented;
+ *     with bf16 weights one GEMM of each depth runs on a second stream owned
+ *     by the handle, forked from and joined back into `stream` by events
+ *     within the same call (also when `stream` is being captured into a
+ *     CUDA graph), so stream order as seen by the caller is unchanged;
  *   - return value: DART_OK or a negative dart_status; argument errors are
  *     detected on the host before anything is enqueued;
  *   - a handle must not be used from two streams or threads at once.
