@@ -77,6 +77,15 @@ MUTANTS = [
     ("candidate set: left in rank order instead of token order",
      "    qsort(cand, (size_t)c->cand_k, sizeof(int), int_cmp);\n",
      ""),
+    ("teacher-forced state: every step from the first token",
+     "    for (int i = 0; i < len; i++) {\n        orc_head(c, Wi, Wo, E, h, path[i], t);\n        memcpy(h, t, sizeof(double) * (size_t)d);\n    }\n    memcpy(h_out",
+     "    for (int i = 0; i < len; i++) {\n        orc_head(c, Wi, Wo, E, h, path[0], t);\n        memcpy(h, t, sizeof(double) * (size_t)d);\n    }\n    memcpy(h_out"),
+    ("teacher-forced children: drafter row of the prefix's last position",
+     "const float *row = Dlog_seq + (size_t)len * V;",
+     "const float *row = Dlog_seq + (size_t)(len > 0 ? len - 1 : 0) * V;"),
+    ("teacher-forced scores: beta not added",
+     "s += lq[path[i]] + c->beta;",
+     "s += lq[path[i]];"),
     ("restricted q~: normalised over the full vocabulary",
      "    double lse = orc_log_softmax(z, K, lq);\n    free(z);",
      "    double *zf = (double *)malloc(sizeof(double) * (size_t)c->V);\n"

@@ -58,6 +58,49 @@ def test_head_matches_library_modules(wdtype):
         assert abs(np.mean(got ** 2) - 1.0) < 1e-5
 
 
+@pytest.mark.parametrize("wdtype,cand_k", [("f32", 0), ("bf16", 0), ("f32", 3)])
+def test_teacher_forced_helpers_match_torch(wdtype, cand_k):
+    """The teacher-forced helpers the GPU parity tests use: the state after a
+    path is the library-module head applied token by token from h_0; the
+    Eq. 5 scores along a path and a prefix's children equal the torch
+    log-softmax (over C_i for cand_k > 0) of the same states."""
+    cfg = tiny(V=9, d=16, L=4, W=4, k=4, wdtype=wdtype, cand_k=cand_k, temperature=0.8)
+    x = rand_inputs(cfg)
+    head = TorchHead(cfg, x["Wi"], x["Wo"], x["E"])
+    E64 = head.E
+    path = np.array([4, 0, 7], np.int32)
+    h = torch.from_numpy(x["h0"][0].astype(np.float64))
+    states = [h]
+    for t in path:
+        h = head(h, int(t))
+        states.append(h)
+    for n in range(len(path) + 1):
+        got = oracle.path_state(cfg, x["Wi"], x["Wo"], x["E"], x["h0"][0], path[:n])
+        np.testing.assert_allclose(got, states[n].numpy(), rtol=0, atol=1e-12)
+    want, acc = [], 0.0
+    for i, t in enumerate(path):
+        if cand_k:
+            lq = child_logq_restricted(cfg, E64, x["Dlog"][0, i], states[i], topK_candidates(x["Dlog"][0, i], cand_k))
+        else:
+            lq = child_logq(cfg, E64, x["Dlog"][0, i], states[i])
+        acc += float(lq[int(t)]) + cfg.beta
+        want.append(acc)
+    got = oracle.path_scores(cfg, x["Wi"], x["Wo"], x["E"], x["Dlog"][0], x["h0"][0], path)
+    np.testing.assert_allclose(got, want, rtol=0, atol=1e-12)
+    n = 2
+    if cand_k:
+        lq = child_logq_restricted(cfg, E64, x["Dlog"][0, n], states[n], topK_candidates(x["Dlog"][0, n], cand_k))
+    else:
+        lq = child_logq(cfg, E64, x["Dlog"][0, n], states[n])
+    kk = 3
+    tok, lqk, lse, allq = oracle.node_children(cfg, x["Wi"], x["Wo"], x["E"], x["Dlog"][0], x["h0"][0], path[:n], kk,
+                                                want_all=True)
+    lqn = lq.numpy()
+    np.testing.assert_allclose(allq, lqn, rtol=0, atol=1e-12)
+    np.testing.assert_array_equal(tok, np.lexsort((np.arange(cfg.V), -lqn))[:kk])
+    np.testing.assert_allclose(lqk, lqn[tok], rtol=0, atol=1e-12)
+
+
 def test_child_logits_and_log_softmax_match_torch():
     cfg = tiny(V=300, d=32, temperature=0.7)
     x = rand_inputs(cfg)
