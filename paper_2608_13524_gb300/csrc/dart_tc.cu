@@ -11,8 +11,11 @@
 //     the epilogue of tile i overlap the MMAs of tile i+1.  The epilogue adds
 //     the drafter row, scales by 1/T and reduces on chip to a running
 //     log-sum-exp and a top-k per node, so no [N,V] logits tensor is written.
-//   * Correction-head GEMMs (split-K): A = W_i or W_o tile, B = the node
-//     inputs; each CTA writes an fp32 partial tile.
+//   * Correction-head GEMMs (split-K): A = W_i[:, 0:d] (or all of W_i) or
+//     W_o tile, B = the node inputs; each CTA writes an fp32 partial tile, or
+//     the k splits of a tile form a cluster that sums them on chip.  The same
+//     kernel, with A = W_i[:, d:2d] and B = E rows as nodes, computes the
+//     per-token table Q[t] = W_i[:, d:2d] . E[t] once per handle.
 // Warp roles (192 threads): warp 0 = TMA producer, warp 1 = TMEM allocator
 // and single-thread MMA issuer, warps 2-5 = epilogue (TMEM lane quarters
 // warp%4).  Every wait is bounded: on timeout the CTA records kDevTimeout in
