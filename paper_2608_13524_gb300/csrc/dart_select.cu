@@ -10,8 +10,9 @@
 //       one block per sequence: global top-B by (score desc, node id asc),
 //       compaction in id order, parent remap, depths, position ids and the
 //       ancestor bit mask.
-//   prep / gather / silu / residual_norm: the elementwise parts of the
-//       fallback correction head around the two GEMMs.
+//   prep / gather / silu / gather_silu / residual_norm: the elementwise parts
+//       of the fallback correction head around the two GEMMs (gather_silu
+//       adds the per-token row of the split first layer's table).
 #include <cstdlib>
 
 #include "dart_device.cuh"
