@@ -185,12 +185,14 @@ int dart_profile_read(dart_handle *h, float *lmhead_ms, int *lmhead_launches);
 
 /* Per-kind breakdown of the same profiling events (every launch is
  * bracketed while profiling is enabled).  Kinds: 0 LM-head scoring,
- * 1 merge + frontier select, 2 head-input gather, 3 head GEMM W_i,
- * 4 SiLU + split, 5 head GEMM W_o, 6 residual + RMSNorm, 7 depth-1 anchor
- * preparation, 8 prune + emit, 9 candidate sets C_d (cand_k > 0, once per
- * round), 10 candidate scoring (cand_k > 0, per depth).  ms[i] / launches[i]
- * receive the summed device time and count of kind i for i < nkinds
- * (nkinds <= 11); resets the events. */
+ * 1 merge + frontier select, 2 head-input gather, 3 head GEMM W_i
+ * (W_i[:, 0:d] over the parents with the split first layer of bf16
+ * weights), 4 SiLU + split, 5 head GEMM W_o, 6 residual + RMSNorm,
+ * 7 depth-1 anchor preparation, 8 prune + emit, 9 candidate sets C_d
+ * (cand_k > 0, once per round), 10 candidate scoring (cand_k > 0, per
+ * depth), 11 gather of the per-token table row + SiLU + split (split first
+ * layer).  ms[i] / launches[i] receive the summed device time and count of
+ * kind i for i < nkinds (nkinds <= 12); resets the events. */
 int dart_profile_read_kinds(dart_handle *h, float *ms, int *launches, int nkinds);
 
 /* Number of kernel launches one dart_build_tree enqueues for this handle. */
