@@ -10,6 +10,7 @@ import os
 import socket
 
 import numpy as np
+import pytest
 import torch
 import torch.distributed as dist
 import torch.multiprocessing as mp
@@ -86,5 +87,7 @@ def _vocab_shards(rank, world, out_dir):
     np.testing.assert_allclose(lq, ref_lq[ref_tk], atol=1e-12)
 
 
-def test_vocab_parallel_merge_gloo(tmp_path):
-    spawn(_vocab_shards, tmp_path)
+@pytest.mark.parametrize("world", [2, 3])
+def test_vocab_parallel_merge_gloo(tmp_path, world):
+    """world = 3 splits the 1003 tokens unevenly (334 / 334 / 335)."""
+    spawn(_vocab_shards, tmp_path, world=world)
