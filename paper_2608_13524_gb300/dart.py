@@ -3,7 +3,7 @@
 Argument marshalling only: every step of the construction runs in the CUDA
 kernels of ``libdart.so``.  Functions keep the C names; tensors are passed by
 ``data_ptr()`` and streams by their CUDA handle.  There is no fallback: if the
-library is missing, importing the binding raises.
+library is missing, the first call into it raises.
 """
 from __future__ import annotations
 
