@@ -109,7 +109,7 @@ def kernel_source_sha():
 def split_head(cfg):
     """True when the library splits the first head layer (bf16 weights):
     each depth streams W_i[:, 0:d] (2 d^2 bytes) instead of all of W_i."""
-    return cfg.wdtype == "bf16" and os.environ.get("DART_SPLIT_HEAD", "1")[:1] != "0"
+    return cfg.wdtype == "bf16" and cfg.head_split != 2
 
 
 def wi_bytes_per_depth(cfg):

@@ -69,6 +69,17 @@ typedef enum {
 
 typedef enum { DART_F32 = 0, DART_BF16 = 1 } dart_dtype;
 
+/* Tuning switches of dart_config (every setting computes the same tree up
+ * to the order of fp32 summation; DART_AUTO leaves the choice to the library). */
+enum { DART_AUTO = 0, DART_ON = 1, DART_OFF = 2 };
+
+/* Extra constructions a handle prepares for (dart_config.variants, bit set);
+ * each allocates its own workspace at dart_init_head. */
+enum {
+    DART_VARIANT_CHAIN_DDTREE = 1, /* dart_build_chain_ddtree */
+    DART_VARIANT_SEQ_HEAP = 2      /* dart_build_seq_heap */
+};
+
 /* Problem definition (Algorithm 1 inputs).
  *   V      vocabulary size, 1 <= V < 2^24, V >= k
  *   d      hidden size of the correction head, multiple of 64, 64 <= d <= 16384
@@ -83,12 +94,24 @@ typedef enum { DART_F32 = 0, DART_BF16 = 1 } dart_dtype;
  *   rms_eps      RMSNorm epsilon (> 0)
  *   pos_offset   position id of the root; a node at depth d gets pos_offset+d
  *   cand_k K of Algorithm 1: 0 scores every node over the full vocabulary;
- *          k <= cand_k <= min(V, 1024) scores it over C_d only */
+ *          k <= cand_k <= min(V, 1024) scores it over C_d only
+ * Tuning (DART_AUTO / DART_ON / DART_OFF; bf16 weights only, ignored for fp32):
+ *   head_split         evaluate W_i . [h_p ; E[t_c]] as W_i[:, 0:d] . h_p plus
+ *                      a row of the per-token table Q[t] = W_i[:, d:2d] . E[t]
+ *                      (V*d floats of workspace, built at dart_init_head);
+ *                      AUTO = ON.  OFF keeps no table (gather + full W_i GEMM)
+ *   head_split_stream  with head_split: run the W_i[:, 0:d] GEMM on a second
+ *                      stream beside the selection of the children; AUTO = ON
+ *   lmhead_ctas_per_sm 1 or 2 LM-head CTAs per SM; 0 = by d (2 if d <= 3072
+ *                      and both fit, else 1)
+ *   variants           bit set of DART_VARIANT_* (0: Algorithm 1 only) */
 typedef struct {
     int V, d, L, W, k, B, nseq;
     float beta, temperature, rms_eps;
     int pos_offset;
     int cand_k;
+    int head_split, head_split_stream, lmhead_ctas_per_sm;
+    int variants;
 } dart_config;
 
 /* Emitted verification tree, caller-allocated, per sequence s:
@@ -142,7 +165,9 @@ int dart_prune_and_emit(dart_handle *h, const dart_tree_out *out, void *stream);
 
 /* The whole round: dart_expand_depth for 1..L, then dart_prune_and_emit.
  * Launched as one cached CUDA graph per distinct (inputs, outputs) pointer
- * set unless the stream is being captured by the caller. */
+ * set unless the stream is being captured by the caller.  The handle keeps
+ * the graphs of its 8 most recently used pointer sets (least recently used
+ * one destroyed first), so a caller rotating buffers does not grow memory. */
 int dart_build_tree(dart_handle *h, const float *drafter_logits, const float *anchor_h,
                     const dart_tree_out *out, void *stream);
 
@@ -176,6 +201,17 @@ int dart_get_states(dart_handle *h, float *states, int *rows, void *stream);
 /* Synchronises `stream` and returns (then clears) the device status word:
  * DART_OK, or DART_ERR_TIMEOUT if a kernel's bounded wait gave up. */
 int dart_status_sync(dart_handle *h, void *stream);
+
+/* Test hook for the failure path of the bounded device waits (no fault is
+ * made): one CTA waits on an mbarrier that nothing completes, with the same
+ * wait routine the kernels use but a limit of `limit_us` microseconds
+ * (1 <= limit_us <= 2000000), gives up, sets the abort flag of its CTA and
+ * the DART_ERR_TIMEOUT bit of the handle's status word; a second thread of
+ * the CTA, waiting with the kernels' own 2 s limit on another such barrier,
+ * must return as soon as it sees the abort flag.  No copy or MMA is in
+ * flight.  elapsed_ns (optional, device int64 [2]) receives the time each of
+ * the two waits took.  The next dart_status_sync returns DART_ERR_TIMEOUT. */
+int dart_test_wait_timeout(dart_handle *h, int limit_us, int64_t *elapsed_ns, void *stream);
 
 /* Profiling: when enabled, CUDA events bracket every LM-head scoring launch
  * (forces non-graph launches); dart_profile_read returns the summed device
@@ -217,10 +253,18 @@ int dart_launches_per_round(dart_handle *h);
  * address (cudaGetSymbolAddress) and sets kernel attributes, so make that
  * first call before any stream capture.  Every call on a device shares the
  * array: calls that overlap on the GPU (other streams, other threads) race;
- * serialise them.  Device-side timeouts are not reported by this entry point. */
+ * serialise them.  Device-side timeouts are not reported by the call
+ * itself: dart_noalloc_status reads them afterwards. */
 int dart_expand_root_noalloc(const dart_config *cfg, const void *E, const float *drafter_logits,
                              const float *anchor_h, int32_t *node_tok, float *node_logq, float *node_lse,
                              int32_t *front_tok, float *front_score, int32_t *front_count, void *stream);
+
+/* After dart_expand_root_noalloc on the current device: synchronises
+ * `stream` and returns DART_ERR_TIMEOUT if a device-side wait of the most
+ * recent call gave up, else DART_OK (the status word lives in the static
+ * array, at a fixed offset; nothing is allocated).  DART_ERR_STATE if no
+ * call has been made on this device yet. */
+int dart_noalloc_status(void *stream);
 
 void dart_destroy(dart_handle *h);
 const char *dart_status_string(int code);

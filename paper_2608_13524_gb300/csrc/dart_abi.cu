@@ -36,12 +36,13 @@ using namespace dart;
 
 namespace {
 
-constexpr int kVersion = 1;
+constexpr int kVersion = 2;
 constexpr int kMaxW = 64, kMaxK = 64, kMaxWK = 4096, kMaxSuper = 1024, kMaxB = 1024;
 constexpr int kMaxD = 16384;
 constexpr int kMaxCandK = 1024;  // candidate-set size K of the restricted scoring
 constexpr int kMaxV = (1 << 24) - 1;
 constexpr int kMaxProfilePairs = 8192;
+constexpr size_t kMaxGraphs = 8;  // cached round graphs per handle (least recently used evicted)
 
 EncodeTiledFn encode_fn() { return tensor_map_encoder(); }
 
@@ -80,6 +81,7 @@ struct DepthPlan {
 struct GraphEntry {
     const void* key[9];
     cudaGraphExec_t exec;
+    unsigned long long last_use;
 };
 
 }  // namespace
@@ -127,6 +129,7 @@ struct dart_handle {
     // graphs
     cudaStream_t cap_stream;
     std::vector<GraphEntry> graphs;
+    unsigned long long graph_clock;
     // profiling
     bool profiling;
     std::vector<cudaEvent_t> ev;
@@ -160,12 +163,16 @@ int validate_cfg(const dart_config* c) {
     if (!(c->temperature >= 0.0f) || !std::isfinite(c->temperature)) return DART_ERR_INVALID;
     if (!(c->rms_eps > 0.0f) || !std::isfinite(c->rms_eps)) return DART_ERR_INVALID;
     if (c->cand_k != 0 && (c->cand_k < c->k || c->cand_k > c->V || c->cand_k > kMaxCandK)) return DART_ERR_INVALID;
+    for (int sw : {c->head_split, c->head_split_stream})
+        if (sw != DART_AUTO && sw != DART_ON && sw != DART_OFF) return DART_ERR_INVALID;
+    if (c->lmhead_ctas_per_sm < 0 || c->lmhead_ctas_per_sm > 2) return DART_ERR_INVALID;
+    if (c->variants & ~(DART_VARIANT_CHAIN_DDTREE | DART_VARIANT_SEQ_HEAP)) return DART_ERR_INVALID;
     return DART_OK;
 }
 
-// Node group of the LM-head kernel (up to 128: one MMA of N = 256 covers the
-// hi and lo products of 128 nodes) and of the head GEMMs (up to 64).
-int pick_ng_tc(int N) { return N <= 16 ? 16 : (N <= 32 ? 32 : (N <= 64 ? 64 : 128)); }
+// Node group of the head GEMMs (up to 64) and of the fp32 LM-head kernel; the
+// tensor-core LM-head kernel's plan comes from plan_lmhead_tc (groups of up
+// to 128 nodes: one MMA of N = 256 covers the hi and lo products of 128).
 int pick_ng_gemm(int N) { return N <= 16 ? 16 : (N <= 32 ? 32 : 64); }
 int pick_ng_f32(int N) { return N <= 16 ? 16 : 32; }
 
@@ -213,30 +220,15 @@ int build_plans(dart_handle* h) {
         DepthPlan& p = h->plans[dep];
         p.P = h->caps[dep - 1];
         p.N = c.nseq * p.P;
-        p.NG = tc ? pick_ng_tc(p.N) : pick_ng_f32(p.N);
-        p.G = (p.N + p.NG - 1) / p.NG;
-        p.nV = std::max(1, std::min(h->num_sms / p.G, tiles));
         if (tc) {
-            // Two CTAs per SM when both fit with >= 4 pipeline stages each: two
-            // independent TMA streams per SM, and one CTA's epilogue / start-up /
-            // tail overlaps the other's stream.  Measured on GB300 it pays for
-            // short rows (d = 2560: -4 % per round) but not for d = 4096, where
-            // the deeper single-CTA pipeline and half as many partial lists win.
-            const int fixed = lmhead_tc_fixed_smem(p.NG, c.k, 16);
-            const int half = h->smem_optin / 2 - 2048;
-            const int st2 = tc_stages(half, tc_stage_bytes(p.NG), fixed);
-            const int smem2 = lmhead_tc_fixed_smem(p.NG, c.k, st2) + st2 * tc_stage_bytes(p.NG);
-            const char* force = getenv("DART_LMHEAD_CTAS_PER_SM");  // tuning override: 1 or 2
-            const bool want2 = force ? atoi(force) == 2 : c.d <= 3072;
-            if (want2 && st2 >= 4 && 2 * lmhead_tc_tmem_cols(p.NG) <= 512 &&
-                lmhead_tc_ctas_per_sm(p.NG, smem2) >= 2) {
-                p.stages = st2;
-                p.nV = std::max(1, std::min(2 * h->num_sms / p.G, tiles));
-            } else {
-                p.stages = tc_stages(h->smem_optin, tc_stage_bytes(p.NG), fixed);
-            }
-            if (p.stages < 2) return DART_ERR_UNSUPPORTED;
-            p.smem = lmhead_tc_fixed_smem(p.NG, c.k, p.stages) + p.stages * tc_stage_bytes(p.NG);
+            LmheadPlan lp;
+            if (!plan_lmhead_tc(p.N, c.V, c.d, c.k, h->num_sms, h->smem_optin, c.lmhead_ctas_per_sm, &lp))
+                return DART_ERR_UNSUPPORTED;
+            p.NG = lp.NG;
+            p.G = lp.G;
+            p.nV = lp.nV;
+            p.stages = lp.stages;
+            p.smem = lp.smem;
             // One group of <= 16 nodes: every CTA streams its own slice of
             // E and the launch is HBM-bound.  Besides the stages it loads
             // before waiting on the previous kernel (which is latency-bound
@@ -249,6 +241,9 @@ int build_plans(dart_handle* h) {
                          ? static_cast<int>(kL2PrefetchBytes / (static_cast<long long>(kTileM) * kBlockK * 2) / p.nV)
                          : 0;
         } else {
+            p.NG = pick_ng_f32(p.N);
+            p.G = (p.N + p.NG - 1) / p.NG;
+            p.nV = std::max(1, std::min(h->num_sms / p.G, tiles));
             p.stages = 0;
             p.l2pf = 0;
             p.smem = lmhead_f32_smem(p.NG, c.k);
@@ -271,11 +266,10 @@ int build_plans(dart_handle* h) {
             // runs over the parents' states, which are already held as hi/lo
             // rows (no gather of the inputs), with half of W_i, beside the
             // selection of the children, and Q[t_c] is added in the SiLU
-            // kernel.  DART_SPLIT_HEAD=0 turns it off.
-            const char* sh = getenv("DART_SPLIT_HEAD");
-            p.split = (tc && !(sh && sh[0] == '0')) ? 1 : 0;
-            const char* ss = getenv("DART_SPLIT_SIDE");  // tuning override: 0 = after merge + select, same stream
-            p.side = (p.split && !(ss && ss[0] == '0')) ? 1 : 0;
+            // kernel.  head_split = DART_OFF turns it off; head_split_stream =
+            // DART_OFF runs its GEMM after merge + select on the same stream.
+            p.split = (tc && c.head_split != DART_OFF) ? 1 : 0;
+            p.side = (p.split && c.head_split_stream != DART_OFF) ? 1 : 0;
             p.g1 = p.split ? gemm_plan(h, c.d, p.N, c.d / kBlockK, tc) : gemm_plan(h, 2 * c.d, p.Nc, c.d / kBlockK, tc);
             p.g2 = gemm_plan(h, c.d, p.Nc, c.d / kBlockK, tc);
             if (tc) {
@@ -321,9 +315,6 @@ int build_plans(dart_handle* h) {
                     } else {
                         g->S = std::max(1, std::min(g->KB, cap / tiles_mg));
                     }
-                    if (getenv("DART_DEBUG_PLAN"))
-                        fprintf(stderr, "dart: depth %d gemm K=%d tiles %d x k-splits %d%s, %d CTAs/SM\n", dep, g->K,
-                                tiles_mg, g->S, cl ? " (cluster)" : "", cps);
                 }
                 p.g1.mode = cluster1 ? (p.split ? kGemmSum : kGemmSiluSplit) : kGemmPartials;
                 p.g2.mode = cluster ? kGemmSum : kGemmPartials;
@@ -795,6 +786,22 @@ int check_inputs(const dart_handle* h, const float* dlog, const float* anchor, b
     return DART_OK;
 }
 
+// Keeps `ge` in the handle's graph cache, destroying the least recently used
+// entry when the cache is full (a graph launched earlier on the caller's
+// stream may still run: cudaGraphExecDestroy defers its release until then),
+// and launches it.
+cudaError_t cache_and_launch(dart_handle* h, const GraphEntry& ge, cudaStream_t st) {
+    if (h->graphs.size() >= kMaxGraphs) {
+        size_t lru = 0;
+        for (size_t i = 1; i < h->graphs.size(); i++)
+            if (h->graphs[i].last_use < h->graphs[lru].last_use) lru = i;
+        cudaGraphExecDestroy(h->graphs[lru].exec);
+        h->graphs.erase(h->graphs.begin() + static_cast<long>(lru));
+    }
+    h->graphs.push_back(ge);
+    return cudaGraphLaunch(ge.exec, st);
+}
+
 }  // namespace
 
 extern "C" {
@@ -911,6 +918,7 @@ int dart_build_tree(dart_handle* h, const float* drafter_logits, const float* an
         if (std::memcmp(g.key, key, sizeof key) == 0) {
             h->next_depth = h->cfg.L + 1;
             h->last_rows = h->plans[h->cfg.L].N;
+            g.last_use = ++h->graph_clock;
             return cuda_err(cudaGraphLaunch(g.exec, st));
         }
     }
@@ -931,8 +939,8 @@ int dart_build_tree(dart_handle* h, const float* drafter_logits, const float* an
         h->next_depth = 1;
         return DART_ERR_CUDA;
     }
-    h->graphs.push_back(ge);
-    return cuda_err(cudaGraphLaunch(ge.exec, st));
+    ge.last_use = ++h->graph_clock;
+    return cuda_err(cache_and_launch(h, ge, st));
 }
 
 int dart_build_tree_host(dart_handle* h, const float* drafter_logits_host, const float* anchor_host,
@@ -1035,6 +1043,13 @@ int dart_status_sync(dart_handle* h, void* stream) {
     if (word & kDevTimeout) return DART_ERR_TIMEOUT;
     if (word & kDevOrphan) return DART_ERR_STATE;
     return DART_OK;
+}
+
+int dart_test_wait_timeout(dart_handle* h, int limit_us, int64_t* elapsed_ns, void* stream) {
+    if (!h || limit_us < 1 || limit_us > 2000000) return DART_ERR_INVALID;
+    if (elapsed_ns && (reinterpret_cast<uintptr_t>(elapsed_ns) & 7u)) return DART_ERR_INVALID;
+    return cuda_err(launch_wait_probe(h->status, static_cast<unsigned long long>(limit_us) * 1000ull,
+                                      reinterpret_cast<long long*>(elapsed_ns), static_cast<cudaStream_t>(stream)));
 }
 
 int dart_set_profiling(dart_handle* h, int enable) {

@@ -118,6 +118,16 @@ int gemm_tc_ctas_per_sm(int NG, int smem);
 int gemm_tc_max_clusters(int NG, int smem, int cluster);  // resident CTAs per SM (occupancy API; needs limits set)
 cudaError_t tc_set_smem_limits(int max_dyn);
 
+// Launch plan of the tensor-core LM-head kernel for N nodes: node group NG
+// (16 / 32 / 64 / 128) and G groups, nV vocabulary ranges, pipeline stages
+// and dynamic shared memory; one or two CTAs per SM (ctas_per_sm_pref 1 or 2,
+// 0 = by d).  False if no plan fits the device.
+struct LmheadPlan {
+    int NG, G, nV, stages, smem;
+};
+bool plan_lmhead_tc(int N, int V, int d, int k, int num_sms, int smem_optin, int ctas_per_sm_pref,
+                    LmheadPlan* out);
+
 // fp32 CUDA-core kernels (dart_f32.cu)
 cudaError_t launch_lmhead_f32(const LmheadArgs& a, cudaStream_t st);
 cudaError_t launch_gemm_f32(const GemmArgs& a, cudaStream_t st);
@@ -189,6 +199,9 @@ struct EmitArgs {
     int* status;
 };
 cudaError_t launch_prune_emit(const EmitArgs& a, cudaStream_t st);
+
+// One CTA whose bounded mbarrier waits run out (see dart_test_wait_timeout).
+cudaError_t launch_wait_probe(int* status, unsigned long long limit_ns, long long* elapsed_ns, cudaStream_t st);
 
 // depth-1 preparation: states <- anchors, and their hi/lo bf16 split
 cudaError_t launch_prep_anchor(const float* anchor, int nseq, int d, float* h, __nv_bfloat16* HL, int bhalf,

@@ -39,6 +39,7 @@ __device__ __align__(256) unsigned char g_scratch[kScratchBytes];
 
 struct DeviceSetup {
     bool ready;
+    bool called;          // a call was enqueued on this device (its status word is meaningful)
     unsigned char* base;  // device address of g_scratch on this device
     int sms, optin;
 };
@@ -49,16 +50,19 @@ typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t,
                                   const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
                                   CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
 
+EncodeTiledFn lookup_encode_tiled() {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+        return reinterpret_cast<EncodeTiledFn>(p);
+    return nullptr;
+}
+
+// Looked up once; the initialisation of a function-local static is
+// thread-safe, so first calls from several threads (on any devices) agree.
 EncodeTiledFn encode_tiled() {
-    static EncodeTiledFn fn = nullptr;
-    if (!fn) {
-        void* p = nullptr;
-        cudaDriverEntryPointQueryResult q;
-        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
-                cudaSuccess &&
-            q == cudaDriverEntryPointSuccess)
-            fn = reinterpret_cast<EncodeTiledFn>(p);
-    }
+    static const EncodeTiledFn fn = lookup_encode_tiled();
     return fn;
 }
 
@@ -121,6 +125,7 @@ extern "C" int dart_expand_root_noalloc(const dart_config* cfg, const void* E, c
         return DART_ERR_INVALID;
     if (c.nseq > kMaxSeqNoAlloc || c.d > kMaxDNoAlloc) return DART_ERR_INVALID;
     if (c.cand_k != 0) return DART_ERR_INVALID;  // full-vocabulary scoring only
+    if (c.lmhead_ctas_per_sm < 0 || c.lmhead_ctas_per_sm > 2) return DART_ERR_INVALID;
     if ((reinterpret_cast<uintptr_t>(E) & 15u) || (reinterpret_cast<uintptr_t>(drafter_logits) & 3u) ||
         (reinterpret_cast<uintptr_t>(anchor_h) & 15u))
         return DART_ERR_INVALID;
@@ -135,27 +140,20 @@ extern "C" int dart_expand_root_noalloc(const dart_config* cfg, const void* E, c
     if (tc_set_smem_limits(ds.optin) != cudaSuccess || select_set_smem_limits(ds.optin - 8192) != cudaSuccess)
         return DART_ERR_CUDA;
 
-    // launch plan of depth 1 (the same rule the handle path uses)
+    // launch plan of depth 1: the handle path's plan (plan_lmhead_tc) for N roots
     const int N = c.nseq;
-    const int NG = N <= 16 ? 16 : (N <= 32 ? 32 : 64);
+    LmheadPlan lp;
+    if (!plan_lmhead_tc(N, c.V, c.d, c.k, ds.sms, ds.optin, c.lmhead_ctas_per_sm, &lp) || lp.G != 1)
+        return DART_ERR_UNSUPPORTED;
+    const int NG = lp.NG, nV = lp.nV;
     const int tiles = (c.V + kTileM - 1) / kTileM;
-    const int fixed = lmhead_tc_fixed_smem(NG, c.k, 16);
-    const int sb = tc_stage_bytes(NG);
-    const int st2 = std::min(16, (ds.optin / 2 - 2048 - fixed) / sb);
-    int stages, nV;
-    if (st2 >= 4 && lmhead_tc_ctas_per_sm(NG, lmhead_tc_fixed_smem(NG, c.k, st2) + st2 * sb) >= 2) {
-        stages = st2;
-        nV = std::max(1, std::min(2 * ds.sms, tiles));
-    } else {
-        stages = std::min(16, (ds.optin - fixed) / sb);
-        nV = std::max(1, std::min(ds.sms, tiles));
-    }
-    if (stages < 2) return DART_ERR_UNSUPPORTED;
-    const int smem = lmhead_tc_fixed_smem(NG, c.k, stages) + stages * sb;
     const int Pn = std::min(c.W, c.k);
 
-    // carve the scratch array; reject sizes beyond it
+    // carve the scratch array (the status word first, at a fixed offset that
+    // dart_noalloc_status reads); reject sizes beyond it
     size_t off = 0;
+    int* status = reinterpret_cast<int*>(ds.base);
+    off += 256;
     auto take = [&](size_t bytes) {
         unsigned char* p = ds.base + off;
         off += round256(bytes);
@@ -169,7 +167,6 @@ extern "C" int dart_expand_root_noalloc(const dart_config* cfg, const void* E, c
     int* child_prow = reinterpret_cast<int*>(take(size_t(N) * Pn * 4));
     int* child_tok = reinterpret_cast<int*>(take(size_t(N) * Pn * 4));
     int* seq_ticket = reinterpret_cast<int*>(take(size_t(N) * 4));
-    int* status = reinterpret_cast<int*>(take(4));
     uint64_t* gthr = reinterpret_cast<uint64_t*>(take(size_t(N) * 8));
     if (off > kScratchBytes) return DART_ERR_INVALID;
 
@@ -200,12 +197,12 @@ extern "C" int dart_expand_root_noalloc(const dart_config* cfg, const void* E, c
     la.dlog_seq_stride = static_cast<long long>(c.L) * c.V;
     la.dlog_row_off = 0;
     la.bhalf = kBhalfNoAlloc;
-    la.stages = stages;
+    la.stages = lp.stages;
     la.part_ms = part_ms;
     la.part_key = part_key;
     la.status = status;
     la.gthr = gthr;
-    if (launch_lmhead_tc(&tmE, &tmH, la, smem, st) != cudaSuccess) return DART_ERR_CUDA;
+    if (launch_lmhead_tc(&tmE, &tmH, la, lp.smem, st) != cudaSuccess) return DART_ERR_CUDA;
 
     SelectArgs sa;
     std::memset(&sa, 0, sizeof sa);
@@ -235,5 +232,25 @@ extern "C" int dart_expand_root_noalloc(const dart_config* cfg, const void* E, c
     sa.seq_ticket = seq_ticket;
     sa.status = status;
     if (launch_merge_select(sa, st) != cudaSuccess) return DART_ERR_CUDA;
+    {
+        std::lock_guard<std::mutex> lock(g_setup_mu);
+        g_setup[dev].called = true;
+    }
     return DART_OK;
+}
+
+extern "C" int dart_noalloc_status(void* stream) {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return DART_ERR_CUDA;
+    if (dev < 0 || dev >= kMaxDevices) return DART_ERR_UNSUPPORTED;
+    unsigned char* base = nullptr;
+    {
+        std::lock_guard<std::mutex> lock(g_setup_mu);
+        if (!g_setup[dev].ready || !g_setup[dev].called) return DART_ERR_STATE;
+        base = g_setup[dev].base;
+    }
+    if (cudaStreamSynchronize(static_cast<cudaStream_t>(stream)) != cudaSuccess) return DART_ERR_CUDA;
+    int word = 0;  // a pageable host int: cudaMemcpy stages it without allocating device memory
+    if (cudaMemcpy(&word, base, sizeof word, cudaMemcpyDeviceToHost) != cudaSuccess) return DART_ERR_CUDA;
+    return (word & kDevTimeout) ? DART_ERR_TIMEOUT : DART_OK;
 }

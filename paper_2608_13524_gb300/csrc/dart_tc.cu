@@ -544,6 +544,35 @@ int lmhead_fixed(int k, int stages) {
            NG * 4 + 8;
 }
 
+// The failure path of the bounded waits, exercised without a fault: two
+// mbarriers that nothing ever completes (count 1, no arrival, no copy or MMA
+// tracked by them).  Thread 0 waits with limit_ns, gives up and records the
+// timeout exactly as the pipeline roles do (abort flag + status bit); thread
+// 32 waits with the kernels' own limit and returns once it sees the abort
+// flag.  Each records how long its wait took.
+__global__ void __launch_bounds__(64) wait_probe_kernel(int* status, unsigned long long limit_ns,
+                                                        long long* elapsed_ns) {
+    __shared__ __align__(8) uint64_t bar[2];
+    __shared__ int abort_flag;
+    if (threadIdx.x == 0) {
+        mbar_init(&bar[0], 1);
+        mbar_init(&bar[1], 1);
+        abort_flag = 0;
+        fence_mbar_init();
+    }
+    __syncthreads();
+    volatile int* abort = &abort_flag;
+    const unsigned long long t0 = globaltimer_ns();
+    long long took = -1;
+    if (threadIdx.x == 0) {
+        if (!mbar_wait(&bar[0], 0, abort, limit_ns)) record_timeout(status, abort);
+        took = static_cast<long long>(globaltimer_ns() - t0);
+    } else if (threadIdx.x == 32) {
+        if (!mbar_wait(&bar[1], 0, abort)) took = static_cast<long long>(globaltimer_ns() - t0);
+    }
+    if (elapsed_ns && took >= 0) elapsed_ns[threadIdx.x == 0 ? 0 : 1] = took;
+}
+
 template <int NG>
 cudaError_t launch_lmhead_ng(const CUtensorMap* tmE, const CUtensorMap* tmH, const LmheadArgs& a, int smem,
                              cudaStream_t st) {
@@ -620,9 +649,6 @@ static int ctas_per_sm(const void* fn, int nthreads, int smem) {
     int n = per_smem > 0 ? sm_smem / per_smem : 1;
     if (per_regs > 0) n = std::min(n, sm_regs / per_regs);
     n = std::min(n, sm_threads / nthreads);
-    if (getenv("DART_DEBUG_PLAN"))
-        fprintf(stderr, "dart: smem %d (+%zu static, +%d reserved) of %d, regs %d x %d of %d -> %d CTAs/SM\n", smem,
-                fa.sharedSizeBytes, reserved, sm_smem, fa.numRegs, nthreads, sm_regs, n);
     return std::max(n, 1);
 }
 
@@ -649,6 +675,36 @@ int lmhead_tc_ctas_per_sm(int NG, int smem) {
         case 64: return ctas_per_sm(reinterpret_cast<const void*>(lmhead_tc_kernel<64>), threads<64>(), smem);
         default: return ctas_per_sm(reinterpret_cast<const void*>(lmhead_tc_kernel<128>), threads<128>(), smem);
     }
+}
+
+bool plan_lmhead_tc(int N, int V, int d, int k, int num_sms, int smem_optin, int ctas_per_sm_pref,
+                    LmheadPlan* out) {
+    LmheadPlan p;
+    p.NG = N <= 16 ? 16 : (N <= 32 ? 32 : (N <= 64 ? 64 : 128));
+    p.G = (N + p.NG - 1) / p.NG;
+    const int tiles = (V + kTileM - 1) / kTileM;
+    p.nV = std::max(1, std::min(num_sms / p.G, tiles));
+    const int sb = tc_stage_bytes(p.NG);
+    const int fixed = lmhead_tc_fixed_smem(p.NG, k, 16);
+    auto stages_in = [&](int budget) { return std::min(16, (budget - fixed) / sb); };
+    // Two CTAs per SM when both fit with >= 4 pipeline stages each: two
+    // independent TMA streams per SM, and one CTA's epilogue / start-up /
+    // tail overlaps the other's stream.  Measured on GB300 it pays for
+    // short rows (d = 2560: -4 % per round) but not for d = 4096, where
+    // the deeper single-CTA pipeline and half as many partial lists win.
+    const int st2 = stages_in(smem_optin / 2 - 2048);
+    const int smem2 = lmhead_tc_fixed_smem(p.NG, k, st2) + st2 * sb;
+    const bool want2 = ctas_per_sm_pref ? ctas_per_sm_pref == 2 : d <= 3072;
+    if (want2 && st2 >= 4 && 2 * lmhead_tc_tmem_cols(p.NG) <= 512 && lmhead_tc_ctas_per_sm(p.NG, smem2) >= 2) {
+        p.stages = st2;
+        p.nV = std::max(1, std::min(2 * num_sms / p.G, tiles));
+    } else {
+        p.stages = stages_in(smem_optin);
+    }
+    if (p.stages < 2) return false;
+    p.smem = lmhead_tc_fixed_smem(p.NG, k, p.stages) + p.stages * sb;
+    *out = p;
+    return true;
 }
 
 cudaError_t tc_set_smem_limits(int max_dyn) {
@@ -687,6 +743,11 @@ cudaError_t launch_gemm_tc(const CUtensorMap* tmA, const CUtensorMap* tmB, const
         case 64: return launch_gemm_ng<64>(tmA, tmB, a, smem, st);
         default: return cudaErrorInvalidValue;
     }
+}
+
+cudaError_t launch_wait_probe(int* status, unsigned long long limit_ns, long long* elapsed_ns, cudaStream_t st) {
+    wait_probe_kernel<<<1, 64, 0, st>>>(status, limit_ns, elapsed_ns);
+    return cudaGetLastError();
 }
 
 }  // namespace dart

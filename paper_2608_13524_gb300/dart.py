@@ -24,13 +24,17 @@ DART_ERR_STATE = -5
 DART_ERR_UNSUPPORTED = -6
 DART_F32 = 0
 DART_BF16 = 1
+DART_AUTO, DART_ON, DART_OFF = 0, 1, 2
+DART_VARIANT_CHAIN_DDTREE = 1
+DART_VARIANT_SEQ_HEAP = 2
 
 
 class DartConfig(C.Structure):
     _fields_ = [("V", C.c_int), ("d", C.c_int), ("L", C.c_int), ("W", C.c_int), ("k", C.c_int),
                 ("B", C.c_int), ("nseq", C.c_int), ("beta", C.c_float),
                 ("temperature", C.c_float), ("rms_eps", C.c_float), ("pos_offset", C.c_int),
-                ("cand_k", C.c_int)]
+                ("cand_k", C.c_int), ("head_split", C.c_int), ("head_split_stream", C.c_int),
+                ("lmhead_ctas_per_sm", C.c_int), ("variants", C.c_int)]
 
 
 class DartTreeOut(C.Structure):
@@ -71,6 +75,8 @@ def lib():
             "dart_get_node_topk": (i, [vp, vp, vp, vp, C.POINTER(i), vp]),
             "dart_get_states": (i, [vp, vp, C.POINTER(i), vp]),
             "dart_status_sync": (i, [vp, vp]),
+            "dart_test_wait_timeout": (i, [vp, i, vp, vp]),
+            "dart_noalloc_status": (i, [vp]),
             "dart_set_profiling": (i, [vp, i]),
             "dart_profile_read": (i, [vp, C.POINTER(f), C.POINTER(i)]),
             "dart_profile_read_kinds": (i, [vp, vp, vp, i]),
@@ -115,10 +121,14 @@ def _stream(stream):
 
 def make_config(cfg) -> DartConfig:
     """From any object with V, d, L, W, k, B, nseq, beta, temperature,
-    rms_eps, pos_offset and optionally cand_k (0: full vocabulary)."""
+    rms_eps, pos_offset and optionally cand_k (0: full vocabulary) and the
+    tuning fields head_split, head_split_stream, lmhead_ctas_per_sm, variants
+    (0: the library's choice)."""
+    g = lambda name: int(getattr(cfg, name, 0))
     return DartConfig(int(cfg.V), int(cfg.d), int(cfg.L), int(cfg.W), int(cfg.k), int(cfg.B),
                       int(cfg.nseq), float(cfg.beta), float(cfg.temperature), float(cfg.rms_eps),
-                      int(cfg.pos_offset), int(getattr(cfg, "cand_k", 0)))
+                      int(cfg.pos_offset), g("cand_k"), g("head_split"), g("head_split_stream"),
+                      g("lmhead_ctas_per_sm"), g("variants"))
 
 
 def alloc_tree_out(cfg, device="cuda", pin=False):
@@ -207,6 +217,13 @@ def dart_status_sync(h, stream=None):
     return int(lib().dart_status_sync(h, _stream(stream)))
 
 
+def dart_test_wait_timeout(h, limit_us, elapsed_ns=None, stream=None):
+    """Runs the bounded-wait probe (see dart.h); the next dart_status_sync
+    returns DART_ERR_TIMEOUT.  elapsed_ns: optional int64 device tensor [2]."""
+    _check(lib().dart_test_wait_timeout(h, int(limit_us), _ptr(elapsed_ns), _stream(stream)),
+           "dart_test_wait_timeout")
+
+
 def dart_set_profiling(h, enable):
     _check(lib().dart_set_profiling(h, int(bool(enable))), "dart_set_profiling")
 
@@ -244,6 +261,12 @@ def dart_expand_root_noalloc(cfg, E, drafter_logits, anchor_h, node_tok, node_lo
                                           _ptr(node_tok), _ptr(node_logq), _ptr(node_lse), _ptr(front_tok),
                                           _ptr(front_score), _ptr(front_count), _stream(stream)),
            "dart_expand_root_noalloc")
+
+
+def dart_noalloc_status(stream=None):
+    """DART_OK or DART_ERR_TIMEOUT for the most recent dart_expand_root_noalloc
+    on the current device (synchronises the stream)."""
+    return int(lib().dart_noalloc_status(_stream(stream)))
 
 
 def dart_destroy(h):

@@ -7,18 +7,17 @@ import bench
 from workloads import NAMED
 
 
-def test_first_head_layer_bytes_per_depth(monkeypatch):
+def test_first_head_layer_bytes_per_depth():
     q8 = NAMED["qwen3-8b"]
-    monkeypatch.delenv("DART_SPLIT_HEAD", raising=False)
-    # split first layer: W_i[:, 0:d] only, d*d bf16 elements
+    # split first layer (the default): W_i[:, 0:d] only, d*d bf16 elements
     assert bench.split_head(q8)
     assert bench.wi_bytes_per_depth(q8) == 4096 * 4096 * 2
-    # unsplit: all of W_i [d][2d]
-    monkeypatch.setenv("DART_SPLIT_HEAD", "0")
-    assert not bench.split_head(q8)
-    assert bench.wi_bytes_per_depth(q8) == 4096 * 2 * 4096 * 2
+    # unsplit (dart_config.head_split = DART_OFF): all of W_i [d][2d]
+    off = q8.replace(head_split=2)
+    assert not bench.split_head(off)
+    assert bench.wi_bytes_per_depth(off) == 4096 * 2 * 4096 * 2
+    assert bench.split_head(q8.replace(head_split=1))
     # the fp32 toy never splits
-    monkeypatch.delenv("DART_SPLIT_HEAD", raising=False)
     toy = NAMED["toy"]
     assert not bench.split_head(toy)
     assert bench.wi_bytes_per_depth(toy) == 2 * toy.d * toy.d * 4
@@ -32,12 +31,9 @@ def test_first_head_layer_bytes_per_depth(monkeypatch):
     ("batched-k64", True, (False, False)),    # 256 children: cluster GEMMs, nothing kept
     ("qwen3-8b", True, (False, False)),       # full vocabulary: the E stream evicts them
 ])
-def test_kept_head_weights_mirrors_the_plan(monkeypatch, name, split, expect):
-    if split:
-        monkeypatch.delenv("DART_SPLIT_HEAD", raising=False)
-    else:
-        monkeypatch.setenv("DART_SPLIT_HEAD", "0")
-    assert bench.kept_head_weights(NAMED[name]) == expect
+def test_kept_head_weights_mirrors_the_plan(name, split, expect):
+    cfg = NAMED[name] if split else NAMED[name].replace(head_split=2)
+    assert bench.kept_head_weights(cfg) == expect
 
 
 def test_whole_job_rate_counts_every_rank():

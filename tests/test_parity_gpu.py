@@ -161,16 +161,17 @@ def test_build_tree_graph_matches_depthwise(dart, cfg):
 VARIANT_CFGS = [SMALL[2], SMALL[5], SMALL[6], RESTRICTED[1]]
 
 
-@pytest.mark.parametrize("env", [{"DART_SPLIT_HEAD": "0"}, {"DART_SPLIT_SIDE": "0"}], ids=["unsplit", "same-stream"])
+@pytest.mark.parametrize("switch", [dict(head_split=2), dict(head_split_stream=2), dict(lmhead_ctas_per_sm=1),
+                                    dict(lmhead_ctas_per_sm=2)],
+                         ids=["unsplit", "same-stream", "lmhead-1cta", "lmhead-2cta"])
 @pytest.mark.parametrize("cfg", VARIANT_CFGS, ids=[c.name for c in VARIANT_CFGS])
-def test_head_update_variants(dart, cfg, env, monkeypatch):
-    """The head-update variants the library keeps behind its tuning switches
-    (read when a handle is created): the unsplit first layer (gather of
-    [h_p ; E[t_c]] and the full W_i GEMM) and the split layer's GEMM on the
-    main stream.  Each matches the oracle, and the graph launch equals the
-    depth-by-depth calls."""
-    for k, v in env.items():
-        monkeypatch.setenv(k, v)
+def test_head_update_variants(dart, cfg, switch):
+    """The variants behind the tuning fields of dart_config: the unsplit first
+    head layer (gather of [h_p ; E[t_c]] and the full W_i GEMM, no table), the
+    split layer's GEMM on the main stream, and one or two LM-head CTAs per SM.
+    Each matches the oracle, and the graph launch equals the depth-by-depth
+    calls."""
+    cfg = cfg.replace(**switch)
     x = make_inputs(cfg)
     dx = to_device(cfg, x)
     ref = oracle.build_tree(cfg, x["Wi"], x["Wo"], x["E"], x["Dlog"], x["h0"])

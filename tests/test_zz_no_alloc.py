@@ -40,20 +40,43 @@ def handle_depth1(dart, cfg, dx):
         dart.dart_destroy(h)
 
 
-@pytest.mark.parametrize("nseq,V,d,W,k,T", [(3, 20000, 512, 8, 12, 0.7), (1, 151936, 4096, 16, 16, 1.0)])
+def outputs(nseq, W, k):
+    """Output tensors pre-filled with values no correct call leaves behind."""
+    return [torch.full((nseq, k), -7, dtype=torch.int32, device="cuda"),
+            torch.full((nseq, k), 7.0, device="cuda"), torch.full((nseq,), 7.0, device="cuda"),
+            torch.full((nseq, W), -7, dtype=torch.int32, device="cuda"),
+            torch.full((nseq, W), 7.0, device="cuda"), torch.full((nseq,), -7, dtype=torch.int32, device="cuda")]
+
+
+def dirty_the_array(dart):
+    """One call of another shape (64 roots, d = 4096, k = 64), so the static
+    array holds this call's partial lists, states and padding rows when the
+    next call starts."""
+    cfg = Config("noalloc-dirty", 64, 30000, 4096, 2, 64, 64, 64, "bf16", 0.5, 8999)
+    x = make_inputs(cfg)
+    dx = to_device(cfg, x)
+    dart.dart_expand_root_noalloc(cfg, dx["E"], dx["Dlog"], dx["h0"], *outputs(64, 64, 64))
+    assert dart.dart_noalloc_status() == dart.DART_OK
+
+
+CASES = [(3, 20000, 512, 8, 12, 0.7),      # 16-node group, W <= k
+         (1, 151936, 4096, 16, 16, 1.0),   # the Qwen3-8B shape
+         (40, 20000, 2560, 6, 4, 0.0),     # 64-node group, W > k (unused frontier ranks), greedy T = 0
+         (17, 9000, 1024, 8, 8, 0.3)]      # 32-node group
+
+
+@pytest.mark.parametrize("nseq,V,d,W,k,T", CASES)
 def test_noalloc_matches_handle_path_twice(dart, nseq, V, d, W, k, T):
     cfg = Config("noalloc", nseq, V, d, 4, W, k, 20, "bf16", T, 9000 + nseq)
     x = make_inputs(cfg)
     dx = to_device(cfg, x)
     ref = handle_depth1(dart, cfg, dx)
     tol = tol_of(cfg)
+    dirty_the_array(dart)
     for call in range(2):  # the second call reuses the array the first one left behind
-        out = [torch.full((nseq, k), -7, dtype=torch.int32, device="cuda"),
-               torch.full((nseq, k), 7.0, device="cuda"), torch.full((nseq,), 7.0, device="cuda"),
-               torch.full((nseq, W), -7, dtype=torch.int32, device="cuda"),
-               torch.full((nseq, W), 7.0, device="cuda"), torch.full((nseq,), -7, dtype=torch.int32, device="cuda")]
+        out = outputs(nseq, W, k)
         dart.dart_expand_root_noalloc(cfg, dx["E"], dx["Dlog"], dx["h0"], *out)
-        torch.cuda.synchronize()
+        assert dart.dart_noalloc_status() == dart.DART_OK
         got = [t.cpu().numpy() for t in out]
         np.testing.assert_array_equal(got[0], ref[0], err_msg=f"node tokens, call {call}")
         np.testing.assert_allclose(got[1], ref[1], atol=tol, rtol=0, err_msg=f"node log q, call {call}")
@@ -61,6 +84,8 @@ def test_noalloc_matches_handle_path_twice(dart, nseq, V, d, W, k, T):
         np.testing.assert_array_equal(got[3], ref[3], err_msg=f"frontier tokens, call {call}")
         np.testing.assert_allclose(got[4], ref[4], atol=tol, rtol=0, err_msg=f"frontier scores, call {call}")
         np.testing.assert_array_equal(got[5], ref[5], err_msg=f"frontier counts, call {call}")
+        if W > k:  # unused frontier ranks of the single parent
+            assert np.all(got[3][:, k:] == -1) and np.all(np.isneginf(got[4][:, k:]))
 
 
 def test_noalloc_rejects_sizes_beyond_its_array(dart):

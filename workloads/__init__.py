@@ -54,6 +54,12 @@ class Config:
     spike_early: float = 6.0   # positions 0..7
     spike_late: float = 3.0    # positions 8..
     cand_k: int = 0            # K of Algorithm 1 (candidate-set size); 0 = full vocabulary
+    # library tuning switches (dart_config; 0 = the library's choice, 1 = on,
+    # 2 = off): they change neither the inputs nor the tree
+    head_split: int = 0
+    head_split_stream: int = 0
+    lmhead_ctas_per_sm: int = 0
+    variants: int = 0          # extra constructions prepared by the handle (bit set)
 
     def replace(self, **kw) -> "Config":
         return dataclasses.replace(self, **kw)
