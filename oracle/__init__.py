@@ -5,7 +5,9 @@ benchmark's CPU-baseline leg may use this package; the product path never
 imports it.  It shares no code with the CUDA path.
 
 The arithmetic lives in ``dart_oracle.c`` (Algorithm 1, Eq. 5, Lemma 1 of the
-paper, each function citing its passage).  This file only builds the C
+paper, and the two constructions Table 2 compares DARTree with: Domino-chain +
+DDTree and sequential correction with heap; each function citing its
+passage).  This file only builds the C
 library and marshals numpy arrays.  ``cfg`` arguments are any object with the
 fields V, d, L, W, k, B, nseq, pos_offset, wdtype ("f32"/"bf16"), beta,
 temperature, rms_eps.
@@ -36,13 +38,16 @@ def build(force: bool = False) -> str:
     if (not force and os.path.exists(_LIB)
             and os.path.getmtime(_LIB) >= os.path.getmtime(_SRC)):
         return _LIB
-    base = ["gcc", "-O2", "-std=c11", "-shared", "-fPIC", _SRC, "-o", _LIB + ".tmp", "-lm"]
+    # a private temporary per process, renamed into place atomically, so
+    # processes that build at the same time never load a half-written file
+    tmp = f"{_LIB}.{os.getpid()}.tmp"
+    base = ["gcc", "-O2", "-std=c11", "-shared", "-fPIC", _SRC, "-o", tmp, "-lm"]
     try:
         subprocess.run(base[:1] + ["-fopenmp"] + base[1:], check=True,
                        capture_output=True)
     except subprocess.CalledProcessError:
         subprocess.run(base, check=True, capture_output=True)
-    os.replace(_LIB + ".tmp", _LIB)
+    os.replace(tmp, _LIB)
     return _LIB
 
 
@@ -69,7 +74,7 @@ def lib():
         _lib.orc_num_threads.restype = C.c_int
         _lib.orc_log_softmax.restype = C.c_double
         _lib.orc_node_children.restype = C.c_double
-        for f in ("orc_build_tree", "orc_prune_emit", "orc_heap_select"):
+        for f in ("orc_build_tree", "orc_prune_emit", "orc_heap_select", "orc_chain_ddtree", "orc_seq_heap"):
             getattr(_lib, f).restype = C.c_int
     return _lib
 
@@ -199,6 +204,46 @@ def heap_select(cfg, st_parent, st_score, st_count, s=0):
     n = lib().orc_heap_select(C.byref(_cfg(cfg)), _p(st_parent), _p(st_score),
                               _p(st_count), C.c_int(s), _p(out))
     return out[:n].copy()
+
+
+# ------------------------------------------- heap-based constructions
+
+def _tree_out(cfg):
+    ns, B = cfg.nseq, cfg.B
+    nw = (B + 63) // 64
+    return dict(tokens=np.empty((ns, B), np.int32), parents=np.empty((ns, B), np.int32),
+                depths=np.empty((ns, B), np.int32), pos_ids=np.empty((ns, B), np.int32),
+                scores=np.empty((ns, B), np.float64), n_nodes=np.empty(ns, np.int32),
+                mask=np.empty((ns, B, nw), np.uint64))
+
+
+def chain_ddtree(cfg, Wi, Wo, E, Dlog, h0):
+    """Domino-chain + DDTree (see ``orc_chain_ddtree``): the emitted tree in
+    pop order plus the chain (chain_tok, chain_lse [nseq][L])."""
+    Wi, Wo, E = _w(cfg, Wi), _w(cfg, Wo), _w(cfg, E)
+    Dlog = np.ascontiguousarray(Dlog, dtype=np.float32)
+    h0 = np.ascontiguousarray(h0, dtype=np.float32)
+    r = _tree_out(cfg)
+    r["chain_tok"] = np.empty((cfg.nseq, cfg.L), np.int32)
+    r["chain_lse"] = np.empty((cfg.nseq, cfg.L), np.float64)
+    lib().orc_chain_ddtree(C.byref(_cfg(cfg)), _p(Wi), _p(Wo), _p(E), _p(Dlog), _p(h0), _p(r["chain_tok"]),
+                           _p(r["chain_lse"]), _p(r["tokens"]), _p(r["parents"]), _p(r["depths"]),
+                           _p(r["pos_ids"]), _p(r["scores"]), _p(r["n_nodes"]), _p(r["mask"]))
+    return r
+
+
+def seq_heap(cfg, Wi, Wo, E, Dlog, h0):
+    """Sequential correction with heap (see ``orc_seq_heap``): the emitted
+    tree in pop order plus expansions [nseq] (children distributions computed)."""
+    Wi, Wo, E = _w(cfg, Wi), _w(cfg, Wo), _w(cfg, E)
+    Dlog = np.ascontiguousarray(Dlog, dtype=np.float32)
+    h0 = np.ascontiguousarray(h0, dtype=np.float32)
+    r = _tree_out(cfg)
+    r["expansions"] = np.empty(cfg.nseq, np.int32)
+    lib().orc_seq_heap(C.byref(_cfg(cfg)), _p(Wi), _p(Wo), _p(E), _p(Dlog), _p(h0), _p(r["tokens"]),
+                       _p(r["parents"]), _p(r["depths"]), _p(r["pos_ids"]), _p(r["scores"]), _p(r["n_nodes"]),
+                       _p(r["mask"]), _p(r["expansions"]))
+    return r
 
 
 # ------------------------------------------------- teacher-forced helpers

@@ -591,3 +591,199 @@ void orc_path_scores(const orc_cfg *c, const void *Wi, const void *Wo, const voi
     free(t);
     free(lq);
 }
+
+/* ------------------------------------------- heap-based constructions */
+
+/* Emission of a tree built by best-first popping (rows in pop order, which is
+ * a topological order: a node is popped after its parent).  Row i holds
+ * token tok[i], parent row par[i] (-1: the root), depth dep[i] and score
+ * sc[i]; mask rows by the ancestor walk; rows n..B-1 are padding. */
+static void emit_pop_order(const orc_cfg *c, int s, int n, const int *tok, const int *par, const int *dep,
+                           const double *sc, int *o_tok, int *o_par, int *o_dep, int *o_pos, double *o_score,
+                           int *o_n, uint64_t *o_mask) {
+    const int B = c->B, nw = (B + 63) / 64;
+    for (int i = 0; i < B; i++) {
+        const size_t o = (size_t)s * B + i;
+        uint64_t *row = o_mask + o * nw;
+        memset(row, 0, sizeof(uint64_t) * nw);
+        if (i < n) {
+            o_tok[o] = tok[i];
+            o_par[o] = par[i];
+            o_dep[o] = dep[i];
+            o_pos[o] = c->pos_offset + dep[i];
+            o_score[o] = sc[i];
+            for (int a = i; a >= 0; a = par[a]) row[a / 64] |= 1ull << (a % 64);
+        } else {
+            o_tok[o] = -1;
+            o_par[o] = -2;
+            o_dep[o] = 0;
+            o_pos[o] = -1;
+            o_score[o] = -INFINITY;
+        }
+    }
+    o_n[s] = n;
+}
+
+/* Sorted child list of a distribution: the m = min(B, entries) best
+ * (log q~ desc, token asc) tokens and their log q~.  lq_all holds log q~ of
+ * every token (-inf outside C_d when the candidate set is restricted). */
+static int child_list(const orc_cfg *c, const double *lq_all, int *ltok, double *llq) {
+    const int nent = c->cand_k > 0 ? c->cand_k : c->V;
+    const int m = c->B < nent ? c->B : nent;
+    orc_topk(lq_all, c->V, m, ltok);
+    for (int j = 0; j < m; j++) llq[j] = lq_all[ltok[j]];
+    return m;
+}
+
+/* One best-first step over the popped nodes (and the root, index -1): every
+ * node p with depth < L offers its best child not yet taken, child rank
+ * next[p] of its sorted list, scored s_p + log q~ + beta (Eq. 5).  Returns
+ * the node whose offer is best by (score desc, node asc; the root first), or
+ * -2 if no finite offer remains.  lists: row p+1 of ltok/llq/llen. */
+static int best_offer(const orc_cfg *c, int n, const int *dep, const double *sc, const int *next,
+                      const int *llen, const double *llq, int lstride, double *best_score) {
+    int best = -2;
+    double bs = -INFINITY;
+    for (int p = -1; p < n; p++) {
+        const int dp = p < 0 ? 0 : dep[p];
+        if (dp >= c->L || next[p + 1] >= llen[p + 1]) continue;
+        const double v = (p < 0 ? 0.0 : sc[p]) + llq[(size_t)(p + 1) * lstride + next[p + 1]] + c->beta;
+        if (v == -INFINITY) continue;
+        if (best == -2 || v > bs) { /* p ascends, so ties keep the earlier node */
+            best = p;
+            bs = v;
+        }
+    }
+    *best_score = bs;
+    return best;
+}
+
+/* Domino-chain + DDTree (Sec. 5.2, Table 2): causal correction along ONE draft
+ * chain, then DDTree (Sec. 3.3) over the chain-conditioned distributions.
+ * Per sequence:
+ *   1. the chain: from r_0, at each depth d = 1..L the corrected distribution
+ *      q~_d(. | y_<d) of the chain prefix (over V, or over C_d when cand_k > 0),
+ *      its argmax y_d (log q~ desc, token asc), and, for d < L, the state
+ *      r(y_1..y_d) = g(r(y_<d), y_d);
+ *   2. DDTree: the chain's distributions are used as position-wise marginals
+ *      shared by every node of a depth; best-first search over prefixes
+ *      scored s = sum_i log q~_i(u_i) + beta d (beta = 0: DDTree's mass
+ *      objective), each pop taking the best offer (next child in
+ *      sorted order of a popped node, DDTree's "next sibling / first child"
+ *      pushes), until B nodes are popped.
+ * Emitted in pop order; chain_tok / chain_lse [nseq][L] receive the chain and
+ * the log-sum-exp of each of its distributions. */
+int orc_chain_ddtree(const orc_cfg *c, const void *Wi, const void *Wo, const void *E, const float *Dlog,
+                     const float *h0, int *chain_tok, double *chain_lse, int *o_tok, int *o_par, int *o_dep,
+                     int *o_pos, double *o_score, int *o_n, uint64_t *o_mask) {
+    const int V = c->V, d = c->d, L = c->L, B = c->B;
+    double *h = (double *)malloc(sizeof(double) * (size_t)d);
+    double *t = (double *)malloc(sizeof(double) * (size_t)d);
+    double *lq = (double *)malloc(sizeof(double) * (size_t)V);
+    int *ltok = (int *)malloc(sizeof(int) * (size_t)L * B);     /* per depth */
+    double *llq = (double *)malloc(sizeof(double) * (size_t)L * B);
+    int *llen = (int *)malloc(sizeof(int) * (size_t)L);
+    int *ptok = (int *)malloc(sizeof(int) * (size_t)B), *ppar = (int *)malloc(sizeof(int) * (size_t)B);
+    int *pdep = (int *)malloc(sizeof(int) * (size_t)B), *next = (int *)malloc(sizeof(int) * (size_t)(B + 1));
+    int *olen = (int *)malloc(sizeof(int) * (size_t)(B + 1));
+    double *psc = (double *)malloc(sizeof(double) * (size_t)B);
+    double *olq = (double *)malloc(sizeof(double) * (size_t)(B + 1) * B); /* offers per node, by its depth */
+    for (int s = 0; s < c->nseq; s++) {
+        /* 1. the chain */
+        for (int j = 0; j < d; j++) h[j] = (double)h0[(size_t)s * d + j];
+        for (int dep = 1; dep <= L; dep++) {
+            const float *drow = Dlog + ((size_t)s * L + dep - 1) * V; /* position dep-1 */
+            chain_lse[(size_t)s * L + dep - 1] = child_logq_all(c, E, drow, h, lq);
+            llen[dep - 1] = child_list(c, lq, ltok + (size_t)(dep - 1) * B, llq + (size_t)(dep - 1) * B);
+            const int y = ltok[(size_t)(dep - 1) * B];
+            chain_tok[(size_t)s * L + dep - 1] = y;
+            if (dep < L) {
+                orc_head(c, Wi, Wo, E, h, y, t);
+                memcpy(h, t, sizeof(double) * (size_t)d);
+            }
+        }
+        /* 2. DDTree over the chain-conditioned marginals */
+        int n = 0;
+        next[0] = 0;
+        olen[0] = llen[0];
+        memcpy(olq, llq, sizeof(double) * (size_t)B);
+        while (n < B) {
+            double v;
+            const int p = best_offer(c, n, pdep, psc, next, olen, olq, B, &v);
+            if (p == -2) break;
+            const int dep = p < 0 ? 1 : pdep[p] + 1;
+            ptok[n] = ltok[(size_t)(dep - 1) * B + next[p + 1]];
+            ppar[n] = p;
+            pdep[n] = dep;
+            psc[n] = v;
+            next[p + 1]++;
+            next[n + 1] = 0;
+            olen[n + 1] = dep < L ? llen[dep] : 0;
+            if (dep < L) memcpy(olq + (size_t)(n + 1) * B, llq + (size_t)dep * B, sizeof(double) * (size_t)B);
+            n++;
+        }
+        emit_pop_order(c, s, n, ptok, ppar, pdep, psc, o_tok, o_par, o_dep, o_pos, o_score, o_n, o_mask);
+    }
+    free(h); free(t); free(lq); free(ltok); free(llq); free(llen);
+    free(ptok); free(ppar); free(pdep); free(next); free(olen); free(psc); free(olq);
+    return 0;
+}
+
+/* Sequential correction with heap (Sec. 4.1, Table 2): exact node-wise
+ * best-first search under the corrected scores.  The root's children are
+ * scored at r_0; each pop takes the best offer among the popped nodes (each
+ * offers its best child not yet taken, by its OWN corrected distribution),
+ * and the popped node, if above depth L, is then corrected: its state
+ * r(u_1..u_d) = g(r(u_<d), u_d) and its children's distribution
+ * q~_{d+1}(. | u_1..u_d) are computed before the next pop.  B pops; emitted in
+ * pop order.  expansions[s] receives the number of correction-head
+ * evaluations of children (the root included). */
+int orc_seq_heap(const orc_cfg *c, const void *Wi, const void *Wo, const void *E, const float *Dlog,
+                 const float *h0, int *o_tok, int *o_par, int *o_dep, int *o_pos, double *o_score, int *o_n,
+                 uint64_t *o_mask, int *expansions) {
+    const int V = c->V, d = c->d, L = c->L, B = c->B;
+    double *hs = (double *)malloc(sizeof(double) * (size_t)(B + 1) * d); /* row p+1: state of node p */
+    double *lq = (double *)malloc(sizeof(double) * (size_t)V);
+    int *ltok = (int *)malloc(sizeof(int) * (size_t)(B + 1) * B);
+    double *llq = (double *)malloc(sizeof(double) * (size_t)(B + 1) * B);
+    int *llen = (int *)malloc(sizeof(int) * (size_t)(B + 1));
+    int *next = (int *)malloc(sizeof(int) * (size_t)(B + 1));
+    int *ptok = (int *)malloc(sizeof(int) * (size_t)B), *ppar = (int *)malloc(sizeof(int) * (size_t)B);
+    int *pdep = (int *)malloc(sizeof(int) * (size_t)B);
+    double *psc = (double *)malloc(sizeof(double) * (size_t)B);
+    for (int s = 0; s < c->nseq; s++) {
+        const float *dl = Dlog + (size_t)s * L * V;
+        for (int j = 0; j < d; j++) hs[j] = (double)h0[(size_t)s * d + j];
+        child_logq_all(c, E, dl, hs, lq);
+        llen[0] = child_list(c, lq, ltok, llq);
+        next[0] = 0;
+        int n = 0, nexp = 1;
+        while (n < B) {
+            double v;
+            const int p = best_offer(c, n, pdep, psc, next, llen, llq, B, &v);
+            if (p == -2) break;
+            const int dep = p < 0 ? 1 : pdep[p] + 1;
+            const int tk = ltok[(size_t)(p + 1) * B + next[p + 1]];
+            ptok[n] = tk;
+            ppar[n] = p;
+            pdep[n] = dep;
+            psc[n] = v;
+            next[p + 1]++;
+            next[n + 1] = 0;
+            llen[n + 1] = 0;
+            if (dep < L) { /* correct the new prefix: its state, then its children */
+                double *hn = hs + (size_t)(n + 1) * d;
+                orc_head(c, Wi, Wo, E, hs + (size_t)(p + 1) * d, tk, hn);
+                child_logq_all(c, E, dl + (size_t)dep * V, hn, lq);
+                llen[n + 1] = child_list(c, lq, ltok + (size_t)(n + 1) * B, llq + (size_t)(n + 1) * B);
+                nexp++;
+            }
+            n++;
+        }
+        expansions[s] = nexp;
+        emit_pop_order(c, s, n, ptok, ppar, pdep, psc, o_tok, o_par, o_dep, o_pos, o_score, o_n, o_mask);
+    }
+    free(hs); free(lq); free(ltok); free(llq); free(llen); free(next);
+    free(ptok); free(ppar); free(pdep); free(psc);
+    return 0;
+}

@@ -6,6 +6,7 @@
   per-shard (max, sum exp, top-k) partials all-gathered and merged equal the
   unsharded log-softmax and top-k of the oracle.
 """
+import datetime
 import os
 import socket
 
@@ -29,7 +30,8 @@ def free_port():
 def _run(rank, world, port, fn, out_dir):
     os.environ["MASTER_ADDR"] = "127.0.0.1"
     os.environ["MASTER_PORT"] = str(port)
-    dist.init_process_group("gloo", rank=rank, world_size=world)
+    # a rank that fails ends the others' next collective within a minute
+    dist.init_process_group("gloo", rank=rank, world_size=world, timeout=datetime.timedelta(seconds=60))
     try:
         fn(rank, world, out_dir)
     finally:
@@ -38,6 +40,7 @@ def _run(rank, world, port, fn, out_dir):
 
 
 def spawn(fn, tmp_path, world=2):
+    oracle.build()  # once, before the ranks start
     mp.spawn(_run, args=(world, free_port(), fn, str(tmp_path)), nprocs=world, join=True)
 
 

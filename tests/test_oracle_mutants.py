@@ -77,6 +77,24 @@ MUTANTS = [
     ("candidate set: left in rank order instead of token order",
      "    qsort(cand, (size_t)c->cand_k, sizeof(int), int_cmp);\n",
      ""),
+    ("chain: the state advanced with depth 1's token at every depth",
+     "orc_head(c, Wi, Wo, E, h, y, t);",
+     "orc_head(c, Wi, Wo, E, h, ltok[0], t);"),
+    ("DDTree: a node's offers scored with its own depth's marginal",
+     "if (dep < L) memcpy(olq + (size_t)(n + 1) * B, llq + (size_t)dep * B, sizeof(double) * (size_t)B);",
+     "if (dep < L) memcpy(olq + (size_t)(n + 1) * B, llq + (size_t)(dep - 1) * B, sizeof(double) * (size_t)B);"),
+    ("sequential heap: children scored at the parent's state",
+     "child_logq_all(c, E, dl + (size_t)dep * V, hn, lq);",
+     "child_logq_all(c, E, dl + (size_t)dep * V, hs + (size_t)(p + 1) * d, lq);"),
+    ("sequential heap: children scored with the parent's drafter row",
+     "child_logq_all(c, E, dl + (size_t)dep * V, hn, lq);",
+     "child_logq_all(c, E, dl + (size_t)(dep - 1) * V, hn, lq);"),
+    ("best-first offers: depth bonus dropped",
+     "+ llq[(size_t)(p + 1) * lstride + next[p + 1]] + c->beta;",
+     "+ llq[(size_t)(p + 1) * lstride + next[p + 1]];"),
+    ("pop-order emission: mask row holds the node only",
+     "for (int a = i; a >= 0; a = par[a]) row[a / 64] |= 1ull << (a % 64);",
+     "row[i / 64] |= 1ull << (i % 64);"),
     ("teacher-forced state: every step from the first token",
      "    for (int i = 0; i < len; i++) {\n        orc_head(c, Wi, Wo, E, h, path[i], t);\n        memcpy(h, t, sizeof(double) * (size_t)d);\n    }\n    memcpy(h_out",
      "    for (int i = 0; i < len; i++) {\n        orc_head(c, Wi, Wo, E, h, path[0], t);\n        memcpy(h, t, sizeof(double) * (size_t)d);\n    }\n    memcpy(h_out"),

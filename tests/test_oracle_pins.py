@@ -564,3 +564,175 @@ def test_restricted_tree_structure():
         for i in range(r["n_nodes"][s]):
             dep = int(r["depths"][s, i])
             assert r["tokens"][s, i] in set(topK_candidates(x["Dlog"][s, dep - 1], cfg.cand_k).tolist())
+
+
+# ------------------------------------ the two constructions of Table 2
+
+def paths_of(r, s=0):
+    """{token path: score} of an emitted tree, and the paths in row order."""
+    out, order = {}, []
+    for i in range(int(r["n_nodes"][s])):
+        path, j = [], i
+        while j >= 0:
+            path.append(int(r["tokens"][s, j]))
+            j = int(r["parents"][s, j])
+        p = tuple(reversed(path))
+        out[p] = float(r["scores"][s, i])
+        order.append(p)
+    return out, order
+
+
+def check_pop_order_tree(cfg, r, s=0):
+    """Rows in pop order: parents precede children, scores never increase
+    along the rows (best-first), depths/positions/mask consistent, padding."""
+    n = int(r["n_nodes"][s])
+    for i in range(n):
+        p = int(r["parents"][s, i])
+        assert -1 <= p < i
+        assert r["depths"][s, i] == (1 if p < 0 else r["depths"][s, p] + 1)
+        assert r["pos_ids"][s, i] == cfg.pos_offset + r["depths"][s, i]
+        if i:
+            assert r["scores"][s, i] <= r["scores"][s, i - 1]
+        anc, j = set(), i
+        while j >= 0:
+            anc.add(j)
+            j = int(r["parents"][s, j])
+        row = r["mask"][s, i]
+        assert {b for b in range(cfg.B) if (int(row[b // 64]) >> (b % 64)) & 1} == anc
+    for i in range(n, cfg.B):
+        assert r["tokens"][s, i] == -1 and r["parents"][s, i] == -2 and not np.any(r["mask"][s, i])
+
+
+def torch_chain(cfg, x, s=0):
+    """The greedy corrected chain with the library head: per depth the
+    clamped log-softmax row, its argmax token and its log-sum-exp."""
+    head = TorchHead(cfg, x["Wi"], x["Wo"], x["E"])
+    h = torch.from_numpy(x["h0"][s].astype(np.float64))
+    Tp = cfg.temperature if cfg.temperature > 0 else 1.0
+    rows, toks, lses = [], [], []
+    K = int(getattr(cfg, "cand_k", 0))
+    for i in range(cfg.L):
+        if K > 0:
+            cand = topK_candidates(x["Dlog"][s, i], K)
+            lq = child_logq_restricted(cfg, head.E, x["Dlog"][s, i], h, cand)
+            z = (torch.from_numpy(x["Dlog"][s, i].astype(np.float64))[torch.from_numpy(cand)] +
+                 head.E[torch.from_numpy(cand)] @ h) / Tp
+        else:
+            lq = child_logq(cfg, head.E, x["Dlog"][s, i], h)
+            z = (torch.from_numpy(x["Dlog"][s, i].astype(np.float64)) + head.E @ h) / Tp
+        t = int(np.lexsort((np.arange(cfg.V), -lq.numpy()))[0])
+        rows.append(lq.numpy())
+        toks.append(t)
+        lses.append(float(torch.logsumexp(z, 0)))
+        h = head(h, t)
+    return rows, toks, lses
+
+
+@pytest.mark.parametrize("cand_k", [0, 4])
+def test_chain_is_the_greedy_corrected_chain(cand_k):
+    """Domino-chain + DDTree, step 1: the chain follows the argmax of the
+    corrected distribution of its own prefix (library head and softmax)."""
+    cfg = tiny(V=23, d=16, L=5, W=1, k=1, B=9, temperature=0.7, cand_k=cand_k)
+    x = rand_inputs(cfg)
+    r = oracle.chain_ddtree(cfg, x["Wi"], x["Wo"], x["E"], x["Dlog"], x["h0"])
+    _, toks, lses = torch_chain(cfg, x)
+    assert list(r["chain_tok"][0]) == toks
+    np.testing.assert_allclose(r["chain_lse"][0], lses, rtol=0, atol=1e-12)
+
+
+@pytest.mark.parametrize("beta", [0.0, -0.2])
+@pytest.mark.parametrize("B", [1, 7, 40])
+def test_chain_ddtree_bruteforce(beta, B):
+    """Domino-chain + DDTree = the top-B prefixes, over every token path, of
+    the sum of the chain-conditioned log-probabilities (+ beta d): exhaustive
+    enumeration on V = 5, L = 3, and the rows come out best first."""
+    cfg = tiny(V=5, d=8, L=3, W=1, k=1, B=B, beta=beta, temperature=1.3)
+    x = rand_inputs(cfg)
+    r = oracle.chain_ddtree(cfg, x["Wi"], x["Wo"], x["E"], x["Dlog"], x["h0"])
+    rows, _, _ = torch_chain(cfg, x)
+    every = {}
+    for n in range(1, cfg.L + 1):
+        for p in itertools.product(range(cfg.V), repeat=n):
+            every[p] = sum(rows[i][t] for i, t in enumerate(p)) + beta * n
+    want = sorted(every.items(), key=lambda kv: -kv[1])[:B]
+    got, _ = paths_of(r)
+    assert set(got) == {p for p, _ in want}
+    for p, sc in want:
+        assert abs(got[p] - sc) < 1e-12
+    check_pop_order_tree(cfg, r)
+
+
+@pytest.mark.parametrize("cand_k", [0, 12])
+def test_zero_E_chain_ddtree_and_seq_heap_are_ddtree(cand_k):
+    """E = 0: the correction is path independent, so both Table 2
+    constructions reduce to DDTree's best-first tree over the drafter's
+    marginals (renormalised over C_d when restricted), in the same pop order."""
+    cfg = tiny(V=40, d=16, L=5, W=1, k=1, B=25, beta=-0.2, cand_k=cand_k)
+    x = rand_inputs(cfg)
+    x["E"] = np.zeros_like(x["E"])
+    rows = []
+    for i in range(cfg.L):
+        z = torch.from_numpy(x["Dlog"][0, i].astype(np.float64))
+        if cand_k:
+            cand = topK_candidates(x["Dlog"][0, i], cand_k)
+            row = np.full(cfg.V, -np.inf)
+            row[cand] = torch.log_softmax(z[torch.from_numpy(cand)], 0).numpy()
+        else:
+            row = torch.log_softmax(z, 0).numpy()
+        rows.append(row + cfg.beta)
+    want = ddtree_topB(rows, cfg.B)
+    for fn in (oracle.chain_ddtree, oracle.seq_heap):
+        r = fn(cfg, x["Wi"], x["Wo"], x["E"], x["Dlog"], x["h0"])
+        got, order = paths_of(r)
+        assert order == [p for p, _ in want]
+        for p, sc in want:
+            assert abs(got[p] - sc) < 1e-12
+        check_pop_order_tree(cfg, r)
+
+
+@pytest.mark.parametrize("beta,temperature", [(0.0, 0.0), (-0.2, 1.0), (-1.5, 0.6)])
+def test_seq_heap_bruteforce(beta, temperature):
+    """Sequential correction with heap = exact best-first under the corrected
+    scores = the top-B of every token path by its Eq. 5 score, each path
+    scored from the root on its own (library head), V = 5, L = 3."""
+    cfg = tiny(V=5, d=8, L=3, W=1, k=1, B=30, beta=beta, temperature=temperature)
+    x = rand_inputs(cfg)
+    every = all_path_scores(cfg, x["Wi"], x["Wo"], x["E"], x["Dlog"][0], x["h0"][0], cfg.L)
+    r = oracle.seq_heap(cfg, x["Wi"], x["Wo"], x["E"], x["Dlog"], x["h0"])
+    want = sorted(every.items(), key=lambda kv: -kv[1])[:cfg.B]
+    got, _ = paths_of(r)
+    assert set(got) == {p for p, _ in want}
+    for p, sc in want:
+        assert abs(got[p] - sc) < 1e-12
+    check_pop_order_tree(cfg, r)
+    # one corrected distribution per popped prefix above depth L, and the root's
+    n_inner = int(np.sum((r["depths"][0, :r["n_nodes"][0]] < cfg.L) & (r["depths"][0, :r["n_nodes"][0]] > 0)))
+    assert r["expansions"][0] == 1 + n_inner
+
+
+def test_seq_heap_restricted_bruteforce():
+    cfg = tiny(V=7, d=8, L=3, W=1, k=1, B=20, cand_k=3, temperature=0.9)
+    x = rand_inputs(cfg)
+    every = all_path_scores(cfg, x["Wi"], x["Wo"], x["E"], x["Dlog"][0], x["h0"][0], cfg.L)
+    r = oracle.seq_heap(cfg, x["Wi"], x["Wo"], x["E"], x["Dlog"], x["h0"])
+    want = sorted(every.items(), key=lambda kv: -kv[1])[:cfg.B]
+    got, _ = paths_of(r)
+    assert set(got) == {p for p, _ in want}
+    for p, sc in want:
+        assert abs(got[p] - sc) < 1e-12
+
+
+def test_seq_heap_equals_dartree_with_a_full_beam():
+    """With a beam wide enough to hold every prefix (W = V^(L-1), k = V),
+    Algorithm 1's supertree is the whole prefix tree and, by Lemma 1, its
+    top-B pruning is the exact best-first tree of the sequential heap."""
+    cfg = tiny(V=4, d=8, L=4, W=64, k=4, B=50, nseq=2, beta=-0.3, temperature=0.8)
+    x = rand_inputs(cfg)
+    a = run(cfg, x)
+    b = oracle.seq_heap(cfg, x["Wi"], x["Wo"], x["E"], x["Dlog"], x["h0"])
+    for s in range(cfg.nseq):
+        pa, _ = paths_of(a, s)
+        pb, _ = paths_of(b, s)
+        assert set(pa) == set(pb)
+        for p in pa:
+            assert abs(pa[p] - pb[p]) < 1e-12
