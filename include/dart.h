@@ -104,7 +104,10 @@ enum {
  *                      stream beside the selection of the children; AUTO = ON
  *   lmhead_ctas_per_sm 1 or 2 LM-head CTAs per SM; 0 = by d (2 if d <= 3072
  *                      and both fit, else 1)
- *   variants           bit set of DART_VARIANT_* (0: Algorithm 1 only) */
+ *   variants           bit set of DART_VARIANT_* (0: Algorithm 1 only); the
+ *                      variants need cand_k = 0 and nseq <= 64, and the
+ *                      chain's search keeps L * min(B, V) scores and tokens in
+ *                      shared memory (DART_ERR_UNSUPPORTED beyond 227 KB) */
 typedef struct {
     int V, d, L, W, k, B, nseq;
     float beta, temperature, rms_eps;
@@ -171,6 +174,52 @@ int dart_prune_and_emit(dart_handle *h, const dart_tree_out *out, void *stream);
 int dart_build_tree(dart_handle *h, const float *drafter_logits, const float *anchor_h,
                     const dart_tree_out *out, void *stream);
 
+/* DARTree (fixed), the paper's first variant (Sec. 5.1): the supertree of
+ * Algorithm 1 is itself the verification tree -- every retained node is
+ * emitted, nothing is pruned (the paper's setting: W = 4 per depth, 64 nodes
+ * over 16 depths).  Requires B >= sum_d |S_d| (at most L*W; else
+ * DART_ERR_INVALID); otherwise as dart_build_tree, whose top-B then keeps
+ * every node. */
+int dart_build_tree_fixed(dart_handle *h, const float *drafter_logits, const float *anchor_h,
+                          const dart_tree_out *out, void *stream);
+
+/* Domino-chain + DDTree, the first alternative construction of Table 2
+ * (Sec. 5.2): causal correction along ONE draft chain -- from r_0, at each
+ * depth d the chain prefix's corrected distribution q~_d(. | y_<d) (full
+ * vocabulary), its argmax y_d (log q~ desc, token asc) continuing the chain
+ * -- then DDTree (Sec. 3.3) over those chain-conditioned distributions used
+ * as position-wise marginals: best-first search over prefixes scored
+ * s = sum_i log q~_i(u_i) + beta d (beta = 0 is DDTree's mass objective),
+ * B pops.  Each pop takes the best "offer" -- every popped node (and the
+ * root) offers its best child not yet taken -- by (score desc, popped node
+ * asc, the root first).  The emitted rows are in pop order (parents first,
+ * scores non-increasing); parents/depths/pos_ids/mask as for dart_build_tree.
+ * Needs a handle made with DART_VARIANT_CHAIN_DDTREE in cfg.variants
+ * (else DART_ERR_STATE).  Cost: L LM-head passes of one node per sequence,
+ * the chain's L-1 head updates, a top-min(B, V) selection per depth and the
+ * search.  Cached as a CUDA graph like dart_build_tree. */
+int dart_build_chain_ddtree(dart_handle *h, const float *drafter_logits, const float *anchor_h,
+                            const dart_tree_out *out, void *stream);
+
+/* Sequential correction with heap, the second alternative construction of
+ * Table 2 (Sec. 4.1): exact node-wise best-first search under the corrected
+ * scores.  The root's children are scored at r_0; each of the B pops takes
+ * the best offer as above -- but every node offers children from its OWN
+ * corrected distribution -- and the popped prefix is then corrected before
+ * the next pop: its state r(u_1..u_d) = g(r(u_<d), u_d) and the distribution
+ * of its children q~_{d+1}(. | u_1..u_d) over the vocabulary (none at depth
+ * L).  For beta <= 0 the result is the top-B of ALL prefixes by Eq. 5.
+ * Emitted in pop order.  Needs DART_VARIANT_SEQ_HEAP in cfg.variants (else
+ * DART_ERR_STATE).  Cost: up to B LM-head passes of one node per sequence,
+ * one after another.  Cached as a CUDA graph like dart_build_tree. */
+int dart_build_seq_heap(dart_handle *h, const float *drafter_logits, const float *anchor_h,
+                        const dart_tree_out *out, void *stream);
+
+/* Test hook after dart_build_chain_ddtree: the chain y [nseq][L] (int32)
+ * and the log-sum-exp of each of its scaled-logit rows lse [nseq][L]
+ * (float).  NULL outputs are skipped; DART_ERR_STATE after any other round. */
+int dart_get_chain(dart_handle *h, int32_t *tok, float *lse, void *stream);
+
 /* dart_build_tree on HOST buffers: copies drafter_logits_host [nseq][L][V]
  * and anchor_host [nseq][d] to handle-owned device staging, builds the tree
  * and copies it back into the host arrays of out_host (same layout as
@@ -227,8 +276,10 @@ int dart_profile_read(dart_handle *h, float *lmhead_ms, int *lmhead_launches);
  * 7 depth-1 anchor preparation, 8 prune + emit, 9 candidate sets C_d
  * (cand_k > 0, once per round), 10 candidate scoring (cand_k > 0, per
  * depth), 11 gather of the per-token table row + SiLU + split (split first
- * layer).  ms[i] / launches[i] receive the summed device time and count of
- * kind i for i < nkinds (nkinds <= 12); resets the events. */
+ * layer), 12 top-K by value over a row of scaled logits (the best-first
+ * constructions), 13 DDTree search, 14 one pop of the sequential search,
+ * 15 its emission.  ms[i] / launches[i] receive the summed device time and
+ * count of kind i for i < nkinds (nkinds <= 16); resets the events. */
 int dart_profile_read_kinds(dart_handle *h, float *ms, int *launches, int nkinds);
 
 /* Number of kernel launches one dart_build_tree enqueues for this handle. */

@@ -18,7 +18,7 @@ LIB = os.path.join(HERE, "libdart.so")
 BUILD_DIR = os.path.join(HERE, "_build")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 SOURCES = ["dart_abi.cu", "dart_tc.cu", "dart_f32.cu", "dart_select.cu", "dart_noalloc.cu", "dart_cand.cu",
-           "dart_attn.cu"]
+           "dart_attn.cu", "dart_heap.cu"]
 
 
 def _nvcc() -> str:

@@ -78,8 +78,11 @@ struct DepthPlan {
     int g1_smem, g2_smem;
 };
 
+// Round graph cache key: the construction (kind) and the pointer set.
+enum RoundKind { kRoundDartree = 0, kRoundChainDdtree = 1, kRoundSeqHeap = 2 };
+
 struct GraphEntry {
-    const void* key[9];
+    const void* key[10];
     cudaGraphExec_t exec;
     unsigned long long last_use;
 };
@@ -115,6 +118,31 @@ struct dart_handle {
     uint64_t* cand_part;  // [nseq * L][slices][cand_k] per-slice top keys of the candidate selection
     int* cand_rticket;    // [nseq * L] slices finished per row
     float* Qtab;          // [V][d] fp32: Q[t] = W_i[:, d:2d] . E[t] (split first head layer), or null
+    // best-first constructions (dart_config.variants): the one-node-per-
+    // sequence plans (W = k = 1) of the chain and of the sequential search
+    dart_config ccfg;
+    std::vector<int> ccaps;
+    std::vector<DepthPlan> cplans;
+    int Bp;                // children kept per distribution: min(B, V)
+    int ddt_S, sh_S;       // top-K slices per row (chain rows, popped-prefix rows)
+    // Domino-chain + DDTree
+    float* zrows;          // [nseq][L][V] the chain's scaled logits
+    float* chain_lse;      // [nseq][L]
+    int* ddt_tok;          // [nseq][L][Bp]
+    float* ddt_z;
+    uint64_t* ddt_part;    // [nseq * L][topk_S][Bp]
+    int* ddt_ticket;       // [nseq * L]
+    // sequential correction with heap (slot 0 = the root, p + 1 = node p)
+    float* sh_tab;         // [nseq][B+1][d]
+    int* sh_ltok;          // [nseq][B+1][Bp]
+    float* sh_lz;
+    float* sh_llse;        // [nseq][B+1]
+    int *sh_next, *sh_npop, *sh_dlog_row;
+    float* sh_offer;
+    float* sh_zrow;        // [nseq][V]
+    uint64_t* sh_part;     // [nseq][topk_S][Bp]
+    int* sh_ticket;        // [nseq]
+    int last_kind;         // construction of the most recent round (RoundKind)
     std::vector<void*> allocs;
     CUtensorMap tmE, tmWi, tmWo, tmH[4], tmX[3], tmA[3];
     CUtensorMap tmWiR, tmEB;  // Q table: A = W_i[:, d:2d] (128-row box), B = E rows as 64-node groups
@@ -209,16 +237,17 @@ int tc_stages(int smem_optin, int stage_bytes, int fixed) {
     return std::min(16, s);
 }
 
-int build_plans(dart_handle* h) {
-    const dart_config& c = h->cfg;
+// Launch plans of every depth for configuration c (the handle's, or the
+// one-node-per-sequence configuration of the best-first constructions).
+int build_plans(dart_handle* h, const dart_config& c, std::vector<int>& caps, std::vector<DepthPlan>& plans) {
     const bool tc = h->wdtype == DART_BF16;
-    h->caps.assign(c.L + 1, 1);
-    for (int i = 1; i <= c.L; i++) h->caps[i] = std::min(c.W, h->caps[i - 1] * c.k);
-    h->plans.resize(c.L + 1);
+    caps.assign(c.L + 1, 1);
+    for (int i = 1; i <= c.L; i++) caps[i] = std::min(c.W, caps[i - 1] * c.k);
+    plans.resize(c.L + 1);
     const int tiles = (c.V + kTileM - 1) / kTileM;
     for (int dep = 1; dep <= c.L; dep++) {
-        DepthPlan& p = h->plans[dep];
-        p.P = h->caps[dep - 1];
+        DepthPlan& p = plans[dep];
+        p.P = caps[dep - 1];
         p.N = c.nseq * p.P;
         if (tc) {
             LmheadPlan lp;
@@ -256,7 +285,7 @@ int build_plans(dart_handle* h) {
             p.cand_ds = cand_score_slices(p.P, c.d, c.nseq, c.cand_k, h->smem_optin);
             if (p.cand_ds == 0) return DART_ERR_UNSUPPORTED;
         }
-        p.Pn = h->caps[dep];
+        p.Pn = caps[dep];
         p.Nc = c.nseq * p.Pn;
         p.split = p.side = 0;
         if (dep < c.L) {
@@ -346,11 +375,12 @@ int build_plans(dart_handle* h) {
 
 size_t max_part_floats(const dart_handle* h) {
     size_t m = 1;
-    for (int dep = 1; dep < h->cfg.L; dep++) {
-        const DepthPlan& p = h->plans[dep];
-        m = std::max(m, static_cast<size_t>(p.g1.S) * p.Nc * h->cfg.d);
-        m = std::max(m, static_cast<size_t>(p.g2.S) * p.Nc * h->cfg.d);
-    }
+    for (const std::vector<DepthPlan>* ps : {&h->plans, &h->cplans})
+        for (int dep = 1; dep + 1 < static_cast<int>(ps->size()); dep++) {
+            const DepthPlan& p = (*ps)[dep];
+            m = std::max(m, static_cast<size_t>(p.g1.S) * std::max(p.N, p.Nc) * h->cfg.d);
+            m = std::max(m, static_cast<size_t>(p.g2.S) * p.Nc * h->cfg.d);
+        }
     return m;
 }
 
@@ -359,11 +389,12 @@ int alloc_workspace(dart_handle* h) {
     const size_t d = c.d;
     int rc = DART_OK;
     size_t max_nvn = 1, max_keys = 1;  // key lists x nodes; keys incl. one padding key per node
-    for (int dep = 1; dep <= c.L; dep++) {
-        const DepthPlan& p = h->plans[dep];
-        max_nvn = std::max(max_nvn, static_cast<size_t>(p.nlist) * p.N);
-        max_keys = std::max(max_keys, (static_cast<size_t>(p.nlist) * p.klist + 1) * p.N);
-    }
+    for (const std::vector<DepthPlan>* ps : {&h->plans, &h->cplans})
+        for (int dep = 1; dep < static_cast<int>(ps->size()); dep++) {
+            const DepthPlan& p = (*ps)[dep];
+            max_nvn = std::max(max_nvn, static_cast<size_t>(p.nlist) * p.N);
+            max_keys = std::max(max_keys, (static_cast<size_t>(p.nlist) * p.klist + 1) * p.N);
+        }
     const size_t super = static_cast<size_t>(c.nseq) * c.L * c.W;
 #define DART_ALLOC(ptr, n) \
     if (rc == DART_OK) rc = dalloc(h, &(ptr), (n));
@@ -395,6 +426,28 @@ int alloc_workspace(dart_handle* h) {
     bool any_split = false;
     for (int dep = 1; dep < c.L; dep++) any_split = any_split || h->plans[dep].split;
     if (any_split) DART_ALLOC(h->Qtab, static_cast<size_t>(c.V) * d)
+    const size_t ns = c.nseq, Bp = h->Bp, S1 = static_cast<size_t>(c.B) + 1;
+    if (c.variants & DART_VARIANT_CHAIN_DDTREE) {
+        DART_ALLOC(h->zrows, ns * c.L * c.V)
+        DART_ALLOC(h->chain_lse, ns * c.L)
+        DART_ALLOC(h->ddt_tok, ns * c.L * Bp)
+        DART_ALLOC(h->ddt_z, ns * c.L * Bp)
+        DART_ALLOC(h->ddt_part, ns * c.L * h->ddt_S * Bp)
+        DART_ALLOC(h->ddt_ticket, ns * c.L)
+    }
+    if (c.variants & DART_VARIANT_SEQ_HEAP) {
+        DART_ALLOC(h->sh_tab, ns * S1 * d)
+        DART_ALLOC(h->sh_ltok, ns * S1 * Bp)
+        DART_ALLOC(h->sh_lz, ns * S1 * Bp)
+        DART_ALLOC(h->sh_llse, ns * S1)
+        DART_ALLOC(h->sh_next, ns * S1)
+        DART_ALLOC(h->sh_offer, ns * S1)
+        DART_ALLOC(h->sh_npop, ns)
+        DART_ALLOC(h->sh_dlog_row, ns)
+        DART_ALLOC(h->sh_zrow, ns * c.V)
+        DART_ALLOC(h->sh_part, ns * h->sh_S * Bp)
+        DART_ALLOC(h->sh_ticket, ns)
+    }
     if (c.cand_k > 0) {
         size_t scr = 1;
         for (int dep = 1; dep <= c.L; dep++)
@@ -422,6 +475,8 @@ int alloc_workspace(dart_handle* h) {
     if (cudaMemset(h->seq_ticket, 0, c.nseq * sizeof(int)) != cudaSuccess) return DART_ERR_CUDA;
     if (cudaMemset(h->status, 0, sizeof(int)) != cudaSuccess) return DART_ERR_CUDA;
     if (cudaMemset(h->tree_count, 0, c.nseq * c.L * sizeof(int)) != cudaSuccess) return DART_ERR_CUDA;
+    if (h->ddt_ticket && cudaMemset(h->ddt_ticket, 0, ns * c.L * sizeof(int)) != cudaSuccess) return DART_ERR_CUDA;
+    if (h->sh_ticket && cudaMemset(h->sh_ticket, 0, ns * sizeof(int)) != cudaSuccess) return DART_ERR_CUDA;
     // one-time kernel attributes
     int max_sel = 0;
     for (int dep = 1; dep <= c.L; dep++)
@@ -436,6 +491,19 @@ int alloc_workspace(dart_handle* h) {
             cudaMemset(h->cand_rticket, 0, static_cast<size_t>(c.nseq) * c.L * sizeof(int)) != cudaSuccess)
             return DART_ERR_CUDA;
         if (cand_set_smem_limits(std::max(cand_topk_smem(c.cand_k), 48 * 1024), score_smem) != cudaSuccess)
+            return DART_ERR_CUDA;
+    }
+    if (c.variants) {
+        // top-K by value over V (the chain's rows, a popped prefix's row); the
+        // candidate top-K of cand_k > 0 shares the kernel: keep the larger limit
+        const int topk = std::max({cand_topk_smem(h->Bp), c.cand_k > 0 ? cand_topk_smem(c.cand_k) : 0, 48 * 1024});
+        int score_smem = 48 * 1024;
+        if (c.cand_k > 0)
+            for (int dep = 1; dep <= c.L; dep++)
+                score_smem = std::max(score_smem, cand_score_smem(h->plans[dep].P, c.d, h->plans[dep].cand_ds));
+        if (cand_set_smem_limits(topk, score_smem) != cudaSuccess) return DART_ERR_CUDA;
+        if ((c.variants & DART_VARIANT_CHAIN_DDTREE) &&
+            heap_set_smem_limits(std::max(ddtree_smem(c.L, h->Bp, c.B), 48 * 1024)) != cudaSuccess)
             return DART_ERR_CUDA;
     }
     if (h->wdtype == DART_BF16) {
@@ -516,7 +584,7 @@ void release(dart_handle* h) {
 
 enum Kind {
     kLmhead = 0, kSelect, kGather, kGemm1, kSilu, kGemm2, kNorm, kPrep, kEmit, kCandTopk, kCandScore, kGatherSilu,
-    kNumKinds
+    kRowTopk, kDdtree, kSeqStep, kSeqEmit, kNumKinds
 };
 
 // Opens an event pair around the next launch when profiling (no-op otherwise).
@@ -539,9 +607,84 @@ void prof_end(dart_handle* h, int i, cudaStream_t st) {
     h->ev_used = i + 2;
 }
 
-int enqueue_depth(dart_handle* h, int dep, const float* dlog, const float* anchor, cudaStream_t st) {
-    const dart_config& c = h->cfg;
-    const DepthPlan& p = h->plans[dep];
+// LM-head launch arguments of plan p (drafter row and cross-CTA bounds are
+// set by the caller); h32: the nodes' fp32 states (fp32 weights).
+LmheadArgs lmhead_args(const dart_handle* h, const dart_config& c, const DepthPlan& p, const float* dlog,
+                       const float* h32) {
+    LmheadArgs la;
+    std::memset(&la, 0, sizeof la);
+    la.V = c.V;
+    la.d = c.d;
+    la.N = p.N;
+    la.NG = p.NG;
+    la.G = p.G;
+    la.nV = p.nV;
+    la.k = c.k;
+    la.tiles = (c.V + kTileM - 1) / kTileM;
+    la.P = p.P;
+    la.invT = c.temperature > 0.0f ? 1.0f / c.temperature : 1.0f;
+    la.dlog = dlog;
+    la.dlog_seq_stride = static_cast<long long>(c.L) * c.V;
+    la.bhalf = kNPadMax;
+    la.stages = p.stages;
+    la.l2pf = p.l2pf;
+    la.part_ms = h->part_ms;
+    la.part_key = h->part_key;
+    la.status = h->status;
+    la.h32 = h32;
+    la.E32 = static_cast<const float*>(h->E);
+    return la;
+}
+
+// Merge + frontier-selection launch arguments of plan p at depth dep.
+SelectArgs select_args(const dart_handle* h, const dart_config& c, const DepthPlan& p, int dep) {
+    SelectArgs sa;
+    std::memset(&sa, 0, sizeof sa);
+    sa.N = p.N;
+    sa.P = p.P;
+    sa.k = c.k;
+    sa.nV = p.nlist;
+    sa.klist = p.klist;
+    sa.W = c.W;
+    sa.L = c.L;
+    sa.nseq = c.nseq;
+    sa.dep = dep;
+    sa.Pn = p.Pn;
+    sa.beta = c.beta;
+    sa.part_ms = h->part_ms;
+    sa.part_key = h->part_key;
+    sa.node_logq = h->node_logq;
+    sa.node_tok = h->node_tok;
+    sa.node_lse = h->node_lse;
+    sa.tree_tok = h->tree_tok;
+    sa.tree_parent = h->tree_parent;
+    sa.tree_score = h->tree_score;
+    sa.tree_count = h->tree_count;
+    sa.child_prow = h->child_prow;
+    sa.child_tok = h->child_tok;
+    sa.seq_ticket = h->seq_ticket;
+    sa.status = h->status;
+    return sa;
+}
+
+// Optional outputs of one depth (the chain of Domino-chain + DDTree): every
+// node's scaled logits z[n][v] -> zout[n * zout_stride + v], and its
+// log-sum-exp -> lse_hist[n * lse_hist_stride].
+struct DepthOutputs {
+    float* zout;
+    long long zout_stride;
+    float* lse_hist;
+    long long lse_hist_stride;
+};
+
+int enqueue_head_update(dart_handle* h, const dart_config& c, const DepthPlan& p, const float* hcur, float* hnext,
+                        bool g1_launched, cudaStream_t st);
+
+// Algorithm 1, one iteration, for configuration c with plans `plans` (the
+// handle's, or the one-node-per-sequence chain's).
+int enqueue_depth(dart_handle* h, const dart_config& c, const std::vector<DepthPlan>& plans, int dep,
+                  const float* dlog, const float* anchor, cudaStream_t st, const DepthOutputs* outs = nullptr) {
+    const DepthPlan& p = plans[dep];
     const bool tc = h->wdtype == DART_BF16;
     cudaError_t e = cudaSuccess;
     if (dep == 1) {
@@ -562,30 +705,13 @@ int enqueue_depth(dart_handle* h, int dep, const float* dlog, const float* ancho
         }
     }
     // 1) LM-head scoring of every prefix in S_{dep-1} (fused log-sum-exp / top-k)
-    LmheadArgs la;
-    std::memset(&la, 0, sizeof la);
-    la.V = c.V;
-    la.d = c.d;
-    la.N = p.N;
-    la.NG = p.NG;
-    la.G = p.G;
-    la.nV = p.nV;
-    la.k = c.k;
-    la.tiles = (c.V + kTileM - 1) / kTileM;
-    la.P = p.P;
-    la.invT = c.temperature > 0.0f ? 1.0f / c.temperature : 1.0f;
-    la.dlog = dlog;
-    la.dlog_seq_stride = static_cast<long long>(c.L) * c.V;
+    LmheadArgs la = lmhead_args(h, c, p, dlog, h->hbuf[h->cur]);
     la.dlog_row_off = static_cast<long long>(dep - 1) * c.V;
-    la.bhalf = kNPadMax;
-    la.stages = p.stages;
-    la.l2pf = p.l2pf;
-    la.part_ms = h->part_ms;
-    la.part_key = h->part_key;
-    la.status = h->status;
-    la.h32 = h->hbuf[h->cur];
-    la.E32 = static_cast<const float*>(h->E);
     la.gthr = h->gthr + static_cast<size_t>(dep - 1) * kNPadMax;
+    if (outs) {
+        la.zout = outs->zout;
+        la.zout_stride = outs->zout_stride;
+    }
     int pi;
     if (c.cand_k > 0) {
         // candidate-restricted scoring: every node against its sequence's C_d
@@ -637,33 +763,12 @@ int enqueue_depth(dart_handle* h, int dep, const float* dlog, const float* ancho
         if (e != cudaSuccess || cudaEventRecord(h->ev_join, h->side) != cudaSuccess) return DART_ERR_CUDA;
     }
     // 2) merge partials, log q~, Eq. 5 scores, global top-W -> S_dep
-    SelectArgs sa;
-    std::memset(&sa, 0, sizeof sa);
-    sa.N = p.N;
-    sa.P = p.P;
-    sa.k = c.k;
-    sa.nV = p.nlist;
-    sa.klist = p.klist;
-    sa.W = c.W;
-    sa.L = c.L;
-    sa.nseq = c.nseq;
-    sa.dep = dep;
-    sa.Pn = p.Pn;
-    sa.beta = c.beta;
-    sa.part_ms = h->part_ms;
-    sa.part_key = h->part_key;
+    SelectArgs sa = select_args(h, c, p, dep);
     sa.gthr = c.cand_k > 0 ? nullptr : la.gthr;
-    sa.node_logq = h->node_logq;
-    sa.node_tok = h->node_tok;
-    sa.node_lse = h->node_lse;
-    sa.tree_tok = h->tree_tok;
-    sa.tree_parent = h->tree_parent;
-    sa.tree_score = h->tree_score;
-    sa.tree_count = h->tree_count;
-    sa.child_prow = h->child_prow;
-    sa.child_tok = h->child_tok;
-    sa.seq_ticket = h->seq_ticket;
-    sa.status = h->status;
+    if (outs) {
+        sa.lse_hist = outs->lse_hist;
+        sa.lse_hist_stride = outs->lse_hist_stride;
+    }
     pi = prof_begin(h, kSelect, st);
     e = launch_merge_select(sa, st);
     prof_end(h, pi, st);
@@ -671,8 +776,24 @@ int enqueue_depth(dart_handle* h, int dep, const float* dlog, const float* ancho
     h->last_rows = p.N;
     if (dep == c.L) return DART_OK;
     // 3) correction-head update of the retained children (Algorithm 1, state update)
-    const float* hcur = h->hbuf[h->cur];
-    float* hnext = h->hbuf[1 - h->cur];
+    const int rc = enqueue_head_update(h, c, p, h->hbuf[h->cur], h->hbuf[1 - h->cur], p.side != 0, st);
+    if (rc != DART_OK) return rc;
+    h->cur = 1 - h->cur;
+    h->last_rows = p.Nc;
+    return DART_OK;
+}
+
+// Correction-head update of the children listed in child_prow / child_tok
+// (Algorithm 1, "update their states"): hnext[c] = RMSNorm(hcur[prow[c]] +
+// W_o SiLU(W_i [hcur[prow[c]] ; E[tok[c]]])), with the hi/lo bf16 split of
+// the result in HL.  With the split first layer the W_i[:, 0:d] GEMM reads
+// the parents' hi/lo rows in HL; g1_launched: it already runs on the side
+// stream (joined here).
+int enqueue_head_update(dart_handle* h, const dart_config& c, const DepthPlan& p, const float* hcur, float* hnext,
+                        bool g1_launched, cudaStream_t st) {
+    const bool tc = h->wdtype == DART_BF16;
+    cudaError_t e = cudaSuccess;
+    int pi;
     if (!p.split) {
         pi = prof_begin(h, kGather, st);
         e = launch_gather_x(p.Nc, c.d, h->child_prow, h->child_tok, hcur, h->E, tc ? 1 : 0, h->XL, kNPadMax, h->X32,
@@ -685,7 +806,7 @@ int enqueue_depth(dart_handle* h, int dep, const float* dlog, const float* ancho
     g1.outL = h->AL;
     g2.out = h->part;
     g1.status = g2.status = h->status;
-    if (!p.side) {  // (on the side stream it was launched after the LM-head)
+    if (!g1_launched) {  // (on the side stream it was launched after the LM-head)
         pi = prof_begin(h, kGemm1, st);
         if (p.split) {
             e = launch_gemm_tc(&h->tmWi, &h->tmH[ng_index(g1.NG)], g1, p.g1_smem, st);
@@ -701,7 +822,7 @@ int enqueue_depth(dart_handle* h, int dep, const float* dlog, const float* ancho
     }
     const bool fused = tc && g1.mode != kGemmPartials;  // SiLU applied in the GEMM's cluster reduction
     if (p.split) {
-        if (p.side && cudaStreamWaitEvent(st, h->ev_join, 0) != cudaSuccess) return DART_ERR_CUDA;
+        if (g1_launched && cudaStreamWaitEvent(st, h->ev_join, 0) != cudaSuccess) return DART_ERR_CUDA;
         pi = prof_begin(h, kGatherSilu, st);
         // (a cluster GEMM wrote the summed U: one "split")
         e = launch_gather_silu(p.Nc, c.d, g1.mode == kGemmPartials ? g1.S : 1, g1.N, h->part, h->child_prow,
@@ -729,10 +850,7 @@ int enqueue_depth(dart_handle* h, int dep, const float* dlog, const float* ancho
     e = launch_residual_norm(p.Nc, c.d, s2, h->part, h->child_prow, hcur, c.rms_eps, hnext, tc ? h->HL : nullptr,
                              kNPadMax, st);
     prof_end(h, pi, st);
-    if (e != cudaSuccess) return DART_ERR_CUDA;
-    h->cur = 1 - h->cur;
-    h->last_rows = p.Nc;
-    return DART_OK;
+    return e == cudaSuccess ? DART_OK : DART_ERR_CUDA;
 }
 
 int check_out(const dart_tree_out* o) {
@@ -772,11 +890,149 @@ int enqueue_emit(dart_handle* h, const dart_tree_out* o, cudaStream_t st) {
 
 int enqueue_round(dart_handle* h, const float* dlog, const float* anchor, const dart_tree_out* out, cudaStream_t st) {
     for (int dep = 1; dep <= h->cfg.L; dep++) {
-        int rc = enqueue_depth(h, dep, dlog, anchor, st);
+        int rc = enqueue_depth(h, h->cfg, h->plans, dep, dlog, anchor, st);
         if (rc != DART_OK) return rc;
     }
     h->next_depth = h->cfg.L + 1;
     return enqueue_emit(h, out, st);
+}
+
+// Domino-chain + DDTree (Table 2): the chain is Algorithm 1 with W = k = 1
+// (one node per sequence and depth: its argmax child continues the chain),
+// which also keeps every depth's scaled logits and log-sum-exp; then the
+// chain's best Bp = min(B, V) children of every depth, best first, and
+// DDTree's best-first search over those position-wise distributions.
+int enqueue_chain_ddtree(dart_handle* h, const float* dlog, const float* anchor, const dart_tree_out* out,
+                         cudaStream_t st) {
+    const dart_config& c = h->cfg;
+    for (int dep = 1; dep <= c.L; dep++) {
+        DepthOutputs o;
+        o.zout = h->zrows + static_cast<size_t>(dep - 1) * c.V;
+        o.zout_stride = static_cast<long long>(c.L) * c.V;
+        o.lse_hist = h->chain_lse + (dep - 1);
+        o.lse_hist_stride = c.L;
+        const int rc = enqueue_depth(h, h->ccfg, h->cplans, dep, dlog, anchor, st, &o);
+        if (rc != DART_OK) return rc;
+    }
+    int pi = prof_begin(h, kRowTopk, st);
+    cudaError_t e = launch_row_topk_by_value(h->zrows, c.nseq * c.L, c.V, h->Bp, h->ddt_S, h->ddt_tok, h->ddt_z,
+                                             h->Bp, h->ddt_part, h->ddt_ticket, st);
+    prof_end(h, pi, st);
+    if (e != cudaSuccess) return DART_ERR_CUDA;
+    DdtArgs a;
+    std::memset(&a, 0, sizeof a);
+    a.L = c.L;
+    a.B = c.B;
+    a.Bp = h->Bp;
+    a.nseq = c.nseq;
+    a.pos_offset = c.pos_offset;
+    a.beta = c.beta;
+    a.tok = h->ddt_tok;
+    a.zval = h->ddt_z;
+    a.lse = h->chain_lse;
+    a.tokens = out->tokens;
+    a.parents = out->parents;
+    a.depths = out->depths;
+    a.pos_ids = out->pos_ids;
+    a.n_nodes = out->n_nodes;
+    a.scores = out->scores;
+    a.mask = out->mask;
+    pi = prof_begin(h, kDdtree, st);
+    e = launch_ddtree(a, st);
+    prof_end(h, pi, st);
+    return e == cudaSuccess ? DART_OK : DART_ERR_CUDA;
+}
+
+// Sequential correction with heap (Sec. 4.1, Table 2): B pops, each
+// correcting the popped prefix before the next: its state (head update of
+// one node per sequence) and its children over the vocabulary (LM-head,
+// merge for the log-sum-exp, the best Bp children best first).  The last pop
+// needs no correction, nor does any pop when L = 1.
+int enqueue_seq_heap(dart_handle* h, const float* dlog, const float* anchor, const dart_tree_out* out,
+                     cudaStream_t st) {
+    const dart_config& c = h->cfg;
+    const dart_config& cc = h->ccfg;
+    const DepthPlan& p = h->cplans[1];  // one node per sequence
+    const bool tc = h->wdtype == DART_BF16;
+    const size_t S1 = static_cast<size_t>(c.B) + 1;
+    SeqHeapArgs a;
+    std::memset(&a, 0, sizeof a);
+    a.L = c.L;
+    a.B = c.B;
+    a.Bp = h->Bp;
+    a.nseq = c.nseq;
+    a.d = c.d;
+    a.pos_offset = c.pos_offset;
+    a.bhalf = kNPadMax;
+    a.beta = c.beta;
+    a.anchor = anchor;
+    a.tab = h->sh_tab;
+    a.ltok = h->sh_ltok;
+    a.lz = h->sh_lz;
+    a.llse = h->sh_llse;
+    a.next = h->sh_next;
+    a.offer = h->sh_offer;
+    a.npop = h->sh_npop;
+    a.hin = h->hbuf[0];
+    a.HL = tc ? h->HL : nullptr;
+    a.hout = h->hbuf[1];
+    a.child_prow = h->child_prow;
+    a.child_tok = h->child_tok;
+    a.dlog_row = h->sh_dlog_row;
+    a.tokens = out->tokens;
+    a.parents = out->parents;
+    a.depths = out->depths;
+    a.pos_ids = out->pos_ids;
+    a.n_nodes = out->n_nodes;
+    a.scores = out->scores;
+    a.mask = out->mask;
+    // scoring of one node per sequence, its best Bp children into slot `slot`
+    auto score = [&](int slot, const float* h32, const int* dlog_row, bool first) -> int {
+        LmheadArgs la = lmhead_args(h, cc, p, dlog, h32);
+        la.dlog_row = dlog_row;  // null: position 0 (the root's children)
+        la.gthr = first ? h->gthr : nullptr;
+        la.zout = h->sh_zrow;
+        la.zout_stride = c.V;
+        int pi = prof_begin(h, kLmhead, st);
+        cudaError_t e = tc ? launch_lmhead_tc(&h->tmE, &h->tmH[ng_index(p.NG)], la, p.smem, st) : launch_lmhead_f32(la, st);
+        prof_end(h, pi, st);
+        if (e != cudaSuccess) return DART_ERR_CUDA;
+        SelectArgs sa = select_args(h, cc, p, 1);
+        sa.gthr = la.gthr;
+        sa.lse_hist = h->sh_llse + slot;
+        sa.lse_hist_stride = static_cast<long long>(S1);
+        pi = prof_begin(h, kSelect, st);
+        e = launch_merge_select(sa, st);
+        prof_end(h, pi, st);
+        if (e != cudaSuccess) return DART_ERR_CUDA;
+        pi = prof_begin(h, kRowTopk, st);
+        e = launch_row_topk_by_value(h->sh_zrow, c.nseq, c.V, h->Bp, h->sh_S, h->sh_ltok + slot * h->Bp,
+                                     h->sh_lz + slot * h->Bp, static_cast<long long>(S1) * h->Bp, h->sh_part,
+                                     h->sh_ticket, st);
+        prof_end(h, pi, st);
+        return e == cudaSuccess ? DART_OK : DART_ERR_CUDA;
+    };
+    int pi = prof_begin(h, kPrep, st);
+    cudaError_t e = launch_prep_anchor(anchor, c.nseq, c.d, h->hbuf[0], tc ? h->HL : nullptr, kNPadMax, h->gthr,
+                                       kNPadMax, st);
+    prof_end(h, pi, st);
+    if (e != cudaSuccess) return DART_ERR_CUDA;
+    int rc = score(0, h->hbuf[0], nullptr, true);
+    if (rc != DART_OK) return rc;
+    for (int t = 0; t < c.B; t++) {
+        pi = prof_begin(h, kSeqStep, st);
+        e = launch_seqheap_step(a, t, st);
+        prof_end(h, pi, st);
+        if (e != cudaSuccess) return DART_ERR_CUDA;
+        if (c.L == 1 || t + 1 == c.B) continue;
+        rc = enqueue_head_update(h, cc, p, h->hbuf[0], h->hbuf[1], false, st);
+        if (rc == DART_OK) rc = score(t + 1, h->hbuf[1], h->sh_dlog_row, false);
+        if (rc != DART_OK) return rc;
+    }
+    pi = prof_begin(h, kSeqEmit, st);
+    e = launch_seqheap_emit(a, st);
+    prof_end(h, pi, st);
+    return e == cudaSuccess ? DART_OK : DART_ERR_CUDA;
 }
 
 int check_inputs(const dart_handle* h, const float* dlog, const float* anchor, bool need_anchor) {
@@ -800,6 +1056,77 @@ cudaError_t cache_and_launch(dart_handle* h, const GraphEntry& ge, cudaStream_t 
     }
     h->graphs.push_back(ge);
     return cudaGraphLaunch(ge.exec, st);
+}
+
+int enqueue_kind(dart_handle* h, int kind, const float* dlog, const float* anchor, const dart_tree_out* out,
+                 cudaStream_t st) {
+    switch (kind) {
+        case kRoundChainDdtree: return enqueue_chain_ddtree(h, dlog, anchor, out, st);
+        case kRoundSeqHeap: return enqueue_seq_heap(h, dlog, anchor, out, st);
+        default: return enqueue_round(h, dlog, anchor, out, st);
+    }
+}
+
+// After a round of `kind`: the state the test hooks see.  Algorithm 1's
+// rounds leave every depth readable; the best-first constructions leave no
+// Algorithm 1 frontier (dart_get_chain reads the chain).
+void finish_round(dart_handle* h, int kind, bool ok) {
+    h->last_kind = kind;
+    if (!ok) {
+        h->next_depth = 1;
+        return;
+    }
+    h->next_depth = h->cfg.L + 1;
+    if (kind == kRoundDartree) h->last_rows = h->plans[h->cfg.L].N;
+}
+
+// One round of construction `kind`: launched as one cached CUDA graph per
+// distinct (kind, inputs, outputs) set, or enqueued directly when profiling
+// or when the caller is capturing the stream.
+int run_round(dart_handle* h, int kind, const float* dlog, const float* anchor, const dart_tree_out* out,
+              void* stream) {
+    if (!h) return DART_ERR_INVALID;
+    int rc = check_inputs(h, dlog, anchor, true);
+    if (rc == DART_OK) rc = check_out(out);
+    if (rc != DART_OK) return rc;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+    if (cudaStreamIsCapturing(st, &cs) != cudaSuccess) return DART_ERR_CUDA;
+    if (h->profiling || cs != cudaStreamCaptureStatusNone) {
+        rc = enqueue_kind(h, kind, dlog, anchor, out, st);
+        finish_round(h, kind, rc == DART_OK);
+        return rc;
+    }
+    const void* key[10] = {reinterpret_cast<const void*>(static_cast<uintptr_t>(kind)),
+                           dlog, anchor, out->tokens, out->parents, out->depths,
+                           out->pos_ids, out->scores, out->n_nodes, out->mask};
+    for (auto& g : h->graphs) {
+        if (std::memcmp(g.key, key, sizeof key) == 0) {
+            finish_round(h, kind, true);
+            g.last_use = ++h->graph_clock;
+            return cuda_err(cudaGraphLaunch(g.exec, st));
+        }
+    }
+    cudaGraph_t graph = nullptr;
+    if (cudaStreamBeginCapture(h->cap_stream, cudaStreamCaptureModeThreadLocal) != cudaSuccess) return DART_ERR_CUDA;
+    rc = enqueue_kind(h, kind, dlog, anchor, out, h->cap_stream);
+    cudaError_t ce = cudaStreamEndCapture(h->cap_stream, &graph);
+    if (rc != DART_OK || ce != cudaSuccess) {
+        if (graph) cudaGraphDestroy(graph);
+        finish_round(h, kind, false);
+        return rc != DART_OK ? rc : DART_ERR_CUDA;
+    }
+    GraphEntry ge;
+    std::memcpy(ge.key, key, sizeof key);
+    ce = cudaGraphInstantiate(&ge.exec, graph, 0);
+    cudaGraphDestroy(graph);
+    if (ce != cudaSuccess) {
+        finish_round(h, kind, false);
+        return DART_ERR_CUDA;
+    }
+    ge.last_use = ++h->graph_clock;
+    finish_round(h, kind, true);
+    return cuda_err(cache_and_launch(h, ge, st));
 }
 
 }  // namespace
@@ -850,7 +1177,22 @@ int dart_init_head(dart_handle** out, const dart_config* cfg, int wdtype, const 
     h->smem_optin = optin;
     h->next_depth = 1;
     if (wdtype == DART_BF16 && tc_set_smem_limits(optin) != cudaSuccess) rc = DART_ERR_CUDA;
-    if (rc == DART_OK) rc = build_plans(h);
+    if (rc == DART_OK) rc = build_plans(h, h->cfg, h->caps, h->plans);
+    if (rc == DART_OK && cfg->variants) {
+        // the best-first constructions score one node per sequence at a time
+        // over the full vocabulary and keep its best min(B, V) children
+        if (cfg->cand_k != 0 || cfg->nseq > 64) rc = DART_ERR_UNSUPPORTED;
+        h->ccfg = *cfg;
+        h->ccfg.W = 1;
+        h->ccfg.k = 1;
+        h->Bp = std::min(cfg->B, cfg->V);
+        h->ddt_S = cand_topk_slices(cfg->V, h->Bp, cfg->nseq * cfg->L, sms);
+        h->sh_S = cand_topk_slices(cfg->V, h->Bp, cfg->nseq, sms);
+        if (rc == DART_OK) rc = build_plans(h, h->ccfg, h->ccaps, h->cplans);
+        if (rc == DART_OK && (cfg->variants & DART_VARIANT_CHAIN_DDTREE) &&
+            ddtree_smem(cfg->L, h->Bp, cfg->B) > optin)
+            rc = DART_ERR_UNSUPPORTED;
+    }
     if (rc == DART_OK) rc = alloc_workspace(h);
     if (rc == DART_OK && wdtype == DART_BF16) rc = make_tensor_maps(h);
     if (rc == DART_OK && h->Qtab) rc = compute_qtab(h, static_cast<cudaStream_t>(stream));
@@ -884,9 +1226,10 @@ int dart_expand_depth(dart_handle* h, int depth, const float* drafter_logits, co
     if (depth < 1 || depth > h->cfg.L) return DART_ERR_INVALID;
     int rc = check_inputs(h, drafter_logits, anchor_h, depth == 1);
     if (rc != DART_OK) return rc;
-    if (depth != 1 && depth != h->next_depth) return DART_ERR_STATE;
-    rc = enqueue_depth(h, depth, drafter_logits, anchor_h, static_cast<cudaStream_t>(stream));
+    if (depth != 1 && (depth != h->next_depth || h->last_kind != kRoundDartree)) return DART_ERR_STATE;
+    rc = enqueue_depth(h, h->cfg, h->plans, depth, drafter_logits, anchor_h, static_cast<cudaStream_t>(stream));
     h->next_depth = rc == DART_OK ? depth + 1 : 1;
+    h->last_kind = kRoundDartree;
     return rc;
 }
 
@@ -894,53 +1237,48 @@ int dart_prune_and_emit(dart_handle* h, const dart_tree_out* out, void* stream) 
     if (!h) return DART_ERR_INVALID;
     int rc = check_out(out);
     if (rc != DART_OK) return rc;
-    if (h->next_depth != h->cfg.L + 1) return DART_ERR_STATE;
+    if (h->next_depth != h->cfg.L + 1 || h->last_kind != kRoundDartree) return DART_ERR_STATE;
     return enqueue_emit(h, out, static_cast<cudaStream_t>(stream));
 }
 
 int dart_build_tree(dart_handle* h, const float* drafter_logits, const float* anchor_h, const dart_tree_out* out,
                     void* stream) {
+    return run_round(h, kRoundDartree, drafter_logits, anchor_h, out, stream);
+}
+
+int dart_build_tree_fixed(dart_handle* h, const float* drafter_logits, const float* anchor_h,
+                          const dart_tree_out* out, void* stream) {
     if (!h) return DART_ERR_INVALID;
-    int rc = check_inputs(h, drafter_logits, anchor_h, true);
-    if (rc == DART_OK) rc = check_out(out);
-    if (rc != DART_OK) return rc;
+    int total = 0;
+    for (int dep = 1; dep <= h->cfg.L; dep++) total += h->caps[dep];
+    if (h->cfg.B < total) return DART_ERR_INVALID;  // every retained node must fit: no pruning
+    return run_round(h, kRoundDartree, drafter_logits, anchor_h, out, stream);
+}
+
+int dart_build_chain_ddtree(dart_handle* h, const float* drafter_logits, const float* anchor_h,
+                            const dart_tree_out* out, void* stream) {
+    if (!h) return DART_ERR_INVALID;
+    if (!(h->cfg.variants & DART_VARIANT_CHAIN_DDTREE)) return DART_ERR_STATE;
+    return run_round(h, kRoundChainDdtree, drafter_logits, anchor_h, out, stream);
+}
+
+int dart_build_seq_heap(dart_handle* h, const float* drafter_logits, const float* anchor_h, const dart_tree_out* out,
+                        void* stream) {
+    if (!h) return DART_ERR_INVALID;
+    if (!(h->cfg.variants & DART_VARIANT_SEQ_HEAP)) return DART_ERR_STATE;
+    return run_round(h, kRoundSeqHeap, drafter_logits, anchor_h, out, stream);
+}
+
+int dart_get_chain(dart_handle* h, int32_t* tok, float* lse, void* stream) {
+    if (!h) return DART_ERR_INVALID;
+    if (h->last_kind != kRoundChainDdtree || h->next_depth != h->cfg.L + 1) return DART_ERR_STATE;
+    const size_t n = static_cast<size_t>(h->cfg.nseq) * h->cfg.L;
     cudaStream_t st = static_cast<cudaStream_t>(stream);
-    cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
-    if (cudaStreamIsCapturing(st, &cs) != cudaSuccess) return DART_ERR_CUDA;
-    if (h->profiling || cs != cudaStreamCaptureStatusNone) {
-        rc = enqueue_round(h, drafter_logits, anchor_h, out, st);
-        if (rc != DART_OK) h->next_depth = 1;
-        return rc;
-    }
-    const void* key[9] = {drafter_logits, anchor_h, out->tokens, out->parents, out->depths,
-                          out->pos_ids,   out->scores, out->n_nodes, out->mask};
-    for (auto& g : h->graphs) {
-        if (std::memcmp(g.key, key, sizeof key) == 0) {
-            h->next_depth = h->cfg.L + 1;
-            h->last_rows = h->plans[h->cfg.L].N;
-            g.last_use = ++h->graph_clock;
-            return cuda_err(cudaGraphLaunch(g.exec, st));
-        }
-    }
-    cudaGraph_t graph = nullptr;
-    if (cudaStreamBeginCapture(h->cap_stream, cudaStreamCaptureModeThreadLocal) != cudaSuccess) return DART_ERR_CUDA;
-    rc = enqueue_round(h, drafter_logits, anchor_h, out, h->cap_stream);
-    cudaError_t ce = cudaStreamEndCapture(h->cap_stream, &graph);
-    if (rc != DART_OK || ce != cudaSuccess) {
-        if (graph) cudaGraphDestroy(graph);
-        h->next_depth = 1;
-        return rc != DART_OK ? rc : DART_ERR_CUDA;
-    }
-    GraphEntry ge;
-    std::memcpy(ge.key, key, sizeof key);
-    ce = cudaGraphInstantiate(&ge.exec, graph, 0);
-    cudaGraphDestroy(graph);
-    if (ce != cudaSuccess) {
-        h->next_depth = 1;
-        return DART_ERR_CUDA;
-    }
-    ge.last_use = ++h->graph_clock;
-    return cuda_err(cache_and_launch(h, ge, st));
+    cudaError_t e = cudaSuccess;
+    // the chain ran with W = 1: its depth-d node of sequence s is tree slot s * L + d - 1
+    if (tok) e = cudaMemcpyAsync(tok, h->tree_tok, n * 4, cudaMemcpyDeviceToDevice, st);
+    if (lse && e == cudaSuccess) e = cudaMemcpyAsync(lse, h->chain_lse, n * 4, cudaMemcpyDeviceToDevice, st);
+    return cuda_err(e);
 }
 
 int dart_build_tree_host(dart_handle* h, const float* drafter_logits_host, const float* anchor_host,
@@ -989,7 +1327,7 @@ int dart_build_tree_host(dart_handle* h, const float* drafter_logits_host, const
 int dart_get_frontier(dart_handle* h, int depth, int32_t* tok, int32_t* parent_slot, float* score, int32_t* count,
                       void* stream) {
     if (!h || depth < 1 || depth > h->cfg.L) return DART_ERR_INVALID;
-    if (depth >= h->next_depth) return DART_ERR_STATE;
+    if (depth >= h->next_depth || h->last_kind != kRoundDartree) return DART_ERR_STATE;
     const dart_config& c = h->cfg;
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     const size_t W = c.W;
@@ -1009,7 +1347,7 @@ int dart_get_frontier(dart_handle* h, int depth, int32_t* tok, int32_t* parent_s
 
 int dart_get_node_topk(dart_handle* h, int32_t* tok, float* logq, float* lse, int* rows, void* stream) {
     if (!h) return DART_ERR_INVALID;
-    if (h->next_depth < 2) return DART_ERR_STATE;
+    if (h->next_depth < 2 || h->last_kind != kRoundDartree) return DART_ERR_STATE;
     const int dep = h->next_depth - 1;
     const int N = h->plans[dep].N;
     if (rows) *rows = N;
@@ -1024,7 +1362,7 @@ int dart_get_node_topk(dart_handle* h, int32_t* tok, float* logq, float* lse, in
 
 int dart_get_states(dart_handle* h, float* states, int* rows, void* stream) {
     if (!h) return DART_ERR_INVALID;
-    if (h->next_depth < 2) return DART_ERR_STATE;
+    if (h->next_depth < 2 || h->last_kind != kRoundDartree) return DART_ERR_STATE;
     const int dep = h->next_depth - 1;
     const int R = dep < h->cfg.L ? h->plans[dep].Nc : h->plans[dep].N;
     if (rows) *rows = R;

@@ -121,7 +121,8 @@ __device__ __forceinline__ void for_row(const float* x, int V, F&& f) {
 // its count) and the last block of the row to finish (atomic ticket; nobody
 // waits) selects the K largest of the S K published keys.
 __global__ void __launch_bounds__(kTopkThreads)
-    cand_topk_kernel(const float* dlog, int V, int K, int S, int* cand_tok, uint64_t* part, int* ticket) {
+    cand_topk_kernel(const float* dlog, int V, int K, int S, int* cand_tok, uint64_t* part, int* ticket,
+                     int by_value, long long out_stride, float* out_val) {
     pdl_trigger();
     pdl_wait();
     extern __shared__ uint64_t csm[];
@@ -266,12 +267,18 @@ __global__ void __launch_bounds__(kTopkThreads)
             if (coll[i] >= kth && coll[i] != 0ull) out[atomicAdd(&cnt[0], 1)] = coll[i];
         __syncthreads();
     }
-    // write the K tokens in ascending order (rank by counting)
+    // write the K tokens in ascending token order, or (by_value) best first
+    // with their values (rank by counting; keys are distinct)
     for (int i = tid; i < K; i += kTopkThreads) {
         const uint32_t tk = key_idx(out[i]);
         int r = 0;
-        for (int j = 0; j < K; j++) r += key_idx(out[j]) < tk;
-        cand_tok[static_cast<size_t>(row) * K + r] = static_cast<int>(tk);
+        if (by_value) {
+            for (int j = 0; j < K; j++) r += out[j] > out[i];
+        } else {
+            for (int j = 0; j < K; j++) r += key_idx(out[j]) < tk;
+        }
+        cand_tok[static_cast<size_t>(row) * out_stride + r] = static_cast<int>(tk);
+        if (out_val) out_val[static_cast<size_t>(row) * out_stride + r] = key_val(out[i]);
     }
 }
 
@@ -429,7 +436,13 @@ cudaError_t cand_set_smem_limits(int topk_smem, int score_smem) {
 cudaError_t launch_cand_topk(const float* dlog, int rows, int V, int K, int S, int* cand_tok, uint64_t* part,
                              int* ticket, cudaStream_t st) {
     return launch_pdl(cand_topk_kernel, dim3(rows * S), dim3(kTopkThreads), cand_topk_smem(K), st, dlog, V, K, S,
-                      cand_tok, part, ticket);
+                      cand_tok, part, ticket, 0, static_cast<long long>(K), static_cast<float*>(nullptr));
+}
+
+cudaError_t launch_row_topk_by_value(const float* x, int rows, int V, int K, int S, int* tok, float* val,
+                                     long long out_stride, uint64_t* part, int* ticket, cudaStream_t st) {
+    return launch_pdl(cand_topk_kernel, dim3(rows * S), dim3(kTopkThreads), cand_topk_smem(K), st, x, V, K, S, tok,
+                      part, ticket, 1, out_stride, val);
 }
 
 cudaError_t launch_cand_score(const CandArgs& a, cudaStream_t st) {

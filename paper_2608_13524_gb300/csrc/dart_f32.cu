@@ -91,9 +91,12 @@ __global__ void __launch_bounds__(kEpiThreads) lmhead_f32_kernel(const LmheadArg
                     const int seq = n / a.P;
                     if (seq != cur_seq) {
                         cur_seq = seq;
-                        dl = valid ? __ldg(a.dlog + seq * a.dlog_seq_stride + a.dlog_row_off + v) : 0.0f;
+                        const long long off = a.dlog_row ? static_cast<long long>(__ldg(a.dlog_row + seq)) * a.V
+                                                         : a.dlog_row_off;
+                        dl = valid ? __ldg(a.dlog + seq * a.dlog_seq_stride + off + v) : 0.0f;
                     }
                     z[j] = (acc[c0 + j] + dl) * a.invT;
+                    if (a.zout && valid) a.zout[static_cast<long long>(n) * a.zout_stride + v] = z[j];
                 }
             }
             (void)epi_chunk(e, NG, a.k, ew, lane, c0, z, nodemask, valid, static_cast<uint32_t>(v), ssum[c0 / 16]);

@@ -79,6 +79,10 @@ struct LmheadArgs {
     const float* h32;     // fp32 states [N][d] (fp32 kernel)
     const float* E32;     // fp32 table [V][d]   (fp32 kernel)
     uint64_t* gthr;       // [N] cross-CTA top-k bounds, zero before the launch (may be null)
+    // optional (null: unused)
+    const int* dlog_row;  // [nseq] drafter row of each sequence's nodes (replaces dlog_row_off / V)
+    float* zout;          // z[n][v] written to zout[n * zout_stride + v] (node groups <= 64)
+    long long zout_stride;
 };
 
 // Skinny split-K GEMM for the correction head: out[split][n][m] =
@@ -154,6 +158,8 @@ struct SelectArgs {
     int* child_tok;
     int* seq_ticket;       // [nseq]
     int* status;
+    float* lse_hist;       // optional: node n's log-sum-exp also to lse_hist[n * lse_hist_stride]
+    long long lse_hist_stride;
 };
 cudaError_t launch_merge_select(const SelectArgs& a, cudaStream_t st);
 int merge_select_smem(int nV, int klist, int k, int W);
@@ -180,6 +186,10 @@ struct CandArgs {
 // leaves them zero).
 cudaError_t launch_cand_topk(const float* dlog, int rows, int V, int K, int S, int* cand_tok, uint64_t* part,
                              int* ticket, cudaStream_t st);
+// The same selection over rows of any fp32 values x [rows][V], written best
+// first (value desc, index asc): tok / val [rows][out_stride], K per row.
+cudaError_t launch_row_topk_by_value(const float* x, int rows, int V, int K, int S, int* tok, float* val,
+                                     long long out_stride, uint64_t* part, int* ticket, cudaStream_t st);
 int cand_topk_slices(int V, int K, int rows, int num_sms);
 cudaError_t launch_cand_score(const CandArgs& a, cudaStream_t st);
 int cand_topk_smem(int K);
@@ -199,6 +209,51 @@ struct EmitArgs {
     int* status;
 };
 cudaError_t launch_prune_emit(const EmitArgs& a, cudaStream_t st);
+
+// Best-first constructions of Table 2 (dart_heap.cu).
+// Domino-chain + DDTree: the chain's best Bp children per depth (value order)
+// tok / zval [nseq][L][Bp] and lse [nseq][L] -> the emitted tree.
+struct DdtArgs {
+    int L, B, Bp, nseq, pos_offset;
+    float beta;
+    const int* tok;
+    const float* zval;
+    const float* lse;
+    int *tokens, *parents, *depths, *pos_ids, *n_nodes;
+    float* scores;
+    uint64_t* mask;
+};
+int ddtree_smem(int L, int Bp, int B);
+cudaError_t heap_set_smem_limits(int ddtree_bytes);
+cudaError_t launch_ddtree(const DdtArgs& a, cudaStream_t st);
+// Sequential correction with heap: per sequence, slot 0 = the root and slot
+// p + 1 = popped node p: state tab [nseq][B+1][d], sorted children ltok / lz
+// [nseq][B+1][Bp] (value order) with their log-sum-exp llse [nseq][B+1],
+// cursor next and offer [nseq][B+1], pops npop [nseq]; the output rows are
+// written in pop order.  hin / HL (rows s, bhalf + s): the head's input for
+// the popped prefix; hout: the head's output; child_prow / child_tok /
+// dlog_row [nseq]: the head update's and the LM-head's per-sequence inputs.
+struct SeqHeapArgs {
+    int L, B, Bp, nseq, d, pos_offset, bhalf;
+    float beta;
+    const float* anchor;  // [nseq][d] r_0 (slot 0 of the table)
+    float* tab;
+    const int* ltok;
+    const float* lz;
+    const float* llse;
+    int* next;
+    float* offer;
+    int* npop;
+    float* hin;
+    __nv_bfloat16* HL;
+    const float* hout;
+    int *child_prow, *child_tok, *dlog_row;
+    int *tokens, *parents, *depths, *pos_ids, *n_nodes;
+    float* scores;
+    uint64_t* mask;
+};
+cudaError_t launch_seqheap_step(const SeqHeapArgs& a, int t, cudaStream_t st);
+cudaError_t launch_seqheap_emit(const SeqHeapArgs& a, cudaStream_t st);
 
 // One CTA whose bounded mbarrier waits run out (see dart_test_wait_timeout).
 cudaError_t launch_wait_probe(int* status, unsigned long long limit_ns, long long* elapsed_ns, cudaStream_t st);

@@ -104,7 +104,10 @@ __global__ void __launch_bounds__(kSelThreads) merge_select_kernel(const SelectA
             a.node_logq[static_cast<size_t>(n) * a.k + j] = lq;
             a.node_tok[static_cast<size_t>(n) * a.k + j] = static_cast<int>(key_idx(x));
         }
-        if (tid == 0) a.node_lse[n] = lse;
+        if (tid == 0) {
+            a.node_lse[n] = lse;
+            if (a.lse_hist) a.lse_hist[static_cast<size_t>(n) * a.lse_hist_stride] = lse;
+        }
     } else {
         for (int j = tid; j < a.k; j += kSelThreads) {
             a.node_logq[static_cast<size_t>(n) * a.k + j] = -INFINITY;

@@ -345,7 +345,9 @@ __global__ void __launch_bounds__(threads<NG>(), 1)
                     const int seq = (g * NG + c0 + j) / a.P;
                     if (seq != cur_seq) {
                         cur_seq = seq;
-                        dl = valid ? __ldg(a.dlog + seq * a.dlog_seq_stride + a.dlog_row_off + v) : 0.0f;
+                        const long long off = a.dlog_row ? static_cast<long long>(__ldg(a.dlog_row + seq)) * a.V
+                                                         : a.dlog_row_off;
+                        dl = valid ? __ldg(a.dlog + seq * a.dlog_seq_stride + off + v) : 0.0f;
                     }
                     z[j] = (z[j] + dl) * a.invT;
                 }
@@ -371,6 +373,12 @@ __global__ void __launch_bounds__(threads<NG>(), 1)
                 load_z(acc, 0, v, valid, z);
                 tc_fence_before();
                 mbar_arrive(&s.tempty[acc]);
+                if (a.zout && valid) {
+                    const int nb = g * NG + (wi >> 2) * 16;
+#pragma unroll
+                    for (int j = 0; j < 16; j++)
+                        if ((nodemask[0] >> j) & 1u) a.zout[static_cast<long long>(nb + j) * a.zout_stride + v] = z[j];
+                }
                 (void)epi_chunk(e, NG, a.k, quarter, lane, (wi >> 2) * 16, z, nodemask[0], valid,
                                 static_cast<uint32_t>(v), ssum[0]);
                 epi_merge(e, NG, a.k, wi, lane, kEpi, etid, a.gthr, g * NG, a.N);

@@ -71,6 +71,10 @@ def lib():
             "dart_prune_and_emit": (i, [vp, C.POINTER(DartTreeOut), vp]),
             "dart_build_tree": (i, [vp, vp, vp, C.POINTER(DartTreeOut), vp]),
             "dart_build_tree_host": (i, [vp, vp, vp, C.POINTER(DartTreeOut), vp]),
+            "dart_build_tree_fixed": (i, [vp, vp, vp, C.POINTER(DartTreeOut), vp]),
+            "dart_build_chain_ddtree": (i, [vp, vp, vp, C.POINTER(DartTreeOut), vp]),
+            "dart_build_seq_heap": (i, [vp, vp, vp, C.POINTER(DartTreeOut), vp]),
+            "dart_get_chain": (i, [vp, vp, vp, vp]),
             "dart_get_frontier": (i, [vp, i, vp, vp, vp, vp, vp]),
             "dart_get_node_topk": (i, [vp, vp, vp, vp, C.POINTER(i), vp]),
             "dart_get_states": (i, [vp, vp, C.POINTER(i), vp]),
@@ -176,6 +180,33 @@ def dart_build_tree(h, drafter_logits, anchor_h, out: DartTreeOut, stream=None):
                                  _stream(stream)), "dart_build_tree")
 
 
+def dart_build_tree_fixed(h, drafter_logits, anchor_h, out: DartTreeOut, stream=None):
+    """DARTree (fixed): every retained node emitted, no pruning (B >= sum |S_d|)."""
+    _check(lib().dart_build_tree_fixed(h, _ptr(drafter_logits), _ptr(anchor_h), C.byref(out),
+                                       _stream(stream)), "dart_build_tree_fixed")
+
+
+def dart_build_chain_ddtree(h, drafter_logits, anchor_h, out: DartTreeOut, stream=None):
+    """Domino-chain + DDTree (the handle needs DART_VARIANT_CHAIN_DDTREE)."""
+    _check(lib().dart_build_chain_ddtree(h, _ptr(drafter_logits), _ptr(anchor_h), C.byref(out),
+                                         _stream(stream)), "dart_build_chain_ddtree")
+
+
+def dart_build_seq_heap(h, drafter_logits, anchor_h, out: DartTreeOut, stream=None):
+    """Sequential correction with heap (the handle needs DART_VARIANT_SEQ_HEAP)."""
+    _check(lib().dart_build_seq_heap(h, _ptr(drafter_logits), _ptr(anchor_h), C.byref(out),
+                                     _stream(stream)), "dart_build_seq_heap")
+
+
+def dart_get_chain(h, cfg, stream=None):
+    """(chain tokens [nseq][L] int32, log-sum-exp [nseq][L] float) after
+    dart_build_chain_ddtree."""
+    tok = torch.empty((cfg.nseq, cfg.L), dtype=torch.int32, device="cuda")
+    lse = torch.empty((cfg.nseq, cfg.L), dtype=torch.float32, device="cuda")
+    _check(lib().dart_get_chain(h, _ptr(tok), _ptr(lse), _stream(stream)), "dart_get_chain")
+    return tok, lse
+
+
 def dart_build_tree_host(h, drafter_logits_host, anchor_host, out_host: DartTreeOut, stream=None):
     _check(lib().dart_build_tree_host(h, _ptr(drafter_logits_host), _ptr(anchor_host),
                                       C.byref(out_host), _stream(stream)), "dart_build_tree_host")
@@ -236,7 +267,8 @@ def dart_profile_read(h):
 
 
 KIND_NAMES = ("lmhead", "merge_select", "gather", "gemm_wi", "silu_split", "gemm_wo", "residual_norm",
-              "prep_anchor", "prune_emit", "cand_topk", "cand_score", "gather_silu")
+              "prep_anchor", "prune_emit", "cand_topk", "cand_score", "gather_silu", "row_topk", "ddtree",
+              "seqheap_step", "seqheap_emit")
 
 
 def dart_profile_read_kinds(h):
@@ -291,6 +323,18 @@ class Dart:
 
     def build_tree(self, drafter_logits, anchor_h, stream=None):
         dart_build_tree(self.h, drafter_logits, anchor_h, self.out, stream)
+        return self.out_t
+
+    def build_tree_fixed(self, drafter_logits, anchor_h, stream=None):
+        dart_build_tree_fixed(self.h, drafter_logits, anchor_h, self.out, stream)
+        return self.out_t
+
+    def build_chain_ddtree(self, drafter_logits, anchor_h, stream=None):
+        dart_build_chain_ddtree(self.h, drafter_logits, anchor_h, self.out, stream)
+        return self.out_t
+
+    def build_seq_heap(self, drafter_logits, anchor_h, stream=None):
+        dart_build_seq_heap(self.h, drafter_logits, anchor_h, self.out, stream)
         return self.out_t
 
     def close(self):

@@ -299,3 +299,112 @@ def validate_frontier_teacher_forced(cfg, x, gst, s, dep, tol_step):
         for r in range(int(gst["st_count"][s, dep - 2])):
             known[(dep - 2) * cfg.W + r] = float(gst["st_score"][s, dep - 2, r])
     validate_depth_teacher_forced(cfg, TeacherForced(cfg, x, s), gst, s, dep, tol_step, known)
+
+
+# ----------------------------------------------- best-first constructions
+
+def pop_order_paths(g, s):
+    """[(token path, score)] of the emitted rows of sequence s, in row order."""
+    out = []
+    for i in range(int(g["n_nodes"][s])):
+        path, j = [], i
+        while j >= 0:
+            path.append(int(g["tokens"][s, j]))
+            j = int(g["parents"][s, j])
+        out.append((tuple(reversed(path)), float(g["scores"][s, i])))
+    return out
+
+
+def check_pop_order_structure(cfg, g, s):
+    """Rows in pop order: parents first, depth = parent's + 1, position ids,
+    scores finite and non-increasing (exact: a child adds log q~ <= 0 and
+    beta <= 0 to its parent's score), ancestor mask, padding."""
+    n = int(g["n_nodes"][s])
+    assert 0 <= n <= cfg.B
+    par = g["parents"][s]
+    for i in range(n):
+        p = int(par[i])
+        assert -1 <= p < i, (s, i, p)
+        assert g["depths"][s, i] == (1 if p < 0 else g["depths"][s, p] + 1)
+        assert 1 <= g["depths"][s, i] <= cfg.L
+        assert g["pos_ids"][s, i] == cfg.pos_offset + g["depths"][s, i]
+        assert np.isfinite(g["scores"][s, i])
+        if i:
+            assert g["scores"][s, i] <= g["scores"][s, i - 1], (s, i)
+        anc, j = set(), i
+        while j >= 0:
+            anc.add(j)
+            j = int(par[j])
+        row = np.asarray(g["mask"][s, i]).view(np.uint64)
+        assert {b for b in range(cfg.B) if (int(row[b // 64]) >> (b % 64)) & 1} == anc, (s, i)
+    for i in range(n, cfg.B):
+        assert g["tokens"][s, i] == -1 and g["parents"][s, i] == -2
+        assert g["depths"][s, i] == 0 and g["pos_ids"][s, i] == -1
+        assert np.isneginf(g["scores"][s, i]) and not np.any(g["mask"][s, i])
+
+
+def compare_pop_order_tree(cfg, ref, g, tol, path_score):
+    """A best-first tree of the GPU (rows in pop order) against the oracle's.
+    path_score(s, path) is the oracle's score of any prefix, so a GPU path the
+    oracle tree lacks is still checked.  Rules: the same node count; every
+    GPU path scored within tol of the oracle's score of that path; the two
+    node sets equal, or differing only across a near tie at the budget cut
+    (each path only one side has scores within 2 tol of the cut); the rows in
+    the oracle's order wherever the oracle's adjacent scores differ by >= tol;
+    the structure of check_pop_order_structure."""
+    rep = dict(near_tie=[], order_ties=0, bit_identical=None, max_score_err=0.0)
+    for s in range(cfg.nseq):
+        check_pop_order_structure(cfg, g, s)
+        gp, rp = pop_order_paths(g, s), pop_order_paths(ref, s)
+        assert len(gp) == len(rp) == int(ref["n_nodes"][s]), (s, len(gp), len(rp))
+        rs = dict(rp)
+        orc = {}
+        for p, sc in gp:
+            o = rs[p] if p in rs else path_score(s, p)
+            orc[p] = o
+            e = abs(sc - o)
+            rep["max_score_err"] = max(rep["max_score_err"], e)
+            assert e <= tol, f"seq {s} path {p}: score off by {e}"
+        if set(orc) != set(rs):
+            cut = rp[-1][1] if rp else np.inf
+            for p in set(orc) - set(rs):
+                assert orc[p] >= cut - 2 * tol, f"seq {s}: GPU path {p} below the oracle's cut"
+            gcut = min(orc.values()) if orc else -np.inf
+            for p in set(rs) - set(orc):
+                assert rs[p] <= gcut + 2 * tol, f"seq {s}: oracle path {p} missing well above the GPU's cut"
+            rep["near_tie"].append((s, float(cut)))
+            continue
+        gaps = [rp[i][1] - rp[i + 1][1] for i in range(len(rp) - 1)]
+        if all(x >= tol for x in gaps):
+            assert [p for p, _ in gp] == [p for p, _ in rp], f"seq {s}: pop order differs"
+        else:
+            rep["order_ties"] += 1
+            for i in range(len(gp) - 1):
+                assert orc[gp[i][0]] >= orc[gp[i + 1][0]] - 2 * tol
+    keys = ("tokens", "parents", "depths", "pos_ids", "n_nodes")
+    rep["bit_identical"] = bool(all(np.array_equal(g[k], ref[k]) for k in keys) and
+                                np.array_equal(np.asarray(g["mask"]).view(np.uint64), ref["mask"]))
+    return rep
+
+
+def chain_path_score(cfg, x, chain):
+    """path_score for Domino-chain + DDTree: a prefix scored with the oracle's
+    distributions of the chain prefixes (`chain` [nseq][L] = the oracle's
+    chain), sum_i log q~_i(u_i | chain_<i) + beta len."""
+    rows = {}
+
+    def row(s, i):
+        if (s, i) not in rows:
+            tf = TeacherForced(cfg, x, s)
+            z = oracle.child_logits(cfg, x["E"], x["Dlog"][s, i], tf.state(tuple(int(t) for t in chain[s][:i])))
+            rows[(s, i)] = oracle.log_softmax(z)[0]
+        return rows[(s, i)]
+
+    return lambda s, p: sum(float(row(s, i)[t]) for i, t in enumerate(p)) + cfg.beta * len(p)
+
+
+def corrected_path_score(cfg, x):
+    """path_score for the sequential search: the prefix's own corrected
+    scores (Eq. 5 along the path, teacher-forced by the oracle)."""
+    return lambda s, p: float(oracle.path_scores(cfg, x["Wi"], x["Wo"], x["E"], x["Dlog"][s], x["h0"][s],
+                                                 np.array(p, np.int32))[-1])

@@ -259,3 +259,72 @@ def test_a_wrong_frontier_after_a_near_tie_fails(tie_case, dep, how):
     x, ref, gst = planted(tie_case, dep, how)
     with pytest.raises(AssertionError):
         compare_with_oracle(TIE, ref, gst, consistent_gpu_tree(TIE, gst), tol_of(TIE), x=x)
+
+
+# ------------------------------------- best-first (pop-order) trees
+
+HEAP = Config("checker-heap", 2, 500, 64, 4, 4, 4, 20, "bf16", 0.5, 93)
+
+
+@pytest.fixture(scope="module")
+def heap_case():
+    x = make_inputs(HEAP)
+    a = oracle.chain_ddtree(HEAP, x["Wi"], x["Wo"], x["E"], x["Dlog"], x["h0"])
+    b = oracle.seq_heap(HEAP, x["Wi"], x["Wo"], x["E"], x["Dlog"], x["h0"])
+    return x, a, b
+
+
+def as_gpu_rows(ref):
+    g = {k: ref[k].copy() for k in ("tokens", "parents", "depths", "pos_ids", "n_nodes")}
+    g["scores"] = ref["scores"].astype(np.float32)
+    g["mask"] = ref["mask"].view(np.int64).copy()
+    return g
+
+
+def scorers(x, a):
+    from parity import chain_path_score, corrected_path_score
+    return chain_path_score(HEAP, x, a["chain_tok"]), corrected_path_score(HEAP, x)
+
+
+def test_oracle_pop_order_trees_pass(heap_case):
+    from parity import compare_pop_order_tree
+    x, a, b = heap_case
+    sa, sb = scorers(x, a)
+    for ref, sc in ((a, sa), (b, sb)):
+        rep = compare_pop_order_tree(HEAP, ref, as_gpu_rows(ref), tol_of(HEAP), sc)
+        assert rep["bit_identical"] and not rep["near_tie"]
+
+
+@pytest.mark.parametrize("which", ["chain", "seq"])
+@pytest.mark.parametrize("plant", ["token", "score", "swap", "mask", "padding", "count", "parent"])
+def test_a_wrong_pop_order_tree_fails(heap_case, which, plant):
+    from parity import compare_pop_order_tree
+    x, a, b = heap_case
+    ref = a if which == "chain" else b
+    sc = scorers(x, a)[0 if which == "chain" else 1]
+    g = as_gpu_rows(ref)
+    tol = tol_of(HEAP)
+    n = int(g["n_nodes"][0])
+    i = int(np.nonzero(g["parents"][0, :n] >= 0)[0][-1])   # a node below depth 1
+    if plant == "token":
+        g["tokens"][0, i] = (g["tokens"][0, i] + 1) % HEAP.V
+    elif plant == "score":
+        g["scores"][0, n - 1] -= np.float32(3 * tol)
+    elif plant == "swap":
+        j = next(j for j in range(n - 1) if ref["scores"][0, j] - ref["scores"][0, j + 1] > tol
+                 and g["parents"][0, j + 1] != j)
+        for k in ("tokens", "parents", "depths", "pos_ids", "scores"):
+            g[k][0, [j, j + 1]] = g[k][0, [j + 1, j]]
+    elif plant == "mask":
+        g["mask"][0, i, 0] &= ~np.int64(1 << int(g["parents"][0, i]))
+    elif plant == "padding":
+        g["tokens"][0, HEAP.B - 1] = 3 if n < HEAP.B else g["tokens"][0, HEAP.B - 1]
+        g["n_nodes"][0] = n - 1
+    elif plant == "count":
+        g["n_nodes"][1] -= 1
+    elif plant == "parent":
+        g["parents"][0, i] = -1
+        g["depths"][0, i] = 1
+        g["pos_ids"][0, i] = HEAP.pos_offset + 1
+    with pytest.raises(AssertionError):
+        compare_pop_order_tree(HEAP, ref, g, tol, sc)
