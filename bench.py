@@ -514,10 +514,243 @@ def run_verify(args, acfg):
         dist.destroy_process_group()
 
 
+# ------------------------------------------------------- extra measurement modes
+
+def gpu_setup():
+    import torch
+    import torch.distributed as dist
+    rank, world, local = dist_env()
+    if world > 1:
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    dev = torch.device("cuda", local if world > 1 else 0)
+    torch.cuda.set_device(dev)
+    return rank, world, dev
+
+
+def device_inputs(cfg, x, dev):
+    import torch
+    tb = lambda a: torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).to(dev).view(torch.bfloat16)
+    tf = lambda a: torch.from_numpy(np.ascontiguousarray(a)).to(dev)
+    conv = tb if cfg.wdtype == "bf16" else tf
+    return conv(x["Wi"]), conv(x["Wo"]), conv(x["E"]), tf(x["Dlog"]), tf(x["h0"])
+
+
+def clock_sampler(dev):
+    import torch
+    props = torch.cuda.get_device_properties(dev)
+    bus = None
+    try:
+        bus = f"{props.pci_domain_id:08X}:{props.pci_bus_id:02X}:{props.pci_device_id:02X}.0"
+    except Exception:
+        pass
+    return ClockSampler(bus)
+
+
+def time_rounds(build, steps, stream, barrier):
+    """Average device ms of `steps` back-to-back rounds (CUDA events on the
+    launching stream; the caller warmed up)."""
+    import torch
+    barrier()
+    a = torch.cuda.Event(enable_timing=True)
+    b = torch.cuda.Event(enable_timing=True)
+    a.record(stream)
+    for _ in range(steps):
+        build()
+    b.record(stream)
+    barrier()
+    return a.elapsed_time(b) / steps
+
+
+def profile_round(dart, h, build, steps, barrier):
+    """Per-kind device time and launch count of `steps` rounds (events around
+    every launch, direct launches), averaged per round."""
+    dart.dart_set_profiling(h, True)
+    build()
+    dart.dart_profile_read_kinds(h)
+    barrier()
+    for _ in range(steps):
+        build()
+    barrier()
+    kinds = dart.dart_profile_read_kinds(h)
+    dart.dart_set_profiling(h, False)
+    return {k: (v[0] / steps, v[1] / steps) for k, v in kinds.items() if v[1]}
+
+
+def run_table2(args, base):
+    """Construction-only latency of the tree constructions of Table 2 and of
+    DARTree (fixed) on the same synthetic inputs: DARTree (the workload's W,
+    k, B, pruned), DARTree (fixed) (W = k = B / L, no pruning), Domino-chain +
+    DDTree and sequential correction with heap (both with the workload's B)."""
+    import torch
+    from paper_2608_13524_gb300 import dart
+    from workloads import make_inputs
+
+    rank, world, dev = gpu_setup()
+    cfg = base.replace(variants=3)
+    wf = max(1, cfg.B // cfg.L)
+    fixed = base.replace(name=base.name + "-fixed", W=wf, k=wf, B=wf * cfg.L)
+    x = make_inputs(cfg, rank=rank)
+    Wi, Wo, E, D, h0 = device_inputs(cfg, x, dev)
+    stream = torch.cuda.current_stream(dev)
+
+    def barrier():
+        if world > 1:
+            torch.distributed.barrier()
+        torch.cuda.synchronize(dev)
+
+    eng = dart.Dart(cfg, Wi, Wo, E)
+    engf = dart.Dart(fixed, Wi, Wo, E)
+    cons = [("dartree", eng, lambda: eng.build_tree(D, h0, stream), cfg),
+            ("dartree_fixed", engf, lambda: engf.build_tree_fixed(D, h0, stream), fixed),
+            ("chain_ddtree", eng, lambda: eng.build_chain_ddtree(D, h0, stream), cfg),
+            ("seq_heap", eng, lambda: eng.build_seq_heap(D, h0, stream), cfg)]
+    for _, e, build, _ in cons:
+        for _ in range(args.warmup):
+            build()
+        if dart.dart_status_sync(e.h, stream) != 0:
+            raise RuntimeError("device status after warm-up")
+    clocks = clock_sampler(dev)
+    clocks.start()
+    time.sleep(0.3)
+    ms = {name: allreduce_max(time_rounds(build, args.steps, stream, barrier), world, dev)
+          for name, _, build, _ in cons}
+    clk = clocks.stop()
+    peak, peak_kind = measured_peak()
+    out = {}
+    launches = 0
+    for name, e, build, c in cons:
+        kinds = profile_round(dart, e.h, build, 2, barrier)  # up to ~2300 launches per round: 2 fit the event pool
+        lm_ms, lm_n = kinds.get("lmhead", (0.0, 0))
+        n_launch = sum(v[1] for v in kinds.values())
+        launches += n_launch * args.steps
+        emitted = tree_to_counts(e.out_t)
+        out[name] = {"us_per_round": ms[name] * 1e3, "vs_dartree": ms[name] / ms["dartree"],
+                     "lmhead_launches_per_round": lm_n, "launches_per_round": n_launch,
+                     "lmhead_us_per_launch": lm_ms * 1e3 / max(lm_n, 1e-9),
+                     "lmhead_hbm_frac": (c.V * c.d * c.bpe + c.V * 4) / (lm_ms / 1e3 / max(lm_n, 1e-9)) / 1e9 / peak
+                     if lm_n else None,
+                     "W": c.W, "k": c.k, "B": c.B, "nodes_emitted": emitted,
+                     "kernel_us_per_round": {k: v[0] * 1e3 for k, v in kinds.items()}}
+    if dart.dart_status_sync(eng.h, stream) != 0 or dart.dart_status_sync(engf.h, stream) != 0:
+        raise RuntimeError("device status after the timed region")
+    eng.close()
+    engf.close()
+    if rank == 0:
+        line = {"metric": "tree-construction µs/round, the constructions of Table 2 on one input",
+                "value": ms["dartree"] * 1e3, "unit": "µs/round", "n_gpus": world, "steps": args.steps,
+                "warmup": args.warmup, "ms_per_step": sum(ms.values()), "higher_is_better": False,
+                "scaling": "weak", "vs_baseline": None, "dtype": "bf16" if cfg.wdtype == "bf16" else "f32",
+                "data": "synthetic",
+                "config": {"workload": base.name, "nseq": cfg.nseq, "V": cfg.V, "d": cfg.d, "L": cfg.L,
+                           "beta": cfg.beta, "T": cfg.temperature, "parallelism": f"replicas x{world}",
+                           "l2": "inputs larger than L2: E streamed by every LM-head pass"},
+                "constructions": out, "gpu_launches": int(launches), "clocks": clk, "peak_hbm_gbs": peak,
+                "peak_kind": peak_kind,
+                "paper_context": "Table 2 (Qwen3-4B, GSM8K, B = 64, RTX 6000 Ada, whole rounds incl. drafting "
+                                 "and verification): DARTree 28.494 ms, Domino-chain + DDTree 28.285 ms, "
+                                 "Seq. correction w. heap 62.703 ms",
+                "e2e": None, "cpu_baseline": None}
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        torch.distributed.destroy_process_group()
+
+
+def tree_to_counts(out_t):
+    return [int(v) for v in out_t["n_nodes"].cpu().tolist()]
+
+
+def run_sweep(args):
+    """The width / budget sweep at the Qwen3-4B shape (Sec. 5.3): every
+    (W, B) point, µs per round, the LM-head kernel's time per launch and its
+    fraction of the measured HBM copy peak, the round's LM-head bytes over
+    the round time against 8 TB/s."""
+    import torch
+    from paper_2608_13524_gb300 import dart
+    from workloads import make_inputs, sweep_configs
+
+    rank, world, dev = gpu_setup()
+    pts = sweep_configs()
+    x = make_inputs(pts[0], rank=rank)
+    Wi, Wo, E, D, h0 = device_inputs(pts[0], x, dev)
+    stream = torch.cuda.current_stream(dev)
+
+    def barrier():
+        if world > 1:
+            torch.distributed.barrier()
+        torch.cuda.synchronize(dev)
+
+    peak, peak_kind = measured_peak()
+    clocks = clock_sampler(dev)
+    clocks.start()
+    time.sleep(0.3)
+    rows, launches, total_exp, total_ms = [], 0, 0, 0.0
+    for cfg in pts:
+        eng = dart.Dart(cfg, Wi, Wo, E)
+        build = lambda: eng.build_tree(D, h0, stream)
+        for _ in range(args.warmup):
+            build()
+        ms = allreduce_max(time_rounds(build, args.steps, stream, barrier), world, dev)
+        kinds = profile_round(dart, eng.h, build, max(2, args.steps // 4), barrier)
+        if dart.dart_status_sync(eng.h, stream) != 0:
+            raise RuntimeError(f"device status after {cfg.name}")
+        lm_ms, lm_n = kinds["lmhead"]
+        lm_s = lm_ms / 1e3 / lm_n
+        launches += dart.dart_launches_per_round(eng.h) * args.steps
+        exp = cfg.expansions_per_round() * world
+        total_exp += exp
+        total_ms += ms
+        rows.append({"W": cfg.W, "B": cfg.B, "us_per_round": ms * 1e3, "node_expansions_per_s": exp / (ms / 1e3),
+                     "lmhead_us_per_launch": lm_s * 1e6,
+                     "lmhead_hbm_frac": cfg.lmhead_bytes_per_depth() / lm_s / 1e9 / peak,
+                     "round_lmhead_frac_of_8tbs": cfg.L * cfg.V * cfg.d * cfg.bpe / (ms / 1e3) / 1e9 / NOMINAL_HBM_GBS,
+                     "nodes_emitted": min(cfg.B, sum(cfg.caps()[1:]))})
+        eng.close()
+    clk = clocks.stop()
+    if rank == 0:
+        line = {"metric": "tree-construction µs/round across the width / budget sweep", "value": total_exp / (total_ms / 1e3),
+                "unit": "node expansions/s (all points)", "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+                "ms_per_step": total_ms / len(pts), "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+                "dtype": "bf16", "data": "synthetic",
+                "config": {"workload": "sweep (Qwen3-4B shape)", "V": pts[0].V, "d": pts[0].d, "L": pts[0].L,
+                           "W": [8, 16, 32, 64], "k": "= W", "B": [32, 128, 512, 1024], "beta": pts[0].beta,
+                           "T": pts[0].temperature, "parallelism": f"replicas x{world}",
+                           "l2": "inputs larger than L2: E (0.78 GB) streamed once per depth"},
+                "sweep": rows, "peak_hbm_gbs": peak, "peak_kind": peak_kind, "gpu_launches": int(launches),
+                "clocks": clk, "e2e": None, "cpu_baseline": None}
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        torch.distributed.destroy_process_group()
+
+
+def ensure_ranks(args):
+    """--gpus N: under torchrun WORLD_SIZE must be N; without it, N > 1
+    relaunches this command as N local ranks (one per GPU) and returns the
+    launcher's exit status."""
+    world = os.environ.get("WORLD_SIZE")
+    if world is not None:
+        if int(world) != args.gpus:
+            sys.stderr.write(f"bench.py: --gpus {args.gpus} but WORLD_SIZE={world}\n")
+            return 2
+        return None
+    if args.gpus <= 1:
+        return None
+    import socket
+    with socket.socket() as sk:
+        sk.bind(("127.0.0.1", 0))
+        port = sk.getsockname()[1]
+    cmd = [sys.executable, "-m", "torch.distributed.run", "--nnodes=1", f"--nproc-per-node={args.gpus}",
+           "--master-addr", "127.0.0.1", "--master-port", str(port), os.path.abspath(__file__)] + sys.argv[1:]
+    return subprocess.run(cmd).returncode
+
+
 def main():
     args = parse()
     if args.warmup < 3:
         args.warmup = 3
+    rc = ensure_ranks(args)
+    if rc is not None:
+        sys.exit(rc)
     from workloads import ATTN_NAMED, NAMED
     if args.config in ATTN_NAMED:
         acfg = ATTN_NAMED[args.config]
@@ -526,7 +759,14 @@ def main():
         else:
             run_verify(args, acfg)
         return
-    cfg = NAMED[args.config]
+    if args.config == "sweep" and args.impl != "reference":
+        run_sweep(args)
+        return
+    if args.config.startswith("table2-") and args.impl != "reference":
+        run_table2(args, NAMED[args.config[len("table2-"):]])
+        return
+    cfg = NAMED[args.config if args.config in NAMED else args.config.split("table2-")[-1]] \
+        if args.config != "sweep" else NAMED["sweep-W16-B128"]
     if args.impl == "reference":
         run_reference(args, cfg)
         return

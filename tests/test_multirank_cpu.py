@@ -105,7 +105,8 @@ def test_reference_arm_under_torchrun_prints_one_line():
     root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
     cmd = [sys.executable, "-m", "torch.distributed.run", "--nnodes=1", "--nproc-per-node", "2",
            "--master-addr", "127.0.0.1", "--master-port", str(free_port()), os.path.join(root, "bench.py"),
-           "--impl", "reference", "--config", "toy", "--steps", "1", "--warmup", "3", "--cpu-seconds", "2"]
+           "--impl", "reference", "--config", "toy", "--gpus", "2", "--steps", "1", "--warmup", "3",
+           "--cpu-seconds", "2"]
     r = subprocess.run(cmd, capture_output=True, text=True, timeout=300, cwd=root)
     assert r.returncode == 0, r.stderr[-2000:]
     lines = [ln for ln in r.stdout.splitlines() if ln.startswith("{")]
@@ -114,3 +115,29 @@ def test_reference_arm_under_torchrun_prints_one_line():
     assert j["impl"] == "reference" and j["n_gpus"] == 2 and j["value"] > 0
     assert j["cpu_baseline"]["kind"] == "oracle" and j["cpu_baseline"]["value"] == j["value"]
     assert j["e2e"]["h2d_bytes_per_step"] == 0 and j["e2e"]["d2h_bytes_per_step"] == 0
+
+
+def test_bench_gpus_flag_spawns_the_ranks_itself():
+    """`bench.py --gpus 2` without a launcher starts two ranks itself (the
+    reference arm: rank 0 prints the one line)."""
+    import json
+    import subprocess
+    import sys
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    env = {k: v for k, v in os.environ.items() if k not in ("RANK", "WORLD_SIZE", "LOCAL_RANK")}
+    cmd = [sys.executable, os.path.join(root, "bench.py"), "--impl", "reference", "--config", "toy", "--gpus", "2",
+           "--steps", "1", "--warmup", "3", "--cpu-seconds", "2"]
+    r = subprocess.run(cmd, capture_output=True, text=True, timeout=300, cwd=root, env=env)
+    assert r.returncode == 0, r.stderr[-2000:]
+    lines = [ln for ln in r.stdout.splitlines() if ln.startswith("{")]
+    assert len(lines) == 1 and json.loads(lines[0])["n_gpus"] == 2
+
+
+def test_bench_refuses_a_world_size_other_than_gpus():
+    import subprocess
+    import sys
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    env = dict(os.environ, WORLD_SIZE="2", RANK="0", LOCAL_RANK="0")
+    cmd = [sys.executable, os.path.join(root, "bench.py"), "--impl", "reference", "--config", "toy", "--gpus", "4"]
+    r = subprocess.run(cmd, capture_output=True, text=True, timeout=120, cwd=root, env=env)
+    assert r.returncode != 0 and "WORLD_SIZE" in r.stderr
