@@ -102,8 +102,14 @@ enum {
  *                      AUTO = ON.  OFF keeps no table (gather + full W_i GEMM)
  *   head_split_stream  with head_split: run the W_i[:, 0:d] GEMM on a second
  *                      stream beside the selection of the children; AUTO = ON
- *   lmhead_ctas_per_sm 1 or 2 LM-head CTAs per SM; 0 = by d (2 if d <= 3072
- *                      and both fit, else 1)
+ *   lmhead_ctas_per_sm 1 or 2 LM-head CTAs per SM; 0 = 2 when both fit and
+ *                      the weights are tiled or d <= 3072, else 1
+ *   weights_tiled      the LM-head streams a copy of E re-laid as 128 x 64
+ *                      tiles of 16 KB contiguous memory (made at
+ *                      dart_init_head: ceil(V/128)*128*d bf16 of workspace)
+ *                      instead of the caller's row-major E; AUTO = ON
+ *   head_weights_tiled the same for the head GEMMs' W_i (its first half with
+ *                      head_split) and W_o (2*d*d or 3*d*d bf16); AUTO = OFF
  *   variants           bit set of DART_VARIANT_* (0: Algorithm 1 only); the
  *                      variants need cand_k = 0 and nseq <= 64, and the
  *                      chain's search keeps L * min(B, V) scores and tokens in
@@ -113,7 +119,7 @@ typedef struct {
     float beta, temperature, rms_eps;
     int pos_offset;
     int cand_k;
-    int head_split, head_split_stream, lmhead_ctas_per_sm;
+    int head_split, head_split_stream, lmhead_ctas_per_sm, weights_tiled, head_weights_tiled;
     int variants;
 } dart_config;
 

@@ -118,6 +118,13 @@ struct dart_handle {
     uint64_t* cand_part;  // [nseq * L][slices][cand_k] per-slice top keys of the candidate selection
     int* cand_rticket;    // [nseq * L] slices finished per row
     float* Qtab;          // [V][d] fp32: Q[t] = W_i[:, d:2d] . E[t] (split first head layer), or null
+    // copies of the streamed weights as 128 x 64 tiles of contiguous 16 KB
+    // (launch_retile), or null: E (weights_tiled), W_i and W_o (head_weights_tiled)
+    bool tiled, wtiled;
+    __nv_bfloat16* Et;    // E [V][d]
+    __nv_bfloat16* Wit;   // W_i[:, 0:Kwi], Kwi = d with the split first layer, else 2d
+    __nv_bfloat16* Wot;   // W_o
+    int Kwi;
     // best-first constructions (dart_config.variants): the one-node-per-
     // sequence plans (W = k = 1) of the chain and of the sequential search
     dart_config ccfg;
@@ -191,7 +198,7 @@ int validate_cfg(const dart_config* c) {
     if (!(c->temperature >= 0.0f) || !std::isfinite(c->temperature)) return DART_ERR_INVALID;
     if (!(c->rms_eps > 0.0f) || !std::isfinite(c->rms_eps)) return DART_ERR_INVALID;
     if (c->cand_k != 0 && (c->cand_k < c->k || c->cand_k > c->V || c->cand_k > kMaxCandK)) return DART_ERR_INVALID;
-    for (int sw : {c->head_split, c->head_split_stream})
+    for (int sw : {c->head_split, c->head_split_stream, c->weights_tiled, c->head_weights_tiled})
         if (sw != DART_AUTO && sw != DART_ON && sw != DART_OFF) return DART_ERR_INVALID;
     if (c->lmhead_ctas_per_sm < 0 || c->lmhead_ctas_per_sm > 2) return DART_ERR_INVALID;
     if (c->variants & ~(DART_VARIANT_CHAIN_DDTREE | DART_VARIANT_SEQ_HEAP)) return DART_ERR_INVALID;
@@ -251,7 +258,7 @@ int build_plans(dart_handle* h, const dart_config& c, std::vector<int>& caps, st
         p.N = c.nseq * p.P;
         if (tc) {
             LmheadPlan lp;
-            if (!plan_lmhead_tc(p.N, c.V, c.d, c.k, h->num_sms, h->smem_optin, c.lmhead_ctas_per_sm, &lp))
+            if (!plan_lmhead_tc(p.N, c.V, c.d, c.k, h->num_sms, h->smem_optin, c.lmhead_ctas_per_sm, h->tiled, &lp))
                 return DART_ERR_UNSUPPORTED;
             p.NG = lp.NG;
             p.G = lp.G;
@@ -347,6 +354,8 @@ int build_plans(dart_handle* h, const dart_config& c, std::vector<int>& caps, st
                 }
                 p.g1.mode = cluster1 ? (p.split ? kGemmSum : kGemmSiluSplit) : kGemmPartials;
                 p.g2.mode = cluster ? kGemmSum : kGemmPartials;
+                p.g1.a_tiled_kb = h->wtiled ? h->Kwi / kBlockK : 0;
+                p.g2.a_tiled_kb = h->wtiled ? c.d / kBlockK : 0;
                 // Candidate-restricted scoring streams nothing through L2
                 // between the depths: with <= 16 children (weight-bound
                 // GEMMs) the largest of {W_i and W_o, W_i (4 d^2 bytes, 2 d^2
@@ -426,6 +435,11 @@ int alloc_workspace(dart_handle* h) {
     bool any_split = false;
     for (int dep = 1; dep < c.L; dep++) any_split = any_split || h->plans[dep].split;
     if (any_split) DART_ALLOC(h->Qtab, static_cast<size_t>(c.V) * d)
+    if (h->tiled) DART_ALLOC(h->Et, static_cast<size_t>((c.V + kTileM - 1) / kTileM) * kTileM * d)
+    if (h->wtiled) {
+        DART_ALLOC(h->Wit, static_cast<size_t>((c.d + kTileM - 1) / kTileM) * kTileM * h->Kwi)
+        DART_ALLOC(h->Wot, static_cast<size_t>((c.d + kTileM - 1) / kTileM) * kTileM * d)
+    }
     const size_t ns = c.nseq, Bp = h->Bp, S1 = static_cast<size_t>(c.B) + 1;
     if (c.variants & DART_VARIANT_CHAIN_DDTREE) {
         DART_ALLOC(h->zrows, ns * c.L * c.V)
@@ -482,30 +496,17 @@ int alloc_workspace(dart_handle* h) {
     for (int dep = 1; dep <= c.L; dep++)
         max_sel = std::max(max_sel, merge_select_smem(h->plans[dep].nlist, h->plans[dep].klist, c.k, c.W));
     if (max_sel > h->smem_optin) return DART_ERR_UNSUPPORTED;
-    if (select_set_smem_limits(std::max(max_sel, 48 * 1024)) != cudaSuccess) return DART_ERR_CUDA;
+    if (select_set_smem_limits() != cudaSuccess) return DART_ERR_CUDA;
     if (c.cand_k > 0) {
-        int score_smem = 48 * 1024;
         for (int dep = 1; dep <= c.L; dep++)
-            score_smem = std::max(score_smem, cand_score_smem(h->plans[dep].P, c.d, h->plans[dep].cand_ds));
+            if (cand_score_smem(h->plans[dep].P, c.d, h->plans[dep].cand_ds) > h->smem_optin - 1024)
+                return DART_ERR_UNSUPPORTED;
         if (cudaMemset(h->cand_ticket, 0, c.nseq * ((c.cand_k + 7) / 8) * sizeof(int)) != cudaSuccess ||
             cudaMemset(h->cand_rticket, 0, static_cast<size_t>(c.nseq) * c.L * sizeof(int)) != cudaSuccess)
             return DART_ERR_CUDA;
-        if (cand_set_smem_limits(std::max(cand_topk_smem(c.cand_k), 48 * 1024), score_smem) != cudaSuccess)
-            return DART_ERR_CUDA;
     }
-    if (c.variants) {
-        // top-K by value over V (the chain's rows, a popped prefix's row); the
-        // candidate top-K of cand_k > 0 shares the kernel: keep the larger limit
-        const int topk = std::max({cand_topk_smem(h->Bp), c.cand_k > 0 ? cand_topk_smem(c.cand_k) : 0, 48 * 1024});
-        int score_smem = 48 * 1024;
-        if (c.cand_k > 0)
-            for (int dep = 1; dep <= c.L; dep++)
-                score_smem = std::max(score_smem, cand_score_smem(h->plans[dep].P, c.d, h->plans[dep].cand_ds));
-        if (cand_set_smem_limits(topk, score_smem) != cudaSuccess) return DART_ERR_CUDA;
-        if ((c.variants & DART_VARIANT_CHAIN_DDTREE) &&
-            heap_set_smem_limits(std::max(ddtree_smem(c.L, h->Bp, c.B), 48 * 1024)) != cudaSuccess)
-            return DART_ERR_CUDA;
-    }
+    if ((c.cand_k > 0 || c.variants) && cand_set_smem_limits() != cudaSuccess) return DART_ERR_CUDA;
+    if ((c.variants & DART_VARIANT_CHAIN_DDTREE) && heap_set_smem_limits() != cudaSuccess) return DART_ERR_CUDA;
     if (h->wdtype == DART_BF16) {
         if (tc_set_smem_limits(h->smem_optin) != cudaSuccess) return DART_ERR_CUDA;
     } else {
@@ -517,8 +518,17 @@ int alloc_workspace(dart_handle* h) {
 int make_tensor_maps(dart_handle* h) {
     const dart_config& c = h->cfg;
     const uint64_t d = c.d;
-    bool ok = encode_bf16_2d(&h->tmE, h->E, d, c.V, kTileM) && encode_bf16_2d(&h->tmWi, h->Wi, 2 * d, d, kTileM) &&
-              encode_bf16_2d(&h->tmWo, h->Wo, d, d, kTileM);
+    // the LM-head's E: [V][d] row-major, or the tiled copy viewed as rows of 64
+    // elements (tile (rt, kb) = rows (rt * d/64 + kb) * 128 .. + 127)
+    auto tiled_rows = [](uint64_t rows, uint64_t cols) {
+        return (rows + kTileM - 1) / kTileM * kTileM * (cols / kBlockK);
+    };
+    bool ok = (h->tiled ? encode_bf16_2d(&h->tmE, h->Et, kBlockK, tiled_rows(c.V, d), kTileM)
+                        : encode_bf16_2d(&h->tmE, h->E, d, c.V, kTileM)) &&
+              (h->wtiled ? encode_bf16_2d(&h->tmWi, h->Wit, kBlockK, tiled_rows(d, h->Kwi), kTileM) &&
+                               encode_bf16_2d(&h->tmWo, h->Wot, kBlockK, tiled_rows(d, d), kTileM)
+                         : encode_bf16_2d(&h->tmWi, h->Wi, 2 * d, d, kTileM) &&
+                               encode_bf16_2d(&h->tmWo, h->Wo, d, d, kTileM));
     const int ngs[3] = {16, 32, 64};
     for (int i = 0; i < 3 && ok; i++) {
         ok = encode_bf16_2d(&h->tmH[i], h->HL, d, 2 * kNPadMax, ngs[i]) &&
@@ -633,6 +643,7 @@ LmheadArgs lmhead_args(const dart_handle* h, const dart_config& c, const DepthPl
     la.status = h->status;
     la.h32 = h32;
     la.E32 = static_cast<const float*>(h->E);
+    la.e_tiled = h->Et ? 1 : 0;
     return la;
 }
 
@@ -1177,6 +1188,9 @@ int dart_init_head(dart_handle** out, const dart_config* cfg, int wdtype, const 
     h->smem_optin = optin;
     h->next_depth = 1;
     if (wdtype == DART_BF16 && tc_set_smem_limits(optin) != cudaSuccess) rc = DART_ERR_CUDA;
+    h->tiled = wdtype == DART_BF16 && cfg->weights_tiled != DART_OFF;
+    h->wtiled = wdtype == DART_BF16 && cfg->head_weights_tiled == DART_ON;
+    h->Kwi = (wdtype == DART_BF16 && cfg->head_split != DART_OFF) ? cfg->d : 2 * cfg->d;
     if (rc == DART_OK) rc = build_plans(h, h->cfg, h->caps, h->plans);
     if (rc == DART_OK && cfg->variants) {
         // the best-first constructions score one node per sequence at a time
@@ -1196,6 +1210,16 @@ int dart_init_head(dart_handle** out, const dart_config* cfg, int wdtype, const 
     if (rc == DART_OK) rc = alloc_workspace(h);
     if (rc == DART_OK && wdtype == DART_BF16) rc = make_tensor_maps(h);
     if (rc == DART_OK && h->Qtab) rc = compute_qtab(h, static_cast<cudaStream_t>(stream));
+    if (rc == DART_OK && (h->tiled || h->wtiled)) {
+        cudaStream_t st0 = static_cast<cudaStream_t>(stream);
+        const __nv_bfloat16* wi = static_cast<const __nv_bfloat16*>(W_i);
+        cudaError_t e = cudaSuccess;
+        if (h->tiled) e = launch_retile(static_cast<const __nv_bfloat16*>(E), cfg->V, cfg->d, cfg->d, h->Et, st0);
+        if (h->wtiled && e == cudaSuccess) e = launch_retile(wi, cfg->d, h->Kwi, 2ll * cfg->d, h->Wit, st0);
+        if (h->wtiled && e == cudaSuccess)
+            e = launch_retile(static_cast<const __nv_bfloat16*>(W_o), cfg->d, cfg->d, cfg->d, h->Wot, st0);
+        rc = cuda_err(e);
+    }
     if (rc == DART_OK && cudaStreamCreateWithFlags(&h->cap_stream, cudaStreamNonBlocking) != cudaSuccess)
         rc = DART_ERR_CUDA;
     if (rc == DART_OK && h->Qtab &&

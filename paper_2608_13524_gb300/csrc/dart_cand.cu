@@ -426,10 +426,9 @@ int cand_score_slices(int P, int d, int nseq, int K, int max_smem) {
 
 int cand_score_smem(int P, int d, int DS) { return P * (d / DS) * 4; }
 
-cudaError_t cand_set_smem_limits(int topk_smem, int score_smem) {
-    cudaError_t e = cudaFuncSetAttribute(cand_topk_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, topk_smem);
-    if (e == cudaSuccess)
-        e = cudaFuncSetAttribute(cand_score_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, score_smem);
+cudaError_t cand_set_smem_limits() {
+    cudaError_t e = set_max_dynamic_smem(reinterpret_cast<const void*>(cand_topk_kernel));
+    if (e == cudaSuccess) e = set_max_dynamic_smem(reinterpret_cast<const void*>(cand_score_kernel));
     return e;
 }
 

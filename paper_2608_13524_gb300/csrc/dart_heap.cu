@@ -283,9 +283,7 @@ __global__ void __launch_bounds__(kHeapThreads) seqheap_emit_kernel(const SeqHea
 
 int ddtree_smem(int L, int Bp, int B) { return (L * Bp * 2 + B * 4 + (B + 1) * 2) * 4; }
 
-cudaError_t heap_set_smem_limits(int ddtree_bytes) {
-    return cudaFuncSetAttribute(ddtree_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, ddtree_bytes);
-}
+cudaError_t heap_set_smem_limits() { return set_max_dynamic_smem(reinterpret_cast<const void*>(ddtree_kernel)); }
 
 cudaError_t launch_ddtree(const DdtArgs& a, cudaStream_t st) {
     return launch_pdl(ddtree_kernel, dim3(a.nseq), dim3(kHeapThreads), ddtree_smem(a.L, a.Bp, a.B), st, a);

@@ -14,6 +14,21 @@ typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t,
                                   CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
 EncodeTiledFn tensor_map_encoder();
 
+// Raises `fn`'s dynamic shared-memory limit to the most the device allows
+// beside the kernel's static shared memory.  Kernel attributes are
+// process-wide: a handle never lowers a limit another handle's plan needs.
+inline cudaError_t set_max_dynamic_smem(const void* fn) {
+    int dev = 0, optin = 0;
+    cudaFuncAttributes fa;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e == cudaSuccess) e = cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
+    if (e == cudaSuccess) e = cudaFuncGetAttributes(&fa, fn);
+    if (e == cudaSuccess)
+        e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 optin - static_cast<int>(fa.sharedSizeBytes));
+    return e;
+}
+
 // Launches `kernel` with programmatic stream serialization (PDL), so its
 // prologue can overlap the tail of the previous kernel in the stream.
 bool pdl_enabled();
@@ -79,6 +94,7 @@ struct LmheadArgs {
     const float* h32;     // fp32 states [N][d] (fp32 kernel)
     const float* E32;     // fp32 table [V][d]   (fp32 kernel)
     uint64_t* gthr;       // [N] cross-CTA top-k bounds, zero before the launch (may be null)
+    int e_tiled;          // the E tensor map is over the tiled copy (launch_retile), not [V][d]
     // optional (null: unused)
     const int* dlog_row;  // [nseq] drafter row of each sequence's nodes (replaces dlog_row_off / V)
     float* zout;          // z[n][v] written to zout[n * zout_stride + v] (node groups <= 64)
@@ -96,6 +112,7 @@ struct GemmArgs {
     int stages;
     int mode;             // tcgen05 path: kGemmPartials, or kGemmSiluSplit / kGemmSum (the k splits are one cluster)
     int keep_a;           // load A (the weights) evict-last: it is read again at the next depth from L2
+    int a_tiled_kb;       // 0: A's tensor map is row-major [M][K]; else over a tiled copy with this many k-blocks per row of tiles
     float* out;           // fp32 path: partials [S][N][M]; kGemmSum: the sum [N][M]
     __nv_bfloat16* outL;  // kGemmSiluSplit: SiLU of the sum as hi rows [N][M], lo rows from row bhalf
     int* status;
@@ -124,12 +141,13 @@ cudaError_t tc_set_smem_limits(int max_dyn);
 
 // Launch plan of the tensor-core LM-head kernel for N nodes: node group NG
 // (16 / 32 / 64 / 128) and G groups, nV vocabulary ranges, pipeline stages
-// and dynamic shared memory; one or two CTAs per SM (ctas_per_sm_pref 1 or 2,
-// 0 = by d).  False if no plan fits the device.
+// and dynamic shared memory; one or two CTAs per SM (ctas_per_sm_pref 1 or 2;
+// 0 = two when E is streamed from its tiled copy or d <= 3072).  False if no
+// plan fits the device.
 struct LmheadPlan {
     int NG, G, nV, stages, smem;
 };
-bool plan_lmhead_tc(int N, int V, int d, int k, int num_sms, int smem_optin, int ctas_per_sm_pref,
+bool plan_lmhead_tc(int N, int V, int d, int k, int num_sms, int smem_optin, int ctas_per_sm_pref, bool e_tiled,
                     LmheadPlan* out);
 
 // fp32 CUDA-core kernels (dart_f32.cu)
@@ -163,7 +181,7 @@ struct SelectArgs {
 };
 cudaError_t launch_merge_select(const SelectArgs& a, cudaStream_t st);
 int merge_select_smem(int nV, int klist, int k, int W);
-cudaError_t select_set_smem_limits(int max_dyn);
+cudaError_t select_set_smem_limits();  // the device maximum (set_max_dynamic_smem)
 
 // candidate-restricted scoring (dart_cand.cu)
 struct CandArgs {
@@ -195,7 +213,7 @@ cudaError_t launch_cand_score(const CandArgs& a, cudaStream_t st);
 int cand_topk_smem(int K);
 int cand_score_slices(int P, int d, int nseq, int K, int max_smem);  // 0: does not fit
 int cand_score_smem(int P, int d, int DS);
-cudaError_t cand_set_smem_limits(int topk_smem, int score_smem);
+cudaError_t cand_set_smem_limits();    // the device maximum for both kernels
 
 struct EmitArgs {
     int L, W, B, nseq, pos_offset;
@@ -224,7 +242,7 @@ struct DdtArgs {
     uint64_t* mask;
 };
 int ddtree_smem(int L, int Bp, int B);
-cudaError_t heap_set_smem_limits(int ddtree_bytes);
+cudaError_t heap_set_smem_limits();    // the device maximum
 cudaError_t launch_ddtree(const DdtArgs& a, cudaStream_t st);
 // Sequential correction with heap: per sequence, slot 0 = the root and slot
 // p + 1 = popped node p: state tab [nseq][B+1][d], sorted children ltok / lz
@@ -254,6 +272,12 @@ struct SeqHeapArgs {
 };
 cudaError_t launch_seqheap_step(const SeqHeapArgs& a, int t, cudaStream_t st);
 cudaError_t launch_seqheap_emit(const SeqHeapArgs& a, cudaStream_t st);
+
+// bf16 [rows][cols] (row pitch `pitch` elements) -> 128 x 64 tiles, each 16 KB contiguous (tile (rt, kb)
+// at index rt * cols / 64 + kb; rows past `rows` zero): every TMA request of
+// the LM-head's E stream then reads one contiguous 16 KB block.
+cudaError_t launch_retile(const __nv_bfloat16* src, int rows, int cols, long long pitch, __nv_bfloat16* dst,
+                          cudaStream_t st);
 
 // One CTA whose bounded mbarrier waits run out (see dart_test_wait_timeout).
 cudaError_t launch_wait_probe(int* status, unsigned long long limit_ns, long long* elapsed_ns, cudaStream_t st);

@@ -94,7 +94,7 @@ int setup_device(int dev, DeviceSetup* out) {
         if (major != 10 || minor != 3) return DART_ERR_UNSUPPORTED;
         void* p = nullptr;
         if (cudaGetSymbolAddress(&p, g_scratch) != cudaSuccess || p == nullptr) return DART_ERR_CUDA;
-        if (tc_set_smem_limits(optin) != cudaSuccess || select_set_smem_limits(optin - 8192) != cudaSuccess)
+        if (tc_set_smem_limits(optin) != cudaSuccess || select_set_smem_limits() != cudaSuccess)
             return DART_ERR_CUDA;
         s.base = static_cast<unsigned char*>(p);
         s.sms = sms;
@@ -135,15 +135,15 @@ extern "C" int dart_expand_root_noalloc(const dart_config* cfg, const void* E, c
     DeviceSetup ds;
     int rc = setup_device(dev, &ds);
     if (rc != DART_OK) return rc;
-    // kernel attributes are process-wide: re-apply limits at least as high as this path needs
-    // (merge_select also has static shared memory, so its dynamic limit stays below optin)
-    if (tc_set_smem_limits(ds.optin) != cudaSuccess || select_set_smem_limits(ds.optin - 8192) != cudaSuccess)
+    // kernel attributes are process-wide: re-apply the device maxima (no call lowers them)
+    if (tc_set_smem_limits(ds.optin) != cudaSuccess || select_set_smem_limits() != cudaSuccess)
         return DART_ERR_CUDA;
 
     // launch plan of depth 1: the handle path's plan (plan_lmhead_tc) for N roots
+    // and a row-major E (this entry point keeps no tiled copy)
     const int N = c.nseq;
     LmheadPlan lp;
-    if (!plan_lmhead_tc(N, c.V, c.d, c.k, ds.sms, ds.optin, c.lmhead_ctas_per_sm, &lp) || lp.G != 1)
+    if (!plan_lmhead_tc(N, c.V, c.d, c.k, ds.sms, ds.optin, c.lmhead_ctas_per_sm, false, &lp) || lp.G != 1)
         return DART_ERR_UNSUPPORTED;
     const int NG = lp.NG, nV = lp.nV;
     const int tiles = (c.V + kTileM - 1) / kTileM;

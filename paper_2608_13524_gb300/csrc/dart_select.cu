@@ -411,9 +411,7 @@ int merge_select_smem(int nV, int klist, int k, int W) {
     return (max(nV * klist, W * k) + kRankMax + 64) * 8 + W * k * 4;
 }
 
-cudaError_t select_set_smem_limits(int max_dyn) {
-    return cudaFuncSetAttribute(merge_select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, max_dyn);
-}
+cudaError_t select_set_smem_limits() { return set_max_dynamic_smem(reinterpret_cast<const void*>(merge_select_kernel)); }
 
 cudaError_t launch_merge_select(const SelectArgs& a, cudaStream_t st) {
     const int smem = merge_select_smem(a.nV, a.klist, a.k, a.W);

@@ -60,7 +60,17 @@ struct Work {
     int kb0, kb1;   // k-block range
     int brow;       // B row of this node group (hi half); lo half at + bhalf
     int lo_kb_end;  // k-blocks >= this carry no lo half
+    int tiled_kb;   // 0: A is row-major [rows][K]; else A is tiled, tile (rt, kb) at rows (rt * tiled_kb + kb) * 128
 };
+
+// TMA coordinates of A tile i (of this CTA's range), k-block kb: in the
+// row-major layout (x = kb * 64, y = row), or in the tiled layout, where the
+// 128 x 64 tile (rt, kb) is 16 KB of contiguous memory, viewed as rows of 64
+// elements: (x = 0, y = (rt * KB + kb) * 128).
+__device__ __forceinline__ int a_x(const Work& w, int kb) { return w.tiled_kb ? 0 : kb * kBlockK; }
+__device__ __forceinline__ int a_y(const Work& w, int i, int kb) {
+    return w.tiled_kb ? ((w.row0 / kTileM + i) * w.tiled_kb + kb) * kTileM : w.row0 + i * kTileM;
+}
 
 template <int NG>
 struct Layout {
@@ -98,12 +108,12 @@ __device__ __forceinline__ void producer(const CUtensorMap* tmA, const CUtensorM
         const int i = static_cast<int>(f) / kbs, kb = w.kb0 + static_cast<int>(f) % kbs;
         const bool lo = kb < w.lo_kb_end;
         mbar_arrive_expect_tx(&full[f], kATileBytes + NG * 128 * (lo ? 2 : 1));
-        tma_load_2d(ring + f * Layout<NG>::kStage, tmA, &full[f], kb * kBlockK, w.row0 + i * kTileM, pol_a);
+        tma_load_2d(ring + f * Layout<NG>::kStage, tmA, &full[f], a_x(w, kb), a_y(w, i, kb), pol_a);
     }
     // and the next `l2pf` into L2, while the previous kernel still runs
     for (uint32_t f = pre; f < pre + static_cast<uint32_t>(l2pf) && f < total; f++) {
         const int i = static_cast<int>(f) / kbs, kb = w.kb0 + static_cast<int>(f) % kbs;
-        tma_prefetch_2d(tmA, kb * kBlockK, w.row0 + i * kTileM);
+        tma_prefetch_2d(tmA, a_x(w, kb), a_y(w, i, kb));
     }
     pdl_wait();
     for (uint32_t f = 0; f < pre; f++) {
@@ -125,7 +135,7 @@ __device__ __forceinline__ void producer(const CUtensorMap* tmA, const CUtensorM
         uint8_t* sA = ring + stage * Layout<NG>::kStage;
         uint8_t* sH = sA + kATileBytes;
         mbar_arrive_expect_tx(&full[stage], kATileBytes + NG * 128 * (lo ? 2 : 1));
-        tma_load_2d(sA, tmA, &full[stage], kb * kBlockK, w.row0 + i * kTileM, pol_a);
+        tma_load_2d(sA, tmA, &full[stage], a_x(w, kb), a_y(w, i, kb), pol_a);
         tma_load_2d(sH, tmB, &full[stage], kb * kBlockK, w.brow, pol_b);
         if (lo) tma_load_2d(sH + NG * 128, tmB, &full[stage], kb * kBlockK, bhalf + w.brow, pol_b);
         fills++;
@@ -295,6 +305,7 @@ __global__ void __launch_bounds__(threads<NG>(), 1)
     w.kb1 = a.d / kBlockK;
     w.brow = g * NG;
     w.lo_kb_end = w.kb1;
+    w.tiled_kb = a.e_tiled ? w.kb1 : 0;
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const uint32_t tmem_base = setup<NG>(s, stages, tmem_cols<NG>());
@@ -460,6 +471,7 @@ __global__ void __launch_bounds__(threads<NG>(), 1)
     w.kb1 = static_cast<int>((static_cast<long long>(split_c + 1) * a.KB) / a.S);
     w.brow = g_c * NG;
     w.lo_kb_end = a.lo_kb_end;
+    w.tiled_kb = a.a_tiled_kb;
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const uint32_t tmem_base = setup<NG>(s, stages, tmem_cols<NG>());
@@ -685,7 +697,7 @@ int lmhead_tc_ctas_per_sm(int NG, int smem) {
     }
 }
 
-bool plan_lmhead_tc(int N, int V, int d, int k, int num_sms, int smem_optin, int ctas_per_sm_pref,
+bool plan_lmhead_tc(int N, int V, int d, int k, int num_sms, int smem_optin, int ctas_per_sm_pref, bool e_tiled,
                     LmheadPlan* out) {
     LmheadPlan p;
     p.NG = N <= 16 ? 16 : (N <= 32 ? 32 : (N <= 64 ? 64 : 128));
@@ -697,12 +709,14 @@ bool plan_lmhead_tc(int N, int V, int d, int k, int num_sms, int smem_optin, int
     auto stages_in = [&](int budget) { return std::min(16, (budget - fixed) / sb); };
     // Two CTAs per SM when both fit with >= 4 pipeline stages each: two
     // independent TMA streams per SM, and one CTA's epilogue / start-up /
-    // tail overlaps the other's stream.  Measured on GB300 it pays for
-    // short rows (d = 2560: -4 % per round) but not for d = 4096, where
-    // the deeper single-CTA pipeline and half as many partial lists win.
+    // tail overlaps the other's stream.  Measured on GB300 (A/B per round):
+    // with E row-major it pays for short rows (d = 2560: -4 %) but not for
+    // d = 4096 (+6 %), where the deeper single-CTA pipeline wins; with E in
+    // contiguous 16 KB tiles two CTAs win at d = 4096 too (-3.6 % against
+    // one CTA on the same tiles, -1.0 % against row-major with one).
     const int st2 = stages_in(smem_optin / 2 - 2048);
     const int smem2 = lmhead_tc_fixed_smem(p.NG, k, st2) + st2 * sb;
-    const bool want2 = ctas_per_sm_pref ? ctas_per_sm_pref == 2 : d <= 3072;
+    const bool want2 = ctas_per_sm_pref ? ctas_per_sm_pref == 2 : (e_tiled || d <= 3072);
     if (want2 && st2 >= 4 && 2 * lmhead_tc_tmem_cols(p.NG) <= 512 && lmhead_tc_ctas_per_sm(p.NG, smem2) >= 2) {
         p.stages = st2;
         p.nV = std::max(1, std::min(2 * num_sms / p.G, tiles));
@@ -755,6 +769,39 @@ cudaError_t launch_gemm_tc(const CUtensorMap* tmA, const CUtensorMap* tmB, const
 
 cudaError_t launch_wait_probe(int* status, unsigned long long limit_ns, long long* elapsed_ns, cudaStream_t st) {
     wait_probe_kernel<<<1, 64, 0, st>>>(status, limit_ns, elapsed_ns);
+    return cudaGetLastError();
+}
+
+namespace {
+
+// dst = src [rows][cols] bf16 (row pitch `pitch`) re-laid as 128 x 64 tiles, tile (rt, kb)
+// (rows 128 rt .., columns 64 kb ..) as 16 KB of contiguous memory at tile
+// index rt * (cols / 64) + kb, rows 128-byte, rows past `rows` zero.  One
+// thread per 16-byte chunk of dst.
+__global__ void retile_kernel(const __nv_bfloat16* src, int rows, int cols, long long pitch, __nv_bfloat16* dst,
+                              long long chunks) {
+    const int KB = cols / kBlockK;
+    for (long long q = blockIdx.x * static_cast<long long>(blockDim.x) + threadIdx.x; q < chunks;
+         q += static_cast<long long>(gridDim.x) * blockDim.x) {
+        const int c8 = static_cast<int>(q & 7);
+        const int r = static_cast<int>((q >> 3) & (kTileM - 1));
+        const long long tile = q >> 10;
+        const long long rt = tile / KB;
+        const int kb = static_cast<int>(tile % KB);
+        const long long row = rt * kTileM + r;
+        uint4 v = make_uint4(0u, 0u, 0u, 0u);
+        if (row < rows) v = *reinterpret_cast<const uint4*>(src + row * pitch + kb * kBlockK + c8 * 8);
+        reinterpret_cast<uint4*>(dst)[q] = v;
+    }
+}
+
+}  // namespace
+
+cudaError_t launch_retile(const __nv_bfloat16* src, int rows, int cols, long long pitch, __nv_bfloat16* dst,
+                          cudaStream_t st) {
+    const long long rt = (rows + kTileM - 1) / kTileM;
+    const long long chunks = rt * (cols / kBlockK) * kTileM * 8;
+    retile_kernel<<<4096, 256, 0, st>>>(src, rows, cols, pitch, dst, chunks);
     return cudaGetLastError();
 }
 

@@ -34,7 +34,8 @@ class DartConfig(C.Structure):
                 ("B", C.c_int), ("nseq", C.c_int), ("beta", C.c_float),
                 ("temperature", C.c_float), ("rms_eps", C.c_float), ("pos_offset", C.c_int),
                 ("cand_k", C.c_int), ("head_split", C.c_int), ("head_split_stream", C.c_int),
-                ("lmhead_ctas_per_sm", C.c_int), ("variants", C.c_int)]
+                ("lmhead_ctas_per_sm", C.c_int), ("weights_tiled", C.c_int), ("head_weights_tiled", C.c_int),
+                ("variants", C.c_int)]
 
 
 class DartTreeOut(C.Structure):
@@ -126,13 +127,13 @@ def _stream(stream):
 def make_config(cfg) -> DartConfig:
     """From any object with V, d, L, W, k, B, nseq, beta, temperature,
     rms_eps, pos_offset and optionally cand_k (0: full vocabulary) and the
-    tuning fields head_split, head_split_stream, lmhead_ctas_per_sm, variants
-    (0: the library's choice)."""
+    tuning fields head_split, head_split_stream, lmhead_ctas_per_sm,
+    weights_tiled, head_weights_tiled, variants (0: the library's choice)."""
     g = lambda name: int(getattr(cfg, name, 0))
     return DartConfig(int(cfg.V), int(cfg.d), int(cfg.L), int(cfg.W), int(cfg.k), int(cfg.B),
                       int(cfg.nseq), float(cfg.beta), float(cfg.temperature), float(cfg.rms_eps),
                       int(cfg.pos_offset), g("cand_k"), g("head_split"), g("head_split_stream"),
-                      g("lmhead_ctas_per_sm"), g("variants"))
+                      g("lmhead_ctas_per_sm"), g("weights_tiled"), g("head_weights_tiled"), g("variants"))
 
 
 def alloc_tree_out(cfg, device="cuda", pin=False):

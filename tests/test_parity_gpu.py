@@ -162,13 +162,15 @@ VARIANT_CFGS = [SMALL[2], SMALL[5], SMALL[6], RESTRICTED[1]]
 
 
 @pytest.mark.parametrize("switch", [dict(head_split=2), dict(head_split_stream=2), dict(lmhead_ctas_per_sm=1),
-                                    dict(lmhead_ctas_per_sm=2)],
-                         ids=["unsplit", "same-stream", "lmhead-1cta", "lmhead-2cta"])
+                                    dict(lmhead_ctas_per_sm=2), dict(weights_tiled=2),
+                                    dict(weights_tiled=2, head_split=2)],
+                         ids=["unsplit", "same-stream", "lmhead-1cta", "lmhead-2cta", "row-major", "row-major-unsplit"])
 @pytest.mark.parametrize("cfg", VARIANT_CFGS, ids=[c.name for c in VARIANT_CFGS])
 def test_head_update_variants(dart, cfg, switch):
     """The variants behind the tuning fields of dart_config: the unsplit first
     head layer (gather of [h_p ; E[t_c]] and the full W_i GEMM, no table), the
-    split layer's GEMM on the main stream, and one or two LM-head CTAs per SM.
+    split layer's GEMM on the main stream, one or two LM-head CTAs per SM, and
+    the caller's row-major weights streamed directly instead of tiled copies.
     Each matches the oracle, and the graph launch equals the depth-by-depth
     calls."""
     cfg = cfg.replace(**switch)
@@ -320,3 +322,28 @@ def test_sweep_oracle_parity(dart, W):
                                        "mask", "prune_gap")})
         rep = compare_with_oracle(cfg, ref, gst, g, tol_of(cfg), x=x)
         report(cfg, rep)
+
+
+def test_handles_with_different_plans_coexist(dart):
+    """Kernel attributes are process-wide: a handle created later with a
+    smaller plan (here one LM-head CTA per SM, half as many partial lists to
+    merge) must not break an earlier handle whose merge needs more shared
+    memory.  Both give the oracle's tree."""
+    big = C("coexist", 1, 20000, 2560, 3, 32, 32, 40, "bf16", 0.0, 81, lmhead_ctas_per_sm=2)
+    small = big.replace(lmhead_ctas_per_sm=1)
+    x = make_inputs(big)
+    dx = to_device(big, x)
+    a = dart.Dart(big, dx["Wi"], dx["Wo"], dx["E"])
+    b = dart.Dart(small, dx["Wi"], dx["Wo"], dx["E"])
+    try:
+        ga = tree_to_numpy(a.build_tree(dx["Dlog"], dx["h0"]))
+        gb = tree_to_numpy(b.build_tree(dx["Dlog"], dx["h0"]))
+        assert dart.dart_status_sync(a.h) == 0 and dart.dart_status_sync(b.h) == 0
+        gst = gpu_supertree(dart, a.h, big)
+    finally:
+        a.close()
+        b.close()
+    ref = oracle.build_tree(big, x["Wi"], x["Wo"], x["E"], x["Dlog"], x["h0"])
+    compare_with_oracle(big, ref, gst, ga, tol_of(big), x=x)
+    for k in ga:
+        np.testing.assert_array_equal(ga[k], gb[k], err_msg=k)

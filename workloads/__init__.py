@@ -59,6 +59,8 @@ class Config:
     head_split: int = 0
     head_split_stream: int = 0
     lmhead_ctas_per_sm: int = 0
+    weights_tiled: int = 0
+    head_weights_tiled: int = 0
     variants: int = 0          # extra constructions prepared by the handle (bit set)
 
     def replace(self, **kw) -> "Config":
