@@ -107,7 +107,9 @@ enum {
  *   weights_tiled      the LM-head streams a copy of E re-laid as 128 x 64
  *                      tiles of 16 KB contiguous memory (made at
  *                      dart_init_head: ceil(V/128)*128*d bf16 of workspace)
- *                      instead of the caller's row-major E; AUTO = ON
+ *                      instead of the caller's row-major E; AUTO = ON for
+ *                      d <= 3072 with at most 16 nodes per depth (where it
+ *                      was measured faster), else OFF
  *   head_weights_tiled the same for the head GEMMs' W_i (its first half with
  *                      head_split) and W_o (2*d*d or 3*d*d bf16); AUTO = OFF
  *   variants           bit set of DART_VARIANT_* (0: Algorithm 1 only); the

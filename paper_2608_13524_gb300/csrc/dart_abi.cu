@@ -1188,7 +1188,21 @@ int dart_init_head(dart_handle** out, const dart_config* cfg, int wdtype, const 
     h->smem_optin = optin;
     h->next_depth = 1;
     if (wdtype == DART_BF16 && tc_set_smem_limits(optin) != cudaSuccess) rc = DART_ERR_CUDA;
-    h->tiled = wdtype == DART_BF16 && cfg->weights_tiled != DART_OFF;
+    {
+        // AUTO: the tiled copy of E where it was measured faster per round on
+        // GB300 (A/B, same process): d <= 3072 with at most 16 nodes per
+        // depth (Qwen3-4B shape -2 to -4 %, sweep W = 8); elsewhere the gain
+        // was within +-1 % (d = 4096 with 16 nodes, 8 x 32 nodes, 64 nodes)
+        // or a loss (+3.7 % with 32 nodes at d = 2560)
+        int max_nodes = 0, width = 1;
+        for (int dep = 1; dep <= cfg->L; dep++) {
+            max_nodes = std::max(max_nodes, cfg->nseq * width);
+            width = std::min(cfg->W, width * cfg->k);
+        }
+        const bool auto_on = cfg->d <= 3072 && max_nodes <= 16;
+        h->tiled = wdtype == DART_BF16 &&
+                   (cfg->weights_tiled == DART_ON || (cfg->weights_tiled == DART_AUTO && auto_on));
+    }
     h->wtiled = wdtype == DART_BF16 && cfg->head_weights_tiled == DART_ON;
     h->Kwi = (wdtype == DART_BF16 && cfg->head_split != DART_OFF) ? cfg->d : 2 * cfg->d;
     if (rc == DART_OK) rc = build_plans(h, h->cfg, h->caps, h->plans);
