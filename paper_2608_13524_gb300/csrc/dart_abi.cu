@@ -71,6 +71,7 @@ struct DepthPlan {
     int l2pf;                            // LM-head: E tiles per CTA prefetched into L2 before its wait
     int nlist, klist;                    // sorted key lists per node and their length (merge input)
     int cand_ds;                         // candidate scoring: d slices per candidate group
+    int f32_ds;                          // fp32 LM-head: blocks per vocabulary range (d slices)
     int Nc, Pn;                          // children (head update) at this depth
     int split;                           // g1 = W_i[:, 0:d] . h over the N parents; E half from the Q table
     int side;                            // split: g1 runs on the side stream beside merge + select
@@ -280,6 +281,11 @@ int build_plans(dart_handle* h, const dart_config& c, std::vector<int>& caps, st
             p.NG = pick_ng_f32(p.N);
             p.G = (p.N + p.NG - 1) / p.NG;
             p.nV = std::max(1, std::min(h->num_sms / p.G, tiles));
+            // fewer vocabulary tiles than SMs: clusters of DS blocks split d
+            // (toy shape, V = 4096: 32 tiles x 4 slices of d = 256)
+            p.f32_ds = 1;
+            while (p.f32_ds < 8 && 2 * p.f32_ds <= c.d / kBlockK && p.nV * p.G * 2 * p.f32_ds <= h->num_sms)
+                p.f32_ds *= 2;
             p.stages = 0;
             p.l2pf = 0;
             p.smem = lmhead_f32_smem(p.NG, c.k);
@@ -644,6 +650,7 @@ LmheadArgs lmhead_args(const dart_handle* h, const dart_config& c, const DepthPl
     la.h32 = h32;
     la.E32 = static_cast<const float*>(h->E);
     la.e_tiled = h->Et ? 1 : 0;
+    la.DS = p.f32_ds > 0 ? p.f32_ds : 1;
     return la;
 }
 
@@ -805,6 +812,15 @@ int enqueue_head_update(dart_handle* h, const dart_config& c, const DepthPlan& p
     const bool tc = h->wdtype == DART_BF16;
     cudaError_t e = cudaSuccess;
     int pi;
+    if (!tc && head_small_f32_slices(c.d) > 0) {
+        // small fp32 heads: the whole update in one launch (one cluster per child)
+        pi = prof_begin(h, kNorm, st);
+        e = launch_head_small_f32(p.Nc, c.d, h->child_prow, h->child_tok, hcur, static_cast<const float*>(h->E),
+                                  static_cast<const float*>(h->Wi), static_cast<const float*>(h->Wo), c.rms_eps, hnext,
+                                  st);
+        prof_end(h, pi, st);
+        return e == cudaSuccess ? DART_OK : DART_ERR_CUDA;
+    }
     if (!p.split) {
         pi = prof_begin(h, kGather, st);
         e = launch_gather_x(p.Nc, c.d, h->child_prow, h->child_tok, hcur, h->E, tc ? 1 : 0, h->XL, kNPadMax, h->X32,

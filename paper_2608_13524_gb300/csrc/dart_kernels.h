@@ -95,6 +95,7 @@ struct LmheadArgs {
     const float* E32;     // fp32 table [V][d]   (fp32 kernel)
     uint64_t* gthr;       // [N] cross-CTA top-k bounds, zero before the launch (may be null)
     int e_tiled;          // the E tensor map is over the tiled copy (launch_retile), not [V][d]
+    int DS;               // fp32 kernel: blocks (one cluster) sharing a vocabulary range, each a slice of d
     // optional (null: unused)
     const int* dlog_row;  // [nseq] drafter row of each sequence's nodes (replaces dlog_row_off / V)
     float* zout;          // z[n][v] written to zout[n * zout_stride + v] (node groups <= 64)
@@ -154,6 +155,13 @@ bool plan_lmhead_tc(int N, int V, int d, int k, int num_sms, int smem_optin, int
 cudaError_t launch_lmhead_f32(const LmheadArgs& a, cudaStream_t st);
 cudaError_t launch_gemm_f32(const GemmArgs& a, cudaStream_t st);
 int lmhead_f32_smem(int NG, int k);
+int lmhead_f32_cw(int N);  // node columns computed for N nodes (4, 8, 16, 32)
+// The whole head update (gather, W_i, SiLU, W_o, residual, RMSNorm) of Nc
+// children in one launch, fp32, d <= 1024: clusters of head_small_f32_slices(d)
+// blocks per child (0 = not applicable).
+int head_small_f32_slices(int d);
+cudaError_t launch_head_small_f32(int Nc, int d, const int* prow, const int* tok, const float* h, const float* E,
+                                  const float* Wi, const float* Wo, float eps, float* hnext, cudaStream_t st);
 cudaError_t f32_set_smem_limits(int max_dyn);
 
 // selection / emission / elementwise kernels (dart_select.cu)

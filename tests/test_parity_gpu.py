@@ -51,6 +51,8 @@ SMALL = [
     C("bf16-manytiles", 1, 320000, 128, 3, 8, 16, 20, "bf16", 1.0, 26),
     C("bf16-k64-many", 1, 200000, 64, 2, 64, 64, 80, "bf16", 0.0, 27),
     C("f32-manytiles", 2, 150000, 64, 3, 16, 16, 30, "f32", 0.0, 28),
+    C("f32-d192", 2, 3000, 192, 4, 6, 4, 15, "f32", 0.5, 29),
+    C("f32-d1024", 1, 2000, 1024, 3, 8, 8, 20, "f32", 0.0, 30),
     TOY,
 ]
 
