@@ -330,7 +330,8 @@ def test_handles_with_different_plans_coexist(dart):
     """Kernel attributes are process-wide: a handle created later with a
     smaller plan (here one LM-head CTA per SM, half as many partial lists to
     merge) must not break an earlier handle whose merge needs more shared
-    memory.  Both give the oracle's tree."""
+    memory.  Both give the oracle's tree (their vocabulary splits differ, so
+    their fp32 sums may differ in the last bits)."""
     big = C("coexist", 1, 20000, 2560, 3, 32, 32, 40, "bf16", 0.0, 81, lmhead_ctas_per_sm=2)
     small = big.replace(lmhead_ctas_per_sm=1)
     x = make_inputs(big)
@@ -342,10 +343,10 @@ def test_handles_with_different_plans_coexist(dart):
         gb = tree_to_numpy(b.build_tree(dx["Dlog"], dx["h0"]))
         assert dart.dart_status_sync(a.h) == 0 and dart.dart_status_sync(b.h) == 0
         gst = gpu_supertree(dart, a.h, big)
+        gstb = gpu_supertree(dart, b.h, small)
     finally:
         a.close()
         b.close()
     ref = oracle.build_tree(big, x["Wi"], x["Wo"], x["E"], x["Dlog"], x["h0"])
     compare_with_oracle(big, ref, gst, ga, tol_of(big), x=x)
-    for k in ga:
-        np.testing.assert_array_equal(ga[k], gb[k], err_msg=k)
+    compare_with_oracle(small, ref, gstb, gb, tol_of(big), x=x)
