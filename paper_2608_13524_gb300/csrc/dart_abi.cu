@@ -69,6 +69,7 @@ int ng_index(int NG) { return NG == 16 ? 0 : (NG == 32 ? 1 : (NG == 64 ? 2 : 3))
 struct DepthPlan {
     int N, P, NG, G, nV, stages, smem;  // LM-head scoring
     int l2pf;                            // LM-head: E tiles per CTA prefetched into L2 before its wait
+    int epf;                             // of those and the stages, how many the previous depth prefetches early
     int nlist, klist;                    // sorted key lists per node and their length (merge input)
     int cand_ds;                         // candidate scoring: d slices per candidate group
     int f32_ds;                          // fp32 LM-head: blocks per vocabulary range (d slices)
@@ -95,6 +96,7 @@ struct dart_handle {
     int wdtype;
     const void *Wi, *Wo, *E;
     int dev, num_sms, smem_optin;
+    long long l2_bytes;   // L2 cache size (plans of the early E prefetch)
     std::vector<int> caps;
     std::vector<DepthPlan> plans;
     int next_depth;  // 1..L+1 (L+1 = all depths expanded)
@@ -277,6 +279,19 @@ int build_plans(dart_handle* h, const dart_config& c, std::vector<int>& caps, st
             p.l2pf = (p.G == 1 && p.NG <= 16)
                          ? static_cast<int>(kL2PrefetchBytes / (static_cast<long long>(kTileM) * kBlockK * 2) / p.nV)
                          : 0;
+            // The previous depth's selection and head update leave HBM idle
+            // for tens of microseconds: a side-stream kernel requests this
+            // launch's first E tiles then, as much as L2 holds beside the
+            // head weights (6 d^2 bytes, re-read every depth).  Measured on
+            // GB300 (tiles per CTA swept, rounds A/B): d = 4096 best near 12
+            // of 37 tiles per CTA (-0.55 %), d = 2560 near 20 of 36 (-3.3 %);
+            // beyond that it evicts the head weights and costs more than it
+            // gains; with several node groups or 32+ nodes it gains nothing.
+            const long long free_l2 = h->l2_bytes - 6ll * c.d * c.d;
+            const long long per_unit = static_cast<long long>(kTileM) * kBlockK * 2 * p.nV;
+            p.epf = (p.l2pf > 0 && free_l2 > 0)
+                        ? static_cast<int>(std::min<long long>(free_l2 / per_unit, p.stages + p.l2pf))
+                        : 0;
         } else {
             p.NG = pick_ng_f32(p.N);
             p.G = (p.N + p.NG - 1) / p.NG;
@@ -288,6 +303,7 @@ int build_plans(dart_handle* h, const dart_config& c, std::vector<int>& caps, st
                 p.f32_ds *= 2;
             p.stages = 0;
             p.l2pf = 0;
+            p.epf = 0;
             p.smem = lmhead_f32_smem(p.NG, c.k);
             if (p.smem > h->smem_optin) return DART_ERR_UNSUPPORTED;
         }
@@ -775,6 +791,14 @@ int enqueue_depth(dart_handle* h, const dart_config& c, const std::vector<DepthP
         g1.status = h->status;
         if (cudaEventRecord(h->ev_fork, st) != cudaSuccess || cudaStreamWaitEvent(h->side, h->ev_fork, 0) != cudaSuccess)
             return DART_ERR_CUDA;
+        // HBM idles while the children are selected: the next LM-head's
+        // first E tiles (its L2-prefetch window) are requested now, beside it
+        if (c.cand_k == 0 && dep < c.L && plans[dep + 1].epf > 0) {
+            const DepthPlan& q = plans[dep + 1];
+            if (launch_lmhead_l2_prefetch(&h->tmE, (c.V + kTileM - 1) / kTileM, q.nV, c.d, q.epf, h->Et ? 1 : 0,
+                                          h->side) != cudaSuccess)
+                return DART_ERR_CUDA;
+        }
         pi = prof_begin(h, kGemm1, h->side);
         e = launch_gemm_tc(&h->tmWi, &h->tmH[ng_index(g1.NG)], g1, p.g1_smem, h->side);
         prof_end(h, pi, h->side);
@@ -1185,11 +1209,12 @@ int dart_init_head(dart_handle** out, const dart_config* cfg, int wdtype, const 
     if (!W_i || !W_o || !E || !aligned16(W_i) || !aligned16(W_o) || !aligned16(E)) return DART_ERR_INVALID;
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess) return DART_ERR_CUDA;
-    int major = 0, minor = 0, sms = 0, optin = 0;
+    int major = 0, minor = 0, sms = 0, optin = 0, l2 = 0;
     if (cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev) != cudaSuccess ||
         cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev) != cudaSuccess ||
         cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
-        cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) != cudaSuccess)
+        cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&l2, cudaDevAttrL2CacheSize, dev) != cudaSuccess)
         return DART_ERR_CUDA;
     if (major != 10 || minor != 3) return DART_ERR_UNSUPPORTED;  // built for sm_103a only
     dart_handle* h = new (std::nothrow) dart_handle();
@@ -1202,6 +1227,7 @@ int dart_init_head(dart_handle** out, const dart_config* cfg, int wdtype, const 
     h->dev = dev;
     h->num_sms = sms;
     h->smem_optin = optin;
+    h->l2_bytes = l2;
     h->next_depth = 1;
     if (wdtype == DART_BF16 && tc_set_smem_limits(optin) != cudaSuccess) rc = DART_ERR_CUDA;
     {

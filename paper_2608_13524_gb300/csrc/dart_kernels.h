@@ -140,6 +140,11 @@ int gemm_tc_ctas_per_sm(int NG, int smem);
 int gemm_tc_max_clusters(int NG, int smem, int cluster);  // resident CTAs per SM (occupancy API; needs limits set)
 cudaError_t tc_set_smem_limits(int max_dyn);
 
+// Prefetch into L2 the first `count` E tiles of each of the nV vocabulary
+// ranges of an LM-head launch (whole-tile split of `tiles` tiles).
+cudaError_t launch_lmhead_l2_prefetch(const CUtensorMap* tmE, int tiles, int nV, int d, int count, int tiled,
+                                      cudaStream_t st);
+
 // Launch plan of the tensor-core LM-head kernel for N nodes: node group NG
 // (16 / 32 / 64 / 128) and G groups, nV vocabulary ranges, pipeline stages
 // and dynamic shared memory; one or two CTAs per SM (ctas_per_sm_pref 1 or 2;

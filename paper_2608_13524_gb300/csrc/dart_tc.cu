@@ -805,4 +805,38 @@ cudaError_t launch_retile(const __nv_bfloat16* src, int rows, int cols, long lon
     return cudaGetLastError();
 }
 
+namespace {
+
+// The first `count` E tiles of every CTA of an LM-head launch (nV vocabulary
+// ranges of whole tiles, the same split as lmhead_tc_kernel) prefetched into
+// L2, one block per range so that every SM's TMA unit issues its own share
+// (one unit issuing them all takes hundreds of microseconds).  Launched beside
+// the selection of the previous depth, while HBM would otherwise wait.
+__global__ void lmhead_l2_prefetch_kernel(const __grid_constant__ CUtensorMap tmE, int tiles, int nV, int KB, int count,
+                                          int tiled) {
+    const int vr = blockIdx.x;
+    if (threadIdx.x != 0 || vr >= nV) return;
+    const int t0 = static_cast<int>((static_cast<long long>(vr) * tiles) / nV);
+    const int t1 = static_cast<int>((static_cast<long long>(vr + 1) * tiles) / nV);
+    Work w;
+    w.ntiles = t1 - t0;
+    w.row0 = t0 * kTileM;
+    w.kb0 = 0;
+    w.kb1 = KB;
+    w.brow = 0;
+    w.lo_kb_end = KB;
+    w.tiled_kb = tiled ? KB : 0;
+    const int total = w.ntiles * KB;
+    for (int f = 0; f < count && f < total; f++) tma_prefetch_2d(&tmE, a_x(w, f % KB), a_y(w, f / KB, f % KB));
+}
+
+}  // namespace
+
+cudaError_t launch_lmhead_l2_prefetch(const CUtensorMap* tmE, int tiles, int nV, int d, int count, int tiled,
+                                      cudaStream_t st) {
+    const int KB = d / kBlockK;
+    lmhead_l2_prefetch_kernel<<<nV, 32, 0, st>>>(*tmE, tiles, nV, KB, count, tiled);
+    return cudaGetLastError();
+}
+
 }  // namespace dart
