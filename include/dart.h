@@ -64,7 +64,8 @@ typedef enum {
     DART_ERR_NOMEM = -3,       /* device or host allocation failed */
     DART_ERR_TIMEOUT = -4,     /* a device-side wait gave up (reported by dart_status_sync) */
     DART_ERR_STATE = -5,       /* call out of order (e.g. depth skipped) */
-    DART_ERR_UNSUPPORTED = -6  /* device is not sm_103 / missing driver entry point */
+    DART_ERR_UNSUPPORTED = -6, /* device is not sm_103 / missing driver entry point */
+    DART_ERR_BOUNDS = -7       /* debug builds only: a device index check failed (dart_status_sync) */
 } dart_status;
 
 typedef enum { DART_F32 = 0, DART_BF16 = 1 } dart_dtype;
@@ -256,8 +257,23 @@ int dart_get_node_topk(dart_handle *h, int32_t *tok, float *logq, float *lse, in
 int dart_get_states(dart_handle *h, float *states, int *rows, void *stream);
 
 /* Synchronises `stream` and returns (then clears) the device status word:
- * DART_OK, or DART_ERR_TIMEOUT if a kernel's bounded wait gave up. */
+ * DART_OK, DART_ERR_TIMEOUT if a kernel's bounded wait gave up, or (debug
+ * builds) DART_ERR_BOUNDS if a data-dependent index failed its check. */
 int dart_status_sync(dart_handle *h, void *stream);
+
+/* 1 in a library compiled with -DDART_DEBUG, else 0.  Debug builds check
+ * every data-dependent index of the selection, emission, gather and heap
+ * kernels (parent slots against the previous depth's count, token ids
+ * against V, output positions against B) before it is used: a failing check
+ * skips the access and sets a bit of the handle's status word, which the next
+ * dart_status_sync returns as DART_ERR_BOUNDS; nothing traps. */
+int dart_debug_build(void);
+
+/* Test hook of the debug checks: one thread evaluates one failing index
+ * check (an index equal to its bound) on `stream`, touching no memory but
+ * the status word.  Debug builds: the next dart_status_sync returns
+ * DART_ERR_BOUNDS; release builds: DART_OK (the checks compile away). */
+int dart_test_bounds_report(dart_handle *h, void *stream);
 
 /* Test hook for the failure path of the bounded device waits (no fault is
  * made): one CTA waits on an mbarrier that nothing completes, with the same

@@ -877,7 +877,7 @@ int enqueue_head_update(dart_handle* h, const dart_config& c, const DepthPlan& p
         pi = prof_begin(h, kGatherSilu, st);
         // (a cluster GEMM wrote the summed U: one "split")
         e = launch_gather_silu(p.Nc, c.d, g1.mode == kGemmPartials ? g1.S : 1, g1.N, h->part, h->child_prow,
-                               h->child_tok, c.V, h->Qtab, h->AL, kNPadMax, st);
+                               h->child_tok, c.V, h->Qtab, h->AL, kNPadMax, h->status, st);
         prof_end(h, pi, st);
         if (e != cudaSuccess) return DART_ERR_CUDA;
     } else if (!fused) {
@@ -988,6 +988,7 @@ int enqueue_chain_ddtree(dart_handle* h, const float* dlog, const float* anchor,
     a.n_nodes = out->n_nodes;
     a.scores = out->scores;
     a.mask = out->mask;
+    a.status = h->status;
     pi = prof_begin(h, kDdtree, st);
     e = launch_ddtree(a, st);
     prof_end(h, pi, st);
@@ -1037,6 +1038,7 @@ int enqueue_seq_heap(dart_handle* h, const float* dlog, const float* anchor, con
     a.n_nodes = out->n_nodes;
     a.scores = out->scores;
     a.mask = out->mask;
+    a.status = h->status;
     // scoring of one node per sequence, its best Bp children into slot `slot`
     auto score = [&](int slot, const float* h32, const int* dlog_row, bool first) -> int {
         LmheadArgs la = lmhead_args(h, cc, p, dlog, h32);
@@ -1195,6 +1197,7 @@ const char* dart_status_string(int code) {
         case DART_ERR_TIMEOUT: return "device wait timed out";
         case DART_ERR_STATE: return "call out of order";
         case DART_ERR_UNSUPPORTED: return "unsupported device or configuration";
+        case DART_ERR_BOUNDS: return "device index check failed (debug build)";
         default: return "unknown status";
     }
 }
@@ -1459,8 +1462,16 @@ int dart_status_sync(dart_handle* h, void* stream) {
     if (cudaMemcpy(&word, h->status, sizeof word, cudaMemcpyDeviceToHost) != cudaSuccess) return DART_ERR_CUDA;
     if (cudaMemset(h->status, 0, sizeof word) != cudaSuccess) return DART_ERR_CUDA;
     if (word & kDevTimeout) return DART_ERR_TIMEOUT;
+    if (word & kDevBounds) return DART_ERR_BOUNDS;
     if (word & kDevOrphan) return DART_ERR_STATE;
     return DART_OK;
+}
+
+int dart_debug_build(void) { return debug_build() ? 1 : 0; }
+
+int dart_test_bounds_report(dart_handle* h, void* stream) {
+    if (!h) return DART_ERR_INVALID;
+    return cuda_err(launch_bounds_probe(h->status, static_cast<cudaStream_t>(stream)));
 }
 
 int dart_test_wait_timeout(dart_handle* h, int limit_us, int64_t* elapsed_ns, void* stream) {

@@ -15,6 +15,23 @@ namespace dart {
 // Device status word bits (read back by dart_status_sync).
 constexpr int kDevTimeout = 1;      // a bounded wait gave up
 constexpr int kDevOrphan = 2;       // pruning kept a node whose parent was cut (impossible for beta <= 0)
+constexpr int kDevBounds = 4;       // debug builds: a data-dependent index failed its check
+
+// Debug builds (-DDART_DEBUG) check data-dependent indices (parent slots,
+// token ids, output positions) before they are used: a failed check sets
+// kDevBounds in the status word and the caller skips the access, so the
+// context stays usable and dart_status_sync reports DART_ERR_BOUNDS.
+// Release builds compile the checks away (the function returns true).
+__device__ __forceinline__ bool bounds_check(int* status, bool ok) {
+#ifdef DART_DEBUG
+    if (!ok && status) atomicOr(status, kDevBounds);
+    return ok;
+#else
+    (void)status;
+    (void)ok;
+    return true;
+#endif
+}
 
 // A wait that has not completed after this long means a bug; give up.
 constexpr unsigned long long kWaitLimitNs = 2000000000ull;  // 2 s

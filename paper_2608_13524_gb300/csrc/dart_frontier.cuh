@@ -39,6 +39,7 @@ __device__ __forceinline__ void select_frontier(const SelectArgs& a, int s, int 
         if (r < cnt) {
             const uint64_t x = top[r];
             const int c = static_cast<int>(key_idx(x));
+            if (!bounds_check(a.status, c < ncand)) continue;
             const int pp = c / a.k;
             const int tok = ctok[c];
             a.tree_tok[tb + r] = tok;

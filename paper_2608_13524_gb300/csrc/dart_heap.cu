@@ -119,7 +119,8 @@ __global__ void __launch_bounds__(kHeapThreads) ddtree_kernel(const DdtArgs a) {
             const float sc = key_val(k);
             const int dep = o == 0 ? 1 : ndep[o - 1] + 1;
             if (lane == 0) {
-                const int c = next[o];
+                int c = next[o];
+                if (!bounds_check(a.status, c < Bp && dep <= L)) c = 0;
                 ntok[n] = tk[(dep - 1) * Bp + c];
                 npar[n] = o - 1;
                 ndep[n] = dep;
@@ -221,8 +222,9 @@ __global__ void __launch_bounds__(kHeapThreads) seqheap_step_kernel(const SeqHea
                 const int o = static_cast<int>(key_idx(best));
                 const float sc = key_val(best);
                 const size_t lb = static_cast<size_t>(s) * S1 + o;
-                const int c = next[o];
+                int c = next[o];
                 const int dep = o == 0 ? 1 : a.depths[ob + o - 1] + 1;
+                if (!bounds_check(a.status, c < Bp && o <= n && dep <= L)) c = 0;
                 const int tok = a.ltok[lb * Bp + c];
                 a.tokens[ob + n] = tok;
                 a.parents[ob + n] = o - 1;

@@ -253,6 +253,7 @@ struct DdtArgs {
     int *tokens, *parents, *depths, *pos_ids, *n_nodes;
     float* scores;
     uint64_t* mask;
+    int* status;
 };
 int ddtree_smem(int L, int Bp, int B);
 cudaError_t heap_set_smem_limits();    // the device maximum
@@ -282,6 +283,7 @@ struct SeqHeapArgs {
     int *tokens, *parents, *depths, *pos_ids, *n_nodes;
     float* scores;
     uint64_t* mask;
+    int* status;
 };
 cudaError_t launch_seqheap_step(const SeqHeapArgs& a, int t, cudaStream_t st);
 cudaError_t launch_seqheap_emit(const SeqHeapArgs& a, cudaStream_t st);
@@ -306,7 +308,10 @@ cudaError_t launch_silu_split(int Nc, int d, int S, const float* part, __nv_bflo
                               cudaStream_t st);
 // a = SiLU(Q[tok[c]] + sum_s part[s][prow[c]]) -> AL (hi/lo); part: [S][Np][d]
 cudaError_t launch_gather_silu(int Nc, int d, int S, int Np, const float* part, const int* prow, const int* tok,
-                               int V, const float* Q, __nv_bfloat16* AL, int bhalf, cudaStream_t st);
+                               int V, const float* Q, __nv_bfloat16* AL, int bhalf, int* status, cudaStream_t st);
+// debug builds (-DDART_DEBUG): one failing index check, reported through `status`
+cudaError_t launch_bounds_probe(int* status, cudaStream_t st);
+bool debug_build();
 // h_next[c] = RMSNorm(h[prow[c]] + sum_s part[s][c]) and its hi/lo split
 cudaError_t launch_residual_norm(int Nc, int d, int S, const float* part, const int* prow, const float* h,
                                  float eps, float* h_next, __nv_bfloat16* HL, int bhalf, cudaStream_t st);

@@ -22,6 +22,7 @@ DART_ERR_NOMEM = -3
 DART_ERR_TIMEOUT = -4
 DART_ERR_STATE = -5
 DART_ERR_UNSUPPORTED = -6
+DART_ERR_BOUNDS = -7
 DART_F32 = 0
 DART_BF16 = 1
 DART_AUTO, DART_ON, DART_OFF = 0, 1, 2
@@ -56,6 +57,15 @@ class DartError(RuntimeError):
 
 
 _lib = None
+_empty = torch.empty
+
+
+def set_output_allocator(fn=None):
+    """Allocator of the device output tensors this module creates (same
+    signature as torch.empty; None restores torch.empty).  Tests pass one
+    that surrounds every output with guard bytes."""
+    global _empty
+    _empty = torch.empty if fn is None else fn
 
 
 def lib():
@@ -81,6 +91,8 @@ def lib():
             "dart_get_states": (i, [vp, vp, C.POINTER(i), vp]),
             "dart_status_sync": (i, [vp, vp]),
             "dart_test_wait_timeout": (i, [vp, i, vp, vp]),
+            "dart_debug_build": (i, []),
+            "dart_test_bounds_report": (i, [vp, vp]),
             "dart_noalloc_status": (i, [vp]),
             "dart_set_profiling": (i, [vp, i]),
             "dart_profile_read": (i, [vp, C.POINTER(f), C.POINTER(i)]),
@@ -141,15 +153,17 @@ def alloc_tree_out(cfg, device="cuda", pin=False):
     ns, B = cfg.nseq, cfg.B
     nw = (B + 63) // 64
     kw = dict(device=device)
+    new = _empty
     if pin:
         kw = dict(device="cpu", pin_memory=True)
-    t = dict(tokens=torch.empty((ns, B), dtype=torch.int32, **kw),
-             parents=torch.empty((ns, B), dtype=torch.int32, **kw),
-             depths=torch.empty((ns, B), dtype=torch.int32, **kw),
-             pos_ids=torch.empty((ns, B), dtype=torch.int32, **kw),
-             scores=torch.empty((ns, B), dtype=torch.float32, **kw),
-             n_nodes=torch.empty((ns,), dtype=torch.int32, **kw),
-             mask=torch.empty((ns, B, nw), dtype=torch.int64, **kw))
+        new = torch.empty
+    t = dict(tokens=new((ns, B), dtype=torch.int32, **kw),
+             parents=new((ns, B), dtype=torch.int32, **kw),
+             depths=new((ns, B), dtype=torch.int32, **kw),
+             pos_ids=new((ns, B), dtype=torch.int32, **kw),
+             scores=new((ns, B), dtype=torch.float32, **kw),
+             n_nodes=new((ns,), dtype=torch.int32, **kw),
+             mask=new((ns, B, nw), dtype=torch.int64, **kw))
     out = DartTreeOut(*(t[k].data_ptr() for k in
                         ("tokens", "parents", "depths", "pos_ids", "scores", "n_nodes", "mask")))
     return t, out
@@ -202,8 +216,8 @@ def dart_build_seq_heap(h, drafter_logits, anchor_h, out: DartTreeOut, stream=No
 def dart_get_chain(h, cfg, stream=None):
     """(chain tokens [nseq][L] int32, log-sum-exp [nseq][L] float) after
     dart_build_chain_ddtree."""
-    tok = torch.empty((cfg.nseq, cfg.L), dtype=torch.int32, device="cuda")
-    lse = torch.empty((cfg.nseq, cfg.L), dtype=torch.float32, device="cuda")
+    tok = _empty((cfg.nseq, cfg.L), dtype=torch.int32, device="cuda")
+    lse = _empty((cfg.nseq, cfg.L), dtype=torch.float32, device="cuda")
     _check(lib().dart_get_chain(h, _ptr(tok), _ptr(lse), _stream(stream)), "dart_get_chain")
     return tok, lse
 
@@ -215,10 +229,10 @@ def dart_build_tree_host(h, drafter_logits_host, anchor_host, out_host: DartTree
 
 def dart_get_frontier(h, depth, cfg, stream=None):
     dev = "cuda"
-    tok = torch.empty((cfg.nseq, cfg.W), dtype=torch.int32, device=dev)
-    par = torch.empty_like(tok)
-    score = torch.empty((cfg.nseq, cfg.W), dtype=torch.float32, device=dev)
-    count = torch.empty((cfg.nseq,), dtype=torch.int32, device=dev)
+    tok = _empty((cfg.nseq, cfg.W), dtype=torch.int32, device=dev)
+    par = _empty(tok.shape, dtype=tok.dtype, device=tok.device)
+    score = _empty((cfg.nseq, cfg.W), dtype=torch.float32, device=dev)
+    count = _empty((cfg.nseq,), dtype=torch.int32, device=dev)
     _check(lib().dart_get_frontier(h, int(depth), _ptr(tok), _ptr(par), _ptr(score), _ptr(count),
                                    _stream(stream)), "dart_get_frontier")
     return tok, par, score, count
@@ -229,9 +243,9 @@ def dart_get_node_topk(h, cfg, stream=None):
     _check(lib().dart_get_node_topk(h, None, None, None, C.byref(rows), _stream(stream)),
            "dart_get_node_topk")
     n = rows.value
-    tok = torch.empty((n, cfg.k), dtype=torch.int32, device="cuda")
-    logq = torch.empty((n, cfg.k), dtype=torch.float32, device="cuda")
-    lse = torch.empty((n,), dtype=torch.float32, device="cuda")
+    tok = _empty((n, cfg.k), dtype=torch.int32, device="cuda")
+    logq = _empty((n, cfg.k), dtype=torch.float32, device="cuda")
+    lse = _empty((n,), dtype=torch.float32, device="cuda")
     _check(lib().dart_get_node_topk(h, _ptr(tok), _ptr(logq), _ptr(lse), C.byref(rows),
                                     _stream(stream)), "dart_get_node_topk")
     return tok, logq, lse
@@ -240,13 +254,21 @@ def dart_get_node_topk(h, cfg, stream=None):
 def dart_get_states(h, cfg, stream=None):
     rows = C.c_int()
     _check(lib().dart_get_states(h, None, C.byref(rows), _stream(stream)), "dart_get_states")
-    st = torch.empty((rows.value, cfg.d), dtype=torch.float32, device="cuda")
+    st = _empty((rows.value, cfg.d), dtype=torch.float32, device="cuda")
     _check(lib().dart_get_states(h, _ptr(st), C.byref(rows), _stream(stream)), "dart_get_states")
     return st
 
 
 def dart_status_sync(h, stream=None):
     return int(lib().dart_status_sync(h, _stream(stream)))
+
+
+def dart_debug_build() -> bool:
+    return bool(lib().dart_debug_build())
+
+
+def dart_test_bounds_report(h, stream=None):
+    _check(lib().dart_test_bounds_report(h, _stream(stream)), "dart_test_bounds_report")
 
 
 def dart_test_wait_timeout(h, limit_us, elapsed_ns=None, stream=None):
@@ -400,9 +422,9 @@ class TreeAttention:
         n = dart_tree_attention_workspace(self.cfg)
         if n == 0:
             raise DartError(DART_ERR_INVALID, "dart_tree_attention_workspace")
-        self.workspace = torch.empty(n, dtype=torch.uint8, device="cuda")
+        self.workspace = _empty((n,), dtype=torch.uint8, device="cuda")
         c = self.cfg
-        self.out = torch.empty((c.nseq, c.B, c.Hq, c.dh), dtype=torch.float32, device="cuda")
+        self.out = _empty((c.nseq, c.B, c.Hq, c.dh), dtype=torch.float32, device="cuda")
 
     def __call__(self, q, k_tree, v_tree, k_ctx, v_ctx, pos_ids, mask, n_nodes, status=None, stream=None):
         dart_tree_attention(self.cfg, q, k_tree, v_tree, k_ctx, v_ctx, pos_ids, mask, n_nodes, self.out,

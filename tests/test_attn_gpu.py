@@ -19,6 +19,7 @@ import numpy as np
 import pytest
 import torch
 
+import canary
 from oracle import tree_attn as ta
 from workloads import ATTN_BATCHED, ATTN_Q4B, ATTN_Q8B, AttnConfig, bf16_bits_to_f32, make_attn_inputs
 
@@ -53,7 +54,7 @@ def gpu_attention(dart, cfg: AttnConfig, x, mask=None, pos_ids=None, n_nodes=Non
     nn = torch.from_numpy(x["n_nodes"]).to(dev) if n_nodes is None else n_nodes
     if mask is None:
         mw = (cfg.B + 63) // 64
-        mask = torch.empty((cfg.nseq, cfg.B, mw), dtype=torch.int64, device=dev)
+        mask = canary.empty((cfg.nseq, cfg.B, mw), dtype=torch.int64, device=dev)
         dart.dart_ancestor_mask(par, nn, mask)
     if pos_ids is None:
         dep = torch.from_numpy(x["depths"]).to(dev)
@@ -135,7 +136,7 @@ def test_ancestor_mask_matches_paths(dart):
     par = torch.from_numpy(x["parents"]).cuda()
     nn = torch.from_numpy(x["n_nodes"]).cuda()
     mw = (cfg.B + 63) // 64
-    mask = torch.empty((cfg.nseq, cfg.B, mw), dtype=torch.int64, device="cuda")
+    mask = canary.empty((cfg.nseq, cfg.B, mw), dtype=torch.int64, device="cuda")
     dart.dart_ancestor_mask(par, nn, mask)
     m = mask.cpu().numpy().view(np.uint64)
     for s in range(cfg.nseq):

@@ -12,6 +12,7 @@ import numpy as np
 import pytest
 import torch
 
+import canary
 from parity import to_device, tol_of
 from workloads import Config, make_inputs
 
@@ -41,11 +42,11 @@ def handle_depth1(dart, cfg, dx):
 
 
 def outputs(nseq, W, k):
-    """Output tensors pre-filled with values no correct call leaves behind."""
-    return [torch.full((nseq, k), -7, dtype=torch.int32, device="cuda"),
-            torch.full((nseq, k), 7.0, device="cuda"), torch.full((nseq,), 7.0, device="cuda"),
-            torch.full((nseq, W), -7, dtype=torch.int32, device="cuda"),
-            torch.full((nseq, W), 7.0, device="cuda"), torch.full((nseq,), -7, dtype=torch.int32, device="cuda")]
+    """Output tensors pre-filled with values no correct call leaves behind,
+    each between guard bytes (checked when the test ends)."""
+    spec = [((nseq, k), torch.int32, -7), ((nseq, k), torch.float32, 7.0), ((nseq,), torch.float32, 7.0),
+            ((nseq, W), torch.int32, -7), ((nseq, W), torch.float32, 7.0), ((nseq,), torch.int32, -7)]
+    return [canary.empty(shape, dtype=dt, device="cuda").fill_(v) for shape, dt, v in spec]
 
 
 def dirty_the_array(dart):
