@@ -116,7 +116,19 @@ enum {
  *   variants           bit set of DART_VARIANT_* (0: Algorithm 1 only); the
  *                      variants need cand_k = 0 and nseq <= 64, and the
  *                      chain's search keeps L * min(B, V) scores and tokens in
- *                      shared memory (DART_ERR_UNSUPPORTED beyond 227 KB) */
+ *                      shared memory (DART_ERR_UNSUPPORTED beyond 227 KB)
+ *   fused_round        fp32 weights: dart_build_tree runs the whole round
+ *                      (every depth's scoring, merge, selection and head
+ *                      update, then prune and emit) as one cooperative
+ *                      kernel, one block per SM with grid-wide barriers,
+ *                      instead of a graph of per-step launches.  Possible
+ *                      with cand_k = 0, at most 32 nodes per depth
+ *                      (nseq * W <= 32), L <= 32, L * W <= 256, k <= 32,
+ *                      d <= 1024, V <= 65536 and the node states and
+ *                      per-block scores within shared memory; AUTO = ON
+ *                      where possible, ON = DART_ERR_UNSUPPORTED where not.
+ *                      The depth-by-depth calls always take the per-step
+ *                      launches (results agree within fp32 rounding) */
 typedef struct {
     int V, d, L, W, k, B, nseq;
     float beta, temperature, rms_eps;
@@ -124,6 +136,7 @@ typedef struct {
     int cand_k;
     int head_split, head_split_stream, lmhead_ctas_per_sm, weights_tiled, head_weights_tiled;
     int variants;
+    int fused_round;
 } dart_config;
 
 /* Emitted verification tree, caller-allocated, per sequence s:
@@ -261,6 +274,16 @@ int dart_get_states(dart_handle *h, float *states, int *rows, void *stream);
  * builds) DART_ERR_BOUNDS if a data-dependent index failed its check. */
 int dart_status_sync(dart_handle *h, void *stream);
 
+/* Test hook of the fused round's grid barrier (handles with fused_round in
+ * effect, else DART_ERR_STATE): two blocks wait at the handle's barrier for
+ * a third that never comes, each gives up after limit_us microseconds
+ * (1 <= limit_us <= 2000000) and sets the DART_ERR_TIMEOUT bit; nothing else
+ * is touched.  The next dart_status_sync returns DART_ERR_TIMEOUT and resets
+ * the barrier, after which the handle's rounds run normally again (before
+ * it, dart_build_tree returns DART_ERR_STATE).  A fused round whose barrier
+ * gave up on its own is reported and reset the same way. */
+int dart_test_barrier_timeout(dart_handle *h, int limit_us, void *stream);
+
 /* 1 in a library compiled with -DDART_DEBUG, else 0.  Debug builds check
  * every data-dependent index of the selection, emission, gather and heap
  * kernels (parent slots against the previous depth's count, token ids
@@ -302,8 +325,10 @@ int dart_profile_read(dart_handle *h, float *lmhead_ms, int *lmhead_launches);
  * depth), 11 gather of the per-token table row + SiLU + split (split first
  * layer), 12 top-K by value over a row of scaled logits (the best-first
  * constructions), 13 DDTree search, 14 one pop of the sequential search,
- * 15 its emission.  ms[i] / launches[i] receive the summed device time and
- * count of kind i for i < nkinds (nkinds <= 16); resets the events. */
+ * 15 its emission, 16 the fused small-problem round (fused_round: one
+ * launch per round), 17 the early L2 prefetch of the next depth's first E
+ * tiles (side stream).  ms[i] / launches[i] receive the summed device time
+ * and count of kind i for i < nkinds (nkinds <= 18); resets the events. */
 int dart_profile_read_kinds(dart_handle *h, float *ms, int *launches, int nkinds);
 
 /* Number of kernel launches one dart_build_tree enqueues for this handle. */

@@ -153,6 +153,21 @@ struct dart_handle {
     uint64_t* sh_part;     // [nseq][topk_S][Bp]
     int* sh_ticket;        // [nseq]
     int last_kind;         // construction of the most recent round (RoundKind)
+    // fused small-problem round (dart_config.fused_round): one cooperative
+    // kernel of fused_G blocks, each scoring at most fused_R vocabulary rows
+    bool fused;
+    bool fused_cluster;    // one cluster per sequence (else one cooperative grid)
+    int fused_nm, fused_G, fused_R;
+    bool fused_ecache, fused_mstage;
+    int fused_stage;       // cluster form: bytes per E stage
+    bool fused_wres;       // cluster form: head weights resident in shared memory
+    size_t fused_smem;
+    float *f_rbuf, *f_abuf, *f_ssqp;
+    float2* f_pms;
+    uint64_t* f_pkey;
+    unsigned* f_bar;       // grid barrier: arrivals, generation
+    int* f_abort;
+    bool f_dirty;          // the barrier probe left the barrier mid-way (until dart_status_sync)
     std::vector<void*> allocs;
     CUtensorMap tmE, tmWi, tmWo, tmH[4], tmX[3], tmA[3];
     CUtensorMap tmWiR, tmEB;  // Q table: A = W_i[:, d:2d] (128-row box), B = E rows as 64-node groups
@@ -201,7 +216,7 @@ int validate_cfg(const dart_config* c) {
     if (!(c->temperature >= 0.0f) || !std::isfinite(c->temperature)) return DART_ERR_INVALID;
     if (!(c->rms_eps > 0.0f) || !std::isfinite(c->rms_eps)) return DART_ERR_INVALID;
     if (c->cand_k != 0 && (c->cand_k < c->k || c->cand_k > c->V || c->cand_k > kMaxCandK)) return DART_ERR_INVALID;
-    for (int sw : {c->head_split, c->head_split_stream, c->weights_tiled, c->head_weights_tiled})
+    for (int sw : {c->head_split, c->head_split_stream, c->weights_tiled, c->head_weights_tiled, c->fused_round})
         if (sw != DART_AUTO && sw != DART_ON && sw != DART_OFF) return DART_ERR_INVALID;
     if (c->lmhead_ctas_per_sm < 0 || c->lmhead_ctas_per_sm > 2) return DART_ERR_INVALID;
     if (c->variants & ~(DART_VARIANT_CHAIN_DDTREE | DART_VARIANT_SEQ_HEAP)) return DART_ERR_INVALID;
@@ -249,6 +264,105 @@ int tc_stages(int smem_optin, int stage_bytes, int fixed) {
 
 // Launch plans of every depth for configuration c (the handle's, or the
 // one-node-per-sequence configuration of the best-first constructions).
+// Whether dart_build_tree runs as one cooperative kernel (fused_round): fp32
+// weights, full-vocabulary scoring, at most 32 nodes per depth, and the
+// kernel's shared memory (node states, per-block score keys, selection
+// buffers) within the device limit; one block per SM, at most 160.
+int plan_fused_round(dart_handle* h) {
+    const dart_config& c = h->cfg;
+    h->fused = false;
+    if (c.fused_round == DART_OFF) return DART_OK;
+    int nmax = 0, pmax = 0;
+    for (int dep = 1; dep <= c.L; dep++) {
+        nmax = std::max(nmax, c.nseq * h->caps[dep - 1]);
+        pmax = std::max(pmax, h->caps[dep - 1]);
+    }
+    const bool base_ok = h->wdtype == DART_F32 && c.cand_k == 0 && c.W <= 32 && c.L <= kRoundMaxL &&
+                         c.L * c.W <= 256 && c.k <= 32 && c.d <= 1024;
+    // the kernel's static shared memory (prune / emit and selection scratch) is below 32 KB
+    const size_t avail = static_cast<size_t>(h->smem_optin) - 32 * 1024;
+    {
+        // one cluster per sequence: where a block's share of E (re-read at
+        // every depth) is at most 512 KB and the sequence's states and slice
+        // keys fit in shared memory
+        const int pm = round_small_nm(pmax);
+        const int R = (c.V + kRoundCluster - 1) / kRoundCluster;
+        if (base_ok && pm > 0 && c.W * c.k <= 256 && static_cast<size_t>(R) * c.d * 4 <= 512 * 1024 &&
+            pm * c.d <= 16384 && static_cast<size_t>(pm) * R * 8 <= 64 * 1024) {
+            // E streams through two stages: the larger the copies, the faster
+            // (one SM's bulk copies complete one after another, at a fixed
+            // latency each: about 340 ns, measured on GB300)
+            // (each block also keeps its rows of the head weights, 12 F d
+            // bytes, where they fit beside stages of at least 32 KB)
+            // (larger stages first: they matter more than resident weights)
+            if (round_cluster_set_attributes() != cudaSuccess) return DART_ERR_CUDA;
+            const size_t cavail = static_cast<size_t>(h->smem_optin) - round_cluster_static_smem(pm);
+            int stage = 0;
+            bool wres = false;
+            size_t smem = 0;
+            for (const int stb : {64 * 1024, 48 * 1024, 32 * 1024}) {
+                for (const bool wr : {true, false}) {
+                    const int st = stb / (c.d * 4) * (c.d * 4);
+                    const size_t sm = round_cluster_smem(pm, c.d, R, c.W, c.k, st, wr);
+                    if (st > 0 && sm <= cavail) {
+                        stage = st;
+                        wres = wr;
+                        smem = sm;
+                        break;
+                    }
+                }
+                if (stage) break;
+            }
+            if (stage) {
+                if (round_cluster_fits(pm, smem)) {
+                    h->fused = true;
+                    h->fused_cluster = true;
+                    h->fused_nm = pm;
+                    h->fused_G = kRoundCluster;
+                    h->fused_R = R;
+                    h->fused_smem = smem;
+                    h->fused_ecache = false;
+                    h->fused_mstage = false;
+                    h->fused_stage = stage;
+                    h->fused_wres = wres;
+                    return DART_OK;
+                }
+            }
+        }
+    }
+    const int G = std::min(h->num_sms, 160);
+    const int R = (c.V + G - 1) / G;
+    const int nm = round_small_nm(nmax);
+    bool ok = base_ok && nm > 0 && c.nseq * c.W <= 32 && c.V <= 65536 && c.nseq <= G;
+    // each block keeps its E slice for the whole round when it is small
+    // (it is read at every depth), and the merge stages a node's lists
+    bool ecache = static_cast<size_t>(R) * (c.d + 4) * 4 <= 64 * 1024;
+    const bool mstage = static_cast<size_t>(8) * G * c.k * 8 <= 80 * 1024;
+    size_t smem = 0;
+    if (ok) {
+        smem = round_small_smem(nm, c.d, R, c.W, c.k, G, ecache, mstage);
+        if (smem > avail && ecache) {
+            ecache = false;
+            smem = round_small_smem(nm, c.d, R, c.W, c.k, G, ecache, mstage);
+        }
+        ok = smem <= avail;
+    }
+    if (ok) {
+        if (round_small_set_smem_limits() != cudaSuccess) return DART_ERR_CUDA;
+        ok = round_small_blocks_per_sm(nm, smem) >= 1;
+    }
+    if (!ok) return c.fused_round == DART_ON ? DART_ERR_UNSUPPORTED : DART_OK;
+    h->fused = true;
+    h->fused_cluster = false;
+    h->fused_nm = nm;
+    h->fused_G = G;
+    h->fused_R = R;
+    h->fused_smem = smem;
+    h->fused_ecache = ecache;
+    h->fused_mstage = mstage;
+    return DART_OK;
+}
+
 int build_plans(dart_handle* h, const dart_config& c, std::vector<int>& caps, std::vector<DepthPlan>& plans) {
     const bool tc = h->wdtype == DART_BF16;
     caps.assign(c.L + 1, 1);
@@ -462,6 +576,16 @@ int alloc_workspace(dart_handle* h) {
         DART_ALLOC(h->Wit, static_cast<size_t>((c.d + kTileM - 1) / kTileM) * kTileM * h->Kwi)
         DART_ALLOC(h->Wot, static_cast<size_t>((c.d + kTileM - 1) / kTileM) * kTileM * d)
     }
+    if (h->fused) {
+        const size_t nc = static_cast<size_t>(c.nseq) * c.W, G = h->fused_G;
+        DART_ALLOC(h->f_rbuf, nc * d)
+        DART_ALLOC(h->f_abuf, nc * d)
+        DART_ALLOC(h->f_ssqp, nc * G)
+        DART_ALLOC(h->f_pms, nc * G)
+        DART_ALLOC(h->f_pkey, nc * G * c.k)
+        DART_ALLOC(h->f_bar, kRoundBarWords)
+        DART_ALLOC(h->f_abort, 1)
+    }
     const size_t ns = c.nseq, Bp = h->Bp, S1 = static_cast<size_t>(c.B) + 1;
     if (c.variants & DART_VARIANT_CHAIN_DDTREE) {
         DART_ALLOC(h->zrows, ns * c.L * c.V)
@@ -513,6 +637,11 @@ int alloc_workspace(dart_handle* h) {
     if (cudaMemset(h->tree_count, 0, c.nseq * c.L * sizeof(int)) != cudaSuccess) return DART_ERR_CUDA;
     if (h->ddt_ticket && cudaMemset(h->ddt_ticket, 0, ns * c.L * sizeof(int)) != cudaSuccess) return DART_ERR_CUDA;
     if (h->sh_ticket && cudaMemset(h->sh_ticket, 0, ns * sizeof(int)) != cudaSuccess) return DART_ERR_CUDA;
+    if (h->fused && (cudaMemset(h->f_bar, 0, kRoundBarWords * sizeof(unsigned)) != cudaSuccess ||
+                     cudaMemset(h->f_abort, 0, sizeof(int)) != cudaSuccess ||
+                     round_small_set_smem_limits() != cudaSuccess ||
+                     (h->fused_cluster && round_cluster_set_attributes() != cudaSuccess)))
+        return DART_ERR_CUDA;
     // one-time kernel attributes
     int max_sel = 0;
     for (int dep = 1; dep <= c.L; dep++)
@@ -616,7 +745,7 @@ void release(dart_handle* h) {
 
 enum Kind {
     kLmhead = 0, kSelect, kGather, kGemm1, kSilu, kGemm2, kNorm, kPrep, kEmit, kCandTopk, kCandScore, kGatherSilu,
-    kRowTopk, kDdtree, kSeqStep, kSeqEmit, kNumKinds
+    kRowTopk, kDdtree, kSeqStep, kSeqEmit, kFusedRound, kL2Prefetch, kNumKinds
 };
 
 // Opens an event pair around the next launch when profiling (no-op otherwise).
@@ -795,9 +924,11 @@ int enqueue_depth(dart_handle* h, const dart_config& c, const std::vector<DepthP
         // first E tiles (its L2-prefetch window) are requested now, beside it
         if (c.cand_k == 0 && dep < c.L && plans[dep + 1].epf > 0) {
             const DepthPlan& q = plans[dep + 1];
-            if (launch_lmhead_l2_prefetch(&h->tmE, (c.V + kTileM - 1) / kTileM, q.nV, c.d, q.epf, h->Et ? 1 : 0,
-                                          h->side) != cudaSuccess)
-                return DART_ERR_CUDA;
+            pi = prof_begin(h, kL2Prefetch, h->side);
+            e = launch_lmhead_l2_prefetch(&h->tmE, (c.V + kTileM - 1) / kTileM, q.nV, c.d, q.epf, h->Et ? 1 : 0,
+                                          h->side);
+            prof_end(h, pi, h->side);
+            if (e != cudaSuccess) return DART_ERR_CUDA;
         }
         pi = prof_begin(h, kGemm1, h->side);
         e = launch_gemm_tc(&h->tmWi, &h->tmH[ng_index(g1.NG)], g1, p.g1_smem, h->side);
@@ -913,7 +1044,7 @@ int check_out(const dart_tree_out* o) {
     return DART_OK;
 }
 
-int enqueue_emit(dart_handle* h, const dart_tree_out* o, cudaStream_t st) {
+EmitArgs emit_args(const dart_handle* h, const dart_tree_out* o) {
     const dart_config& c = h->cfg;
     EmitArgs a;
     a.L = c.L;
@@ -933,13 +1064,76 @@ int enqueue_emit(dart_handle* h, const dart_tree_out* o, cudaStream_t st) {
     a.scores = o->scores;
     a.mask = o->mask;
     a.status = h->status;
+    return a;
+}
+
+int enqueue_emit(dart_handle* h, const dart_tree_out* o, cudaStream_t st) {
+    const EmitArgs a = emit_args(h, o);
     const int pi = prof_begin(h, kEmit, st);
     const cudaError_t e = launch_prune_emit(a, st);
     prof_end(h, pi, st);
     return e == cudaSuccess ? DART_OK : DART_ERR_CUDA;
 }
 
+// The fused small-problem round: one cooperative kernel (dart_round.cu).
+int enqueue_fused_round(dart_handle* h, const float* dlog, const float* anchor, const dart_tree_out* out,
+                        cudaStream_t st) {
+    const dart_config& c = h->cfg;
+    if (h->f_dirty) return DART_ERR_STATE;  // dart_status_sync first (it resets the barrier)
+    RoundArgs a;
+    std::memset(&a, 0, sizeof a);
+    a.V = c.V;
+    a.d = c.d;
+    a.L = c.L;
+    a.W = c.W;
+    a.k = c.k;
+    a.nseq = c.nseq;
+    a.G = h->fused_G;
+    a.R = h->fused_R;
+    a.ecache = h->fused_ecache ? 1 : 0;
+    a.mstage = h->fused_mstage ? 1 : 0;
+    a.stage_bytes = h->fused_stage;
+    a.wres = h->fused_wres ? 1 : 0;
+    for (int i = 0; i <= c.L; i++) a.caps[i] = h->caps[i];
+    a.beta = c.beta;
+    a.invT = c.temperature > 0.0f ? 1.0f / c.temperature : 1.0f;
+    a.eps = c.rms_eps;
+    a.E = static_cast<const float*>(h->E);
+    a.Wi = static_cast<const float*>(h->Wi);
+    a.Wo = static_cast<const float*>(h->Wo);
+    a.dlog = dlog;
+    a.anchor = anchor;
+    a.h0 = h->hbuf[0];
+    a.h1 = h->hbuf[1];
+    a.rbuf = h->f_rbuf;
+    a.abuf = h->f_abuf;
+    a.ssqp = h->f_ssqp;
+    a.pms = h->f_pms;
+    a.pkey = h->f_pkey;
+    a.node_logq = h->node_logq;
+    a.node_lse = h->node_lse;
+    a.node_tok = h->node_tok;
+    a.tree_tok = h->tree_tok;
+    a.tree_parent = h->tree_parent;
+    a.tree_count = h->tree_count;
+    a.tree_score = h->tree_score;
+    a.child_prow = h->child_prow;
+    a.child_tok = h->child_tok;
+    a.status = h->status;
+    a.bar = h->f_bar;
+    a.abort = h->f_abort;
+    a.emit = emit_args(h, out);
+    const int pi = prof_begin(h, kFusedRound, st);
+    const cudaError_t e = h->fused_cluster ? launch_round_cluster_f32(a, h->fused_nm, h->fused_smem, st)
+                                           : launch_round_small_f32(a, h->fused_nm, h->fused_smem, st);
+    prof_end(h, pi, st);
+    h->cur = (c.L - 1) & 1;  // depth L's states: the parity buffer of depth L
+    h->next_depth = c.L + 1;
+    return e == cudaSuccess ? DART_OK : DART_ERR_CUDA;
+}
+
 int enqueue_round(dart_handle* h, const float* dlog, const float* anchor, const dart_tree_out* out, cudaStream_t st) {
+    if (h->fused) return enqueue_fused_round(h, dlog, anchor, out, st);
     for (int dep = 1; dep <= h->cfg.L; dep++) {
         int rc = enqueue_depth(h, h->cfg, h->plans, dep, dlog, anchor, st);
         if (rc != DART_OK) return rc;
@@ -1145,7 +1339,8 @@ int run_round(dart_handle* h, int kind, const float* dlog, const float* anchor, 
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
     if (cudaStreamIsCapturing(st, &cs) != cudaSuccess) return DART_ERR_CUDA;
-    if (h->profiling || cs != cudaStreamCaptureStatusNone) {
+    // (the fused round is one launch already: no graph)
+    if (h->profiling || cs != cudaStreamCaptureStatusNone || (kind == kRoundDartree && h->fused)) {
         rc = enqueue_kind(h, kind, dlog, anchor, out, st);
         finish_round(h, kind, rc == DART_OK);
         return rc;
@@ -1251,6 +1446,7 @@ int dart_init_head(dart_handle** out, const dart_config* cfg, int wdtype, const 
     h->wtiled = wdtype == DART_BF16 && cfg->head_weights_tiled == DART_ON;
     h->Kwi = (wdtype == DART_BF16 && cfg->head_split != DART_OFF) ? cfg->d : 2 * cfg->d;
     if (rc == DART_OK) rc = build_plans(h, h->cfg, h->caps, h->plans);
+    if (rc == DART_OK) rc = plan_fused_round(h);
     if (rc == DART_OK && cfg->variants) {
         // the best-first constructions score one node per sequence at a time
         // over the full vocabulary and keep its best min(B, V) children
@@ -1461,13 +1657,29 @@ int dart_status_sync(dart_handle* h, void* stream) {
     if (cudaStreamSynchronize(st) != cudaSuccess) return DART_ERR_CUDA;
     if (cudaMemcpy(&word, h->status, sizeof word, cudaMemcpyDeviceToHost) != cudaSuccess) return DART_ERR_CUDA;
     if (cudaMemset(h->status, 0, sizeof word) != cudaSuccess) return DART_ERR_CUDA;
-    if (word & kDevTimeout) return DART_ERR_TIMEOUT;
+    if (word & kDevTimeout) {
+        // a fused round that gave up left its grid barrier mid-way
+        if (h->f_bar && (cudaMemset(h->f_bar, 0, kRoundBarWords * sizeof(unsigned)) != cudaSuccess ||
+                         cudaMemset(h->f_abort, 0, sizeof(int)) != cudaSuccess))
+            return DART_ERR_CUDA;
+        h->f_dirty = false;
+        return DART_ERR_TIMEOUT;
+    }
     if (word & kDevBounds) return DART_ERR_BOUNDS;
     if (word & kDevOrphan) return DART_ERR_STATE;
     return DART_OK;
 }
 
 int dart_debug_build(void) { return debug_build() ? 1 : 0; }
+
+int dart_test_barrier_timeout(dart_handle* h, int limit_us, void* stream) {
+    if (!h || limit_us < 1 || limit_us > 2000000) return DART_ERR_INVALID;
+    if (!h->fused) return DART_ERR_STATE;
+    h->f_dirty = true;
+    return cuda_err(launch_barrier_probe(h->f_bar, h->f_abort, h->status,
+                                         static_cast<unsigned long long>(limit_us) * 1000ull,
+                                         static_cast<cudaStream_t>(stream)));
+}
 
 int dart_test_bounds_report(dart_handle* h, void* stream) {
     if (!h) return DART_ERR_INVALID;
@@ -1518,6 +1730,7 @@ int dart_profile_read(dart_handle* h, float* lmhead_ms, int* lmhead_launches) {
 int dart_launches_per_round(dart_handle* h) {
     if (!h) return DART_ERR_INVALID;
     const int L = h->cfg.L;
+    if (h->fused) return 1;
     // prep, (LM-head + select) per depth, then per depth but the last:
     // gather, W_i GEMM, [SiLU,] W_o GEMM, residual-norm; or with the split
     // first layer: W_i[:, 0:d] GEMM, gather + SiLU, W_o GEMM, residual-norm;

@@ -288,6 +288,58 @@ struct SeqHeapArgs {
 cudaError_t launch_seqheap_step(const SeqHeapArgs& a, int t, cudaStream_t st);
 cudaError_t launch_seqheap_emit(const SeqHeapArgs& a, cudaStream_t st);
 
+// The whole round of a small fp32 problem in one cooperative kernel
+// (dart_round.cu): G blocks (one per SM, at most 160), each scoring a slice
+// of at most R vocabulary rows.  caps[dep] = nodes per sequence at depth dep
+// (caps[0] = 1).  h0 / h1: the normalised states of odd / even depths
+// [nodes][d]; rbuf, abuf [children][d]; ssqp [children][G] per-block sums of
+// r^2; pms [nodes][G] and pkey [nodes][G][k] the per-slice (max, sum exp)
+// and best keys; bar (kRoundBarWords words, zero: arrivals, generation and
+// the one-sequence arrival ticket on separate 128-byte lines) and abort
+// (zero) the grid barrier.  ecache: each block keeps its E slice in shared
+// memory for the whole round; mstage: the merge stages a node's G*k keys in
+// shared memory.
+constexpr int kRoundMaxL = 32;
+constexpr int kRoundBarWords = 96;
+struct RoundArgs {
+    int V, d, L, W, k, nseq, G, R;
+    int ecache, mstage;
+    int stage_bytes;  // cluster form: bytes of each of the two E stages (a multiple of d * 4)
+    int wres;         // cluster form: each block keeps its W_i and W_o rows in shared memory
+    int caps[kRoundMaxL + 1];
+    float beta, invT, eps;
+    const float *E, *Wi, *Wo, *dlog, *anchor;
+    float *h0, *h1, *rbuf, *abuf, *ssqp;
+    float2* pms;
+    uint64_t* pkey;
+    float *node_logq, *node_lse;
+    int* node_tok;
+    int *tree_tok, *tree_parent, *tree_count;
+    float* tree_score;
+    int *child_prow, *child_tok;
+    int* status;
+    unsigned* bar;
+    int* abort;
+    EmitArgs emit;
+};
+int round_small_nm(int nmax);  // node slots of the kernel instance: 4, 8, 16, 32 (0: too many)
+size_t round_small_smem(int nm, int d, int R, int W, int k, int G, bool ecache, bool mstage);
+cudaError_t round_small_set_smem_limits();
+int round_small_blocks_per_sm(int nm, size_t smem);
+cudaError_t launch_round_small_f32(const RoundArgs& a, int nm, size_t smem, cudaStream_t st);
+// The same round with one cluster of kRoundCluster blocks per sequence
+// (G = kRoundCluster, R = the rows of a block's vocabulary slice): pm node
+// slots per sequence (4, 8, 16, 32)
+constexpr int kRoundCluster = 16;
+size_t round_cluster_smem(int pm, int d, int R, int W, int k, int stage_bytes, bool wres);
+cudaError_t round_cluster_set_attributes();
+bool round_cluster_fits(int pm, size_t smem);
+size_t round_cluster_static_smem(int pm);
+cudaError_t launch_round_cluster_f32(const RoundArgs& a, int pm, size_t smem, cudaStream_t st);
+// two blocks at a grid barrier of three that give up after limit_ns (test hook)
+cudaError_t launch_barrier_probe(unsigned* bar, int* abort, int* status, unsigned long long limit_ns,
+                                 cudaStream_t st);
+
 // bf16 [rows][cols] (row pitch `pitch` elements) -> 128 x 64 tiles, each 16 KB contiguous (tile (rt, kb)
 // at index rt * cols / 64 + kb; rows past `rows` zero): every TMA request of
 // the LM-head's E stream then reads one contiguous 16 KB block.

@@ -64,6 +64,8 @@ def test_debug_build_passes_the_parity_cases(dart):
            "tests/test_parity_gpu.py::test_build_tree_graph_matches_depthwise",
            "tests/test_parity_gpu.py::test_neg_inf_drafter_logits",
            "tests/test_parity_gpu.py::test_restricted_candidates_and_neg_inf",
+           "tests/test_parity_gpu.py::test_fused_round_parity",
+           "tests/test_parity_gpu.py::test_fused_round_neg_inf_and_states",
            "tests/test_heap_gpu.py::test_chain_ddtree_and_seq_heap_parity",
            "tests/test_heap_gpu.py::test_variants_and_algorithm1_on_one_handle",
            "tests/test_heap_gpu.py::test_dartree_fixed"]

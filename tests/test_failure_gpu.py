@@ -98,3 +98,44 @@ def test_the_graph_cache_is_bounded_and_rotating_buffers_stay_correct(dart):
                 np.testing.assert_array_equal(g[k], ref[k], err_msg=k)
     finally:
         eng.close()
+
+
+def test_a_grid_barrier_that_runs_out_is_reported_and_the_fused_round_recovers(dart):
+    """The fused round's grid barrier with a short limit and a block that
+    never arrives (no copy or computation in flight): DART_ERR_TIMEOUT, the
+    handle refuses rounds until the status is read, then the barrier is reset
+    and the next round is the oracle's tree again."""
+    # (V = 60000: the grid form of the fused round, whose barrier this is)
+    cfg = Config("barrier-timeout", 1, 60000, 128, 4, 4, 4, 12, "f32", 0.0, 80, fused_round=1)
+    x = make_inputs(cfg)
+    dx = to_device(cfg, x)
+    eng = dart.Dart(cfg, dx["Wi"], dx["Wo"], dx["E"])
+    try:
+        before = tree_to_numpy(eng.build_tree(dx["Dlog"], dx["h0"]))
+        assert dart.dart_status_sync(eng.h) == dart.DART_OK
+        t0 = time.perf_counter()
+        dart.dart_test_barrier_timeout(eng.h, 300)
+        with pytest.raises(dart.DartError) as e:
+            eng.build_tree(dx["Dlog"], dx["h0"])
+        assert e.value.code == dart.DART_ERR_STATE
+        assert dart.dart_status_sync(eng.h) == dart.DART_ERR_TIMEOUT
+        assert time.perf_counter() - t0 < 1.5
+        assert dart.dart_status_sync(eng.h) == dart.DART_OK
+        after = tree_to_numpy(eng.build_tree(dx["Dlog"], dx["h0"]))
+        assert dart.dart_status_sync(eng.h) == dart.DART_OK
+        for k in before:
+            np.testing.assert_array_equal(after[k], before[k], err_msg=k)
+        gst = gpu_supertree(dart, eng.h, cfg)
+    finally:
+        eng.close()
+    ref = oracle.build_tree(cfg, x["Wi"], x["Wo"], x["E"], x["Dlog"], x["h0"])
+    compare_with_oracle(cfg, ref, gst, after, tol_of(cfg), x=x)
+    # a handle without the fused round has no barrier to probe
+    cfg2 = cfg.replace(fused_round=2)
+    eng = dart.Dart(cfg2, dx["Wi"], dx["Wo"], dx["E"])
+    try:
+        with pytest.raises(dart.DartError) as e:
+            dart.dart_test_barrier_timeout(eng.h, 300)
+        assert e.value.code == dart.DART_ERR_STATE
+    finally:
+        eng.close()

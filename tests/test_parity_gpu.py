@@ -137,7 +137,9 @@ GRAPH = SMALL[:6] + RESTRICTED[:3]
 def test_build_tree_graph_matches_depthwise(dart, cfg):
     """dart_build_tree (one cached CUDA graph) equals the depth-by-depth
     calls, is deterministic across repeated launches, and the host-buffer
-    variant returns the same tree."""
+    variant returns the same tree.  (fp32: the graph of per-step launches;
+    the fused round is compared with the oracle below.)"""
+    cfg = cfg.replace(fused_round=2)
     x = make_inputs(cfg)
     dx = to_device(cfg, x)
     _, gst_ref, g_ref = run_depthwise(dart, cfg, dx)
@@ -158,6 +160,94 @@ def test_build_tree_graph_matches_depthwise(dart, cfg):
             np.testing.assert_array_equal(ht[k].numpy(), g_ref[k], err_msg=k)
     finally:
         eng.close()
+
+
+# fp32 problems small enough for the fused round: one cluster per sequence
+# where a block's share of E is small, else one cooperative grid (the V = 64K
+# case; at most 32 nodes per depth)
+FUSED = [c for c in SMALL if c.wdtype == "f32" and c.V <= 65536] + [
+    C("f32-fused-nseq4", 4, 6000, 256, 5, 8, 8, 30, "f32", 0.7, 41),
+    C("f32-fused-V64k", 1, 65536, 128, 3, 16, 16, 25, "f32", 0.0, 42),
+    C("f32-fused-k32", 2, 4000, 64, 4, 16, 32, 40, "f32", 0.0, 43),
+    C("f32-fused-L8W32", 1, 3000, 64, 8, 32, 8, 120, "f32", 0.3, 44),
+    C("f32-fused-chain", 1, 2000, 128, 6, 1, 1, 6, "f32", 0.0, 45),
+    C("f32-fused-B1", 2, 1500, 128, 4, 4, 4, 1, "f32", 0.0, 46, pos_offset=9),
+    C("f32-fused-Vk", 1, 8, 64, 4, 8, 8, 30, "f32", 0.0, 47),
+]
+
+
+@pytest.mark.parametrize("cfg", FUSED, ids=[c.name for c in FUSED])
+def test_fused_round_parity(dart, cfg):
+    """The whole round as one kernel launch: the oracle's tree
+    (compare_with_oracle), bit-identical on repeated launches and through the
+    host-buffer entry point."""
+    cfg = cfg.replace(fused_round=1)
+    x = make_inputs(cfg)
+    dx = to_device(cfg, x)
+    ref = oracle.build_tree(cfg, x["Wi"], x["Wo"], x["E"], x["Dlog"], x["h0"])
+    eng = dart.Dart(cfg, dx["Wi"], dx["Wo"], dx["E"])
+    try:
+        assert dart.dart_launches_per_round(eng.h) == 1
+        g = tree_to_numpy(eng.build_tree(dx["Dlog"], dx["h0"]))
+        assert dart.dart_status_sync(eng.h) == 0
+        gst = gpu_supertree(dart, eng.h, cfg)
+        for it in range(2):
+            again = tree_to_numpy(eng.build_tree(dx["Dlog"], dx["h0"]))
+            for k in g:
+                np.testing.assert_array_equal(again[k], g[k], err_msg=f"{k} (launch {it + 2})")
+        ht, hout = dart.alloc_tree_out(cfg, pin=True)
+        dart.dart_build_tree_host(eng.h, dx["Dlog"].cpu().pin_memory(), dx["h0"].cpu().pin_memory(), hout)
+        assert dart.dart_status_sync(eng.h) == 0
+        for k in g:
+            np.testing.assert_array_equal(ht[k].numpy(), g[k], err_msg=k)
+    finally:
+        eng.close()
+    compare_with_oracle(cfg, ref, gst, g, tol_of(cfg), x=x)
+
+
+def test_fused_round_neg_inf_and_states(dart):
+    """-inf drafter logits through the fused round, and the state hook after
+    it: depth L's states equal the depth-by-depth path's within fp32
+    rounding."""
+    cfg = C("f32-fused-neginf", 2, 700, 128, 4, 6, 4, 40, "f32", 0.0, 48, fused_round=1)
+    x = make_inputs(cfg)
+    x["Dlog"][0, 1, 3:] = -np.inf      # depth 2 of seq 0: only tokens 0..2 possible
+    x["Dlog"][1, 0, :] = -np.inf       # depth 1 of seq 1: no child at all
+    x["Dlog"][1, 0, 5] = 0.0           #   ... except token 5
+    dx = to_device(cfg, x)
+    ref = oracle.build_tree(cfg, x["Wi"], x["Wo"], x["E"], x["Dlog"], x["h0"])
+    per, _, _ = run_depthwise(dart, cfg, dx)
+    eng = dart.Dart(cfg, dx["Wi"], dx["Wo"], dx["E"])
+    try:
+        g = tree_to_numpy(eng.build_tree(dx["Dlog"], dx["h0"]))
+        assert dart.dart_status_sync(eng.h) == 0
+        gst = gpu_supertree(dart, eng.h, cfg)
+        st = dart.dart_get_states(eng.h, cfg).cpu().numpy()
+    finally:
+        eng.close()
+    compare_with_oracle(cfg, ref, gst, g, tol_of(cfg), x=x)
+    assert int(gst["st_count"][1, 0]) == 1 and int(gst["st_tok"][1, 0, 0]) == 5
+    np.testing.assert_allclose(st, per[-1]["states"], rtol=0, atol=1e-4)
+
+
+def test_fused_round_eligibility(dart):
+    """fused_round = ON where the problem does not fit is refused at
+    dart_init_head; AUTO then takes the per-step launches."""
+    x = None
+    for cfg in (C("f32-wide", 1, 1500, 64, 3, 40, 4, 20, "f32", 0.7, 12),          # W > 32
+                C("f32-bigV", 1, 70000, 64, 2, 4, 4, 8, "f32", 0.0, 13),           # V > 65536, E slices > 512 KB
+                C("bf16-small", 1, 1000, 128, 3, 4, 4, 8, "bf16", 0.0, 14)):        # bf16 weights
+        x = make_inputs(cfg)
+        dx = to_device(cfg, x)
+        wd = dart.DART_BF16 if cfg.wdtype == "bf16" else dart.DART_F32
+        with pytest.raises(dart.DartError) as e:
+            dart.dart_init_head(cfg.replace(fused_round=1), wd, dx["Wi"], dx["Wo"], dx["E"])
+        assert e.value.code == dart.DART_ERR_UNSUPPORTED
+        h = dart.dart_init_head(cfg, wd, dx["Wi"], dx["Wo"], dx["E"])
+        try:
+            assert dart.dart_launches_per_round(h) > 1
+        finally:
+            dart.dart_destroy(h)
 
 
 VARIANT_CFGS = [SMALL[2], SMALL[5], SMALL[6], RESTRICTED[1]]

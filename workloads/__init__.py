@@ -62,6 +62,7 @@ class Config:
     weights_tiled: int = 0
     head_weights_tiled: int = 0
     variants: int = 0          # extra constructions prepared by the handle (bit set)
+    fused_round: int = 0       # fp32: the whole round as one cooperative kernel (where possible)
 
     def replace(self, **kw) -> "Config":
         return dataclasses.replace(self, **kw)
