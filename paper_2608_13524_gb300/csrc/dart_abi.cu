@@ -1733,11 +1733,20 @@ int dart_launches_per_round(dart_handle* h) {
     if (h->fused) return 1;
     // prep, (LM-head + select) per depth, then per depth but the last:
     // gather, W_i GEMM, [SiLU,] W_o GEMM, residual-norm; or with the split
-    // first layer: W_i[:, 0:d] GEMM, gather + SiLU, W_o GEMM, residual-norm;
-    // prune-emit
+    // first layer: W_i[:, 0:d] GEMM, gather + SiLU, W_o GEMM, residual-norm,
+    // and beside them the early prefetch of the next depth's E tiles; or
+    // (fp32, d <= 1024) the whole update in one launch; prune-emit
+    const bool tc = h->wdtype == DART_BF16;
     int n = 1 + 2 * L + 1 + (h->cfg.cand_k > 0 ? 1 : 0);
-    for (int dep = 1; dep < L; dep++)
-        n += (h->plans[dep].split || (h->wdtype == DART_BF16 && h->plans[dep].g1.mode != kGemmPartials)) ? 4 : 5;
+    for (int dep = 1; dep < L; dep++) {
+        const DepthPlan& p = h->plans[dep];
+        if (!tc && head_small_f32_slices(h->cfg.d) > 0) {
+            n += 1;
+            continue;
+        }
+        n += (p.split || (tc && p.g1.mode != kGemmPartials)) ? 4 : 5;
+        if (p.side && h->cfg.cand_k == 0 && h->plans[dep + 1].epf > 0) n += 1;
+    }
     return n;
 }
 

@@ -440,3 +440,29 @@ def test_handles_with_different_plans_coexist(dart):
     ref = oracle.build_tree(big, x["Wi"], x["Wo"], x["E"], x["Dlog"], x["h0"])
     compare_with_oracle(big, ref, gst, ga, tol_of(big), x=x)
     compare_with_oracle(small, ref, gstb, gb, tol_of(big), x=x)
+
+
+LAUNCH_CFGS = [SMALL[0], SMALL[0].replace(fused_round=2), SMALL[1], SMALL[2], SMALL[5], SMALL[19],
+               RESTRICTED[1], RESTRICTED[0]]
+
+
+@pytest.mark.parametrize("cfg", LAUNCH_CFGS, ids=[f"{c.name}-{c.fused_round}" for c in LAUNCH_CFGS])
+def test_launches_per_round_matches_the_profiled_round(dart, cfg):
+    """dart_launches_per_round (the bench's kernel-launch count) equals the
+    launches one profiled round brackets, kind by kind summed (every launch
+    of a round is bracketed while profiling is on)."""
+    x = make_inputs(cfg)
+    dx = to_device(cfg, x)
+    eng = dart.Dart(cfg, dx["Wi"], dx["Wo"], dx["E"])
+    try:
+        eng.build_tree(dx["Dlog"], dx["h0"])
+        dart.dart_set_profiling(eng.h, True)
+        dart.dart_profile_read_kinds(eng.h)
+        eng.build_tree(dx["Dlog"], dx["h0"])
+        kinds = dart.dart_profile_read_kinds(eng.h)
+        dart.dart_set_profiling(eng.h, False)
+        assert dart.dart_status_sync(eng.h) == 0
+        counted = sum(n for _, n in kinds.values())
+        assert counted == dart.dart_launches_per_round(eng.h), kinds
+    finally:
+        eng.close()
