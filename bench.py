@@ -879,9 +879,9 @@ def main():
     if kinds.get("round_f32", (0.0, 0))[1] > 0:
         # the fused small-problem round: one launch per round reads E and the
         # drafter rows once per depth and the head weights once per head update
-        rl_kind, rl_name = "round_f32", "round_small_f32_kernel (whole round)"
+        rl_kind, rl_name = "round_f32", "fused fp32 round kernel (whole round)"
         bytes_launch = cfg.L * cfg.lmhead_bytes_per_depth() + (cfg.L - 1) * 3 * cfg.d * cfg.d * cfg.bpe
-        rl_note = "one launch per round; latency-bound (grid barriers), its bytes fit in L2"
+        rl_note = "one launch per round; latency-bound (cluster or grid barriers between steps), its bytes fit in L2"
     elif cfg.cand_k == 0:
         rl_kind, rl_name, bytes_launch, rl_note = "lmhead", "lmhead_tc_kernel", cfg.lmhead_bytes_per_depth(), None
     elif not wi_kept:
