@@ -287,7 +287,7 @@ int plan_fused_round(dart_handle* h) {
         // keys fit in shared memory
         const int pm = round_small_nm(pmax);
         const int R = (c.V + kRoundCluster - 1) / kRoundCluster;
-        if (base_ok && pm > 0 && c.W * c.k <= 256 && static_cast<size_t>(R) * c.d * 4 <= 512 * 1024 &&
+        if (base_ok && pm > 0 && c.W * c.k <= 256 && R <= 8 * 256 && static_cast<size_t>(R) * c.d * 4 <= 512 * 1024 &&
             pm * c.d <= 16384 && static_cast<size_t>(pm) * R * 8 <= 64 * 1024) {
             // E streams through two stages: the larger the copies, the faster
             // (one SM's bulk copies complete one after another, at a fixed

@@ -720,7 +720,8 @@ __global__ void __launch_bounds__(kRoundThreads, 1) round_cluster_f32_kernel(con
     // the merged children lists of the nodes this block merged: [NP][k]
     float* nlq = xbuf + NP * d;
     int* ntok = reinterpret_cast<int*>(nlq + NP * k);
-    float* wis = reinterpret_cast<float*>((reinterpret_cast<uintptr_t>(ntok + NP * k) + 15) & ~static_cast<uintptr_t>(15));
+    float* dls = reinterpret_cast<float*>(ntok + NP * k);  // [R] the depth's drafter logits of the block's rows
+    float* wis = reinterpret_cast<float*>((reinterpret_cast<uintptr_t>(dls + a.R) + 15) & ~static_cast<uintptr_t>(15));
     float* wos = wis + F * 2 * d;
     volatile int* abort = &misc[0];
 
@@ -782,6 +783,16 @@ __global__ void __launch_bounds__(kRoundThreads, 1) round_cluster_f32_kernel(con
     for (int dep = 1; dep <= a.L; dep++) {
         const int P = a.caps[dep - 1], Pn = a.caps[dep];
         float* hcur = (dep & 1) ? a.h0 : a.h1;
+        // the depth's drafter logits of this block's rows, requested first
+        // (they arrive while the states are gathered)
+        const float* drow = a.dlog + (static_cast<size_t>(s) * a.L + dep - 1) * a.V;
+        constexpr int kDl = 8;  // R <= 8 * kRoundThreads
+        float dlr[kDl];
+#pragma unroll
+        for (int u = 0; u < kDl; u++) {
+            const int r = tid + u * kRoundThreads;
+            dlr[u] = r < R ? __ldg(drow + v0 + r) : 0.0f;
+        }
         // A1: the depth's states: the anchor, or r / rms(r) of the previous
         // depth's children gathered from the blocks that own the features
         if (dep == 1) {
@@ -807,6 +818,11 @@ __global__ void __launch_bounds__(kRoundThreads, 1) round_cluster_f32_kernel(con
                 }
             }
         }
+#pragma unroll
+        for (int u = 0; u < kDl; u++) {
+            const int r = tid + u * kRoundThreads;
+            if (r < R) dls[r] = dlr[u];
+        }
         __syncthreads();
         for (int q = tid; q < P * F; q += kRoundThreads) {
             const int p = q / F, i = static_cast<int>(rank) * F + q % F;
@@ -814,7 +830,6 @@ __global__ void __launch_bounds__(kRoundThreads, 1) round_cluster_f32_kernel(con
         }
         // A2: z of this block's rows for the P nodes: warps take RS rows at a
         // time, lanes split d; the partial sums are reduce-scattered
-        const float* drow = a.dlog + (static_cast<size_t>(s) * a.L + dep - 1) * a.V;
         for (int ch = 0; ch < nch; ch++) {
             const int g = (dep - 1) * nch + ch;
             const int st = g & 1;
@@ -848,7 +863,7 @@ __global__ void __launch_bounds__(kRoundThreads, 1) round_cluster_f32_kernel(con
                 const int row = ch * CR + r0 + r;
                 if (n < P && r0 + r < rows) {
                     const int vv = v0 + row;
-                    kz[n * a.R + row] = make_key((v[0] + __ldg(drow + vv)) * a.invT, static_cast<uint32_t>(vv));
+                    kz[n * a.R + row] = make_key((v[0] + dls[row]) * a.invT, static_cast<uint32_t>(vv));
                 }
             }
             __syncthreads();  // stage st is free again
@@ -1095,7 +1110,8 @@ size_t round_cluster_smem_pm(int d, int R, int W, int k, int stage_bytes, bool w
     const int F = d / kCS;
     return static_cast<size_t>(NP) * d * 4 + static_cast<size_t>(NP) * k * 8 + 3 * static_cast<size_t>(NP) * F * 4 +
            2 * static_cast<size_t>(stage_bytes) + static_cast<size_t>(NP) * R * 8 + static_cast<size_t>(NP) * d * 4 +
-           static_cast<size_t>(NP) * k * 8 + 16 + (wres ? static_cast<size_t>(F) * 3 * d * 4 : 0);
+           static_cast<size_t>(NP) * k * 8 + static_cast<size_t>(R) * 4 + 16 +
+           (wres ? static_cast<size_t>(F) * 3 * d * 4 : 0);
 }
 
 int round_small_nm(int nmax) { return nmax <= 4 ? 4 : (nmax <= 8 ? 8 : (nmax <= 16 ? 16 : (nmax <= 32 ? 32 : 0))); }
