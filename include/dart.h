@@ -128,7 +128,17 @@ enum {
  *                      per-block scores within shared memory; AUTO = ON
  *                      where possible, ON = DART_ERR_UNSUPPORTED where not.
  *                      The depth-by-depth calls always take the per-step
- *                      launches (results agree within fp32 rounding) */
+ *                      launches (results agree within fp32 rounding)
+ *   topk_bound         bf16 weights, cand_k = 0, V >= max(64, 2k): a
+ *                      small kernel before each LM-head launch bounds every
+ *                      node's k-th best score from below (its k-th best,
+ *                      less an error bound, over the rows of largest drafter
+ *                      logit in max(64, 2k) vocabulary chunks), and the
+ *                      LM-head's top-k filter starts from that bound instead
+ *                      of offering every logit of its first tiles to the
+ *                      list merges.  The tree is unchanged.  AUTO = ON for
+ *                      k >= 32 at depths of more than 32 nodes (where it was
+ *                      measured faster) */
 typedef struct {
     int V, d, L, W, k, B, nseq;
     float beta, temperature, rms_eps;
@@ -137,6 +147,7 @@ typedef struct {
     int head_split, head_split_stream, lmhead_ctas_per_sm, weights_tiled, head_weights_tiled;
     int variants;
     int fused_round;
+    int topk_bound;
 } dart_config;
 
 /* Emitted verification tree, caller-allocated, per sequence s:
@@ -327,8 +338,9 @@ int dart_profile_read(dart_handle *h, float *lmhead_ms, int *lmhead_launches);
  * constructions), 13 DDTree search, 14 one pop of the sequential search,
  * 15 its emission, 16 the fused small-problem round (fused_round: one
  * launch per round), 17 the early L2 prefetch of the next depth's first E
- * tiles (side stream).  ms[i] / launches[i] receive the summed device time
- * and count of kind i for i < nkinds (nkinds <= 18); resets the events. */
+ * tiles (side stream), 18 the starting bound of the top-k filters
+ * (topk_bound).  ms[i] / launches[i] receive the summed device time and
+ * count of kind i for i < nkinds (nkinds <= 19); resets the events. */
 int dart_profile_read_kinds(dart_handle *h, float *ms, int *launches, int nkinds);
 
 /* Number of kernel launches one dart_build_tree enqueues for this handle. */

@@ -20,7 +20,7 @@ DEBUG_LIB = os.path.join(HERE, "libdart_debug.so")
 DEBUG_BUILD_DIR = os.path.join(HERE, "_build_debug")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 SOURCES = ["dart_abi.cu", "dart_tc.cu", "dart_f32.cu", "dart_select.cu", "dart_noalloc.cu", "dart_cand.cu",
-           "dart_attn.cu", "dart_heap.cu", "dart_round.cu"]
+           "dart_attn.cu", "dart_heap.cu", "dart_round.cu", "dart_bound.cu"]
 
 
 def _nvcc() -> str:

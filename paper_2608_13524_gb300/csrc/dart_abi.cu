@@ -70,6 +70,7 @@ struct DepthPlan {
     int N, P, NG, G, nV, stages, smem;  // LM-head scoring
     int l2pf;                            // LM-head: E tiles per CTA prefetched into L2 before its wait
     int epf;                             // of those and the stages, how many the previous depth prefetches early
+    int bound;                           // seed rows per sequence of the seed pass before this depth's LM-head (0: none)
     int nlist, klist;                    // sorted key lists per node and their length (merge input)
     int cand_ds;                         // candidate scoring: d slices per candidate group
     int f32_ds;                          // fp32 LM-head: blocks per vocabulary range (d slices)
@@ -115,6 +116,7 @@ struct dart_handle {
     float* tree_score;
     int *child_prow, *child_tok, *seq_ticket, *status;
     uint64_t* gthr;  // [L][kNPadMax] cross-CTA top-k bounds of every depth, zeroed per round
+    float* bound_y;     // [kNPadMax][kBoundR] seed scores less their error bounds (topk_bound)
     int* cand_tok;   // [nseq][L][cand_k] candidate sets C_d (cand_k > 0)
     float* cand_scratch;  // candidate scoring partial dot products
     int* cand_ticket;     // [nseq][ceil(cand_k/8)]
@@ -216,7 +218,8 @@ int validate_cfg(const dart_config* c) {
     if (!(c->temperature >= 0.0f) || !std::isfinite(c->temperature)) return DART_ERR_INVALID;
     if (!(c->rms_eps > 0.0f) || !std::isfinite(c->rms_eps)) return DART_ERR_INVALID;
     if (c->cand_k != 0 && (c->cand_k < c->k || c->cand_k > c->V || c->cand_k > kMaxCandK)) return DART_ERR_INVALID;
-    for (int sw : {c->head_split, c->head_split_stream, c->weights_tiled, c->head_weights_tiled, c->fused_round})
+    for (int sw : {c->head_split, c->head_split_stream, c->weights_tiled, c->head_weights_tiled, c->fused_round,
+                   c->topk_bound})
         if (sw != DART_AUTO && sw != DART_ON && sw != DART_OFF) return DART_ERR_INVALID;
     if (c->lmhead_ctas_per_sm < 0 || c->lmhead_ctas_per_sm > 2) return DART_ERR_INVALID;
     if (c->variants & ~(DART_VARIANT_CHAIN_DDTREE | DART_VARIANT_SEQ_HEAP)) return DART_ERR_INVALID;
@@ -255,6 +258,9 @@ GemmArgs gemm_plan(const dart_handle* h, int K, int Nc, int lo_kb_end, bool tc) 
 }
 
 constexpr long long kL2PrefetchBytes = 64ll << 20;  // about half of the 126 MB L2
+// Starting bound of the LM-head's top-k filters (topk_bound): at most this
+// many seed rows per sequence (2k rounded up to 64; scratch per node).
+constexpr int kBoundR = 2 * kMaxK;
 constexpr long long kL2KeepBytes = 72ll << 20;      // head weights kept in L2 across depths, at most
 
 int tc_stages(int smem_optin, int stage_bytes, int fixed) {
@@ -406,6 +412,26 @@ int build_plans(dart_handle* h, const dart_config& c, std::vector<int>& caps, st
             p.epf = (p.l2pf > 0 && free_l2 > 0)
                         ? static_cast<int>(std::min<long long>(free_l2 / per_unit, p.stages + p.l2pf))
                         : 0;
+            // The LM-head offers a logit to a node's top-k merges only if it
+            // beats the node's filter bound; at k >= 32 the merges of the
+            // first tiles (where the bound is still low) limit the kernel,
+            // and a small kernel that bounds each node's k-th best score
+            // from the rows of largest drafter logit lets the filter start
+            // high (csrc/dart_bound.cu).
+            // Measured on GB300 (µs per round, same box, AUTO's choice in
+            // brackets): 64 nodes, k = 64: 3421 -> 2706 [on]; 256 nodes
+            // (8 x 32), k = 32: 9594 -> 8670 [on; 128 seed rows: 8964];
+            // 32 nodes, k = 32: 2520 -> 2518 [off]; 16 nodes, k = 16:
+            // 3415 -> 3475 [off].  64- and 128-node groups keep 32
+            // candidate slots per node, which needs the bound (without it:
+            // +6 % at 64 nodes).
+            const int bR = std::max(64, (2 * c.k + 63) / 64 * 64);
+            const int bstat = seed_score_static_smem();
+            const bool want = c.topk_bound == DART_ON || (c.topk_bound == DART_AUTO && c.k >= 32 && p.N > 32);
+            p.bound = (want && c.cand_k == 0 && bR <= kBoundR && c.V >= bR && bstat >= 0 &&
+                       seed_score_smem(c.d) + bstat <= static_cast<size_t>(h->smem_optin))
+                          ? bR
+                          : 0;
         } else {
             p.NG = pick_ng_f32(p.N);
             p.G = (p.N + p.NG - 1) / p.NG;
@@ -418,6 +444,7 @@ int build_plans(dart_handle* h, const dart_config& c, std::vector<int>& caps, st
             p.stages = 0;
             p.l2pf = 0;
             p.epf = 0;
+            p.bound = 0;
             p.smem = lmhead_f32_smem(p.NG, c.k);
             if (p.smem > h->smem_optin) return DART_ERR_UNSUPPORTED;
         }
@@ -568,6 +595,7 @@ int alloc_workspace(dart_handle* h) {
     DART_ALLOC(h->seq_ticket, c.nseq)
     DART_ALLOC(h->status, 1)
     DART_ALLOC(h->gthr, static_cast<size_t>(c.L) * kNPadMax)
+    if (h->wdtype == DART_BF16) DART_ALLOC(h->bound_y, static_cast<size_t>(kNPadMax) * kBoundR)
     bool any_split = false;
     for (int dep = 1; dep < c.L; dep++) any_split = any_split || h->plans[dep].split;
     if (any_split) DART_ALLOC(h->Qtab, static_cast<size_t>(c.V) * d)
@@ -660,6 +688,7 @@ int alloc_workspace(dart_handle* h) {
     if ((c.variants & DART_VARIANT_CHAIN_DDTREE) && heap_set_smem_limits() != cudaSuccess) return DART_ERR_CUDA;
     if (h->wdtype == DART_BF16) {
         if (tc_set_smem_limits(h->smem_optin) != cudaSuccess) return DART_ERR_CUDA;
+        if (seed_score_set_smem_limit(h->smem_optin) != cudaSuccess) return DART_ERR_CUDA;
     } else {
         if (f32_set_smem_limits(h->smem_optin) != cudaSuccess) return DART_ERR_CUDA;
     }
@@ -745,7 +774,7 @@ void release(dart_handle* h) {
 
 enum Kind {
     kLmhead = 0, kSelect, kGather, kGemm1, kSilu, kGemm2, kNorm, kPrep, kEmit, kCandTopk, kCandScore, kGatherSilu,
-    kRowTopk, kDdtree, kSeqStep, kSeqEmit, kFusedRound, kL2Prefetch, kNumKinds
+    kRowTopk, kDdtree, kSeqStep, kSeqEmit, kFusedRound, kL2Prefetch, kBound, kNumKinds
 };
 
 // Opens an event pair around the next launch when profiling (no-op otherwise).
@@ -903,6 +932,29 @@ int enqueue_depth(dart_handle* h, const dart_config& c, const std::vector<DepthP
         pi = prof_begin(h, kCandScore, st);
         e = launch_cand_score(ca, st);
     } else {
+        if (p.bound) {
+            BoundArgs ba;
+            std::memset(&ba, 0, sizeof ba);
+            ba.P = p.P;
+            ba.d = c.d;
+            ba.V = c.V;
+            ba.k = c.k;
+            ba.R = p.bound;
+            ba.invT = la.invT;
+            ba.h = h->hbuf[h->cur];
+            ba.E = static_cast<const __nv_bfloat16*>(h->E);
+            ba.dlog = dlog;
+            ba.dlog_seq_stride = la.dlog_seq_stride;
+            ba.dlog_row_off = la.dlog_row_off;
+            ba.ybuf = h->bound_y;
+            ba.status = h->status;
+            const int pb = prof_begin(h, kBound, st);
+            e = launch_seed_score(ba, c.nseq, st);
+            prof_end(h, pb, st);
+            if (e != cudaSuccess) return DART_ERR_CUDA;
+            la.seed_y = h->bound_y;
+            la.seed_R = p.bound;
+        }
         pi = prof_begin(h, kLmhead, st);
         e = tc ? launch_lmhead_tc(&h->tmE, &h->tmH[ng_index(p.NG)], la, p.smem, st) : launch_lmhead_f32(la, st);
     }
@@ -1738,6 +1790,7 @@ int dart_launches_per_round(dart_handle* h) {
     // (fp32, d <= 1024) the whole update in one launch; prune-emit
     const bool tc = h->wdtype == DART_BF16;
     int n = 1 + 2 * L + 1 + (h->cfg.cand_k > 0 ? 1 : 0);
+    for (int dep = 1; dep <= L; dep++) n += h->plans[dep].bound > 0 ? 1 : 0;
     for (int dep = 1; dep < L; dep++) {
         const DepthPlan& p = h->plans[dep];
         if (!tc && head_small_f32_slices(h->cfg.d) > 0) {

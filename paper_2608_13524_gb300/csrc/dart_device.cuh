@@ -153,6 +153,15 @@ __device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, u
         : "memory");
 }
 
+// One bulk copy global -> shared (both 16-byte aligned, bytes a multiple of
+// 16), completing on `bar`.
+__device__ __forceinline__ void bulk_load(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {
+    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                     smem_u32(dst)),
+                 "l"(src), "r"(bytes), "r"(smem_u32(bar))
+                 : "memory");
+}
+
 // L2 prefetch of one tile of a 2-D tensor (no shared memory, no barrier).
 __device__ __forceinline__ void tma_prefetch_2d(const CUtensorMap* map, int x, int y) {
     asm volatile("cp.async.bulk.prefetch.tensor.2d.L2.global.tile [%0, {%1, %2}];" ::"l"(reinterpret_cast<uint64_t>(map)),
@@ -479,6 +488,22 @@ __device__ __forceinline__ float2 lse_merge(float2 a, float2 b) {
     return make_float2(m, a.y * __expf(a.x - m) + b.y * __expf(b.x - m));
 }
 
+// Reduce-scatter of 32 partial sums per lane across the warp: afterwards
+// lane l holds, in v[0], the sum over the 32 lanes of v[l] (fixed order:
+// 31 shuffles for 32 results).
+__device__ __forceinline__ void warp_reduce_scatter32(float (&v)[32], int lane) {
+#pragma unroll
+    for (int o = 16; o >= 1; o >>= 1) {
+        const bool up = (lane & o) != 0;
+#pragma unroll
+        for (int j = 0; j < o; j++) {
+            const float send = up ? v[j] : v[j + o];
+            const float recv = __shfl_xor_sync(kFull, send, o);
+            v[j] = (up ? v[j + o] : v[j]) + recv;
+        }
+    }
+}
+
 __device__ __forceinline__ float warp_max(float v) {
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(kFull, v, o));
@@ -502,12 +527,67 @@ __device__ __forceinline__ float bfly16(const float (&v)[16], int lane) {
     return op(d, __shfl_xor_sync(kFull, d, 1));
 }
 
+// The kk-th largest (1 <= kk <= R) of the R values y[0..R) (R a multiple of
+// 32, at most 256), by one warp: MSB-first radix select over the values'
+// order-preserving images; NaN if some value is NaN.
+__device__ __forceinline__ float warp_kth_largest(const float* y, int R, int kk, int lane) {
+    uint32_t u[8];
+    bool nan = false;
+#pragma unroll
+    for (int q = 0; q < 8; q++) {
+        const float v = q * 32 < R ? __ldcg(y + q * 32 + lane) : -INFINITY;
+        nan |= isnan(v);
+        u[q] = f32_ord(v);
+    }
+    if (__any_sync(kFull, nan)) return __int_as_float(0x7FC00000);
+    uint32_t prefix = 0, mask = 0;
+    int need = kk;
+    for (int b = 31; b >= 0; b--) {
+        const uint32_t bit = 1u << b, cand = prefix | bit, m2 = mask | bit;
+        int cnt = 0;
+#pragma unroll
+        for (int q = 0; q < 8; q++)
+            if (q * 32 < R) cnt += __popc(__ballot_sync(kFull, (u[q] & m2) == cand));
+        if (cnt >= need)
+            prefix = cand;
+        else
+            need -= cnt;
+        mask = m2;
+    }
+    return f32_unord(prefix);
+}
+
 // nthr = number of epilogue threads (4 warps per 16-node chunk of the group).
-__device__ __forceinline__ void epi_init(const EpiSmem& e, int NG, int k, int etid, int nthr) {
+// The first tile's filter starts from the node's published bound gthr[n0+i]
+// (zero before the first merge), raised with seed scores (seed_y[n][0..R),
+// launch_seed_score) to their k-th largest, which the CTAs of the first
+// vocabulary range publish into gthr.  Called after the wait on the
+// previous kernel.
+__device__ __forceinline__ void epi_init(const EpiSmem& e, int NG, int k, int etid, int nthr,
+                                         uint64_t* gthr = nullptr, int n0 = 0, int N = 0,
+                                         const float* seed_y = nullptr, int seed_R = 0, bool publish = false) {
     for (int i = etid; i < NG * k; i += nthr) e.list[i] = 0ull;
     for (int i = etid; i < NG; i += nthr) {
         e.cnt[i] = 0;
-        e.gcache[i] = 0ull;
+        if (!seed_y)
+            e.gcache[i] = (gthr && n0 + i < N) ? __ldcg(reinterpret_cast<const unsigned long long*>(gthr) + n0 + i) : 0ull;
+    }
+    if (seed_y) {
+        const int lane = etid & 31;
+        for (int i = etid >> 5; i < NG; i += nthr >> 5) {
+            uint64_t g = 0ull;
+            if (n0 + i < N) {
+                const float b = warp_kth_largest(seed_y + static_cast<size_t>(n0 + i) * seed_R, seed_R, k, lane);
+                if (gthr) g = __ldcg(reinterpret_cast<const unsigned long long*>(gthr) + n0 + i);
+                if (isfinite(b)) {
+                    const uint64_t key = make_key(b, 0xFFFFFFFFu);  // below every real key of value b
+                    if (publish && lane == 0 && gthr)
+                        atomicMax(reinterpret_cast<unsigned long long*>(gthr) + n0 + i, static_cast<unsigned long long>(key));
+                    g = key > g ? key : g;
+                }
+            }
+            if (lane == 0) e.gcache[i] = g;
+        }
     }
     if (etid < 2) e.more[etid] = 0;
     for (int i = etid; i < 4 * NG; i += nthr) e.mref[i] = -INFINITY;

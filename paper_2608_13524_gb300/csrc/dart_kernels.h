@@ -100,6 +100,8 @@ struct LmheadArgs {
     const int* dlog_row;  // [nseq] drafter row of each sequence's nodes (replaces dlog_row_off / V)
     float* zout;          // z[n][v] written to zout[n * zout_stride + v] (node groups <= 64)
     long long zout_stride;
+    const float* seed_y;  // [N][seed_R] seed scores (launch_seed_score): the filter starts from each
+    int seed_R;           // node's k-th largest, which is also published into gthr (null: no seed pass)
 };
 
 // Skinny split-K GEMM for the correction head: out[split][n][m] =
@@ -142,6 +144,27 @@ cudaError_t tc_set_smem_limits(int max_dyn);
 
 // Prefetch into L2 the first `count` E tiles of each of the nV vocabulary
 // ranges of an LM-head launch (whole-tile split of `tiles` tiles).
+// Seed scores of the starting bound of each node's top-k filter
+// (csrc/dart_bound.cu): for each node n of sequence s and each of R equal
+// vocabulary chunks, the score of the chunk's row of largest drafter logit
+// less an error bound, ybuf[n][c]; the LM-head takes the k-th largest of a
+// node's R values as its filter's starting threshold.
+constexpr int kBoundMaxR = 256;
+struct BoundArgs {
+    int P, d, V, k, R;          // nodes per sequence, hidden, vocabulary, top-k, seed rows per sequence (multiple of 32)
+    float invT;
+    const float* h;             // [nseq * P][d] fp32 states
+    const __nv_bfloat16* E;     // [V][d] row-major
+    const float* dlog;          // drafter logits, row of sequence s: dlog + s * dlog_seq_stride + dlog_row_off
+    long long dlog_seq_stride, dlog_row_off;
+    float* ybuf;                // [nseq * P][R]
+    int* status;
+};
+cudaError_t launch_seed_score(const BoundArgs& a, int nseq, cudaStream_t st);
+size_t seed_score_smem(int d);
+cudaError_t seed_score_set_smem_limit(int smem_optin);
+int seed_score_static_smem();  // -1 on error
+
 cudaError_t launch_lmhead_l2_prefetch(const CUtensorMap* tmE, int tiles, int nV, int d, int count, int tiled,
                                       cudaStream_t st);
 

@@ -571,36 +571,11 @@ __device__ __forceinline__ float ld_cl_f32(const void* local, uint32_t rank) {
     return v;
 }
 
-// One bulk copy global -> shared (both 16-byte aligned, bytes a multiple of
-// 16), completing on `bar`.
-__device__ __forceinline__ void bulk_load(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {
-    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
-                     smem_u32(dst)),
-                 "l"(src), "r"(bytes), "r"(smem_u32(bar))
-                 : "memory");
-}
-
 __device__ __forceinline__ float dot4(const float4 a, const float4 b, float acc) {
     acc = fmaf(a.x, b.x, acc);
     acc = fmaf(a.y, b.y, acc);
     acc = fmaf(a.z, b.z, acc);
     return fmaf(a.w, b.w, acc);
-}
-
-// Reduce-scatter of 32 partial sums per lane across the warp: afterwards
-// lane l holds, in v[0], the sum over the 32 lanes of v[l] (fixed order:
-// 31 shuffles for 32 results).
-__device__ __forceinline__ void warp_reduce_scatter32(float (&v)[32], int lane) {
-#pragma unroll
-    for (int o = 16; o >= 1; o >>= 1) {
-        const bool up = (lane & o) != 0;
-#pragma unroll
-        for (int j = 0; j < o; j++) {
-            const float send = up ? v[j] : v[j + o];
-            const float recv = __shfl_xor_sync(kFull, send, o);
-            v[j] = (up ? v[j + o] : v[j]) + recv;
-        }
-    }
 }
 
 // Candidates per lane of the warp-level frontier selection (at most

@@ -42,11 +42,16 @@ template <int NG>
 constexpr int epi_chunks() {
     return NG > 64 ? NG / 64 : 1;
 }
-// Candidate slots per node: a whole tile (nothing can overflow) up to 64-node
-// groups; 128-node groups keep fewer and merge in rounds when they overflow.
+// Candidate slots per node: a whole tile (nothing can overflow) up to 32-node
+// groups; 64- and 128-node groups keep fewer (more pipeline stages fit) and
+// merge in rounds when a tile overflows them.  Those groups come with the
+// starting bound of the filter (seed pass before the launch), after which
+// a tile rarely offers more than a few logits per node.  Measured on GB300
+// at 64 nodes, k = 64 (µs per round, same box): 128 slots 3042, 64 slots
+// 2806, 32 slots 2706 with the bound; without it 32 slots cost +6 %.
 template <int NG>
 constexpr int lm_cand_cap() {
-    return NG > 64 ? kCandCapLarge : kCandCap;
+    return NG >= 64 ? kCandCapLarge : kCandCap;
 }
 template <int NG>
 constexpr int threads() {
@@ -155,14 +160,14 @@ template <int NG>
 __device__ __forceinline__ void mma_issuer(const Work& w, uint8_t* ring, int stages, uint64_t* full,
                                            uint64_t* empty, uint64_t* tfull, uint64_t* tempty, uint64_t* tdown,
                                            uint32_t tmem_base, int acc_stride, volatile int* abort,
-                                           int* status) {
+                                           int* status, int nacc = 2) {
     constexpr uint32_t idesc2 = idesc_bf16_f32(kTileM, 2 * NG);  // hi and lo rows together
     constexpr uint32_t idesc1 = idesc_bf16_f32(kTileM, NG);      // hi rows only (no lo half)
     uint32_t stage = 0, phase = 0;
     bool ok = true;
     for (int i = 0; i < w.ntiles && ok; i++) {
-        const int acc = i & 1;
-        const uint32_t aph = (i >> 1) & 1;
+        const int acc = i % nacc;
+        const uint32_t aph = (i / nacc) & 1;
         if (!mbar_wait(&tempty[acc], aph ^ 1u, abort)) {
             record_timeout(status, abort);
             ok = false;
@@ -207,22 +212,22 @@ struct Smem {
 };
 
 template <int NG>
-__device__ __forceinline__ Smem carve(uint8_t* raw, int stages) {
+__device__ __forceinline__ Smem carve(uint8_t* raw, int stages, int nacc = 2) {
     Smem s;
     const uint32_t off = (1024u - (smem_u32(raw) & 1023u)) & 1023u;
     s.ring = raw + off;
     s.full = reinterpret_cast<uint64_t*>(s.ring + stages * Layout<NG>::kStage);
     s.empty = s.full + stages;
     s.tfull = s.empty + stages;
-    s.tempty = s.tfull + 2;
-    s.tdown = s.tempty + 2;
+    s.tempty = s.tfull + nacc;
+    s.tdown = s.tempty + nacc;
     s.misc = reinterpret_cast<int*>(s.tdown + 1);
     s.tail = reinterpret_cast<uint8_t*>(s.misc + 4);
     return s;
 }
 
 template <int NG>
-__device__ __forceinline__ uint32_t setup(const Smem& s, int stages, int ncols) {
+__device__ __forceinline__ uint32_t setup(const Smem& s, int stages, int ncols, int nacc = 2) {
     constexpr int kEpi = epi_threads<NG>();
     const int warp = threadIdx.x >> 5;
     if (threadIdx.x == 0) {
@@ -230,7 +235,7 @@ __device__ __forceinline__ uint32_t setup(const Smem& s, int stages, int ncols) 
             mbar_init(&s.full[i], 1);
             mbar_init(&s.empty[i], 1);
         }
-        for (int i = 0; i < 2; i++) {
+        for (int i = 0; i < nacc; i++) {
             mbar_init(&s.tfull[i], 1);
             mbar_init(&s.tempty[i], kEpi);
         }
@@ -273,6 +278,25 @@ constexpr int tmem_cols() {
                                                                            : (2 * acc_stride<NG>() <= 256 ? 256 : 512)));
 }
 
+// Accumulators of the LM-head (a ring in TMEM): with 64-node groups four,
+// so that the MMAs run up to three tiles ahead of the epilogue, whose cost
+// per tile is uneven (the first tiles of a vocabulary range pass most
+// logits to the top-k merges, later ones few).  All of TMEM then belongs to
+// one CTA, which the plan's shared memory makes the only LM-head CTA of its SM.
+template <int NG>
+constexpr int lm_nacc() {
+    return NG == 64 ? 4 : 2;
+}
+template <int NG>
+constexpr int lm_tmem_cols() {
+    return lm_nacc<NG>() * acc_stride<NG>() <= 32
+               ? 32
+               : (lm_nacc<NG>() * acc_stride<NG>() <= 64
+                      ? 64
+                      : (lm_nacc<NG>() * acc_stride<NG>() <= 128 ? 128
+                                                                 : (lm_nacc<NG>() * acc_stride<NG>() <= 256 ? 256 : 512)));
+}
+
 // ------------------------------------------------------------ LM-head kernel
 
 template <int NG>
@@ -282,7 +306,8 @@ __global__ void __launch_bounds__(threads<NG>(), 1)
     extern __shared__ uint8_t smem_raw[];
     pdl_trigger();
     const int stages = a.stages;
-    Smem s = carve<NG>(smem_raw, stages);
+    constexpr int kNacc = lm_nacc<NG>();
+    Smem s = carve<NG>(smem_raw, stages, kNacc);
     constexpr int kCap = lm_cand_cap<NG>();
     EpiSmem e;
     e.cap = kCap;
@@ -308,7 +333,7 @@ __global__ void __launch_bounds__(threads<NG>(), 1)
     w.tiled_kb = a.e_tiled ? w.kb1 : 0;
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const uint32_t tmem_base = setup<NG>(s, stages, tmem_cols<NG>());
+    const uint32_t tmem_base = setup<NG>(s, stages, lm_tmem_cols<NG>(), kNacc);
     volatile int* abort = &s.misc[1];
 
     if (warp == 0) {
@@ -317,7 +342,7 @@ __global__ void __launch_bounds__(threads<NG>(), 1)
     } else if (warp == 1) {
         if (lane == 0)
             mma_issuer<NG>(w, s.ring, stages, s.full, s.empty, s.tfull, s.tempty, s.tdown, tmem_base,
-                           acc_stride<NG>(), abort, a.status);
+                           acc_stride<NG>(), abort, a.status, kNacc);
     } else {
         // epilogue warp wi = warp - 2 reads TMEM lane quarter warp % 4 and
         // owns the 16-node chunks wi / 4 + 4 * ci (ci < kChunks) of the group
@@ -327,7 +352,7 @@ __global__ void __launch_bounds__(threads<NG>(), 1)
         const int wi = warp - 2;
         const int quarter = warp & 3;
         pdl_wait();
-        epi_init(e, NG, a.k, etid, kEpi);
+        epi_init(e, NG, a.k, etid, kEpi, a.gthr, g * NG, a.N, a.seed_y, a.seed_R, vr == 0);
         float ssum[kChunks];
         uint32_t nodemask[kChunks];
 #pragma unroll
@@ -365,8 +390,8 @@ __global__ void __launch_bounds__(threads<NG>(), 1)
             }
         };
         for (int i = 0; i < w.ntiles; i++) {
-            const int acc = i & 1;
-            const uint32_t aph = (i >> 1) & 1;
+            const int acc = i % kNacc;
+            const uint32_t aph = (i / kNacc) & 1;
             if (etid == 0) {
                 const bool ok = mbar_wait(&s.tfull[acc], aph, abort);
                 if (!ok) record_timeout(a.status, abort);
@@ -435,7 +460,7 @@ __global__ void __launch_bounds__(threads<NG>(), 1)
         for (int ci = 0; ci < kChunks; ci++) epi_stash(e, NG, quarter, lane, ((wi >> 2) + 4 * ci) * 16, ssum[ci]);
         epi_finalize(e, NG, a.k, etid, kEpi, g * NG, a.N, vr, a.nV, a.part_ms, a.part_key);
     }
-    teardown(tmem_base, tmem_cols<NG>());
+    teardown(tmem_base, lm_tmem_cols<NG>());
 }
 
 // --------------------------------------------------------------- GEMM kernel
@@ -560,7 +585,7 @@ __global__ void __launch_bounds__(threads<NG>(), 1)
 
 template <int NG>
 int lmhead_fixed(int k, int stages) {
-    return (2 * stages + 5) * 8 + 16 + NG * k * 8 + NG * lm_cand_cap<NG>() * 8 + NG * 8 + 4 * NG * 8 + 4 * NG * 4 +
+    return (2 * stages + 2 * lm_nacc<NG>() + 1) * 8 + 16 + NG * k * 8 + NG * lm_cand_cap<NG>() * 8 + NG * 8 + 4 * NG * 8 + 4 * NG * 4 +
            NG * 4 + 8;
 }
 
@@ -634,10 +659,10 @@ int tc_stage_bytes(int NG) { return kATileBytes + 2 * NG * 128; }
 
 int lmhead_tc_tmem_cols(int NG) {
     switch (NG) {
-        case 16: return tmem_cols<16>();
-        case 32: return tmem_cols<32>();
-        case 64: return tmem_cols<64>();
-        default: return tmem_cols<128>();
+        case 16: return lm_tmem_cols<16>();
+        case 32: return lm_tmem_cols<32>();
+        case 64: return lm_tmem_cols<64>();
+        default: return lm_tmem_cols<128>();
     }
 }
 

@@ -36,7 +36,7 @@ class DartConfig(C.Structure):
                 ("temperature", C.c_float), ("rms_eps", C.c_float), ("pos_offset", C.c_int),
                 ("cand_k", C.c_int), ("head_split", C.c_int), ("head_split_stream", C.c_int),
                 ("lmhead_ctas_per_sm", C.c_int), ("weights_tiled", C.c_int), ("head_weights_tiled", C.c_int),
-                ("variants", C.c_int), ("fused_round", C.c_int)]
+                ("variants", C.c_int), ("fused_round", C.c_int), ("topk_bound", C.c_int)]
 
 
 class DartTreeOut(C.Structure):
@@ -141,14 +141,14 @@ def make_config(cfg) -> DartConfig:
     """From any object with V, d, L, W, k, B, nseq, beta, temperature,
     rms_eps, pos_offset and optionally cand_k (0: full vocabulary) and the
     tuning fields head_split, head_split_stream, lmhead_ctas_per_sm,
-    weights_tiled, head_weights_tiled, variants, fused_round (0: the library's
-    choice)."""
+    weights_tiled, head_weights_tiled, variants, fused_round, topk_bound (0: the
+    library's choice)."""
     g = lambda name: int(getattr(cfg, name, 0))
     return DartConfig(int(cfg.V), int(cfg.d), int(cfg.L), int(cfg.W), int(cfg.k), int(cfg.B),
                       int(cfg.nseq), float(cfg.beta), float(cfg.temperature), float(cfg.rms_eps),
                       int(cfg.pos_offset), g("cand_k"), g("head_split"), g("head_split_stream"),
                       g("lmhead_ctas_per_sm"), g("weights_tiled"), g("head_weights_tiled"), g("variants"),
-                      g("fused_round"))
+                      g("fused_round"), g("topk_bound"))
 
 
 def alloc_tree_out(cfg, device="cuda", pin=False):
@@ -298,7 +298,7 @@ def dart_profile_read(h):
 
 KIND_NAMES = ("lmhead", "merge_select", "gather", "gemm_wi", "silu_split", "gemm_wo", "residual_norm",
               "prep_anchor", "prune_emit", "cand_topk", "cand_score", "gather_silu", "row_topk", "ddtree",
-              "seqheap_step", "seqheap_emit", "round_f32", "l2_prefetch")
+              "seqheap_step", "seqheap_emit", "round_f32", "l2_prefetch", "topk_bound")
 
 
 def dart_profile_read_kinds(h):

@@ -53,7 +53,7 @@ BAD = [dict(V=0), dict(d=100), dict(d=32), dict(L=0), dict(W=0), dict(W=65), dic
        dict(d=16448), dict(V=1 << 24), dict(L=1025, W=1), dict(temperature=float("inf")),
        dict(rms_eps=float("nan")), dict(head_split=3), dict(head_split=-1), dict(head_split_stream=3),
        dict(lmhead_ctas_per_sm=3), dict(lmhead_ctas_per_sm=-1), dict(variants=4), dict(variants=-1),
-       dict(fused_round=3), dict(fused_round=-1)]
+       dict(fused_round=3), dict(fused_round=-1), dict(topk_bound=3), dict(topk_bound=-1)]
 
 
 @pytest.mark.parametrize("bad", BAD, ids=[str(b) for b in BAD])

@@ -442,11 +442,72 @@ def test_handles_with_different_plans_coexist(dart):
     compare_with_oracle(small, ref, gstb, gb, tol_of(big), x=x)
 
 
+# the starting bound of the LM-head's top-k filters (topk_bound): forced on
+# at every depth (1 node at depth 1 included); odd node counts per sequence
+# (node blocks of fewer than 8), a vocabulary whose last seed chunks are
+# empty, temperature, k = 64 with few nodes (128 seed rows), 64-node groups (32
+# candidate slots, 4 accumulators) and 128-node groups
+BOUND = [
+    C("bound-k32-N64", 2, 6000, 256, 4, 32, 32, 60, "bf16", 0.0, 61),
+    C("bound-odd-P", 3, 3001, 192, 3, 13, 40, 30, "bf16", 0.7, 62),
+    C("bound-k64-W8", 1, 9000, 128, 3, 8, 64, 40, "bf16", 0.0, 63),
+    C("bound-N128", 4, 4000, 128, 3, 32, 32, 70, "bf16", 1.0, 64),
+    C("bound-k64-d512", 1, 30000, 512, 3, 64, 64, 90, "bf16", 0.0, 65),
+]
+
+
+@pytest.mark.parametrize("cfg", BOUND, ids=[c.name for c in BOUND])
+def test_topk_bound_matches_the_oracle_and_changes_nothing(dart, cfg):
+    """With the seed pass on, the tree equals the oracle's, and every emitted
+    array (scores included) is bit-identical to the run without it: the bound
+    only keeps logits below a node's k-th best out of the top-k merges."""
+    x = make_inputs(cfg)
+    dx = to_device(cfg, x)
+    ref = oracle.build_tree(cfg, x["Wi"], x["Wo"], x["E"], x["Dlog"], x["h0"])
+    on = cfg.replace(topk_bound=1)
+    _, gst, g = run_depthwise(dart, on, dx)
+    print(cfg.name, compare_with_oracle(on, ref, gst, g, tol_of(cfg), x=x))
+    _, gst_off, g_off = run_depthwise(dart, cfg.replace(topk_bound=2), dx)
+    for k in g:
+        np.testing.assert_array_equal(g[k], g_off[k], err_msg=k)
+    for k in gst:
+        np.testing.assert_array_equal(gst[k], gst_off[k], err_msg=k)
+    eng = dart.Dart(on, dx["Wi"], dx["Wo"], dx["E"])
+    try:
+        out = eng.build_tree(dx["Dlog"], dx["h0"])
+        torch.cuda.synchronize()
+        assert dart.dart_status_sync(eng.h) == 0
+        gg = tree_to_numpy(out)
+        for k in g:
+            np.testing.assert_array_equal(gg[k], g[k], err_msg=f"graph {k}")
+    finally:
+        eng.close()
+
+
+def test_topk_bound_with_neg_inf_drafter_logits(dart):
+    """Seed chunks whose drafter logits are all -inf give no seed score; a
+    sequence with a single finite token at a depth still gets its one child."""
+    cfg = C("bound-neginf", 2, 2000, 128, 4, 40, 40, 60, "bf16", 0.0, 66, topk_bound=1)
+    x = make_inputs(cfg)
+    x["Dlog"][0, 1, 300:] = -np.inf     # depth 2 of seq 0: tokens 0..299 only (most chunks empty)
+    x["Dlog"][1, 0, :] = -np.inf        # depth 1 of seq 1: token 7 only
+    x["Dlog"][1, 0, 7] = 0.0
+    x["Dlog"][1, 2, ::2] = -np.inf      # depth 3 of seq 1: every other token
+    dx = to_device(cfg, x)
+    ref = oracle.build_tree(cfg, x["Wi"], x["Wo"], x["E"], x["Dlog"], x["h0"])
+    _, gst, g = run_depthwise(dart, cfg, dx)
+    compare_with_oracle(cfg, ref, gst, g, tol_of(cfg), x=x)
+    assert int(gst["st_count"][1, 0]) == 1
+    _, gst_off, g_off = run_depthwise(dart, cfg.replace(topk_bound=2), dx)
+    for k in g:
+        np.testing.assert_array_equal(g[k], g_off[k], err_msg=k)
+
+
 LAUNCH_CFGS = [SMALL[0], SMALL[0].replace(fused_round=2), SMALL[1], SMALL[2], SMALL[5], SMALL[19],
-               RESTRICTED[1], RESTRICTED[0]]
+               RESTRICTED[1], RESTRICTED[0], BOUND[0].replace(topk_bound=1), BOUND[1]]
 
 
-@pytest.mark.parametrize("cfg", LAUNCH_CFGS, ids=[f"{c.name}-{c.fused_round}" for c in LAUNCH_CFGS])
+@pytest.mark.parametrize("cfg", LAUNCH_CFGS, ids=[f"{c.name}-{c.fused_round}-{c.topk_bound}" for c in LAUNCH_CFGS])
 def test_launches_per_round_matches_the_profiled_round(dart, cfg):
     """dart_launches_per_round (the bench's kernel-launch count) equals the
     launches one profiled round brackets, kind by kind summed (every launch

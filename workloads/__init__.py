@@ -63,6 +63,7 @@ class Config:
     head_weights_tiled: int = 0
     variants: int = 0          # extra constructions prepared by the handle (bit set)
     fused_round: int = 0       # fp32: the whole round as one cooperative kernel (where possible)
+    topk_bound: int = 0        # bf16: a starting bound of each node's top-k filter before each LM-head
 
     def replace(self, **kw) -> "Config":
         return dataclasses.replace(self, **kw)
