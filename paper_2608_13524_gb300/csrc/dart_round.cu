@@ -618,6 +618,46 @@ __device__ void select_frontier_cluster(const SelectArgs& a, int s, int prev_cou
     const int cnt = min(a.W, valid);
     __syncwarp();  // every lane has read fscore before it is overwritten
     const size_t tb = (static_cast<size_t>(s) * a.L + a.dep - 1) * a.W;
+    auto keep = [&](int r, uint64_t tp, int tk) {
+        const int pp = static_cast<int>(key_idx(tp)) / a.k;
+        const float sc = key_val(tp);
+        fscore[r] = sc;
+        a.tree_tok[tb + r] = tk;
+        a.tree_parent[tb + r] = a.dep == 1 ? -1 : pp;
+        a.tree_score[tb + r] = sc;
+        if (r < a.Pn) {
+            cprow[r] = pp;
+            ctokr[r] = tk;
+            a.child_prow[s * a.Pn + r] = s * a.P + pp;
+            a.child_tok[s * a.Pn + r] = tk;
+        }
+    };
+    auto empty = [&](int r) {
+        a.tree_tok[tb + r] = -1;
+        a.tree_parent[tb + r] = -1;
+        a.tree_score[tb + r] = -INFINITY;
+        if (r < a.Pn) {
+            cprow[r] = -1;
+            ctokr[r] = 0;
+            a.child_prow[s * a.Pn + r] = -1;
+            a.child_tok[s * a.Pn + r] = 0;
+        }
+    };
+    if (ncand <= 32) {
+        // one candidate per lane: its rank among all keys (distinct) in one
+        // pass of 32 independent shuffles instead of W dependent maxima
+        const uint64_t mine = key[0];
+        int rank = 0;
+#pragma unroll
+        for (int src = 0; src < 32; src++) rank += shfl_u64(mine, src) > mine ? 1 : 0;
+        if (mine != 0ull && rank < cnt) keep(rank, mine, tok[0]);
+        for (int r = cnt + lane; r < a.W; r += 32) empty(r);
+        if (lane == 0) {
+            *fcount = cnt;
+            a.tree_count[s * a.L + a.dep - 1] = cnt;
+        }
+        return;
+    }
     for (int r = 0; r < a.W; r++) {
         uint64_t best = 0ull;
 #pragma unroll
@@ -628,30 +668,11 @@ __device__ void select_frontier_cluster(const SelectArgs& a, int s, int prev_cou
             for (int u = 0; u < kCandLane; u++) {
                 if (key[u] == tp) {  // the one owner lane (the keys are distinct)
                     key[u] = 0ull;
-                    const int pp = static_cast<int>(key_idx(tp)) / a.k;
-                    const float sc = key_val(tp);
-                    fscore[r] = sc;
-                    a.tree_tok[tb + r] = tok[u];
-                    a.tree_parent[tb + r] = a.dep == 1 ? -1 : pp;
-                    a.tree_score[tb + r] = sc;
-                    if (r < a.Pn) {
-                        cprow[r] = pp;
-                        ctokr[r] = tok[u];
-                        a.child_prow[s * a.Pn + r] = s * a.P + pp;
-                        a.child_tok[s * a.Pn + r] = tok[u];
-                    }
+                    keep(r, tp, tok[u]);
                 }
             }
         } else if (lane == 0) {
-            a.tree_tok[tb + r] = -1;
-            a.tree_parent[tb + r] = -1;
-            a.tree_score[tb + r] = -INFINITY;
-            if (r < a.Pn) {
-                cprow[r] = -1;
-                ctokr[r] = 0;
-                a.child_prow[s * a.Pn + r] = -1;
-                a.child_tok[s * a.Pn + r] = 0;
-            }
+            empty(r);
         }
     }
     if (lane == 0) {
@@ -896,6 +917,15 @@ __global__ void __launch_bounds__(kRoundThreads, 1) round_cluster_f32_kernel(con
                 acc = (lane & o) ? lse_merge(other, acc) : lse_merge(acc, other);
             }
             const float lse = acc.x == -INFINITY ? -INFINITY : acc.x + logf(acc.y);
+            auto put = [&](int j, uint64_t tp) {
+                const float z = tp != 0ull ? key_val(tp) : -INFINITY;
+                const float lq = (lse != -INFINITY && z != -INFINITY) ? fminf(z - lse, 0.0f) : -INFINITY;
+                const int tkn = tp != 0ull ? static_cast<int>(key_idx(tp)) : -1;
+                lq_out[j] = lq;
+                tok_out[j] = tkn;
+                nlq[p * k + j] = lq;
+                ntok[p * k + j] = tkn;
+            };
             int ptr = 0;
             uint64_t head = lane < kCS ? ld_cl_u64(&pkey_s[p * k], static_cast<uint32_t>(lane)) : 0ull;
             uint64_t nxt = lane < kCS && k > 1 ? ld_cl_u64(&pkey_s[p * k + 1], static_cast<uint32_t>(lane)) : 0ull;
@@ -906,15 +936,7 @@ __global__ void __launch_bounds__(kRoundThreads, 1) round_cluster_f32_kernel(con
                     head = nxt;
                     nxt = ptr + 1 < k ? ld_cl_u64(&pkey_s[p * k + ptr + 1], static_cast<uint32_t>(lane)) : 0ull;
                 }
-                if (lane == 0) {
-                    const float z = tp != 0ull ? key_val(tp) : -INFINITY;
-                    const float lq = (lse != -INFINITY && z != -INFINITY) ? fminf(z - lse, 0.0f) : -INFINITY;
-                    const int tkn = tp != 0ull ? static_cast<int>(key_idx(tp)) : -1;
-                    lq_out[j] = lq;
-                    tok_out[j] = tkn;
-                    nlq[p * k + j] = lq;
-                    ntok[p * k + j] = tkn;
-                }
+                if (lane == 0) put(j, tp);
             }
             if (lane == 0) a.node_lse[n] = lse;
         }

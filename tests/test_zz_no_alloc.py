@@ -89,6 +89,38 @@ def test_noalloc_matches_handle_path_twice(dart, nseq, V, d, W, k, T):
             assert np.all(got[3][:, k:] == -1) and np.all(np.isneginf(got[4][:, k:]))
 
 
+@pytest.mark.parametrize("nseq,V,d,W,k,T", [(3, 20000, 512, 8, 12, 0.7), (40, 5000, 256, 6, 4, 0.0)])
+def test_noalloc_matches_the_oracle(dart, nseq, V, d, W, k, T):
+    """Depth 1 of Algorithm 1 from the allocation-free entry point against the
+    fp64 oracle directly: each root's k best children (tokens exact where the
+    oracle's gaps exceed the tolerance), log q~, log-sum-exp, and the
+    frontier S_1 with its scores and size."""
+    import oracle
+    cfg = Config("noalloc-oracle", nseq, V, d, 1, W, k, 20, "bf16", T, 9100 + nseq)
+    x = make_inputs(cfg)
+    dx = to_device(cfg, x)
+    ref = oracle.build_tree(cfg, x["Wi"], x["Wo"], x["E"], x["Dlog"], x["h0"])
+    tol = tol_of(cfg)
+    out = outputs(nseq, W, k)
+    dart.dart_expand_root_noalloc(cfg, dx["E"], dx["Dlog"], dx["h0"], *out)
+    assert dart.dart_noalloc_status() == dart.DART_OK
+    tok, logq, lse, ftok, fsc, fcnt = [t.cpu().numpy() for t in out]
+    for s in range(nseq):
+        rl, rt = ref["nd_logq"][s, 0, 0, :k], ref["nd_tok"][s, 0, 0, :k]
+        assert abs(float(lse[s]) - ref["nd_lse"][s, 0, 0]) <= tol
+        fin = np.isfinite(rl)
+        assert np.all(np.abs(logq[s][fin] - rl[fin]) <= tol)
+        gaps = -np.diff(ref["nd_logq"][s, 0, 0])
+        if np.all(gaps[:k] >= tol):
+            np.testing.assert_array_equal(tok[s], rt)
+        n = int(ref["st_count"][s, 0])
+        assert int(fcnt[s]) == n
+        rs = ref["st_score"][s, 0, :n]
+        assert np.all(np.abs(fsc[s, :n] - rs) <= tol)
+        if n < 2 or np.all(-np.diff(rs) >= tol):
+            np.testing.assert_array_equal(ftok[s, :n], ref["st_tok"][s, 0, :n])
+
+
 def test_noalloc_rejects_sizes_beyond_its_array(dart):
     lib = dart.lib()
     big = Config("toolarge", 65, 1000, 128, 2, 2, 2, 4, "bf16", 0.0, 1)
