@@ -992,8 +992,19 @@ __global__ void __launch_bounds__(kRoundThreads, 1) round_cluster_f32_kernel(con
                 a.wres ? wis + static_cast<size_t>(fok ? il : 0) * 2 * d
                        : a.Wi + static_cast<size_t>(rank * F + (fok ? il : 0)) * 2 * d);
             float acc[NP];
+            // each child's operand [h_p ; E[t_c]] as two row pointers, the
+            // slot's parent read once (one shared-memory load per product)
+            const float4* hrow[NP];
+            const float4* xrow[NP];
+            bool use[NP];
 #pragma unroll
-            for (int c = 0; c < NP; c++) acc[c] = 0.0f;
+            for (int c = 0; c < NP; c++) {
+                acc[c] = 0.0f;
+                const int cp = c < Pn ? cpar[c] : -1;
+                use[c] = cp >= 0;
+                hrow[c] = hs4 + (cp >= 0 ? cp : 0) * d4;
+                xrow[c] = xb4 + c * d4 - d4;
+            }
             for (int q0 = sl; q0 < 2 * d4; q0 += 16 * 8) {
                 float4 wv[8];
 #pragma unroll
@@ -1005,8 +1016,7 @@ __global__ void __launch_bounds__(kRoundThreads, 1) round_cluster_f32_kernel(con
                     if (q < 2 * d4) {
 #pragma unroll
                         for (int c = 0; c < NP; c++) {
-                            if (c < Pn && cpar[c] >= 0)
-                                acc[c] = dot4(wv[u], q < d4 ? hs4[cpar[c] * d4 + q] : xb4[c * d4 + q - d4], acc[c]);
+                            if (use[c]) acc[c] = dot4(wv[u], (q < d4 ? hrow[c] : xrow[c])[q], acc[c]);
                         }
                     }
                 }
@@ -1033,8 +1043,12 @@ __global__ void __launch_bounds__(kRoundThreads, 1) round_cluster_f32_kernel(con
             const float4* wr = reinterpret_cast<const float4*>(a.wres ? wos + static_cast<size_t>(fok ? il : 0) * d
                                                                        : a.Wo + static_cast<size_t>(i) * d);
             float acc[NP];
+            bool use[NP];
 #pragma unroll
-            for (int c = 0; c < NP; c++) acc[c] = 0.0f;
+            for (int c = 0; c < NP; c++) {
+                acc[c] = 0.0f;
+                use[c] = c < Pn && cpar[c] >= 0;
+            }
             for (int q0 = sl; q0 < d4; q0 += 16 * 8) {
                 float4 wv[8];
 #pragma unroll
@@ -1046,7 +1060,7 @@ __global__ void __launch_bounds__(kRoundThreads, 1) round_cluster_f32_kernel(con
                     if (q < d4) {
 #pragma unroll
                         for (int c = 0; c < NP; c++)
-                            if (c < Pn && cpar[c] >= 0) acc[c] = dot4(wv[u], xb4[c * d4 + q], acc[c]);
+                            if (use[c]) acc[c] = dot4(wv[u], xb4[c * d4 + q], acc[c]);
                     }
                 }
             }
