@@ -136,9 +136,9 @@ enum {
  *                      logit in max(64, 2k) vocabulary chunks), and the
  *                      LM-head's top-k filter starts from that bound instead
  *                      of offering every logit of its first tiles to the
- *                      list merges.  The tree is unchanged.  AUTO = ON for
- *                      k >= 32 at depths of more than 32 nodes (where it was
- *                      measured faster) */
+ *                      list merges.  The tree is unchanged.  AUTO = ON at
+ *                      depths of more than 32 nodes (where it was measured
+ *                      faster) */
 typedef struct {
     int V, d, L, W, k, B, nseq;
     float beta, temperature, rms_eps;

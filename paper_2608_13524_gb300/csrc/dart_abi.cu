@@ -419,15 +419,16 @@ int build_plans(dart_handle* h, const dart_config& c, std::vector<int>& caps, st
             // from the rows of largest drafter logit lets the filter start
             // high (csrc/dart_bound.cu).
             // Measured on GB300 (µs per round, same box, AUTO's choice in
-            // brackets): 64 nodes, k = 64: 3421 -> 2706 [on]; 256 nodes
-            // (8 x 32), k = 32: 9594 -> 8670 [on; 128 seed rows: 8964];
-            // 32 nodes, k = 32: 2520 -> 2518 [off]; 16 nodes, k = 16:
-            // 3415 -> 3475 [off].  64- and 128-node groups keep 32
-            // candidate slots per node, which needs the bound (without it:
-            // +6 % at 64 nodes).
+            // brackets): 64 nodes, k = 64: 3421 -> 2706 [on]; 64 nodes
+            // (4 x 16), k = 16: 2743 -> 2664 [on]; 256 nodes (8 x 32),
+            // k = 32: 9594 -> 8670 [on; 128 seed rows: 8964]; 256 nodes,
+            // k = 8: 8495 -> 8286 [on]; 32 nodes, k = 32: 2520 -> 2518
+            // [off]; 16 nodes, k = 16: 3415 -> 3475 [off].  64- and
+            // 128-node groups keep 32 candidate slots per node, which needs
+            // the bound (without it: +6 % at 64 nodes, k = 64).
             const int bR = std::max(64, (2 * c.k + 63) / 64 * 64);
             const int bstat = seed_score_static_smem();
-            const bool want = c.topk_bound == DART_ON || (c.topk_bound == DART_AUTO && c.k >= 32 && p.N > 32);
+            const bool want = c.topk_bound == DART_ON || (c.topk_bound == DART_AUTO && p.N > 32);
             p.bound = (want && c.cand_k == 0 && bR <= kBoundR && c.V >= bR && bstat >= 0 &&
                        seed_score_smem(c.d) + bstat <= static_cast<size_t>(h->smem_optin))
                           ? bR
