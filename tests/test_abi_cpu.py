@@ -141,3 +141,14 @@ def test_tree_attention_rejects_a_small_workspace_on_host():
     p = (C.cast(buf, C.c_void_p).value + 255) & ~255
     rc = lib.dart_tree_attention(C.byref(cfg), p, p, p, p, p, p, p, p, p, p, need - 1, None, None)
     assert rc == dart.DART_ERR_INVALID
+
+
+def test_profiling_kind_names_match_the_header():
+    """The binding names as many profiling kinds as dart_profile_read_kinds
+    accepts (include/dart.h), and the kinds numbered there are in the same
+    order (the last one: the starting bound of the top-k filters)."""
+    hdr = open(os.path.join(ROOT, "include", "dart.h")).read()
+    n = int(re.search(r"nkinds <= (\d+)", hdr).group(1))
+    assert len(dart.KIND_NAMES) == n
+    assert dart.KIND_NAMES[-1] == "topk_bound" and re.search(rf"{n - 1} the starting bound of the top-k filters", hdr)
+    assert dart.KIND_NAMES[16] == "round_f32" and dart.KIND_NAMES[17] == "l2_prefetch"
