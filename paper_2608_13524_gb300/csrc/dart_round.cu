@@ -825,7 +825,21 @@ __global__ void __launch_bounds__(kRoundThreads, 1) round_cluster_f32_kernel(con
             hcur[static_cast<size_t>(s * P + p) * d + i] = hs[p * d + i];
         }
         // A2: z of this block's rows for the P nodes: warps take RS rows at a
-        // time, lanes split d; the partial sums are reduce-scattered
+        // time, lanes split d; the partial sums are reduce-scattered.  Where
+        // the nodes' states fit (NP * d/128 float4 per lane <= 8) each lane
+        // keeps its share of them in registers for all chunks of the depth
+        constexpr int kQR = NP <= 8 ? 8 / NP : 1;
+        const bool hreg = NP <= 8 && d4 <= 32 * kQR;
+        float4 hr[kQR * NP];
+        if (hreg) {
+#pragma unroll
+            for (int qi = 0; qi < kQR; qi++) {
+                const int q = lane + 32 * qi;
+#pragma unroll
+                for (int n = 0; n < NP; n++)
+                    hr[qi * NP + n] = (q < d4 && n < P) ? hs4[n * d4 + q] : make_float4(0.f, 0.f, 0.f, 0.f);
+            }
+        }
         for (int ch = 0; ch < nch; ch++) {
             const int g = (dep - 1) * nch + ch;
             const int st = g & 1;
@@ -843,15 +857,30 @@ __global__ void __launch_bounds__(kRoundThreads, 1) round_cluster_f32_kernel(con
                 float v[32];
 #pragma unroll
                 for (int j = 0; j < 32; j++) v[j] = 0.0f;
-                for (int q = lane; q < d4; q += 32) {
-                    float4 hq[NP];
+                if (hreg) {
 #pragma unroll
-                    for (int n = 0; n < NP; n++) hq[n] = n < P ? hs4[n * d4 + q] : make_float4(0.f, 0.f, 0.f, 0.f);
+                    for (int qi = 0; qi < kQR; qi++) {
+                        const int q = lane + 32 * qi;
+                        if (q < d4) {
 #pragma unroll
-                    for (int r = 0; r < RS; r++) {
-                        const float4 e = r0 + r < rows ? e4[(r0 + r) * d4 + q] : make_float4(0.f, 0.f, 0.f, 0.f);
+                            for (int r = 0; r < RS; r++) {
+                                const float4 e = r0 + r < rows ? e4[(r0 + r) * d4 + q] : make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll
-                        for (int n = 0; n < NP; n++) v[r * NP + n] = dot4(e, hq[n], v[r * NP + n]);
+                                for (int n = 0; n < NP; n++) v[r * NP + n] = dot4(e, hr[qi * NP + n], v[r * NP + n]);
+                            }
+                        }
+                    }
+                } else {
+                    for (int q = lane; q < d4; q += 32) {
+                        float4 hq[NP];
+#pragma unroll
+                        for (int n = 0; n < NP; n++) hq[n] = n < P ? hs4[n * d4 + q] : make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+                        for (int r = 0; r < RS; r++) {
+                            const float4 e = r0 + r < rows ? e4[(r0 + r) * d4 + q] : make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+                            for (int n = 0; n < NP; n++) v[r * NP + n] = dot4(e, hq[n], v[r * NP + n]);
+                        }
                     }
                 }
                 warp_reduce_scatter32(v, lane);
